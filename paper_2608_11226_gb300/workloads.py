@@ -1,0 +1,400 @@
+"""Seeded synthetic inputs for the batched PPO power-controller path.
+
+This module only *generates inputs*: power traces shaped like the paper's
+GRPO telemetry, phase labels, initial network weights, fleet start offsets
+and the numeric parameters of each workload preset.  It performs none of the
+method's arithmetic (no actuator, window, reward, network, GAE or PPO math);
+both the CUDA library and the CPU oracle consume what it produces.
+
+Shapes follow the paper's workloads:
+  * half-second samples (Sec. 4.4), clamped to the A100 envelope of 86 W idle
+    to 434 W maximum excursion (Sec. 3);
+  * the 7B run's cadence of about 81 samples per GRPO step with a
+    generation plateau and a short update burst (Sec. 5, Table 1);
+  * 72B cluster steps of about 55 s (110 samples) with sub-second
+    pipeline-overlap spikes, median 0.5 s, 90th percentile 2 s (Sec. 6.3);
+  * a 16-GPU fleet of 2x72B@4, 2x14B@2 and 4x7B@1 jobs whose per-device
+    means follow the ledger (Sec. 6.9) and whose fleet mean is 2.95 kW
+    (Sec. 8, Table 9); multi-GPU jobs' devices are anti-correlated at -0.13
+    (Sec. 6.3).
+"""
+from __future__ import annotations
+
+import dataclasses
+import math
+from typing import Dict, List, Optional, Tuple
+
+import numpy as np
+
+IDLE_W = 86.0
+MAX_W = 434.0
+DT_S = 0.5
+# tokens per generation-phase sample of the 7B run: 1,731,712 tokens over
+# 40,624 samples (Table 3, Sec. 5)
+T0_7B = 1731712.0 / 40624.0
+
+# actuator kinds / observation kinds / reward kinds (numeric codes shared by
+# the C-ABI header and the oracle's own header, each of which defines them)
+ACT_SET_LEVEL = 0   # action a selects level a directly
+ACT_INCDEC = 1      # hold, G-1, G+1, b-1, b+1 (Sec. 4.1)
+OBS_TINY8 = 0
+OBS_7B16 = 1
+OBS_OCC32 = 2
+OBS_OCC64 = 3
+REWARD_FIXED = 0     # G1 design (Sec. 4.2)
+REWARD_LAGRANGE = 1  # Eq. 6
+DTYPE_F32 = 0
+DTYPE_BF16 = 1
+
+OBS_DIM = {OBS_TINY8: 8, OBS_7B16: 16, OBS_OCC32: 32, OBS_OCC64: 64}
+
+
+@dataclasses.dataclass
+class EnvSpec:
+    n_envs: int
+    n_channels: int
+    trace_len: int
+    n_actions: int
+    obs_kind: int
+    actuator_kind: int
+    n_levels: int
+    level_init: int
+    g_min: int
+    g_max: int
+    b_min: int
+    b_max: int
+    b_init: int
+    episode_len: int
+    budget_q: int              # budget in 1/64 W
+    scale_phase_mask: int      # bit k set: samples of phase k are actuated
+    level_scale: List[List[float]]   # [n_levels][C] (used by ACT_SET_LEVEL)
+    level_tokens: List[float]        # [n_levels] tokens per generation sample
+    reward_kind: int
+    reward_window: int         # 1 or 60 samples
+    r_ok: float
+    r_viol: float
+    bonus_coef: float
+    seed: int
+
+    @property
+    def obs_dim(self) -> int:
+        return OBS_DIM[self.obs_kind]
+
+
+@dataclasses.dataclass
+class NetSpec:
+    obs_dim: int
+    hidden: int
+    n_actions: int
+    dtype: int
+
+
+@dataclasses.dataclass
+class PPOSpec:
+    epochs: int
+    minibatch: int
+    lr: float = 3e-4
+    clip: float = 0.2
+    vf_coef: float = 0.5
+    ent_coef: float = 0.0
+    max_grad_norm: float = 0.5
+    beta1: float = 0.9
+    beta2: float = 0.999
+    eps: float = 1e-8
+    gamma: float = 0.99
+    lam: float = 0.95
+
+
+@dataclasses.dataclass
+class Workload:
+    name: str
+    env: EnvSpec
+    net: NetSpec
+    ppo: PPOSpec
+    horizon: int
+    trace: np.ndarray          # [C][L] float32
+    phase: np.ndarray          # [L] uint8 (0 generation, 1 update)
+    lam_penalty: float = 1.0   # Lagrange multiplier passed to the rollout
+
+
+# --------------------------------------------------------------------------
+# traces
+# --------------------------------------------------------------------------
+
+def _clamp(x: np.ndarray) -> np.ndarray:
+    return np.clip(x, IDLE_W, MAX_W).astype(np.float32)
+
+
+def _largest_remainder(weights: np.ndarray, total: int) -> np.ndarray:
+    """Integer durations >= 1 proportional to `weights` summing to `total`."""
+    raw = weights / weights.sum() * total
+    base = np.maximum(np.floor(raw).astype(np.int64), 1)
+    rem = total - int(base.sum())
+    if rem > 0:
+        order = np.argsort(-(raw - np.floor(raw)), kind="stable")
+        base[order[:rem]] += 1
+    elif rem < 0:
+        order = np.argsort(-base, kind="stable")
+        i = 0
+        while rem < 0:
+            j = order[i % len(order)]
+            if base[j] > 1:
+                base[j] -= 1
+                rem += 1
+            i += 1
+    return base
+
+
+def tiny_trace(seed: int = 0, length: int = 4000) -> Tuple[np.ndarray, np.ndarray]:
+    """61-sample N(340,15) generation plateau, then a 20-sample N(390,10) update burst."""
+    rng = np.random.Generator(np.random.PCG64(seed))
+    t = np.arange(length)
+    in_update = (t % 81) >= 61
+    x = np.where(in_update, 390.0 + 10.0 * rng.standard_normal(length),
+                 340.0 + 15.0 * rng.standard_normal(length))
+    return _clamp(x)[None, :], in_update.astype(np.uint8)
+
+
+def _grpo_cadence(rng, n_steps: int, total: int, gen_med: float, upd_med: float):
+    gen = gen_med * np.exp(0.25 * rng.standard_normal(n_steps))
+    upd = upd_med * np.exp(0.25 * rng.standard_normal(n_steps))
+    durs = _largest_remainder(np.stack([gen, upd], 1).reshape(-1), total)
+    phase = np.repeat(np.tile(np.array([0, 1], np.uint8), n_steps), durs)
+    return phase
+
+
+def trace_7b(seed: int = 0, length: int = 60000, n_steps: int = 500):
+    """500 GRPO steps with lognormal generation/update durations (medians 100/20 samples)."""
+    rng = np.random.Generator(np.random.PCG64(seed))
+    phase = _grpo_cadence(rng, n_steps, length, 100.0, 20.0)
+    mean = np.where(phase == 1, 390.0, 340.0)
+    x = mean + 15.0 * rng.standard_normal(length)
+    return _clamp(x)[None, :], phase
+
+
+def _spikes(rng, length: int, start_prob: float = 0.01) -> np.ndarray:
+    """0/1 mask of 1-4 sample spikes (median 1 sample = 0.5 s, p90 4 samples = 2 s)."""
+    mask = np.zeros(length, np.float64)
+    starts = np.nonzero(rng.random(length) < start_prob)[0]
+    durs = rng.choice([1, 2, 3, 4], size=len(starts), p=[0.5, 0.2, 0.15, 0.15])
+    for s, d in zip(starts, durs):
+        mask[s:s + d] = 1.0
+    return mask
+
+
+def trace_72b(seed: int = 0, length: int = 22000, n_channels: int = 4,
+              samples_per_step: int = 110, corr: float = 0.8):
+    """4 channels: per-step plateau U(250,330) shared, noise with pairwise correlation `corr`."""
+    rng = np.random.Generator(np.random.PCG64(seed))
+    n_steps = (length + samples_per_step - 1) // samples_per_step
+    level = np.repeat(rng.uniform(250.0, 330.0, n_steps), samples_per_step)[:length]
+    z0 = rng.standard_normal(length)
+    x = np.empty((n_channels, length))
+    a, b = math.sqrt(corr), math.sqrt(1.0 - corr)
+    spike = 60.0 * _spikes(rng, length)
+    for c in range(n_channels):
+        x[c] = level + 15.0 * (a * z0 + b * rng.standard_normal(length)) + spike
+    return _clamp(x), np.zeros(length, np.uint8)
+
+
+def _correlated_normals(rng, k: int, n: int, rho: float) -> np.ndarray:
+    cov = np.full((k, k), rho) + (1.0 - rho) * np.eye(k)
+    chol = np.linalg.cholesky(cov)
+    return chol @ rng.standard_normal((k, n))
+
+
+FLEET_JOBS = [  # (kind, gpus) -- Sec. 8: 2x72B@4, 2x14B@2, 4x7B@1
+    ("72B", 4), ("72B", 4), ("14B", 2), ("14B", 2),
+    ("7B", 1), ("7B", 1), ("7B", 1), ("7B", 1),
+]
+# per-device mean power of each job kind (Sec. 6.9 ledger)
+FLEET_DEVICE_MEAN_W = {"7B": 314.9, "14B": 190.7, "72B": 147.0}
+FLEET_MEAN_KW = 2.95
+FLEET_NAMEPLATE_W = 16 * 400.0
+
+
+def fleet_traces(seed: int = 0, length: int = 380000):
+    """16 per-GPU traces; returns (traces [16][L] f32, job_of_gpu [16] i32)."""
+    rng = np.random.Generator(np.random.PCG64(seed))
+    total_mean = sum(FLEET_DEVICE_MEAN_W[k] * g for k, g in FLEET_JOBS)
+    scale = FLEET_MEAN_KW * 1000.0 / total_mean
+    rows, job_of_gpu = [], []
+    for j, (kind, gpus) in enumerate(FLEET_JOBS):
+        target = FLEET_DEVICE_MEAN_W[kind] * scale
+        if kind == "7B":
+            phase = _grpo_cadence(rng, length // 120 + 1, length + 0, 100.0, 20.0)[:length]
+            base = np.where(phase == 1, 1.15, 1.0)
+            noise = 15.0 * rng.standard_normal((1, length))
+            shape = base[None, :] * target + noise
+        else:
+            sps = 110 if kind == "72B" else 90
+            n_steps = length // sps + 1
+            step_level = np.repeat(rng.uniform(0.9, 1.1, n_steps), sps)[:length]
+            noise = 12.0 * _correlated_normals(rng, gpus, length, -0.13)
+            spike = 40.0 * _spikes(rng, length) if kind == "72B" else 0.0
+            shape = step_level[None, :] * target + noise + spike
+        shape = shape * (target / shape.mean(axis=1, keepdims=True))
+        for g in range(gpus):
+            rows.append(shape[g])
+            job_of_gpu.append(j)
+    return _clamp(np.stack(rows)), np.asarray(job_of_gpu, np.int32)
+
+
+def fleet_offsets(n: int, n_jobs: int, length: int, seed: int = 0) -> np.ndarray:
+    """[N][J] int32 job start offsets in [0, L); composition 0 is the aligned one."""
+    rng = np.random.Generator(np.random.PCG64(seed + 1000))
+    off = rng.integers(0, length, size=(n, n_jobs), dtype=np.int64).astype(np.int32)
+    if n > 0:
+        off[0, :] = 0
+    return off
+
+
+def budget_q(watts: float) -> int:
+    """Budget in the 1/64 W fixed-point unit, rounded to nearest."""
+    return int(round(watts * 64.0))
+
+
+# --------------------------------------------------------------------------
+# initial weights (SB3-style orthogonal initialisation; inputs to both sides)
+# --------------------------------------------------------------------------
+
+def _orthogonal(rng, rows: int, cols: int, gain: float) -> np.ndarray:
+    a = rng.standard_normal((max(rows, cols), min(rows, cols)))
+    q, r = np.linalg.qr(a)
+    q = q * np.sign(np.diag(r))[None, :]
+    if rows < cols:
+        q = q.T
+    return (gain * q[:rows, :cols]).astype(np.float32)
+
+
+def param_count(obs_dim: int, hidden: int, n_actions: int) -> int:
+    pol = hidden * obs_dim + hidden + hidden * hidden + hidden + n_actions * hidden + n_actions
+    val = hidden * obs_dim + hidden + hidden * hidden + hidden + hidden + 1
+    return pol + val
+
+
+def init_params(net: NetSpec, seed: int = 0, bias_scale: float = 0.0) -> np.ndarray:
+    """Flat fp32 parameter vector in the canonical layout:
+
+    policy: W1[H][D] b1[H] W2[H][H] b2[H] W3[A][H] b3[A]
+    value:  V1[H][D] c1[H] V2[H][H] c2[H] V3[1][H] c3[1]
+    """
+    rng = np.random.Generator(np.random.PCG64(seed + 77))
+    D, H, A = net.obs_dim, net.hidden, net.n_actions
+    g = math.sqrt(2.0)
+
+    def bias(n):
+        return (bias_scale * rng.standard_normal(n)).astype(np.float32)
+
+    parts = [
+        _orthogonal(rng, H, D, g).ravel(), bias(H),
+        _orthogonal(rng, H, H, g).ravel(), bias(H),
+        _orthogonal(rng, A, H, 0.01).ravel(), bias(A),
+        _orthogonal(rng, H, D, g).ravel(), bias(H),
+        _orthogonal(rng, H, H, g).ravel(), bias(H),
+        _orthogonal(rng, 1, H, 1.0).ravel(), bias(1),
+    ]
+    p = np.concatenate(parts).astype(np.float32)
+    assert p.size == param_count(D, H, A)
+    return p
+
+
+# --------------------------------------------------------------------------
+# presets
+# --------------------------------------------------------------------------
+
+def _incdec_tokens(g_max: int) -> List[float]:
+    # tokens per generation sample at group size G with b = b_init = 4:
+    # proportional to G, equal to the 7B run's rate at the launch setting G = 4
+    return [T0_7B * g / 4.0 for g in range(g_max + 1)]
+
+
+def _occ_tables(n_levels: int, n_channels: int):
+    # 16 concurrency levels spanning the 22.5% mean-power swing and the 5.2x
+    # throughput ratio of the generation-batch knob (Table 4); 189.1 tok/s at
+    # full occupancy (Table 5) is 94.55 tokens per half-second sample
+    scale = [[0.775 + 0.225 * l / (n_levels - 1)] * n_channels for l in range(n_levels)]
+    toks = [94.55 * 5.2 ** ((l - (n_levels - 1)) / (n_levels - 1)) for l in range(n_levels)]
+    return scale, toks
+
+
+def make_tiny(n_envs: int = 64, seed: int = 0) -> Workload:
+    trace, phase = tiny_trace(seed)
+    env = EnvSpec(
+        n_envs=n_envs, n_channels=1, trace_len=trace.shape[1], n_actions=3,
+        obs_kind=OBS_TINY8, actuator_kind=ACT_SET_LEVEL, n_levels=3, level_init=1,
+        g_min=0, g_max=2, b_min=1, b_max=1, b_init=1, episode_len=500,
+        budget_q=budget_q(300.0), scale_phase_mask=0b01,
+        level_scale=[[0.85], [1.0], [1.15]],
+        level_tokens=[0.8 * T0_7B, 1.0 * T0_7B, 1.2 * T0_7B],
+        reward_kind=REWARD_FIXED, reward_window=1, r_ok=1.0, r_viol=-8.0, bonus_coef=1.0,
+        seed=seed)
+    net = NetSpec(8, 64, 3, DTYPE_F32)
+    return Workload("tiny", env, net, PPOSpec(epochs=4, minibatch=2048), 128, trace, phase)
+
+
+def make_7b(n_envs: int = 4096, seed: int = 0) -> Workload:
+    trace, phase = trace_7b(seed)
+    env = EnvSpec(
+        n_envs=n_envs, n_channels=1, trace_len=trace.shape[1], n_actions=5,
+        obs_kind=OBS_7B16, actuator_kind=ACT_INCDEC, n_levels=9, level_init=4,
+        g_min=3, g_max=8, b_min=1, b_max=8, b_init=4, episode_len=500,
+        budget_q=budget_q(314.6), scale_phase_mask=0b11,
+        level_scale=[[1.0]] * 9, level_tokens=_incdec_tokens(8),
+        reward_kind=REWARD_FIXED, reward_window=1, r_ok=1.0, r_viol=-8.0, bonus_coef=1.0,
+        seed=seed)
+    net = NetSpec(16, 128, 5, DTYPE_F32)
+    return Workload("7b", env, net, PPOSpec(epochs=4, minibatch=8192), 512, trace, phase)
+
+
+def _occ_workload(name: str, n_envs: int, length: int, obs_kind: int, hidden: int,
+                  horizon: int, seed: int, ppo: PPOSpec) -> Workload:
+    trace, phase = trace_72b(seed, length=length)
+    C = trace.shape[0]
+    scale, toks = _occ_tables(16, C)
+    # budget: cluster mean power at the default level (7) divided by the 0.888
+    # batch-4-to-budget ratio of Sec. 4.5
+    mean_cluster = float(trace.astype(np.float64).sum(axis=0).mean()) * scale[7][0]
+    env = EnvSpec(
+        n_envs=n_envs, n_channels=C, trace_len=length, n_actions=16,
+        obs_kind=obs_kind, actuator_kind=ACT_SET_LEVEL, n_levels=16, level_init=7,
+        g_min=0, g_max=15, b_min=1, b_max=1, b_init=1, episode_len=500,
+        budget_q=budget_q(mean_cluster / 0.888), scale_phase_mask=0b11,
+        level_scale=scale, level_tokens=toks,
+        reward_kind=REWARD_LAGRANGE, reward_window=60, r_ok=1.0, r_viol=-8.0, bonus_coef=0.0,
+        seed=seed)
+    net = NetSpec(OBS_DIM[obs_kind], hidden, 16, DTYPE_BF16)
+    return Workload(name, env, net, ppo, horizon, trace, phase)
+
+
+def make_72b(n_envs: int = 65536, seed: int = 0) -> Workload:
+    return _occ_workload("72b", n_envs, 22000, OBS_OCC32, 256, 1024, seed,
+                         PPOSpec(epochs=4, minibatch=65536, ent_coef=0.01))
+
+
+def make_stress(n_envs: int = 262144, seed: int = 0, horizon: int = 2048) -> Workload:
+    return _occ_workload("stress", n_envs, 380000, OBS_OCC64, 512, horizon, seed,
+                         PPOSpec(epochs=4, minibatch=65536, ent_coef=0.01))
+
+
+PRESETS = {"tiny": make_tiny, "7b": make_7b, "72b": make_72b, "stress": make_stress}
+
+
+@dataclasses.dataclass
+class FleetWorkload:
+    traces: np.ndarray      # [G][L] float32
+    job_of_gpu: np.ndarray  # [G] int32
+    n_jobs: int
+    offsets: np.ndarray     # [N][J] int32
+    horizon: int
+    windows: np.ndarray     # [W] int32
+    budget_q: int
+
+
+def make_fleet(n_compositions: int = 1_000_000, length: int = 380000, seed: int = 0,
+               windows=(1, 60, 600)) -> FleetWorkload:
+    traces, job = fleet_traces(seed, length)
+    J = int(job.max()) + 1
+    off = fleet_offsets(n_compositions, J, length, seed)
+    return FleetWorkload(traces, job, J, off, length, np.asarray(windows, np.int32),
+                         budget_q(0.5 * FLEET_NAMEPLATE_W))

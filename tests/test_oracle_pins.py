@@ -1,0 +1,447 @@
+"""Pins of the CPU oracle against what the paper and the mathematics fix.
+
+Each test checks the oracle against something other than itself: published
+known-answer vectors, brute force on tiny inputs, closed forms, finite
+differences, library routines for special cases, and invariants.
+"""
+import math
+import os
+
+import numpy as np
+import pytest
+import torch
+
+import oracle as O
+from paper_2608_11226_gb300 import workloads as W
+from tests.envref import BruteEnv
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+# --------------------------------------------------------------------- Philox
+def test_philox_known_answers():
+    rows = 0
+    for line in open(os.path.join(GOLDEN, "philox4x32_10_kat.txt")):
+        if line.startswith("#") or not line.strip():
+            continue
+        v = [int(x, 16) for x in line.split()]
+        out = O.philox4x32_10(v[0:4], v[4:6])
+        assert list(out) == v[6:10]
+        rows += 1
+    assert rows == 3
+
+
+# -------------------------------------------------------------------- Feistel
+@pytest.mark.parametrize("n", [1, 2, 3, 5, 64, 1000, 8192, 10007])
+def test_feistel_is_a_permutation(n):
+    keys = O.perm_keys(7, 1, 3)
+    p = O.feistel_perm(n, keys)
+    assert sorted(p.tolist()) == list(range(n))
+    if n >= 64:  # not the identity and differs across epochs
+        assert not np.array_equal(p, np.arange(n))
+        assert not np.array_equal(p, O.feistel_perm(n, O.perm_keys(7, 2, 3)))
+
+
+# ----------------------------------------------------------------------- bf16
+def test_bf16_round_matches_torch():
+    rng = np.random.default_rng(0)
+    x = np.concatenate([rng.standard_normal(2000) * 10.0 ** rng.integers(-6, 6, 2000),
+                        [1.0, -1.0, 1.00390625, 1.01171875, 3.0e-3]])
+    ref = torch.tensor(x.astype(np.float32)).to(torch.bfloat16).to(torch.float64).numpy()
+    got = np.array([O.bf16_round(float(np.float32(v))) for v in x])
+    assert np.array_equal(got, ref)
+
+
+# ------------------------------------------------------------------- actuator
+def test_group_size_actuator_formula():
+    """Sec. 4.1: P = trace * (0.8 + 0.2 G / G_max), here G_max = 8."""
+    spec = W.make_7b(n_envs=4).env
+    for G, want in zip(range(3, 9), [0.875, 0.9, 0.925, 0.95, 0.975, 1.0]):
+        assert O.actuator_scale(spec, G) == np.float32(want)
+
+
+# -------------------------------------------------------- env vs brute force
+def _brute_compare(wl, n_envs, T, iters=1, seed_actions=0):
+    spec = wl.env
+    ids = list(range(n_envs))
+    env = O.OracleEnv(spec, wl.trace, wl.phase, ids)
+    brutes = [BruteEnv(spec, wl.trace.astype(np.float32), wl.phase, e, O.philox4x32_10) for e in ids]
+    rng = np.random.default_rng(seed_actions)
+    params = W.init_params(wl.net)
+    for it in range(iters):
+        forced = rng.integers(0, spec.n_actions, size=(T, n_envs)).astype(np.uint8)
+        out = env.rollout(params, wl.net.hidden, wl.net.dtype == 1, T, it, lam=0.7, forced=forced)
+        for i, b in enumerate(brutes):
+            v1 = v60 = 0
+            en = 0
+            tok = exc = 0.0
+            for t in range(T):
+                o = b.obs()
+                assert np.array_equal(out["obs"][t, i], o), (it, t, i)
+                st = b.step(int(forced[t, i]), 0.7, t, it)
+                assert out["done"][t, i] == st["done"]
+                assert abs(out["reward"][t, i] - st["r"]) <= 1e-12 * max(1.0, abs(st["r"]))
+                v1 += st["v1"]; v60 += st["v60"]; en += st["q"]
+                tok += st["tokens"]; exc += st["excess"]
+            assert np.array_equal(out["obs_last"][i], b.obs())
+            assert list(out["viol"][i]) == [v1, v60]
+            assert out["energy_q"][i] == en
+            assert abs(out["tokens"][i] - tok) <= 1e-9 * max(1.0, tok)
+            assert abs(out["excess"][i] - exc) <= 1e-9 * max(1.0, exc)
+
+
+def test_env_tiny_matches_bruteforce():
+    _brute_compare(W.make_tiny(n_envs=3), 3, 620, iters=2)
+
+
+def test_env_7b_matches_bruteforce():
+    _brute_compare(W.make_7b(n_envs=3), 3, 520)
+
+
+def test_env_72b_matches_bruteforce():
+    wl = W.make_72b(n_envs=2)
+    _brute_compare(wl, 2, 510)
+
+
+def test_env_occ64_matches_bruteforce():
+    wl = W._occ_workload("occ64", 2, 3000, W.OBS_OCC64, 32, 64, 0, W.PPOSpec(1, 64))
+    _brute_compare(wl, 2, 505)
+
+
+def _const_spec(level_w_q: int, budget: int):
+    """Constant trace whose actuated sample is exactly level_w_q / 64 W."""
+    trace = np.full((1, 2000), level_w_q / 64.0, np.float32)
+    phase = np.zeros(2000, np.uint8)
+    spec = W.EnvSpec(
+        n_envs=1, n_channels=1, trace_len=2000, n_actions=2, obs_kind=W.OBS_TINY8,
+        actuator_kind=W.ACT_SET_LEVEL, n_levels=2, level_init=0, g_min=0, g_max=1, b_min=1,
+        b_max=1, b_init=1, episode_len=500, budget_q=budget, scale_phase_mask=0b11,
+        level_scale=[[1.0], [1.0]], level_tokens=[10.0, 10.0], reward_kind=W.REWARD_FIXED,
+        reward_window=60, r_ok=1.0, r_viol=-8.0, bonus_coef=0.0, seed=3)
+    return spec, trace, phase
+
+
+@pytest.mark.parametrize("delta,expect", [(1, 1), (0, 0), (-1, 0)])
+def test_violation_counts_hand_computed(delta, expect):
+    """Eq. 2 on a constant trace at B + delta/64 W: every sample violates iff delta > 0."""
+    B = 300 * 64
+    spec, trace, phase = _const_spec(B + delta, B)
+    env = O.OracleEnv(spec, trace, phase, [0])
+    T = 700
+    out = env.rollout(np.zeros(W.param_count(8, 4, 2), np.float32), 4, False, T, 0,
+                      forced=np.zeros((T, 1), np.uint8))
+    assert list(out["viol"][0]) == [expect * T, expect * T]
+    assert out["energy_q"][0] == T * (B + delta)
+    assert np.all(out["reward"] == (-8.0 if expect else 1.0))
+    assert out["done"][:, 0].sum() == 1 and out["done"][499, 0] == 1
+    # Eq. 3: X = max(0, P30 - B) * dt = (1/64 W) * 0.5 s per violating sample
+    assert out["excess"][0] == pytest.approx(expect * T * 0.5 / 64.0, rel=1e-12)
+
+
+def test_episode_offsets_in_range():
+    wl = W.make_7b(n_envs=256)
+    env = O.OracleEnv(wl.env, wl.trace, wl.phase, list(range(256)))
+    st = env.state.view(np.int32).reshape(256, -1)
+    pos = st[:, 0]
+    assert pos.min() >= 60 and pos.max() <= wl.env.trace_len - 500
+    assert len(np.unique(pos)) > 200
+
+
+# ------------------------------------------------------------------------ MLP
+def _torch_mlp(net, params, obs, bf16=False):
+    D, H, A = net.obs_dim, net.hidden, net.n_actions
+    p = torch.tensor(params.astype(np.float64))
+    sizes = [H * D, H, H * H, H, A * H, A, H * D, H, H * H, H, H, 1]
+    parts = list(torch.split(p, sizes))
+    x = torch.tensor(obs.astype(np.float64))
+
+    def rb(t):
+        return t.float().to(torch.bfloat16).double() if bf16 else t
+
+    def net_fwd(W1, b1, W2, b2, W3, b3, out):
+        h = rb(torch.tanh(rb(x) @ rb(W1.view(H, D)).T + b1))
+        h = rb(torch.tanh(h @ rb(W2.view(H, H)).T + b2))
+        return h @ rb(W3.view(out, H)).T + b3
+
+    return net_fwd(*parts[:6], A).numpy(), net_fwd(*parts[6:], 1).numpy()[:, 0]
+
+
+@pytest.mark.parametrize("bf16", [False, True])
+def test_mlp_matches_torch(bf16):
+    net = W.NetSpec(16, 32, 5, int(bf16))
+    params = W.init_params(net, seed=3, bias_scale=0.1)
+    obs = np.random.default_rng(1).standard_normal((50, 16)).astype(np.float32)
+    lg, v = O.mlp_forward(net, params, obs)
+    tl, tv = _torch_mlp(net, params, obs, bf16)
+    tol = 1e-12 if not bf16 else 1e-2
+    assert np.allclose(lg, tl, rtol=tol, atol=tol) and np.allclose(v, tv, rtol=tol, atol=tol)
+
+
+def test_mlp_hand_computed_2_2_2():
+    net = W.NetSpec(2, 2, 2, 0)
+    # policy W1=[[1,0],[0,1]] b1=0; W2=[[1,1],[0,-1]] b2=[0,0.5]; W3=[[1,0],[0,2]] b3=[0.1,0]
+    pol = [1, 0, 0, 1, 0, 0, 1, 1, 0, -1, 0, 0.5, 1, 0, 0, 2, 0.1, 0]
+    val = [2, 0, 0, 0, 0, 0, 1, 0, 0, 0, 0, 0, 3, 0, -1]
+    params = np.array(pol + val, np.float32)
+    x = np.array([[0.5, -0.25]], np.float32)
+    lg, v = O.mlp_forward(net, params, x)
+    h1 = np.tanh([0.5, -0.25])
+    h2 = np.tanh([h1[0] + h1[1], -h1[1] + 0.5])
+    assert lg[0] == pytest.approx([h2[0] + float(np.float32(0.1)), 2 * h2[1]], rel=1e-12)
+    g = np.tanh(np.tanh(1.0))
+    assert v[0] == pytest.approx(3 * g - 1.0, rel=1e-12)
+
+
+def test_mlp_zero_weights_uniform():
+    net = W.NetSpec(8, 16, 3, 0)
+    params = np.zeros(W.param_count(8, 16, 3), np.float32)
+    params[-1] = 0.75  # value output bias
+    lg, v = O.mlp_forward(net, params, np.ones((4, 8), np.float32))
+    assert np.all(lg == 0.0) and np.all(v == 0.75)
+
+
+# -------------------------------------------------------------------- sampler
+def _bias_only_params(net, b3):
+    p = np.zeros(W.param_count(net.obs_dim, net.hidden, net.n_actions), np.float32)
+    D, H, A = net.obs_dim, net.hidden, net.n_actions
+    off = H * D + H + H * H + H + A * H
+    p[off:off + A] = b3
+    return p
+
+
+def test_sampler_inverse_cdf_and_frequencies():
+    wl = W.make_7b(n_envs=64)
+    b3 = np.array([0.3, -1.0, 1.2, 0.0, -0.4], np.float32)
+    params = _bias_only_params(wl.net, b3)
+    ids = list(range(64))
+    env = O.OracleEnv(wl.env, wl.trace, wl.phase, ids)
+    T = 512
+    out = env.rollout(params, wl.net.hidden, False, T, 5)
+    z = b3.astype(np.float64)
+    pr = np.exp(z - z.max()) / np.exp(z - z.max()).sum()
+    cdf = np.cumsum(pr)
+    key = [wl.env.seed & 0xFFFFFFFF, wl.env.seed >> 32]
+    for t in range(0, T, 37):
+        for i in ids:
+            u = (int(O.philox4x32_10([i, t, 5, 0], key)[0]) >> 8) / 2.0 ** 24
+            assert out["act_own"][t, i] == int(np.searchsorted(cdf, u, side="right"))
+    counts = np.bincount(out["act_own"].ravel(), minlength=5)
+    n = counts.sum()
+    sigma = np.sqrt(n * pr * (1 - pr))
+    assert np.all(np.abs(counts - n * pr) < 5 * sigma)
+    lp = np.log(pr)
+    assert np.allclose(out["logp"], lp[out["act_own"]], rtol=1e-12, atol=1e-12)
+    det = O.OracleEnv(wl.env, wl.trace, wl.phase, ids).rollout(params, wl.net.hidden, False, 8, 5,
+                                                                deterministic=True)
+    assert np.all(det["act_own"] == 2)
+
+
+# ------------------------------------------------------------------------ GAE
+def test_gae_closed_form_constant():
+    T, E, g, l, r, v = 50, 3, 0.99, 0.95, 0.75, 2.0  # r, v exact in fp32
+    adv, ret = O.gae(np.full((T, E), r), np.full((T, E), v), np.zeros((T, E)), np.full(E, v), g, l)
+    t = np.arange(T)
+    want = (r + (g - 1) * v) * (1 - (g * l) ** (T - t)) / (1 - g * l)
+    assert np.allclose(adv[:, 0], want, rtol=1e-12)
+    assert np.allclose(ret, adv + v)
+
+
+def test_gae_special_cases():
+    rng = np.random.default_rng(0)
+    T, E = 40, 4
+    r = rng.standard_normal((T, E)).astype(np.float32)
+    v = rng.standard_normal((T, E)).astype(np.float32)
+    lv = rng.standard_normal(E).astype(np.float32)
+    d = (rng.random((T, E)) < 0.1).astype(np.uint8)
+    r64, v64, lv64 = r.astype(np.float64), v.astype(np.float64), lv.astype(np.float64)
+    vn = np.vstack([v64[1:], lv64[None]])
+    # lambda = 0: A = delta
+    adv, _ = O.gae(r, v, d, lv, 0.99, 0.0)
+    assert np.allclose(adv, r64 + 0.99 * (1 - d) * vn - v64, rtol=1e-12, atol=1e-12)
+    # gamma = lambda = 1, no dones: A_t = sum_{k>=t} r_k + V_T - V_t
+    adv, _ = O.gae(r, v, np.zeros_like(d), lv, 1.0, 1.0)
+    want = np.cumsum(r64[::-1], 0)[::-1] + lv64[None] - v64
+    assert np.allclose(adv, want, rtol=1e-10, atol=1e-10)
+    # every step terminal: A_t = r_t - V_t
+    adv, _ = O.gae(r, v, np.ones_like(d), lv, 0.99, 0.95)
+    assert np.allclose(adv, r64 - v64, rtol=1e-12, atol=1e-12)
+
+
+# ------------------------------------------------------------------------ PPO
+def _ppo_batch(net, M, seed=0):
+    rng = np.random.default_rng(seed)
+    obs = rng.standard_normal((M, net.obs_dim)).astype(np.float32)
+    act = rng.integers(0, net.n_actions, M).astype(np.uint8)
+    lpo = (np.log(1.0 / net.n_actions) + 0.3 * rng.standard_normal(M)).astype(np.float32)
+    adv = rng.standard_normal(M).astype(np.float32)
+    ret = rng.standard_normal(M).astype(np.float32)
+    return obs, act, lpo, adv, ret
+
+
+def _torch_ppo_loss(net, params, obs, act, lpo, adv, ret, clip, vf, ent):
+    D, H, A = net.obs_dim, net.hidden, net.n_actions
+    p = torch.tensor(params, dtype=torch.float64, requires_grad=True)
+    sizes = [H * D, H, H * H, H, A * H, A, H * D, H, H * H, H, H, 1]
+    W1, b1, W2, b2, W3, b3, V1, c1, V2, c2, V3, c3 = torch.split(p, sizes)
+    x = torch.tensor(obs, dtype=torch.float64)
+    z = torch.tanh(torch.tanh(x @ W1.view(H, D).T + b1) @ W2.view(H, H).T + b2) @ W3.view(A, H).T + b3
+    V = (torch.tanh(torch.tanh(x @ V1.view(H, D).T + c1) @ V2.view(H, H).T + c2) @ V3.view(1, H).T + c3)[:, 0]
+    logp_all = torch.log_softmax(z, -1)
+    lp = logp_all[torch.arange(len(act)), torch.tensor(act, dtype=torch.long)]
+    a = torch.tensor(adv, dtype=torch.float64)
+    a = (a - a.mean()) / (a.std() + 1e-8)
+    rho = torch.exp(lp - torch.tensor(lpo, dtype=torch.float64))
+    pg = -torch.min(rho * a, torch.clamp(rho, 1 - clip, 1 + clip) * a).mean()
+    vl = ((torch.tensor(ret, dtype=torch.float64) - V) ** 2).mean()
+    H_ = -(logp_all.exp() * logp_all).sum(-1).mean()
+    loss = pg + vf * vl - ent * H_
+    loss.backward()
+    return loss.item(), p.grad.numpy()
+
+
+def test_ppo_gradient_matches_autograd_and_finite_differences():
+    net = W.NetSpec(6, 8, 4, 0)
+    params = W.init_params(net, seed=5, bias_scale=0.1).astype(np.float64)
+    batch = _ppo_batch(net, 32)
+    loss, grad, _ = O.ppo_minibatch_grad(net, params, *batch, 0.2, 0.5, 0.01)
+    tl, tg = _torch_ppo_loss(net, params, *batch, 0.2, 0.5, 0.01)
+    assert loss == pytest.approx(tl, rel=1e-12)
+    assert np.allclose(grad, tg, rtol=1e-9, atol=1e-12)
+    rng = np.random.default_rng(1)
+    h = 1e-6
+    for k in rng.choice(len(params), 40, replace=False):
+        pp, pm = params.copy(), params.copy()
+        pp[k] += h
+        pm[k] -= h
+        lp_, _, _ = O.ppo_minibatch_grad(net, pp, *batch, 0.2, 0.5, 0.01, want_grad=False)
+        lm_, _, _ = O.ppo_minibatch_grad(net, pm, *batch, 0.2, 0.5, 0.01, want_grad=False)
+        fd = (lp_ - lm_) / (2 * h)
+        assert abs(fd - grad[k]) <= 1e-6 * max(1.0, abs(grad[k])), k
+
+
+def test_ppo_first_minibatch_ratio_one_policy_loss_zero():
+    """With logp_old = logp under the current params, rho = 1 and the
+    clipped surrogate is -mean(normalised advantage) = 0."""
+    net = W.NetSpec(6, 8, 4, 0)
+    params = W.init_params(net, seed=2, bias_scale=0.1)
+    obs, act, _, adv, ret = _ppo_batch(net, 64)
+    lg, _ = O.mlp_forward(net, params, obs)
+    lse = lg.max(1) + np.log(np.exp(lg - lg.max(1, keepdims=True)).sum(1))
+    lpo = (lg[np.arange(64), act] - lse).astype(np.float32)
+    _, _, st = O.ppo_minibatch_grad(net, params.astype(np.float64), obs, act, lpo, adv, ret,
+                                    0.2, 0.5, 0.0)
+    assert abs(st[0]) < 1e-6 and st[4] == 0.0 and abs(st[3]) < 1e-12
+
+
+def test_ppo_clip_cases_two_samples():
+    """Two samples, normalised advantages +-1/sqrt(2)*sqrt(2)... rho set via logp_old."""
+    net = W.NetSpec(2, 2, 2, 0)
+    params = np.zeros(W.param_count(2, 2, 2), np.float64)  # uniform policy, logp = log 0.5
+    obs = np.zeros((2, 2), np.float32)
+    act = np.array([0, 1], np.uint8)
+    adv = np.array([1.0, -1.0], np.float32)   # normalised: +-1/sqrt(2) * ... (mean 0, std sqrt 2)
+    ret = np.zeros(2, np.float32)
+    an = np.array([1.0, -1.0]) / (np.sqrt(2.0) + 1e-8)
+    for rho in (0.5, 0.9, 1.0, 1.1, 1.5):
+        lpo = np.full(2, math.log(0.5) - math.log(rho), np.float32)
+        r = math.exp(math.log(0.5) - float(np.float32(math.log(0.5) - math.log(rho))))
+        _, _, st = O.ppo_minibatch_grad(net, params, obs, act, lpo, adv, ret, 0.2, 0.5, 0.0)
+        rc = min(max(r, 0.8), 1.2)
+        want = -np.mean(np.minimum(r * an, rc * an))
+        assert st[0] == pytest.approx(want, rel=1e-9, abs=1e-12)
+        assert st[4] == (1.0 if abs(r - 1) > 0.2 else 0.0)
+
+
+def test_ppo_adam_first_step_is_signed_lr():
+    net = W.NetSpec(6, 8, 4, 0)
+    params = W.init_params(net, seed=4, bias_scale=0.1)
+    N = 256
+    obs, act, lpo, adv, ret = _ppo_batch(net, N, seed=3)
+    ppo = W.PPOSpec(epochs=1, minibatch=N, max_grad_norm=1e9)
+    P, m, v, t, st = O.ppo_update(net, ppo, params, np.zeros(params.size), np.zeros(params.size), 0,
+                                  obs, act, lpo, adv, ret, seed=1, iteration=0, max_steps=1)
+    _, g, _ = O.ppo_minibatch_grad(net, params.astype(np.float64), obs, act, lpo, adv, ret,
+                                   0.2, 0.5, 0.0)
+    step = P - params.astype(np.float64)
+    big = np.abs(g) > 1e-5
+    assert t == 1 and st[7] == 1
+    assert np.allclose(step[big], -3e-4 * np.sign(g[big]), rtol=1e-3)
+    # a full-batch minibatch sees every sample once, so the permutation does not matter
+    assert np.allclose(m, 0.1 * g, rtol=1e-12, atol=1e-300)
+
+
+def test_ppo_grad_norm_clip():
+    net = W.NetSpec(6, 8, 4, 0)
+    params = W.init_params(net, seed=4, bias_scale=0.1)
+    obs, act, lpo, adv, ret = _ppo_batch(net, 64, seed=9)
+    ppo = W.PPOSpec(epochs=1, minibatch=64, max_grad_norm=1e-3)
+    _, m, _, _, st = O.ppo_update(net, ppo, params, np.zeros(params.size), np.zeros(params.size),
+                                  0, obs, act, lpo, adv, ret, seed=1, iteration=0, max_steps=1)
+    # m = (1 - beta1) * clipped gradient; the clipped gradient has norm max_norm * n / (n + 1e-6)
+    n = st[6]
+    assert np.linalg.norm(m / 0.1) == pytest.approx(1e-3 * n / (n + 1e-6), rel=1e-9)
+
+
+# ---------------------------------------------------------------------- fleet
+def _brute_fleet(traces, job, J, offsets, H, windows, Bq):
+    q = np.rint(traces.astype(np.float32) * np.float32(64)).astype(np.int64)
+    G, L = q.shape
+    N = offsets.shape[0]
+    counts = np.zeros((N, len(windows)), np.int64)
+    peaks = np.zeros((N, len(windows)), np.int64)
+    t = np.arange(H)
+    for n in range(N):
+        P = sum(q[g, (t + offsets[n, job[g]]) % L] for g in range(G))
+        for wi, w in enumerate(windows):
+            S = np.array([P[tt - w + 1:tt + 1].sum() for tt in range(w - 1, H)])
+            counts[n, wi] = int((S > Bq * w).sum())
+            peaks[n, wi] = int(S.max()) if len(S) else 0
+    return counts, peaks
+
+
+def test_fleet_matches_bruteforce():
+    rng = np.random.default_rng(0)
+    G, L, J = 6, 700, 3
+    traces = (300 + 60 * rng.standard_normal((G, L))).astype(np.float32)
+    job = np.array([0, 0, 1, 2, 2, 2], np.int32)
+    off = rng.integers(0, L, (9, J)).astype(np.int32)
+    off[0] = 0
+    windows = np.array([1, 7, 60, 600], np.int32)
+    Bq = 6 * 300 * 64
+    for H in (L, 650, 599, 1):
+        c, p = O.fleet_windows(traces, job, J, off, H, windows, Bq)
+        bc, bp = _brute_fleet(traces, job, J, off, H, windows, Bq)
+        assert np.array_equal(c, bc) and np.array_equal(p, bp)
+
+
+def test_fleet_invariants():
+    fw = W.make_fleet(n_compositions=6, length=3000, windows=(1, 60, 600))
+    c, p = O.fleet_windows(fw.traces, fw.job_of_gpu, fw.n_jobs, fw.offsets, fw.horizon,
+                           fw.windows, fw.budget_q)
+    q = np.rint(fw.traces * np.float32(64)).astype(np.int64)
+    # (iii) the aligned composition is the direct sum of the traces
+    direct = q.sum(0)
+    assert p[0, 0] == direct.max()
+    assert c[0, 0] == int((direct > fw.budget_q).sum())
+    # (ii) the composed peak never exceeds the sum of per-job peaks
+    for wi, w in enumerate(fw.windows):
+        per_job = 0
+        for j in range(fw.n_jobs):
+            pj = q[fw.job_of_gpu == j].sum(0)
+            _, pk = O.fleet_windows(pj[None].astype(np.float32) / 64.0, [0], 1,
+                                    np.zeros((1, 1), np.int32), fw.horizon, [w], 0)
+            per_job += pk[0, 0]
+        assert np.all(p[:, wi] <= per_job)
+    # (iv) one job and one trace reduce to the single-trace window analysis
+    c1, p1 = O.fleet_windows(fw.traces[:1], [0], 1, np.zeros((1, 1), np.int32), fw.horizon,
+                             [60], fw.budget_q // 16)
+    S = np.convolve(q[0], np.ones(60, np.int64), mode="valid")
+    assert c1[0, 0] == int((S > 60 * (fw.budget_q // 16)).sum()) and p1[0, 0] == S.max()
+
+
+def test_fleet_constant_hand_counted():
+    traces = np.full((2, 100), 10.0, np.float32)  # q = 640 each, sum 1280
+    off = np.array([[0, 0], [5, 17]], np.int32)
+    for Bq, want in ((1279, [100, 41]), (1280, [0, 0])):
+        c, p = O.fleet_windows(traces, [0, 1], 2, off, 100, [1, 60], Bq)
+        assert c.tolist() == [want, want] and p.tolist() == [[1280, 76800]] * 2
