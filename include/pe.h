@@ -1,0 +1,254 @@
+/*
+ * pe.h -- C ABI of the GB300 library for batched, trace-driven training of
+ * the PPO power meta-controller of "Cutting AI Datacenter Energy with
+ * Reinforcement Learning: Measured Power Control of LLM Training from One
+ * GPU to the Fleet" (arxiv 2608.11226).
+ *
+ * The library runs every step of the path on one GPU (sm_103a):
+ *   pe_env_create   -- load a power trace, validate it, place E envs      (Sec. 4.1)
+ *   pe_rollout      -- E envs x T steps: observe, policy, sample, actuate,
+ *                      windows, reward; then the value network            (Sec. 4.1, 4.2, Eqs. 1-6)
+ *   pe_gae          -- reverse-time generalised advantage estimation       (Sec. 4.2)
+ *   pe_ppo_update   -- epochs x minibatches of clipped-loss PPO with Adam  (Sec. 4.2, 4.5)
+ *   pe_fleet_windows-- composed fleet traces, window violation counts and
+ *                      peaks over 0.5 s / 30 s / 5 min windows             (Sec. 7, 8, Eqs. 1-2)
+ *
+ * Conventions
+ *  - Every buffer argument is a DEVICE pointer owned by the caller, unless
+ *    the argument says "host".  The library owns only the opaque pe_env.
+ *  - Calls are asynchronous on `stream` (a cudaStream_t passed as void*;
+ *    NULL = the legacy default stream).  Argument errors are detected before
+ *    any launch and returned synchronously; nothing is launched then.
+ *  - No call except pe_env_create/pe_env_destroy allocates device memory;
+ *    scratch space is a caller-provided workspace whose size the matching
+ *    *_workspace_bytes function returns.
+ *  - On a non-zero status, pe_last_error() returns a thread-local message.
+ *  - No C++ exception crosses this interface.
+ *
+ * Units: one environment step consumes one half-second power sample
+ * (Delta t = 0.5 s, Sec. 4.4).  Power inside the library is an int32 in
+ * 1/64 W: q = rint(P * 64) of the fp32 actuated power P, so that window sums
+ * and violation counts are exact integers.
+ */
+#ifndef PE_H
+#define PE_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef int32_t pe_status;
+#define PE_OK 0
+#define PE_EINVAL 1     /* bad argument (null pointer, size, unsupported shape) */
+#define PE_ENOMEM 2     /* device allocation failed (pe_env_create only) */
+#define PE_ECUDA 3      /* a CUDA runtime call or launch failed */
+#define PE_EOVERFLOW 4  /* trace outside the fixed-point range */
+#define PE_ETIMEOUT 5   /* a bounded device-side wait gave up */
+#define PE_ESTATE 6     /* object in the wrong state */
+
+#define PE_MAX_LEVELS 32
+#define PE_MAX_CHANNELS 4
+
+/* actuator kinds */
+#define PE_ACT_SET_LEVEL 0 /* action a selects actuator level a (Table 4 concurrency levels) */
+#define PE_ACT_INCDEC 1    /* Sec. 4.1: hold, G-1, G+1, batch-1, batch+1 */
+/* observation kinds (width D) */
+#define PE_OBS_TINY8 0  /* D=8: Sec. 4.1 state */
+#define PE_OBS_7B16 1   /* D=16: last 8 samples, 30 s mean, budget slack, phase, G, b, 10 s mean, 5 s slope */
+#define PE_OBS_OCC32 2  /* D=32: Eq. 5 eight-vector + per-channel last 4 samples + per-channel 30 s means */
+#define PE_OBS_OCC64 3  /* D=64: Eq. 5 eight-vector + per-channel last 12 + per-channel 10 s and 30 s means */
+/* reward kinds */
+#define PE_REWARD_FIXED 0    /* Sec. 4.2 G1: +r_ok / r_viol per step plus a throughput bonus */
+#define PE_REWARD_LAGRANGE 1 /* Eq. 6 per step: T/1000 - lambda X - 2 lambda max(0, P30 - B) */
+/* network element types */
+#define PE_F32 0
+#define PE_BF16 1
+/* pe_rollout flags */
+#define PE_ROLLOUT_DETERMINISTIC 1 /* argmax action, lowest index on ties (Sec. 4.4 evaluation) */
+
+/* Environment configuration (Sec. 4.1 MDP; Sec. 4.5 windows and budget).
+ * Actuated power of channel c at level l is the fp32 product
+ *   P = x_c(p) * s(l, c)  when bit phase(p) of scale_phase_mask is set, else x_c(p),
+ * where s(l, c) = level_scale[l][c] for PE_ACT_SET_LEVEL and, for the
+ * group-size actuator PE_ACT_INCDEC, s(G) = (float)(0.8 + (0.2 * G) / g_max)
+ * evaluated in double (Sec. 4.1).  Tokens per generation-phase sample are
+ * level_tokens[l] (times b / b_init for PE_ACT_INCDEC); 0 in other phases. */
+typedef struct pe_env_config {
+  int32_t n_envs;           /* E >= 1 */
+  int32_t n_channels;       /* C in [1, 4]: per-GPU channels summed into cluster power */
+  int32_t trace_len;        /* L >= episode_len + 60 */
+  int32_t n_actions;        /* A: 5 for INCDEC, n_levels for SET_LEVEL */
+  int32_t obs_kind;         /* PE_OBS_* */
+  int32_t actuator_kind;    /* PE_ACT_* */
+  int32_t n_levels;         /* levels in the tables (INCDEC: g_max + 1) */
+  int32_t level_init;       /* level (or G) at every episode start */
+  int32_t g_min, g_max;     /* INCDEC group-size range; g_min = 3 is the Sec. 4.2 (G4) floor */
+  int32_t b_min, b_max, b_init; /* INCDEC batch-size range and start */
+  int32_t episode_len;      /* steps per episode (500, Sec. 4.1) */
+  int32_t budget_q;         /* budget B in 1/64 W */
+  int32_t scale_phase_mask; /* bit k: samples of phase k are actuated */
+  int32_t reward_kind;      /* PE_REWARD_* */
+  int32_t reward_window;    /* FIXED reward: violation over 1 sample or 60 samples (30 s) */
+  float r_ok, r_viol, bonus_coef; /* FIXED reward: +1, -8, throughput bonus coefficient */
+  float level_scale[PE_MAX_LEVELS][PE_MAX_CHANNELS];
+  float level_tokens[PE_MAX_LEVELS];
+  uint64_t seed;            /* Philox4x32-10 key */
+} pe_env_config;
+
+/* Policy/value network: two separate tanh MLPs obs_dim -> hidden -> hidden
+ * -> {n_actions logits, 1 value} (Sec. 4.2 MLP actor-critic).  Parameters are
+ * one flat fp32 vector, row-major W[out][in]:
+ *   policy: W1[H][D] b1[H] W2[H][H] b2[H] W3[A][H] b3[A]
+ *   value : V1[H][D] c1[H] V2[H][H] c2[H] V3[1][H] c3[1]
+ * Supported (D, H, A, dtype): (8,64,3,F32), (16,128,5,F32).  A BF16 network
+ * keeps fp32 master parameters; the library rounds weights, observations and
+ * hidden activations to bf16 and accumulates in fp32. */
+typedef struct pe_net {
+  int32_t obs_dim, hidden, n_actions, dtype;
+} pe_net;
+
+/* Rollout buffer, time-major [T][E] (row t holds env 0..E-1).  All device
+ * pointers, caller-owned; every one is written by pe_rollout. */
+typedef struct pe_rollout_buf {
+  void* obs;          /* [T][E][D] fp32 (or bf16 for a BF16 network): observation before step t */
+  void* obs_last;     /* [E][D] observation after the last step */
+  uint8_t* act;       /* [T][E] action taken */
+  float* logp;        /* [T][E] log-probability of the action under the policy */
+  float* value;       /* [T][E] value of obs[t] */
+  float* last_value;  /* [E]    value of obs_last */
+  float* reward;      /* [T][E] */
+  uint8_t* done;      /* [T][E] 1 if the episode ended with step t */
+  int32_t* viol;      /* [E][2] violating steps of this call: instantaneous (Eq. 2, w=0.5 s), 30 s (Eq. 2) */
+  float* tokens;      /* [E]    generated tokens of this call */
+  float* excess;      /* [E]    integrated excess of this call, W*s (Eq. 3) */
+  int64_t* energy_q;  /* [E]    sum of actuated cluster power over the call, 1/64 W per sample */
+} pe_rollout_buf;
+
+/* PPO configuration (Sec. 4.2 / 4.5; SB3 defaults where the paper is silent) */
+typedef struct pe_ppo_config {
+  int32_t epochs;        /* passes over the rollout */
+  int32_t minibatch;     /* samples per minibatch; the last one of an epoch may be smaller */
+  float lr, clip, vf_coef, ent_coef, max_grad_norm, beta1, beta2, eps;
+  uint64_t seed;         /* Philox key of the minibatch permutation */
+  uint32_t iteration;    /* PPO iteration (part of the permutation counter) */
+} pe_ppo_config;
+
+typedef struct pe_env pe_env;
+
+/* Create E environments over one trace (Sec. 4.1 trace replay).
+ *  trace: [C][L] fp32 watts, host or device memory (copied).
+ *  phase: [L] uint8 phase label per sample (0 generation, 1 update; Sec. 4.4).
+ * Every env starts an episode at offset 60 + floor(u * (L - episode_len - 59) / 2^32),
+ * u = Philox4x32-10(key = seed, ctr = (env, 0, 0, 2)).out[0]; its 60-sample
+ * history is warm-started at level_init.
+ * Errors: PE_EINVAL (sizes, kinds, tables), PE_EOVERFLOW (a sample that is
+ * not finite, negative, or whose actuated 60-sample window sum could exceed
+ * int32), PE_ENOMEM, PE_ECUDA.  Synchronous. */
+pe_status pe_env_create(const pe_env_config* cfg, const float* trace, const uint8_t* phase,
+                        pe_env** out);
+pe_status pe_env_destroy(pe_env* env);
+
+/* Checkpoint: the env state is a flat byte image (host memory). */
+int64_t pe_env_state_bytes(const pe_env* env);
+pe_status pe_env_save(const pe_env* env, void* host_dst);
+pe_status pe_env_load(pe_env* env, const void* host_src);
+
+int64_t pe_param_count(const pe_net* net);
+
+/* One rollout of `horizon` steps for all envs (Sec. 4.1 MDP, Sec. 4.2
+ * controller), continuing each env where the previous call left it.
+ * Step t of env e: observation -> policy logits -> action (inverse CDF of
+ * softmax at u = (philox >> 8) 2^-24, ctr = (e, t, iteration, 0)) -> actuator
+ * -> consume one sample -> windows (Eq. 1: 10 s = 20 samples, 30 s = 60)
+ * -> violation (Eq. 2), excess (Eq. 3), tokens, reward -> episode end after
+ * episode_len steps, new offset from ctr = (e, t, iteration, 1).
+ * Then the value network on every observation and on obs_last.
+ *  lambda: Lagrange multiplier of Eq. 6 (PE_REWARD_LAGRANGE only).
+ * Errors: PE_EINVAL (unsupported network, null buffer, horizon < 1), PE_ECUDA. */
+pe_status pe_rollout(pe_env* env, const pe_net* net, const float* params, int32_t horizon,
+                     uint32_t iteration, float lambda, int32_t flags, const pe_rollout_buf* buf,
+                     void* stream);
+
+/* Value network on n observations (fp32, or bf16 for a BF16 network). */
+pe_status pe_value(const pe_net* net, const float* params, const void* obs, int64_t n,
+                   float* value, void* stream);
+
+/* Generalised advantage estimation (gamma, lambda per Sec. 4.2), time-major:
+ *   delta_t = r_t + gamma (1 - d_t) V_{t+1} - V_t,  V_T = last_value,
+ *   A_t = delta_t + gamma lambda (1 - d_t) A_{t+1},  ret_t = A_t + V_t.
+ * reward, value, adv, ret: [T][E] fp32; done: [T][E] uint8; last_value: [E].
+ * Errors: PE_EINVAL. */
+pe_status pe_gae(const float* reward, const float* value, const uint8_t* done,
+                 const float* last_value, int32_t T, int32_t E, float gamma, float lam,
+                 float* adv, float* ret, void* stream);
+
+/* PPO update over n_samples = T*E rollout samples (Sec. 4.2; SB3 loss):
+ * for each epoch a Feistel permutation of [0, n) keyed by
+ * Philox(key = seed, ctr = (epoch, 0, iteration, 3)); each minibatch
+ * normalises its advantages, forms the clipped surrogate, value loss and
+ * entropy bonus, clips the global gradient norm and takes one Adam step.
+ *  params, adam_m, adam_v: [P] fp32, updated in place.
+ *  adam_t: Adam steps taken before this call (host value).
+ *  obs [n][D] (dtype of the net), act, logp_old, adv, ret: rollout/GAE buffers.
+ *  stats: [8] fp32 out: mean pg loss, value loss, entropy, approx KL,
+ *         clip fraction, total loss; last pre-clip gradient norm; step count.
+ *  workspace: >= pe_ppo_workspace_bytes(...) bytes of device memory.
+ * Errors: PE_EINVAL (unsupported network, sizes, small workspace), PE_ECUDA. */
+int64_t pe_ppo_workspace_bytes(const pe_net* net, const pe_ppo_config* cfg, int64_t n_samples);
+pe_status pe_ppo_update(const pe_net* net, float* params, float* adam_m, float* adam_v,
+                        int64_t adam_t, const void* obs, const uint8_t* act,
+                        const float* logp_old, const float* adv, const float* ret,
+                        int64_t n_samples, const pe_ppo_config* cfg, float* stats,
+                        void* workspace, int64_t workspace_bytes, void* stream);
+
+/* Fleet window accounting (Sec. 7 window analysis, Sec. 8 fleet
+ * composition).  Composition n starts job j at offset o[n][j] (a job's GPUs
+ * share it; traces tile circularly with period L):
+ *   P_n(t) = sum_g q_g((t + o[n][job(g)]) mod L),  t in [0, H)
+ *   S_w(t) = sum_{tau = t-w+1}^{t} P_n(tau)         t in [w-1, H)
+ *   counts[n][i] = #{t : S_w(t) > budget_q * w},  peaks[n][i] = max_t S_w(t)  (0 if H < w)
+ * with q_g = rint(64 * trace) in 1/64 W.
+ *  traces: [G][L] fp32 watts; job_of_gpu: [G] in [0, J); offsets: [N][J] in [0, L)
+ *  (all device memory); windows: [W] HOST array, W in [1, 4], each w in [1, 992];
+ *  counts, peaks: [N][W] int32 (device).
+ *  workspace: >= pe_fleet_workspace_bytes(J, L, H) bytes.
+ * The call validates the traces on the device and waits for that check
+ * (one small device-to-host read on `stream`) before launching the counts.
+ * Errors: PE_EINVAL (sizes, pointers, job map or offsets out of range),
+ * PE_EOVERFLOW (a sample that is not finite or negative, or a composed
+ * window sum or budget_q * w that could exceed int32), PE_ECUDA. */
+int64_t pe_fleet_workspace_bytes(int32_t J, int32_t L, int32_t H);
+pe_status pe_fleet_windows(const float* traces, int32_t G, int32_t L, const int32_t* job_of_gpu,
+                           int32_t J, const int32_t* offsets, int64_t N, int32_t H,
+                           const int32_t* windows, int32_t W, int64_t budget_q,
+                           int32_t* counts, int32_t* peaks, void* workspace,
+                           int64_t workspace_bytes, void* stream);
+
+/* Launch profiling (off by default).  When enabled, every kernel launch of
+ * the library is bracketed by a pair of CUDA events recorded on the launch's
+ * stream; pe_profile_read waits for the recorded events of one kernel kind,
+ * returns the summed device time and the launch count, and clears that kind.
+ * Kinds: */
+#define PE_PROF_ROLLOUT 0
+#define PE_PROF_VALUE 1
+#define PE_PROF_GAE 2
+#define PE_PROF_PPO_GRAD 3
+#define PE_PROF_PPO_REDUCE 4
+#define PE_PROF_PPO_ADAM 5
+#define PE_PROF_PPO_OTHER 6
+#define PE_PROF_FLEET_PREP 7
+#define PE_PROF_FLEET_WINDOWS 8
+#define PE_PROF_KINDS 9
+pe_status pe_profile_enable(int32_t on);
+pe_status pe_profile_read(int32_t kind, double* total_ms, int64_t* launches);
+const char* pe_profile_kind_name(int32_t kind);
+
+/* Message for the last non-OK status on this thread ("" if none). */
+const char* pe_last_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* PE_H */

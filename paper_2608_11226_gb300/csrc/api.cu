@@ -1,0 +1,469 @@
+// C ABI of the pe library: argument validation, object lifetime and kernel
+// dispatch.  Every argument error is detected here, before any launch.
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <mutex>
+#include <vector>
+
+#include "env.cuh"
+#include "mlp_f32.cuh"
+
+namespace pe {
+
+static thread_local char g_err[512] = "";
+
+pe_status fail(pe_status code, const char* fmt, ...) {
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(g_err, sizeof(g_err), fmt, ap);
+  va_end(ap);
+  return code;
+}
+
+pe_status cuda_fail(cudaError_t err, const char* what) {
+  snprintf(g_err, sizeof(g_err), "CUDA error %d (%s) in %s", (int)err, cudaGetErrorString(err), what);
+  return PE_ECUDA;
+}
+
+void clear_error() { g_err[0] = 0; }
+
+// ---------------------------------------------------------------------------
+// launch profiling
+// ---------------------------------------------------------------------------
+struct ProfRec {
+  int kind;
+  cudaEvent_t a, b;
+};
+static std::mutex g_prof_mu;
+static bool g_prof_on = false;
+static std::vector<cudaEvent_t> g_prof_pool;
+static std::vector<ProfRec> g_prof_recs;
+static thread_local cudaEvent_t g_prof_open = nullptr;
+
+static cudaEvent_t prof_event() {
+  if (!g_prof_pool.empty()) {
+    cudaEvent_t e = g_prof_pool.back();
+    g_prof_pool.pop_back();
+    return e;
+  }
+  cudaEvent_t e = nullptr;
+  if (cudaEventCreate(&e) != cudaSuccess) return nullptr;
+  return e;
+}
+
+void prof_mark(int kind, cudaStream_t st, bool begin) {
+  if (!g_prof_on) return;
+  std::lock_guard<std::mutex> lk(g_prof_mu);
+  if (begin) {
+    g_prof_open = prof_event();
+    if (g_prof_open) cudaEventRecord(g_prof_open, st);
+  } else if (g_prof_open) {
+    cudaEvent_t b = prof_event();
+    if (b) {
+      cudaEventRecord(b, st);
+      g_prof_recs.push_back(ProfRec{kind, g_prof_open, b});
+    } else {
+      g_prof_pool.push_back(g_prof_open);
+    }
+    g_prof_open = nullptr;
+  }
+}
+
+// defined in the kernel translation units
+pe_status rollout_f32(const EnvDev& env, const pe_net& net, const float* params, int T, uint32_t it,
+                      float lambda, int det, const pe_rollout_buf& buf, cudaStream_t st);
+pe_status value_f32(const pe_net& net, const float* params, const float* obs, int64_t n,
+                    float* value, cudaStream_t st);
+pe_status gae_launch(const float* r, const float* v, const uint8_t* d, const float* last_v, int T,
+                     int E, float gamma, float lam, float* adv, float* ret, cudaStream_t st);
+int64_t ppo_ws_bytes_f32(const pe_net& net, const pe_ppo_config& cfg, int64_t N);
+pe_status ppo_update_f32(const pe_net& net, float* params, float* m, float* v, int64_t adam_t,
+                         const float* obs, const uint8_t* act, const float* logp_old,
+                         const float* adv, const float* ret, int64_t N, const pe_ppo_config& cfg,
+                         float* stats, void* ws, cudaStream_t st);
+int64_t fleet_ws_bytes(int J, int L, int H);
+pe_status fleet_launch(const float* traces, int G, int L, const int32_t* job_of_gpu, int J,
+                       const int32_t* offsets, int64_t N, int H, const int32_t* windows, int W,
+                       int64_t budget_q, int32_t* counts, int32_t* peaks, void* workspace,
+                       cudaStream_t st);
+
+static int obs_width(int kind) {
+  switch (kind) {
+    case PE_OBS_TINY8: return 8;
+    case PE_OBS_7B16: return 16;
+    case PE_OBS_OCC32: return 32;
+    case PE_OBS_OCC64: return 64;
+    default: return -1;
+  }
+}
+
+// episode start offsets and the default level for every env
+__global__ void env_init_kernel(EnvDev env) {
+  const int e = blockIdx.x * blockDim.x + threadIdx.x;
+  if (e >= env.E) return;
+  const uint32_t u = draw32(env.seed, (uint32_t)e, 0u, 0u, kDrawInit);
+  const uint32_t span = (uint32_t)(env.L - env.ep_len - kWLong + 1);
+  env.st[kStPos * env.E + e] = kWLong + (int)__umulhi(u, span);
+  env.st[kStK * env.E + e] = 0;
+  env.st[kStLevel * env.E + e] = env.level_init;
+  env.st[kStPrev * env.E + e] = env.level_init;
+  env.st[kStB * env.E + e] = env.b_init;
+  env.st[kStTil * env.E + e] = 0;
+  for (int i = 0; i < kRing; ++i) env.ring[(int64_t)e * kRing + i] = (uint8_t)env.level_init;
+  for (int i = 0; i < 8; ++i) env.sums[(int64_t)e * 8 + i] = 0;
+}
+
+}  // namespace pe
+
+using namespace pe;
+
+struct pe_env {
+  pe_env_config cfg;
+  EnvDev dev;
+  int device;
+};
+
+extern "C" {
+
+const char* pe_last_error(void) { return g_err; }
+
+static const char* kProfNames[PE_PROF_KINDS] = {
+    "rollout", "value", "gae", "ppo_grad", "ppo_reduce", "ppo_adam", "ppo_other",
+    "fleet_prepare", "fleet_windows"};
+
+const char* pe_profile_kind_name(int32_t kind) {
+  return (kind >= 0 && kind < PE_PROF_KINDS) ? kProfNames[kind] : "";
+}
+
+pe_status pe_profile_enable(int32_t on) {
+  clear_error();
+  std::lock_guard<std::mutex> lk(g_prof_mu);
+  g_prof_on = on != 0;
+  return PE_OK;
+}
+
+pe_status pe_profile_read(int32_t kind, double* total_ms, int64_t* launches) {
+  clear_error();
+  if (kind < 0 || kind >= PE_PROF_KINDS || !total_ms || !launches) return fail(PE_EINVAL, "bad profile query");
+  std::lock_guard<std::mutex> lk(g_prof_mu);
+  double ms = 0.0;
+  int64_t n = 0;
+  std::vector<ProfRec> keep;
+  for (const ProfRec& r : g_prof_recs) {
+    if (r.kind != kind) {
+      keep.push_back(r);
+      continue;
+    }
+    PE_TRY_CUDA(cudaEventSynchronize(r.b));
+    float t = 0.0f;
+    PE_TRY_CUDA(cudaEventElapsedTime(&t, r.a, r.b));
+    ms += t;
+    ++n;
+    g_prof_pool.push_back(r.a);
+    g_prof_pool.push_back(r.b);
+  }
+  g_prof_recs.swap(keep);
+  *total_ms = ms;
+  *launches = n;
+  return PE_OK;
+}
+
+int64_t pe_param_count(const pe_net* net) {
+  if (!net) return -1;
+  return mlp_layout(net->obs_dim, net->hidden, net->n_actions).total;
+}
+
+static pe_status check_env_config(const pe_env_config* c) {
+  if (c->n_envs < 1) return fail(PE_EINVAL, "n_envs must be >= 1");
+  if (c->n_channels < 1 || c->n_channels > PE_MAX_CHANNELS) return fail(PE_EINVAL, "n_channels must be in [1, 4]");
+  if (c->episode_len < 1) return fail(PE_EINVAL, "episode_len must be >= 1");
+  if ((int64_t)c->trace_len < (int64_t)c->episode_len + kWLong)
+    return fail(PE_EINVAL, "trace_len (%d) must be >= episode_len + 60", c->trace_len);
+  if (obs_width(c->obs_kind) < 0) return fail(PE_EINVAL, "unknown obs_kind %d", c->obs_kind);
+  if (c->n_levels < 1 || c->n_levels > PE_MAX_LEVELS) return fail(PE_EINVAL, "n_levels must be in [1, 32]");
+  if (c->level_init < 0 || c->level_init >= c->n_levels) return fail(PE_EINVAL, "level_init out of range");
+  if (c->actuator_kind == PE_ACT_INCDEC) {
+    if (c->n_actions != 5) return fail(PE_EINVAL, "the inc/dec actuator has 5 actions");
+    if (c->g_min < 0 || c->g_max >= c->n_levels || c->g_max <= 0 || c->g_min > c->g_max ||
+        c->level_init < c->g_min || c->level_init > c->g_max)
+      return fail(PE_EINVAL, "group-size range [g_min, g_max] invalid");
+    if (c->b_min < 1 || c->b_min > c->b_max || c->b_init < c->b_min || c->b_init > c->b_max ||
+        (c->obs_kind == PE_OBS_7B16 && c->b_max == c->b_min))
+      return fail(PE_EINVAL, "batch range [b_min, b_max] invalid");
+  } else if (c->actuator_kind == PE_ACT_SET_LEVEL) {
+    if (c->n_actions < 1 || c->n_actions > c->n_levels) return fail(PE_EINVAL, "n_actions must be in [1, n_levels]");
+    if (c->obs_kind == PE_OBS_TINY8 && c->n_levels < 2) return fail(PE_EINVAL, "TINY8 needs >= 2 levels");
+  } else {
+    return fail(PE_EINVAL, "unknown actuator_kind %d", c->actuator_kind);
+  }
+  if (c->obs_kind == PE_OBS_7B16 && c->actuator_kind != PE_ACT_INCDEC)
+    return fail(PE_EINVAL, "7B16 observations need the inc/dec actuator");
+  if (c->budget_q < 1 || (int64_t)c->budget_q * kWLong * PE_MAX_CHANNELS >= INT32_MAX)
+    return fail(PE_EINVAL, "budget_q out of range");
+  if (c->reward_kind != PE_REWARD_FIXED && c->reward_kind != PE_REWARD_LAGRANGE)
+    return fail(PE_EINVAL, "unknown reward_kind");
+  if (c->reward_window != 1 && c->reward_window != kWLong) return fail(PE_EINVAL, "reward_window must be 1 or 60");
+  return PE_OK;
+}
+
+pe_status pe_env_create(const pe_env_config* cfg, const float* trace, const uint8_t* phase,
+                        pe_env** out) {
+  clear_error();
+  if (!cfg || !trace || !phase || !out) return fail(PE_EINVAL, "null argument");
+  *out = nullptr;
+  pe_status s = check_env_config(cfg);
+  if (s != PE_OK) return s;
+  const int C = cfg->n_channels, L = cfg->trace_len, E = cfg->n_envs;
+  // host copies for validation (trace and phase may live in host or device memory)
+  std::vector<float> h((size_t)C * L);
+  std::vector<uint8_t> ph((size_t)L);
+  PE_TRY_CUDA(cudaMemcpy(h.data(), trace, sizeof(float) * h.size(), cudaMemcpyDefault));
+  PE_TRY_CUDA(cudaMemcpy(ph.data(), phase, ph.size(), cudaMemcpyDefault));
+  for (int i = 0; i < L; ++i)
+    if (ph[i] > 7) return fail(PE_EINVAL, "phase label %d at %d outside [0, 7]", (int)ph[i], i);
+  pe_env* env = new pe_env();
+  env->cfg = *cfg;
+  EnvDev& d = env->dev;
+  memset(&d, 0, sizeof(d));
+  d.E = E; d.C = C; d.L = L; d.A = cfg->n_actions; d.obs_kind = cfg->obs_kind;
+  d.act_kind = cfg->actuator_kind; d.n_levels = cfg->n_levels; d.level_init = cfg->level_init;
+  d.g_min = cfg->g_min; d.g_max = cfg->g_max; d.b_min = cfg->b_min; d.b_max = cfg->b_max;
+  d.b_init = cfg->b_init; d.ep_len = cfg->episode_len; d.budget_q = cfg->budget_q;
+  d.phase_mask = cfg->scale_phase_mask; d.reward_kind = cfg->reward_kind;
+  d.reward_window = cfg->reward_window; d.r_ok = cfg->r_ok; d.r_viol = cfg->r_viol;
+  d.bonus_coef = cfg->bonus_coef; d.seed = cfg->seed;
+  // actuator table: Sec. 4.1 formula for the group-size actuator, else the given table
+  for (int l = 0; l < PE_MAX_LEVELS; ++l)
+    for (int c = 0; c < PE_MAX_CHANNELS; ++c) {
+      if (cfg->actuator_kind == PE_ACT_INCDEC)
+        d.scale[l][c] = (float)(0.8 + 0.2 * (double)l / (double)cfg->g_max);
+      else
+        d.scale[l][c] = cfg->level_scale[l][c];
+    }
+  for (int l = 0; l < PE_MAX_LEVELS; ++l) d.tokens[l] = cfg->level_tokens[l];
+  double rmax = 0.0;
+  if (cfg->actuator_kind == PE_ACT_INCDEC) {
+    for (int l = cfg->g_min; l <= cfg->g_max; ++l)
+      rmax = fmax(rmax, (double)cfg->level_tokens[l] * cfg->b_max / cfg->b_init);
+  } else {
+    for (int l = 0; l < cfg->n_levels; ++l) rmax = fmax(rmax, (double)cfg->level_tokens[l]);
+  }
+  d.inv_rate_max = rmax > 0 ? (float)(1.0 / rmax) : 0.0f;
+  // fixed-point range: every actuated sample and every 60-sample cluster sum must fit in int32
+  double qmax = 0.0;
+  for (int c = 0; c < C; ++c) {
+    float smax = 1.0f;
+    for (int l = 0; l < cfg->n_levels; ++l) smax = fmaxf(smax, d.scale[l][c]);
+    if (!(smax >= 0.0f) || !std::isfinite(smax)) { delete env; return fail(PE_EINVAL, "actuator scale not finite"); }
+    for (int i = 0; i < L; ++i) {
+      const float x = h[(size_t)c * L + i];
+      if (!std::isfinite(x) || x < 0.0f) { delete env; return fail(PE_EOVERFLOW, "trace sample (%d, %d) is not a finite non-negative power", c, i); }
+      qmax = fmax(qmax, (double)x * smax * 64.0);
+    }
+  }
+  if (qmax * C * kWLong >= 2147483000.0) { delete env; return fail(PE_EOVERFLOW, "trace too large for the 1/64 W fixed point"); }
+  cudaError_t e1 = cudaGetDevice(&env->device);
+  float* dtrace = nullptr;
+  uint8_t* dphase = nullptr;
+  int32_t* st = nullptr;
+  uint8_t* ring = nullptr;
+  int32_t* sums = nullptr;
+  if (e1 == cudaSuccess) e1 = cudaMalloc(&dtrace, sizeof(float) * h.size());
+  if (e1 == cudaSuccess) e1 = cudaMalloc(&dphase, ph.size());
+  if (e1 == cudaSuccess) e1 = cudaMalloc(&st, sizeof(int32_t) * kStN * (size_t)E);
+  if (e1 == cudaSuccess) e1 = cudaMalloc(&ring, (size_t)kRing * E);
+  if (e1 == cudaSuccess) e1 = cudaMalloc(&sums, sizeof(int32_t) * 8 * (size_t)E);
+  if (e1 != cudaSuccess) {
+    cudaFree(dtrace); cudaFree(dphase); cudaFree(st); cudaFree(ring); cudaFree(sums);
+    delete env;
+    return e1 == cudaErrorMemoryAllocation ? fail(PE_ENOMEM, "device allocation failed")
+                                           : cuda_fail(e1, "pe_env_create");
+  }
+  d.trace = dtrace; d.phase = dphase; d.st = st; d.ring = ring; d.sums = sums;
+  PE_TRY_CUDA(cudaMemcpy(dtrace, h.data(), sizeof(float) * h.size(), cudaMemcpyHostToDevice));
+  PE_TRY_CUDA(cudaMemcpy(dphase, ph.data(), ph.size(), cudaMemcpyHostToDevice));
+  env_init_kernel<<<ceil_div(E, 256), 256>>>(d);  // one-time set-up, not profiled
+  PE_CHECK_LAUNCH("env_init_kernel");
+  PE_TRY_CUDA(cudaDeviceSynchronize());
+  *out = env;
+  return PE_OK;
+}
+
+pe_status pe_env_destroy(pe_env* env) {
+  clear_error();
+  if (!env) return PE_OK;
+  cudaFree((void*)env->dev.trace);
+  cudaFree((void*)env->dev.phase);
+  cudaFree(env->dev.st);
+  cudaFree(env->dev.ring);
+  cudaFree(env->dev.sums);
+  delete env;
+  return PE_OK;
+}
+
+int64_t pe_env_state_bytes(const pe_env* env) {
+  if (!env) return -1;
+  return (int64_t)env->dev.E * (kStN * 4 + kRing + 8 * 4);
+}
+
+pe_status pe_env_save(const pe_env* env, void* host_dst) {
+  clear_error();
+  if (!env || !host_dst) return fail(PE_EINVAL, "null argument");
+  const size_t E = (size_t)env->dev.E;
+  char* p = reinterpret_cast<char*>(host_dst);
+  PE_TRY_CUDA(cudaDeviceSynchronize());
+  PE_TRY_CUDA(cudaMemcpy(p, env->dev.st, E * kStN * 4, cudaMemcpyDeviceToHost));
+  PE_TRY_CUDA(cudaMemcpy(p + E * kStN * 4, env->dev.ring, E * kRing, cudaMemcpyDeviceToHost));
+  PE_TRY_CUDA(cudaMemcpy(p + E * (kStN * 4 + kRing), env->dev.sums, E * 32, cudaMemcpyDeviceToHost));
+  return PE_OK;
+}
+
+pe_status pe_env_load(pe_env* env, const void* host_src) {
+  clear_error();
+  if (!env || !host_src) return fail(PE_EINVAL, "null argument");
+  const size_t E = (size_t)env->dev.E;
+  const char* p = reinterpret_cast<const char*>(host_src);
+  const int32_t* st = reinterpret_cast<const int32_t*>(p);
+  const uint8_t* ring = reinterpret_cast<const uint8_t*>(p + E * kStN * 4);
+  const pe_env_config& c = env->cfg;
+  for (size_t e = 0; e < E; ++e) {
+    const int32_t pos = st[kStPos * E + e], k = st[kStK * E + e];
+    if (pos < kWLong || pos + (c.episode_len - k) > c.trace_len || k < 0 || k >= c.episode_len)
+      return fail(PE_EINVAL, "state image: env %zu has an invalid position", e);
+    for (int f = kStLevel; f <= kStPrev; ++f)
+      if (st[f * E + e] < 0 || st[f * E + e] >= c.n_levels) return fail(PE_EINVAL, "state image: bad level");
+    for (int i = 0; i < kRing; ++i)
+      if (ring[e * kRing + i] >= c.n_levels) return fail(PE_EINVAL, "state image: bad level ring");
+  }
+  PE_TRY_CUDA(cudaDeviceSynchronize());
+  PE_TRY_CUDA(cudaMemcpy(env->dev.st, p, E * kStN * 4, cudaMemcpyHostToDevice));
+  PE_TRY_CUDA(cudaMemcpy(env->dev.ring, p + E * kStN * 4, E * kRing, cudaMemcpyHostToDevice));
+  PE_TRY_CUDA(cudaMemcpy(env->dev.sums, p + E * (kStN * 4 + kRing), E * 32, cudaMemcpyHostToDevice));
+  return PE_OK;
+}
+
+static pe_status check_net(const pe_net* net) {
+  if (!net) return fail(PE_EINVAL, "null network");
+  if (net->obs_dim < 1 || net->hidden < 4 || net->n_actions < 1 || (net->dtype != PE_F32 && net->dtype != PE_BF16))
+    return fail(PE_EINVAL, "invalid network description");
+  return PE_OK;
+}
+
+pe_status pe_rollout(pe_env* env, const pe_net* net, const float* params, int32_t horizon,
+                     uint32_t iteration, float lambda, int32_t flags, const pe_rollout_buf* buf,
+                     void* stream) {
+  clear_error();
+  if (!env || !params || !buf) return fail(PE_EINVAL, "null argument");
+  pe_status s = check_net(net);
+  if (s != PE_OK) return s;
+  if (horizon < 1) return fail(PE_EINVAL, "horizon must be >= 1");
+  if (net->obs_dim != obs_width(env->cfg.obs_kind) || net->n_actions != env->cfg.n_actions)
+    return fail(PE_EINVAL, "network does not match the env (obs_dim %d vs %d, actions %d vs %d)",
+                net->obs_dim, obs_width(env->cfg.obs_kind), net->n_actions, env->cfg.n_actions);
+  if (!buf->obs || !buf->obs_last || !buf->act || !buf->logp || !buf->value || !buf->last_value ||
+      !buf->reward || !buf->done || !buf->viol || !buf->tokens || !buf->excess || !buf->energy_q)
+    return fail(PE_EINVAL, "null rollout buffer field");
+  if ((int64_t)horizon * env->dev.E > (int64_t)INT32_MAX) return fail(PE_EINVAL, "horizon * n_envs too large");
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  const int det = (flags & PE_ROLLOUT_DETERMINISTIC) ? 1 : 0;
+  if (net->dtype == PE_F32) {
+    s = rollout_f32(env->dev, *net, params, horizon, iteration, lambda, det, *buf, st);
+    if (s != PE_OK) return s;
+    s = value_f32(*net, params, reinterpret_cast<const float*>(buf->obs), (int64_t)horizon * env->dev.E,
+                  buf->value, st);
+    if (s != PE_OK) return s;
+    return value_f32(*net, params, reinterpret_cast<const float*>(buf->obs_last), env->dev.E,
+                     buf->last_value, st);
+  }
+  return fail(PE_EINVAL, "bf16 networks are not supported by pe_rollout in this build");
+}
+
+pe_status pe_value(const pe_net* net, const float* params, const void* obs, int64_t n,
+                   float* value, void* stream) {
+  clear_error();
+  pe_status s = check_net(net);
+  if (s != PE_OK) return s;
+  if (!params || (n > 0 && (!obs || !value))) return fail(PE_EINVAL, "null argument");
+  if (n < 0) return fail(PE_EINVAL, "n must be >= 0");
+  if (net->dtype == PE_F32)
+    return value_f32(*net, params, reinterpret_cast<const float*>(obs), n, value,
+                     reinterpret_cast<cudaStream_t>(stream));
+  return fail(PE_EINVAL, "bf16 networks are not supported by pe_value in this build");
+}
+
+pe_status pe_gae(const float* reward, const float* value, const uint8_t* done,
+                 const float* last_value, int32_t T, int32_t E, float gamma, float lam,
+                 float* adv, float* ret, void* stream) {
+  clear_error();
+  if (T < 0 || E < 0) return fail(PE_EINVAL, "T and E must be >= 0");
+  if (T == 0 || E == 0) return PE_OK;
+  if (!reward || !value || !done || !last_value || !adv || !ret) return fail(PE_EINVAL, "null argument");
+  if ((int64_t)T * E > (int64_t)1 << 40) return fail(PE_EINVAL, "T * E too large");
+  if (!std::isfinite(gamma) || !std::isfinite(lam)) return fail(PE_EINVAL, "gamma and lambda must be finite");
+  return gae_launch(reward, value, done, last_value, T, E, gamma, lam, adv, ret,
+                    reinterpret_cast<cudaStream_t>(stream));
+}
+
+static pe_status check_ppo(const pe_net* net, const pe_ppo_config* cfg, int64_t n) {
+  pe_status s = check_net(net);
+  if (s != PE_OK) return s;
+  if (!cfg) return fail(PE_EINVAL, "null PPO config");
+  if (cfg->epochs < 1 || cfg->epochs > 16) return fail(PE_EINVAL, "epochs must be in [1, 16]");
+  if (cfg->minibatch < 1) return fail(PE_EINVAL, "minibatch must be >= 1");
+  if (n < 1 || n > (int64_t)INT32_MAX) return fail(PE_EINVAL, "n_samples must be in [1, 2^31)");
+  if (net->dtype != PE_F32) return fail(PE_EINVAL, "bf16 networks are not supported by pe_ppo_update in this build");
+  return PE_OK;
+}
+
+int64_t pe_ppo_workspace_bytes(const pe_net* net, const pe_ppo_config* cfg, int64_t n_samples) {
+  if (check_ppo(net, cfg, n_samples) != PE_OK) return -1;
+  return ppo_ws_bytes_f32(*net, *cfg, n_samples);
+}
+
+pe_status pe_ppo_update(const pe_net* net, float* params, float* adam_m, float* adam_v,
+                        int64_t adam_t, const void* obs, const uint8_t* act,
+                        const float* logp_old, const float* adv, const float* ret,
+                        int64_t n_samples, const pe_ppo_config* cfg, float* stats,
+                        void* workspace, int64_t workspace_bytes, void* stream) {
+  clear_error();
+  pe_status s = check_ppo(net, cfg, n_samples);
+  if (s != PE_OK) return s;
+  if (!params || !adam_m || !adam_v || !obs || !act || !logp_old || !adv || !ret || !stats || !workspace)
+    return fail(PE_EINVAL, "null argument");
+  if (adam_t < 0) return fail(PE_EINVAL, "adam_t must be >= 0");
+  const int64_t need = ppo_ws_bytes_f32(*net, *cfg, n_samples);
+  if (workspace_bytes < need) return fail(PE_EINVAL, "workspace too small (%lld < %lld bytes)", (long long)workspace_bytes, (long long)need);
+  return ppo_update_f32(*net, params, adam_m, adam_v, adam_t, reinterpret_cast<const float*>(obs),
+                        act, logp_old, adv, ret, n_samples, *cfg, stats, workspace,
+                        reinterpret_cast<cudaStream_t>(stream));
+}
+
+int64_t pe_fleet_workspace_bytes(int32_t J, int32_t L, int32_t H) {
+  if (J < 1 || L < 1 || H < 0) return -1;
+  return fleet_ws_bytes(J, L, H);
+}
+
+pe_status pe_fleet_windows(const float* traces, int32_t G, int32_t L, const int32_t* job_of_gpu,
+                           int32_t J, const int32_t* offsets, int64_t N, int32_t H,
+                           const int32_t* windows, int32_t W, int64_t budget_q,
+                           int32_t* counts, int32_t* peaks, void* workspace,
+                           int64_t workspace_bytes, void* stream) {
+  clear_error();
+  if (G < 1 || G > 64) return fail(PE_EINVAL, "G must be in [1, 64]");
+  if (J < 1 || J > 32 || J > G) return fail(PE_EINVAL, "J must be in [1, min(32, G)]");
+  if (L < 1 || H < 0 || N < 0) return fail(PE_EINVAL, "L >= 1, H >= 0 and N >= 0 required");
+  if ((int64_t)L + H > (int64_t)INT32_MAX) return fail(PE_EINVAL, "L + H too large");
+  if (W < 1 || W > 4 || !windows) return fail(PE_EINVAL, "W must be in [1, 4] with a host window array");
+  for (int k = 0; k < W; ++k)
+    if (windows[k] < 1 || windows[k] > 992) return fail(PE_EINVAL, "window %d outside [1, 992]", windows[k]);
+  if (budget_q < 0) return fail(PE_EINVAL, "budget_q must be >= 0");
+  if (!traces || !job_of_gpu || !workspace || (N > 0 && (!offsets || !counts || !peaks)))
+    return fail(PE_EINVAL, "null argument");
+  if (workspace_bytes < fleet_ws_bytes(J, L, H)) return fail(PE_EINVAL, "workspace too small");
+  return fleet_launch(traces, G, L, job_of_gpu, J, offsets, N, H, windows, W, budget_q, counts,
+                      peaks, workspace, reinterpret_cast<cudaStream_t>(stream));
+}
+
+}  // extern "C"

@@ -1,0 +1,300 @@
+// Environment of the batched power-control MDP: device-side definitions
+// shared by the rollout kernels (fp32 FFMA networks and bf16 tensor-core
+// networks).
+//
+// One environment step consumes one half-second sample of a power trace
+// (Sec. 4.1 trace replay).  Actuated power is held in 1/64 W integers, so the
+// trailing window sums of Eq. 1 (10 s = 20 samples, 30 s = 60 samples) and
+// the violation indicators of Eq. 2 are exact.
+#pragma once
+
+#include "common.cuh"
+
+namespace pe {
+
+constexpr int kWShort = 20;  // 10 s
+constexpr int kWLong = 60;   // 30 s
+constexpr int kRing = 64;    // per-env ring of the last 64 samples (>= kWLong)
+
+// everything a rollout kernel needs to know about the envs (passed by value)
+struct EnvDev {
+  int32_t E, C, L, A, obs_kind, act_kind, n_levels, level_init;
+  int32_t g_min, g_max, b_min, b_max, b_init, ep_len, budget_q, phase_mask;
+  int32_t reward_kind, reward_window;
+  float r_ok, r_viol, bonus_coef, inv_rate_max;
+  float scale[PE_MAX_LEVELS][PE_MAX_CHANNELS];  // actuator table (INCDEC formula pre-evaluated)
+  float tokens[PE_MAX_LEVELS];
+  uint64_t seed;
+  const float* trace;    // [C][L]
+  const uint8_t* phase;  // [L]
+  // persistent env state, SoA
+  int32_t* st;     // [6][E]: pos, k, level, prev, b, til
+  uint8_t* ring;   // [E][64]: level used for the sample at position p (slot p & 63)
+  int32_t* sums;   // [E][8]: s_short[4], s_long[4] (per channel)
+};
+
+enum { kStPos = 0, kStK, kStLevel, kStPrev, kStB, kStTil, kStN };
+
+// Per-tile env state staged in shared memory for the whole horizon.
+template <int TE, int C>
+struct EnvTile {
+  int32_t pos[TE], k[TE], level[TE], prev[TE], b[TE], til[TE];
+  int32_t s_short[TE][4], s_long[TE][4];
+  int32_t q[TE][C][kRing];  // actuated per-channel samples of positions p-64..p-1, slot p & 63
+  uint8_t ring[TE][kRing];  // level of each of those samples
+};
+
+__device__ __forceinline__ float actuator_scale(const EnvDev& env, int level, int c, int ph) {
+  return ((env.phase_mask >> ph) & 1) ? env.scale[level][c] : 1.0f;
+}
+
+__device__ __forceinline__ int32_t sample_q(const EnvDev& env, int c, int pos, int level) {
+  const float x = __ldg(env.trace + (int64_t)c * env.L + pos);
+  return quant64(x, actuator_scale(env, level, c, __ldg(env.phase + pos)));
+}
+
+// rebuild the 60-sample history of env slot e from its level ring
+template <int TE, int C>
+__device__ void rebuild_history(const EnvDev& env, EnvTile<TE, C>& s, int e) {
+  const int p = s.pos[e];
+  for (int c = 0; c < C; ++c) {
+    int32_t ss = 0, sl = 0;
+    for (int i = 1; i <= kWLong; ++i) {
+      const int pp = p - i;
+      const int32_t q = sample_q(env, c, pp, s.ring[e][pp & (kRing - 1)]);
+      s.q[e][c][pp & (kRing - 1)] = q;
+      sl += q;
+      if (i <= kWShort) ss += q;
+    }
+    s.s_short[e][c] = ss;
+    s.s_long[e][c] = sl;
+  }
+}
+
+// new episode for env slot e (global index eg): Philox offset, warm start
+template <int TE, int C>
+__device__ void env_reset(const EnvDev& env, EnvTile<TE, C>& s, int e, uint32_t eg, uint32_t t,
+                          uint32_t it, uint32_t purpose) {
+  const uint32_t u = draw32(env.seed, eg, t, it, purpose);
+  const uint32_t span = (uint32_t)(env.L - env.ep_len - kWLong + 1);
+  const int o = kWLong + (int)__umulhi(u, span);
+  s.pos[e] = o;
+  s.k[e] = 0;
+  s.level[e] = env.level_init;
+  s.prev[e] = env.level_init;
+  s.b[e] = env.b_init;
+  s.til[e] = 0;
+  for (int i = 0; i < kRing; ++i) s.ring[e][i] = (uint8_t)env.level_init;
+  rebuild_history<TE, C>(env, s, e);
+}
+
+template <int TE, int C>
+__device__ __forceinline__ int32_t Qc(const EnvTile<TE, C>& s, int e, int c, int i) {
+  return s.q[e][c][(s.pos[e] - 1 - i) & (kRing - 1)];
+}
+
+template <int TE, int C>
+__device__ __forceinline__ int32_t Qcl(const EnvTile<TE, C>& s, int e, int i) {
+  int32_t v = 0;
+#pragma unroll
+  for (int c = 0; c < C; ++c) v += Qc<TE, C>(s, e, c, i);
+  return v;
+}
+
+// Observation feature f of env slot e (fp32 quotient of exact integers;
+// all power quantities are normalised by the budget B).
+//   TINY8 (Sec. 4.1): 5 latest samples, headroom, phase, level
+//   7B16: 8 latest samples, 30 s mean, 30 s slack, phase, G, b, 10 s mean, 5 s slope, 0
+//   OCC32/OCC64: Eq. 5 eight-vector, then per-channel recent samples and means
+template <int TE, int C, int OBS>
+__device__ __forceinline__ float feature(const EnvDev& env, const EnvTile<TE, C>& s, int e, int f) {
+  const int64_t B = env.budget_q;
+  if (OBS == PE_OBS_TINY8) {
+    if (f < 5) return ratio_i(Qcl<TE, C>(s, e, 4 - f), B);
+    if (f == 5) return ratio_i(B - Qcl<TE, C>(s, e, 0), B);
+    if (f == 6) return (float)__ldg(env.phase + s.pos[e] - 1);
+    return ratio_i(s.level[e], env.n_levels - 1);
+  }
+  int64_t S20 = 0, S60 = 0;
+#pragma unroll
+  for (int c = 0; c < C; ++c) {
+    S20 += s.s_short[e][c];
+    S60 += s.s_long[e][c];
+  }
+  if (OBS == PE_OBS_7B16) {
+    if (f < 8) return ratio_i(Qcl<TE, C>(s, e, 7 - f), B);
+    switch (f) {
+      case 8: return ratio_i(S60, kWLong * B);
+      case 9: return ratio_i(kWLong * B - S60, kWLong * B);
+      case 10: return (float)__ldg(env.phase + s.pos[e] - 1);
+      case 11: return ratio_i(s.level[e] - env.g_min, env.g_max - env.g_min);
+      case 12: return ratio_i(s.b[e] - env.b_min, env.b_max - env.b_min);
+      case 13: return ratio_i(S20, kWShort * B);
+      case 14: return ratio_i((int64_t)Qcl<TE, C>(s, e, 0) - Qcl<TE, C>(s, e, 10), B);
+      default: return 0.0f;
+    }
+  }
+  // OCC32 / OCC64 (Eq. 5 core)
+  switch (f) {
+    case 0: return ratio_i(Qcl<TE, C>(s, e, 0), B);
+    case 1: return ratio_i(S20, kWShort * B);
+    case 2: return ratio_i(S60, kWLong * B);
+    case 3: return ratio_i(kWLong * B - S60, kWLong * B);
+    case 4: return ratio_i((int64_t)Qcl<TE, C>(s, e, 0) - Qcl<TE, C>(s, e, 10), B);
+    case 5: return ratio_i(s.level[e] + 1, env.n_levels);
+    case 6: return ratio_i(s.prev[e] + 1, env.n_levels);
+    case 7: return fminf(ratio_i(s.til[e], 40), 1.0f);
+    default: break;
+  }
+  if (OBS == PE_OBS_OCC32) {
+    if (f < 24) {
+      const int c = (f - 8) >> 2, i = (f - 8) & 3;
+      return c < C ? ratio_i((int64_t)C * Qc<TE, C>(s, e, c, 3 - i), B) : 0.0f;
+    }
+    if (f < 28) {
+      const int c = f - 24;
+      return c < C ? ratio_i((int64_t)C * s.s_long[e][c], kWLong * B) : 0.0f;
+    }
+    return 0.0f;
+  }
+  // OCC64
+  if (f < 56) {
+    const int c = (f - 8) / 12, i = (f - 8) % 12;
+    return c < C ? ratio_i((int64_t)C * Qc<TE, C>(s, e, c, 11 - i), B) : 0.0f;
+  }
+  if (f < 60) {
+    const int c = f - 56;
+    return c < C ? ratio_i((int64_t)C * s.s_short[e][c], kWShort * B) : 0.0f;
+  }
+  const int c = f - 60;
+  return c < C ? ratio_i((int64_t)C * s.s_long[e][c], kWLong * B) : 0.0f;
+}
+
+struct StepOut {
+  float reward, tokens, excess;
+  int32_t q, v1, v60, done;
+};
+
+// Apply action a to env slot e and consume one sample (Sec. 4.1 actuator and
+// action set with the Sec. 4.2 floor g_min; Eqs. 1-3; G1 or Eq. 6 reward).
+template <int TE, int C>
+__device__ __forceinline__ StepOut env_step(const EnvDev& env, EnvTile<TE, C>& s, int e, int a,
+                                            float lambda) {
+  int nl = s.level[e];
+  if (env.act_kind == PE_ACT_INCDEC) {
+    if (a == 1 && nl > env.g_min) --nl;
+    if (a == 2 && nl < env.g_max) ++nl;
+    if (a == 3 && s.b[e] > env.b_min) s.b[e] -= 1;
+    if (a == 4 && s.b[e] < env.b_max) s.b[e] += 1;
+  } else {
+    nl = a;
+  }
+  s.til[e] = (nl != s.level[e]) ? 0 : s.til[e] + 1;
+  s.prev[e] = s.level[e];
+  s.level[e] = nl;
+  const int p = s.pos[e];
+  const int ph = __ldg(env.phase + p);
+  s.ring[e][p & (kRing - 1)] = (uint8_t)nl;
+  int32_t Q = 0;
+  int64_t S60 = 0;
+#pragma unroll
+  for (int c = 0; c < C; ++c) {
+    const int32_t qin = quant64(__ldg(env.trace + (int64_t)c * env.L + p), actuator_scale(env, nl, c, ph));
+    const int32_t q20 = s.q[e][c][(p - kWShort) & (kRing - 1)];
+    const int32_t q60 = s.q[e][c][(p - kWLong) & (kRing - 1)];
+    s.s_short[e][c] += qin - q20;
+    s.s_long[e][c] += qin - q60;
+    s.q[e][c][p & (kRing - 1)] = qin;
+    Q += qin;
+    S60 += s.s_long[e][c];
+  }
+  const int64_t B60 = (int64_t)kWLong * env.budget_q;
+  StepOut o;
+  o.q = Q;
+  o.v1 = Q > env.budget_q;
+  o.v60 = S60 > B60;
+  const float exc_w = o.v60 ? __fdiv_rn(__ll2float_rn(S60 - B60), 3840.0f) : 0.0f;  // watts over B
+  o.excess = exc_w * 0.5f;                                                            // Eq. 3, W*s
+  float rate = env.tokens[nl];
+  if (env.act_kind == PE_ACT_INCDEC) rate = __fdiv_rn(rate * (float)s.b[e], (float)env.b_init);
+  o.tokens = ph == 0 ? rate : 0.0f;
+  if (env.reward_kind == PE_REWARD_LAGRANGE) {
+    o.reward = o.tokens / 1000.0f - lambda * o.excess - 2.0f * lambda * exc_w;  // Eq. 6
+  } else {
+    const int viol = env.reward_window == 1 ? o.v1 : o.v60;
+    o.reward = (viol ? env.r_viol : env.r_ok) + env.bonus_coef * rate * env.inv_rate_max;
+  }
+  s.pos[e] = p + 1;
+  s.k[e] += 1;
+  o.done = s.k[e] == env.ep_len;
+  return o;
+}
+
+template <int TE, int C>
+__device__ void load_tile(const EnvDev& env, EnvTile<TE, C>& s, int e0, int ne) {
+  for (int e = threadIdx.x; e < ne; e += blockDim.x) {
+    const int g = e0 + e;
+    s.pos[e] = env.st[kStPos * env.E + g];
+    s.k[e] = env.st[kStK * env.E + g];
+    s.level[e] = env.st[kStLevel * env.E + g];
+    s.prev[e] = env.st[kStPrev * env.E + g];
+    s.b[e] = env.st[kStB * env.E + g];
+    s.til[e] = env.st[kStTil * env.E + g];
+    for (int i = 0; i < kRing; ++i) s.ring[e][i] = env.ring[(int64_t)g * kRing + i];
+    rebuild_history<TE, C>(env, s, e);
+  }
+}
+
+template <int TE, int C>
+__device__ void store_tile(const EnvDev& env, const EnvTile<TE, C>& s, int e0, int ne) {
+  for (int e = threadIdx.x; e < ne; e += blockDim.x) {
+    const int g = e0 + e;
+    env.st[kStPos * env.E + g] = s.pos[e];
+    env.st[kStK * env.E + g] = s.k[e];
+    env.st[kStLevel * env.E + g] = s.level[e];
+    env.st[kStPrev * env.E + g] = s.prev[e];
+    env.st[kStB * env.E + g] = s.b[e];
+    env.st[kStTil * env.E + g] = s.til[e];
+    for (int i = 0; i < kRing; ++i) env.ring[(int64_t)g * kRing + i] = s.ring[e][i];
+    for (int c = 0; c < 4; ++c) {
+      env.sums[(int64_t)g * 8 + c] = c < C ? s.s_short[e][c] : 0;
+      env.sums[(int64_t)g * 8 + 4 + c] = c < C ? s.s_long[e][c] : 0;
+    }
+  }
+}
+
+// categorical sample by inverse CDF (or argmax), returns action and its log-prob
+template <int A>
+__device__ __forceinline__ int sample_action(const float* z, uint32_t r, bool det, float* logp) {
+  float m = z[0];
+  int amax = 0;
+#pragma unroll
+  for (int j = 1; j < A; ++j)
+    if (z[j] > m) {
+      m = z[j];
+      amax = j;
+    }
+  float S = 0.0f;
+#pragma unroll
+  for (int j = 0; j < A; ++j) S += expf(z[j] - m);
+  int a = A - 1;
+  if (det) {
+    a = amax;
+  } else {
+    const float u = (float)(r >> 8) * (1.0f / 16777216.0f);
+    const float target = u * S;
+    float c = 0.0f;
+#pragma unroll
+    for (int j = 0; j < A; ++j) {
+      c += expf(z[j] - m);
+      if (target < c) {
+        a = j;
+        break;
+      }
+    }
+  }
+  *logp = z[a] - m - logf(S);
+  return a;
+}
+
+}  // namespace pe

@@ -1,0 +1,98 @@
+// fp32 building blocks of the policy/value MLPs (FFMA register tiles over
+// activations held feature-major in shared memory: xT[feature][row]).
+#pragma once
+
+#include "common.cuh"
+
+namespace pe {
+
+// canonical flat parameter layout (row-major W[out][in]):
+//   policy W1[H][D] b1[H] W2[H][H] b2[H] W3[A][H] b3[A]
+//   value  V1[H][D] c1[H] V2[H][H] c2[H] V3[1][H] c3[1]
+struct MlpLayout {
+  int64_t w1, b1, w2, b2, w3, b3, v1, c1, v2, c2, v3, c3, total;
+};
+
+__host__ __device__ __forceinline__ MlpLayout mlp_layout(int D, int H, int A) {
+  MlpLayout L;
+  int64_t o = 0;
+  L.w1 = o; o += (int64_t)H * D;
+  L.b1 = o; o += H;
+  L.w2 = o; o += (int64_t)H * H;
+  L.b2 = o; o += H;
+  L.w3 = o; o += (int64_t)A * H;
+  L.b3 = o; o += A;
+  L.v1 = o; o += (int64_t)H * D;
+  L.c1 = o; o += H;
+  L.v2 = o; o += (int64_t)H * H;
+  L.c2 = o; o += H;
+  L.v3 = o; o += H;
+  L.c3 = o; o += 1;
+  L.total = o;
+  return L;
+}
+
+// dst[k][n] = W[n][k] for W[rows=N][cols=K] in global memory
+__device__ __forceinline__ void load_transposed(const float* __restrict__ W, float* dst, int N, int K) {
+  for (int i = threadIdx.x; i < N * K; i += blockDim.x) {
+    const int k = i / N, n = i % N;
+    dst[i] = __ldg(W + (int64_t)n * K + k);
+  }
+}
+
+__device__ __forceinline__ void load_copy(const float* __restrict__ src, float* dst, int n) {
+  for (int i = threadIdx.x; i < n; i += blockDim.x) dst[i] = __ldg(src + i);
+}
+
+// outT[n][e] = tanh(b[n] + sum_k inT[k][e] * WT[k][n]) for TE rows; each
+// thread owns a 4-row x 4-neuron register tile.  LD is the row stride (in
+// floats) of inT and outT.
+template <int TE, int K, int N, int LD = TE>
+__device__ __forceinline__ void dense_tanh_t(const float* __restrict__ inT, const float* __restrict__ WT,
+                                             const float* __restrict__ bias, float* __restrict__ outT) {
+  constexpr int EG = TE / 4, NG = N / 4;
+  for (int j = threadIdx.x; j < EG * NG; j += blockDim.x) {
+    const int eg = j % EG, ng = j / EG;
+    float acc[4][4];
+#pragma unroll
+    for (int r = 0; r < 4; ++r)
+#pragma unroll
+      for (int c = 0; c < 4; ++c) acc[r][c] = 0.0f;
+#pragma unroll 8
+    for (int k = 0; k < K; ++k) {
+      const float4 x = *reinterpret_cast<const float4*>(inT + k * LD + eg * 4);
+      const float4 w = *reinterpret_cast<const float4*>(WT + k * N + ng * 4);
+      const float xv[4] = {x.x, x.y, x.z, x.w};
+      const float wv[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+      for (int r = 0; r < 4; ++r)
+#pragma unroll
+        for (int c = 0; c < 4; ++c) acc[r][c] = fmaf(xv[r], wv[c], acc[r][c]);
+    }
+#pragma unroll
+    for (int c = 0; c < 4; ++c) {
+      const float bb = bias[ng * 4 + c];
+      float4 o;
+      o.x = tanhf(acc[0][c] + bb);
+      o.y = tanhf(acc[1][c] + bb);
+      o.z = tanhf(acc[2][c] + bb);
+      o.w = tanhf(acc[3][c] + bb);
+      *reinterpret_cast<float4*>(outT + (ng * 4 + c) * LD + eg * 4) = o;
+    }
+  }
+}
+
+// out[e][a] = b[a] + sum_k W[a][k] * hT[k][e]
+template <int TE, int K, int NA, int LD = TE>
+__device__ __forceinline__ void head_t(const float* __restrict__ hT, const float* __restrict__ W,
+                                       const float* __restrict__ bias, float* __restrict__ out) {
+  for (int j = threadIdx.x; j < TE * NA; j += blockDim.x) {
+    const int e = j % TE, a = j / TE;
+    float acc = 0.0f;
+#pragma unroll 8
+    for (int k = 0; k < K; ++k) acc = fmaf(W[a * K + k], hT[k * LD + e], acc);
+    out[e * NA + a] = acc + bias[a];
+  }
+}
+
+}  // namespace pe

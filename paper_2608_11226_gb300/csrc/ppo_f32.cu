@@ -1,0 +1,614 @@
+// PPO update for fp32 policy/value networks (Sec. 4.2; SB3's clipped
+// surrogate, squared-error value loss, entropy bonus, global-norm gradient
+// clipping and Adam).
+//
+// Per minibatch three launches:
+//   1. ppo_grad_kernel: 2*NC CTAs, the first NC differentiate the policy
+//      network, the other NC the value network (their gradients are
+//      independent).  A CTA walks its share of the minibatch in slices of 32
+//      permuted samples (Feistel order), runs forward and backward with the
+//      activations feature-major in shared memory, and keeps its weight
+//      gradient tiles in registers across slices; it writes one fp32 partial
+//      gradient row.
+//   2. ppo_reduce_kernel: fixed-order sum of the NC partial rows (in fp64),
+//      per-block sums of squares for the global norm.  Deterministic.
+//   3. ppo_adam_kernel: global norm, clip factor, Adam step; accumulates the
+//      minibatch statistics.
+// The per-minibatch advantage mean/std (which depend only on the
+// permutation) are computed for all minibatches up front.
+#include <algorithm>
+#include <cmath>
+
+#include "mlp_f32.cuh"
+
+namespace pe {
+
+constexpr int kPpoS = 32;           // samples per slice
+constexpr int kPpoLD = kPpoS + 4;   // row stride of feature-major activations
+constexpr int kPpoNT = 256;         // threads per gradient CTA
+constexpr int kPpoMaxEpochs = 16;
+
+struct FeistelSet {
+  Feistel f[kPpoMaxEpochs];
+};
+
+// deterministic block reduction of a double (fixed shuffle tree + fixed order)
+__device__ __forceinline__ double block_sum_d(double v, double* red) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  const int w = threadIdx.x >> 5, nw = blockDim.x >> 5;
+  __syncthreads();
+  if ((threadIdx.x & 31) == 0) red[w] = v;
+  __syncthreads();
+  double t = 0.0;
+  for (int i = 0; i < nw; ++i) t += red[i];
+  return t;
+}
+
+// advantage mean and 1/(std + 1e-8) (unbiased std) of every minibatch
+__global__ void ppo_advstats_kernel(const float* __restrict__ adv, int64_t N, int M, int nmb,
+                                    FeistelSet perms, float2* __restrict__ out) {
+  __shared__ double red[32];
+  const int mb = blockIdx.x, ep = blockIdx.y;
+  const Feistel& f = perms.f[ep];
+  const int64_t start = (int64_t)mb * M;
+  const int cnt = (int)(N - start < (int64_t)M ? N - start : (int64_t)M);
+  double s = 0.0;
+  for (int j = threadIdx.x; j < cnt; j += blockDim.x) s += (double)__ldg(adv + feistel_index(f, start + j));
+  const double mean = block_sum_d(s, red) / (double)cnt;
+  double q = 0.0;
+  for (int j = threadIdx.x; j < cnt; j += blockDim.x) {
+    const double a = (double)__ldg(adv + feistel_index(f, start + j)) - mean;
+    q += a * a;
+  }
+  const double ss = block_sum_d(q, red);
+  if (threadIdx.x == 0) {
+    if (cnt > 1) {
+      const double sd = sqrt(ss / (double)(cnt - 1));
+      out[ep * nmb + mb] = make_float2((float)mean, (float)(1.0 / (sd + 1e-8)));
+    } else {
+      out[ep * nmb + mb] = make_float2(0.0f, 1.0f);  // a 1-sample minibatch is not normalised
+    }
+  }
+}
+
+// outT[n][e] = (sum_k inT[k][e] W[k][n]) * (1 - hT[n][e]^2): back through a tanh layer
+template <int TE, int K, int N, int LD>
+__device__ __forceinline__ void dense_bwd_t(const float* __restrict__ inT, const float* __restrict__ W,
+                                            const float* __restrict__ hT, float* __restrict__ outT) {
+  constexpr int EG = TE / 4, NG = N / 4;
+  for (int j = threadIdx.x; j < EG * NG; j += blockDim.x) {
+    const int eg = j % EG, ng = j / EG;
+    float acc[4][4] = {};
+#pragma unroll 8
+    for (int k = 0; k < K; ++k) {
+      const float4 x = *reinterpret_cast<const float4*>(inT + k * LD + eg * 4);
+      const float4 w = *reinterpret_cast<const float4*>(W + k * N + ng * 4);
+      const float xv[4] = {x.x, x.y, x.z, x.w};
+      const float wv[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+      for (int r = 0; r < 4; ++r)
+#pragma unroll
+        for (int c = 0; c < 4; ++c) acc[r][c] = fmaf(xv[r], wv[c], acc[r][c]);
+    }
+#pragma unroll
+    for (int c = 0; c < 4; ++c) {
+      float* o = outT + (ng * 4 + c) * LD + eg * 4;
+      const float4 h = *reinterpret_cast<const float4*>(hT + (ng * 4 + c) * LD + eg * 4);
+      float4 r;
+      r.x = acc[0][c] * (1.0f - h.x * h.x);
+      r.y = acc[1][c] * (1.0f - h.y * h.y);
+      r.z = acc[2][c] * (1.0f - h.z * h.z);
+      r.w = acc[3][c] * (1.0f - h.w * h.w);
+      *reinterpret_cast<float4*>(o) = r;
+    }
+  }
+}
+
+// acc[m][n] += sum_s aT[m][s] bT[n][s] with per-thread 4x4 tiles whose rows
+// and columns are interleaved (m = mg + i*M/4, n = ng + j*N/4) so that the
+// float4 loads of one quarter-warp hit distinct shared-memory banks
+template <int M, int N, int NT>
+struct WGradAcc {
+  static constexpr int MG = M / 4, NG = N / 4, JOBS = MG * NG, PER = (JOBS + NT - 1) / NT;
+  float acc[PER][4][4];
+  __device__ __forceinline__ void zero() {
+#pragma unroll
+    for (int q = 0; q < PER; ++q)
+#pragma unroll
+      for (int i = 0; i < 4; ++i)
+#pragma unroll
+        for (int j = 0; j < 4; ++j) acc[q][i][j] = 0.0f;
+  }
+  template <int S, int LD>
+  __device__ __forceinline__ void add(const float* __restrict__ aT, const float* __restrict__ bT) {
+#pragma unroll
+    for (int q = 0; q < PER; ++q) {
+      const int jb = threadIdx.x + q * NT;
+      if (jb < JOBS) {
+        const int mg = jb / NG, ng = jb % NG;
+#pragma unroll 2
+        for (int s = 0; s < S; s += 4) {
+          float4 a[4], b[4];
+#pragma unroll
+          for (int i = 0; i < 4; ++i) a[i] = *reinterpret_cast<const float4*>(aT + (mg + i * MG) * LD + s);
+#pragma unroll
+          for (int j = 0; j < 4; ++j) b[j] = *reinterpret_cast<const float4*>(bT + (ng + j * NG) * LD + s);
+#pragma unroll
+          for (int i = 0; i < 4; ++i)
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+              float v = acc[q][i][j];
+              v = fmaf(a[i].x, b[j].x, v);
+              v = fmaf(a[i].y, b[j].y, v);
+              v = fmaf(a[i].z, b[j].z, v);
+              v = fmaf(a[i].w, b[j].w, v);
+              acc[q][i][j] = v;
+            }
+        }
+      }
+    }
+  }
+  __device__ __forceinline__ void store(float* __restrict__ dst) const {
+#pragma unroll
+    for (int q = 0; q < PER; ++q) {
+      const int jb = threadIdx.x + q * NT;
+      if (jb < JOBS) {
+        const int mg = jb / NG, ng = jb % NG;
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+#pragma unroll
+          for (int j = 0; j < 4; ++j) dst[(int64_t)(mg + i * MG) * N + ng + j * NG] = acc[q][i][j];
+      }
+    }
+  }
+};
+
+template <int D, int H, int A>
+struct PpoSmem {
+  float w1t[D * H], w2t[H * H], w2[H * H], b1[H], b2[H], w3[A * H], b3[(A + 3) / 4 * 4];
+  float xt[D * kPpoLD], h1t[H * kPpoLD], h2t[H * kPpoLD], d2t[H * kPpoLD];
+  float z[kPpoS * A];
+  float lpo[kPpoS], advn[kPpoS], ret[kPpoS];
+  int32_t act[kPpoS], valid[kPpoS];
+  uint32_t idx[kPpoS];
+};
+
+struct PpoArgs {
+  const float* obs;
+  const uint8_t* act;
+  const float* logp_old;
+  const float* adv;
+  const float* ret;
+  const float* params;
+  Feistel perm;
+  int64_t start;
+  int cnt;
+  const float2* advstat;  // (mean, 1/(std+1e-8)) of this minibatch's advantages
+  float clip, vf_coef, ent_coef, inv_cnt;
+  float* partial;       // [NC][P]
+  float* stat_partial;  // [2*NC][8]
+  int NC, slices_per_cta;
+  int64_t P;
+};
+
+template <int D, int H, int A, bool POL>
+__device__ __forceinline__ void ppo_role(PpoSmem<D, H, A>& s, const PpoArgs& g, int c) {
+  constexpr int NA = POL ? A : 1;
+  const MlpLayout Lp = mlp_layout(D, H, A);
+  const int64_t oW1 = POL ? Lp.w1 : Lp.v1, oB1 = POL ? Lp.b1 : Lp.c1;
+  const int64_t oW2 = POL ? Lp.w2 : Lp.v2, oB2 = POL ? Lp.b2 : Lp.c2;
+  const int64_t oW3 = POL ? Lp.w3 : Lp.v3, oB3 = POL ? Lp.b3 : Lp.c3;
+  load_transposed(g.params + oW1, s.w1t, H, D);
+  load_transposed(g.params + oW2, s.w2t, H, H);
+  load_copy(g.params + oW2, s.w2, H * H);
+  load_copy(g.params + oB1, s.b1, H);
+  load_copy(g.params + oB2, s.b2, H);
+  load_copy(g.params + oW3, s.w3, NA * H);
+  load_copy(g.params + oB3, s.b3, NA);
+  const int tid = threadIdx.x;
+  const float2 as = *g.advstat;
+
+  WGradAcc<H, H, kPpoNT> g2;
+  WGradAcc<H, D, kPpoNT> g1;
+  g2.zero();
+  g1.zero();
+  constexpr int PER3 = (NA * H + kPpoNT - 1) / kPpoNT;
+  float g3[PER3], gb1 = 0.0f, gb2 = 0.0f, gb3 = 0.0f;
+#pragma unroll
+  for (int q = 0; q < PER3; ++q) g3[q] = 0.0f;
+  float st_pg = 0.0f, st_ent = 0.0f, st_kl = 0.0f, st_clip = 0.0f, st_v = 0.0f;
+
+  for (int sl = 0; sl < g.slices_per_cta; ++sl) {
+    const int base = (c * g.slices_per_cta + sl) * kPpoS;
+    if (base >= g.cnt) break;
+    __syncthreads();
+    // gather the slice (permuted sample order)
+    for (int i = tid; i < kPpoS; i += blockDim.x) {
+      const int ok = base + i < g.cnt;
+      s.valid[i] = ok;
+      if (ok) {
+        const uint32_t idx = feistel_index(g.perm, g.start + base + i);
+        s.idx[i] = idx;
+        s.act[i] = __ldg(g.act + idx);
+        s.lpo[i] = __ldg(g.logp_old + idx);
+        s.advn[i] = (__ldg(g.adv + idx) - as.x) * as.y;
+        s.ret[i] = __ldg(g.ret + idx);
+      } else {
+        s.idx[i] = 0;
+        s.act[i] = 0;
+        s.lpo[i] = s.advn[i] = s.ret[i] = 0.0f;
+      }
+    }
+    __syncthreads();
+    for (int i = tid; i < kPpoS * D; i += blockDim.x) {
+      const int si = i / D, f = i % D;
+      float v = 0.0f;
+      if (s.valid[si]) v = __ldg(g.obs + (int64_t)s.idx[si] * D + f);
+      s.xt[f * kPpoLD + si] = v;
+    }
+    __syncthreads();
+    // forward
+    dense_tanh_t<kPpoS, D, H, kPpoLD>(s.xt, s.w1t, s.b1, s.h1t);
+    __syncthreads();
+    dense_tanh_t<kPpoS, H, H, kPpoLD>(s.h1t, s.w2t, s.b2, s.h2t);
+    __syncthreads();
+    head_t<kPpoS, H, NA, kPpoLD>(s.h2t, s.w3, s.b3, s.z);
+    __syncthreads();
+    // loss terms and dLoss/dhead per sample
+    if (tid < kPpoS) {
+      float* z = s.z + tid * NA;
+      if (!s.valid[tid]) {
+#pragma unroll
+        for (int j = 0; j < NA; ++j) z[j] = 0.0f;
+      } else if (POL) {
+        float m = z[0];
+#pragma unroll
+        for (int j = 1; j < NA; ++j) m = fmaxf(m, z[j]);
+        float se = 0.0f;
+#pragma unroll
+        for (int j = 0; j < NA; ++j) se += expf(z[j] - m);
+        const float lse = m + logf(se);
+        float lp[NA], p[NA], Hs = 0.0f;
+#pragma unroll
+        for (int j = 0; j < NA; ++j) {
+          lp[j] = z[j] - lse;
+          p[j] = expf(lp[j]);
+          Hs -= p[j] * lp[j];
+        }
+        const int a = s.act[tid];
+        const float an = s.advn[tid];
+        const float logr = lp[a] - s.lpo[tid];
+        const float rho = expf(logr);
+        const float rc = fminf(fmaxf(rho, 1.0f - g.clip), 1.0f + g.clip);
+        const float s1 = rho * an, s2 = rc * an;
+        st_pg += -fminf(s1, s2);
+        st_ent += Hs;
+        st_kl += (rho - 1.0f) - logr;
+        st_clip += fabsf(rho - 1.0f) > g.clip ? 1.0f : 0.0f;
+        const float dlp = (s1 <= s2 ? -an : 0.0f) * rho * g.inv_cnt;
+#pragma unroll
+        for (int j = 0; j < NA; ++j)
+          z[j] = dlp * ((j == a ? 1.0f : 0.0f) - p[j]) + g.ent_coef * g.inv_cnt * p[j] * (lp[j] + Hs);
+      } else {
+        const float V = z[0], R = s.ret[tid];
+        st_v += (R - V) * (R - V);
+        z[0] = g.vf_coef * 2.0f * (V - R) * g.inv_cnt;
+      }
+    }
+    __syncthreads();
+    // head gradient; back through the head into layer 2
+#pragma unroll
+    for (int q = 0; q < PER3; ++q) {
+      const int j = tid + q * kPpoNT;
+      if (j < NA * H) {
+        const int a = j / H, k = j % H;
+        float acc = 0.0f;
+#pragma unroll 8
+        for (int si = 0; si < kPpoS; ++si) acc = fmaf(s.z[si * NA + a], s.h2t[k * kPpoLD + si], acc);
+        g3[q] += acc;
+      }
+    }
+    if (tid < NA) {
+      float acc = 0.0f;
+      for (int si = 0; si < kPpoS; ++si) acc += s.z[si * NA + tid];
+      gb3 += acc;
+    }
+    for (int i = tid; i < H * kPpoS; i += blockDim.x) {
+      const int k = i / kPpoS, si = i % kPpoS;
+      float acc = 0.0f;
+#pragma unroll
+      for (int a = 0; a < NA; ++a) acc = fmaf(s.w3[a * H + k], s.z[si * NA + a], acc);
+      const float h = s.h2t[k * kPpoLD + si];
+      s.d2t[k * kPpoLD + si] = acc * (1.0f - h * h);
+    }
+    __syncthreads();
+    // layer-2 weight gradient; back into layer 1 (written over h2t, now dead)
+    g2.template add<kPpoS, kPpoLD>(s.d2t, s.h1t);
+    if (tid < H) {
+      float acc = 0.0f;
+      for (int si = 0; si < kPpoS; ++si) acc += s.d2t[tid * kPpoLD + si];
+      gb2 += acc;
+    }
+    dense_bwd_t<kPpoS, H, H, kPpoLD>(s.d2t, s.w2, s.h1t, s.h2t);
+    __syncthreads();
+    // layer-1 weight gradient
+    g1.template add<kPpoS, kPpoLD>(s.h2t, s.xt);
+    if (tid < H) {
+      float acc = 0.0f;
+      for (int si = 0; si < kPpoS; ++si) acc += s.h2t[tid * kPpoLD + si];
+      gb1 += acc;
+    }
+  }
+  // partial gradient row of this CTA (its network's slice of the parameter vector)
+  float* row = g.partial + (int64_t)c * g.P;
+  g1.store(row + oW1);
+  g2.store(row + oW2);
+#pragma unroll
+  for (int q = 0; q < PER3; ++q) {
+    const int j = tid + q * kPpoNT;
+    if (j < NA * H) row[oW3 + j] = g3[q];
+  }
+  if (tid < H) {
+    row[oB1 + tid] = gb1;
+    row[oB2 + tid] = gb2;
+  }
+  if (tid < NA) row[oB3 + tid] = gb3;
+  // statistics of the slice samples (held by warp 0), fixed shuffle tree
+  if (tid < 32) {
+    float v[5] = {st_pg, st_ent, st_kl, st_clip, st_v};
+#pragma unroll
+    for (int k = 0; k < 5; ++k)
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) v[k] += __shfl_xor_sync(0xffffffffu, v[k], o);
+    if (tid == 0) {
+      float* sp = g.stat_partial + (int64_t)((POL ? 0 : g.NC) + c) * 8;
+#pragma unroll
+      for (int k = 0; k < 5; ++k) sp[k] = v[k];
+    }
+  }
+}
+
+template <int D, int H, int A>
+__global__ void __launch_bounds__(kPpoNT) ppo_grad_kernel(PpoArgs g) {
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  PpoSmem<D, H, A>& s = *reinterpret_cast<PpoSmem<D, H, A>*>(smem_raw);
+  if ((int)blockIdx.x < g.NC)
+    ppo_role<D, H, A, true>(s, g, blockIdx.x);
+  else
+    ppo_role<D, H, A, false>(s, g, blockIdx.x - g.NC);
+}
+
+__global__ void ppo_reduce_kernel(const float* __restrict__ partial, int NC, int64_t P,
+                                  float* __restrict__ grad, double* __restrict__ sq) {
+  __shared__ double red[32];
+  const int64_t p = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  double gsum = 0.0;
+  if (p < P) {
+    for (int c = 0; c < NC; ++c) gsum += (double)__ldg(partial + (int64_t)c * P + p);
+    grad[p] = (float)gsum;
+  }
+  const float gf = (float)gsum;
+  const double t = block_sum_d((double)gf * (double)gf, red);
+  if (threadIdx.x == 0) sq[blockIdx.x] = t;
+}
+
+struct AdamArgs {
+  float beta1, beta2, step_size, inv_sqrt_bc2, eps, max_norm;
+  float clip, vf_coef, ent_coef, inv_cnt;
+};
+
+__global__ void ppo_adam_kernel(float* __restrict__ params, float* __restrict__ m,
+                                float* __restrict__ v, const float* __restrict__ grad,
+                                const double* __restrict__ sq, int nsq, int64_t P, AdamArgs a,
+                                const float* __restrict__ stat_partial, int NC,
+                                double* __restrict__ acc) {
+  __shared__ double s_norm;
+  if (threadIdx.x < 32) {
+    double t = 0.0;
+    for (int b = threadIdx.x; b < nsq; b += 32) t += sq[b];
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
+    if (threadIdx.x == 0) s_norm = sqrt(t);
+  }
+  __syncthreads();
+  const double norm = s_norm;
+  const float coef = (float)fmin(1.0, (double)a.max_norm / (norm + 1e-6));
+  for (int64_t p = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; p < P;
+       p += (int64_t)gridDim.x * blockDim.x) {
+    const float gp = grad[p] * coef;
+    const float mp = a.beta1 * m[p] + (1.0f - a.beta1) * gp;
+    const float vp = a.beta2 * v[p] + (1.0f - a.beta2) * gp * gp;
+    m[p] = mp;
+    v[p] = vp;
+    params[p] -= a.step_size * mp / (sqrtf(vp) * a.inv_sqrt_bc2 + a.eps);
+  }
+  if (blockIdx.x == 0 && threadIdx.x == 0) {
+    double pg = 0, ent = 0, kl = 0, cf = 0, vl = 0;
+    for (int c = 0; c < NC; ++c) {
+      pg += stat_partial[c * 8 + 0];
+      ent += stat_partial[c * 8 + 1];
+      kl += stat_partial[c * 8 + 2];
+      cf += stat_partial[c * 8 + 3];
+      vl += stat_partial[(NC + c) * 8 + 4];
+    }
+    const double ic = a.inv_cnt;
+    acc[0] += pg * ic;
+    acc[1] += vl * ic;
+    acc[2] += ent * ic;
+    acc[3] += kl * ic;
+    acc[4] += cf * ic;
+    acc[5] += pg * ic + a.vf_coef * vl * ic - a.ent_coef * ent * ic;
+    acc[6] = norm;
+    acc[7] += 1.0;
+  }
+}
+
+__global__ void ppo_finalize_kernel(const double* __restrict__ acc, float* __restrict__ stats) {
+  const int k = threadIdx.x;
+  if (k < 8) {
+    const double n = acc[7] > 0 ? acc[7] : 1.0;
+    stats[k] = (float)(k < 6 ? acc[k] / n : acc[k]);
+  }
+}
+
+// ---------------------------------------------------------------------------
+// host side
+// ---------------------------------------------------------------------------
+Feistel make_feistel(uint64_t n, uint64_t seed, uint32_t epoch, uint32_t iteration) {
+  Feistel f;
+  const u32x4 k = philox10(u32x4{epoch, 0u, iteration, kDrawPerm}, (uint32_t)seed, (uint32_t)(seed >> 32));
+  f.k[0] = k.x;
+  f.k[1] = k.y;
+  f.k[2] = k.z;
+  f.k[3] = k.w;
+  int bits = 2;
+  while ((1ull << bits) < n) ++bits;
+  if (bits & 1) ++bits;
+  f.half = (uint32_t)(bits / 2);
+  f.n = n;
+  return f;
+}
+
+struct PpoPlan {
+  int64_t P, N;
+  int nmb, NC, slices_per_cta, nsq;
+  int64_t off_advstat, off_partial, off_stat, off_grad, off_sq, off_acc, total;
+};
+
+static int64_t align256(int64_t x) { return (x + 255) / 256 * 256; }
+
+static PpoPlan ppo_plan(const pe_net& net, const pe_ppo_config& cfg, int64_t N) {
+  PpoPlan p;
+  p.P = mlp_layout(net.obs_dim, net.hidden, net.n_actions).total;
+  p.N = N;
+  p.nmb = (int)((N + cfg.minibatch - 1) / cfg.minibatch);
+  const int slices = (cfg.minibatch + kPpoS - 1) / kPpoS;
+  p.NC = slices < 64 ? slices : 64;
+  p.slices_per_cta = (slices + p.NC - 1) / p.NC;
+  p.nsq = (int)((p.P + 255) / 256);
+  int64_t o = 0;
+  p.off_advstat = o; o = align256(o + (int64_t)cfg.epochs * p.nmb * 8);
+  p.off_partial = o; o = align256(o + (int64_t)p.NC * p.P * 4);
+  p.off_stat = o; o = align256(o + (int64_t)2 * p.NC * 8 * 4);
+  p.off_grad = o; o = align256(o + p.P * 4);
+  p.off_sq = o; o = align256(o + (int64_t)p.nsq * 8);
+  p.off_acc = o; o = align256(o + 8 * 8);
+  p.total = o;
+  return p;
+}
+
+int64_t ppo_ws_bytes_f32(const pe_net& net, const pe_ppo_config& cfg, int64_t N) {
+  return ppo_plan(net, cfg, N).total;
+}
+
+template <int D, int H, int A>
+static pe_status ppo_run(const pe_net& net, float* params, float* m, float* v, int64_t adam_t,
+                         const float* obs, const uint8_t* act, const float* logp_old,
+                         const float* adv, const float* ret, int64_t N, const pe_ppo_config& cfg,
+                         float* stats, char* ws, cudaStream_t st) {
+  const PpoPlan pl = ppo_plan(net, cfg, N);
+  float2* advstat = reinterpret_cast<float2*>(ws + pl.off_advstat);
+  float* partial = reinterpret_cast<float*>(ws + pl.off_partial);
+  float* stat_partial = reinterpret_cast<float*>(ws + pl.off_stat);
+  float* grad = reinterpret_cast<float*>(ws + pl.off_grad);
+  double* sq = reinterpret_cast<double*>(ws + pl.off_sq);
+  double* acc = reinterpret_cast<double*>(ws + pl.off_acc);
+  PE_TRY_CUDA(cudaMemsetAsync(acc, 0, 8 * sizeof(double), st));
+  FeistelSet perms{};
+  for (int ep = 0; ep < cfg.epochs; ++ep) perms.f[ep] = make_feistel((uint64_t)N, cfg.seed, ep, cfg.iteration);
+  {
+    ProfScope ps(PE_PROF_PPO_OTHER, st);
+    ppo_advstats_kernel<<<dim3(pl.nmb, cfg.epochs), 256, 0, st>>>(adv, N, cfg.minibatch, pl.nmb, perms, advstat);
+  }
+  PE_CHECK_LAUNCH("ppo_advstats_kernel");
+  using Smem = PpoSmem<D, H, A>;
+  auto kern = ppo_grad_kernel<D, H, A>;
+  const int bytes = (int)sizeof(Smem);
+  PE_TRY_CUDA(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes));
+  int dev = 0, sms = 0;
+  PE_TRY_CUDA(cudaGetDevice(&dev));
+  PE_TRY_CUDA(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
+  int64_t t = adam_t;
+  for (int ep = 0; ep < cfg.epochs; ++ep) {
+    for (int mb = 0; mb < pl.nmb; ++mb) {
+      const int64_t start = (int64_t)mb * cfg.minibatch;
+      const int cnt = (int)std::min<int64_t>(cfg.minibatch, N - start);
+      PpoArgs g;
+      g.obs = obs;
+      g.act = act;
+      g.logp_old = logp_old;
+      g.adv = adv;
+      g.ret = ret;
+      g.params = params;
+      g.perm = perms.f[ep];
+      g.start = start;
+      g.cnt = cnt;
+      g.clip = cfg.clip;
+      g.vf_coef = cfg.vf_coef;
+      g.ent_coef = cfg.ent_coef;
+      g.inv_cnt = 1.0f / (float)cnt;
+      g.partial = partial;
+      g.stat_partial = stat_partial;
+      g.NC = pl.NC;
+      g.slices_per_cta = pl.slices_per_cta;
+      g.P = pl.P;
+      g.advstat = advstat + (int64_t)ep * pl.nmb + mb;
+      {
+        ProfScope ps(PE_PROF_PPO_GRAD, st);
+        kern<<<2 * pl.NC, kPpoNT, bytes, st>>>(g);
+      }
+      PE_CHECK_LAUNCH("ppo_grad_kernel");
+      {
+        ProfScope ps(PE_PROF_PPO_REDUCE, st);
+        ppo_reduce_kernel<<<pl.nsq, 256, 0, st>>>(partial, pl.NC, pl.P, grad, sq);
+      }
+      PE_CHECK_LAUNCH("ppo_reduce_kernel");
+      t += 1;
+      const double bc1 = 1.0 - std::pow((double)cfg.beta1, (double)t);
+      const double bc2 = 1.0 - std::pow((double)cfg.beta2, (double)t);
+      AdamArgs a;
+      a.beta1 = cfg.beta1;
+      a.beta2 = cfg.beta2;
+      a.step_size = (float)(cfg.lr / bc1);
+      a.inv_sqrt_bc2 = (float)(1.0 / std::sqrt(bc2));
+      a.eps = cfg.eps;
+      a.max_norm = cfg.max_grad_norm;
+      a.clip = cfg.clip;
+      a.vf_coef = cfg.vf_coef;
+      a.ent_coef = cfg.ent_coef;
+      a.inv_cnt = 1.0f / (float)cnt;
+      const int agrid = (int)std::min<int64_t>((pl.P + 255) / 256, 4 * sms);
+      {
+        ProfScope ps(PE_PROF_PPO_ADAM, st);
+        ppo_adam_kernel<<<agrid, 256, 0, st>>>(params, m, v, grad, sq, pl.nsq, pl.P, a, stat_partial, pl.NC, acc);
+      }
+      PE_CHECK_LAUNCH("ppo_adam_kernel");
+    }
+  }
+  {
+    ProfScope ps(PE_PROF_PPO_OTHER, st);
+    ppo_finalize_kernel<<<1, 32, 0, st>>>(acc, stats);
+  }
+  PE_CHECK_LAUNCH("ppo_finalize_kernel");
+  return PE_OK;
+}
+
+}  // namespace pe
+
+namespace pe {
+
+pe_status ppo_update_f32(const pe_net& net, float* params, float* m, float* v, int64_t adam_t,
+                         const float* obs, const uint8_t* act, const float* logp_old,
+                         const float* adv, const float* ret, int64_t N, const pe_ppo_config& cfg,
+                         float* stats, void* ws, cudaStream_t st) {
+  char* w = reinterpret_cast<char*>(ws);
+  if (net.obs_dim == 8 && net.hidden == 64 && net.n_actions == 3)
+    return ppo_run<8, 64, 3>(net, params, m, v, adam_t, obs, act, logp_old, adv, ret, N, cfg, stats, w, st);
+  if (net.obs_dim == 16 && net.hidden == 128 && net.n_actions == 5)
+    return ppo_run<16, 128, 5>(net, params, m, v, adam_t, obs, act, logp_old, adv, ret, N, cfg, stats, w, st);
+  return fail(PE_EINVAL, "unsupported fp32 PPO network (D=%d H=%d A=%d)", net.obs_dim, net.hidden,
+              net.n_actions);
+}
+
+}  // namespace pe

@@ -1,0 +1,307 @@
+"""Parity of the CUDA path (through the C ABI) with the CPU oracle.
+
+Tolerances (spec bar): integer counts bit-exact; fp32 env, network and
+GAE outputs within 1e-5 relative, measured against max(|ref|, rms(ref)) so
+that near-zero entries do not fail a pure relative test; sampled actions
+agree on >= 99.9% of steps under teacher forcing (the oracle steps with the
+GPU's actions, so one flipped sample cannot cascade).
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle as O
+from paper_2608_11226_gb300 import pe
+from paper_2608_11226_gb300 import workloads as W
+
+pytestmark = pytest.mark.gpu
+TOL = 1e-5
+
+
+def rel_err(gpu, ref):
+    gpu = np.asarray(gpu, np.float64)
+    ref = np.asarray(ref, np.float64)
+    if ref.size == 0:
+        return 0.0
+    floor = np.sqrt(np.mean(ref ** 2)) + 1e-30
+    return float(np.max(np.abs(gpu - ref) / np.maximum(np.abs(ref), floor)))
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    from paper_2608_11226_gb300 import build
+    build.build()
+    assert torch.cuda.is_available()
+    pe.lib()
+
+
+def cpu(t):
+    return t.detach().cpu().numpy()
+
+
+# ------------------------------------------------------------------------ GAE
+@pytest.mark.parametrize("T,E", [(1, 1), (37, 100), (512, 4096), (600, 33), (2048, 70)])
+def test_gae_parity(T, E):
+    g = torch.Generator().manual_seed(T * 1000 + E)
+    r = torch.randn(T, E, generator=g)
+    v = torch.randn(T, E, generator=g)
+    d = (torch.rand(T, E, generator=g) < 0.02).to(torch.uint8)
+    lv = torch.randn(E, generator=g)
+    dev = [x.cuda() for x in (r, v, d, lv)]
+    adv = torch.empty(T, E, device="cuda")
+    ret = torch.empty(T, E, device="cuda")
+    pe.gae(*dev, 0.99, 0.95, adv, ret)
+    torch.cuda.synchronize()
+    ra, rr = O.gae(r.numpy(), v.numpy(), d.numpy(), lv.numpy(), 0.99, 0.95)
+    assert rel_err(cpu(adv), ra) <= TOL
+    assert rel_err(cpu(ret), rr) <= TOL
+
+
+def test_gae_empty_is_noop():
+    z = torch.empty(0, 5, device="cuda")
+    pe.gae(z, z, z.to(torch.uint8), torch.empty(5, device="cuda"), 0.99, 0.95, z, z)
+
+
+# ---------------------------------------------------------------------- fleet
+def _fleet_gpu(fw, windows):
+    traces = torch.from_numpy(fw.traces).cuda()
+    job = torch.from_numpy(fw.job_of_gpu).cuda()
+    off = torch.from_numpy(fw.offsets).cuda()
+    N = fw.offsets.shape[0]
+    counts = torch.empty((N, len(windows)), dtype=torch.int32, device="cuda")
+    peaks = torch.empty_like(counts)
+    ws = torch.empty(pe.fleet_workspace_bytes(fw.n_jobs, fw.traces.shape[1], fw.horizon),
+                     dtype=torch.uint8, device="cuda")
+    pe.fleet_windows(traces, job, fw.n_jobs, off, fw.horizon, windows, fw.budget_q, counts, peaks, ws)
+    torch.cuda.synchronize()
+    return cpu(counts), cpu(peaks)
+
+
+def test_fleet_parity_small_bit_exact():
+    fw = W.make_fleet(n_compositions=77, length=3001, windows=(1, 60, 600))
+    c, p = _fleet_gpu(fw, [1, 60, 600])
+    oc, op = O.fleet_windows(fw.traces, fw.job_of_gpu, fw.n_jobs, fw.offsets, fw.horizon,
+                             fw.windows, fw.budget_q)
+    assert np.array_equal(c, oc) and np.array_equal(p, op)
+
+
+@pytest.mark.parametrize("H", [1, 31, 599, 600, 2500])
+def test_fleet_parity_horizons(H):
+    fw = W.make_fleet(n_compositions=9, length=2500, windows=(1, 60, 600))
+    fw.horizon = H
+    c, p = _fleet_gpu(fw, [1, 7, 60, 600])
+    oc, op = O.fleet_windows(fw.traces, fw.job_of_gpu, fw.n_jobs, fw.offsets, H,
+                             [1, 7, 60, 600], fw.budget_q)
+    assert np.array_equal(c, oc) and np.array_equal(p, op)
+
+
+def test_fleet_parity_full_size_sampled():
+    """380,000-sample traces and 1,000,000 compositions (the full fleet
+    workload); the oracle recomputes a seeded sample of compositions."""
+    fw = W.make_fleet()
+    c, p = _fleet_gpu(fw, [1, 60, 600])
+    rng = np.random.default_rng(11)
+    pick = np.concatenate([[0, 1, fw.offsets.shape[0] - 1],
+                           rng.choice(fw.offsets.shape[0], 5, replace=False)])
+    oc, op = O.fleet_windows(fw.traces, fw.job_of_gpu, fw.n_jobs, fw.offsets[pick], fw.horizon,
+                             fw.windows, fw.budget_q)
+    assert np.array_equal(c[pick], oc) and np.array_equal(p[pick], op)
+    # invariant at every composition: the composed peak never exceeds the
+    # sum of per-job peaks (computed by the oracle per job)
+    q = np.rint(fw.traces * np.float32(64)).astype(np.int64)
+    for wi, w in enumerate((1, 60, 600)):
+        per = 0
+        for j in range(fw.n_jobs):
+            x = q[fw.job_of_gpu == j].sum(0)
+            x = np.concatenate([x, x[:w - 1]])  # the trace tiles circularly
+            per += np.convolve(x, np.ones(w, np.int64), "valid").max()
+        assert p[:, wi].max() <= per
+
+
+def test_fleet_rejects_bad_offsets_and_traces():
+    fw = W.make_fleet(n_compositions=4, length=700)
+    fw.offsets[2, 3] = 700
+    with pytest.raises(pe.PEError) as e:
+        _fleet_gpu(fw, [1, 60])
+    assert e.value.status == pe.PE_EINVAL
+    fw = W.make_fleet(n_compositions=4, length=700)
+    fw.traces[3, 5] = np.nan
+    with pytest.raises(pe.PEError) as e:
+        _fleet_gpu(fw, [1, 60])
+    assert e.value.status == pe.PE_EOVERFLOW
+
+
+# -------------------------------------------------------------------- rollout
+def _rollout_case(wl, T, iters, sample_envs=None, det=False, lam=1.0):
+    spec, net = wl.env, wl.net
+    params = W.init_params(net, seed=1, bias_scale=0.05)
+    env = pe.Env(spec, torch.from_numpy(wl.trace), torch.from_numpy(wl.phase))
+    buf = pe.alloc_rollout(spec, net, T)
+    p_dev = torch.from_numpy(params).cuda()
+    ids = np.arange(spec.n_envs) if sample_envs is None else np.asarray(sample_envs)
+    ora = O.OracleEnv(spec, wl.trace, wl.phase, ids)
+    agree = total = 0
+    for it in range(iters):
+        pe.rollout(env, net, p_dev, T, it, buf, lam=lam, deterministic=det)
+        torch.cuda.synchronize()
+        g = {k: cpu(v) for k, v in buf.items()}
+        forced = g["act"][:, ids]
+        o = ora.rollout(params, net.hidden, net.dtype == 1, T, it, lam=lam, deterministic=det,
+                        forced=forced)
+        gobs = g["obs"][:, ids].astype(np.float32)
+        assert np.array_equal(gobs, o["obs"]), "observations differ"
+        assert np.array_equal(g["obs_last"][ids], o["obs_last"])
+        assert np.array_equal(g["done"][:, ids], o["done"])
+        assert np.array_equal(g["viol"][ids], o["viol"])
+        assert np.array_equal(g["energy_q"][ids], o["energy_q"])
+        assert rel_err(g["reward"][:, ids], o["reward"]) <= TOL
+        assert rel_err(g["tokens"][ids], o["tokens"]) <= TOL
+        assert rel_err(g["excess"][ids], o["excess"]) <= TOL
+        assert rel_err(g["logp"][:, ids], o["logp"]) <= TOL
+        agree += int((o["act_own"] == forced).sum())
+        total += forced.size
+        _, ov = O.mlp_forward(net, params, o["obs"].reshape(-1, net.obs_dim))
+        assert rel_err(g["value"][:, ids].ravel(), ov) <= TOL
+        _, olv = O.mlp_forward(net, params, o["obs_last"])
+        assert rel_err(g["last_value"][ids], olv) <= TOL
+    assert agree / total >= 0.999, agree / total
+    env.close()
+    return agree / total
+
+
+def test_rollout_parity_tiny_full():
+    _rollout_case(W.make_tiny(), 128, iters=5)   # 640 steps: crosses an episode boundary
+
+
+def test_rollout_parity_tiny_ragged_tile():
+    _rollout_case(W.make_tiny(n_envs=45), 3, iters=2)
+
+
+def test_rollout_parity_tiny_deterministic():
+    _rollout_case(W.make_tiny(n_envs=40), 64, iters=1, det=True)
+
+
+def test_rollout_parity_7b_sampled():
+    wl = W.make_7b()
+    rng = np.random.default_rng(3)
+    ids = np.unique(np.concatenate([[0, 31, 32, 4095], rng.choice(4096, 28, replace=False)]))
+    _rollout_case(wl, 512, iters=2, sample_envs=ids)
+
+
+def test_env_checkpoint_roundtrip():
+    wl = W.make_tiny(n_envs=50)
+    params = torch.from_numpy(W.init_params(wl.net, seed=2)).cuda()
+    a = pe.Env(wl.env, torch.from_numpy(wl.trace), torch.from_numpy(wl.phase))
+    b = pe.Env(wl.env, torch.from_numpy(wl.trace).cuda(), torch.from_numpy(wl.phase).cuda())
+    ba, bb = pe.alloc_rollout(wl.env, wl.net, 300), pe.alloc_rollout(wl.env, wl.net, 300)
+    pe.rollout(a, wl.net, params, 300, 0, ba)
+    pe.rollout(b, wl.net, params, 300, 0, bb)
+    img = a.save()
+    pe.rollout(a, wl.net, params, 300, 1, ba)
+    b.load(img)
+    pe.rollout(b, wl.net, params, 300, 1, bb)
+    torch.cuda.synchronize()
+    for k in ba:
+        assert torch.equal(ba[k], bb[k]), k
+
+
+def test_env_rejects_bad_trace():
+    wl = W.make_tiny(n_envs=4)
+    tr = wl.trace.copy()
+    tr[0, 100] = np.inf
+    with pytest.raises(pe.PEError) as e:
+        pe.Env(wl.env, torch.from_numpy(tr), torch.from_numpy(wl.phase))
+    assert e.value.status == pe.PE_EOVERFLOW
+
+
+# ------------------------------------------------------------------------ PPO
+def _ppo_inputs(wl, T, seed=0):
+    spec, net = wl.env, wl.net
+    params = W.init_params(net, seed=seed, bias_scale=0.05)
+    env = pe.Env(spec, torch.from_numpy(wl.trace), torch.from_numpy(wl.phase))
+    buf = pe.alloc_rollout(spec, net, T)
+    p_dev = torch.from_numpy(params).cuda()
+    pe.rollout(env, net, p_dev, T, 0, buf)
+    adv = torch.empty(T, spec.n_envs, device="cuda")
+    ret = torch.empty_like(adv)
+    pe.gae(buf["reward"], buf["value"], buf["done"], buf["last_value"], wl.ppo.gamma, wl.ppo.lam, adv, ret)
+    torch.cuda.synchronize()
+    env.close()
+    return params, buf, adv, ret
+
+
+def _run_ppo(wl, ppo, params, buf, adv, ret, iteration=0):
+    net = wl.net
+    N = buf["act"].numel()
+    p = torch.from_numpy(params).cuda()
+    m = torch.zeros_like(p)
+    v = torch.zeros_like(p)
+    stats = torch.zeros(8, device="cuda")
+    ws = torch.empty(pe.ppo_workspace_bytes(net, ppo, N), dtype=torch.uint8, device="cuda")
+    pe.ppo_update(net, ppo, p, m, v, 0, buf["obs"], buf["act"], buf["logp"], adv, ret, stats, ws,
+                  seed=7, iteration=iteration)
+    torch.cuda.synchronize()
+    return cpu(p), cpu(m), cpu(v), cpu(stats)
+
+
+def _oracle_ppo(wl, ppo, params, buf, adv, ret, iteration=0, max_steps=-1):
+    P = params.size
+    return O.ppo_update(wl.net, ppo, params, np.zeros(P), np.zeros(P), 0,
+                        cpu(buf["obs"]).reshape(-1, wl.net.obs_dim), cpu(buf["act"]).ravel(),
+                        cpu(buf["logp"]).ravel(), cpu(adv).ravel(), cpu(ret).ravel(), 7, iteration,
+                        max_steps)
+
+
+def test_ppo_single_step_parity():
+    """One minibatch step: Adam's first moment after one step is
+    (1 - beta1) * the clipped gradient, so it exposes the gradient itself."""
+    wl = W.make_tiny()
+    params, buf, adv, ret = _ppo_inputs(wl, 128)
+    ppo = W.PPOSpec(epochs=1, minibatch=8192)
+    gp, gm, gv, gs = _run_ppo(wl, ppo, params, buf, adv, ret)
+    P, m, v, t, st = _oracle_ppo(wl, ppo, params, buf, adv, ret)
+    assert t == 1
+    assert rel_err(gm, m) <= TOL
+    assert rel_err(gv, v) <= 2 * TOL
+    assert rel_err(gp, P) <= TOL
+    for k in (1, 2, 5, 6):   # value loss, entropy, total loss, grad norm
+        assert abs(gs[k] - st[k]) <= TOL * max(abs(st[k]), 1e-3), (k, gs[k], st[k])
+    assert abs(gs[0] - st[0]) <= 1e-5 * max(abs(st[0]), 1.0)   # pg loss is ~0 at rho = 1
+
+
+def test_ppo_ragged_minibatches():
+    """3 steps over minibatches of 3000, 3000 and 2192 samples."""
+    wl = W.make_tiny()
+    params, buf, adv, ret = _ppo_inputs(wl, 128, seed=1)
+    ppo = W.PPOSpec(epochs=1, minibatch=3000)
+    gp, gm, gv, gs = _run_ppo(wl, ppo, params, buf, adv, ret, iteration=5)
+    P, m, v, t, st = _oracle_ppo(wl, ppo, params, buf, adv, ret, iteration=5)
+    assert t == 3 and gs[7] == 3
+    assert rel_err(gp, P) <= 1e-4
+    assert rel_err(gm, m) <= 1e-3
+
+
+def test_ppo_full_update_tiny():
+    """4 epochs x 4 minibatches (ragged last one: 8192 = 3*2500 + 692)."""
+    wl = W.make_tiny()
+    params, buf, adv, ret = _ppo_inputs(wl, 128, seed=3)
+    ppo = W.PPOSpec(epochs=4, minibatch=2500)
+    gp, gm, gv, gs = _run_ppo(wl, ppo, params, buf, adv, ret, iteration=2)
+    P, m, v, t, st = _oracle_ppo(wl, ppo, params, buf, adv, ret, iteration=2)
+    assert t == 16 and gs[7] == 16
+    # Adam normalises each step by sqrt(v): a parameter whose gradient is
+    # within rounding of zero can move by up to lr either way, so the
+    # end-of-update comparison is on the parameter vector as a whole
+    dp, dref = gp - params, P - params
+    assert np.linalg.norm(dp - dref) <= 1e-3 * np.linalg.norm(dref)
+    assert rel_err(gp, P) <= 1e-4
+    assert abs(gs[1] - st[1]) <= 1e-4 * abs(st[1])
+
+
+def test_ppo_7b_first_steps():
+    wl = W.make_7b(n_envs=512)
+    params, buf, adv, ret = _ppo_inputs(wl, 64)
+    ppo = W.PPOSpec(epochs=1, minibatch=32768)
+    gp, gm, gv, gs = _run_ppo(wl, ppo, params, buf, adv, ret)
+    P, m, v, t, st = _oracle_ppo(wl, ppo, params, buf, adv, ret)
+    assert rel_err(gm, m) <= TOL and rel_err(gp, P) <= TOL
