@@ -1,0 +1,433 @@
+#!/usr/bin/env python
+"""Benchmark of the batched PPO power-controller path on GB300.
+
+One step = one PPO iteration of the 7B workload (4,096 envs x 512 steps over
+a 60,000-sample trace, 5 actions, fp32 16-128-128 policy/value MLPs):
+rollout (env + policy + sampler, then the value network), GAE, and the PPO
+update (4 epochs x 256 minibatches of 8,192).  Metric: env-steps/s
+(E * T per step).  The fleet accounting (1,000,000 compositions of 16
+traces x 380,000 samples, windows 1/60/600) is timed in the same run and
+reported under "fleet" as window-samples/s.
+
+Timing: W untimed warm-up steps, then K steps each bracketed by CUDA events
+on the launch stream; an L2 flush (256 MB write) runs between timed steps,
+outside the events.  Multi-GPU (torchrun): independent replicas (one per
+rank, seed = rank), barrier + max over ranks; value = all ranks' env-steps
+divided by the slowest rank's time.
+
+--impl reference times the CPU oracle on a bounded sample of the same
+workload (the paper ships no GPU implementation to compare against).
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+import torch  # noqa: E402
+
+METRIC = "PPO controller env-steps/s and fleet window-samples/s on 1 GB300; % HBM roofline"
+FP32_LANES_PER_SM = 128
+N_SM = 152
+SM_MAX_MHZ = 2070.0
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--fleet-n", type=int, default=1_000_000)
+    ap.add_argument("--fleet-steps", type=int, default=3)
+    ap.add_argument("--cpu-envs", type=int, default=48, help="envs in the oracle CPU sample")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    return ap.parse_args()
+
+
+# --------------------------------------------------------------------------- clocks
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            out, _ = self.proc.communicate(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+            out, _ = self.proc.communicate()
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in out.splitlines():
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                mx.append(float(f[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, f[5:9]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "samples": len(sm),
+                "reasons": sorted(reasons)}
+
+
+# --------------------------------------------------------------------------- helpers
+def ppo_flops_per_sample(D, H, A):
+    fwd = (D * H + H * H + H * A) + (D * H + H * H + H)
+    bwd = (2 * H * A + 2 * H * H + D * H) + (2 * H + 2 * H * H + D * H)
+    return 2 * (fwd + bwd)
+
+
+def load_traffic(kernel: str):
+    """dram bytes per launch from the committed ncu summary, if present."""
+    path = os.path.join(ROOT, "profiles", f"{kernel}.md")
+    if not os.path.exists(path):
+        return None
+    for line in open(path):
+        if line.strip().startswith("traffic_bytes_per_launch:"):
+            v = line.split(":", 1)[1].strip()
+            return None if v in ("", "null") else float(v)
+    return None
+
+
+def dist_setup():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl")
+    else:
+        torch.cuda.set_device(0)
+    return world, rank, local
+
+
+def barrier(world):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def max_over_ranks(x: float, world: int) -> float:
+    if world == 1:
+        return x
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device="cuda")
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+# --------------------------------------------------------------------------- our path
+class Trainer:
+    """State of one 7B PPO training replica on the device."""
+
+    def __init__(self, seed: int):
+        from paper_2608_11226_gb300 import pe
+        from paper_2608_11226_gb300 import workloads as W
+        self.pe, self.W = pe, W
+        self.wl = W.make_7b(seed=seed)
+        wl = self.wl
+        self.E, self.T = wl.env.n_envs, wl.horizon
+        self.env = pe.Env(wl.env, torch.from_numpy(wl.trace), torch.from_numpy(wl.phase))
+        self.buf = pe.alloc_rollout(wl.env, wl.net, self.T)
+        self.params = torch.from_numpy(W.init_params(wl.net, seed=seed)).cuda()
+        self.m = torch.zeros_like(self.params)
+        self.v = torch.zeros_like(self.params)
+        self.adv = torch.empty(self.T, self.E, device="cuda")
+        self.ret = torch.empty_like(self.adv)
+        self.stats = torch.zeros(8, device="cuda")
+        N = self.E * self.T
+        self.ws = torch.empty(pe.ppo_workspace_bytes(wl.net, wl.ppo, N), dtype=torch.uint8, device="cuda")
+        self.adam_t = 0
+        self.it = 0
+        self.seed = seed
+        self.steps_per_update = wl.ppo.epochs * ((N + wl.ppo.minibatch - 1) // wl.ppo.minibatch)
+
+    def step(self):
+        pe, wl = self.pe, self.wl
+        pe.rollout(self.env, wl.net, self.params, self.T, self.it, self.buf)
+        pe.gae(self.buf["reward"], self.buf["value"], self.buf["done"], self.buf["last_value"],
+               wl.ppo.gamma, wl.ppo.lam, self.adv, self.ret)
+        pe.ppo_update(wl.net, wl.ppo, self.params, self.m, self.v, self.adam_t, self.buf["obs"],
+                      self.buf["act"], self.buf["logp"], self.adv, self.ret, self.stats, self.ws,
+                      seed=1000 + self.seed, iteration=self.it)
+        self.adam_t += self.steps_per_update
+        self.it += 1
+
+
+def run_ours(args, world, rank, local):
+    from paper_2608_11226_gb300 import build, pe
+    from paper_2608_11226_gb300 import workloads as W
+    build.build()
+    pe.lib()
+    tr = Trainer(seed=rank)
+    flush = torch.empty(64 * 1024 * 1024, dtype=torch.float32, device="cuda")  # 256 MB > L2
+    for _ in range(args.warmup):
+        tr.step()
+    torch.cuda.synchronize()
+    # ---- timed region (device time, CUDA events on the launch stream)
+    for k in range(pe.PE_PROF_KINDS):
+        pe.profile_read(k)
+    clocks = ClockSampler(local)
+    barrier(world)
+    torch.cuda.synchronize()
+    clocks.start()
+    pe.profile_enable(True)
+    stream = torch.cuda.current_stream()
+    evs = []
+    for _ in range(args.steps):
+        flush.fill_(1.0)
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        tr.step()
+        b.record(stream)
+        evs.append((a, b))
+    torch.cuda.synchronize()
+    pe.profile_enable(False)
+    barrier(world)
+    clk = clocks.stop()
+    total_ms = sum(a.elapsed_time(b) for a, b in evs)
+    prof = {pe.profile_kind_name(k): pe.profile_read(k) for k in range(pe.PE_PROF_KINDS)}
+    total_ms = max_over_ranks(total_ms, world)
+    ms_step = total_ms / args.steps
+    env_steps = tr.E * tr.T
+    value = env_steps * world * args.steps / (total_ms / 1e3)
+    launches = sum(n for _, n in prof.values())
+    # ---- dominant kernel roofline (fp32 FFMA bound)
+    gms, gn = prof["ppo_grad"]
+    net = tr.wl.net
+    fl_launch = ppo_flops_per_sample(net.obs_dim, net.hidden, net.n_actions) * tr.wl.ppo.minibatch
+    peak_tflops = N_SM * FP32_LANES_PER_SM * 2 * SM_MAX_MHZ * 1e6 / 1e12
+    ach = fl_launch / (gms / gn / 1e3) / 1e12 if gn else None
+    roof = {"kernel": "ppo_grad_kernel", "bound": "alu", "achieved": ach, "peak": peak_tflops,
+            "unit": "TFLOP/s", "frac": (ach / peak_tflops) if ach else None,
+            "traffic": load_traffic("ppo_grad_kernel"),
+            "peak_source": "derived: 152 SMs x 128 FP32 lanes x 2 FLOP x 2070 MHz",
+            "avg_launch_ms": gms / gn if gn else None, "launches": gn,
+            "flop_per_launch": fl_launch}
+    kernels = {k: {"ms_per_step": ms / args.steps, "launches_per_step": n / args.steps,
+                   "share": ms / sum(x for x, _ in prof.values()) if n else 0.0}
+               for k, (ms, n) in prof.items() if n}
+    # GAE roofline (HBM): 17 algorithmic bytes per env-step
+    gae_ms, gae_n = prof["gae"]
+    gae_gbs = 17.0 * env_steps / (gae_ms / gae_n / 1e3) / 1e9 if gae_n else None
+    peaks = json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json"))) if os.path.exists(
+        os.path.join(ROOT, "MEASURED_PEAKS.json")) else {"hbm_gbs": 6800.0}
+    hbm = float(peaks.get("hbm_gbs", 6800.0))
+    gae_roof = {"kernel": "gae_kernel", "bound": "hbm", "achieved": gae_gbs, "peak": hbm,
+                "unit": "GB/s", "frac": gae_gbs / hbm if gae_gbs else None,
+                "traffic": load_traffic("gae_kernel")}
+
+    # ---- end to end through host buffers: model state uploaded from pinned
+    # host memory every step, parameters + statistics + counters read back
+    host_in = [x.cpu().pin_memory() for x in (tr.params, tr.m, tr.v)]
+    host_out = {k: torch.empty(x.shape, dtype=x.dtype).pin_memory() for k, x in
+                (("params", tr.params), ("m", tr.m), ("v", tr.v), ("stats", tr.stats),
+                 ("viol", tr.buf["viol"]), ("tokens", tr.buf["tokens"]),
+                 ("excess", tr.buf["excess"]), ("energy_q", tr.buf["energy_q"]))}
+    h2d = sum(x.numel() * x.element_size() for x in host_in)
+    d2h = sum(x.numel() * x.element_size() for x in host_out.values())
+    e2e_steps = max(3, args.steps // 2)
+    barrier(world)
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    for _ in range(e2e_steps):
+        tr.params.copy_(host_in[0], non_blocking=True)
+        tr.m.copy_(host_in[1], non_blocking=True)
+        tr.v.copy_(host_in[2], non_blocking=True)
+        tr.step()
+        for k, dst in host_out.items():
+            src = {"params": tr.params, "m": tr.m, "v": tr.v, "stats": tr.stats}.get(k)
+            dst.copy_(tr.buf[k] if src is None else src, non_blocking=True)
+        torch.cuda.current_stream().synchronize()
+        _ = float(host_out["stats"][5])
+    e2e_s = max_over_ranks(time.perf_counter() - t0, world)
+    e2e = {"value": env_steps * world * e2e_steps / e2e_s, "unit": "env-steps/s",
+           "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h}
+
+    # ---- fleet accounting
+    fleet = run_fleet(args, world) if args.fleet_n > 0 else None
+
+    out = {"metric": METRIC, "value": value, "unit": "env-steps/s", "n_gpus": world,
+           "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_step,
+           "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+           "data": "synthetic",
+           "config": {"workload": "7b: 4096 envs x 512 steps on a 60,000-sample 7B-GRPO-shaped "
+                                  "trace, 5 actions, MLP 16-128-128 fp32, GAE, PPO 4 epochs x "
+                                  "minibatch 8192", "n_envs": tr.E, "horizon": tr.T,
+                      "parallelism": f"replicas x{world}" if world > 1 else "1 GPU",
+                      "l2": "flushed between timed steps (256 MB write)"},
+           "roofline": roof, "gae_roofline": gae_roof, "kernels": kernels,
+           "gpu_launches": launches, "clocks": clk, "e2e": e2e, "fleet": fleet,
+           "ppo_stats_last": [float(x) for x in tr.stats.cpu()]}
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        out["cpu_baseline"] = cpu_baseline(args.cpu_envs)
+    if rank == 0:
+        print(json.dumps(out), flush=True)
+
+
+def run_fleet(args, world):
+    from paper_2608_11226_gb300 import pe
+    from paper_2608_11226_gb300 import workloads as W
+    fw = W.make_fleet(n_compositions=args.fleet_n)
+    G, L = fw.traces.shape
+    traces = torch.from_numpy(fw.traces).cuda()
+    job = torch.from_numpy(fw.job_of_gpu).cuda()
+    off = torch.from_numpy(fw.offsets).cuda()
+    N = fw.offsets.shape[0]
+    windows = [1, 60, 600]
+    counts = torch.empty((N, 3), dtype=torch.int32, device="cuda")
+    peaks = torch.empty_like(counts)
+    ws = torch.empty(pe.fleet_workspace_bytes(fw.n_jobs, L, fw.horizon), dtype=torch.uint8, device="cuda")
+    pe.fleet_windows(traces, job, fw.n_jobs, off, fw.horizon, windows, fw.budget_q, counts, peaks, ws)
+    torch.cuda.synchronize()
+    for k in range(pe.PE_PROF_KINDS):
+        pe.profile_read(k)
+    barrier(world)
+    pe.profile_enable(True)
+    stream = torch.cuda.current_stream()
+    a = torch.cuda.Event(enable_timing=True)
+    b = torch.cuda.Event(enable_timing=True)
+    a.record(stream)
+    for _ in range(args.fleet_steps):
+        pe.fleet_windows(traces, job, fw.n_jobs, off, fw.horizon, windows, fw.budget_q, counts,
+                         peaks, ws)
+    b.record(stream)
+    torch.cuda.synchronize()
+    pe.profile_enable(False)
+    ms = max_over_ranks(a.elapsed_time(b), world)
+    wms, wn = pe.profile_read(pe.PE_PROF_FLEET_WINDOWS)
+    pe.profile_read(pe.PE_PROF_FLEET_PREP)
+    H = fw.horizon
+    ws_per_call = sum(N * (H - w + 1) for w in windows)
+    composed = N * H
+    c = counts.cpu().numpy()
+    p = peaks.cpu().numpy()
+    return {"metric": "fleet window-samples/s", "value": ws_per_call * world * args.fleet_steps / (ms / 1e3),
+            "unit": "window-samples/s", "ms_per_call": ms / args.fleet_steps,
+            "config": {"workload": "fleet: 16 traces x 380,000 samples (2x72B@4, 2x14B@2, 4x7B@1), "
+                                   f"{N} offset compositions, windows 1/60/600, budget 0.5 x nameplate",
+                       "n": N, "horizon": H},
+            "kernel_ms_per_launch": wms / wn if wn else None,
+            "composed_samples_per_s": composed / (wms / wn / 1e3) if wn else None,
+            "logical_l2_gbs": 4.0 * fw.n_jobs * composed / (wms / wn / 1e3) / 1e9 if wn else None,
+            "violation_fraction_mean": [float(c[:, i].mean() / (H - w + 1)) for i, w in enumerate(windows)],
+            "peak_fraction_of_nameplate_max": [float(p[:, i].max() / (64.0 * w) / W.FLEET_NAMEPLATE_W)
+                                               for i, w in enumerate(windows)],
+            "traffic": load_traffic("fleet_windows_kernel")}
+
+
+# --------------------------------------------------------------------------- CPU oracle
+def oracle_iteration(n_envs: int, seed: int = 0, iteration: int = 0):
+    """One PPO iteration of the 7B workload on a sample of n_envs envs, by the
+    CPU oracle (rollout, value, GAE, PPO update with the minibatch scaled by
+    n_envs / 4096 so that the update takes the same 256 minibatch steps)."""
+    import oracle as O
+    from paper_2608_11226_gb300 import workloads as W
+    wl = W.make_7b(seed=seed)
+    net = wl.net
+    params = W.init_params(net, seed=seed)
+    env = O.OracleEnv(wl.env, wl.trace, wl.phase, np.arange(n_envs))
+    T = wl.horizon
+    t0 = time.perf_counter()
+    o = env.rollout(params, net.hidden, False, T, iteration)
+    _, v = O.mlp_forward(net, params, o["obs"].reshape(-1, net.obs_dim))
+    _, lv = O.mlp_forward(net, params, o["obs_last"])
+    adv, ret = O.gae(o["reward"].astype(np.float32), v.reshape(T, n_envs).astype(np.float32),
+                     o["done"], lv.astype(np.float32), wl.ppo.gamma, wl.ppo.lam)
+    mb = max(1, wl.ppo.minibatch * n_envs // wl.env.n_envs)
+    ppo = W.PPOSpec(epochs=wl.ppo.epochs, minibatch=mb)
+    P = params.size
+    O.ppo_update(net, ppo, params, np.zeros(P), np.zeros(P), 0, o["obs"].reshape(-1, net.obs_dim),
+                 o["act_own"].ravel(), o["logp"].astype(np.float32).ravel(),
+                 adv.astype(np.float32).ravel(), ret.astype(np.float32).ravel(), 7, iteration)
+    return time.perf_counter() - t0, n_envs * T
+
+
+def cpu_baseline(n_envs: int):
+    import oracle as O
+    O.build()
+    dt, steps = oracle_iteration(n_envs)
+    return {"value": steps / dt, "unit": "env-steps/s", "cores": 1, "kind": "oracle",
+            "sample": f"one PPO iteration of the 7b workload on {n_envs} of 4096 envs "
+                      f"(512 steps each, minibatch scaled to keep 256 minibatch steps); {dt:.1f} s"}
+
+
+def run_reference(args, world, rank):
+    if rank != 0:
+        return
+    import oracle as O
+    O.build()
+    n = max(1, args.cpu_envs // 3)
+    for _ in range(args.warmup):
+        oracle_iteration(n)
+    tot = 0.0
+    steps = 0
+    for k in range(args.steps):
+        dt, s = oracle_iteration(n, iteration=k)
+        tot += dt
+        steps += s
+    value = steps / tot
+    out = {"metric": METRIC, "value": value, "unit": "env-steps/s", "n_gpus": world,
+           "steps": args.steps, "warmup": args.warmup, "ms_per_step": tot / args.steps * 1e3,
+           "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+           "data": "synthetic", "impl": "reference",
+           "config": {"workload": "7b: 4096 envs x 512 steps on a 60,000-sample 7B-GRPO-shaped "
+                                  "trace, 5 actions, MLP 16-128-128 fp32, GAE, PPO 4 epochs x "
+                                  "minibatch 8192", "sample_envs": n},
+           "cpu_baseline": {"value": value, "unit": "env-steps/s", "cores": 1, "kind": "oracle",
+                            "sample": f"{n} of 4096 envs per step, minibatch scaled to keep 256 "
+                                      "minibatch steps"},
+           "e2e": {"value": value, "unit": "env-steps/s", "h2d_bytes_per_step": 0,
+                   "d2h_bytes_per_step": 0}}
+    print(json.dumps(out), flush=True)
+
+
+def main():
+    args = parse()
+    if args.impl == "reference":
+        world = int(os.environ.get("WORLD_SIZE", "1"))
+        rank = int(os.environ.get("RANK", "0"))
+        run_reference(args, world, rank)
+        return
+    world, rank, local = dist_setup()
+    run_ours(args, world, rank, local)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

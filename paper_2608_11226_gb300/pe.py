@@ -23,6 +23,9 @@ PE_OK, PE_EINVAL, PE_ENOMEM, PE_ECUDA, PE_EOVERFLOW, PE_ETIMEOUT, PE_ESTATE = ra
 PE_F32, PE_BF16 = 0, 1
 PE_ROLLOUT_DETERMINISTIC = 1
 MAX_LEVELS, MAX_CH = 32, 4
+(PE_PROF_ROLLOUT, PE_PROF_VALUE, PE_PROF_GAE, PE_PROF_PPO_GRAD, PE_PROF_PPO_REDUCE,
+ PE_PROF_PPO_ADAM, PE_PROF_PPO_OTHER, PE_PROF_FLEET_PREP, PE_PROF_FLEET_WINDOWS) = range(9)
+PE_PROF_KINDS = 9
 
 
 class PEError(RuntimeError):
@@ -63,7 +66,8 @@ class PPOConfig(C.Structure):
 EXPORTS = (
     "pe_env_create", "pe_env_destroy", "pe_env_state_bytes", "pe_env_save", "pe_env_load",
     "pe_param_count", "pe_rollout", "pe_value", "pe_gae", "pe_ppo_workspace_bytes",
-    "pe_ppo_update", "pe_fleet_workspace_bytes", "pe_fleet_windows", "pe_last_error")
+    "pe_ppo_update", "pe_fleet_workspace_bytes", "pe_fleet_windows", "pe_profile_enable",
+    "pe_profile_read", "pe_profile_kind_name", "pe_last_error")
 
 
 def lib():
@@ -90,6 +94,9 @@ def lib():
             "pe_fleet_workspace_bytes": (i64, [i32, i32, i32]),
             "pe_fleet_windows": (i32, [vp, i32, i32, vp, i32, vp, i64, i32, vp, i32, i64, vp,
                                        vp, vp, i64, vp]),
+            "pe_profile_enable": (i32, [i32]),
+            "pe_profile_read": (i32, [i32, C.POINTER(C.c_double), C.POINTER(C.c_int64)]),
+            "pe_profile_kind_name": (C.c_char_p, [i32]),
             "pe_last_error": (C.c_char_p, []),
         }
         for name, (res, args) in sig.items():
@@ -251,3 +258,19 @@ def fleet_windows(traces, job_of_gpu, J: int, offsets, H: int, windows: Sequence
     _check(lib().pe_fleet_windows(_ptr(traces), G, L, _ptr(job_of_gpu), J, _ptr(offsets), N, H,
                                   w, len(windows), budget_q, _ptr(counts), _ptr(peaks),
                                   _ptr(workspace), workspace.numel(), _stream(stream)))
+
+
+def profile_enable(on: bool):
+    _check(lib().pe_profile_enable(int(bool(on))))
+
+
+def profile_read(kind: int):
+    """(summed device ms, launches) of one kernel kind since the last read."""
+    ms = C.c_double()
+    n = C.c_int64()
+    _check(lib().pe_profile_read(kind, C.byref(ms), C.byref(n)))
+    return ms.value, n.value
+
+
+def profile_kind_name(kind: int) -> str:
+    return lib().pe_profile_kind_name(kind).decode()
