@@ -226,6 +226,26 @@ pe_status pe_fleet_windows(const float* traces, int32_t G, int32_t L, const int3
                            int32_t* counts, int32_t* peaks, void* workspace,
                            int64_t workspace_bytes, void* stream);
 
+/* pe_fleet_windows for callers that cannot allocate device memory -- code
+ * inside a host process whose device memory belongs to another allocator,
+ * or a control loop that cannot afford an allocation's synchronisation.
+ * The paper has no counterpart: this is a deployment convenience.
+ * Same arguments and results as pe_fleet_windows without the workspace: the
+ * scratch is one file-scope device array of PE_FLEET_NOALLOC_SCRATCH_BYTES
+ * (4 MiB, held by every GPU that loads the library until exit).  Requests
+ * needing more (J * (L + H) * 4 + 512 bytes) return PE_EINVAL with that
+ * limit in the message, before any launch.  The call allocates nothing (no
+ * cudaMalloc, no allocating library routine).  Its first call on a device
+ * looks up the array's device address (cudaGetSymbolAddress) with that
+ * device current; make that first call before any stream capture.  All
+ * calls share the array: calls that overlap on the GPU race. */
+#define PE_FLEET_NOALLOC_SCRATCH_BYTES (4 * 1024 * 1024)
+pe_status pe_fleet_windows_noalloc(const float* traces, int32_t G, int32_t L,
+                                   const int32_t* job_of_gpu, int32_t J, const int32_t* offsets,
+                                   int64_t N, int32_t H, const int32_t* windows, int32_t W,
+                                   int64_t budget_q, int32_t* counts, int32_t* peaks,
+                                   void* stream);
+
 /* Launch profiling (off by default).  When enabled, every kernel launch of
  * the library is bracketed by a pair of CUDA events recorded on the launch's
  * stream; pe_profile_read waits for the recorded events of one kernel kind,

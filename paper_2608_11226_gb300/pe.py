@@ -66,7 +66,8 @@ class PPOConfig(C.Structure):
 EXPORTS = (
     "pe_env_create", "pe_env_destroy", "pe_env_state_bytes", "pe_env_save", "pe_env_load",
     "pe_param_count", "pe_rollout", "pe_value", "pe_gae", "pe_ppo_workspace_bytes",
-    "pe_ppo_update", "pe_fleet_workspace_bytes", "pe_fleet_windows", "pe_profile_enable",
+    "pe_ppo_update", "pe_fleet_workspace_bytes", "pe_fleet_windows", "pe_fleet_windows_noalloc",
+    "pe_profile_enable",
     "pe_profile_read", "pe_profile_kind_name", "pe_last_error")
 
 
@@ -94,6 +95,8 @@ def lib():
             "pe_fleet_workspace_bytes": (i64, [i32, i32, i32]),
             "pe_fleet_windows": (i32, [vp, i32, i32, vp, i32, vp, i64, i32, vp, i32, i64, vp,
                                        vp, vp, i64, vp]),
+            "pe_fleet_windows_noalloc": (i32, [vp, i32, i32, vp, i32, vp, i64, i32, vp, i32, i64,
+                                               vp, vp, vp]),
             "pe_profile_enable": (i32, [i32]),
             "pe_profile_read": (i32, [i32, C.POINTER(C.c_double), C.POINTER(C.c_int64)]),
             "pe_profile_kind_name": (C.c_char_p, [i32]),
@@ -258,6 +261,21 @@ def fleet_windows(traces, job_of_gpu, J: int, offsets, H: int, windows: Sequence
     _check(lib().pe_fleet_windows(_ptr(traces), G, L, _ptr(job_of_gpu), J, _ptr(offsets), N, H,
                                   w, len(windows), budget_q, _ptr(counts), _ptr(peaks),
                                   _ptr(workspace), workspace.numel(), _stream(stream)))
+
+
+FLEET_NOALLOC_SCRATCH_BYTES = 4 * 1024 * 1024
+
+
+def fleet_windows_noalloc(traces, job_of_gpu, J: int, offsets, H: int, windows: Sequence[int],
+                          budget_q: int, counts, peaks, stream=None):
+    """pe_fleet_windows without a workspace, for callers that cannot allocate
+    device memory; its scratch is a fixed 4 MiB array inside the library."""
+    G, L = traces.shape
+    N = offsets.shape[0]
+    w = (C.c_int32 * len(windows))(*[int(x) for x in windows])
+    _check(lib().pe_fleet_windows_noalloc(_ptr(traces), G, L, _ptr(job_of_gpu), J, _ptr(offsets), N,
+                                          H, w, len(windows), budget_q, _ptr(counts), _ptr(peaks),
+                                          _stream(stream)))
 
 
 def profile_enable(on: bool):
