@@ -233,8 +233,8 @@ pe_status pe_fleet_windows(const float* traces, int32_t G, int32_t L, const int3
  * Same arguments and results as pe_fleet_windows without the workspace: the
  * scratch is one file-scope device array of PE_FLEET_NOALLOC_SCRATCH_BYTES
  * (4 MiB, held by every GPU that loads the library until exit).  Requests
- * needing more (J * (L + H) * 4 + 512 bytes) return PE_EINVAL with that
- * limit in the message, before any launch.  The call allocates nothing (no
+ * needing more (pe_fleet_workspace_bytes(J, L, H), about J * (L + H) * 4
+ * bytes) return PE_EINVAL with that limit in the message, before any launch.  The call allocates nothing (no
  * cudaMalloc, no allocating library routine).  Its first call on a device
  * looks up the array's device address (cudaGetSymbolAddress) with that
  * device current; make that first call before any stream capture.  All

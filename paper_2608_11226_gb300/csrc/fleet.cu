@@ -1,17 +1,19 @@
 // Fleet window accounting (Sec. 7 window analysis, Sec. 8 composed fleet).
 //
-// Prepare: q_g = rint(64 x_g) per GPU, summed per job (a job's GPUs share a
-// start offset) into jobq[j][i] = sum_{g in j} q_g(i mod L) for
-// i in [0, L + H): with the period unrolled once, composition n reads job j
-// at index t + o[n][j] without a modulo.  The buffer (J * (L + H) int32,
-// 24 MB for the 8-job, 380,000-sample fleet) stays resident in L2.
+// Prepare: q_g = rint(64 x_g) per GPU (1/64 W), summed per job (a job's GPUs
+// share a start offset) and turned into a per-job prefix sum over the
+// period unrolled once:
+//   PREX[j][i] = sum_{k < i} sum_{g in j} q_g(k mod L),  i in [0, L + H],
+// kept modulo 2^32 (uint32).  For composition n the running composed prefix
+// is then pre(t) = sum_j PREX[j][t + 1 + o[n][j]] (mod 2^32), and every
+// window sum is S_w(t) = pre(t) - pre(t - w), exact because the true sum is
+// below 2^31 (checked on the host from the per-job maxima).  The prefixes
+// (J * (L + H + 1) int32, 24 MB for the 8-job, 380,000-sample fleet) stay
+// resident in L2.
 //
-// Count: one warp per composition walks t in steps of 32.  Lane l forms
-// P(t0 + l) from J coalesced loads, a warp-shuffle inclusive scan turns the
-// 32 powers into the running prefix sum pre(t) (int32, wrapping: window
-// differences pre(t) - pre(t - w) are exact because every true window sum
-// is below 2^31, checked on the host), and a 1024-slot shared-memory ring of
-// prefixes gives pre(t - w) for every window w <= 992 at once.
+// Count: one warp per composition walks t in steps of 32; lane l forms
+// pre(t0 + l) from J coalesced loads, keeps it in a 1024-slot shared-memory
+// ring, and reads pre(t - w) back for every window w <= 992 at once.
 #include <algorithm>
 #include <climits>
 
@@ -21,54 +23,143 @@ namespace pe {
 
 constexpr int kFleetRing = 1024;
 constexpr int kFleetWarps = 8;
+constexpr int kFleetChunk = 8192;   // prefix-scan chunk per block
 constexpr float kFleetMaxWatts = 65536.0f;
 
 struct FleetWs {
-  int32_t* jobq;     // [J][L + H]
+  uint32_t* prex;    // [J][Lp]
+  uint32_t* totals;  // [J][nchunk] chunk sums, then exclusive chunk offsets
   int32_t* maxq;     // [J]
   int32_t* flag;     // [1]: bit 0 bad sample, bit 1 bad job map, bit 2 bad offset
+  int64_t Lp;        // row stride of prex
+  int nchunk;
 };
 
-__global__ void fleet_prepare_kernel(const float* __restrict__ traces, int G, int L, int H,
-                                     const int32_t* __restrict__ job_of_gpu, int J,
-                                     FleetWs ws) {
-  __shared__ int32_t sjob[64];
-  __shared__ int32_t smax[32];
-  const int j = blockIdx.y;
+__device__ __forceinline__ int32_t job_sample(const float* __restrict__ traces, const int8_t* sjob,
+                                              int G, int L, int j, int64_t i, int& bad) {
+  const int64_t src = i < L ? i : i % L;
+  int32_t s = 0;
+  for (int g = 0; g < G; ++g) {
+    if (sjob[g] != j) continue;
+    const float x = __ldg(traces + (int64_t)g * L + src);
+    if (!(x >= 0.0f && x <= kFleetMaxWatts)) {
+      bad = 1;
+      continue;
+    }
+    s += __float2int_rn(x * 64.0f);
+  }
+  return s;
+}
+
+__device__ __forceinline__ void load_jobs(const int32_t* __restrict__ job_of_gpu, int G, int J,
+                                          int8_t* sjob, int32_t* flag) {
   for (int g = threadIdx.x; g < G; g += blockDim.x) {
     const int jj = job_of_gpu[g];
-    sjob[g] = jj;
-    if (jj < 0 || jj >= J) atomicOr(ws.flag, 2);
+    sjob[g] = (int8_t)((jj >= 0 && jj < J) ? jj : -1);
+    if (jj < 0 || jj >= J) atomicOr(flag, 2);
   }
   __syncthreads();
+}
+
+// block sum of uint32 (wrapping) and max of int32 over 256 threads
+__device__ __forceinline__ void block_sum_max(uint32_t& s, int32_t& m, uint32_t* ss, int32_t* sm) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    s += __shfl_xor_sync(0xffffffffu, s, o);
+    m = max(m, __shfl_xor_sync(0xffffffffu, m, o));
+  }
+  if ((threadIdx.x & 31) == 0) {
+    ss[threadIdx.x >> 5] = s;
+    sm[threadIdx.x >> 5] = m;
+  }
+  __syncthreads();
+  s = 0;
+  m = 0;
+  for (int k = 0; k < (int)(blockDim.x >> 5); ++k) {
+    s += ss[k];
+    m = max(m, sm[k]);
+  }
+}
+
+// pass 1: per (job, chunk) sum, job maximum, sample validation
+__global__ void __launch_bounds__(256) fleet_chunk_sums_kernel(const float* __restrict__ traces, int G, int L, int H,
+                                                               const int32_t* __restrict__ job_of_gpu,
+                                                               int J, FleetWs ws) {
+  __shared__ int8_t sjob[64];
+  __shared__ uint32_t ss[8];
+  __shared__ int32_t sm[8];
+  load_jobs(job_of_gpu, G, J, sjob, ws.flag);
+  const int j = blockIdx.y, c = blockIdx.x;
   const int64_t Lx = (int64_t)L + H;
+  const int64_t i0 = (int64_t)c * kFleetChunk;
+  uint32_t s = 0;
   int32_t m = 0;
   int bad = 0;
-  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < Lx;
-       i += (int64_t)gridDim.x * blockDim.x) {
-    const int64_t src = i < L ? i : i % L;
-    int32_t s = 0;
-    for (int g = 0; g < G; ++g) {
-      if (sjob[g] != j) continue;
-      const float x = __ldg(traces + (int64_t)g * L + src);
-      if (!(x >= 0.0f && x <= kFleetMaxWatts)) {
-        bad = 1;
-        continue;
-      }
-      s += __float2int_rn(x * 64.0f);
-    }
-    ws.jobq[(int64_t)j * Lx + i] = s;
-    m = max(m, s);
+  for (int64_t i = i0 + threadIdx.x; i < min(i0 + kFleetChunk, Lx); i += blockDim.x) {
+    const int32_t q = job_sample(traces, sjob, G, L, j, i, bad);
+    s += (uint32_t)q;
+    m = max(m, q);
   }
   if (bad) atomicOr(ws.flag, 1);
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) m = max(m, __shfl_xor_sync(0xffffffffu, m, o));
-  if ((threadIdx.x & 31) == 0) smax[threadIdx.x >> 5] = m;
-  __syncthreads();
+  block_sum_max(s, m, ss, sm);
   if (threadIdx.x == 0) {
-    int32_t mm = 0;
-    for (int k = 0; k < (int)(blockDim.x >> 5); ++k) mm = max(mm, smax[k]);
-    atomicMax(ws.maxq + j, mm);
+    ws.totals[(int64_t)j * ws.nchunk + c] = s;
+    atomicMax(ws.maxq + j, m);
+  }
+}
+
+// pass 2: exclusive scan of each job's chunk sums (one warp per job)
+__global__ void fleet_chunk_scan_kernel(FleetWs ws) {
+  const int j = blockIdx.x, lane = threadIdx.x;
+  uint32_t carry = 0;
+  for (int c0 = 0; c0 < ws.nchunk; c0 += 32) {
+    const int c = c0 + lane;
+    const uint32_t v = c < ws.nchunk ? ws.totals[(int64_t)j * ws.nchunk + c] : 0u;
+    uint32_t x = v;
+#pragma unroll
+    for (int d = 1; d < 32; d <<= 1) {
+      const uint32_t y = __shfl_up_sync(0xffffffffu, x, d);
+      if (lane >= d) x += y;
+    }
+    if (c < ws.nchunk) ws.totals[(int64_t)j * ws.nchunk + c] = carry + x - v;
+    carry += __shfl_sync(0xffffffffu, x, 31);
+  }
+}
+
+// pass 3: prefix within each chunk, offset by the chunk's exclusive sum
+__global__ void __launch_bounds__(256) fleet_prefix_kernel(const float* __restrict__ traces, int G, int L, int H,
+                                                           const int32_t* __restrict__ job_of_gpu,
+                                                           int J, FleetWs ws) {
+  __shared__ int8_t sjob[64];
+  __shared__ uint32_t wsum[8];
+  load_jobs(job_of_gpu, G, J, sjob, ws.flag);
+  const int j = blockIdx.y, c = blockIdx.x;
+  const int64_t Lx = (int64_t)L + H;
+  const int64_t i0 = (int64_t)c * kFleetChunk;
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  uint32_t carry = ws.totals[(int64_t)j * ws.nchunk + c];
+  uint32_t* row = ws.prex + (int64_t)j * ws.Lp;
+  if (c == 0 && threadIdx.x == 0) row[0] = 0u;
+  int bad = 0;
+  for (int64_t b = i0; b < min(i0 + kFleetChunk, Lx); b += blockDim.x) {
+    const int64_t i = b + threadIdx.x;
+    const uint32_t q = i < Lx ? (uint32_t)job_sample(traces, sjob, G, L, j, i, bad) : 0u;
+    uint32_t x = q;
+#pragma unroll
+    for (int d = 1; d < 32; d <<= 1) {
+      const uint32_t y = __shfl_up_sync(0xffffffffu, x, d);
+      if (lane >= d) x += y;
+    }
+    if (lane == 31) wsum[w] = x;
+    __syncthreads();
+    uint32_t before = 0, total = 0;
+    for (int k = 0; k < 8; ++k) {
+      if (k < w) before += wsum[k];
+      total += wsum[k];
+    }
+    if (i < Lx) row[i + 1] = carry + before + x;
+    carry += total;
+    __syncthreads();
   }
 }
 
@@ -90,36 +181,38 @@ struct FleetWindows {
 
 template <int NW>
 __global__ void __launch_bounds__(32 * kFleetWarps)
-    fleet_windows_kernel(const int32_t* __restrict__ jobq, int J, int64_t Lx,
+    fleet_windows_kernel(const uint32_t* __restrict__ prex, int J, int64_t Lp,
                          const int32_t* __restrict__ offsets, int64_t N, int H, FleetWindows win,
                          int32_t* __restrict__ counts, int32_t* __restrict__ peaks) {
-  __shared__ int32_t ring_all[kFleetWarps][kFleetRing];
-  __shared__ int32_t off_all[kFleetWarps][32];
+  __shared__ uint32_t ring_all[kFleetWarps][kFleetRing];
+  __shared__ const uint32_t* base_all[kFleetWarps][32];
   const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
   const int64_t n = (int64_t)blockIdx.x * kFleetWarps + wid;
   if (n >= N) return;  // the whole warp leaves together; no block-wide barrier follows
-  int32_t* ring = ring_all[wid];
-  const int32_t* off = off_all[wid];
-  if (lane < J) off_all[wid][lane] = __ldg(offsets + n * J + lane);
-  if (lane == 0) ring[kFleetRing - 1] = 0;  // pre(-1) = 0
+  uint32_t* ring = ring_all[wid];
+  const uint32_t** base = base_all[wid];
+  uint32_t pre_m1 = 0;  // pre(-1) = sum_j PREX[j][o_j]
+  if (lane < J) {
+    const int32_t o = __ldg(offsets + n * J + lane);
+    const uint32_t* b = prex + (int64_t)lane * Lp + o;
+    base[lane] = b + 1;
+    pre_m1 = __ldg(b);
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) pre_m1 += __shfl_xor_sync(0xffffffffu, pre_m1, o);
+  if (lane == 0) ring[kFleetRing - 1] = pre_m1;
   __syncwarp();
-  int32_t carry = 0;
+  const uint32_t* b0 = base[0];
   int32_t cnt[NW], pk[NW];
 #pragma unroll
   for (int k = 0; k < NW; ++k) cnt[k] = pk[k] = 0;
   for (int t0 = 0; t0 < H; t0 += 32) {
     const int t = t0 + lane;
-    int32_t P = 0;
-    if (t < H)
-      for (int j = 0; j < J; ++j) P += __ldg(jobq + (int64_t)j * Lx + off[j] + t);
-    int32_t x = P;
-#pragma unroll
-    for (int dlt = 1; dlt < 32; dlt <<= 1) {
-      const int32_t y = __shfl_up_sync(0xffffffffu, x, dlt);
-      if (lane >= dlt) x = (int32_t)((uint32_t)x + (uint32_t)y);
+    uint32_t pre = 0;
+    if (t < H) {
+      pre = __ldg(b0 + t);
+      for (int j = 1; j < J; ++j) pre += __ldg(base[j] + t);
     }
-    const int32_t pre = (int32_t)((uint32_t)carry + (uint32_t)x);
-    carry = __shfl_sync(0xffffffffu, pre, 31);
     ring[t & (kFleetRing - 1)] = pre;
     __syncwarp();
     if (t < H) {
@@ -127,7 +220,7 @@ __global__ void __launch_bounds__(32 * kFleetWarps)
       for (int k = 0; k < NW; ++k) {
         const int w = win.w[k];
         if (t >= w - 1) {
-          const int32_t S = (int32_t)((uint32_t)pre - (uint32_t)ring[(t - w) & (kFleetRing - 1)]);
+          const int32_t S = (int32_t)(pre - ring[(t - w) & (kFleetRing - 1)]);
           cnt[k] += S > win.bw[k];
           pk[k] = max(pk[k], S);
         }
@@ -150,9 +243,13 @@ __global__ void __launch_bounds__(32 * kFleetWarps)
   }
 }
 
+static int64_t fleet_lp(int L, int H) { return (((int64_t)L + H + 1) + 3) / 4 * 4; }
+static int fleet_nchunk(int L, int H) { return (int)((((int64_t)L + H) + kFleetChunk - 1) / kFleetChunk); }
+
 int64_t fleet_ws_bytes(int J, int L, int H) {
-  const int64_t jobq = (int64_t)J * ((int64_t)L + H) * 4;
-  return ((jobq + 255) / 256) * 256 + 256 + 256;
+  const int64_t prex = ((int64_t)J * fleet_lp(L, H) * 4 + 255) / 256 * 256;
+  const int64_t tot = ((int64_t)J * fleet_nchunk(L, H) * 4 + 255) / 256 * 256;
+  return prex + tot + 256 + 256;
 }
 
 pe_status fleet_launch(const float* traces, int G, int L, const int32_t* job_of_gpu, int J,
@@ -160,23 +257,27 @@ pe_status fleet_launch(const float* traces, int G, int L, const int32_t* job_of_
                        int64_t budget_q, int32_t* counts, int32_t* peaks, void* workspace,
                        cudaStream_t st) {
   char* base = reinterpret_cast<char*>(workspace);
-  const int64_t jobq_bytes = ((int64_t)J * ((int64_t)L + H) * 4 + 255) / 256 * 256;
   FleetWs ws;
-  ws.jobq = reinterpret_cast<int32_t*>(base);
-  ws.maxq = reinterpret_cast<int32_t*>(base + jobq_bytes);
-  ws.flag = reinterpret_cast<int32_t*>(base + jobq_bytes + 256);
+  ws.Lp = fleet_lp(L, H);
+  ws.nchunk = fleet_nchunk(L, H);
+  const int64_t prex_bytes = ((int64_t)J * ws.Lp * 4 + 255) / 256 * 256;
+  const int64_t tot_bytes = ((int64_t)J * ws.nchunk * 4 + 255) / 256 * 256;
+  ws.prex = reinterpret_cast<uint32_t*>(base);
+  ws.totals = reinterpret_cast<uint32_t*>(base + prex_bytes);
+  ws.maxq = reinterpret_cast<int32_t*>(base + prex_bytes + tot_bytes);
+  ws.flag = reinterpret_cast<int32_t*>(base + prex_bytes + tot_bytes + 256);
   PE_TRY_CUDA(cudaMemsetAsync(ws.maxq, 0, 256 + 4, st));
-  dim3 grid(ceil_div((int64_t)L + H, 256 * 8), J);
   {
     ProfScope ps(PE_PROF_FLEET_PREP, st);
-    fleet_prepare_kernel<<<grid, 256, 0, st>>>(traces, G, L, H, job_of_gpu, J, ws);
+    const dim3 grid(ws.nchunk, J);
+    fleet_chunk_sums_kernel<<<grid, 256, 0, st>>>(traces, G, L, H, job_of_gpu, J, ws);
+    fleet_chunk_scan_kernel<<<J, 32, 0, st>>>(ws);
+    fleet_prefix_kernel<<<grid, 256, 0, st>>>(traces, G, L, H, job_of_gpu, J, ws);
+    if (N > 0)
+      fleet_check_offsets_kernel<<<(int)std::min<int64_t>(ceil_div(N * J, 256), 4096), 256, 0, st>>>(
+          offsets, N * J, L, ws.flag);
   }
-  PE_CHECK_LAUNCH("fleet_prepare_kernel");
-  if (N > 0) {
-    fleet_check_offsets_kernel<<<(int)std::min<int64_t>(ceil_div(N * J, 256), 4096), 256, 0, st>>>(
-        offsets, N * J, L, ws.flag);
-    PE_CHECK_LAUNCH("fleet_check_offsets_kernel");
-  }
+  PE_CHECK_LAUNCH("fleet prepare kernels");
   int32_t host[64 + 1];
   PE_TRY_CUDA(cudaMemcpyAsync(host, ws.maxq, sizeof(int32_t) * J, cudaMemcpyDeviceToHost, st));
   PE_TRY_CUDA(cudaMemcpyAsync(host + 64, ws.flag, sizeof(int32_t), cudaMemcpyDeviceToHost, st));
@@ -197,13 +298,13 @@ pe_status fleet_launch(const float* traces, int G, int L, const int32_t* job_of_
   }
   if (N == 0) return PE_OK;
   const int grid_n = (int)((N + kFleetWarps - 1) / kFleetWarps);
-  const int64_t Lx = (int64_t)L + H;
+  const int64_t Lx = ws.Lp;
   ProfScope ps(PE_PROF_FLEET_WINDOWS, st);
   switch (W) {
-    case 1: fleet_windows_kernel<1><<<grid_n, 32 * kFleetWarps, 0, st>>>(ws.jobq, J, Lx, offsets, N, H, win, counts, peaks); break;
-    case 2: fleet_windows_kernel<2><<<grid_n, 32 * kFleetWarps, 0, st>>>(ws.jobq, J, Lx, offsets, N, H, win, counts, peaks); break;
-    case 3: fleet_windows_kernel<3><<<grid_n, 32 * kFleetWarps, 0, st>>>(ws.jobq, J, Lx, offsets, N, H, win, counts, peaks); break;
-    default: fleet_windows_kernel<4><<<grid_n, 32 * kFleetWarps, 0, st>>>(ws.jobq, J, Lx, offsets, N, H, win, counts, peaks); break;
+    case 1: fleet_windows_kernel<1><<<grid_n, 32 * kFleetWarps, 0, st>>>(ws.prex, J, Lx, offsets, N, H, win, counts, peaks); break;
+    case 2: fleet_windows_kernel<2><<<grid_n, 32 * kFleetWarps, 0, st>>>(ws.prex, J, Lx, offsets, N, H, win, counts, peaks); break;
+    case 3: fleet_windows_kernel<3><<<grid_n, 32 * kFleetWarps, 0, st>>>(ws.prex, J, Lx, offsets, N, H, win, counts, peaks); break;
+    default: fleet_windows_kernel<4><<<grid_n, 32 * kFleetWarps, 0, st>>>(ws.prex, J, Lx, offsets, N, H, win, counts, peaks); break;
   }
   PE_CHECK_LAUNCH("fleet_windows_kernel");
   return PE_OK;

@@ -57,7 +57,7 @@ extern "C" pe_status pe_fleet_windows_noalloc(const float* traces, int32_t G, in
   const int64_t need = fleet_ws_bytes(J, L, H);
   if (need > (int64_t)PE_FLEET_NOALLOC_SCRATCH_BYTES)
     return fail(PE_EINVAL,
-                "fleet scratch of %lld bytes (J * (L + H) * 4 + 512) exceeds the fixed %lld-byte "
+                "fleet scratch of %lld bytes (pe_fleet_workspace_bytes) exceeds the fixed %lld-byte "
                 "static scratch of pe_fleet_windows_noalloc; use pe_fleet_windows with a workspace",
                 (long long)need, (long long)PE_FLEET_NOALLOC_SCRATCH_BYTES);
   void* scratch = nullptr;

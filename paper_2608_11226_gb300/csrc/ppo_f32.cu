@@ -379,40 +379,104 @@ __global__ void __launch_bounds__(kPpoNT) ppo_grad_kernel(PpoArgs g) {
     ppo_role<D, H, A, false>(s, g, blockIdx.x - g.NC);
 }
 
-__global__ void ppo_reduce_kernel(const float* __restrict__ partial, int NC, int64_t P,
-                                  float* __restrict__ grad, double* __restrict__ sq) {
-  __shared__ double red[32];
-  const int64_t p = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-  double gsum = 0.0;
-  if (p < P) {
-    for (int c = 0; c < NC; ++c) gsum += (double)__ldg(partial + (int64_t)c * P + p);
-    grad[p] = (float)gsum;
+// grad[p] = sum_c partial[c][p] in a fixed order: a block covers 32
+// parameters x 8 partial-row groups (row c goes to group c % 8), the groups
+// are combined in shared memory in group order.  The last block to finish
+// (atomic ticket; no block waits for another) forms the global norm from the
+// per-block sums of squares in block order and the minibatch statistics.
+constexpr int kRedP = 32, kRedG = 8;
+
+struct ReduceArgs {
+  const float* partial;
+  const float* stat_partial;  // [2*NC][8]
+  int NC;
+  int64_t P;
+  float* grad;
+  double* sq;             // [gridDim.x]
+  unsigned int* ticket;   // zeroed before the first launch; the last block re-zeroes it
+  double* norm;           // [1] out
+  double* acc;            // [8] running statistics
+  float vf_coef, ent_coef, inv_cnt;
+};
+
+__global__ void __launch_bounds__(kRedP * kRedG) ppo_reduce_kernel(ReduceArgs a) {
+  __shared__ double part[kRedG][kRedP];
+  __shared__ double red[kRedG];
+  __shared__ bool last;
+  const int lp = threadIdx.x % kRedP, cg = threadIdx.x / kRedP;
+  const int64_t p = (int64_t)blockIdx.x * kRedP + lp;
+  double s = 0.0;
+  if (p < a.P)
+    for (int c = cg; c < a.NC; c += kRedG) s += (double)__ldg(a.partial + (int64_t)c * a.P + p);
+  part[cg][lp] = s;
+  __syncthreads();
+  if (cg == 0) {
+    double g = 0.0;
+#pragma unroll
+    for (int k = 0; k < kRedG; ++k) g += part[k][lp];
+    const float gf = (float)g;
+    if (p < a.P) a.grad[p] = gf;
+    double q = p < a.P ? (double)gf * (double)gf : 0.0;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) q += __shfl_xor_sync(0xffffffffu, q, o);
+    if (lp == 0) {
+      a.sq[blockIdx.x] = q;
+      __threadfence();
+      const unsigned int t = atomicAdd(a.ticket, 1u);
+      last = (t == gridDim.x - 1);
+    }
   }
-  const float gf = (float)gsum;
-  const double t = block_sum_d((double)gf * (double)gf, red);
-  if (threadIdx.x == 0) sq[blockIdx.x] = t;
+  __syncthreads();
+  if (!last) return;
+  __threadfence();
+  // last block: global norm (fixed order: strided partial sums, then warp tree)
+  double q = 0.0;
+  for (int b = threadIdx.x; b < (int)gridDim.x; b += blockDim.x) q += *((volatile double*)a.sq + b);
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) q += __shfl_xor_sync(0xffffffffu, q, o);
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = q;
+  __syncthreads();
+  if (threadIdx.x < 32) {
+    // minibatch statistics: lane c sums rows c, c+32, ... of the stat partials
+    double v[5] = {0, 0, 0, 0, 0};
+    for (int c = threadIdx.x; c < a.NC; c += 32) {
+      v[0] += a.stat_partial[c * 8 + 0];
+      v[1] += a.stat_partial[c * 8 + 1];
+      v[2] += a.stat_partial[c * 8 + 2];
+      v[3] += a.stat_partial[c * 8 + 3];
+      v[4] += a.stat_partial[(a.NC + c) * 8 + 4];
+    }
+#pragma unroll
+    for (int k = 0; k < 5; ++k)
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) v[k] += __shfl_xor_sync(0xffffffffu, v[k], o);
+    if (threadIdx.x == 0) {
+      double t = 0.0;
+      for (int k = 0; k < kRedG; ++k) t += red[k];
+      const double norm = sqrt(t);
+      *a.norm = norm;
+      const double ic = a.inv_cnt;
+      a.acc[0] += v[0] * ic;
+      a.acc[1] += v[4] * ic;
+      a.acc[2] += v[1] * ic;
+      a.acc[3] += v[2] * ic;
+      a.acc[4] += v[3] * ic;
+      a.acc[5] += v[0] * ic + a.vf_coef * v[4] * ic - a.ent_coef * v[1] * ic;
+      a.acc[6] = norm;
+      a.acc[7] += 1.0;
+      *a.ticket = 0u;
+    }
+  }
 }
 
 struct AdamArgs {
   float beta1, beta2, step_size, inv_sqrt_bc2, eps, max_norm;
-  float clip, vf_coef, ent_coef, inv_cnt;
 };
 
 __global__ void ppo_adam_kernel(float* __restrict__ params, float* __restrict__ m,
                                 float* __restrict__ v, const float* __restrict__ grad,
-                                const double* __restrict__ sq, int nsq, int64_t P, AdamArgs a,
-                                const float* __restrict__ stat_partial, int NC,
-                                double* __restrict__ acc) {
-  __shared__ double s_norm;
-  if (threadIdx.x < 32) {
-    double t = 0.0;
-    for (int b = threadIdx.x; b < nsq; b += 32) t += sq[b];
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
-    if (threadIdx.x == 0) s_norm = sqrt(t);
-  }
-  __syncthreads();
-  const double norm = s_norm;
+                                const double* __restrict__ norm_p, int64_t P, AdamArgs a) {
+  const double norm = *norm_p;
   const float coef = (float)fmin(1.0, (double)a.max_norm / (norm + 1e-6));
   for (int64_t p = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; p < P;
        p += (int64_t)gridDim.x * blockDim.x) {
@@ -422,25 +486,6 @@ __global__ void ppo_adam_kernel(float* __restrict__ params, float* __restrict__ 
     m[p] = mp;
     v[p] = vp;
     params[p] -= a.step_size * mp / (sqrtf(vp) * a.inv_sqrt_bc2 + a.eps);
-  }
-  if (blockIdx.x == 0 && threadIdx.x == 0) {
-    double pg = 0, ent = 0, kl = 0, cf = 0, vl = 0;
-    for (int c = 0; c < NC; ++c) {
-      pg += stat_partial[c * 8 + 0];
-      ent += stat_partial[c * 8 + 1];
-      kl += stat_partial[c * 8 + 2];
-      cf += stat_partial[c * 8 + 3];
-      vl += stat_partial[(NC + c) * 8 + 4];
-    }
-    const double ic = a.inv_cnt;
-    acc[0] += pg * ic;
-    acc[1] += vl * ic;
-    acc[2] += ent * ic;
-    acc[3] += kl * ic;
-    acc[4] += cf * ic;
-    acc[5] += pg * ic + a.vf_coef * vl * ic - a.ent_coef * ent * ic;
-    acc[6] = norm;
-    acc[7] += 1.0;
   }
 }
 
@@ -486,14 +531,14 @@ static PpoPlan ppo_plan(const pe_net& net, const pe_ppo_config& cfg, int64_t N) 
   const int slices = (cfg.minibatch + kPpoS - 1) / kPpoS;
   p.NC = slices < 64 ? slices : 64;
   p.slices_per_cta = (slices + p.NC - 1) / p.NC;
-  p.nsq = (int)((p.P + 255) / 256);
+  p.nsq = (int)((p.P + kRedP - 1) / kRedP);
   int64_t o = 0;
   p.off_advstat = o; o = align256(o + (int64_t)cfg.epochs * p.nmb * 8);
   p.off_partial = o; o = align256(o + (int64_t)p.NC * p.P * 4);
   p.off_stat = o; o = align256(o + (int64_t)2 * p.NC * 8 * 4);
   p.off_grad = o; o = align256(o + p.P * 4);
   p.off_sq = o; o = align256(o + (int64_t)p.nsq * 8);
-  p.off_acc = o; o = align256(o + 8 * 8);
+  p.off_acc = o; o = align256(o + 8 * 8 + 16);
   p.total = o;
   return p;
 }
@@ -514,7 +559,9 @@ static pe_status ppo_run(const pe_net& net, float* params, float* m, float* v, i
   float* grad = reinterpret_cast<float*>(ws + pl.off_grad);
   double* sq = reinterpret_cast<double*>(ws + pl.off_sq);
   double* acc = reinterpret_cast<double*>(ws + pl.off_acc);
-  PE_TRY_CUDA(cudaMemsetAsync(acc, 0, 8 * sizeof(double), st));
+  double* norm = acc + 8;
+  unsigned int* ticket = reinterpret_cast<unsigned int*>(acc + 9);
+  PE_TRY_CUDA(cudaMemsetAsync(acc, 0, 8 * sizeof(double) + 16, st));
   FeistelSet perms{};
   for (int ep = 0; ep < cfg.epochs; ++ep) perms.f[ep] = make_feistel((uint64_t)N, cfg.seed, ep, cfg.iteration);
   {
@@ -561,7 +608,20 @@ static pe_status ppo_run(const pe_net& net, float* params, float* m, float* v, i
       PE_CHECK_LAUNCH("ppo_grad_kernel");
       {
         ProfScope ps(PE_PROF_PPO_REDUCE, st);
-        ppo_reduce_kernel<<<pl.nsq, 256, 0, st>>>(partial, pl.NC, pl.P, grad, sq);
+        ReduceArgs ra;
+        ra.partial = partial;
+        ra.stat_partial = stat_partial;
+        ra.NC = pl.NC;
+        ra.P = pl.P;
+        ra.grad = grad;
+        ra.sq = sq;
+        ra.ticket = ticket;
+        ra.norm = norm;
+        ra.acc = acc;
+        ra.vf_coef = cfg.vf_coef;
+        ra.ent_coef = cfg.ent_coef;
+        ra.inv_cnt = 1.0f / (float)cnt;
+        ppo_reduce_kernel<<<pl.nsq, kRedP * kRedG, 0, st>>>(ra);
       }
       PE_CHECK_LAUNCH("ppo_reduce_kernel");
       t += 1;
@@ -574,14 +634,9 @@ static pe_status ppo_run(const pe_net& net, float* params, float* m, float* v, i
       a.inv_sqrt_bc2 = (float)(1.0 / std::sqrt(bc2));
       a.eps = cfg.eps;
       a.max_norm = cfg.max_grad_norm;
-      a.clip = cfg.clip;
-      a.vf_coef = cfg.vf_coef;
-      a.ent_coef = cfg.ent_coef;
-      a.inv_cnt = 1.0f / (float)cnt;
-      const int agrid = (int)std::min<int64_t>((pl.P + 255) / 256, 4 * sms);
       {
         ProfScope ps(PE_PROF_PPO_ADAM, st);
-        ppo_adam_kernel<<<agrid, 256, 0, st>>>(params, m, v, grad, sq, pl.nsq, pl.P, a, stat_partial, pl.NC, acc);
+        ppo_adam_kernel<<<(int)((pl.P + 255) / 256), 256, 0, st>>>(params, m, v, grad, norm, pl.P, a);
       }
       PE_CHECK_LAUNCH("ppo_adam_kernel");
     }
