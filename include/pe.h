@@ -102,7 +102,7 @@ typedef struct pe_env_config {
  * one flat fp32 vector, row-major W[out][in]:
  *   policy: W1[H][D] b1[H] W2[H][H] b2[H] W3[A][H] b3[A]
  *   value : V1[H][D] c1[H] V2[H][H] c2[H] V3[1][H] c3[1]
- * Supported (D, H, A, dtype): (8,64,3,F32), (16,128,5,F32).  A BF16 network
+ * Supported (D, H, A, dtype): (8,64,3,F32), (16,128,5,F32), (32,256,16,BF16).  A BF16 network
  * keeps fp32 master parameters; the library rounds weights, observations and
  * hidden activations to bf16 and accumulates in fp32. */
 typedef struct pe_net {
@@ -166,14 +166,22 @@ int64_t pe_param_count(const pe_net* net);
  * episode_len steps, new offset from ctr = (e, t, iteration, 1).
  * Then the value network on every observation and on obs_last.
  *  lambda: Lagrange multiplier of Eq. 6 (PE_REWARD_LAGRANGE only).
- * Errors: PE_EINVAL (unsupported network, null buffer, horizon < 1), PE_ECUDA. */
+ *  workspace: >= pe_rollout_workspace_bytes(env, net) bytes of device memory
+ *  (0 for fp32 networks: NULL is accepted).  BF16 networks (D=32, H=256,
+ *  A=16, 4 channels) run on the tcgen05 tensor cores.
+ * Errors: PE_EINVAL (unsupported network, null buffer, horizon < 1, small
+ * workspace), PE_ECUDA; a bounded tensor-core wait that gives up on the
+ * device is reported by pe_device_check. */
+int64_t pe_rollout_workspace_bytes(const pe_env* env, const pe_net* net);
 pe_status pe_rollout(pe_env* env, const pe_net* net, const float* params, int32_t horizon,
                      uint32_t iteration, float lambda, int32_t flags, const pe_rollout_buf* buf,
-                     void* stream);
+                     void* workspace, int64_t workspace_bytes, void* stream);
 
-/* Value network on n observations (fp32, or bf16 for a BF16 network). */
+/* Value network on n observations (fp32, or bf16 for a BF16 network).
+ * workspace: >= pe_value_workspace_bytes(net) bytes (0 for fp32). */
+int64_t pe_value_workspace_bytes(const pe_net* net);
 pe_status pe_value(const pe_net* net, const float* params, const void* obs, int64_t n,
-                   float* value, void* stream);
+                   float* value, void* workspace, int64_t workspace_bytes, void* stream);
 
 /* Generalised advantage estimation (gamma, lambda per Sec. 4.2), time-major:
  *   delta_t = r_t + gamma (1 - d_t) V_{t+1} - V_t,  V_T = last_value,
@@ -264,6 +272,10 @@ pe_status pe_fleet_windows_noalloc(const float* traces, int32_t G, int32_t L,
 pe_status pe_profile_enable(int32_t on);
 pe_status pe_profile_read(int32_t kind, double* total_ms, int64_t* launches);
 const char* pe_profile_kind_name(int32_t kind);
+
+/* Synchronise `stream`, then report device-side errors of earlier launches:
+ * PE_ETIMEOUT if a bounded tensor-core wait gave up (the flag is cleared). */
+pe_status pe_device_check(void* stream);
 
 /* Message for the last non-OK status on this thread ("" if none). */
 const char* pe_last_error(void);

@@ -84,6 +84,13 @@ pe_status ppo_update_f32(const pe_net& net, float* params, float* m, float* v, i
                          const float* adv, const float* ret, int64_t N, const pe_ppo_config& cfg,
                          float* stats, void* ws, cudaStream_t st);
 int64_t fleet_ws_bytes(int J, int L, int H);
+int64_t rollout_bf16_ws_bytes(const pe_net& net, int64_t E);
+pe_status rollout_bf16(const EnvDev& env, const pe_net& net, const float* params, int T, uint32_t it,
+                       float lambda, int det, const pe_rollout_buf& buf, void* ws, cudaStream_t st);
+pe_status value_bf16(const pe_net& net, const float* params, const void* obs, int64_t n, float* value,
+                     void* ws, cudaStream_t st);
+int64_t value_bf16_ws_bytes(const pe_net& net);
+pe_status device_check(cudaStream_t st);
 pe_status fleet_launch(const float* traces, int G, int L, const int32_t* job_of_gpu, int J,
                        const int32_t* offsets, int64_t N, int H, const int32_t* windows, int W,
                        int64_t budget_q, int32_t* counts, int32_t* peaks, void* workspace,
@@ -99,20 +106,26 @@ static int obs_width(int kind) {
   }
 }
 
-// episode start offsets and the default level for every env
+// first episode of every env (Sec. 4.1 random offset, warm-started history and
+// window sums), through the same reset as later episodes
+template <int C>
 __global__ void env_init_kernel(EnvDev env) {
   const int e = blockIdx.x * blockDim.x + threadIdx.x;
   if (e >= env.E) return;
-  const uint32_t u = draw32(env.seed, (uint32_t)e, 0u, 0u, kDrawInit);
-  const uint32_t span = (uint32_t)(env.L - env.ep_len - kWLong + 1);
-  env.st[kStPos * env.E + e] = kWLong + (int)__umulhi(u, span);
-  env.st[kStK * env.E + e] = 0;
-  env.st[kStLevel * env.E + e] = env.level_init;
-  env.st[kStPrev * env.E + e] = env.level_init;
-  env.st[kStB * env.E + e] = env.b_init;
-  env.st[kStTil * env.E + e] = 0;
-  for (int i = 0; i < kRing; ++i) env.ring[(int64_t)e * kRing + i] = (uint8_t)env.level_init;
-  for (int i = 0; i < 8; ++i) env.sums[(int64_t)e * 8 + i] = 0;
+  RegAcc<C> a;
+  a.ring = env.ring + (int64_t)e * kRing;
+  env_reset<C>(env, a, (uint32_t)e, 0u, 0u, kDrawInit);
+  store_reg<C>(env, e, a);
+}
+
+static void launch_env_init(const EnvDev& d) {
+  const int grid = ceil_div(d.E, 256);
+  switch (d.C) {
+    case 1: env_init_kernel<1><<<grid, 256>>>(d); break;
+    case 2: env_init_kernel<2><<<grid, 256>>>(d); break;
+    case 3: env_init_kernel<3><<<grid, 256>>>(d); break;
+    default: env_init_kernel<4><<<grid, 256>>>(d); break;
+  }
 }
 
 }  // namespace pe
@@ -284,7 +297,7 @@ pe_status pe_env_create(const pe_env_config* cfg, const float* trace, const uint
   d.trace = dtrace; d.phase = dphase; d.st = st; d.ring = ring; d.sums = sums;
   PE_TRY_CUDA(cudaMemcpy(dtrace, h.data(), sizeof(float) * h.size(), cudaMemcpyHostToDevice));
   PE_TRY_CUDA(cudaMemcpy(dphase, ph.data(), ph.size(), cudaMemcpyHostToDevice));
-  env_init_kernel<<<ceil_div(E, 256), 256>>>(d);  // one-time set-up, not profiled
+  launch_env_init(d);  // one-time set-up, not profiled
   PE_CHECK_LAUNCH("env_init_kernel");
   PE_TRY_CUDA(cudaDeviceSynchronize());
   *out = env;
@@ -351,9 +364,15 @@ static pe_status check_net(const pe_net* net) {
   return PE_OK;
 }
 
+int64_t pe_rollout_workspace_bytes(const pe_env* env, const pe_net* net) {
+  if (!env || !net) return -1;
+  if (net->dtype == PE_F32) return 0;
+  return rollout_bf16_ws_bytes(*net, env->dev.E);
+}
+
 pe_status pe_rollout(pe_env* env, const pe_net* net, const float* params, int32_t horizon,
                      uint32_t iteration, float lambda, int32_t flags, const pe_rollout_buf* buf,
-                     void* stream) {
+                     void* workspace, int64_t workspace_bytes, void* stream) {
   clear_error();
   if (!env || !params || !buf) return fail(PE_EINVAL, "null argument");
   pe_status s = check_net(net);
@@ -377,20 +396,38 @@ pe_status pe_rollout(pe_env* env, const pe_net* net, const float* params, int32_
     return value_f32(*net, params, reinterpret_cast<const float*>(buf->obs_last), env->dev.E,
                      buf->last_value, st);
   }
-  return fail(PE_EINVAL, "bf16 networks are not supported by pe_rollout in this build");
+  const int64_t need = rollout_bf16_ws_bytes(*net, env->dev.E);
+  if (need < 0) return fail(PE_EINVAL, "unsupported bf16 network (D=%d H=%d)", net->obs_dim, net->hidden);
+  if (!workspace || workspace_bytes < need)
+    return fail(PE_EINVAL, "workspace too small (%lld < %lld bytes)", (long long)workspace_bytes, (long long)need);
+  return rollout_bf16(env->dev, *net, params, horizon, iteration, lambda, det, *buf, workspace, st);
+}
+
+int64_t pe_value_workspace_bytes(const pe_net* net) {
+  if (!net) return -1;
+  if (net->dtype == PE_F32) return 0;
+  return value_bf16_ws_bytes(*net);
 }
 
 pe_status pe_value(const pe_net* net, const float* params, const void* obs, int64_t n,
-                   float* value, void* stream) {
+                   float* value, void* workspace, int64_t workspace_bytes, void* stream) {
   clear_error();
   pe_status s = check_net(net);
   if (s != PE_OK) return s;
   if (!params || (n > 0 && (!obs || !value))) return fail(PE_EINVAL, "null argument");
   if (n < 0) return fail(PE_EINVAL, "n must be >= 0");
-  if (net->dtype == PE_F32)
-    return value_f32(*net, params, reinterpret_cast<const float*>(obs), n, value,
-                     reinterpret_cast<cudaStream_t>(stream));
-  return fail(PE_EINVAL, "bf16 networks are not supported by pe_value in this build");
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  if (net->dtype == PE_F32) return value_f32(*net, params, reinterpret_cast<const float*>(obs), n, value, st);
+  const int64_t need = value_bf16_ws_bytes(*net);
+  if (need < 0) return fail(PE_EINVAL, "unsupported bf16 value network (D=%d H=%d)", net->obs_dim, net->hidden);
+  if (!workspace || workspace_bytes < need)
+    return fail(PE_EINVAL, "workspace too small (%lld < %lld bytes)", (long long)workspace_bytes, (long long)need);
+  return value_bf16(*net, params, obs, n, value, workspace, st);
+}
+
+pe_status pe_device_check(void* stream) {
+  clear_error();
+  return device_check(reinterpret_cast<cudaStream_t>(stream));
 }
 
 pe_status pe_gae(const float* reward, const float* value, const uint8_t* done,

@@ -53,121 +53,167 @@ __device__ __forceinline__ int32_t sample_q(const EnvDev& env, int c, int pos, i
   return quant64(x, actuator_scale(env, level, c, __ldg(env.phase + pos)));
 }
 
-// rebuild the 60-sample history of env slot e from its level ring
+// ---------------------------------------------------------------------------
+// Two views of one env's state with the same interface:
+//   TileAcc -- a slot of an EnvTile in shared memory, with the actuated
+//              per-channel samples of the last 64 positions cached;
+//   RegAcc  -- scalars in registers, level ring in global memory, samples
+//              recomputed from the trace and the ring when needed.
+// The features, the step and the reset below are written once over either.
+// ---------------------------------------------------------------------------
 template <int TE, int C>
-__device__ void rebuild_history(const EnvDev& env, EnvTile<TE, C>& s, int e) {
-  const int p = s.pos[e];
+struct TileAcc {
+  EnvTile<TE, C>& s;
+  int e;
+  __device__ int32_t& pos() { return s.pos[e]; }
+  __device__ int32_t& k() { return s.k[e]; }
+  __device__ int32_t& level() { return s.level[e]; }
+  __device__ int32_t& prev() { return s.prev[e]; }
+  __device__ int32_t& b() { return s.b[e]; }
+  __device__ int32_t& til() { return s.til[e]; }
+  __device__ int32_t& ss(int c) { return s.s_short[e][c]; }
+  __device__ int32_t& sl(int c) { return s.s_long[e][c]; }
+  __device__ uint8_t level_at(int p) const { return s.ring[e][p & (kRing - 1)]; }
+  __device__ void set_level_at(int p, int l) { s.ring[e][p & (kRing - 1)] = (uint8_t)l; }
+  // actuated sample of channel c at a recent position p (p in [pos-64, pos))
+  __device__ int32_t q_at(const EnvDev&, int c, int p) const { return s.q[e][c][p & (kRing - 1)]; }
+  __device__ void push(int c, int p, int32_t q) { s.q[e][c][p & (kRing - 1)] = q; }
+};
+
+template <int C>
+struct RegAcc {
+  int32_t pos_, k_, level_, prev_, b_, til_;
+  int32_t ss_[C], sl_[C];
+  uint8_t* ring;  // global [64]
+  __device__ int32_t& pos() { return pos_; }
+  __device__ int32_t& k() { return k_; }
+  __device__ int32_t& level() { return level_; }
+  __device__ int32_t& prev() { return prev_; }
+  __device__ int32_t& b() { return b_; }
+  __device__ int32_t& til() { return til_; }
+  __device__ int32_t& ss(int c) { return ss_[c]; }
+  __device__ int32_t& sl(int c) { return sl_[c]; }
+  __device__ uint8_t level_at(int p) const { return ring[p & (kRing - 1)]; }
+  __device__ void set_level_at(int p, int l) { ring[p & (kRing - 1)] = (uint8_t)l; }
+  __device__ int32_t q_at(const EnvDev& env, int c, int p) const { return sample_q(env, c, p, level_at(p)); }
+  __device__ void push(int, int, int32_t) {}
+};
+
+// 60-sample history before the current position at the recorded levels
+template <int C, class Acc>
+__device__ void rebuild_history(const EnvDev& env, Acc& a) {
+  const int p = a.pos();
   for (int c = 0; c < C; ++c) {
     int32_t ss = 0, sl = 0;
     for (int i = 1; i <= kWLong; ++i) {
       const int pp = p - i;
-      const int32_t q = sample_q(env, c, pp, s.ring[e][pp & (kRing - 1)]);
-      s.q[e][c][pp & (kRing - 1)] = q;
+      const int32_t q = sample_q(env, c, pp, a.level_at(pp));
+      a.push(c, pp, q);
       sl += q;
       if (i <= kWShort) ss += q;
     }
-    s.s_short[e][c] = ss;
-    s.s_long[e][c] = sl;
+    a.ss(c) = ss;
+    a.sl(c) = sl;
   }
 }
 
-// new episode for env slot e (global index eg): Philox offset, warm start
-template <int TE, int C>
-__device__ void env_reset(const EnvDev& env, EnvTile<TE, C>& s, int e, uint32_t eg, uint32_t t,
-                          uint32_t it, uint32_t purpose) {
+// new episode (Sec. 4.1: random offset; Sec. 4.5: warm start at the default level)
+template <int C, class Acc>
+__device__ void env_reset(const EnvDev& env, Acc& a, uint32_t eg, uint32_t t, uint32_t it,
+                          uint32_t purpose) {
   const uint32_t u = draw32(env.seed, eg, t, it, purpose);
   const uint32_t span = (uint32_t)(env.L - env.ep_len - kWLong + 1);
   const int o = kWLong + (int)__umulhi(u, span);
-  s.pos[e] = o;
-  s.k[e] = 0;
-  s.level[e] = env.level_init;
-  s.prev[e] = env.level_init;
-  s.b[e] = env.b_init;
-  s.til[e] = 0;
-  for (int i = 0; i < kRing; ++i) s.ring[e][i] = (uint8_t)env.level_init;
-  rebuild_history<TE, C>(env, s, e);
+  a.pos() = o;
+  a.k() = 0;
+  a.level() = env.level_init;
+  a.prev() = env.level_init;
+  a.b() = env.b_init;
+  a.til() = 0;
+  for (int i = 0; i < kRing; ++i) a.set_level_at(i, env.level_init);
+  rebuild_history<C>(env, a);
 }
 
-template <int TE, int C>
-__device__ __forceinline__ int32_t Qc(const EnvTile<TE, C>& s, int e, int c, int i) {
-  return s.q[e][c][(s.pos[e] - 1 - i) & (kRing - 1)];
+template <int C, class Acc>
+__device__ __forceinline__ int32_t Qc(const EnvDev& env, Acc& a, int c, int i) {
+  return a.q_at(env, c, a.pos() - 1 - i);
 }
 
-template <int TE, int C>
-__device__ __forceinline__ int32_t Qcl(const EnvTile<TE, C>& s, int e, int i) {
+template <int C, class Acc>
+__device__ __forceinline__ int32_t Qcl(const EnvDev& env, Acc& a, int i) {
   int32_t v = 0;
 #pragma unroll
-  for (int c = 0; c < C; ++c) v += Qc<TE, C>(s, e, c, i);
+  for (int c = 0; c < C; ++c) v += Qc<C>(env, a, c, i);
   return v;
 }
 
-// Observation feature f of env slot e (fp32 quotient of exact integers;
-// all power quantities are normalised by the budget B).
+// Observation feature f (fp32 quotient of exact integers; all power
+// quantities are normalised by the budget B).
 //   TINY8 (Sec. 4.1): 5 latest samples, headroom, phase, level
 //   7B16: 8 latest samples, 30 s mean, 30 s slack, phase, G, b, 10 s mean, 5 s slope, 0
 //   OCC32/OCC64: Eq. 5 eight-vector, then per-channel recent samples and means
-template <int TE, int C, int OBS>
-__device__ __forceinline__ float feature(const EnvDev& env, const EnvTile<TE, C>& s, int e, int f) {
+template <int C, int OBS, class Acc>
+__device__ __forceinline__ float feature(const EnvDev& env, Acc& a, int f) {
   const int64_t B = env.budget_q;
   if (OBS == PE_OBS_TINY8) {
-    if (f < 5) return ratio_i(Qcl<TE, C>(s, e, 4 - f), B);
-    if (f == 5) return ratio_i(B - Qcl<TE, C>(s, e, 0), B);
-    if (f == 6) return (float)__ldg(env.phase + s.pos[e] - 1);
-    return ratio_i(s.level[e], env.n_levels - 1);
+    if (f < 5) return ratio_i(Qcl<C>(env, a, 4 - f), B);
+    if (f == 5) return ratio_i(B - Qcl<C>(env, a, 0), B);
+    if (f == 6) return (float)__ldg(env.phase + a.pos() - 1);
+    return ratio_i(a.level(), env.n_levels - 1);
   }
   int64_t S20 = 0, S60 = 0;
 #pragma unroll
   for (int c = 0; c < C; ++c) {
-    S20 += s.s_short[e][c];
-    S60 += s.s_long[e][c];
+    S20 += a.ss(c);
+    S60 += a.sl(c);
   }
   if (OBS == PE_OBS_7B16) {
-    if (f < 8) return ratio_i(Qcl<TE, C>(s, e, 7 - f), B);
+    if (f < 8) return ratio_i(Qcl<C>(env, a, 7 - f), B);
     switch (f) {
       case 8: return ratio_i(S60, kWLong * B);
       case 9: return ratio_i(kWLong * B - S60, kWLong * B);
-      case 10: return (float)__ldg(env.phase + s.pos[e] - 1);
-      case 11: return ratio_i(s.level[e] - env.g_min, env.g_max - env.g_min);
-      case 12: return ratio_i(s.b[e] - env.b_min, env.b_max - env.b_min);
+      case 10: return (float)__ldg(env.phase + a.pos() - 1);
+      case 11: return ratio_i(a.level() - env.g_min, env.g_max - env.g_min);
+      case 12: return ratio_i(a.b() - env.b_min, env.b_max - env.b_min);
       case 13: return ratio_i(S20, kWShort * B);
-      case 14: return ratio_i((int64_t)Qcl<TE, C>(s, e, 0) - Qcl<TE, C>(s, e, 10), B);
+      case 14: return ratio_i((int64_t)Qcl<C>(env, a, 0) - Qcl<C>(env, a, 10), B);
       default: return 0.0f;
     }
   }
   // OCC32 / OCC64 (Eq. 5 core)
   switch (f) {
-    case 0: return ratio_i(Qcl<TE, C>(s, e, 0), B);
+    case 0: return ratio_i(Qcl<C>(env, a, 0), B);
     case 1: return ratio_i(S20, kWShort * B);
     case 2: return ratio_i(S60, kWLong * B);
     case 3: return ratio_i(kWLong * B - S60, kWLong * B);
-    case 4: return ratio_i((int64_t)Qcl<TE, C>(s, e, 0) - Qcl<TE, C>(s, e, 10), B);
-    case 5: return ratio_i(s.level[e] + 1, env.n_levels);
-    case 6: return ratio_i(s.prev[e] + 1, env.n_levels);
-    case 7: return fminf(ratio_i(s.til[e], 40), 1.0f);
+    case 4: return ratio_i((int64_t)Qcl<C>(env, a, 0) - Qcl<C>(env, a, 10), B);
+    case 5: return ratio_i(a.level() + 1, env.n_levels);
+    case 6: return ratio_i(a.prev() + 1, env.n_levels);
+    case 7: return fminf(ratio_i(a.til(), 40), 1.0f);
     default: break;
   }
   if (OBS == PE_OBS_OCC32) {
     if (f < 24) {
       const int c = (f - 8) >> 2, i = (f - 8) & 3;
-      return c < C ? ratio_i((int64_t)C * Qc<TE, C>(s, e, c, 3 - i), B) : 0.0f;
+      return c < C ? ratio_i((int64_t)C * Qc<C>(env, a, c, 3 - i), B) : 0.0f;
     }
     if (f < 28) {
       const int c = f - 24;
-      return c < C ? ratio_i((int64_t)C * s.s_long[e][c], kWLong * B) : 0.0f;
+      return c < C ? ratio_i((int64_t)C * a.sl(c), kWLong * B) : 0.0f;
     }
     return 0.0f;
   }
   // OCC64
   if (f < 56) {
     const int c = (f - 8) / 12, i = (f - 8) % 12;
-    return c < C ? ratio_i((int64_t)C * Qc<TE, C>(s, e, c, 11 - i), B) : 0.0f;
+    return c < C ? ratio_i((int64_t)C * Qc<C>(env, a, c, 11 - i), B) : 0.0f;
   }
   if (f < 60) {
     const int c = f - 56;
-    return c < C ? ratio_i((int64_t)C * s.s_short[e][c], kWShort * B) : 0.0f;
+    return c < C ? ratio_i((int64_t)C * a.ss(c), kWShort * B) : 0.0f;
   }
   const int c = f - 60;
-  return c < C ? ratio_i((int64_t)C * s.s_long[e][c], kWLong * B) : 0.0f;
+  return c < C ? ratio_i((int64_t)C * a.sl(c), kWLong * B) : 0.0f;
 }
 
 struct StepOut {
@@ -175,39 +221,38 @@ struct StepOut {
   int32_t q, v1, v60, done;
 };
 
-// Apply action a to env slot e and consume one sample (Sec. 4.1 actuator and
-// action set with the Sec. 4.2 floor g_min; Eqs. 1-3; G1 or Eq. 6 reward).
-template <int TE, int C>
-__device__ __forceinline__ StepOut env_step(const EnvDev& env, EnvTile<TE, C>& s, int e, int a,
-                                            float lambda) {
-  int nl = s.level[e];
+// Apply action act and consume one sample (Sec. 4.1 actuator and action set
+// with the Sec. 4.2 floor g_min; Eqs. 1-3; G1 or Eq. 6 reward).
+template <int C, class Acc>
+__device__ __forceinline__ StepOut env_step(const EnvDev& env, Acc& a, int act, float lambda) {
+  int nl = a.level();
   if (env.act_kind == PE_ACT_INCDEC) {
-    if (a == 1 && nl > env.g_min) --nl;
-    if (a == 2 && nl < env.g_max) ++nl;
-    if (a == 3 && s.b[e] > env.b_min) s.b[e] -= 1;
-    if (a == 4 && s.b[e] < env.b_max) s.b[e] += 1;
+    if (act == 1 && nl > env.g_min) --nl;
+    if (act == 2 && nl < env.g_max) ++nl;
+    if (act == 3 && a.b() > env.b_min) a.b() -= 1;
+    if (act == 4 && a.b() < env.b_max) a.b() += 1;
   } else {
-    nl = a;
+    nl = act;
   }
-  s.til[e] = (nl != s.level[e]) ? 0 : s.til[e] + 1;
-  s.prev[e] = s.level[e];
-  s.level[e] = nl;
-  const int p = s.pos[e];
+  a.til() = (nl != a.level()) ? 0 : a.til() + 1;
+  a.prev() = a.level();
+  a.level() = nl;
+  const int p = a.pos();
   const int ph = __ldg(env.phase + p);
-  s.ring[e][p & (kRing - 1)] = (uint8_t)nl;
   int32_t Q = 0;
   int64_t S60 = 0;
 #pragma unroll
   for (int c = 0; c < C; ++c) {
     const int32_t qin = quant64(__ldg(env.trace + (int64_t)c * env.L + p), actuator_scale(env, nl, c, ph));
-    const int32_t q20 = s.q[e][c][(p - kWShort) & (kRing - 1)];
-    const int32_t q60 = s.q[e][c][(p - kWLong) & (kRing - 1)];
-    s.s_short[e][c] += qin - q20;
-    s.s_long[e][c] += qin - q60;
-    s.q[e][c][p & (kRing - 1)] = qin;
+    const int32_t q20 = a.q_at(env, c, p - kWShort);
+    const int32_t q60 = a.q_at(env, c, p - kWLong);
+    a.ss(c) += qin - q20;
+    a.sl(c) += qin - q60;
+    a.push(c, p, qin);
     Q += qin;
-    S60 += s.s_long[e][c];
+    S60 += a.sl(c);
   }
+  a.set_level_at(p, nl);  // after the window updates: slot p & 63 held position p - 64
   const int64_t B60 = (int64_t)kWLong * env.budget_q;
   StepOut o;
   o.q = Q;
@@ -216,7 +261,7 @@ __device__ __forceinline__ StepOut env_step(const EnvDev& env, EnvTile<TE, C>& s
   const float exc_w = o.v60 ? __fdiv_rn(__ll2float_rn(S60 - B60), 3840.0f) : 0.0f;  // watts over B
   o.excess = exc_w * 0.5f;                                                            // Eq. 3, W*s
   float rate = env.tokens[nl];
-  if (env.act_kind == PE_ACT_INCDEC) rate = __fdiv_rn(rate * (float)s.b[e], (float)env.b_init);
+  if (env.act_kind == PE_ACT_INCDEC) rate = __fdiv_rn(rate * (float)a.b(), (float)env.b_init);
   o.tokens = ph == 0 ? rate : 0.0f;
   if (env.reward_kind == PE_REWARD_LAGRANGE) {
     o.reward = o.tokens / 1000.0f - lambda * o.excess - 2.0f * lambda * exc_w;  // Eq. 6
@@ -224,9 +269,9 @@ __device__ __forceinline__ StepOut env_step(const EnvDev& env, EnvTile<TE, C>& s
     const int viol = env.reward_window == 1 ? o.v1 : o.v60;
     o.reward = (viol ? env.r_viol : env.r_ok) + env.bonus_coef * rate * env.inv_rate_max;
   }
-  s.pos[e] = p + 1;
-  s.k[e] += 1;
-  o.done = s.k[e] == env.ep_len;
+  a.pos() = p + 1;
+  a.k() += 1;
+  o.done = a.k() == env.ep_len;
   return o;
 }
 
@@ -241,7 +286,8 @@ __device__ void load_tile(const EnvDev& env, EnvTile<TE, C>& s, int e0, int ne) 
     s.b[e] = env.st[kStB * env.E + g];
     s.til[e] = env.st[kStTil * env.E + g];
     for (int i = 0; i < kRing; ++i) s.ring[e][i] = env.ring[(int64_t)g * kRing + i];
-    rebuild_history<TE, C>(env, s, e);
+    TileAcc<TE, C> a{s, e};
+    rebuild_history<C>(env, a);
   }
 }
 
@@ -260,6 +306,40 @@ __device__ void store_tile(const EnvDev& env, const EnvTile<TE, C>& s, int e0, i
       env.sums[(int64_t)g * 8 + c] = c < C ? s.s_short[e][c] : 0;
       env.sums[(int64_t)g * 8 + 4 + c] = c < C ? s.s_long[e][c] : 0;
     }
+  }
+}
+
+// register view of env g (level ring stays in global memory)
+template <int C>
+__device__ __forceinline__ RegAcc<C> load_reg(const EnvDev& env, int g) {
+  RegAcc<C> a;
+  a.pos_ = env.st[kStPos * env.E + g];
+  a.k_ = env.st[kStK * env.E + g];
+  a.level_ = env.st[kStLevel * env.E + g];
+  a.prev_ = env.st[kStPrev * env.E + g];
+  a.b_ = env.st[kStB * env.E + g];
+  a.til_ = env.st[kStTil * env.E + g];
+  a.ring = env.ring + (int64_t)g * kRing;
+#pragma unroll
+  for (int c = 0; c < C; ++c) {
+    a.ss_[c] = env.sums[(int64_t)g * 8 + c];
+    a.sl_[c] = env.sums[(int64_t)g * 8 + 4 + c];
+  }
+  return a;
+}
+
+template <int C>
+__device__ __forceinline__ void store_reg(const EnvDev& env, int g, const RegAcc<C>& a) {
+  env.st[kStPos * env.E + g] = a.pos_;
+  env.st[kStK * env.E + g] = a.k_;
+  env.st[kStLevel * env.E + g] = a.level_;
+  env.st[kStPrev * env.E + g] = a.prev_;
+  env.st[kStB * env.E + g] = a.b_;
+  env.st[kStTil * env.E + g] = a.til_;
+#pragma unroll
+  for (int c = 0; c < 4; ++c) {
+    env.sums[(int64_t)g * 8 + c] = c < C ? a.ss_[c] : 0;
+    env.sums[(int64_t)g * 8 + 4 + c] = c < C ? a.sl_[c] : 0;
   }
 }
 

@@ -1,0 +1,427 @@
+// bf16 policy/value MLPs on the 5th-generation tensor cores (tcgen05), and the
+// decoupled rollout that uses them (72B workload: D=32, H=256, A=16, C=4).
+//
+// A policy/value network is tanh(W2 tanh(W1 x + b1) + b2) followed by a
+// linear head (Sec. 4.2 actor-critic), evaluated on 128-row tiles:
+//   - the fp32 master parameters are first converted once per call into a
+//     bf16 "weight image": each matrix laid out exactly as the kernel keeps it
+//     in shared memory (K-major, 128-byte or 64-byte swizzle);
+//   - a persistent CTA copies the image into shared memory with one bulk copy
+//     (cp.async.bulk, completion on an mbarrier) and keeps it for all its tiles;
+//   - per layer one thread issues tcgen05.mma (M=128, K=16 per instruction)
+//     into TMEM; eight warps read the fp32 accumulators back (tcgen05.ld),
+//     add the bias, apply tanh, round to bf16 and write the next layer's A
+//     operand into shared memory in the swizzled layout.
+// Precision: bf16 observations, weights and hidden activations, fp32
+// accumulation, fp32 bias and tanh -- the quantisation points the oracle
+// emulates.
+#include <type_traits>
+
+#include "env.cuh"
+#include "mlp_f32.cuh"
+#include "tc.cuh"
+
+namespace pe {
+
+// set when a bounded tensor-core wait gives up; read and cleared by pe_device_check
+__device__ int32_t g_tc_error = 0;
+
+constexpr int kTcRows = 128;     // rows (envs / samples) per tile, the MMA M
+constexpr int kTcThreads = 256;  // 8 warps: 4 TMEM lane quadrants x 2 column halves
+constexpr int kHeadN = 16;       // head width (logits or value padded to 16)
+
+// byte sizes of the weight image parts of one network (D, H)
+template <int D, int H>
+struct Img {
+  static constexpr int RB1 = D == 32 ? 64 : 128;        // layer-1 row bytes (SW64 for D=32)
+  static constexpr int W1 = H * RB1 * (D * 2 / RB1);     // H rows x D bf16
+  static constexpr int W2 = H * H * 2;                   // H rows x H bf16 (SW128)
+  static constexpr int W3 = kHeadN * H * 2;              // 16 rows x H bf16 (SW128)
+  static constexpr int TOTAL = W1 + W2 + W3;
+  static constexpr int ACT = kTcRows * H * 2;            // hidden activation tile
+  static_assert(D == 32 || D == 64, "obs width");
+  static_assert(H % 64 == 0 && H <= 256, "hidden width");
+  static_assert(TOTAL + ACT + 3 * 1024 <= 232448, "weights and one activation tile must fit in shared memory");
+};
+
+// fp32 canonical parameters -> bf16 swizzled weight image of one network
+// (policy: W1 W2 W3 of A rows; value: V1 V2 V3 of 1 row), rows >= nout of the
+// head are zero.
+template <int D, int H>
+__global__ void weight_image_kernel(const float* __restrict__ params, int A, int value_net,
+                                    uint8_t* __restrict__ img) {
+  using I = Img<D, H>;
+  const MlpLayout Lp = mlp_layout(D, H, A);
+  const float* w1 = params + (value_net ? Lp.v1 : Lp.w1);
+  const float* w2 = params + (value_net ? Lp.v2 : Lp.w2);
+  const float* w3 = params + (value_net ? Lp.v3 : Lp.w3);
+  const int nout = value_net ? 1 : A;
+  const int total = H * D + H * H + kHeadN * H;
+  for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < total; i += gridDim.x * blockDim.x) {
+    if (i < H * D) {
+      const int r = i / D, k = i % D;
+      *reinterpret_cast<__nv_bfloat16*>(img + tc::swz_offset<I::RB1>(r, k, H)) = __float2bfloat16_rn(w1[i]);
+    } else if (i < H * D + H * H) {
+      const int j = i - H * D, r = j / H, k = j % H;
+      *reinterpret_cast<__nv_bfloat16*>(img + I::W1 + tc::swz_offset<128>(r, k, H)) = __float2bfloat16_rn(w2[j]);
+    } else {
+      const int j = i - H * D - H * H, r = j / H, k = j % H;
+      const float v = r < nout ? w3[r * H + k] : 0.0f;
+      *reinterpret_cast<__nv_bfloat16*>(img + I::W1 + I::W2 + tc::swz_offset<128>(r, k, kHeadN)) =
+          __float2bfloat16_rn(v);
+    }
+  }
+}
+
+template <int D, int H>
+struct MlpBf16Smem {
+  // operand images (bulk-copied): W1 | W2 | W3, then the activation tile
+  alignas(1024) uint8_t w[Img<D, H>::TOTAL];
+  alignas(1024) uint8_t act[Img<D, H>::ACT];  // X (layer-1 A operand) aliases its start
+  float b1[H], b2[H], b3[kHeadN];
+  uint64_t bar_w, bar_mma;
+  uint32_t tmem_base;
+  int32_t err;
+};
+
+// fp32 epilogue of one layer: TMEM columns [col0, col0+H) -> tanh(. + b) -> bf16 A tile
+template <int H>
+__device__ __forceinline__ void epilogue_tanh(uint32_t tmem, int col0, const float* bias, uint8_t* act) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int quad = warp & 3, half = warp >> 2;
+  const int row = quad * 32 + lane;
+  const uint32_t lane_addr = tmem + ((uint32_t)(quad * 32) << 16);
+#pragma unroll 1
+  for (int j = 0; j < H / 2 / 16; ++j) {
+    const int c = half * (H / 2) + j * 16;
+    float v[16];
+    tc::tmem_ld16(lane_addr + (uint32_t)(col0 + c), v);
+    uint32_t p[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i)
+      p[i] = tc::pack_bf16(tanhf(v[2 * i] + bias[c + 2 * i]), tanhf(v[2 * i + 1] + bias[c + 2 * i + 1]));
+    *reinterpret_cast<uint4*>(act + tc::swz_offset<128>(row, c, kTcRows)) = make_uint4(p[0], p[1], p[2], p[3]);
+    *reinterpret_cast<uint4*>(act + tc::swz_offset<128>(row, c + 8, kTcRows)) = make_uint4(p[4], p[5], p[6], p[7]);
+  }
+}
+
+// One MLP over n rows of bf16 observations [n][D]; writes out[r * out_stride + j]
+// for j < nout.  Persistent over 128-row tiles.  *err is set to 1 if a bounded
+// wait timed out.
+template <int D, int H>
+__global__ void __launch_bounds__(kTcThreads, 1)
+    mlp_bf16_kernel(const uint8_t* __restrict__ img, const float* __restrict__ params, int A,
+                    int value_net, const __nv_bfloat16* __restrict__ obs, int64_t n,
+                    float* __restrict__ out, int out_stride, int nout, int32_t* __restrict__ err) {
+  using I = Img<D, H>;
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  // align the dynamic shared window to 1024 B for the swizzle atoms
+  uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
+  MlpBf16Smem<D, H>& s = *reinterpret_cast<MlpBf16Smem<D, H>*>(base);
+  const int tid = threadIdx.x, warp = tid >> 5;
+  const MlpLayout Lp = mlp_layout(D, H, A);
+  if (tid == 0) {
+    s.err = 0;
+    tc::mbar_init(&s.bar_w, 1);
+    tc::mbar_init(&s.bar_mma, 1);
+    tc::fence_mbar_init();
+  }
+  if (warp == 0) tc::tmem_alloc(&s.tmem_base, 512);
+  for (int i = tid; i < H; i += blockDim.x) {
+    s.b1[i] = __ldg(params + (value_net ? Lp.c1 : Lp.b1) + i);
+    s.b2[i] = __ldg(params + (value_net ? Lp.c2 : Lp.b2) + i);
+  }
+  if (tid < kHeadN) s.b3[tid] = tid < nout ? __ldg(params + (value_net ? Lp.c3 : Lp.b3) + tid) : 0.0f;
+  tc::fence_before();
+  __syncthreads();
+  tc::fence_after();
+  const uint32_t tmem = s.tmem_base;
+  if (tid == 0) {
+    tc::mbar_expect_tx(&s.bar_w, (uint32_t)I::TOTAL);
+    tc::bulk_g2s(s.w, img, (uint32_t)I::TOTAL, &s.bar_w);
+  }
+  if (!tc::mbar_wait(&s.bar_w, 0)) atomicExch(&s.err, 1);
+  __syncthreads();
+
+  const uint32_t w1 = tc::smem_u32(s.w), w2 = w1 + I::W1, w3 = w2 + I::W2;
+  const uint32_t xa = tc::smem_u32(s.act);
+  constexpr uint32_t kId1 = tc::idesc_bf16(kTcRows, H);
+  constexpr uint32_t kIdH = tc::idesc_bf16(kTcRows, kHeadN);
+  uint32_t phase = 0;
+  const int64_t tiles = (n + kTcRows - 1) / kTcRows;
+  for (int64_t tile = blockIdx.x; tile < tiles && s.err == 0; tile += gridDim.x) {
+    const int64_t r0 = tile * kTcRows;
+    const int nr = (int)(n - r0 < kTcRows ? n - r0 : kTcRows);
+    // observation tile -> X (D bf16 per row, swizzled like W1)
+    constexpr int CPR = D / 8;  // 16-byte chunks per row
+    for (int i = tid; i < kTcRows * CPR; i += blockDim.x) {
+      const int r = i / CPR, c = i % CPR;
+      uint4 v = make_uint4(0, 0, 0, 0);
+      if (r < nr) v = __ldg(reinterpret_cast<const uint4*>(obs + (r0 + r) * D) + c);
+      *reinterpret_cast<uint4*>(s.act + tc::swz_offset<I::RB1>(r, c * 8, kTcRows)) = v;
+    }
+    tc::fence_async_smem();
+    __syncthreads();
+    // layer 1: D1[128 x H] (TMEM cols 0..H) = X W1^T
+    if (tid == 0) {
+      tc::fence_after();
+#pragma unroll
+      for (int kk = 0; kk < D / 16; ++kk)
+        tc::mma_bf16(tmem, tc::desc_kmajor(xa + kk * 32, 8 * I::RB1, I::RB1 == 64 ? tc::kLayoutSW64 : tc::kLayoutSW128),
+                     tc::desc_kmajor(w1 + kk * 32, 8 * I::RB1, I::RB1 == 64 ? tc::kLayoutSW64 : tc::kLayoutSW128),
+                     kId1, kk > 0);
+      tc::mma_commit(&s.bar_mma);
+    }
+    if (!tc::mbar_wait(&s.bar_mma, phase)) atomicExch(&s.err, 1);
+    phase ^= 1;
+    tc::fence_after();
+    epilogue_tanh<H>(tmem, 0, s.b1, s.act);
+    tc::fence_before();
+    tc::fence_async_smem();
+    __syncthreads();
+    // layer 2: D2 (TMEM cols 256..256+H) = H1 W2^T
+    if (tid == 0) {
+      tc::fence_after();
+#pragma unroll 1
+      for (int kb = 0; kb < H / 64; ++kb)
+#pragma unroll
+        for (int kk = 0; kk < 4; ++kk)
+          tc::mma_bf16(tmem + 256, tc::desc_kmajor(xa + kb * kTcRows * 128 + kk * 32, 1024, tc::kLayoutSW128),
+                       tc::desc_kmajor(w2 + kb * H * 128 + kk * 32, 1024, tc::kLayoutSW128), kId1,
+                       (kb | kk) != 0);
+      tc::mma_commit(&s.bar_mma);
+    }
+    if (!tc::mbar_wait(&s.bar_mma, phase)) atomicExch(&s.err, 1);
+    phase ^= 1;
+    tc::fence_after();
+    epilogue_tanh<H>(tmem, 256, s.b2, s.act);
+    tc::fence_before();
+    tc::fence_async_smem();
+    __syncthreads();
+    // head: D3 (TMEM cols 0..16) = H2 W3^T
+    if (tid == 0) {
+      tc::fence_after();
+#pragma unroll 1
+      for (int kb = 0; kb < H / 64; ++kb)
+#pragma unroll
+        for (int kk = 0; kk < 4; ++kk)
+          tc::mma_bf16(tmem, tc::desc_kmajor(xa + kb * kTcRows * 128 + kk * 32, 1024, tc::kLayoutSW128),
+                       tc::desc_kmajor(w3 + kb * kHeadN * 128 + kk * 32, 1024, tc::kLayoutSW128), kIdH,
+                       (kb | kk) != 0);
+      tc::mma_commit(&s.bar_mma);
+    }
+    if (!tc::mbar_wait(&s.bar_mma, phase)) atomicExch(&s.err, 1);
+    phase ^= 1;
+    tc::fence_after();
+    if (warp < 4) {
+      const int row = warp * 32 + (tid & 31);
+      float v[16];
+      tc::tmem_ld16(tmem + ((uint32_t)(warp * 32) << 16), v);
+      if (row < nr) {
+        float* o = out + (r0 + row) * out_stride;
+#pragma unroll
+        for (int j = 0; j < kHeadN; ++j)
+          if (j < nout) o[j] = v[j] + s.b3[j];
+      }
+    }
+    tc::fence_before();
+    __syncthreads();
+  }
+  if (tid == 0 && s.err) {
+    atomicExch(&g_tc_error, 1);
+    if (err) atomicExch(err, 1);
+  }
+  __syncthreads();
+  if (warp == 0) tc::tmem_dealloc(tmem, 512);
+}
+
+// ---------------------------------------------------------------------------
+// decoupled bf16 rollout: per step, an env kernel (one thread per env: act on
+// the previous step's logits, then observe) and the tensor-core policy kernel
+// ---------------------------------------------------------------------------
+struct ActArgs {
+  const float* logits;  // [E][16]
+  int t;                // step whose action is taken (-1: observe only)
+  uint32_t it;
+  float lambda;
+  int det;
+  int T;                // horizon (t + 1 == T: write obs_last)
+};
+
+template <int C, int OBS, int D, int A>
+__global__ void __launch_bounds__(128) env_actobs_kernel(EnvDev env, ActArgs a, pe_rollout_buf buf) {
+  const int e = blockIdx.x * blockDim.x + threadIdx.x;
+  if (e >= env.E) return;
+  RegAcc<C> acc = load_reg<C>(env, e);
+  if (a.t >= 0) {
+    float z[A];
+    const float4* lz = reinterpret_cast<const float4*>(a.logits + (int64_t)e * kHeadN);
+#pragma unroll
+    for (int j = 0; j < A / 4; ++j) {
+      const float4 q = lz[j];
+      z[4 * j] = q.x;
+      z[4 * j + 1] = q.y;
+      z[4 * j + 2] = q.z;
+      z[4 * j + 3] = q.w;
+    }
+    const uint32_t r = a.det ? 0u : draw32(env.seed, (uint32_t)e, (uint32_t)a.t, a.it, kDrawAction);
+    float lp;
+    const int act = sample_action<A>(z, r, a.det != 0, &lp);
+    const StepOut so = env_step<C>(env, acc, act, a.lambda);
+    const int64_t row = (int64_t)a.t * env.E + e;
+    buf.act[row] = (uint8_t)act;
+    buf.logp[row] = lp;
+    buf.reward[row] = so.reward;
+    buf.done[row] = (uint8_t)so.done;
+    if (a.t == 0) {
+      buf.viol[2 * e] = so.v1;
+      buf.viol[2 * e + 1] = so.v60;
+      buf.tokens[e] = so.tokens;
+      buf.excess[e] = so.excess;
+      buf.energy_q[e] = so.q;
+    } else {
+      buf.viol[2 * e] += so.v1;
+      buf.viol[2 * e + 1] += so.v60;
+      buf.tokens[e] += so.tokens;
+      buf.excess[e] += so.excess;
+      buf.energy_q[e] += so.q;
+    }
+    if (so.done) env_reset<C>(env, acc, (uint32_t)e, (uint32_t)a.t, a.it, kDrawReset);
+  }
+  // observation for step t + 1 (or the final one)
+  __nv_bfloat16* dst = (a.t + 1 < a.T)
+                           ? reinterpret_cast<__nv_bfloat16*>(buf.obs) + ((int64_t)(a.t + 1) * env.E + e) * D
+                           : reinterpret_cast<__nv_bfloat16*>(buf.obs_last) + (int64_t)e * D;
+#pragma unroll 1
+  for (int f0 = 0; f0 < D; f0 += 8) {
+    uint32_t p[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i)
+      p[i] = tc::pack_bf16(feature<C, OBS>(env, acc, f0 + 2 * i), feature<C, OBS>(env, acc, f0 + 2 * i + 1));
+    *reinterpret_cast<uint4*>(dst + f0) = make_uint4(p[0], p[1], p[2], p[3]);
+  }
+  store_reg<C>(env, e, acc);
+}
+
+// workspace: weight image (policy), weight image (value), logits [E][16], error word
+template <int D, int H>
+static int64_t bf16_ws_bytes(int64_t E) {
+  const int64_t img = (Img<D, H>::TOTAL + 1023) / 1024 * 1024;
+  return 2 * img + (E * kHeadN * 4 + 255) / 256 * 256 + 256;
+}
+
+template <int D, int H>
+static pe_status launch_mlp(const uint8_t* img, const float* params, int A, int value_net,
+                            const void* obs, int64_t n, float* out, int out_stride, int nout,
+                            int32_t* err, cudaStream_t st, int prof_kind) {
+  if (n <= 0) return PE_OK;
+  auto kern = mlp_bf16_kernel<D, H>;
+  const int bytes = (int)sizeof(MlpBf16Smem<D, H>) + 1024;
+  PE_TRY_CUDA(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes));
+  int dev = 0, sms = 0;
+  PE_TRY_CUDA(cudaGetDevice(&dev));
+  PE_TRY_CUDA(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
+  const int64_t tiles = (n + kTcRows - 1) / kTcRows;
+  const int grid = (int)(tiles < sms ? tiles : sms);
+  {
+    ProfScope ps(prof_kind, st);
+    kern<<<grid, kTcThreads, bytes, st>>>(img, params, A, value_net,
+                                          reinterpret_cast<const __nv_bfloat16*>(obs), n, out,
+                                          out_stride, nout, err);
+  }
+  PE_CHECK_LAUNCH("mlp_bf16_kernel");
+  return PE_OK;
+}
+
+template <int D, int H>
+static pe_status make_images(const float* params, int A, uint8_t* ws, cudaStream_t st, bool policy) {
+  const int64_t img = (Img<D, H>::TOTAL + 1023) / 1024 * 1024;
+  ProfScope ps(PE_PROF_VALUE, st);
+  if (policy) weight_image_kernel<D, H><<<64, 256, 0, st>>>(params, A, 0, ws);
+  weight_image_kernel<D, H><<<64, 256, 0, st>>>(params, A, 1, ws + img);
+  PE_CHECK_LAUNCH("weight_image_kernel");
+  return PE_OK;
+}
+
+template <int C, int OBS, int D, int H, int A>
+static pe_status rollout_bf16_impl(const EnvDev& env, const float* params, int T, uint32_t it,
+                                   float lambda, int det, const pe_rollout_buf& buf, void* wsv,
+                                   cudaStream_t st) {
+  uint8_t* ws = reinterpret_cast<uint8_t*>(wsv);
+  const int64_t img = (Img<D, H>::TOTAL + 1023) / 1024 * 1024;
+  float* logits = reinterpret_cast<float*>(ws + 2 * img);
+  int32_t* err = reinterpret_cast<int32_t*>(ws + 2 * img + (env.E * (int64_t)kHeadN * 4 + 255) / 256 * 256);
+  PE_TRY_CUDA(cudaMemsetAsync(err, 0, 4, st));
+  pe_status s = make_images<D, H>(params, A, ws, st, true);
+  if (s != PE_OK) return s;
+  const int grid = ceil_div(env.E, 128);
+  ActArgs a{logits, -1, it, lambda, det, T};
+  {
+    ProfScope ps(PE_PROF_ROLLOUT, st);
+    env_actobs_kernel<C, OBS, D, A><<<grid, 128, 0, st>>>(env, a, buf);
+  }
+  PE_CHECK_LAUNCH("env_actobs_kernel");
+  for (int t = 0; t < T; ++t) {
+    const void* obs_t = reinterpret_cast<const __nv_bfloat16*>(buf.obs) + (int64_t)t * env.E * D;
+    s = launch_mlp<D, H>(ws, params, A, 0, obs_t, env.E, logits, kHeadN, A, err, st, PE_PROF_ROLLOUT);
+    if (s != PE_OK) return s;
+    a.t = t;
+    {
+      ProfScope ps(PE_PROF_ROLLOUT, st);
+      env_actobs_kernel<C, OBS, D, A><<<grid, 128, 0, st>>>(env, a, buf);
+    }
+    PE_CHECK_LAUNCH("env_actobs_kernel");
+  }
+  s = launch_mlp<D, H>(ws + img, params, A, 1, buf.obs, (int64_t)T * env.E, buf.value, 1, 1, err, st, PE_PROF_VALUE);
+  if (s != PE_OK) return s;
+  return launch_mlp<D, H>(ws + img, params, A, 1, buf.obs_last, env.E, buf.last_value, 1, 1, err, st, PE_PROF_VALUE);
+}
+
+int64_t rollout_bf16_ws_bytes(const pe_net& net, int64_t E) {
+  if (net.obs_dim == 32 && net.hidden == 256) return bf16_ws_bytes<32, 256>(E);
+  return -1;
+}
+
+pe_status rollout_bf16(const EnvDev& env, const pe_net& net, const float* params, int T, uint32_t it,
+                       float lambda, int det, const pe_rollout_buf& buf, void* ws, cudaStream_t st) {
+  if (net.obs_dim == 32 && net.hidden == 256 && net.n_actions == 16 && env.C == 4 && env.obs_kind == PE_OBS_OCC32)
+    return rollout_bf16_impl<4, PE_OBS_OCC32, 32, 256, 16>(env, params, T, it, lambda, det, buf, ws, st);
+  return fail(PE_EINVAL, "unsupported bf16 network/env combination (D=%d H=%d A=%d C=%d obs=%d)",
+              net.obs_dim, net.hidden, net.n_actions, env.C, env.obs_kind);
+}
+
+pe_status value_bf16(const pe_net& net, const float* params, const void* obs, int64_t n, float* value,
+                     void* wsv, cudaStream_t st) {
+  uint8_t* ws = reinterpret_cast<uint8_t*>(wsv);
+  auto run = [&](auto dtag, auto htag) -> pe_status {
+    constexpr int D = decltype(dtag)::value, H = decltype(htag)::value;
+    const int64_t img = (Img<D, H>::TOTAL + 1023) / 1024 * 1024;
+    int32_t* err = reinterpret_cast<int32_t*>(ws + 2 * img);
+    PE_TRY_CUDA(cudaMemsetAsync(err, 0, 4, st));
+    pe_status s = make_images<D, H>(params, net.n_actions, ws, st, false);
+    if (s != PE_OK) return s;
+    return launch_mlp<D, H>(ws + img, params, net.n_actions, 1, obs, n, value, 1, 1, err, st, PE_PROF_VALUE);
+  };
+  if (net.obs_dim == 32 && net.hidden == 256)
+    return run(std::integral_constant<int, 32>{}, std::integral_constant<int, 256>{});
+  return fail(PE_EINVAL, "unsupported bf16 value network (D=%d H=%d)", net.obs_dim, net.hidden);
+}
+
+pe_status device_check(cudaStream_t st) {
+  PE_TRY_CUDA(cudaStreamSynchronize(st));
+  int32_t flag = 0;
+  PE_TRY_CUDA(cudaMemcpyFromSymbol(&flag, g_tc_error, sizeof(flag)));
+  if (flag) {
+    const int32_t zero = 0;
+    PE_TRY_CUDA(cudaMemcpyToSymbol(g_tc_error, &zero, sizeof(zero)));
+    return fail(PE_ETIMEOUT, "a bounded tensor-core wait timed out in an earlier launch");
+  }
+  return PE_OK;
+}
+
+int64_t value_bf16_ws_bytes(const pe_net& net) {
+  if (net.obs_dim == 32 && net.hidden == 256) return bf16_ws_bytes<32, 256>(0);
+  return -1;
+}
+
+}  // namespace pe

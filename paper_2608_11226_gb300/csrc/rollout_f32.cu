@@ -52,7 +52,8 @@ __global__ void __launch_bounds__(TE / 4 * H / 4)
       const int e = idx / D, f = idx % D;
       float v = 0.0f;
       if (e < ne) {
-        v = feature<TE, C, OBS>(env, s.env, e, f);
+        TileAcc<TE, C> acc{s.env, e};
+        v = feature<C, OBS>(env, acc, f);
         dst[idx] = v;
       }
       s.xt[f * TE + e] = v;
@@ -73,7 +74,8 @@ __global__ void __launch_bounds__(TE / 4 * H / 4)
       const uint32_t r = det ? 0u : draw32(env.seed, eg, (uint32_t)t, it, kDrawAction);
       float lp;
       const int a = sample_action<A>(s.logits + e * A, r, det != 0, &lp);
-      const StepOut so = env_step<TE, C>(env, s.env, e, a, lambda);
+      TileAcc<TE, C> acc{s.env, e};
+      const StepOut so = env_step<C>(env, acc, a, lambda);
       const int64_t row = (int64_t)t * env.E + eg;
       buf.act[row] = (uint8_t)a;
       buf.logp[row] = lp;
@@ -84,7 +86,7 @@ __global__ void __launch_bounds__(TE / 4 * H / 4)
       energy += so.q;
       tok += so.tokens;
       exc += so.excess;
-      if (so.done) env_reset<TE, C>(env, s.env, e, eg, (uint32_t)t, it, kDrawReset);
+      if (so.done) env_reset<C>(env, acc, eg, (uint32_t)t, it, kDrawReset);
     }
     __syncthreads();
   }

@@ -65,7 +65,8 @@ class PPOConfig(C.Structure):
 
 EXPORTS = (
     "pe_env_create", "pe_env_destroy", "pe_env_state_bytes", "pe_env_save", "pe_env_load",
-    "pe_param_count", "pe_rollout", "pe_value", "pe_gae", "pe_ppo_workspace_bytes",
+    "pe_param_count", "pe_rollout_workspace_bytes", "pe_rollout", "pe_value_workspace_bytes",
+    "pe_value", "pe_device_check", "pe_gae", "pe_ppo_workspace_bytes",
     "pe_ppo_update", "pe_fleet_workspace_bytes", "pe_fleet_windows", "pe_fleet_windows_noalloc",
     "pe_profile_enable",
     "pe_profile_read", "pe_profile_kind_name", "pe_last_error")
@@ -86,8 +87,11 @@ def lib():
             "pe_env_save": (i32, [vp, vp]),
             "pe_env_load": (i32, [vp, vp]),
             "pe_param_count": (i64, [vp]),
-            "pe_rollout": (i32, [vp, vp, vp, i32, u32, C.c_float, i32, vp, vp]),
-            "pe_value": (i32, [vp, vp, vp, i64, vp, vp]),
+            "pe_rollout_workspace_bytes": (i64, [vp, vp]),
+            "pe_rollout": (i32, [vp, vp, vp, i32, u32, C.c_float, i32, vp, vp, i64, vp]),
+            "pe_value_workspace_bytes": (i64, [vp]),
+            "pe_value": (i32, [vp, vp, vp, i64, vp, vp, i64, vp]),
+            "pe_device_check": (i32, [vp]),
             "pe_gae": (i32, [vp, vp, vp, vp, i32, i32, C.c_float, C.c_float, vp, vp, vp]),
             "pe_ppo_workspace_bytes": (i64, [vp, vp, i64]),
             "pe_ppo_update": (i32, [vp, vp, vp, vp, i64, vp, vp, vp, vp, vp, i64, vp, vp, vp,
@@ -204,19 +208,43 @@ def _rollout_buf(b: Dict[str, torch.Tensor]) -> RolloutBuf:
         "tokens", "excess", "energy_q")])
 
 
+def rollout_workspace_bytes(env: Env, net: W.NetSpec) -> int:
+    return int(lib().pe_rollout_workspace_bytes(env._h, C.byref(net_desc(net))))
+
+
+def alloc_workspace(nbytes: int, device="cuda") -> Optional[torch.Tensor]:
+    return torch.empty(max(int(nbytes), 1), dtype=torch.uint8, device=device)
+
+
 def rollout(env: Env, net: W.NetSpec, params: torch.Tensor, T: int, iteration: int,
             buf: Dict[str, torch.Tensor], lam: float = 1.0, deterministic: bool = False,
-            stream=None):
+            workspace: Optional[torch.Tensor] = None, stream=None):
     rb = _rollout_buf(buf)
+    if workspace is None and net.dtype != PE_F32:
+        workspace = alloc_workspace(rollout_workspace_bytes(env, net))
+    nbytes = 0 if workspace is None else workspace.numel()
     _check(lib().pe_rollout(env._h, C.byref(net_desc(net)), _ptr(params), T, iteration, lam,
                             PE_ROLLOUT_DETERMINISTIC if deterministic else 0, C.byref(rb),
-                            _stream(stream)))
+                            _ptr(workspace), nbytes, _stream(stream)))
 
 
-def value(net: W.NetSpec, params: torch.Tensor, obs: torch.Tensor, out: torch.Tensor, stream=None):
+def value_workspace_bytes(net: W.NetSpec) -> int:
+    return int(lib().pe_value_workspace_bytes(C.byref(net_desc(net))))
+
+
+def value(net: W.NetSpec, params: torch.Tensor, obs: torch.Tensor, out: torch.Tensor,
+          workspace: Optional[torch.Tensor] = None, stream=None):
     n = obs.numel() // net.obs_dim
+    if workspace is None and net.dtype != PE_F32:
+        workspace = alloc_workspace(value_workspace_bytes(net))
+    nbytes = 0 if workspace is None else workspace.numel()
     _check(lib().pe_value(C.byref(net_desc(net)), _ptr(params), _ptr(obs), n, _ptr(out),
-                          _stream(stream)))
+                          _ptr(workspace), nbytes, _stream(stream)))
+
+
+def device_check(stream=None):
+    """Synchronise and raise PEError(PE_ETIMEOUT) if a bounded device wait gave up."""
+    _check(lib().pe_device_check(_stream(stream)))
 
 
 def gae(reward, value_, done, last_value, gamma: float, lam: float, adv, ret, stream=None):

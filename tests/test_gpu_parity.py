@@ -27,6 +27,20 @@ def rel_err(gpu, ref):
     return float(np.max(np.abs(gpu - ref) / np.maximum(np.abs(ref), floor)))
 
 
+def bf16_ok(gpu, ref, tol=2e-2, tail=1e-3):
+    """bf16-network outputs: normwise relative error <= tol, and at most a
+    `tail` fraction of elements beyond tol in the rms-floored relative error.
+    Rare 1-ulp bf16 rounding flips of hidden activations (fp32 accumulation on
+    the GPU, fp64 in the oracle) cascade into a few larger deviations."""
+    gpu = np.asarray(gpu, np.float64).ravel()
+    ref = np.asarray(ref, np.float64).ravel()
+    d = np.abs(gpu - ref)
+    norm = d.max() / max(np.abs(ref).max(), 1e-30)
+    floor = np.sqrt(np.mean(ref ** 2)) + 1e-30
+    frac = float(np.mean(d / np.maximum(np.abs(ref), floor) > tol))
+    return norm <= tol and frac <= tail
+
+
 @pytest.fixture(scope="module", autouse=True)
 def _built():
     from paper_2608_11226_gb300 import build
@@ -134,36 +148,45 @@ def test_fleet_rejects_bad_offsets_and_traces():
 # -------------------------------------------------------------------- rollout
 def _rollout_case(wl, T, iters, sample_envs=None, det=False, lam=1.0):
     spec, net = wl.env, wl.net
+    bf16 = net.dtype == pe.PE_BF16
     params = W.init_params(net, seed=1, bias_scale=0.05)
     env = pe.Env(spec, torch.from_numpy(wl.trace), torch.from_numpy(wl.phase))
     buf = pe.alloc_rollout(spec, net, T)
     p_dev = torch.from_numpy(params).cuda()
     ids = np.arange(spec.n_envs) if sample_envs is None else np.asarray(sample_envs)
+    ids_d = torch.from_numpy(ids).cuda()
     ora = O.OracleEnv(spec, wl.trace, wl.phase, ids)
+    ws = pe.alloc_workspace(pe.rollout_workspace_bytes(env, net)) if bf16 else None
     agree = total = 0
     for it in range(iters):
-        pe.rollout(env, net, p_dev, T, it, buf, lam=lam, deterministic=det)
-        torch.cuda.synchronize()
-        g = {k: cpu(v) for k, v in buf.items()}
-        forced = g["act"][:, ids]
-        o = ora.rollout(params, net.hidden, net.dtype == 1, T, it, lam=lam, deterministic=det,
-                        forced=forced)
-        gobs = g["obs"][:, ids].astype(np.float32)
-        assert np.array_equal(gobs, o["obs"]), "observations differ"
-        assert np.array_equal(g["obs_last"][ids], o["obs_last"])
-        assert np.array_equal(g["done"][:, ids], o["done"])
-        assert np.array_equal(g["viol"][ids], o["viol"])
-        assert np.array_equal(g["energy_q"][ids], o["energy_q"])
-        assert rel_err(g["reward"][:, ids], o["reward"]) <= TOL
-        assert rel_err(g["tokens"][ids], o["tokens"]) <= TOL
-        assert rel_err(g["excess"][ids], o["excess"]) <= TOL
-        assert rel_err(g["logp"][:, ids], o["logp"]) <= TOL
+        pe.rollout(env, net, p_dev, T, it, buf, lam=lam, deterministic=det, workspace=ws)
+        pe.device_check()
+        g = {}
+        for k, v in buf.items():
+            sel = v[:, ids_d] if v.dim() >= 2 and k in ("obs", "act", "logp", "value", "reward", "done") else v[ids_d]
+            g[k] = cpu(sel.float() if sel.dtype == torch.bfloat16 else sel)
+        forced = g["act"]
+        o = ora.rollout(params, net.hidden, bf16, T, it, lam=lam, deterministic=det, forced=forced)
+        want_obs, want_last = o["obs"], o["obs_last"]
+        if bf16:   # the buffer holds observations rounded to bf16 (RNE), as the oracle feeds its network
+            want_obs = torch.from_numpy(want_obs).to(torch.bfloat16).float().numpy()
+            want_last = torch.from_numpy(want_last).to(torch.bfloat16).float().numpy()
+        assert np.array_equal(g["obs"], want_obs), "observations differ"
+        assert np.array_equal(g["obs_last"], want_last)
+        assert np.array_equal(g["done"], o["done"])
+        assert np.array_equal(g["viol"], o["viol"])
+        assert np.array_equal(g["energy_q"], o["energy_q"])
+        assert rel_err(g["reward"], o["reward"]) <= TOL
+        assert rel_err(g["tokens"], o["tokens"]) <= TOL
+        assert rel_err(g["excess"], o["excess"]) <= TOL
+        close = (lambda a, b: bf16_ok(a, b)) if bf16 else (lambda a, b: rel_err(a, b) <= TOL)
+        assert close(g["logp"], o["logp"])
         agree += int((o["act_own"] == forced).sum())
         total += forced.size
         _, ov = O.mlp_forward(net, params, o["obs"].reshape(-1, net.obs_dim))
-        assert rel_err(g["value"][:, ids].ravel(), ov) <= TOL
+        assert close(g["value"].ravel(), ov)
         _, olv = O.mlp_forward(net, params, o["obs_last"])
-        assert rel_err(g["last_value"][ids], olv) <= TOL
+        assert close(g["last_value"], olv)
     assert agree / total >= 0.999, agree / total
     env.close()
     return agree / total
@@ -186,6 +209,33 @@ def test_rollout_parity_7b_sampled():
     rng = np.random.default_rng(3)
     ids = np.unique(np.concatenate([[0, 31, 32, 4095], rng.choice(4096, 28, replace=False)]))
     _rollout_case(wl, 512, iters=2, sample_envs=ids)
+
+
+def test_rollout_parity_72b_small():
+    """bf16 tensor-core policy/value (D=32, H=256, A=16), 4 channels, Eq. 6
+    reward; 512 envs x 600 steps crosses an episode boundary."""
+    _rollout_case(W.make_72b(n_envs=512), 600, iters=1, lam=0.7)
+
+
+def test_rollout_parity_72b_full_size_sampled():
+    """The full 72B workload (65,536 envs x 1,024 steps); the oracle replays
+    a seeded sample of envs including both ends and a tile boundary."""
+    wl = W.make_72b()
+    rng = np.random.default_rng(5)
+    ids = np.unique(np.concatenate([[0, 127, 128, 65535], rng.choice(65536, 12, replace=False)]))
+    _rollout_case(wl, 1024, iters=1, sample_envs=ids)
+
+
+def test_value_bf16_parity_ragged():
+    net = W.NetSpec(32, 256, 16, pe.PE_BF16)
+    params = W.init_params(net, seed=4, bias_scale=0.1)
+    for n in (1, 127, 129, 5000):
+        obs = torch.randn(n, 32, generator=torch.Generator().manual_seed(n)).to(torch.bfloat16)
+        out = torch.empty(n, device="cuda")
+        pe.value(net, torch.from_numpy(params).cuda(), obs.cuda(), out)
+        pe.device_check()
+        _, ov = O.mlp_forward(net, params, obs.float().numpy())
+        assert bf16_ok(cpu(out), ov)
 
 
 def test_env_checkpoint_roundtrip():
