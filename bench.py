@@ -50,6 +50,9 @@ def parse():
     ap.add_argument("--fleet-steps", type=int, default=3)
     ap.add_argument("--cpu-envs", type=int, default=48, help="envs in the oracle CPU sample")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--r72b-steps", type=int, default=2, help="timed 72B rollouts (0: skip)")
+    ap.add_argument("--r72b-envs", type=int, default=65536)
+    ap.add_argument("--r72b-horizon", type=int, default=1024)
     return ap.parse_args()
 
 
@@ -228,12 +231,15 @@ def run_ours(args, world, rank, local):
     # ---- dominant kernel roofline (fp32 FFMA bound)
     gms, gn = prof["ppo_grad"]
     net = tr.wl.net
-    fl_launch = ppo_flops_per_sample(net.obs_dim, net.hidden, net.n_actions) * tr.wl.ppo.minibatch
+    # one launch is either the persistent update (all epochs x minibatches) or one minibatch
+    samples_per_launch = (tr.E * tr.T * tr.wl.ppo.epochs) if gn == args.steps else tr.wl.ppo.minibatch
+    kname = "ppo_persistent_kernel" if gn == args.steps else "ppo_grad_kernel"
+    fl_launch = ppo_flops_per_sample(net.obs_dim, net.hidden, net.n_actions) * samples_per_launch
     peak_tflops = N_SM * FP32_LANES_PER_SM * 2 * SM_MAX_MHZ * 1e6 / 1e12
     ach = fl_launch / (gms / gn / 1e3) / 1e12 if gn else None
-    roof = {"kernel": "ppo_grad_kernel", "bound": "alu", "achieved": ach, "peak": peak_tflops,
+    roof = {"kernel": kname, "bound": "alu", "achieved": ach, "peak": peak_tflops,
             "unit": "TFLOP/s", "frac": (ach / peak_tflops) if ach else None,
-            "traffic": load_traffic("ppo_grad_kernel"),
+            "traffic": load_traffic(kname),
             "peak_source": "derived: 152 SMs x 128 FP32 lanes x 2 FLOP x 2070 MHz",
             "avg_launch_ms": gms / gn if gn else None, "launches": gn,
             "flop_per_launch": fl_launch}
@@ -279,6 +285,7 @@ def run_ours(args, world, rank, local):
 
     # ---- fleet accounting
     fleet = run_fleet(args, world) if args.fleet_n > 0 else None
+    r72b = run_72b(args, world, peaks) if args.r72b_steps > 0 else None
 
     out = {"metric": METRIC, "value": value, "unit": "env-steps/s", "n_gpus": world,
            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_step,
@@ -290,7 +297,7 @@ def run_ours(args, world, rank, local):
                       "parallelism": f"replicas x{world}" if world > 1 else "1 GPU",
                       "l2": "flushed between timed steps (256 MB write)"},
            "roofline": roof, "gae_roofline": gae_roof, "kernels": kernels,
-           "gpu_launches": launches, "clocks": clk, "e2e": e2e, "fleet": fleet,
+           "gpu_launches": launches, "clocks": clk, "e2e": e2e, "fleet": fleet, "rollout_72b": r72b,
            "ppo_stats_last": [float(x) for x in tr.stats.cpu()]}
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         out["cpu_baseline"] = cpu_baseline(args.cpu_envs)
@@ -347,6 +354,82 @@ def run_fleet(args, world):
             "peak_fraction_of_nameplate_max": [float(p[:, i].max() / (64.0 * w) / W.FLEET_NAMEPLATE_W)
                                                for i, w in enumerate(windows)],
             "traffic": load_traffic("fleet_windows_kernel")}
+
+
+def run_72b(args, world, peaks):
+    """The 72B workload's rollout (65,536 envs x 1,024 steps, bf16 32-256-256
+    policy/value MLPs on the tcgen05 tensor cores, 4 channels, Eq. 6 reward),
+    timed the same way; reports env-steps/s and the tensor-core MLP kernel's
+    achieved bf16 TFLOP/s against the measured sustained bf16 peak."""
+    from paper_2608_11226_gb300 import pe
+    from paper_2608_11226_gb300 import workloads as W
+    wl = W.make_72b(n_envs=args.r72b_envs, seed=0)
+    spec, net = wl.env, wl.net
+    env = pe.Env(spec, torch.from_numpy(wl.trace), torch.from_numpy(wl.phase))
+    T, E = args.r72b_horizon, spec.n_envs
+    buf = pe.alloc_rollout(spec, net, T)
+    params = torch.from_numpy(W.init_params(net, seed=0)).cuda()
+    ws = pe.alloc_workspace(pe.rollout_workspace_bytes(env, net))
+    pe.rollout(env, net, params, T, 0, buf, lam=1.0, workspace=ws)
+    pe.device_check()
+    for k in range(pe.PE_PROF_KINDS):
+        pe.profile_read(k)
+    barrier(world)
+    pe.profile_enable(True)
+    stream = torch.cuda.current_stream()
+    a = torch.cuda.Event(enable_timing=True)
+    b = torch.cuda.Event(enable_timing=True)
+    a.record(stream)
+    for it in range(args.r72b_steps):
+        pe.rollout(env, net, params, T, it + 1, buf, lam=1.0, workspace=ws)
+    b.record(stream)
+    torch.cuda.synchronize()
+    pe.profile_enable(False)
+    pe.device_check()
+    ms = max_over_ranks(a.elapsed_time(b), world) / args.r72b_steps
+    prof = {pe.profile_kind_name(k): pe.profile_read(k) for k in range(pe.PE_PROF_KINDS)}
+    D, H, A = net.obs_dim, net.hidden, net.n_actions
+    pol_flop = 2.0 * E * (D * H + H * H + H * A)          # one policy launch (E rows)
+    val_flop = 2.0 * (T + 1) * E * (D * H + H * H + H)   # the value launches of one rollout
+    # GAE over the 72B rollout buffer (T*E = 67M env-steps, 1.14 GB of algorithmic traffic)
+    adv = torch.empty(T, E, device="cuda")
+    ret = torch.empty_like(adv)
+    pe.gae(buf["reward"], buf["value"], buf["done"], buf["last_value"], 0.99, 0.95, adv, ret)
+    torch.cuda.synchronize()
+    pe.profile_read(pe.PE_PROF_GAE)
+    pe.profile_enable(True)
+    for _ in range(3):
+        pe.gae(buf["reward"], buf["value"], buf["done"], buf["last_value"], 0.99, 0.95, adv, ret)
+    torch.cuda.synchronize()
+    pe.profile_enable(False)
+    gms, gn = pe.profile_read(pe.PE_PROF_GAE)
+    gae_gbs = 17.0 * T * E / (gms / gn / 1e3) / 1e9 if gn else None
+    hbm = float(peaks.get("hbm_gbs", 6800.0))
+    del adv, ret
+    pms, pn = prof["mlp_policy_tc"]
+    vms, vn = prof["mlp_value_tc"]
+    peak = float(peaks.get("bf16_tflops_sustained", 1728.9))
+    pol = pol_flop / (pms / pn / 1e3) / 1e12 if pn else None
+    val = val_flop * args.r72b_steps / (vms / 1e3) / 1e12 if vn else None
+    env.close()
+    return {"metric": "72B rollout env-steps/s", "value": E * T * world / (ms / 1e3),
+            "unit": "env-steps/s", "ms_per_rollout": ms,
+            "config": {"workload": f"72b: {E} envs x {T} steps, 4-channel 22,000-sample trace, "
+                                   "16 levels, MLP 32-256-256 bf16 (tcgen05), value on all T*E obs",
+                       "n_envs": E, "horizon": T},
+            "kernels": {k: {"ms_per_rollout": v[0] / args.r72b_steps,
+                            "launches_per_rollout": v[1] / args.r72b_steps} for k, v in prof.items() if v[1]},
+            "roofline_policy_mlp": {"kernel": f"mlp_bf16_kernel (policy, {E} rows)", "bound": "tensor",
+                                    "achieved": pol, "peak": peak, "unit": "TFLOP/s",
+                                    "frac": pol / peak if pol else None,
+                                    "traffic": load_traffic("mlp_bf16_kernel")},
+            "roofline_value_mlp": {"kernel": "mlp_bf16_kernel (value, T*E rows)", "bound": "tensor",
+                                   "achieved": val, "peak": peak, "unit": "TFLOP/s",
+                                   "frac": val / peak if val else None},
+            "roofline_gae": {"kernel": f"gae_kernel ({T} x {E})", "bound": "hbm", "achieved": gae_gbs,
+                             "peak": hbm, "unit": "GB/s", "frac": gae_gbs / hbm if gae_gbs else None,
+                             "avg_launch_ms": gms / gn if gn else None,
+                             "traffic": load_traffic("gae_kernel")}}
 
 
 # --------------------------------------------------------------------------- CPU oracle

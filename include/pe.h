@@ -268,7 +268,9 @@ pe_status pe_fleet_windows_noalloc(const float* traces, int32_t G, int32_t L,
 #define PE_PROF_PPO_OTHER 6
 #define PE_PROF_FLEET_PREP 7
 #define PE_PROF_FLEET_WINDOWS 8
-#define PE_PROF_KINDS 9
+#define PE_PROF_MLP_POLICY 9  /* tensor-core policy network launches (bf16 rollout) */
+#define PE_PROF_MLP_VALUE 10  /* tensor-core value network launches */
+#define PE_PROF_KINDS 11
 pe_status pe_profile_enable(int32_t on);
 pe_status pe_profile_read(int32_t kind, double* total_ms, int64_t* launches);
 const char* pe_profile_kind_name(int32_t kind);

@@ -144,7 +144,7 @@ const char* pe_last_error(void) { return g_err; }
 
 static const char* kProfNames[PE_PROF_KINDS] = {
     "rollout", "value", "gae", "ppo_grad", "ppo_reduce", "ppo_adam", "ppo_other",
-    "fleet_prepare", "fleet_windows"};
+    "fleet_prepare", "fleet_windows", "mlp_policy_tc", "mlp_value_tc"};
 
 const char* pe_profile_kind_name(int32_t kind) {
   return (kind >= 0 && kind < PE_PROF_KINDS) ? kProfNames[kind] : "";

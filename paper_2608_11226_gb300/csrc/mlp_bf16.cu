@@ -363,7 +363,7 @@ static pe_status rollout_bf16_impl(const EnvDev& env, const float* params, int T
   PE_CHECK_LAUNCH("env_actobs_kernel");
   for (int t = 0; t < T; ++t) {
     const void* obs_t = reinterpret_cast<const __nv_bfloat16*>(buf.obs) + (int64_t)t * env.E * D;
-    s = launch_mlp<D, H>(ws, params, A, 0, obs_t, env.E, logits, kHeadN, A, err, st, PE_PROF_ROLLOUT);
+    s = launch_mlp<D, H>(ws, params, A, 0, obs_t, env.E, logits, kHeadN, A, err, st, PE_PROF_MLP_POLICY);
     if (s != PE_OK) return s;
     a.t = t;
     {
@@ -372,9 +372,9 @@ static pe_status rollout_bf16_impl(const EnvDev& env, const float* params, int T
     }
     PE_CHECK_LAUNCH("env_actobs_kernel");
   }
-  s = launch_mlp<D, H>(ws + img, params, A, 1, buf.obs, (int64_t)T * env.E, buf.value, 1, 1, err, st, PE_PROF_VALUE);
+  s = launch_mlp<D, H>(ws + img, params, A, 1, buf.obs, (int64_t)T * env.E, buf.value, 1, 1, err, st, PE_PROF_MLP_VALUE);
   if (s != PE_OK) return s;
-  return launch_mlp<D, H>(ws + img, params, A, 1, buf.obs_last, env.E, buf.last_value, 1, 1, err, st, PE_PROF_VALUE);
+  return launch_mlp<D, H>(ws + img, params, A, 1, buf.obs_last, env.E, buf.last_value, 1, 1, err, st, PE_PROF_MLP_VALUE);
 }
 
 int64_t rollout_bf16_ws_bytes(const pe_net& net, int64_t E) {
@@ -400,7 +400,7 @@ pe_status value_bf16(const pe_net& net, const float* params, const void* obs, in
     PE_TRY_CUDA(cudaMemsetAsync(err, 0, 4, st));
     pe_status s = make_images<D, H>(params, net.n_actions, ws, st, false);
     if (s != PE_OK) return s;
-    return launch_mlp<D, H>(ws + img, params, net.n_actions, 1, obs, n, value, 1, 1, err, st, PE_PROF_VALUE);
+    return launch_mlp<D, H>(ws + img, params, net.n_actions, 1, obs, n, value, 1, 1, err, st, PE_PROF_MLP_VALUE);
   };
   if (net.obs_dim == 32 && net.hidden == 256)
     return run(std::integral_constant<int, 32>{}, std::integral_constant<int, 256>{});

@@ -44,40 +44,59 @@ __device__ __forceinline__ void load_copy(const float* __restrict__ src, float* 
   for (int i = threadIdx.x; i < n; i += blockDim.x) dst[i] = __ldg(src + i);
 }
 
+// RT consecutive floats (RT = 2 or 4) from shared memory
+template <int RT>
+__device__ __forceinline__ void load_rt(const float* p, float (&v)[RT]) {
+  if constexpr (RT == 4) {
+    const float4 q = *reinterpret_cast<const float4*>(p);
+    v[0] = q.x; v[1] = q.y; v[2] = q.z; v[3] = q.w;
+  } else {
+    const float2 q = *reinterpret_cast<const float2*>(p);
+    v[0] = q.x; v[1] = q.y;
+  }
+}
+
+template <int RT>
+__device__ __forceinline__ void store_rt(float* p, const float (&v)[RT]) {
+  if constexpr (RT == 4) {
+    *reinterpret_cast<float4*>(p) = make_float4(v[0], v[1], v[2], v[3]);
+  } else {
+    *reinterpret_cast<float2*>(p) = make_float2(v[0], v[1]);
+  }
+}
+
 // outT[n][e] = tanh(b[n] + sum_k inT[k][e] * WT[k][n]) for TE rows; each
-// thread owns a 4-row x 4-neuron register tile.  LD is the row stride (in
+// thread owns an RT-row x 4-neuron register tile.  LD is the row stride (in
 // floats) of inT and outT.
-template <int TE, int K, int N, int LD = TE>
+template <int TE, int K, int N, int LD = TE, int RT = 4>
 __device__ __forceinline__ void dense_tanh_t(const float* __restrict__ inT, const float* __restrict__ WT,
                                              const float* __restrict__ bias, float* __restrict__ outT) {
-  constexpr int EG = TE / 4, NG = N / 4;
+  constexpr int EG = TE / RT, NG = N / 4;
   for (int j = threadIdx.x; j < EG * NG; j += blockDim.x) {
     const int eg = j % EG, ng = j / EG;
-    float acc[4][4];
+    float acc[RT][4];
 #pragma unroll
-    for (int r = 0; r < 4; ++r)
+    for (int r = 0; r < RT; ++r)
 #pragma unroll
       for (int c = 0; c < 4; ++c) acc[r][c] = 0.0f;
 #pragma unroll 8
     for (int k = 0; k < K; ++k) {
-      const float4 x = *reinterpret_cast<const float4*>(inT + k * LD + eg * 4);
+      float xv[RT];
+      load_rt<RT>(inT + k * LD + eg * RT, xv);
       const float4 w = *reinterpret_cast<const float4*>(WT + k * N + ng * 4);
-      const float xv[4] = {x.x, x.y, x.z, x.w};
       const float wv[4] = {w.x, w.y, w.z, w.w};
 #pragma unroll
-      for (int r = 0; r < 4; ++r)
+      for (int r = 0; r < RT; ++r)
 #pragma unroll
         for (int c = 0; c < 4; ++c) acc[r][c] = fmaf(xv[r], wv[c], acc[r][c]);
     }
 #pragma unroll
     for (int c = 0; c < 4; ++c) {
       const float bb = bias[ng * 4 + c];
-      float4 o;
-      o.x = tanhf(acc[0][c] + bb);
-      o.y = tanhf(acc[1][c] + bb);
-      o.z = tanhf(acc[2][c] + bb);
-      o.w = tanhf(acc[3][c] + bb);
-      *reinterpret_cast<float4*>(outT + (ng * 4 + c) * LD + eg * 4) = o;
+      float o[RT];
+#pragma unroll
+      for (int r = 0; r < RT; ++r) o[r] = tanhf(acc[r][c] + bb);
+      store_rt<RT>(outT + (ng * 4 + c) * LD + eg * RT, o);
     }
   }
 }

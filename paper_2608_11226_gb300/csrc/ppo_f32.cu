@@ -18,6 +18,7 @@
 // permutation) are computed for all minibatches up front.
 #include <algorithm>
 #include <cmath>
+#include <vector>
 
 #include "mlp_f32.cuh"
 
@@ -25,7 +26,8 @@ namespace pe {
 
 constexpr int kPpoS = 32;           // samples per slice
 constexpr int kPpoLD = kPpoS + 4;   // row stride of feature-major activations
-constexpr int kPpoNT = 256;         // threads per gradient CTA
+constexpr int kPpoNT = 512;         // threads per gradient CTA
+constexpr int kPpoRT = 2;           // sample rows per thread tile in the dense layers
 constexpr int kPpoMaxEpochs = 16;
 
 struct FeistelSet {
@@ -73,45 +75,56 @@ __global__ void ppo_advstats_kernel(const float* __restrict__ adv, int64_t N, in
 }
 
 // outT[n][e] = (sum_k inT[k][e] W[k][n]) * (1 - hT[n][e]^2): back through a tanh layer
-template <int TE, int K, int N, int LD>
+template <int TE, int K, int N, int LD, int RT>
 __device__ __forceinline__ void dense_bwd_t(const float* __restrict__ inT, const float* __restrict__ W,
                                             const float* __restrict__ hT, float* __restrict__ outT) {
-  constexpr int EG = TE / 4, NG = N / 4;
+  constexpr int EG = TE / RT, NG = N / 4;
   for (int j = threadIdx.x; j < EG * NG; j += blockDim.x) {
     const int eg = j % EG, ng = j / EG;
-    float acc[4][4] = {};
+    float acc[RT][4];
+#pragma unroll
+    for (int r = 0; r < RT; ++r)
+#pragma unroll
+      for (int c = 0; c < 4; ++c) acc[r][c] = 0.0f;
 #pragma unroll 8
     for (int k = 0; k < K; ++k) {
-      const float4 x = *reinterpret_cast<const float4*>(inT + k * LD + eg * 4);
+      float xv[RT];
+      load_rt<RT>(inT + k * LD + eg * RT, xv);
       const float4 w = *reinterpret_cast<const float4*>(W + k * N + ng * 4);
-      const float xv[4] = {x.x, x.y, x.z, x.w};
       const float wv[4] = {w.x, w.y, w.z, w.w};
 #pragma unroll
-      for (int r = 0; r < 4; ++r)
+      for (int r = 0; r < RT; ++r)
 #pragma unroll
         for (int c = 0; c < 4; ++c) acc[r][c] = fmaf(xv[r], wv[c], acc[r][c]);
     }
 #pragma unroll
     for (int c = 0; c < 4; ++c) {
-      float* o = outT + (ng * 4 + c) * LD + eg * 4;
-      const float4 h = *reinterpret_cast<const float4*>(hT + (ng * 4 + c) * LD + eg * 4);
-      float4 r;
-      r.x = acc[0][c] * (1.0f - h.x * h.x);
-      r.y = acc[1][c] * (1.0f - h.y * h.y);
-      r.z = acc[2][c] * (1.0f - h.z * h.z);
-      r.w = acc[3][c] * (1.0f - h.w * h.w);
-      *reinterpret_cast<float4*>(o) = r;
+      float h[RT], o[RT];
+      load_rt<RT>(hT + (ng * 4 + c) * LD + eg * RT, h);
+#pragma unroll
+      for (int r = 0; r < RT; ++r) o[r] = acc[r][c] * (1.0f - h[r] * h[r]);
+      store_rt<RT>(outT + (ng * 4 + c) * LD + eg * RT, o);
     }
   }
 }
 
-// acc[m][n] += sum_s aT[m][s] bT[n][s] with per-thread 4x4 tiles whose rows
-// and columns are interleaved (m = mg + i*M/4, n = ng + j*N/4) so that the
-// float4 loads of one quarter-warp hit distinct shared-memory banks
+// acc[m][n] += sum_s aT[m][s] bT[n][s].  Each thread owns 4x4 tiles whose rows
+// and columns are interleaved (m = mg + i*M/4, n = ng + j*N/4); a warp covers
+// WM x WN (mg, ng) pairs, so one float4 load of the warp touches WM (or WN)
+// distinct rows in distinct shared-memory bank groups: one wavefront each.
 template <int M, int N, int NT>
 struct WGradAcc {
-  static constexpr int MG = M / 4, NG = N / 4, JOBS = MG * NG, PER = (JOBS + NT - 1) / NT;
+  static constexpr int MG = M / 4, NG = N / 4;
+  static constexpr int WN = NG < 4 ? NG : 4, WM = 32 / WN;
+  static constexpr int TM = (MG + WM - 1) / WM, TN = NG / WN;
+  static constexpr int NWARP = NT / 32, WT = TM * TN, PER = (WT + NWARP - 1) / NWARP;
   float acc[PER][4][4];
+  __device__ __forceinline__ bool job(int q, int& mg, int& ng) const {
+    const int wt = (int)(threadIdx.x >> 5) + q * NWARP, lane = threadIdx.x & 31;
+    mg = (wt / TN) * WM + lane / WN;
+    ng = (wt % TN) * WN + lane % WN;
+    return wt < WT && mg < MG;
+  }
   __device__ __forceinline__ void zero() {
 #pragma unroll
     for (int q = 0; q < PER; ++q)
@@ -124,9 +137,8 @@ struct WGradAcc {
   __device__ __forceinline__ void add(const float* __restrict__ aT, const float* __restrict__ bT) {
 #pragma unroll
     for (int q = 0; q < PER; ++q) {
-      const int jb = threadIdx.x + q * NT;
-      if (jb < JOBS) {
-        const int mg = jb / NG, ng = jb % NG;
+      int mg, ng;
+      if (job(q, mg, ng)) {
 #pragma unroll 2
         for (int s = 0; s < S; s += 4) {
           float4 a[4], b[4];
@@ -152,9 +164,8 @@ struct WGradAcc {
   __device__ __forceinline__ void store(float* __restrict__ dst) const {
 #pragma unroll
     for (int q = 0; q < PER; ++q) {
-      const int jb = threadIdx.x + q * NT;
-      if (jb < JOBS) {
-        const int mg = jb / NG, ng = jb % NG;
+      int mg, ng;
+      if (job(q, mg, ng)) {
 #pragma unroll
         for (int i = 0; i < 4; ++i)
 #pragma unroll
@@ -188,6 +199,7 @@ struct PpoArgs {
   float clip, vf_coef, ent_coef, inv_cnt;
   float* partial;       // [NC][P]
   float* stat_partial;  // [2*NC][8]
+  float* grad_out;      // [P] reduced gradient (persistent kernel)
   int NC, slices_per_cta;
   int64_t P;
 };
@@ -199,13 +211,19 @@ __device__ __forceinline__ void ppo_role(PpoSmem<D, H, A>& s, const PpoArgs& g, 
   const int64_t oW1 = POL ? Lp.w1 : Lp.v1, oB1 = POL ? Lp.b1 : Lp.c1;
   const int64_t oW2 = POL ? Lp.w2 : Lp.v2, oB2 = POL ? Lp.b2 : Lp.c2;
   const int64_t oW3 = POL ? Lp.w3 : Lp.v3, oB3 = POL ? Lp.b3 : Lp.c3;
-  load_transposed(g.params + oW1, s.w1t, H, D);
-  load_transposed(g.params + oW2, s.w2t, H, H);
-  load_copy(g.params + oW2, s.w2, H * H);
-  load_copy(g.params + oB1, s.b1, H);
-  load_copy(g.params + oB2, s.b2, H);
-  load_copy(g.params + oW3, s.w3, NA * H);
-  load_copy(g.params + oB3, s.b3, NA);
+  // parameters are read through L2 (not the non-coherent L1 path): inside the
+  // persistent update other CTAs rewrite them between minibatches
+  for (int i = threadIdx.x; i < H * D; i += blockDim.x) s.w1t[i] = __ldcg(g.params + oW1 + (int64_t)(i % H) * D + i / H);
+  for (int i = threadIdx.x; i < H * H; i += blockDim.x) {
+    s.w2t[i] = __ldcg(g.params + oW2 + (int64_t)(i % H) * H + i / H);
+    s.w2[i] = __ldcg(g.params + oW2 + i);
+  }
+  for (int i = threadIdx.x; i < H; i += blockDim.x) {
+    s.b1[i] = __ldcg(g.params + oB1 + i);
+    s.b2[i] = __ldcg(g.params + oB2 + i);
+  }
+  for (int i = threadIdx.x; i < NA * H; i += blockDim.x) s.w3[i] = __ldcg(g.params + oW3 + i);
+  for (int i = threadIdx.x; i < NA; i += blockDim.x) s.b3[i] = __ldcg(g.params + oB3 + i);
   const int tid = threadIdx.x;
   const float2 as = *g.advstat;
 
@@ -249,9 +267,9 @@ __device__ __forceinline__ void ppo_role(PpoSmem<D, H, A>& s, const PpoArgs& g, 
     }
     __syncthreads();
     // forward
-    dense_tanh_t<kPpoS, D, H, kPpoLD>(s.xt, s.w1t, s.b1, s.h1t);
+    dense_tanh_t<kPpoS, D, H, kPpoLD, kPpoRT>(s.xt, s.w1t, s.b1, s.h1t);
     __syncthreads();
-    dense_tanh_t<kPpoS, H, H, kPpoLD>(s.h1t, s.w2t, s.b2, s.h2t);
+    dense_tanh_t<kPpoS, H, H, kPpoLD, kPpoRT>(s.h1t, s.w2t, s.b2, s.h2t);
     __syncthreads();
     head_t<kPpoS, H, NA, kPpoLD>(s.h2t, s.w3, s.b3, s.z);
     __syncthreads();
@@ -330,7 +348,7 @@ __device__ __forceinline__ void ppo_role(PpoSmem<D, H, A>& s, const PpoArgs& g, 
       for (int si = 0; si < kPpoS; ++si) acc += s.d2t[tid * kPpoLD + si];
       gb2 += acc;
     }
-    dense_bwd_t<kPpoS, H, H, kPpoLD>(s.d2t, s.w2, s.h1t, s.h2t);
+    dense_bwd_t<kPpoS, H, H, kPpoLD, kPpoRT>(s.d2t, s.w2, s.h1t, s.h2t);
     __syncthreads();
     // layer-1 weight gradient
     g1.template add<kPpoS, kPpoLD>(s.h2t, s.xt);
@@ -377,6 +395,173 @@ __global__ void __launch_bounds__(kPpoNT) ppo_grad_kernel(PpoArgs g) {
     ppo_role<D, H, A, true>(s, g, blockIdx.x);
   else
     ppo_role<D, H, A, false>(s, g, blockIdx.x - g.NC);
+}
+
+// ---------------------------------------------------------------------------
+// Persistent form of the whole update: one cooperative launch runs every
+// minibatch step as three phases separated by grid barriers -- gradient
+// partials (as ppo_grad_kernel), a fixed-order reduction of each CTA's slice
+// of the parameter vector, and the clipped Adam step on that slice.  The
+// cooperative launch guarantees that all CTAs are resident, and every
+// barrier wait is bounded: on timeout the kernel records an error and stops.
+// ---------------------------------------------------------------------------
+struct PpoLoop {
+  PpoArgs g;              // per-minibatch fields are filled in by the kernel
+  const float2* advstat;  // [epochs][nmb]
+  FeistelSet perms;
+  int64_t N;
+  int minibatch, nmb, epochs;
+  float* params;
+  float* m;
+  float* v;
+  double* sq;              // [gridDim.x]
+  double* acc;             // [8] running statistics
+  unsigned int* bar;       // [2]: arrival count, generation
+  int32_t* err;
+  double* bc;              // [2 * steps]: step_size, 1/sqrt(bc2) per Adam step
+  float beta1, beta2, eps, max_norm;
+};
+
+__device__ __forceinline__ bool grid_barrier(unsigned int* bar, int* s_ok) {
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    volatile unsigned int* gen = bar + 1;
+    const unsigned int g0 = *gen;
+    __threadfence();
+    const unsigned int arrived = atomicAdd(bar, 1u) + 1u;
+    bool ok = true;
+    if (arrived == gridDim.x) {
+      atomicExch(bar, 0u);
+      __threadfence();
+      atomicAdd(bar + 1, 1u);
+    } else {
+      const long long t0 = clock64();
+      while (*gen == g0) {
+        if (clock64() - t0 > 4000000000LL) {  // about 2 s at the maximum SM clock
+          ok = false;
+          break;
+        }
+        __nanosleep(64);
+      }
+    }
+    __threadfence();
+    *s_ok = ok;
+  }
+  __syncthreads();
+  return *s_ok != 0;
+}
+
+template <int D, int H, int A>
+__global__ void __launch_bounds__(kPpoNT, 1) ppo_persistent_kernel(PpoLoop L) {
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  PpoSmem<D, H, A>& s = *reinterpret_cast<PpoSmem<D, H, A>*>(smem_raw);
+  __shared__ int s_ok;
+  __shared__ double s_part[4][128];
+  __shared__ double s_red[kPpoNT / 32];
+  __shared__ double s_norm;
+  const int NC = L.g.NC, tid = threadIdx.x;
+  const int64_t P = L.g.P;
+  const int64_t per = (P + gridDim.x - 1) / gridDim.x;
+  const int64_t p0 = (int64_t)blockIdx.x * per, p1 = p0 + per < P ? p0 + per : P;
+  const int pl = tid & 127, rg = tid >> 7;  // 4 row groups x 128 parameter lanes
+  int step = 0;
+  for (int ep = 0; ep < L.epochs; ++ep) {
+    for (int mb = 0; mb < L.nmb; ++mb, ++step) {
+      const int64_t start = (int64_t)mb * L.minibatch;
+      const int cnt = (int)(L.N - start < L.minibatch ? L.N - start : L.minibatch);
+      PpoArgs g = L.g;
+      g.perm = L.perms.f[ep];
+      g.start = start;
+      g.cnt = cnt;
+      g.inv_cnt = 1.0f / (float)cnt;
+      g.advstat = L.advstat + (int64_t)ep * L.nmb + mb;
+      // phase 1: gradient partials of this CTA's role and samples
+      if ((int)blockIdx.x < NC)
+        ppo_role<D, H, A, true>(s, g, blockIdx.x);
+      else
+        ppo_role<D, H, A, false>(s, g, blockIdx.x - NC);
+      if (!grid_barrier(L.bar, &s_ok)) {
+        if (tid == 0) atomicExch(L.err, 1);
+        return;
+      }
+      // phase 2: grad[p] = sum_c partial[c][p] in row order (4 row groups,
+      // combined in group order), and this CTA's sum of squares
+      double q = 0.0;
+      for (int64_t pb = p0; pb < p1; pb += 128) {
+        const int64_t p = pb + pl;
+        double gs = 0.0;
+        if (p < p1) {
+#pragma unroll 4
+          for (int c = rg; c < NC; c += 4) gs += (double)__ldcg(g.partial + (int64_t)c * P + p);
+        }
+        s_part[rg][pl] = gs;
+        __syncthreads();
+        if (rg == 0 && p < p1) {
+          const float gf = (float)(((s_part[0][pl] + s_part[1][pl]) + s_part[2][pl]) + s_part[3][pl]);
+          L.g.grad_out[p] = gf;
+          q += (double)gf * (double)gf;
+        }
+        __syncthreads();
+      }
+      const double qb = block_sum_d(q, s_red);
+      if (tid == 0) L.sq[blockIdx.x] = qb;
+      if (blockIdx.x == 0 && tid < 32) {
+        double v[5] = {0, 0, 0, 0, 0};
+        for (int c = tid; c < NC; c += 32) {
+          v[0] += __ldcg(g.stat_partial + c * 8 + 0);
+          v[1] += __ldcg(g.stat_partial + c * 8 + 1);
+          v[2] += __ldcg(g.stat_partial + c * 8 + 2);
+          v[3] += __ldcg(g.stat_partial + c * 8 + 3);
+          v[4] += __ldcg(g.stat_partial + (NC + c) * 8 + 4);
+        }
+#pragma unroll
+        for (int k = 0; k < 5; ++k)
+#pragma unroll
+          for (int o = 16; o > 0; o >>= 1) v[k] += __shfl_xor_sync(0xffffffffu, v[k], o);
+        if (tid == 0) {
+          const double ic = g.inv_cnt;
+          L.acc[0] += v[0] * ic;
+          L.acc[1] += v[4] * ic;
+          L.acc[2] += v[1] * ic;
+          L.acc[3] += v[2] * ic;
+          L.acc[4] += v[3] * ic;
+          L.acc[5] += v[0] * ic + g.vf_coef * v[4] * ic - g.ent_coef * v[1] * ic;
+        }
+      }
+      if (!grid_barrier(L.bar, &s_ok)) {
+        if (tid == 0) atomicExch(L.err, 1);
+        return;
+      }
+      // phase 3: global norm (fixed order), clip factor, Adam on this slice
+      if (tid < 32) {
+        double t = 0.0;
+        for (int b = tid; b < (int)gridDim.x; b += 32) t += __ldcg(L.sq + b);
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
+        if (tid == 0) s_norm = sqrt(t);
+      }
+      __syncthreads();
+      const double norm = s_norm;
+      const float coef = (float)fmin(1.0, (double)L.max_norm / (norm + 1e-6));
+      const float step_size = (float)L.bc[2 * step], inv_sqrt_bc2 = (float)L.bc[2 * step + 1];
+      for (int64_t p = p0 + tid; p < p1; p += blockDim.x) {
+        const float gp = L.g.grad_out[p] * coef;
+        const float mp = L.beta1 * L.m[p] + (1.0f - L.beta1) * gp;
+        const float vp = L.beta2 * L.v[p] + (1.0f - L.beta2) * gp * gp;
+        L.m[p] = mp;
+        L.v[p] = vp;
+        L.params[p] -= step_size * mp / (sqrtf(vp) * inv_sqrt_bc2 + L.eps);
+      }
+      if (blockIdx.x == 0 && tid == 0) {
+        L.acc[6] = norm;
+        L.acc[7] += 1.0;
+      }
+      if (!grid_barrier(L.bar, &s_ok)) {
+        if (tid == 0) atomicExch(L.err, 1);
+        return;
+      }
+    }
+  }
 }
 
 // grad[p] = sum_c partial[c][p] in a fixed order: a block covers 32
@@ -489,11 +674,14 @@ __global__ void ppo_adam_kernel(float* __restrict__ params, float* __restrict__ 
   }
 }
 
-__global__ void ppo_finalize_kernel(const double* __restrict__ acc, float* __restrict__ stats) {
+// stats[7] is the Adam step count, or -1 if a bounded grid-barrier wait gave up
+__global__ void ppo_finalize_kernel(const double* __restrict__ acc, const int32_t* __restrict__ err,
+                                    float* __restrict__ stats) {
   const int k = threadIdx.x;
   if (k < 8) {
     const double n = acc[7] > 0 ? acc[7] : 1.0;
     stats[k] = (float)(k < 6 ? acc[k] / n : acc[k]);
+    if (k == 7 && *err) stats[7] = -1.0f;
   }
 }
 
@@ -517,8 +705,8 @@ Feistel make_feistel(uint64_t n, uint64_t seed, uint32_t epoch, uint32_t iterati
 
 struct PpoPlan {
   int64_t P, N;
-  int nmb, NC, slices_per_cta, nsq;
-  int64_t off_advstat, off_partial, off_stat, off_grad, off_sq, off_acc, total;
+  int nmb, NC, slices_per_cta, nsq, steps;
+  int64_t off_advstat, off_partial, off_stat, off_grad, off_sq, off_acc, off_bar, off_bc, total;
 };
 
 static int64_t align256(int64_t x) { return (x + 255) / 256 * 256; }
@@ -532,13 +720,16 @@ static PpoPlan ppo_plan(const pe_net& net, const pe_ppo_config& cfg, int64_t N) 
   p.NC = slices < 64 ? slices : 64;
   p.slices_per_cta = (slices + p.NC - 1) / p.NC;
   p.nsq = (int)((p.P + kRedP - 1) / kRedP);
+  p.steps = cfg.epochs * p.nmb;
   int64_t o = 0;
   p.off_advstat = o; o = align256(o + (int64_t)cfg.epochs * p.nmb * 8);
   p.off_partial = o; o = align256(o + (int64_t)p.NC * p.P * 4);
   p.off_stat = o; o = align256(o + (int64_t)2 * p.NC * 8 * 4);
   p.off_grad = o; o = align256(o + p.P * 4);
-  p.off_sq = o; o = align256(o + (int64_t)p.nsq * 8);
+  p.off_sq = o; o = align256(o + (int64_t)(p.nsq > 2 * p.NC ? p.nsq : 2 * p.NC) * 8);
   p.off_acc = o; o = align256(o + 8 * 8 + 16);
+  p.off_bar = o; o = align256(o + 16);
+  p.off_bc = o; o = align256(o + (int64_t)p.steps * 16);
   p.total = o;
   return p;
 }
@@ -576,74 +767,134 @@ static pe_status ppo_run(const pe_net& net, float* params, float* m, float* v, i
   int dev = 0, sms = 0;
   PE_TRY_CUDA(cudaGetDevice(&dev));
   PE_TRY_CUDA(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
-  int64_t t = adam_t;
-  for (int ep = 0; ep < cfg.epochs; ++ep) {
-    for (int mb = 0; mb < pl.nmb; ++mb) {
-      const int64_t start = (int64_t)mb * cfg.minibatch;
-      const int cnt = (int)std::min<int64_t>(cfg.minibatch, N - start);
-      PpoArgs g;
-      g.obs = obs;
-      g.act = act;
-      g.logp_old = logp_old;
-      g.adv = adv;
-      g.ret = ret;
-      g.params = params;
-      g.perm = perms.f[ep];
-      g.start = start;
-      g.cnt = cnt;
-      g.clip = cfg.clip;
-      g.vf_coef = cfg.vf_coef;
-      g.ent_coef = cfg.ent_coef;
-      g.inv_cnt = 1.0f / (float)cnt;
-      g.partial = partial;
-      g.stat_partial = stat_partial;
-      g.NC = pl.NC;
-      g.slices_per_cta = pl.slices_per_cta;
-      g.P = pl.P;
-      g.advstat = advstat + (int64_t)ep * pl.nmb + mb;
-      {
-        ProfScope ps(PE_PROF_PPO_GRAD, st);
-        kern<<<2 * pl.NC, kPpoNT, bytes, st>>>(g);
+  unsigned int* bar = reinterpret_cast<unsigned int*>(ws + pl.off_bar);
+  int32_t* bar_err = reinterpret_cast<int32_t*>(ws + pl.off_bar + 8);
+  PE_TRY_CUDA(cudaMemsetAsync(bar, 0, 16, st));
+  // cooperative persistent update when every CTA can be resident at once
+  auto pk = ppo_persistent_kernel<D, H, A>;
+  PE_TRY_CUDA(cudaFuncSetAttribute(pk, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes));
+  int per_sm = 0, coop = 0;
+  PE_TRY_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, pk, kPpoNT, bytes));
+  PE_TRY_CUDA(cudaDeviceGetAttribute(&coop, cudaDevAttrCooperativeLaunch, dev));
+  if (coop && per_sm * sms >= 2 * pl.NC) {
+    std::vector<double> bc(2 * (size_t)pl.steps);
+    for (int k = 0; k < pl.steps; ++k) {
+      const double tt = (double)(adam_t + k + 1);
+      bc[2 * k] = cfg.lr / (1.0 - std::pow((double)cfg.beta1, tt));
+      bc[2 * k + 1] = 1.0 / std::sqrt(1.0 - std::pow((double)cfg.beta2, tt));
+    }
+    double* bc_dev = reinterpret_cast<double*>(ws + pl.off_bc);
+    PE_TRY_CUDA(cudaMemcpyAsync(bc_dev, bc.data(), bc.size() * sizeof(double), cudaMemcpyHostToDevice, st));
+    PpoLoop L;
+    L.g.obs = obs;
+    L.g.act = act;
+    L.g.logp_old = logp_old;
+    L.g.adv = adv;
+    L.g.ret = ret;
+    L.g.params = params;
+    L.g.clip = cfg.clip;
+    L.g.vf_coef = cfg.vf_coef;
+    L.g.ent_coef = cfg.ent_coef;
+    L.g.partial = partial;
+    L.g.stat_partial = stat_partial;
+    L.g.grad_out = grad;
+    L.g.NC = pl.NC;
+    L.g.slices_per_cta = pl.slices_per_cta;
+    L.g.P = pl.P;
+    L.advstat = advstat;
+    L.perms = perms;
+    L.N = N;
+    L.minibatch = cfg.minibatch;
+    L.nmb = pl.nmb;
+    L.epochs = cfg.epochs;
+    L.params = params;
+    L.m = m;
+    L.v = v;
+    L.sq = sq;
+    L.acc = acc;
+    L.bar = bar;
+    L.err = bar_err;
+    L.bc = bc_dev;
+    L.beta1 = cfg.beta1;
+    L.beta2 = cfg.beta2;
+    L.eps = cfg.eps;
+    L.max_norm = cfg.max_grad_norm;
+    void* kargs[] = {&L};
+    {
+      ProfScope ps(PE_PROF_PPO_GRAD, st);
+      PE_TRY_CUDA(cudaLaunchCooperativeKernel((void*)pk, dim3(2 * pl.NC), dim3(kPpoNT), kargs, (size_t)bytes, st));
+    }
+    PE_CHECK_LAUNCH("ppo_persistent_kernel");
+  } else {
+    int64_t t = adam_t;
+    for (int ep = 0; ep < cfg.epochs; ++ep) {
+      for (int mb = 0; mb < pl.nmb; ++mb) {
+        const int64_t start = (int64_t)mb * cfg.minibatch;
+        const int cnt = (int)std::min<int64_t>(cfg.minibatch, N - start);
+        PpoArgs g;
+        g.obs = obs;
+        g.act = act;
+        g.logp_old = logp_old;
+        g.adv = adv;
+        g.ret = ret;
+        g.params = params;
+        g.perm = perms.f[ep];
+        g.start = start;
+        g.cnt = cnt;
+        g.clip = cfg.clip;
+        g.vf_coef = cfg.vf_coef;
+        g.ent_coef = cfg.ent_coef;
+        g.inv_cnt = 1.0f / (float)cnt;
+        g.partial = partial;
+        g.stat_partial = stat_partial;
+        g.NC = pl.NC;
+        g.slices_per_cta = pl.slices_per_cta;
+        g.P = pl.P;
+        g.advstat = advstat + (int64_t)ep * pl.nmb + mb;
+        {
+          ProfScope ps(PE_PROF_PPO_GRAD, st);
+          kern<<<2 * pl.NC, kPpoNT, bytes, st>>>(g);
+        }
+        PE_CHECK_LAUNCH("ppo_grad_kernel");
+        {
+          ProfScope ps(PE_PROF_PPO_REDUCE, st);
+          ReduceArgs ra;
+          ra.partial = partial;
+          ra.stat_partial = stat_partial;
+          ra.NC = pl.NC;
+          ra.P = pl.P;
+          ra.grad = grad;
+          ra.sq = sq;
+          ra.ticket = ticket;
+          ra.norm = norm;
+          ra.acc = acc;
+          ra.vf_coef = cfg.vf_coef;
+          ra.ent_coef = cfg.ent_coef;
+          ra.inv_cnt = 1.0f / (float)cnt;
+          ppo_reduce_kernel<<<pl.nsq, kRedP * kRedG, 0, st>>>(ra);
+        }
+        PE_CHECK_LAUNCH("ppo_reduce_kernel");
+        t += 1;
+        const double bc1 = 1.0 - std::pow((double)cfg.beta1, (double)t);
+        const double bc2 = 1.0 - std::pow((double)cfg.beta2, (double)t);
+        AdamArgs a;
+        a.beta1 = cfg.beta1;
+        a.beta2 = cfg.beta2;
+        a.step_size = (float)(cfg.lr / bc1);
+        a.inv_sqrt_bc2 = (float)(1.0 / std::sqrt(bc2));
+        a.eps = cfg.eps;
+        a.max_norm = cfg.max_grad_norm;
+        {
+          ProfScope ps(PE_PROF_PPO_ADAM, st);
+          ppo_adam_kernel<<<(int)((pl.P + 255) / 256), 256, 0, st>>>(params, m, v, grad, norm, pl.P, a);
+        }
+        PE_CHECK_LAUNCH("ppo_adam_kernel");
       }
-      PE_CHECK_LAUNCH("ppo_grad_kernel");
-      {
-        ProfScope ps(PE_PROF_PPO_REDUCE, st);
-        ReduceArgs ra;
-        ra.partial = partial;
-        ra.stat_partial = stat_partial;
-        ra.NC = pl.NC;
-        ra.P = pl.P;
-        ra.grad = grad;
-        ra.sq = sq;
-        ra.ticket = ticket;
-        ra.norm = norm;
-        ra.acc = acc;
-        ra.vf_coef = cfg.vf_coef;
-        ra.ent_coef = cfg.ent_coef;
-        ra.inv_cnt = 1.0f / (float)cnt;
-        ppo_reduce_kernel<<<pl.nsq, kRedP * kRedG, 0, st>>>(ra);
-      }
-      PE_CHECK_LAUNCH("ppo_reduce_kernel");
-      t += 1;
-      const double bc1 = 1.0 - std::pow((double)cfg.beta1, (double)t);
-      const double bc2 = 1.0 - std::pow((double)cfg.beta2, (double)t);
-      AdamArgs a;
-      a.beta1 = cfg.beta1;
-      a.beta2 = cfg.beta2;
-      a.step_size = (float)(cfg.lr / bc1);
-      a.inv_sqrt_bc2 = (float)(1.0 / std::sqrt(bc2));
-      a.eps = cfg.eps;
-      a.max_norm = cfg.max_grad_norm;
-      {
-        ProfScope ps(PE_PROF_PPO_ADAM, st);
-        ppo_adam_kernel<<<(int)((pl.P + 255) / 256), 256, 0, st>>>(params, m, v, grad, norm, pl.P, a);
-      }
-      PE_CHECK_LAUNCH("ppo_adam_kernel");
     }
   }
   {
     ProfScope ps(PE_PROF_PPO_OTHER, st);
-    ppo_finalize_kernel<<<1, 32, 0, st>>>(acc, stats);
+    ppo_finalize_kernel<<<1, 32, 0, st>>>(acc, bar_err, stats);
   }
   PE_CHECK_LAUNCH("ppo_finalize_kernel");
   return PE_OK;

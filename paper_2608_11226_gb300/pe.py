@@ -24,8 +24,9 @@ PE_F32, PE_BF16 = 0, 1
 PE_ROLLOUT_DETERMINISTIC = 1
 MAX_LEVELS, MAX_CH = 32, 4
 (PE_PROF_ROLLOUT, PE_PROF_VALUE, PE_PROF_GAE, PE_PROF_PPO_GRAD, PE_PROF_PPO_REDUCE,
- PE_PROF_PPO_ADAM, PE_PROF_PPO_OTHER, PE_PROF_FLEET_PREP, PE_PROF_FLEET_WINDOWS) = range(9)
-PE_PROF_KINDS = 9
+ PE_PROF_PPO_ADAM, PE_PROF_PPO_OTHER, PE_PROF_FLEET_PREP, PE_PROF_FLEET_WINDOWS,
+ PE_PROF_MLP_POLICY, PE_PROF_MLP_VALUE) = range(11)
+PE_PROF_KINDS = 11
 
 
 class PEError(RuntimeError):
