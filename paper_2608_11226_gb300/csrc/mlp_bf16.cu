@@ -27,7 +27,7 @@ namespace pe {
 __device__ int32_t g_tc_error = 0;
 
 constexpr int kTcRows = 128;     // rows (envs / samples) per tile, the MMA M
-constexpr int kTcThreads = 256;  // 8 warps: 4 TMEM lane quadrants x 2 column halves
+constexpr int kTcThreads = 512;  // 16 warps: 4 TMEM lane quadrants x 4 column slices
 constexpr int kHeadN = 16;       // head width (logits or value padded to 16)
 
 // byte sizes of the weight image parts of one network (D, H)
@@ -79,29 +79,45 @@ struct MlpBf16Smem {
   alignas(1024) uint8_t w[Img<D, H>::TOTAL];
   alignas(1024) uint8_t act[Img<D, H>::ACT];  // X (layer-1 A operand) aliases its start
   float b1[H], b2[H], b3[kHeadN];
-  uint64_t bar_w, bar_mma;
+  uint64_t bar_w, bar_mma, bar_hi;  // bar_mma: first column half (and the head), bar_hi: second half
   uint32_t tmem_base;
   int32_t err;
 };
 
-// fp32 epilogue of one layer: TMEM columns [col0, col0+H) -> tanh(. + b) -> bf16 A tile
+// fp32 epilogue of one layer for this warp's H/4 columns, in two parts so that
+// the arithmetic can overlap the tensor core while the store waits for it:
+//   epi_compute: TMEM -> tanh(. + b) -> packed bf16 pairs in registers
+//   epi_store:   registers -> the next layer's A tile (swizzled)
+// Warp w reads TMEM lanes 32*(w%4)..+31 (its rows) and column slice w/4.
 template <int H>
-__device__ __forceinline__ void epilogue_tanh(uint32_t tmem, int col0, const float* bias, uint8_t* act) {
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int quad = warp & 3, half = warp >> 2;
-  const int row = quad * 32 + lane;
+__device__ __forceinline__ void epi_compute(uint32_t tmem, int col0, const float* bias,
+                                            uint32_t (&pk)[H / 8]) {
+  const int warp = threadIdx.x >> 5;
+  const int quad = warp & 3, slice = warp >> 2;
   const uint32_t lane_addr = tmem + ((uint32_t)(quad * 32) << 16);
-#pragma unroll 1
-  for (int j = 0; j < H / 2 / 16; ++j) {
-    const int c = half * (H / 2) + j * 16;
+#pragma unroll
+  for (int j = 0; j < H / 64; ++j) {
+    const int c = slice * (H / 4) + j * 16;
     float v[16];
     tc::tmem_ld16(lane_addr + (uint32_t)(col0 + c), v);
-    uint32_t p[8];
 #pragma unroll
     for (int i = 0; i < 8; ++i)
-      p[i] = tc::pack_bf16(tanhf(v[2 * i] + bias[c + 2 * i]), tanhf(v[2 * i + 1] + bias[c + 2 * i + 1]));
-    *reinterpret_cast<uint4*>(act + tc::swz_offset<128>(row, c, kTcRows)) = make_uint4(p[0], p[1], p[2], p[3]);
-    *reinterpret_cast<uint4*>(act + tc::swz_offset<128>(row, c + 8, kTcRows)) = make_uint4(p[4], p[5], p[6], p[7]);
+      pk[j * 8 + i] = tc::pack_bf16(tanhf(v[2 * i] + bias[c + 2 * i]), tanhf(v[2 * i + 1] + bias[c + 2 * i + 1]));
+  }
+}
+
+template <int H>
+__device__ __forceinline__ void epi_store(const uint32_t (&pk)[H / 8], uint8_t* act) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int quad = warp & 3, slice = warp >> 2;
+  const int row = quad * 32 + lane;
+#pragma unroll
+  for (int j = 0; j < H / 64; ++j) {
+    const int c = slice * (H / 4) + j * 16;
+    *reinterpret_cast<uint4*>(act + tc::swz_offset<128>(row, c, kTcRows)) =
+        make_uint4(pk[j * 8 + 0], pk[j * 8 + 1], pk[j * 8 + 2], pk[j * 8 + 3]);
+    *reinterpret_cast<uint4*>(act + tc::swz_offset<128>(row, c + 8, kTcRows)) =
+        make_uint4(pk[j * 8 + 4], pk[j * 8 + 5], pk[j * 8 + 6], pk[j * 8 + 7]);
   }
 }
 
@@ -124,6 +140,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     s.err = 0;
     tc::mbar_init(&s.bar_w, 1);
     tc::mbar_init(&s.bar_mma, 1);
+    tc::mbar_init(&s.bar_hi, 1);
     tc::fence_mbar_init();
   }
   if (warp == 0) tc::tmem_alloc(&s.tmem_base, 512);
@@ -145,9 +162,9 @@ __global__ void __launch_bounds__(kTcThreads, 1)
 
   const uint32_t w1 = tc::smem_u32(s.w), w2 = w1 + I::W1, w3 = w2 + I::W2;
   const uint32_t xa = tc::smem_u32(s.act);
-  constexpr uint32_t kId1 = tc::idesc_bf16(kTcRows, H);
+  constexpr uint32_t kIdHalf = tc::idesc_bf16(kTcRows, H / 2);
   constexpr uint32_t kIdH = tc::idesc_bf16(kTcRows, kHeadN);
-  uint32_t phase = 0;
+  uint32_t phase = 0, phase_hi = 0;
   const int64_t tiles = (n + kTcRows - 1) / kTcRows;
   for (int64_t tile = blockIdx.x; tile < tiles && s.err == 0; tile += gridDim.x) {
     const int64_t r0 = tile * kTcRows;
@@ -162,20 +179,39 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     }
     tc::fence_async_smem();
     __syncthreads();
+    // Each layer's N = H outputs are issued as two halves of H/2 columns with
+    // separate commits, so that the warps of the first column half run their
+    // epilogue while the tensor core computes the second half.
+    const bool hi_half = (warp >> 2) >= 2;  // column slices 2, 3
     // layer 1: D1[128 x H] (TMEM cols 0..H) = X W1^T
     if (tid == 0) {
       tc::fence_after();
+#pragma unroll 1
+      for (int h = 0; h < 2; ++h) {
 #pragma unroll
-      for (int kk = 0; kk < D / 16; ++kk)
-        tc::mma_bf16(tmem, tc::desc_kmajor(xa + kk * 32, 8 * I::RB1, I::RB1 == 64 ? tc::kLayoutSW64 : tc::kLayoutSW128),
-                     tc::desc_kmajor(w1 + kk * 32, 8 * I::RB1, I::RB1 == 64 ? tc::kLayoutSW64 : tc::kLayoutSW128),
-                     kId1, kk > 0);
-      tc::mma_commit(&s.bar_mma);
+        for (int kk = 0; kk < D / 16; ++kk)
+          tc::mma_bf16(tmem + h * (H / 2),
+                       tc::desc_kmajor(xa + kk * 32, 8 * I::RB1, I::RB1 == 64 ? tc::kLayoutSW64 : tc::kLayoutSW128),
+                       tc::desc_kmajor(w1 + h * (H / 2) * I::RB1 + kk * 32, 8 * I::RB1,
+                                       I::RB1 == 64 ? tc::kLayoutSW64 : tc::kLayoutSW128),
+                       kIdHalf, kk > 0);
+        tc::mma_commit(h == 0 ? &s.bar_mma : &s.bar_hi);
+      }
     }
-    if (!tc::mbar_wait(&s.bar_mma, phase)) atomicExch(&s.err, 1);
-    phase ^= 1;
+    // epilogue 1: the first column half computes as soon as its MMAs are done;
+    // every warp stores only after all layer-1 MMAs have read X (same buffer)
+    uint32_t pk[H / 8];
+    if (!hi_half) {
+      if (!tc::mbar_wait(&s.bar_mma, phase)) atomicExch(&s.err, 1);
+      tc::fence_after();
+      epi_compute<H>(tmem, 0, s.b1, pk);
+    }
+    if (!tc::mbar_wait(&s.bar_hi, phase_hi)) atomicExch(&s.err, 1);
     tc::fence_after();
-    epilogue_tanh<H>(tmem, 0, s.b1, s.act);
+    if (hi_half) epi_compute<H>(tmem, 0, s.b1, pk);
+    epi_store<H>(pk, s.act);
+    phase ^= 1;
+    phase_hi ^= 1;
     tc::fence_before();
     tc::fence_async_smem();
     __syncthreads();
@@ -183,18 +219,30 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     if (tid == 0) {
       tc::fence_after();
 #pragma unroll 1
-      for (int kb = 0; kb < H / 64; ++kb)
+      for (int h = 0; h < 2; ++h) {
+#pragma unroll 1
+        for (int kb = 0; kb < H / 64; ++kb)
 #pragma unroll
-        for (int kk = 0; kk < 4; ++kk)
-          tc::mma_bf16(tmem + 256, tc::desc_kmajor(xa + kb * kTcRows * 128 + kk * 32, 1024, tc::kLayoutSW128),
-                       tc::desc_kmajor(w2 + kb * H * 128 + kk * 32, 1024, tc::kLayoutSW128), kId1,
-                       (kb | kk) != 0);
-      tc::mma_commit(&s.bar_mma);
+          for (int kk = 0; kk < 4; ++kk)
+            tc::mma_bf16(tmem + 256 + h * (H / 2),
+                         tc::desc_kmajor(xa + kb * kTcRows * 128 + kk * 32, 1024, tc::kLayoutSW128),
+                         tc::desc_kmajor(w2 + kb * H * 128 + h * (H / 2) * 128 + kk * 32, 1024, tc::kLayoutSW128),
+                         kIdHalf, (kb | kk) != 0);
+        tc::mma_commit(h == 0 ? &s.bar_mma : &s.bar_hi);
+      }
     }
-    if (!tc::mbar_wait(&s.bar_mma, phase)) atomicExch(&s.err, 1);
-    phase ^= 1;
+    // epilogue 2: as epilogue 1 (H2 overwrites H1, which the MMAs read)
+    if (!hi_half) {
+      if (!tc::mbar_wait(&s.bar_mma, phase)) atomicExch(&s.err, 1);
+      tc::fence_after();
+      epi_compute<H>(tmem, 256, s.b2, pk);
+    }
+    if (!tc::mbar_wait(&s.bar_hi, phase_hi)) atomicExch(&s.err, 1);
     tc::fence_after();
-    epilogue_tanh<H>(tmem, 256, s.b2, s.act);
+    if (hi_half) epi_compute<H>(tmem, 256, s.b2, pk);
+    epi_store<H>(pk, s.act);
+    phase ^= 1;
+    phase_hi ^= 1;
     tc::fence_before();
     tc::fence_async_smem();
     __syncthreads();

@@ -71,6 +71,28 @@ def test_gae_parity(T, E):
     assert rel_err(cpu(ret), rr) <= TOL
 
 
+@pytest.mark.parametrize("T,E", [(64, 16384), (2048, 131072)])
+def test_gae_parity_vector_paths(T, E):
+    """The 2- and 4-env-per-thread vector kernels (chosen for E >= 16,384 and
+    T*E >= 2^28); envs are independent, so the oracle checks sampled columns
+    including both ends of a 128-env CTA span."""
+    g = torch.Generator(device="cuda").manual_seed(E)
+    r = torch.randn(T, E, device="cuda", generator=g)
+    v = torch.randn(T, E, device="cuda", generator=g)
+    d = (torch.rand(T, E, device="cuda", generator=g) < 0.02).to(torch.uint8)
+    lv = torch.randn(E, device="cuda", generator=g)
+    adv = torch.empty(T, E, device="cuda")
+    ret = torch.empty(T, E, device="cuda")
+    pe.gae(r, v, d, lv, 0.99, 0.95, adv, ret)
+    torch.cuda.synchronize()
+    rng = np.random.default_rng(T)
+    cols = np.unique(np.concatenate([[0, 1, 127, 128, E - 1], rng.choice(E, 59, replace=False)]))
+    ci = torch.from_numpy(cols).cuda()
+    ra, rr = O.gae(cpu(r[:, ci]), cpu(v[:, ci]), cpu(d[:, ci]), cpu(lv[ci]), 0.99, 0.95)
+    assert rel_err(cpu(adv[:, ci]), ra) <= TOL
+    assert rel_err(cpu(ret[:, ci]), rr) <= TOL
+
+
 def test_gae_empty_is_noop():
     z = torch.empty(0, 5, device="cuda")
     pe.gae(z, z, z.to(torch.uint8), torch.empty(5, device="cuda"), 0.99, 0.95, z, z)
