@@ -102,7 +102,8 @@ typedef struct pe_env_config {
  * one flat fp32 vector, row-major W[out][in]:
  *   policy: W1[H][D] b1[H] W2[H][H] b2[H] W3[A][H] b3[A]
  *   value : V1[H][D] c1[H] V2[H][H] c2[H] V3[1][H] c3[1]
- * Supported (D, H, A, dtype): (8,64,3,F32), (16,128,5,F32), (32,256,16,BF16).  A BF16 network
+ * Supported (D, H, A, dtype): (8,64,3,F32), (16,128,5,F32), (32,256,16,BF16),
+ * (64,512,16,BF16).  A BF16 network
  * keeps fp32 master parameters; the library rounds weights, observations and
  * hidden activations to bf16 and accumulates in fp32. */
 typedef struct pe_net {
@@ -167,8 +168,8 @@ int64_t pe_param_count(const pe_net* net);
  * Then the value network on every observation and on obs_last.
  *  lambda: Lagrange multiplier of Eq. 6 (PE_REWARD_LAGRANGE only).
  *  workspace: >= pe_rollout_workspace_bytes(env, net) bytes of device memory
- *  (0 for fp32 networks: NULL is accepted).  BF16 networks (D=32, H=256,
- *  A=16, 4 channels) run on the tcgen05 tensor cores.
+ *  (0 for fp32 networks: NULL is accepted).  BF16 networks (D=32, H=256 or
+ *  D=64, H=512; A=16, 4 channels) run on the tcgen05 tensor cores.
  * Errors: PE_EINVAL (unsupported network, null buffer, horizon < 1, small
  * workspace), PE_ECUDA; a bounded tensor-core wait that gives up on the
  * device is reported by pe_device_check. */

@@ -284,6 +284,261 @@ __global__ void __launch_bounds__(kTcThreads, 1)
 }
 
 // ---------------------------------------------------------------------------
+// Streamed variant for networks whose weights do not fit in shared memory
+// (Stress: D=64, H=512; 592 KB of bf16 weights).  The 128-row activation
+// tile stays resident (128 KB); the weights flow through a two-slot ring of
+// 32 KB stages, each the B operand of one (N-half, K-block) of a layer:
+//   layer 1: 2 stages (N-halves of W1, K=64), layer 2: 16 stages (2 N-halves x
+//   8 K-blocks of W2), head: 1 stage (W3, 16 rows x 8 K-blocks).
+// A producer warp (warp 16) issues cp.async.bulk for stage s into slot s%2
+// once the MMAs that read the slot's previous stage have completed (signalled
+// by tcgen05.commit on the slot's "empty" barrier); one thread of warp 1
+// waits for the slot's "full" barrier and issues the MMAs.  The 16 compute
+// warps synchronise with a named barrier so that the producer never waits
+// on them.
+// ---------------------------------------------------------------------------
+constexpr int kStageBytes = 32768;
+constexpr int kStreamStages = 19;  // per tile (H = 512, D = 64)
+constexpr int kComputeThreads = 512;
+constexpr int kStreamThreads = kComputeThreads + 32;
+
+template <int D, int H>
+struct ImgS {
+  static_assert(D == 64 && H == 512, "streamed layout is laid out for D = 64, H = 512");
+  static constexpr int HEAD_OFF = 18 * kStageBytes;
+  static constexpr int TOTAL = HEAD_OFF + kHeadN * H * 2;  // 592 KB
+  __host__ __device__ static int stage_off(int s) { return s * kStageBytes; }
+  __host__ __device__ static int stage_bytes(int s) { return s < 18 ? kStageBytes : kHeadN * H * 2; }
+};
+
+template <int D, int H>
+__global__ void weight_image_stream_kernel(const float* __restrict__ params, int A, int value_net,
+                                           uint8_t* __restrict__ img) {
+  using I = ImgS<D, H>;
+  const MlpLayout Lp = mlp_layout(D, H, A);
+  const float* w1 = params + (value_net ? Lp.v1 : Lp.w1);
+  const float* w2 = params + (value_net ? Lp.v2 : Lp.w2);
+  const float* w3 = params + (value_net ? Lp.v3 : Lp.w3);
+  const int nout = value_net ? 1 : A;
+  const int total = H * D + H * H + kHeadN * H;
+  for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < total; i += gridDim.x * blockDim.x) {
+    uint32_t off;
+    float v;
+    if (i < H * D) {
+      const int r = i / D, k = i % D;
+      off = (r / 256) * kStageBytes + tc::swz_offset<128>(r % 256, k, 256);
+      v = w1[i];
+    } else if (i < H * D + H * H) {
+      const int j = i - H * D, r = j / H, k = j % H;
+      const int stage = 2 + (r / 256) * 8 + k / 64;
+      off = stage * kStageBytes + tc::swz_offset<128>(r % 256, k % 64, 256);
+      v = w2[j];
+    } else {
+      const int j = i - H * D - H * H, r = j / H, k = j % H;
+      off = I::HEAD_OFF + tc::swz_offset<128>(r, k, kHeadN);
+      v = r < nout ? w3[r * H + k] : 0.0f;
+    }
+    *reinterpret_cast<__nv_bfloat16*>(img + off) = __float2bfloat16_rn(v);
+  }
+}
+
+template <int D, int H>
+struct MlpStreamSmem {
+  alignas(1024) uint8_t act[kTcRows * H * 2];
+  alignas(1024) uint8_t ring[2][kStageBytes];
+  float b1[H], b2[H], b3[kHeadN];
+  uint64_t full[2], empty[2], bar_mma;
+  uint32_t tmem_base;
+  int32_t err;
+};
+
+__device__ __forceinline__ void compute_sync() { asm volatile("bar.sync 1, 512;" ::: "memory"); }
+
+template <int D, int H>
+__global__ void __launch_bounds__(kStreamThreads, 1)
+    mlp_bf16_stream_kernel(const uint8_t* __restrict__ img, const float* __restrict__ params, int A,
+                           int value_net, const __nv_bfloat16* __restrict__ obs, int64_t n,
+                           float* __restrict__ out, int out_stride, int nout, int32_t* __restrict__ err) {
+  using I = ImgS<D, H>;
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
+  MlpStreamSmem<D, H>& s = *reinterpret_cast<MlpStreamSmem<D, H>*>(base);
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const MlpLayout Lp = mlp_layout(D, H, A);
+  if (tid == 0) {
+    s.err = 0;
+    for (int i = 0; i < 2; ++i) {
+      tc::mbar_init(&s.full[i], 1);
+      tc::mbar_init(&s.empty[i], 1);
+    }
+    tc::mbar_init(&s.bar_mma, 1);
+    tc::fence_mbar_init();
+  }
+  if (warp == 0) tc::tmem_alloc(&s.tmem_base, 512);
+  for (int i = tid; i < H; i += blockDim.x) {
+    s.b1[i] = __ldg(params + (value_net ? Lp.c1 : Lp.b1) + i);
+    s.b2[i] = __ldg(params + (value_net ? Lp.c2 : Lp.b2) + i);
+  }
+  if (tid < kHeadN) s.b3[tid] = tid < nout ? __ldg(params + (value_net ? Lp.c3 : Lp.b3) + tid) : 0.0f;
+  tc::fence_before();
+  __syncthreads();
+  tc::fence_after();
+  const uint32_t tmem = s.tmem_base;
+  const int64_t tiles = (n + kTcRows - 1) / kTcRows;
+  const int my_tiles = (int)((tiles - blockIdx.x + gridDim.x - 1) / gridDim.x);
+
+  if (warp == kComputeThreads / 32) {
+    // producer: every stage of every tile of this CTA, in consumption order
+    if (lane == 0) {
+      int gs = 0;
+      for (int t = 0; t < my_tiles; ++t) {
+        for (int st = 0; st < kStreamStages; ++st, ++gs) {
+          const int slot = gs & 1;
+          if (gs >= 2 && !tc::mbar_wait(&s.empty[slot], ((gs - 2) >> 1) & 1)) {
+            atomicExch(&s.err, 1);
+            t = my_tiles;
+            break;
+          }
+          tc::mbar_expect_tx(&s.full[slot], (uint32_t)I::stage_bytes(st));
+          tc::bulk_g2s(s.ring[slot], img + I::stage_off(st), (uint32_t)I::stage_bytes(st), &s.full[slot]);
+        }
+      }
+    }
+  } else {
+    const bool issuer = (tid == 32);
+    const uint32_t xa = tc::smem_u32(s.act);
+    const uint32_t r0a = tc::smem_u32(s.ring[0]), r1a = tc::smem_u32(s.ring[1]);
+    constexpr uint32_t kIdN = tc::idesc_bf16(kTcRows, 256);
+    constexpr uint32_t kIdH = tc::idesc_bf16(kTcRows, kHeadN);
+    uint32_t phase = 0;
+    int gs = 0;  // global stage counter of the issuing thread
+    const int quad = warp & 3, slice = warp >> 2, row = quad * 32 + lane;
+    const uint32_t lane_addr = tmem + ((uint32_t)(quad * 32) << 16);
+    for (int t = 0; t < my_tiles; ++t) {
+      if (s.err) break;
+      const int64_t tile = blockIdx.x + (int64_t)t * gridDim.x;
+      const int64_t rbase = tile * kTcRows;
+      const int nr = (int)(n - rbase < kTcRows ? n - rbase : kTcRows);
+      // observation tile (D = 64 bf16 = one 128-byte K-block per row)
+      for (int i = tid; i < kTcRows * (D / 8); i += kComputeThreads) {
+        const int r = i / (D / 8), c = i % (D / 8);
+        uint4 v = make_uint4(0, 0, 0, 0);
+        if (r < nr) v = __ldg(reinterpret_cast<const uint4*>(obs + (rbase + r) * D) + c);
+        *reinterpret_cast<uint4*>(s.act + tc::swz_offset<128>(r, c * 8, kTcRows)) = v;
+      }
+      tc::fence_async_smem();
+      compute_sync();
+      // one weight stage: wait for its slot, issue its MMAs, release the slot
+      auto run_stage = [&](int stg, auto&& body) {
+        const int slot = gs & 1;
+        if (!tc::mbar_wait(&s.full[slot], (gs >> 1) & 1)) atomicExch(&s.err, 1);
+        tc::fence_after();
+        body(slot ? r1a : r0a);
+        tc::mma_commit(&s.empty[slot]);
+        ++gs;
+        (void)stg;
+      };
+      // layer 1: D1 (TMEM cols 0..512) = X W1^T, two N-halves
+      if (issuer) {
+        for (int h = 0; h < 2; ++h)
+          run_stage(h, [&](uint32_t ra) {
+#pragma unroll
+            for (int kk = 0; kk < D / 16; ++kk)
+              tc::mma_bf16(tmem + h * 256, tc::desc_kmajor(xa + kk * 32, 1024, tc::kLayoutSW128),
+                           tc::desc_kmajor(ra + kk * 32, 1024, tc::kLayoutSW128), kIdN, kk > 0);
+          });
+        tc::mma_commit(&s.bar_mma);
+      }
+      if (!tc::mbar_wait(&s.bar_mma, phase)) atomicExch(&s.err, 1);
+      phase ^= 1;
+      tc::fence_after();
+      // epilogue 1: 128 columns per warp, chunk by chunk
+#pragma unroll 1
+      for (int j = 0; j < H / 4 / 16; ++j) {
+        const int c = slice * (H / 4) + j * 16;
+        float v[16];
+        tc::tmem_ld16(lane_addr + (uint32_t)c, v);
+        uint32_t p[8];
+#pragma unroll
+        for (int i = 0; i < 8; ++i)
+          p[i] = tc::pack_bf16(tanhf(v[2 * i] + s.b1[c + 2 * i]), tanhf(v[2 * i + 1] + s.b1[c + 2 * i + 1]));
+        *reinterpret_cast<uint4*>(s.act + tc::swz_offset<128>(row, c, kTcRows)) = make_uint4(p[0], p[1], p[2], p[3]);
+        *reinterpret_cast<uint4*>(s.act + tc::swz_offset<128>(row, c + 8, kTcRows)) = make_uint4(p[4], p[5], p[6], p[7]);
+      }
+      tc::fence_before();
+      tc::fence_async_smem();
+      compute_sync();
+      // layer 2: D2 (TMEM cols 0..512) = H1 W2^T, 2 N-halves x 8 K-blocks
+      if (issuer) {
+        tc::fence_after();
+        for (int h = 0; h < 2; ++h)
+          for (int kb = 0; kb < H / 64; ++kb)
+            run_stage(2 + h * 8 + kb, [&](uint32_t ra) {
+#pragma unroll
+              for (int kk = 0; kk < 4; ++kk)
+                tc::mma_bf16(tmem + h * 256, tc::desc_kmajor(xa + kb * kTcRows * 128 + kk * 32, 1024, tc::kLayoutSW128),
+                             tc::desc_kmajor(ra + kk * 32, 1024, tc::kLayoutSW128), kIdN, (kb | kk) != 0);
+            });
+        tc::mma_commit(&s.bar_mma);
+      }
+      if (!tc::mbar_wait(&s.bar_mma, phase)) atomicExch(&s.err, 1);
+      phase ^= 1;
+      tc::fence_after();
+#pragma unroll 1
+      for (int j = 0; j < H / 4 / 16; ++j) {
+        const int c = slice * (H / 4) + j * 16;
+        float v[16];
+        tc::tmem_ld16(lane_addr + (uint32_t)c, v);
+        uint32_t p[8];
+#pragma unroll
+        for (int i = 0; i < 8; ++i)
+          p[i] = tc::pack_bf16(tanhf(v[2 * i] + s.b2[c + 2 * i]), tanhf(v[2 * i + 1] + s.b2[c + 2 * i + 1]));
+        *reinterpret_cast<uint4*>(s.act + tc::swz_offset<128>(row, c, kTcRows)) = make_uint4(p[0], p[1], p[2], p[3]);
+        *reinterpret_cast<uint4*>(s.act + tc::swz_offset<128>(row, c + 8, kTcRows)) = make_uint4(p[4], p[5], p[6], p[7]);
+      }
+      tc::fence_before();
+      tc::fence_async_smem();
+      compute_sync();
+      // head: D3 (TMEM cols 0..16) = H2 W3^T (one 16 KB stage)
+      if (issuer) {
+        tc::fence_after();
+        run_stage(18, [&](uint32_t ra) {
+#pragma unroll 1
+          for (int kb = 0; kb < H / 64; ++kb)
+#pragma unroll
+            for (int kk = 0; kk < 4; ++kk)
+              tc::mma_bf16(tmem, tc::desc_kmajor(xa + kb * kTcRows * 128 + kk * 32, 1024, tc::kLayoutSW128),
+                           tc::desc_kmajor(ra + kb * kHeadN * 128 + kk * 32, 1024, tc::kLayoutSW128), kIdH,
+                           (kb | kk) != 0);
+        });
+        tc::mma_commit(&s.bar_mma);
+      }
+      if (!tc::mbar_wait(&s.bar_mma, phase)) atomicExch(&s.err, 1);
+      phase ^= 1;
+      tc::fence_after();
+      if (warp < 4) {
+        float v[16];
+        tc::tmem_ld16(lane_addr, v);
+        if (row < nr) {
+          float* o = out + (rbase + row) * out_stride;
+#pragma unroll
+          for (int j = 0; j < kHeadN; ++j)
+            if (j < nout) o[j] = v[j] + s.b3[j];
+        }
+      }
+      tc::fence_before();
+      compute_sync();
+    }
+  }
+  __syncthreads();
+  if (tid == 0 && s.err) {
+    atomicExch(&g_tc_error, 1);
+    if (err) atomicExch(err, 1);
+  }
+  if (warp == 0) tc::tmem_dealloc(tmem, 512);
+}
+
+// ---------------------------------------------------------------------------
 // decoupled bf16 rollout: per step, an env kernel (one thread per env: act on
 // the previous step's logits, then observe) and the tensor-core policy kernel
 // ---------------------------------------------------------------------------
@@ -352,10 +607,22 @@ __global__ void __launch_bounds__(128) env_actobs_kernel(EnvDev env, ActArgs a, 
 }
 
 // workspace: weight image (policy), weight image (value), logits [E][16], error word
+template <int D, int H, bool STREAM = (H > 256)>
+struct NetKind;
+template <int D, int H>
+struct NetKind<D, H, false> {
+  static constexpr bool kStream = false;
+  static constexpr int64_t kImgPad = (Img<D, H>::TOTAL + 1023) / 1024 * 1024;
+};
+template <int D, int H>
+struct NetKind<D, H, true> {
+  static constexpr bool kStream = true;
+  static constexpr int64_t kImgPad = (ImgS<D, H>::TOTAL + 1023) / 1024 * 1024;
+};
+
 template <int D, int H>
 static int64_t bf16_ws_bytes(int64_t E) {
-  const int64_t img = (Img<D, H>::TOTAL + 1023) / 1024 * 1024;
-  return 2 * img + (E * kHeadN * 4 + 255) / 256 * 256 + 256;
+  return 2 * NetKind<D, H>::kImgPad + (E * kHeadN * 4 + 255) / 256 * 256 + 256;
 }
 
 template <int D, int H>
@@ -363,19 +630,24 @@ static pe_status launch_mlp(const uint8_t* img, const float* params, int A, int 
                             const void* obs, int64_t n, float* out, int out_stride, int nout,
                             int32_t* err, cudaStream_t st, int prof_kind) {
   if (n <= 0) return PE_OK;
-  auto kern = mlp_bf16_kernel<D, H>;
-  const int bytes = (int)sizeof(MlpBf16Smem<D, H>) + 1024;
-  PE_TRY_CUDA(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes));
   int dev = 0, sms = 0;
   PE_TRY_CUDA(cudaGetDevice(&dev));
   PE_TRY_CUDA(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
   const int64_t tiles = (n + kTcRows - 1) / kTcRows;
   const int grid = (int)(tiles < sms ? tiles : sms);
-  {
+  const __nv_bfloat16* o = reinterpret_cast<const __nv_bfloat16*>(obs);
+  if constexpr (NetKind<D, H>::kStream) {
+    auto kern = mlp_bf16_stream_kernel<D, H>;
+    const int bytes = (int)sizeof(MlpStreamSmem<D, H>) + 1024;
+    PE_TRY_CUDA(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes));
     ProfScope ps(prof_kind, st);
-    kern<<<grid, kTcThreads, bytes, st>>>(img, params, A, value_net,
-                                          reinterpret_cast<const __nv_bfloat16*>(obs), n, out,
-                                          out_stride, nout, err);
+    kern<<<grid, kStreamThreads, bytes, st>>>(img, params, A, value_net, o, n, out, out_stride, nout, err);
+  } else {
+    auto kern = mlp_bf16_kernel<D, H>;
+    const int bytes = (int)sizeof(MlpBf16Smem<D, H>) + 1024;
+    PE_TRY_CUDA(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes));
+    ProfScope ps(prof_kind, st);
+    kern<<<grid, kTcThreads, bytes, st>>>(img, params, A, value_net, o, n, out, out_stride, nout, err);
   }
   PE_CHECK_LAUNCH("mlp_bf16_kernel");
   return PE_OK;
@@ -383,10 +655,15 @@ static pe_status launch_mlp(const uint8_t* img, const float* params, int A, int 
 
 template <int D, int H>
 static pe_status make_images(const float* params, int A, uint8_t* ws, cudaStream_t st, bool policy) {
-  const int64_t img = (Img<D, H>::TOTAL + 1023) / 1024 * 1024;
+  const int64_t img = NetKind<D, H>::kImgPad;
   ProfScope ps(PE_PROF_VALUE, st);
-  if (policy) weight_image_kernel<D, H><<<64, 256, 0, st>>>(params, A, 0, ws);
-  weight_image_kernel<D, H><<<64, 256, 0, st>>>(params, A, 1, ws + img);
+  if constexpr (NetKind<D, H>::kStream) {
+    if (policy) weight_image_stream_kernel<D, H><<<128, 256, 0, st>>>(params, A, 0, ws);
+    weight_image_stream_kernel<D, H><<<128, 256, 0, st>>>(params, A, 1, ws + img);
+  } else {
+    if (policy) weight_image_kernel<D, H><<<64, 256, 0, st>>>(params, A, 0, ws);
+    weight_image_kernel<D, H><<<64, 256, 0, st>>>(params, A, 1, ws + img);
+  }
   PE_CHECK_LAUNCH("weight_image_kernel");
   return PE_OK;
 }
@@ -396,7 +673,7 @@ static pe_status rollout_bf16_impl(const EnvDev& env, const float* params, int T
                                    float lambda, int det, const pe_rollout_buf& buf, void* wsv,
                                    cudaStream_t st) {
   uint8_t* ws = reinterpret_cast<uint8_t*>(wsv);
-  const int64_t img = (Img<D, H>::TOTAL + 1023) / 1024 * 1024;
+  const int64_t img = NetKind<D, H>::kImgPad;
   float* logits = reinterpret_cast<float*>(ws + 2 * img);
   int32_t* err = reinterpret_cast<int32_t*>(ws + 2 * img + (env.E * (int64_t)kHeadN * 4 + 255) / 256 * 256);
   PE_TRY_CUDA(cudaMemsetAsync(err, 0, 4, st));
@@ -427,6 +704,7 @@ static pe_status rollout_bf16_impl(const EnvDev& env, const float* params, int T
 
 int64_t rollout_bf16_ws_bytes(const pe_net& net, int64_t E) {
   if (net.obs_dim == 32 && net.hidden == 256) return bf16_ws_bytes<32, 256>(E);
+  if (net.obs_dim == 64 && net.hidden == 512) return bf16_ws_bytes<64, 512>(E);
   return -1;
 }
 
@@ -434,25 +712,10 @@ pe_status rollout_bf16(const EnvDev& env, const pe_net& net, const float* params
                        float lambda, int det, const pe_rollout_buf& buf, void* ws, cudaStream_t st) {
   if (net.obs_dim == 32 && net.hidden == 256 && net.n_actions == 16 && env.C == 4 && env.obs_kind == PE_OBS_OCC32)
     return rollout_bf16_impl<4, PE_OBS_OCC32, 32, 256, 16>(env, params, T, it, lambda, det, buf, ws, st);
+  if (net.obs_dim == 64 && net.hidden == 512 && net.n_actions == 16 && env.C == 4 && env.obs_kind == PE_OBS_OCC64)
+    return rollout_bf16_impl<4, PE_OBS_OCC64, 64, 512, 16>(env, params, T, it, lambda, det, buf, ws, st);
   return fail(PE_EINVAL, "unsupported bf16 network/env combination (D=%d H=%d A=%d C=%d obs=%d)",
               net.obs_dim, net.hidden, net.n_actions, env.C, env.obs_kind);
-}
-
-pe_status value_bf16(const pe_net& net, const float* params, const void* obs, int64_t n, float* value,
-                     void* wsv, cudaStream_t st) {
-  uint8_t* ws = reinterpret_cast<uint8_t*>(wsv);
-  auto run = [&](auto dtag, auto htag) -> pe_status {
-    constexpr int D = decltype(dtag)::value, H = decltype(htag)::value;
-    const int64_t img = (Img<D, H>::TOTAL + 1023) / 1024 * 1024;
-    int32_t* err = reinterpret_cast<int32_t*>(ws + 2 * img);
-    PE_TRY_CUDA(cudaMemsetAsync(err, 0, 4, st));
-    pe_status s = make_images<D, H>(params, net.n_actions, ws, st, false);
-    if (s != PE_OK) return s;
-    return launch_mlp<D, H>(ws + img, params, net.n_actions, 1, obs, n, value, 1, 1, err, st, PE_PROF_MLP_VALUE);
-  };
-  if (net.obs_dim == 32 && net.hidden == 256)
-    return run(std::integral_constant<int, 32>{}, std::integral_constant<int, 256>{});
-  return fail(PE_EINVAL, "unsupported bf16 value network (D=%d H=%d)", net.obs_dim, net.hidden);
 }
 
 pe_status device_check(cudaStream_t st) {
@@ -467,8 +730,28 @@ pe_status device_check(cudaStream_t st) {
   return PE_OK;
 }
 
+template <int D, int H>
+static pe_status value_bf16_impl(const pe_net& net, const float* params, const void* obs, int64_t n,
+                                 float* value, uint8_t* ws, cudaStream_t st) {
+  const int64_t img = NetKind<D, H>::kImgPad;
+  int32_t* err = reinterpret_cast<int32_t*>(ws + 2 * img);
+  PE_TRY_CUDA(cudaMemsetAsync(err, 0, 4, st));
+  pe_status s = make_images<D, H>(params, net.n_actions, ws, st, false);
+  if (s != PE_OK) return s;
+  return launch_mlp<D, H>(ws + img, params, net.n_actions, 1, obs, n, value, 1, 1, err, st, PE_PROF_MLP_VALUE);
+}
+
+pe_status value_bf16(const pe_net& net, const float* params, const void* obs, int64_t n, float* value,
+                     void* wsv, cudaStream_t st) {
+  uint8_t* ws = reinterpret_cast<uint8_t*>(wsv);
+  if (net.obs_dim == 32 && net.hidden == 256) return value_bf16_impl<32, 256>(net, params, obs, n, value, ws, st);
+  if (net.obs_dim == 64 && net.hidden == 512) return value_bf16_impl<64, 512>(net, params, obs, n, value, ws, st);
+  return fail(PE_EINVAL, "unsupported bf16 value network (D=%d H=%d)", net.obs_dim, net.hidden);
+}
+
 int64_t value_bf16_ws_bytes(const pe_net& net) {
   if (net.obs_dim == 32 && net.hidden == 256) return bf16_ws_bytes<32, 256>(0);
+  if (net.obs_dim == 64 && net.hidden == 512) return bf16_ws_bytes<64, 512>(0);
   return -1;
 }
 

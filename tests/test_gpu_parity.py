@@ -248,6 +248,33 @@ def test_rollout_parity_72b_full_size_sampled():
     _rollout_case(wl, 1024, iters=1, sample_envs=ids)
 
 
+def test_rollout_parity_stress_small():
+    """Stress network (D=64, H=512: weights streamed through a two-slot ring)
+    on 512 envs x 520 steps of the 380,000-sample 4-channel trace."""
+    _rollout_case(W.make_stress(n_envs=512, horizon=520), 520, iters=1, lam=0.4)
+
+
+def test_rollout_parity_stress_full_size_sampled():
+    """The full Stress workload (262,144 envs x 2,048 steps, 64-512-512 bf16);
+    the oracle replays a seeded sample of envs."""
+    wl = W.make_stress()
+    rng = np.random.default_rng(9)
+    ids = np.unique(np.concatenate([[0, 262143], rng.choice(262144, 6, replace=False)]))
+    _rollout_case(wl, 2048, iters=1, sample_envs=ids)
+
+
+def test_value_bf16_stress_ragged():
+    net = W.NetSpec(64, 512, 16, pe.PE_BF16)
+    params = W.init_params(net, seed=6, bias_scale=0.1)
+    for n in (1, 255, 3000):
+        obs = torch.randn(n, 64, generator=torch.Generator().manual_seed(n)).to(torch.bfloat16)
+        out = torch.empty(n, device="cuda")
+        pe.value(net, torch.from_numpy(params).cuda(), obs.cuda(), out)
+        pe.device_check()
+        _, ov = O.mlp_forward(net, params, obs.float().numpy())
+        assert bf16_ok(cpu(out), ov)
+
+
 def test_value_bf16_parity_ragged():
     net = W.NetSpec(32, 256, 16, pe.PE_BF16)
     params = W.init_params(net, seed=4, bias_scale=0.1)
