@@ -204,6 +204,11 @@ pe_status pe_gae(const float* reward, const float* value, const uint8_t* done,
  *  stats: [8] fp32 out: mean pg loss, value loss, entropy, approx KL,
  *         clip fraction, total loss; last pre-clip gradient norm; step count.
  *  workspace: >= pe_ppo_workspace_bytes(...) bytes of device memory.
+ * BF16 networks: the forward pass rounds the weights (not the biases) of the
+ * fp32 masters to bf16 once per minibatch; the head gradient and the hidden
+ * pre-activation gradients enter the backward products as bf16 with fp32
+ * accumulation; Adam updates the fp32 masters.  stats[7] = -1 if a bounded
+ * wait of the tensor-core forward timed out.
  * Errors: PE_EINVAL (unsupported network, sizes, small workspace), PE_ECUDA. */
 int64_t pe_ppo_workspace_bytes(const pe_net* net, const pe_ppo_config* cfg, int64_t n_samples);
 pe_status pe_ppo_update(const pe_net* net, float* params, float* adam_m, float* adam_v,

@@ -79,6 +79,10 @@ def lib():
                                             f64, f64, f64, vp, vp]),
             "or_ppo_update": (i64, [i32, i32, i32, vp, vp, vp, i64, i64, vp, vp, vp, vp, vp,
                                     vp, u64, u32, i64, vp]),
+            "or_ppo_minibatch_grad_ex": (f64, [i32, i32, i32, i32, vp, i64, vp, vp, vp, vp, vp,
+                                               f64, f64, f64, vp, vp]),
+            "or_ppo_update_ex": (i64, [i32, i32, i32, i32, vp, vp, vp, i64, i64, vp, vp, vp, vp,
+                                       vp, vp, u64, u32, i64, vp]),
             "or_fleet_windows": (i32, [i32, i32, vp, vp, i32, vp, i64, i32, vp, i32, i64,
                                        vp, vp]),
         }
@@ -217,12 +221,13 @@ def ppo_cfg(ppo) -> PPOCfg:
 
 def ppo_minibatch_grad(net, params64: np.ndarray, obs, act, logp_old, adv, ret, clip: float,
                        vf_coef: float, ent_coef: float, want_grad: bool = True):
+    """bf16 networks expect params64 to hold the bf16-rounded weights."""
     params64 = np.ascontiguousarray(params64, np.float64)
     M = len(act)
     grad = np.zeros_like(params64) if want_grad else None
     stats = np.zeros(5, np.float64)
-    loss = lib().or_ppo_minibatch_grad(
-        net.obs_dim, net.hidden, net.n_actions, _p(params64), M,
+    loss = lib().or_ppo_minibatch_grad_ex(
+        net.obs_dim, net.hidden, net.n_actions, int(net.dtype == 1), _p(params64), M,
         _p(np.ascontiguousarray(obs, np.float32)), _p(np.ascontiguousarray(act, np.uint8)),
         _p(np.ascontiguousarray(logp_old, np.float32)), _p(np.ascontiguousarray(adv, np.float32)),
         _p(np.ascontiguousarray(ret, np.float32)), clip, vf_coef, ent_coef, _p(grad), _p(stats))
@@ -238,8 +243,8 @@ def ppo_update(net, ppo, params, adam_m, adam_v, adam_t: int, obs, act, logp_old
     N = int(np.asarray(act).size)
     stats = np.zeros(8, np.float64)
     cfg = ppo_cfg(ppo)
-    t = lib().or_ppo_update(
-        net.obs_dim, net.hidden, net.n_actions, _p(P), _p(m), _p(v), adam_t, N,
+    t = lib().or_ppo_update_ex(
+        net.obs_dim, net.hidden, net.n_actions, int(net.dtype == 1), _p(P), _p(m), _p(v), adam_t, N,
         _p(np.ascontiguousarray(obs, np.float32)), _p(np.ascontiguousarray(act, np.uint8)),
         _p(np.ascontiguousarray(logp_old, np.float32)), _p(np.ascontiguousarray(adv, np.float32)),
         _p(np.ascontiguousarray(ret, np.float32)), C.byref(cfg), seed, iteration, max_steps,

@@ -543,10 +543,20 @@ void or_gae(int32_t T, int32_t E, const float* r, const float* v, const uint8_t*
  * entropy bonus.  Returns the minibatch loss; `grad` receives dLoss/dparams.
  * stats: [pg_loss, v_loss, entropy, approx_kl, clip_frac].
  * ---------------------------------------------------------------------- */
-double or_ppo_minibatch_grad(int32_t D, int32_t H, int32_t A, const double* P, int64_t M,
-                             const float* obs, const uint8_t* act, const float* logp_old,
-                             const float* adv, const float* ret, double clip, double vf_coef,
-                             double ent_coef, double* grad, double* stats) {
+/* bf16 networks (bf16 != 0): the forward pass rounds observations, weights
+ * and hidden activations to bf16 as in the rollout (P must hold the
+ * bf16-rounded weights), and the backward pass feeds every matrix product
+ * bf16 operands: the head gradient dz, and the layer gradients
+ * da2 = dh2 (1 - h2^2) and da1 = dh1 (1 - h1^2) are rounded to bf16 before
+ * they are used; the layer bias gradients sum the rounded values, the head
+ * bias gradient the unrounded dz. */
+static double rb(double x, int32_t bf16) { return bf16 ? or_bf16_round(x) : x; }
+
+double or_ppo_minibatch_grad_ex(int32_t D, int32_t H, int32_t A, int32_t bf16, const double* P,
+                                int64_t M, const float* obs, const uint8_t* act,
+                                const float* logp_old, const float* adv, const float* ret,
+                                double clip, double vf_coef, double ent_coef, double* grad,
+                                double* stats) {
   or_layout L = layout_of(D, H, A);
   double mean = 0.0, var = 0.0, sd = 0.0;
   for (int64_t i = 0; i < M; ++i) mean += (double)adv[i];
@@ -570,9 +580,9 @@ double or_ppo_minibatch_grad(int32_t D, int32_t H, int32_t A, const double* P, i
   double pg = 0.0, vl = 0.0, ent = 0.0, kl = 0.0, cf = 0.0;
   const double invM = 1.0 / (double)M;
   for (int64_t s = 0; s < M; ++s) {
-    obs_to_double(D, obs + s * D, x, 0);
-    policy_fwd(D, H, A, P, x, h1, h2, z, 0);
-    double V = value_fwd(D, H, A, P, x, g1, g2, 0);
+    obs_to_double(D, obs + s * D, x, bf16);
+    policy_fwd(D, H, A, P, x, h1, h2, z, bf16);
+    double V = value_fwd(D, H, A, P, x, g1, g2, bf16);
     double m = z[0];
     for (int32_t j = 1; j < A; ++j)
       if (z[j] > m) m = z[j];
@@ -603,15 +613,16 @@ double or_ppo_minibatch_grad(int32_t D, int32_t H, int32_t A, const double* P, i
       double p = exp(lp[j]);
       dz[j] = dlp * ((j == a ? 1.0 : 0.0) - p) + ent_coef * invM * p * (lp[j] + Hs);
     }
-    /* policy backward */
+    /* policy backward (bf16: dz enters the products rounded; db3 takes it unrounded) */
     for (int32_t j = 0; j < A; ++j) {
-      for (int32_t k = 0; k < H; ++k) grad[L.w3 + (int64_t)j * H + k] += dz[j] * h2[k];
+      const double dzb = rb(dz[j], bf16);
+      for (int32_t k = 0; k < H; ++k) grad[L.w3 + (int64_t)j * H + k] += dzb * h2[k];
       grad[L.b3 + j] += dz[j];
     }
     for (int32_t k = 0; k < H; ++k) {
       double acc = 0.0;
-      for (int32_t j = 0; j < A; ++j) acc += P[L.w3 + (int64_t)j * H + k] * dz[j];
-      da[k] = acc * (1.0 - h2[k] * h2[k]);
+      for (int32_t j = 0; j < A; ++j) acc += P[L.w3 + (int64_t)j * H + k] * rb(dz[j], bf16);
+      da[k] = rb(acc * (1.0 - h2[k] * h2[k]), bf16);
     }
     for (int32_t k = 0; k < H; ++k) {
       for (int32_t l = 0; l < H; ++l) grad[L.w2 + (int64_t)k * H + l] += da[k] * h1[l];
@@ -620,7 +631,7 @@ double or_ppo_minibatch_grad(int32_t D, int32_t H, int32_t A, const double* P, i
     for (int32_t l = 0; l < H; ++l) {
       double acc = 0.0;
       for (int32_t k = 0; k < H; ++k) acc += P[L.w2 + (int64_t)k * H + l] * da[k];
-      dh[l] = acc * (1.0 - h1[l] * h1[l]);
+      dh[l] = rb(acc * (1.0 - h1[l] * h1[l]), bf16);
     }
     for (int32_t l = 0; l < H; ++l) {
       for (int32_t d = 0; d < D; ++d) grad[L.w1 + (int64_t)l * D + d] += dh[l] * x[d];
@@ -628,9 +639,10 @@ double or_ppo_minibatch_grad(int32_t D, int32_t H, int32_t A, const double* P, i
     }
     /* value backward */
     const double dV = vf_coef * 2.0 * (V - (double)ret[s]) * invM;
+    const double dVb = rb(dV, bf16);
     for (int32_t k = 0; k < H; ++k) {
-      grad[L.v3 + k] += dV * g2[k];
-      da[k] = P[L.v3 + k] * dV * (1.0 - g2[k] * g2[k]);
+      grad[L.v3 + k] += dVb * g2[k];
+      da[k] = rb(P[L.v3 + k] * dVb * (1.0 - g2[k] * g2[k]), bf16);
     }
     grad[L.c3] += dV;
     for (int32_t k = 0; k < H; ++k) {
@@ -640,7 +652,7 @@ double or_ppo_minibatch_grad(int32_t D, int32_t H, int32_t A, const double* P, i
     for (int32_t l = 0; l < H; ++l) {
       double acc = 0.0;
       for (int32_t k = 0; k < H; ++k) acc += P[L.v2 + (int64_t)k * H + l] * da[k];
-      dh[l] = acc * (1.0 - g1[l] * g1[l]);
+      dh[l] = rb(acc * (1.0 - g1[l] * g1[l]), bf16);
     }
     for (int32_t l = 0; l < H; ++l) {
       for (int32_t d = 0; d < D; ++d) grad[L.v1 + (int64_t)l * D + d] += dh[l] * x[d];
@@ -658,18 +670,29 @@ double or_ppo_minibatch_grad(int32_t D, int32_t H, int32_t A, const double* P, i
   return pg * invM - ent_coef * ent * invM + vf_coef * vl * invM;
 }
 
+double or_ppo_minibatch_grad(int32_t D, int32_t H, int32_t A, const double* P, int64_t M,
+                             const float* obs, const uint8_t* act, const float* logp_old,
+                             const float* adv, const float* ret, double clip, double vf_coef,
+                             double ent_coef, double* grad, double* stats) {
+  return or_ppo_minibatch_grad_ex(D, H, A, 0, P, M, obs, act, logp_old, adv, ret, clip, vf_coef,
+                                  ent_coef, grad, stats);
+}
+
 /* PPO update: `epochs` passes over the N = T*E samples of one rollout, each
  * in a fresh Feistel order split into minibatches of `minibatch` (the last
  * one ragged); every minibatch: gradient, global-norm clip
  * (g *= max_norm / (|g| + 1e-6) when that is < 1), Adam (Kingma & Ba 2015,
  * Algorithm 1).  Returns the Adam step count after the update.
  * stats: [pg, v, entropy, kl, clip_frac, loss, last grad norm, steps]. */
-int64_t or_ppo_update(int32_t D, int32_t H, int32_t A, double* P, double* adam_m, double* adam_v,
-                      int64_t adam_t, int64_t N, const float* obs, const uint8_t* act,
-                      const float* logp_old, const float* adv, const float* ret,
-                      const or_ppo_cfg* cfg, uint64_t seed, uint32_t iteration,
-                      int64_t max_steps, double* stats) {
+int64_t or_ppo_update_ex(int32_t D, int32_t H, int32_t A, int32_t bf16, double* P, double* adam_m,
+                         double* adam_v, int64_t adam_t, int64_t N, const float* obs,
+                         const uint8_t* act, const float* logp_old, const float* adv,
+                         const float* ret, const or_ppo_cfg* cfg, uint64_t seed,
+                         uint32_t iteration, int64_t max_steps, double* stats) {
   or_layout L = layout_of(D, H, A);
+  /* the bf16 network computes with its fp32 master parameters rounded to bf16
+   * (weights only; biases stay fp32); the Adam step updates the masters */
+  double* Pc = bf16 ? (double*)malloc(sizeof(double) * (size_t)L.total) : P;
   const int64_t M = cfg->minibatch;
   const int64_t nmb = (N + M - 1) / M;
   double* g = (double*)malloc(sizeof(double) * (size_t)L.total);
@@ -696,8 +719,15 @@ int64_t or_ppo_update(int32_t D, int32_t H, int32_t A, double* P, double* adam_m
         br[j] = ret[idx];
       }
       double st[5];
-      double loss = or_ppo_minibatch_grad(D, H, A, P, cnt, bo, ba, bl, bv, br, cfg->clip,
-                                          cfg->vf_coef, cfg->ent_coef, g, st);
+      if (bf16) {
+        int64_t mats[6][2] = {{L.w1, (int64_t)H * D}, {L.w2, (int64_t)H * H}, {L.w3, (int64_t)A * H},
+                              {L.v1, (int64_t)H * D}, {L.v2, (int64_t)H * H}, {L.v3, (int64_t)H}};
+        for (int64_t i = 0; i < L.total; ++i) Pc[i] = (double)(float)P[i];
+        for (int mm = 0; mm < 6; ++mm)
+          for (int64_t i = 0; i < mats[mm][1]; ++i) Pc[mats[mm][0] + i] = or_bf16_round(Pc[mats[mm][0] + i]);
+      }
+      double loss = or_ppo_minibatch_grad_ex(D, H, A, bf16, Pc, cnt, bo, ba, bl, bv, br, cfg->clip,
+                                             cfg->vf_coef, cfg->ent_coef, g, st);
       double nrm = 0.0;
       for (int64_t i = 0; i < L.total; ++i) nrm += g[i] * g[i];
       nrm = sqrt(nrm);
@@ -726,7 +756,17 @@ done:
     stats[7] = (double)steps;
   }
   free(g); free(bo); free(ba); free(bl); free(bv); free(br);
+  if (bf16) free(Pc);
   return adam_t;
+}
+
+int64_t or_ppo_update(int32_t D, int32_t H, int32_t A, double* P, double* adam_m, double* adam_v,
+                      int64_t adam_t, int64_t N, const float* obs, const uint8_t* act,
+                      const float* logp_old, const float* adv, const float* ret,
+                      const or_ppo_cfg* cfg, uint64_t seed, uint32_t iteration,
+                      int64_t max_steps, double* stats) {
+  return or_ppo_update_ex(D, H, A, 0, P, adam_m, adam_v, adam_t, N, obs, act, logp_old, adv, ret,
+                          cfg, seed, iteration, max_steps, stats);
 }
 
 /* ------------------------------------------------------------------------

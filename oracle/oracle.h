@@ -91,6 +91,16 @@ double or_ppo_minibatch_grad(int32_t D, int32_t H, int32_t A, const double* para
                              const float* obs, const uint8_t* act, const float* logp_old,
                              const float* adv, const float* ret, double clip, double vf_coef,
                              double ent_coef, double* grad, double* stats);
+double or_ppo_minibatch_grad_ex(int32_t D, int32_t H, int32_t A, int32_t bf16, const double* params,
+                                int64_t M, const float* obs, const uint8_t* act,
+                                const float* logp_old, const float* adv, const float* ret,
+                                double clip, double vf_coef, double ent_coef, double* grad,
+                                double* stats);
+int64_t or_ppo_update_ex(int32_t D, int32_t H, int32_t A, int32_t bf16, double* params,
+                         double* adam_m, double* adam_v, int64_t adam_t, int64_t N,
+                         const float* obs, const uint8_t* act, const float* logp_old,
+                         const float* adv, const float* ret, const or_ppo_cfg* cfg, uint64_t seed,
+                         uint32_t iteration, int64_t max_steps, double* stats);
 int64_t or_ppo_update(int32_t D, int32_t H, int32_t A, double* params, double* adam_m,
                       double* adam_v, int64_t adam_t, int64_t N, const float* obs,
                       const uint8_t* act, const float* logp_old, const float* adv,

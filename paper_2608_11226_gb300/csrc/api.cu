@@ -83,6 +83,11 @@ pe_status ppo_update_f32(const pe_net& net, float* params, float* m, float* v, i
                          const float* obs, const uint8_t* act, const float* logp_old,
                          const float* adv, const float* ret, int64_t N, const pe_ppo_config& cfg,
                          float* stats, void* ws, cudaStream_t st);
+int64_t ppo_ws_bytes_bf16(const pe_net& net, const pe_ppo_config& cfg, int64_t N);
+pe_status ppo_update_bf16(const pe_net& net, float* params, float* m, float* v, int64_t adam_t,
+                          const void* obs, const uint8_t* act, const float* logp_old, const float* adv,
+                          const float* ret, int64_t N, const pe_ppo_config& cfg, float* stats, void* ws,
+                          cudaStream_t st);
 int64_t fleet_ws_bytes(int J, int L, int H);
 int64_t rollout_bf16_ws_bytes(const pe_net& net, int64_t E);
 pe_status rollout_bf16(const EnvDev& env, const pe_net& net, const float* params, int T, uint32_t it,
@@ -450,13 +455,16 @@ static pe_status check_ppo(const pe_net* net, const pe_ppo_config* cfg, int64_t 
   if (cfg->epochs < 1 || cfg->epochs > 16) return fail(PE_EINVAL, "epochs must be in [1, 16]");
   if (cfg->minibatch < 1) return fail(PE_EINVAL, "minibatch must be >= 1");
   if (n < 1 || n > (int64_t)INT32_MAX) return fail(PE_EINVAL, "n_samples must be in [1, 2^31)");
-  if (net->dtype != PE_F32) return fail(PE_EINVAL, "bf16 networks are not supported by pe_ppo_update in this build");
   return PE_OK;
+}
+
+static int64_t ppo_ws_bytes(const pe_net& net, const pe_ppo_config& cfg, int64_t n) {
+  return net.dtype == PE_BF16 ? ppo_ws_bytes_bf16(net, cfg, n) : ppo_ws_bytes_f32(net, cfg, n);
 }
 
 int64_t pe_ppo_workspace_bytes(const pe_net* net, const pe_ppo_config* cfg, int64_t n_samples) {
   if (check_ppo(net, cfg, n_samples) != PE_OK) return -1;
-  return ppo_ws_bytes_f32(*net, *cfg, n_samples);
+  return ppo_ws_bytes(*net, *cfg, n_samples);
 }
 
 pe_status pe_ppo_update(const pe_net* net, float* params, float* adam_m, float* adam_v,
@@ -470,8 +478,12 @@ pe_status pe_ppo_update(const pe_net* net, float* params, float* adam_m, float* 
   if (!params || !adam_m || !adam_v || !obs || !act || !logp_old || !adv || !ret || !stats || !workspace)
     return fail(PE_EINVAL, "null argument");
   if (adam_t < 0) return fail(PE_EINVAL, "adam_t must be >= 0");
-  const int64_t need = ppo_ws_bytes_f32(*net, *cfg, n_samples);
+  const int64_t need = ppo_ws_bytes(*net, *cfg, n_samples);
+  if (need < 0) return fail(PE_EINVAL, "unsupported PPO network");
   if (workspace_bytes < need) return fail(PE_EINVAL, "workspace too small (%lld < %lld bytes)", (long long)workspace_bytes, (long long)need);
+  if (net->dtype == PE_BF16)
+    return ppo_update_bf16(*net, params, adam_m, adam_v, adam_t, obs, act, logp_old, adv, ret, n_samples, *cfg,
+                           stats, workspace, reinterpret_cast<cudaStream_t>(stream));
   return ppo_update_f32(*net, params, adam_m, adam_v, adam_t, reinterpret_cast<const float*>(obs),
                         act, logp_old, adv, ret, n_samples, *cfg, stats, workspace,
                         reinterpret_cast<cudaStream_t>(stream));

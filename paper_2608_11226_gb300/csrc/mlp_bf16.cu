@@ -26,6 +26,16 @@ namespace pe {
 // set when a bounded tensor-core wait gives up; read and cleared by pe_device_check
 __device__ int32_t g_tc_error = 0;
 
+// optional extras of a forward pass used by the PPO update: rows gathered
+// through an index array, and the bf16 input and hidden activations saved
+// row-major ([n][D], [n][H]) for the backward pass
+struct MlpSave {
+  const uint32_t* gather;  // row r of the tile reads obs row gather[r] (NULL: row r)
+  __nv_bfloat16* x;        // [n][D] or NULL
+  __nv_bfloat16* h1;       // [n][H] or NULL
+  __nv_bfloat16* h2;       // [n][H] or NULL
+};
+
 constexpr int kTcRows = 128;     // rows (envs / samples) per tile, the MMA M
 constexpr int kTcThreads = 512;  // 16 warps: 4 TMEM lane quadrants x 4 column slices
 constexpr int kHeadN = 16;       // head width (logits or value padded to 16)
@@ -107,17 +117,23 @@ __device__ __forceinline__ void epi_compute(uint32_t tmem, int col0, const float
 }
 
 template <int H>
-__device__ __forceinline__ void epi_store(const uint32_t (&pk)[H / 8], uint8_t* act) {
+__device__ __forceinline__ void epi_store(const uint32_t (&pk)[H / 8], uint8_t* act,
+                                          __nv_bfloat16* gsave, int64_t r0, int nr) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int quad = warp & 3, slice = warp >> 2;
   const int row = quad * 32 + lane;
 #pragma unroll
   for (int j = 0; j < H / 64; ++j) {
     const int c = slice * (H / 4) + j * 16;
-    *reinterpret_cast<uint4*>(act + tc::swz_offset<128>(row, c, kTcRows)) =
-        make_uint4(pk[j * 8 + 0], pk[j * 8 + 1], pk[j * 8 + 2], pk[j * 8 + 3]);
-    *reinterpret_cast<uint4*>(act + tc::swz_offset<128>(row, c + 8, kTcRows)) =
-        make_uint4(pk[j * 8 + 4], pk[j * 8 + 5], pk[j * 8 + 6], pk[j * 8 + 7]);
+    const uint4 lo = make_uint4(pk[j * 8 + 0], pk[j * 8 + 1], pk[j * 8 + 2], pk[j * 8 + 3]);
+    const uint4 hi = make_uint4(pk[j * 8 + 4], pk[j * 8 + 5], pk[j * 8 + 6], pk[j * 8 + 7]);
+    *reinterpret_cast<uint4*>(act + tc::swz_offset<128>(row, c, kTcRows)) = lo;
+    *reinterpret_cast<uint4*>(act + tc::swz_offset<128>(row, c + 8, kTcRows)) = hi;
+    if (gsave && row < nr) {
+      uint4* g = reinterpret_cast<uint4*>(gsave + (r0 + row) * H + c);
+      g[0] = lo;
+      g[1] = hi;
+    }
   }
 }
 
@@ -128,7 +144,8 @@ template <int D, int H>
 __global__ void __launch_bounds__(kTcThreads, 1)
     mlp_bf16_kernel(const uint8_t* __restrict__ img, const float* __restrict__ params, int A,
                     int value_net, const __nv_bfloat16* __restrict__ obs, int64_t n,
-                    float* __restrict__ out, int out_stride, int nout, int32_t* __restrict__ err) {
+                    float* __restrict__ out, int out_stride, int nout, int32_t* __restrict__ err,
+                    MlpSave save) {
   using I = Img<D, H>;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   // align the dynamic shared window to 1024 B for the swizzle atoms
@@ -174,7 +191,11 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     for (int i = tid; i < kTcRows * CPR; i += blockDim.x) {
       const int r = i / CPR, c = i % CPR;
       uint4 v = make_uint4(0, 0, 0, 0);
-      if (r < nr) v = __ldg(reinterpret_cast<const uint4*>(obs + (r0 + r) * D) + c);
+      if (r < nr) {
+        const int64_t src = save.gather ? (int64_t)__ldg(save.gather + r0 + r) : r0 + r;
+        v = __ldg(reinterpret_cast<const uint4*>(obs + src * D) + c);
+        if (save.x) *(reinterpret_cast<uint4*>(save.x + (r0 + r) * D) + c) = v;
+      }
       *reinterpret_cast<uint4*>(s.act + tc::swz_offset<I::RB1>(r, c * 8, kTcRows)) = v;
     }
     tc::fence_async_smem();
@@ -209,7 +230,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     if (!tc::mbar_wait(&s.bar_hi, phase_hi)) atomicExch(&s.err, 1);
     tc::fence_after();
     if (hi_half) epi_compute<H>(tmem, 0, s.b1, pk);
-    epi_store<H>(pk, s.act);
+    epi_store<H>(pk, s.act, save.h1, r0, nr);
     phase ^= 1;
     phase_hi ^= 1;
     tc::fence_before();
@@ -240,7 +261,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     if (!tc::mbar_wait(&s.bar_hi, phase_hi)) atomicExch(&s.err, 1);
     tc::fence_after();
     if (hi_half) epi_compute<H>(tmem, 256, s.b2, pk);
-    epi_store<H>(pk, s.act);
+    epi_store<H>(pk, s.act, save.h2, r0, nr);
     phase ^= 1;
     phase_hi ^= 1;
     tc::fence_before();
@@ -358,7 +379,8 @@ template <int D, int H>
 __global__ void __launch_bounds__(kStreamThreads, 1)
     mlp_bf16_stream_kernel(const uint8_t* __restrict__ img, const float* __restrict__ params, int A,
                            int value_net, const __nv_bfloat16* __restrict__ obs, int64_t n,
-                           float* __restrict__ out, int out_stride, int nout, int32_t* __restrict__ err) {
+                           float* __restrict__ out, int out_stride, int nout, int32_t* __restrict__ err,
+                           MlpSave save) {
   using I = ImgS<D, H>;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
@@ -423,7 +445,11 @@ __global__ void __launch_bounds__(kStreamThreads, 1)
       for (int i = tid; i < kTcRows * (D / 8); i += kComputeThreads) {
         const int r = i / (D / 8), c = i % (D / 8);
         uint4 v = make_uint4(0, 0, 0, 0);
-        if (r < nr) v = __ldg(reinterpret_cast<const uint4*>(obs + (rbase + r) * D) + c);
+        if (r < nr) {
+          const int64_t src = save.gather ? (int64_t)__ldg(save.gather + rbase + r) : rbase + r;
+          v = __ldg(reinterpret_cast<const uint4*>(obs + src * D) + c);
+          if (save.x) *(reinterpret_cast<uint4*>(save.x + (rbase + r) * D) + c) = v;
+        }
         *reinterpret_cast<uint4*>(s.act + tc::swz_offset<128>(r, c * 8, kTcRows)) = v;
       }
       tc::fence_async_smem();
@@ -464,6 +490,11 @@ __global__ void __launch_bounds__(kStreamThreads, 1)
           p[i] = tc::pack_bf16(tanhf(v[2 * i] + s.b1[c + 2 * i]), tanhf(v[2 * i + 1] + s.b1[c + 2 * i + 1]));
         *reinterpret_cast<uint4*>(s.act + tc::swz_offset<128>(row, c, kTcRows)) = make_uint4(p[0], p[1], p[2], p[3]);
         *reinterpret_cast<uint4*>(s.act + tc::swz_offset<128>(row, c + 8, kTcRows)) = make_uint4(p[4], p[5], p[6], p[7]);
+        if (save.h1 && row < nr) {
+          uint4* g = reinterpret_cast<uint4*>(save.h1 + (rbase + row) * H + c);
+          g[0] = make_uint4(p[0], p[1], p[2], p[3]);
+          g[1] = make_uint4(p[4], p[5], p[6], p[7]);
+        }
       }
       tc::fence_before();
       tc::fence_async_smem();
@@ -495,6 +526,11 @@ __global__ void __launch_bounds__(kStreamThreads, 1)
           p[i] = tc::pack_bf16(tanhf(v[2 * i] + s.b2[c + 2 * i]), tanhf(v[2 * i + 1] + s.b2[c + 2 * i + 1]));
         *reinterpret_cast<uint4*>(s.act + tc::swz_offset<128>(row, c, kTcRows)) = make_uint4(p[0], p[1], p[2], p[3]);
         *reinterpret_cast<uint4*>(s.act + tc::swz_offset<128>(row, c + 8, kTcRows)) = make_uint4(p[4], p[5], p[6], p[7]);
+        if (save.h2 && row < nr) {
+          uint4* g = reinterpret_cast<uint4*>(save.h2 + (rbase + row) * H + c);
+          g[0] = make_uint4(p[0], p[1], p[2], p[3]);
+          g[1] = make_uint4(p[4], p[5], p[6], p[7]);
+        }
       }
       tc::fence_before();
       tc::fence_async_smem();
@@ -628,7 +664,7 @@ static int64_t bf16_ws_bytes(int64_t E) {
 template <int D, int H>
 static pe_status launch_mlp(const uint8_t* img, const float* params, int A, int value_net,
                             const void* obs, int64_t n, float* out, int out_stride, int nout,
-                            int32_t* err, cudaStream_t st, int prof_kind) {
+                            int32_t* err, cudaStream_t st, int prof_kind, MlpSave save = MlpSave{}) {
   if (n <= 0) return PE_OK;
   int dev = 0, sms = 0;
   PE_TRY_CUDA(cudaGetDevice(&dev));
@@ -641,13 +677,13 @@ static pe_status launch_mlp(const uint8_t* img, const float* params, int A, int 
     const int bytes = (int)sizeof(MlpStreamSmem<D, H>) + 1024;
     PE_TRY_CUDA(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes));
     ProfScope ps(prof_kind, st);
-    kern<<<grid, kStreamThreads, bytes, st>>>(img, params, A, value_net, o, n, out, out_stride, nout, err);
+    kern<<<grid, kStreamThreads, bytes, st>>>(img, params, A, value_net, o, n, out, out_stride, nout, err, save);
   } else {
     auto kern = mlp_bf16_kernel<D, H>;
     const int bytes = (int)sizeof(MlpBf16Smem<D, H>) + 1024;
     PE_TRY_CUDA(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes));
     ProfScope ps(prof_kind, st);
-    kern<<<grid, kTcThreads, bytes, st>>>(img, params, A, value_net, o, n, out, out_stride, nout, err);
+    kern<<<grid, kTcThreads, bytes, st>>>(img, params, A, value_net, o, n, out, out_stride, nout, err, save);
   }
   PE_CHECK_LAUNCH("mlp_bf16_kernel");
   return PE_OK;
@@ -747,6 +783,35 @@ pe_status value_bf16(const pe_net& net, const float* params, const void* obs, in
   if (net.obs_dim == 32 && net.hidden == 256) return value_bf16_impl<32, 256>(net, params, obs, n, value, ws, st);
   if (net.obs_dim == 64 && net.hidden == 512) return value_bf16_impl<64, 512>(net, params, obs, n, value, ws, st);
   return fail(PE_EINVAL, "unsupported bf16 value network (D=%d H=%d)", net.obs_dim, net.hidden);
+}
+
+// forward of one bf16 network over gathered minibatch rows, saving x, h1 and
+// h2 (used by the bf16 PPO update); img must hold the network's weight image
+int64_t bf16_image_bytes(const pe_net& net) {
+  if (net.obs_dim == 32 && net.hidden == 256) return NetKind<32, 256>::kImgPad;
+  if (net.obs_dim == 64 && net.hidden == 512) return NetKind<64, 512>::kImgPad;
+  return -1;
+}
+
+pe_status bf16_make_images(const pe_net& net, const float* params, uint8_t* two_images, cudaStream_t st) {
+  if (net.obs_dim == 32 && net.hidden == 256) return make_images<32, 256>(params, net.n_actions, two_images, st, true);
+  if (net.obs_dim == 64 && net.hidden == 512) return make_images<64, 512>(params, net.n_actions, two_images, st, true);
+  return fail(PE_EINVAL, "unsupported bf16 network");
+}
+
+pe_status bf16_forward_save(const pe_net& net, const uint8_t* img, const float* params, int value_net,
+                            const void* obs, const uint32_t* gather, int64_t n, float* out, int out_stride,
+                            __nv_bfloat16* x, __nv_bfloat16* h1, __nv_bfloat16* h2, int32_t* err,
+                            cudaStream_t st) {
+  const MlpSave sv{gather, x, h1, h2};
+  const int nout = value_net ? 1 : net.n_actions;
+  if (net.obs_dim == 32 && net.hidden == 256)
+    return launch_mlp<32, 256>(img, params, net.n_actions, value_net, obs, n, out, out_stride, nout, err, st,
+                               PE_PROF_PPO_GRAD, sv);
+  if (net.obs_dim == 64 && net.hidden == 512)
+    return launch_mlp<64, 512>(img, params, net.n_actions, value_net, obs, n, out, out_stride, nout, err, st,
+                               PE_PROF_PPO_GRAD, sv);
+  return fail(PE_EINVAL, "unsupported bf16 network");
 }
 
 int64_t value_bf16_ws_bytes(const pe_net& net) {

@@ -734,6 +734,20 @@ static PpoPlan ppo_plan(const pe_net& net, const pe_ppo_config& cfg, int64_t N) 
   return p;
 }
 
+// advantage statistics of every (epoch, minibatch), shared with the bf16 update
+pe_status launch_advstats(const float* adv, int64_t N, int M, int nmb, int epochs, uint64_t seed,
+                          uint32_t iteration, float2* out, cudaStream_t st) {
+  if (epochs < 1 || epochs > kPpoMaxEpochs) return fail(PE_EINVAL, "epochs must be in [1, %d]", kPpoMaxEpochs);
+  FeistelSet perms{};
+  for (int ep = 0; ep < epochs; ++ep) perms.f[ep] = make_feistel((uint64_t)N, seed, ep, iteration);
+  {
+    ProfScope ps(PE_PROF_PPO_OTHER, st);
+    ppo_advstats_kernel<<<dim3(nmb, epochs), 256, 0, st>>>(adv, N, M, nmb, perms, out);
+  }
+  PE_CHECK_LAUNCH("ppo_advstats_kernel");
+  return PE_OK;
+}
+
 int64_t ppo_ws_bytes_f32(const pe_net& net, const pe_ppo_config& cfg, int64_t N) {
   return ppo_plan(net, cfg, N).total;
 }

@@ -346,7 +346,7 @@ def _run_ppo(wl, ppo, params, buf, adv, ret, iteration=0):
 def _oracle_ppo(wl, ppo, params, buf, adv, ret, iteration=0, max_steps=-1):
     P = params.size
     return O.ppo_update(wl.net, ppo, params, np.zeros(P), np.zeros(P), 0,
-                        cpu(buf["obs"]).reshape(-1, wl.net.obs_dim), cpu(buf["act"]).ravel(),
+                        cpu(buf["obs"].float()).reshape(-1, wl.net.obs_dim), cpu(buf["act"]).ravel(),
                         cpu(buf["logp"]).ravel(), cpu(adv).ravel(), cpu(ret).ravel(), 7, iteration,
                         max_steps)
 
@@ -404,3 +404,34 @@ def test_ppo_7b_first_steps():
     gp, gm, gv, gs = _run_ppo(wl, ppo, params, buf, adv, ret)
     P, m, v, t, st = _oracle_ppo(wl, ppo, params, buf, adv, ret)
     assert rel_err(gm, m) <= TOL and rel_err(gp, P) <= TOL
+
+
+# ------------------------------------------------------------------ bf16 PPO
+@pytest.mark.parametrize("preset,E,T", [("72b", 64, 64), ("stress", 32, 64)])
+def test_ppo_bf16_single_step(preset, E, T):
+    """One minibatch over all N = T*E samples of a bf16 network: tensor-core
+    forward over the permuted rows, cuBLASLt backward products, own loss,
+    reduction and Adam.  Adam's first moment after one step is 0.1 x the
+    clipped gradient."""
+    wl = W.make_72b(n_envs=E) if preset == "72b" else W.make_stress(n_envs=E, horizon=T)
+    params, buf, adv, ret = _ppo_inputs(wl, T, seed=2)
+    ppo = W.PPOSpec(epochs=1, minibatch=T * E, ent_coef=0.01)
+    gp, gm, gv, gs = _run_ppo(wl, ppo, params, buf, adv, ret, iteration=1)
+    P, m, v, t, st = _oracle_ppo(wl, ppo, params, buf, adv, ret, iteration=1)
+    assert t == 1 and gs[7] == 1
+    assert bf16_ok(gm, m), (np.abs(gm - m).max() / np.abs(m).max())
+    for k in (1, 2, 6):   # value loss, entropy, grad norm
+        assert abs(gs[k] - st[k]) <= 2e-2 * max(abs(st[k]), 1e-3), (k, gs[k], st[k])
+
+
+def test_ppo_bf16_ragged_epochs_72b():
+    """2 epochs x 3 minibatches (1500, 1500, 1096) on the 72B network."""
+    wl = W.make_72b(n_envs=64)
+    params, buf, adv, ret = _ppo_inputs(wl, 64, seed=4)
+    ppo = W.PPOSpec(epochs=2, minibatch=1500, ent_coef=0.01)
+    gp, gm, gv, gs = _run_ppo(wl, ppo, params, buf, adv, ret, iteration=3)
+    P, m, v, t, st = _oracle_ppo(wl, ppo, params, buf, adv, ret, iteration=3)
+    assert t == 6 and gs[7] == 6
+    dp, dref = gp - params, P - params
+    assert np.linalg.norm(dp - dref) <= 0.1 * np.linalg.norm(dref), np.linalg.norm(dp - dref) / np.linalg.norm(dref)
+    assert abs(gs[1] - st[1]) <= 2e-2 * abs(st[1])

@@ -319,6 +319,104 @@ def test_ppo_gradient_matches_autograd_and_finite_differences():
         assert abs(fd - grad[k]) <= 1e-6 * max(1.0, abs(grad[k])), k
 
 
+def _rb(t):
+    return t.float().to(torch.bfloat16).double()
+
+
+class _RoundFwd(torch.autograd.Function):
+    """bf16 rounding in the forward pass, identity in the backward pass."""
+
+    @staticmethod
+    def forward(ctx, t):
+        return _rb(t)
+
+    @staticmethod
+    def backward(ctx, g):
+        return g
+
+
+class _RoundBwd(torch.autograd.Function):
+    """Identity in the forward pass, bf16 rounding of the incoming gradient."""
+
+    @staticmethod
+    def forward(ctx, t):
+        return t.clone()
+
+    @staticmethod
+    def backward(ctx, g):
+        return _rb(g)
+
+
+class _TanhRound(torch.autograd.Function):
+    """y = bf16(tanh(a)); the derivative uses the stored (rounded) y."""
+
+    @staticmethod
+    def forward(ctx, a):
+        y = _rb(torch.tanh(a))
+        ctx.save_for_backward(y)
+        return y
+
+    @staticmethod
+    def backward(ctx, g):
+        (y,) = ctx.saved_tensors
+        return g * (1.0 - y * y)
+
+
+def _torch_ppo_loss_bf16(net, params, obs, act, lpo, adv, ret, clip, vf, ent):
+    """Autograd of the bf16 network: weights and inputs rounded on the way in,
+    tanh outputs stored rounded, and the gradients at the three product inputs
+    (head output, both pre-activations) rounded on the way back; the head bias
+    sees the unrounded head gradient."""
+    D, H, A = net.obs_dim, net.hidden, net.n_actions
+    p = torch.tensor(params, dtype=torch.float64, requires_grad=True)
+    sizes = [H * D, H, H * H, H, A * H, A, H * D, H, H * H, H, H, 1]
+    W1, b1, W2, b2, W3, b3, V1, c1, V2, c2, V3, c3 = torch.split(p, sizes)
+    x = _rb(torch.tensor(obs, dtype=torch.float64))
+
+    def fwd(Wa, ba, Wb, bb, Wc, bc, out):
+        h1 = _TanhRound.apply(_RoundBwd.apply(x @ _RoundFwd.apply(Wa.view(H, D)).T + ba))
+        h2 = _TanhRound.apply(_RoundBwd.apply(h1 @ _RoundFwd.apply(Wb.view(H, H)).T + bb))
+        return _RoundBwd.apply(h2 @ _RoundFwd.apply(Wc.view(out, H)).T) + bc
+
+    z = fwd(W1, b1, W2, b2, W3, b3, A)
+    V = fwd(V1, c1, V2, c2, V3, c3, 1)[:, 0]
+    logp_all = torch.log_softmax(z, -1)
+    lp = logp_all[torch.arange(len(act)), torch.tensor(act, dtype=torch.long)]
+    a = torch.tensor(adv, dtype=torch.float64)
+    a = (a - a.mean()) / (a.std() + 1e-8)
+    rho = torch.exp(lp - torch.tensor(lpo, dtype=torch.float64))
+    pg = -torch.min(rho * a, torch.clamp(rho, 1 - clip, 1 + clip) * a).mean()
+    vl = ((torch.tensor(ret, dtype=torch.float64) - V) ** 2).mean()
+    H_ = -(logp_all.exp() * logp_all).sum(-1).mean()
+    loss = pg + vf * vl - ent * H_
+    loss.backward()
+    return loss.item(), p.grad.numpy()
+
+
+def test_ppo_bf16_gradient_matches_autograd_with_rounding():
+    """bf16 networks: the oracle's hand-written backward equals autograd of
+    the network with bf16 rounding at the same points, and differs from the
+    unrounded-backward gradient by no more than bf16 rounding."""
+    net = W.NetSpec(6, 16, 4, 1)
+    params = W.init_params(net, seed=6, bias_scale=0.1).astype(np.float64)
+    batch = _ppo_batch(net, 48, seed=2)
+    # the minibatch gradient takes the weights already rounded (the update
+    # rounds its fp32 masters once per minibatch); biases stay unrounded
+    D, H, A = 6, 16, 4
+    sizes = [H * D, H, H * H, H, A * H, A, H * D, H, H * H, H, H, 1]
+    parts = np.split(params, np.cumsum(sizes)[:-1])
+    params = np.concatenate([_rb(torch.tensor(q)).numpy() if i % 2 == 0 else q for i, q in enumerate(parts)])
+    loss, grad, _ = O.ppo_minibatch_grad(net, params, *batch, 0.2, 0.5, 0.01)
+    tl, tg = _torch_ppo_loss_bf16(net, params, *batch, 0.2, 0.5, 0.01)
+    assert loss == pytest.approx(tl, rel=1e-12)
+    assert np.allclose(grad, tg, rtol=1e-9, atol=1e-12)
+    # the forward of the bf16 network differs from the fp64 one (rounding is applied)
+    l64, g64, _ = O.ppo_minibatch_grad(W.NetSpec(6, 16, 4, 0), params, *batch, 0.2, 0.5, 0.01)
+    assert 1e-6 < abs(loss - l64) / abs(l64) < 5e-2
+    d = np.abs(grad - g64).max() / np.abs(g64).max()
+    assert 1e-5 < d < 5e-2
+
+
 def test_ppo_first_minibatch_ratio_one_policy_loss_zero():
     """With logp_old = logp under the current params, rho = 1 and the
     clipped surrogate is -mean(normalised advantage) = 0."""
