@@ -53,6 +53,10 @@ def parse():
     ap.add_argument("--r72b-steps", type=int, default=2, help="timed 72B rollouts (0: skip)")
     ap.add_argument("--r72b-envs", type=int, default=65536)
     ap.add_argument("--r72b-horizon", type=int, default=1024)
+    ap.add_argument("--r72b-ppo-minibatches", type=int, default=16,
+                    help="72B PPO minibatch steps of 65,536 samples timed (0: skip)")
+    ap.add_argument("--gae-large", type=int, nargs=2, default=[2048, 262144], metavar=("T", "E"),
+                    help="GAE roofline size (Stress: 2048 x 262144); T=0 skips it")
     return ap.parse_args()
 
 
@@ -286,6 +290,7 @@ def run_ours(args, world, rank, local):
     # ---- fleet accounting
     fleet = run_fleet(args, world) if args.fleet_n > 0 else None
     r72b = run_72b(args, world, peaks) if args.r72b_steps > 0 else None
+    gae_large = run_gae_large(args, world, peaks) if args.gae_large[0] > 0 else None
 
     out = {"metric": METRIC, "value": value, "unit": "env-steps/s", "n_gpus": world,
            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_step,
@@ -298,6 +303,7 @@ def run_ours(args, world, rank, local):
                       "l2": "flushed between timed steps (256 MB write)"},
            "roofline": roof, "gae_roofline": gae_roof, "kernels": kernels,
            "gpu_launches": launches, "clocks": clk, "e2e": e2e, "fleet": fleet, "rollout_72b": r72b,
+           "gae_roofline_stress_size": gae_large,
            "ppo_stats_last": [float(x) for x in tr.stats.cpu()]}
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         out["cpu_baseline"] = cpu_baseline(args.cpu_envs)
@@ -405,6 +411,7 @@ def run_72b(args, world, peaks):
     gms, gn = pe.profile_read(pe.PE_PROF_GAE)
     gae_gbs = 17.0 * T * E / (gms / gn / 1e3) / 1e9 if gn else None
     hbm = float(peaks.get("hbm_gbs", 6800.0))
+    ppo72 = run_72b_ppo(args, world, peaks, wl, buf, adv, ret) if args.r72b_ppo_minibatches > 0 else None
     del adv, ret
     pms, pn = prof["mlp_policy_tc"]
     vms, vn = prof["mlp_value_tc"]
@@ -429,7 +436,95 @@ def run_72b(args, world, peaks):
             "roofline_gae": {"kernel": f"gae_kernel ({T} x {E})", "bound": "hbm", "achieved": gae_gbs,
                              "peak": hbm, "unit": "GB/s", "frac": gae_gbs / hbm if gae_gbs else None,
                              "avg_launch_ms": gms / gn if gn else None,
-                             "traffic": load_traffic("gae_kernel")}}
+                             "traffic": load_traffic("gae_kernel")},
+            "ppo_update": ppo72}
+
+
+def run_72b_ppo(args, world, peaks, wl, buf, adv, ret):
+    """bf16 PPO update of the 72B networks on the first K x 65,536 samples of
+    the 72B rollout (one epoch, K minibatch steps): tensor-core forward over
+    the permuted rows, cuBLASLt backward products, own loss/reduction/Adam.
+    Reports samples/s and the whole step's bf16 FLOP rate against the
+    measured sustained bf16 peak."""
+    from paper_2608_11226_gb300 import pe
+    from paper_2608_11226_gb300 import workloads as W
+    net = wl.net
+    mb = 65536
+    n = min(args.r72b_ppo_minibatches * mb, buf["act"].numel())
+    ppo = W.PPOSpec(epochs=1, minibatch=mb, ent_coef=0.01)
+    D = net.obs_dim
+    obs = buf["obs"].view(-1, D)[:n]
+    act = buf["act"].view(-1)[:n]
+    lpo = buf["logp"].view(-1)[:n]
+    a_ = adv.view(-1)[:n]
+    r_ = ret.view(-1)[:n]
+    params = torch.from_numpy(W.init_params(net, seed=0)).cuda()
+    m = torch.zeros_like(params)
+    v = torch.zeros_like(params)
+    stats = torch.zeros(8, device="cuda")
+    ws = pe.alloc_workspace(pe.ppo_workspace_bytes(net, ppo, n))
+    pe.ppo_update(net, ppo, params, m, v, 0, obs, act, lpo, a_, r_, stats, ws, seed=7, iteration=0)
+    torch.cuda.synchronize()
+    for k in range(pe.PE_PROF_KINDS):
+        pe.profile_read(k)
+    barrier(world)
+    pe.profile_enable(True)
+    stream = torch.cuda.current_stream()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    pe.ppo_update(net, ppo, params, m, v, 1, obs, act, lpo, a_, r_, stats, ws, seed=7, iteration=1)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    pe.profile_enable(False)
+    ms = max_over_ranks(e0.elapsed_time(e1), world)
+    prof = {pe.profile_kind_name(k): pe.profile_read(k) for k in range(pe.PE_PROF_KINDS)}
+    steps = (n + mb - 1) // mb
+    fl = ppo_flops_per_sample(net.obs_dim, net.hidden, net.n_actions) * n
+    peak = float(peaks.get("bf16_tflops_sustained", 1728.9))
+    ach = fl / (ms / 1e3) / 1e12
+    st = [float(x) for x in stats.cpu()]
+    del ws
+    return {"metric": "72B PPO update samples/s", "value": n * world / (ms / 1e3), "unit": "samples/s",
+            "ms_per_minibatch_step": ms / steps, "minibatch": mb, "steps": steps,
+            "kernels": {k: {"ms_per_step": v_[0] / steps, "launches_per_step": v_[1] / steps}
+                        for k, v_ in prof.items() if v_[1]},
+            "roofline": {"kernel": "bf16 PPO minibatch step (all kernels)", "bound": "tensor",
+                         "achieved": ach, "peak": peak, "unit": "TFLOP/s", "frac": ach / peak,
+                         "flop_per_sample": ppo_flops_per_sample(net.obs_dim, net.hidden, net.n_actions)},
+            "stats": st}
+
+
+def run_gae_large(args, world, peaks):
+    """GAE alone at the Stress size (2,048 x 262,144 env-steps, 9.1 GB of
+    algorithmic traffic), on seeded device-resident inputs."""
+    from paper_2608_11226_gb300 import pe
+    T, E = args.gae_large
+    g = torch.Generator(device="cuda").manual_seed(0)
+    r = torch.randn(T, E, device="cuda", generator=g)
+    v = torch.randn(T, E, device="cuda", generator=g)
+    d = (torch.rand(T, E, device="cuda", generator=g) < 0.002).to(torch.uint8)
+    lv = torch.randn(E, device="cuda", generator=g)
+    adv = torch.empty(T, E, device="cuda")
+    ret = torch.empty_like(adv)
+    pe.gae(r, v, d, lv, 0.99, 0.95, adv, ret)
+    torch.cuda.synchronize()
+    pe.profile_read(pe.PE_PROF_GAE)
+    barrier(world)
+    pe.profile_enable(True)
+    for _ in range(5):
+        pe.gae(r, v, d, lv, 0.99, 0.95, adv, ret)
+    torch.cuda.synchronize()
+    pe.profile_enable(False)
+    gms, gn = pe.profile_read(pe.PE_PROF_GAE)
+    ms = max_over_ranks(gms / gn, world)
+    gbs = 17.0 * T * E / (ms / 1e3) / 1e9
+    hbm = float(peaks.get("hbm_gbs", 6800.0))
+    del r, v, d, adv, ret
+    torch.cuda.empty_cache()
+    return {"kernel": f"gae_kernel ({T} x {E})", "bound": "hbm", "achieved": gbs, "peak": hbm,
+            "unit": "GB/s", "frac": gbs / hbm, "avg_launch_ms": ms,
+            "env_steps_per_s": T * E * world / (ms / 1e3), "traffic": load_traffic("gae_kernel")}
 
 
 # --------------------------------------------------------------------------- CPU oracle

@@ -169,7 +169,8 @@ int64_t pe_param_count(const pe_net* net);
  *  lambda: Lagrange multiplier of Eq. 6 (PE_REWARD_LAGRANGE only).
  *  workspace: >= pe_rollout_workspace_bytes(env, net) bytes of device memory
  *  (0 for fp32 networks: NULL is accepted).  BF16 networks (D=32, H=256 or
- *  D=64, H=512; A=16, 4 channels) run on the tcgen05 tensor cores.
+ *  D=64, H=512; A=16, 4 channels) run on the tcgen05 tensor cores; their
+ *  workspace must be 256-byte and buf->obs / obs_last 16-byte aligned.
  * Errors: PE_EINVAL (unsupported network, null buffer, horizon < 1, small
  * workspace), PE_ECUDA; a bounded tensor-core wait that gives up on the
  * device is reported by pe_device_check. */
@@ -179,7 +180,8 @@ pe_status pe_rollout(pe_env* env, const pe_net* net, const float* params, int32_
                      void* workspace, int64_t workspace_bytes, void* stream);
 
 /* Value network on n observations (fp32, or bf16 for a BF16 network).
- * workspace: >= pe_value_workspace_bytes(net) bytes (0 for fp32). */
+ * workspace: >= pe_value_workspace_bytes(net) bytes (0 for fp32); for a BF16
+ * network the workspace must be 256-byte and obs 16-byte aligned. */
 int64_t pe_value_workspace_bytes(const pe_net* net);
 pe_status pe_value(const pe_net* net, const float* params, const void* obs, int64_t n,
                    float* value, void* workspace, int64_t workspace_bytes, void* stream);
@@ -203,7 +205,8 @@ pe_status pe_gae(const float* reward, const float* value, const uint8_t* done,
  *  obs [n][D] (dtype of the net), act, logp_old, adv, ret: rollout/GAE buffers.
  *  stats: [8] fp32 out: mean pg loss, value loss, entropy, approx KL,
  *         clip fraction, total loss; last pre-clip gradient norm; step count.
- *  workspace: >= pe_ppo_workspace_bytes(...) bytes of device memory.
+ *  workspace: >= pe_ppo_workspace_bytes(...) bytes of device memory, 256-byte
+ *  aligned; obs 16-byte aligned (rows are read as 16-byte vectors).
  * BF16 networks: the forward pass rounds the weights (not the biases) of the
  * fp32 masters to bf16 once per minibatch; the head gradient and the hidden
  * pre-activation gradients enter the backward products as bf16 with fp32

@@ -375,6 +375,8 @@ int64_t pe_rollout_workspace_bytes(const pe_env* env, const pe_net* net) {
   return rollout_bf16_ws_bytes(*net, env->dev.E);
 }
 
+static bool misaligned(const void* p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) & (a - 1)) != 0; }
+
 pe_status pe_rollout(pe_env* env, const pe_net* net, const float* params, int32_t horizon,
                      uint32_t iteration, float lambda, int32_t flags, const pe_rollout_buf* buf,
                      void* workspace, int64_t workspace_bytes, void* stream) {
@@ -405,6 +407,8 @@ pe_status pe_rollout(pe_env* env, const pe_net* net, const float* params, int32_
   if (need < 0) return fail(PE_EINVAL, "unsupported bf16 network (D=%d H=%d)", net->obs_dim, net->hidden);
   if (!workspace || workspace_bytes < need)
     return fail(PE_EINVAL, "workspace too small (%lld < %lld bytes)", (long long)workspace_bytes, (long long)need);
+  if (misaligned(workspace, 256) || misaligned(buf->obs, 16) || misaligned(buf->obs_last, 16))
+    return fail(PE_EINVAL, "bf16 rollout: workspace must be 256-byte and obs buffers 16-byte aligned");
   return rollout_bf16(env->dev, *net, params, horizon, iteration, lambda, det, *buf, workspace, st);
 }
 
@@ -427,6 +431,8 @@ pe_status pe_value(const pe_net* net, const float* params, const void* obs, int6
   if (need < 0) return fail(PE_EINVAL, "unsupported bf16 value network (D=%d H=%d)", net->obs_dim, net->hidden);
   if (!workspace || workspace_bytes < need)
     return fail(PE_EINVAL, "workspace too small (%lld < %lld bytes)", (long long)workspace_bytes, (long long)need);
+  if (misaligned(workspace, 256) || misaligned(obs, 16))
+    return fail(PE_EINVAL, "bf16 value: workspace must be 256-byte and obs 16-byte aligned");
   return value_bf16(*net, params, obs, n, value, workspace, st);
 }
 
@@ -481,6 +487,8 @@ pe_status pe_ppo_update(const pe_net* net, float* params, float* adam_m, float* 
   const int64_t need = ppo_ws_bytes(*net, *cfg, n_samples);
   if (need < 0) return fail(PE_EINVAL, "unsupported PPO network");
   if (workspace_bytes < need) return fail(PE_EINVAL, "workspace too small (%lld < %lld bytes)", (long long)workspace_bytes, (long long)need);
+  if (misaligned(workspace, 256) || misaligned(obs, 16))
+    return fail(PE_EINVAL, "workspace must be 256-byte and obs 16-byte aligned");
   if (net->dtype == PE_BF16)
     return ppo_update_bf16(*net, params, adam_m, adam_v, adam_t, obs, act, logp_old, adv, ret, n_samples, *cfg,
                            stats, workspace, reinterpret_cast<cudaStream_t>(stream));

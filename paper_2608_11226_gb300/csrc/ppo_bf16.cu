@@ -270,37 +270,53 @@ struct AssembleArgs {
   const float* db1p[2];
   const float* w3g[2];     // [16][H] head weight gradients (padded)
   const float* lossp;      // [nlb][32]
+  double* stat5;           // [5] minibatch loss statistics out
   int nrb, nlb, H, A;
   int64_t ob1[2], ob2[2], ob3[2], ow3[2];
 };
 
-// biases (fixed-order sums of the partials), head weights, nothing else
+// bias gradients: one warp per bias element sums its column of partials
+// (lane-strided, then a fixed shuffle tree: deterministic); the head weight
+// gradients are copied out of their padded 16-row buffers
 __global__ void assemble_kernel(AssembleArgs a) {
-  const int i = blockIdx.x * blockDim.x + threadIdx.x;
-  const int per = 2 * a.H + kHead * a.H + kHead;
-  if (i >= 2 * per) return;
-  const int net = i / per, j = i % per;
-  if (j < a.H) {
-    float s = 0.0f;
-    for (int b = 0; b < a.nrb; ++b) s += a.db2p[net][(int64_t)b * a.H + j];
-    a.grad[a.ob2[net] + j] = s;
-  } else if (j < 2 * a.H) {
-    const int c = j - a.H;
-    float s = 0.0f;
-    for (int b = 0; b < a.nrb; ++b) s += a.db1p[net][(int64_t)b * a.H + c];
-    a.grad[a.ob1[net] + c] = s;
-  } else if (j < 2 * a.H + kHead * a.H) {
-    const int q = j - 2 * a.H, r = q / a.H;
+  const int warp = (int)((blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5), lane = threadIdx.x & 31;
+  const int nb = 2 * a.H + kHead;  // bias elements per net: b2, b1, b3 (padded)
+  if (warp >= 2 * nb && warp < 2 * nb + 5) {
+    // minibatch loss statistics (pg, entropy, kl, clip, value) for the Adam kernel
+    const int k = warp - 2 * nb;
+    double s = 0.0;
+    for (int b = lane; b < a.nlb; b += 32) s += (double)a.lossp[(int64_t)b * kPartW + k];
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+    if (lane == 0) a.stat5[k] = s;
+  }
+  if (warp < 2 * nb) {
+    const int net = warp / nb, j = warp % nb;
     const int nout = net ? 1 : a.A;
-    if (r < nout) a.grad[a.ow3[net] + q] = a.w3g[net][q];
-  } else {
-    const int r = j - 2 * a.H - kHead * a.H;
-    const int nout = net ? 1 : a.A;
-    if (r < nout) {
-      float s = 0.0f;
-      for (int b = 0; b < a.nlb; ++b) s += a.lossp[(int64_t)b * kPartW + (net ? 21 : 5 + r)];
-      a.grad[a.ob3[net] + r] = s;
+    float s = 0.0f;
+    if (j < 2 * a.H) {
+      const float* src = j < a.H ? a.db2p[net] + j : a.db1p[net] + (j - a.H);
+      for (int b = lane; b < a.nrb; b += 32) s += src[(int64_t)b * a.H];
+    } else if (j - 2 * a.H < nout) {
+      const int col = net ? 21 : 5 + (j - 2 * a.H);
+      for (int b = lane; b < a.nlb; b += 32) s += a.lossp[(int64_t)b * kPartW + col];
     }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+    if (lane == 0) {
+      if (j < a.H) a.grad[a.ob2[net] + j] = s;
+      else if (j < 2 * a.H) a.grad[a.ob1[net] + (j - a.H)] = s;
+      else if (j - 2 * a.H < nout) a.grad[a.ob3[net] + (j - 2 * a.H)] = s;
+    }
+  }
+  // head weights: threads of the whole grid stride over 2 x 16 x H entries
+  const int64_t tid = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+  const int64_t per = (int64_t)kHead * a.H;
+  for (int64_t i = tid; i < 2 * per; i += (int64_t)gridDim.x * blockDim.x) {
+    const int net = (int)(i / per);
+    const int64_t q = i % per;
+    const int r = (int)(q / a.H);
+    if (r < (net ? 1 : a.A)) a.grad[a.ow3[net] + q] = a.w3g[net][q];
   }
 }
 
@@ -329,8 +345,7 @@ struct AdamBf16Args {
   int nsq;
   int64_t P;
   float beta1, beta2, step_size, inv_sqrt_bc2, eps, max_norm, vf_coef, ent_coef, inv_cnt;
-  const float* lossp;
-  int nlb;
+  const double* stat5;
   double* acc;
 };
 
@@ -355,9 +370,8 @@ __global__ void adam_bf16_kernel(AdamBf16Args a) {
     a.params[p] -= a.step_size * mp / (sqrtf(vp) * a.inv_sqrt_bc2 + a.eps);
   }
   if (blockIdx.x == 0 && threadIdx.x == 0) {
-    double v5[5] = {0, 0, 0, 0, 0};
-    for (int b = 0; b < a.nlb; ++b)
-      for (int k = 0; k < 5; ++k) v5[k] += a.lossp[(int64_t)b * kPartW + k];
+    double v5[5];
+    for (int k = 0; k < 5; ++k) v5[k] = a.stat5[k];
     const double ic = a.inv_cnt;
     a.acc[0] += v5[0] * ic;
     a.acc[1] += v5[4] * ic;
@@ -388,7 +402,7 @@ struct Bf16Plan {
   int nmb, mb, D, H, A, nrb, nlb, nsq;
   int64_t img;
   int64_t o_adv, o_idx, o_img, o_wb, o_x, o_h[4], o_zp, o_zv, o_dz[2], o_dh, o_da2, o_da1, o_db2[2], o_db1[2],
-      o_w3g[2], o_loss, o_grad, o_sq, o_acc, o_lt, total;
+      o_w3g[2], o_loss, o_grad, o_sq, o_acc, o_stat5, o_lt, total;
 };
 
 static int64_t al(int64_t x) { return (x + 1023) / 1024 * 1024; }
@@ -427,6 +441,7 @@ static Bf16Plan bf16_plan(const pe_net& net, const pe_ppo_config& cfg, int64_t N
   p.o_grad = o; o = al(o + p.P * 4);
   p.o_sq = o; o = al(o + (int64_t)p.nsq * 8);
   p.o_acc = o; o = al(o + 8 * 8 + 8);
+  p.o_stat5 = o; o = al(o + 5 * 8);
   p.o_lt = o; o = al(o + kLtWorkspace);
   p.total = o;
   return p;
@@ -467,6 +482,7 @@ pe_status ppo_update_bf16(const pe_net& net, float* params, float* m, float* v, 
   double* sq = reinterpret_cast<double*>(at(pl.o_sq));
   double* acc = reinterpret_cast<double*>(at(pl.o_acc));
   int32_t* err = reinterpret_cast<int32_t*>(acc + 8);
+  double* stat5 = reinterpret_cast<double*>(at(pl.o_stat5));
   void* lt_ws = at(pl.o_lt);
   const int D = pl.D, H = pl.H, A = pl.A;
   const MlpLayout Lp = mlp_layout(D, H, A);
@@ -549,6 +565,7 @@ pe_status ppo_update_bf16(const pe_net& net, float* params, float* m, float* v, 
         aa.w3g[i] = w3g[i];
       }
       aa.lossp = lossp;
+      aa.stat5 = stat5;
       aa.nrb = nrb;
       aa.nlb = nlb;
       aa.H = H;
@@ -557,7 +574,7 @@ pe_status ppo_update_bf16(const pe_net& net, float* params, float* m, float* v, 
       aa.ob2[0] = Lp.b2; aa.ob2[1] = Lp.c2;
       aa.ob3[0] = Lp.b3; aa.ob3[1] = Lp.c3;
       aa.ow3[0] = Lp.w3; aa.ow3[1] = Lp.v3;
-      const int per = 2 * H + kHead * H + kHead;
+      const int asm_warps = 2 * (2 * H + kHead) + 5;
       t += 1;
       AdamBf16Args ad;
       ad.params = params;
@@ -576,12 +593,11 @@ pe_status ppo_update_bf16(const pe_net& net, float* params, float* m, float* v, 
       ad.vf_coef = cfg.vf_coef;
       ad.ent_coef = cfg.ent_coef;
       ad.inv_cnt = 1.0f / (float)cnt;
-      ad.lossp = lossp;
-      ad.nlb = nlb;
+      ad.stat5 = stat5;
       ad.acc = acc;
       {
         ProfScope ps(PE_PROF_PPO_ADAM, st);
-        assemble_kernel<<<ceil_div(2 * per, 256), 256, 0, st>>>(aa);
+        assemble_kernel<<<ceil_div(asm_warps * 32, 256), 256, 0, st>>>(aa);
         sumsq_kernel<<<pl.nsq, 256, 0, st>>>(grad, pl.P, sq);
         adam_bf16_kernel<<<ceil_div(pl.P, 256), 256, 0, st>>>(ad);
       }

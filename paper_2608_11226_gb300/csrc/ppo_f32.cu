@@ -24,10 +24,10 @@
 
 namespace pe {
 
-constexpr int kPpoS = 32;           // samples per slice
+constexpr int kPpoS = 64;           // samples per slice
 constexpr int kPpoLD = kPpoS + 4;   // row stride of feature-major activations
 constexpr int kPpoNT = 512;         // threads per gradient CTA
-constexpr int kPpoRT = 2;           // sample rows per thread tile in the dense layers
+constexpr int kPpoRT = 4;           // sample rows per thread tile in the dense layers
 constexpr int kPpoMaxEpochs = 16;
 
 struct FeistelSet {
@@ -74,10 +74,11 @@ __global__ void ppo_advstats_kernel(const float* __restrict__ adv, int64_t N, in
   }
 }
 
-// outT[n][e] = (sum_k inT[k][e] W[k][n]) * (1 - hT[n][e]^2): back through a tanh layer
+// back through a tanh layer, in place: hT[n][e] <- (sum_k inT[k][e] W[k][n]) * (1 - hT[n][e]^2).
+// Each thread reads hT only at the elements it writes.
 template <int TE, int K, int N, int LD, int RT>
-__device__ __forceinline__ void dense_bwd_t(const float* __restrict__ inT, const float* __restrict__ W,
-                                            const float* __restrict__ hT, float* __restrict__ outT) {
+__device__ __forceinline__ void dense_bwd_inplace(const float* __restrict__ inT, const float* __restrict__ W,
+                                                  float* hT) {
   constexpr int EG = TE / RT, NG = N / 4;
   for (int j = threadIdx.x; j < EG * NG; j += blockDim.x) {
     const int eg = j % EG, ng = j / EG;
@@ -103,7 +104,7 @@ __device__ __forceinline__ void dense_bwd_t(const float* __restrict__ inT, const
       load_rt<RT>(hT + (ng * 4 + c) * LD + eg * RT, h);
 #pragma unroll
       for (int r = 0; r < RT; ++r) o[r] = acc[r][c] * (1.0f - h[r] * h[r]);
-      store_rt<RT>(outT + (ng * 4 + c) * LD + eg * RT, o);
+      store_rt<RT>(hT + (ng * 4 + c) * LD + eg * RT, o);
     }
   }
 }
@@ -175,14 +176,18 @@ struct WGradAcc {
   }
 };
 
+// Shared memory of one gradient CTA: the role's weights (W1 and W2
+// transposed for the forward pass, W2 as stored for the backward pass) and
+// one 64-sample slice of feature-major activations.  h2t holds h2, then the
+// layer-2 pre-activation gradient; h1t holds h1, then the layer-1 one.
 template <int D, int H, int A>
 struct PpoSmem {
-  float w1t[D * H], w2t[H * H], w2[H * H], b1[H], b2[H], w3[A * H], b3[(A + 3) / 4 * 4];
-  float xt[D * kPpoLD], h1t[H * kPpoLD], h2t[H * kPpoLD], d2t[H * kPpoLD];
+  float w1t[D * H], w2t[H * H], w2[H * H], w3[A * H], b1[H], b2[H], b3[8];
+  float xt[D * kPpoLD], h1t[H * kPpoLD], h2t[H * kPpoLD];
   float z[kPpoS * A];
   float lpo[kPpoS], advn[kPpoS], ret[kPpoS];
   int32_t act[kPpoS], valid[kPpoS];
-  uint32_t idx[kPpoS];
+  float stat[kPpoS / 32][8];
 };
 
 struct PpoArgs {
@@ -192,6 +197,7 @@ struct PpoArgs {
   const float* adv;
   const float* ret;
   const float* params;
+  const float* params_t;  // W1, W2, V1, V2 stored transposed ([in][out]) at their own offsets
   Feistel perm;
   int64_t start;
   int cnt;
@@ -204,77 +210,131 @@ struct PpoArgs {
   int64_t P;
 };
 
+// Transposed copy of an updated parameter, for the hidden-layer matrices.
+template <int D, int H, int A>
+__device__ __forceinline__ void store_transposed(float* pt, int64_t p, float val) {
+  const MlpLayout L = mlp_layout(D, H, A);
+  if (p < L.b1) {
+    const int64_t q = p - L.w1;
+    pt[L.w1 + (q % D) * H + q / D] = val;
+  } else if (p >= L.w2 && p < L.b2) {
+    const int64_t q = p - L.w2;
+    pt[L.w2 + (q % H) * H + q / H] = val;
+  } else if (p >= L.v1 && p < L.c1) {
+    const int64_t q = p - L.v1;
+    pt[L.v1 + (q % D) * H + q / D] = val;
+  } else if (p >= L.v2 && p < L.c2) {
+    const int64_t q = p - L.v2;
+    pt[L.v2 + (q % H) * H + q / H] = val;
+  }
+}
+
+template <int D, int H, int A>
+__global__ void ppo_transpose_kernel(const float* __restrict__ params, float* __restrict__ pt) {
+  const int64_t P = mlp_layout(D, H, A).total;
+  for (int64_t p = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; p < P; p += (int64_t)gridDim.x * blockDim.x)
+    store_transposed<D, H, A>(pt, p, params[p]);
+}
+
+// One role (policy or value network) of the minibatch gradient over this
+// CTA's slices: forward, loss, backward; weight-gradient partials in
+// registers, written as this CTA's row of the partial-sum matrix.
 template <int D, int H, int A, bool POL>
 __device__ __forceinline__ void ppo_role(PpoSmem<D, H, A>& s, const PpoArgs& g, int c) {
   constexpr int NA = POL ? A : 1;
+  constexpr int S = kPpoS, LD = kPpoLD;
+  static_assert(D % 4 == 0 && H % 32 == 0 && S * (D / 4) <= 256 && 256 + S <= kPpoNT && 4 * H <= kPpoNT,
+                "gradient CTA layout");
   const MlpLayout Lp = mlp_layout(D, H, A);
   const int64_t oW1 = POL ? Lp.w1 : Lp.v1, oB1 = POL ? Lp.b1 : Lp.c1;
   const int64_t oW2 = POL ? Lp.w2 : Lp.v2, oB2 = POL ? Lp.b2 : Lp.c2;
   const int64_t oW3 = POL ? Lp.w3 : Lp.v3, oB3 = POL ? Lp.b3 : Lp.c3;
+  const int tid = threadIdx.x;
   // parameters are read through L2 (not the non-coherent L1 path): inside the
   // persistent update other CTAs rewrite them between minibatches
-  for (int i = threadIdx.x; i < H * D; i += blockDim.x) s.w1t[i] = __ldcg(g.params + oW1 + (int64_t)(i % H) * D + i / H);
-  for (int i = threadIdx.x; i < H * H; i += blockDim.x) {
-    s.w2t[i] = __ldcg(g.params + oW2 + (int64_t)(i % H) * H + i / H);
+  for (int i = tid; i < H * D; i += blockDim.x) s.w1t[i] = __ldcg(g.params_t + oW1 + i);
+  for (int i = tid; i < H * H; i += blockDim.x) {
+    s.w2t[i] = __ldcg(g.params_t + oW2 + i);
     s.w2[i] = __ldcg(g.params + oW2 + i);
   }
-  for (int i = threadIdx.x; i < H; i += blockDim.x) {
+  for (int i = tid; i < H; i += blockDim.x) {
     s.b1[i] = __ldcg(g.params + oB1 + i);
     s.b2[i] = __ldcg(g.params + oB2 + i);
   }
-  for (int i = threadIdx.x; i < NA * H; i += blockDim.x) s.w3[i] = __ldcg(g.params + oW3 + i);
-  for (int i = threadIdx.x; i < NA; i += blockDim.x) s.b3[i] = __ldcg(g.params + oB3 + i);
-  const int tid = threadIdx.x;
+  for (int i = tid; i < NA * H; i += blockDim.x) s.w3[i] = __ldcg(g.params + oW3 + i);
+  for (int i = tid; i < NA; i += blockDim.x) s.b3[i] = __ldcg(g.params + oB3 + i);
   const float2 as = *g.advstat;
 
   WGradAcc<H, H, kPpoNT> g2;
   WGradAcc<H, D, kPpoNT> g1;
   g2.zero();
   g1.zero();
-  constexpr int PER3 = (NA * H + kPpoNT - 1) / kPpoNT;
-  float g3[PER3], gb1 = 0.0f, gb2 = 0.0f, gb3 = 0.0f;
+  // head backward: thread (k = tid / 4, quarter q = tid % 4) owns row k of the
+  // head weight gradient and of the layer-2 bias gradient over samples 4i + q
+  const int hk = tid >> 2, hq = tid & 3;
+  float g3[NA], gb2 = 0.0f, gb1 = 0.0f, gb3 = 0.0f;
 #pragma unroll
-  for (int q = 0; q < PER3; ++q) g3[q] = 0.0f;
-  float st_pg = 0.0f, st_ent = 0.0f, st_kl = 0.0f, st_clip = 0.0f, st_v = 0.0f;
+  for (int a = 0; a < NA; ++a) g3[a] = 0.0f;
+  float st[5] = {0.0f, 0.0f, 0.0f, 0.0f, 0.0f};  // pg, entropy, kl, clip, value (threads < S)
 
   for (int sl = 0; sl < g.slices_per_cta; ++sl) {
-    const int base = (c * g.slices_per_cta + sl) * kPpoS;
+    const int base = (c * g.slices_per_cta + sl) * S;
     if (base >= g.cnt) break;
     __syncthreads();
-    // gather the slice (permuted sample order)
-    for (int i = tid; i < kPpoS; i += blockDim.x) {
-      const int ok = base + i < g.cnt;
-      s.valid[i] = ok;
+    // gather the slice (permuted sample order): observations as float4 rows,
+    // per-sample scalars by threads 256..256+S
+    constexpr int F4 = D / 4;
+    if (tid < S * F4) {
+      const int si = tid / F4, f = tid % F4;
+      float4 v = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+      if (base + si < g.cnt) {
+        const uint32_t idx = feistel_index(g.perm, g.start + base + si);
+        v = __ldg(reinterpret_cast<const float4*>(g.obs + (int64_t)idx * D) + f);
+      }
+      s.xt[(4 * f + 0) * LD + si] = v.x;
+      s.xt[(4 * f + 1) * LD + si] = v.y;
+      s.xt[(4 * f + 2) * LD + si] = v.z;
+      s.xt[(4 * f + 3) * LD + si] = v.w;
+    } else if (tid >= 256 && tid < 256 + S) {
+      const int si = tid - 256;
+      const int ok = base + si < g.cnt;
+      s.valid[si] = ok;
       if (ok) {
-        const uint32_t idx = feistel_index(g.perm, g.start + base + i);
-        s.idx[i] = idx;
-        s.act[i] = __ldg(g.act + idx);
-        s.lpo[i] = __ldg(g.logp_old + idx);
-        s.advn[i] = (__ldg(g.adv + idx) - as.x) * as.y;
-        s.ret[i] = __ldg(g.ret + idx);
+        const uint32_t idx = feistel_index(g.perm, g.start + base + si);
+        s.act[si] = __ldg(g.act + idx);
+        s.lpo[si] = __ldg(g.logp_old + idx);
+        s.advn[si] = (__ldg(g.adv + idx) - as.x) * as.y;
+        s.ret[si] = __ldg(g.ret + idx);
       } else {
-        s.idx[i] = 0;
-        s.act[i] = 0;
-        s.lpo[i] = s.advn[i] = s.ret[i] = 0.0f;
+        s.act[si] = 0;
+        s.lpo[si] = s.advn[si] = s.ret[si] = 0.0f;
       }
     }
     __syncthreads();
-    for (int i = tid; i < kPpoS * D; i += blockDim.x) {
-      const int si = i / D, f = i % D;
-      float v = 0.0f;
-      if (s.valid[si]) v = __ldg(g.obs + (int64_t)s.idx[si] * D + f);
-      s.xt[f * kPpoLD + si] = v;
+    // forward
+    dense_tanh_t<S, D, H, LD, kPpoRT>(s.xt, s.w1t, s.b1, s.h1t);
+    __syncthreads();
+    dense_tanh_t<S, H, H, LD, kPpoRT>(s.h1t, s.w2t, s.b2, s.h2t);
+    __syncthreads();
+    // head: 4 interleaved K-parts per output in adjacent lanes, shuffle-combined
+    {
+      constexpr int JOBS = (S * NA * 4 + 31) / 32 * 32;
+      for (int j = tid; j < JOBS; j += blockDim.x) {
+        const int part = j & 3, o = j >> 2;
+        const int si = o % S, a = o / S;
+        float acc = 0.0f;
+        if (o < S * NA) {
+#pragma unroll 8
+          for (int k = part; k < H; k += 4) acc = fmaf(s.w3[a * H + k], s.h2t[k * LD + si], acc);
+        }
+        acc += __shfl_xor_sync(0xffffffffu, acc, 1);
+        acc += __shfl_xor_sync(0xffffffffu, acc, 2);
+        if (part == 0 && o < S * NA) s.z[si * NA + a] = acc + s.b3[a];
+      }
     }
     __syncthreads();
-    // forward
-    dense_tanh_t<kPpoS, D, H, kPpoLD, kPpoRT>(s.xt, s.w1t, s.b1, s.h1t);
-    __syncthreads();
-    dense_tanh_t<kPpoS, H, H, kPpoLD, kPpoRT>(s.h1t, s.w2t, s.b2, s.h2t);
-    __syncthreads();
-    head_t<kPpoS, H, NA, kPpoLD>(s.h2t, s.w3, s.b3, s.z);
-    __syncthreads();
-    // loss terms and dLoss/dhead per sample
-    if (tid < kPpoS) {
+    // loss terms and dLoss/dhead per sample (written over the head outputs)
+    if (tid < S) {
       float* z = s.z + tid * NA;
       if (!s.valid[tid]) {
 #pragma unroll
@@ -296,65 +356,68 @@ __device__ __forceinline__ void ppo_role(PpoSmem<D, H, A>& s, const PpoArgs& g, 
         }
         const int a = s.act[tid];
         const float an = s.advn[tid];
-        const float logr = lp[a] - s.lpo[tid];
+        float lpa = 0.0f;
+#pragma unroll
+        for (int j = 0; j < NA; ++j)
+          if (j == a) lpa = lp[j];
+        const float logr = lpa - s.lpo[tid];
         const float rho = expf(logr);
         const float rc = fminf(fmaxf(rho, 1.0f - g.clip), 1.0f + g.clip);
         const float s1 = rho * an, s2 = rc * an;
-        st_pg += -fminf(s1, s2);
-        st_ent += Hs;
-        st_kl += (rho - 1.0f) - logr;
-        st_clip += fabsf(rho - 1.0f) > g.clip ? 1.0f : 0.0f;
+        st[0] += -fminf(s1, s2);
+        st[1] += Hs;
+        st[2] += (rho - 1.0f) - logr;
+        st[3] += fabsf(rho - 1.0f) > g.clip ? 1.0f : 0.0f;
         const float dlp = (s1 <= s2 ? -an : 0.0f) * rho * g.inv_cnt;
 #pragma unroll
         for (int j = 0; j < NA; ++j)
           z[j] = dlp * ((j == a ? 1.0f : 0.0f) - p[j]) + g.ent_coef * g.inv_cnt * p[j] * (lp[j] + Hs);
       } else {
         const float V = z[0], R = s.ret[tid];
-        st_v += (R - V) * (R - V);
+        st[4] += (R - V) * (R - V);
         z[0] = g.vf_coef * 2.0f * (V - R) * g.inv_cnt;
       }
     }
     __syncthreads();
-    // head gradient; back through the head into layer 2
+    // head weight gradient, back through the head into layer 2 (in place over h2)
+    if (hk < H) {
+      float w3k[NA];
 #pragma unroll
-    for (int q = 0; q < PER3; ++q) {
-      const int j = tid + q * kPpoNT;
-      if (j < NA * H) {
-        const int a = j / H, k = j % H;
-        float acc = 0.0f;
-#pragma unroll 8
-        for (int si = 0; si < kPpoS; ++si) acc = fmaf(s.z[si * NA + a], s.h2t[k * kPpoLD + si], acc);
-        g3[q] += acc;
+      for (int a = 0; a < NA; ++a) w3k[a] = s.w3[a * H + hk];
+#pragma unroll 4
+      for (int i = 0; i < S / 4; ++i) {
+        const int si = 4 * i + hq;
+        const float h = s.h2t[hk * LD + si];
+        float d = 0.0f;
+#pragma unroll
+        for (int a = 0; a < NA; ++a) {
+          const float dz = s.z[si * NA + a];
+          g3[a] = fmaf(dz, h, g3[a]);
+          d = fmaf(w3k[a], dz, d);
+        }
+        const float d2 = d * (1.0f - h * h);
+        s.h2t[hk * LD + si] = d2;
+        gb2 += d2;
       }
     }
     if (tid < NA) {
       float acc = 0.0f;
-      for (int si = 0; si < kPpoS; ++si) acc += s.z[si * NA + tid];
+      for (int si = 0; si < S; ++si) acc += s.z[si * NA + tid];
       gb3 += acc;
     }
-    for (int i = tid; i < H * kPpoS; i += blockDim.x) {
-      const int k = i / kPpoS, si = i % kPpoS;
-      float acc = 0.0f;
-#pragma unroll
-      for (int a = 0; a < NA; ++a) acc = fmaf(s.w3[a * H + k], s.z[si * NA + a], acc);
-      const float h = s.h2t[k * kPpoLD + si];
-      s.d2t[k * kPpoLD + si] = acc * (1.0f - h * h);
-    }
     __syncthreads();
-    // layer-2 weight gradient; back into layer 1 (written over h2t, now dead)
-    g2.template add<kPpoS, kPpoLD>(s.d2t, s.h1t);
-    if (tid < H) {
-      float acc = 0.0f;
-      for (int si = 0; si < kPpoS; ++si) acc += s.d2t[tid * kPpoLD + si];
-      gb2 += acc;
-    }
-    dense_bwd_t<kPpoS, H, H, kPpoLD, kPpoRT>(s.d2t, s.w2, s.h1t, s.h2t);
+    // layer-2 weight gradient
+    g2.template add<S, LD>(s.h2t, s.h1t);
     __syncthreads();
-    // layer-1 weight gradient
-    g1.template add<kPpoS, kPpoLD>(s.h2t, s.xt);
-    if (tid < H) {
+    // back into layer 1 (in place over h1)
+    dense_bwd_inplace<S, H, H, LD, kPpoRT>(s.h2t, s.w2, s.h1t);
+    __syncthreads();
+    // layer-1 weight and bias gradients (the bias by the warps the tiles leave idle)
+    g1.template add<S, LD>(s.h1t, s.xt);
+    if (tid >= kPpoNT - H) {
+      const int n = tid - (kPpoNT - H), lane = tid & 31;
       float acc = 0.0f;
-      for (int si = 0; si < kPpoS; ++si) acc += s.h2t[tid * kPpoLD + si];
+      for (int i = 0; i < S; ++i) acc += s.h1t[n * LD + ((i + lane) & (S - 1))];
       gb1 += acc;
     }
   }
@@ -363,26 +426,37 @@ __device__ __forceinline__ void ppo_role(PpoSmem<D, H, A>& s, const PpoArgs& g, 
   g1.store(row + oW1);
   g2.store(row + oW2);
 #pragma unroll
-  for (int q = 0; q < PER3; ++q) {
-    const int j = tid + q * kPpoNT;
-    if (j < NA * H) row[oW3 + j] = g3[q];
+  for (int a = 0; a < NA; ++a) {
+    g3[a] += __shfl_xor_sync(0xffffffffu, g3[a], 1);
+    g3[a] += __shfl_xor_sync(0xffffffffu, g3[a], 2);
   }
-  if (tid < H) {
-    row[oB1 + tid] = gb1;
-    row[oB2 + tid] = gb2;
+  gb2 += __shfl_xor_sync(0xffffffffu, gb2, 1);
+  gb2 += __shfl_xor_sync(0xffffffffu, gb2, 2);
+  if (hq == 0 && hk < H) {
+#pragma unroll
+    for (int a = 0; a < NA; ++a) row[oW3 + (int64_t)a * H + hk] = g3[a];
+    row[oB2 + hk] = gb2;
   }
+  if (tid >= kPpoNT - H) row[oB1 + tid - (kPpoNT - H)] = gb1;
   if (tid < NA) row[oB3 + tid] = gb3;
-  // statistics of the slice samples (held by warp 0), fixed shuffle tree
-  if (tid < 32) {
-    float v[5] = {st_pg, st_ent, st_kl, st_clip, st_v};
+  // statistics of the CTA's samples (held by threads < S), fixed shuffle tree
+  if (tid < S) {
 #pragma unroll
     for (int k = 0; k < 5; ++k)
 #pragma unroll
-      for (int o = 16; o > 0; o >>= 1) v[k] += __shfl_xor_sync(0xffffffffu, v[k], o);
-    if (tid == 0) {
-      float* sp = g.stat_partial + (int64_t)((POL ? 0 : g.NC) + c) * 8;
+      for (int o = 16; o > 0; o >>= 1) st[k] += __shfl_xor_sync(0xffffffffu, st[k], o);
+    if ((tid & 31) == 0)
 #pragma unroll
-      for (int k = 0; k < 5; ++k) sp[k] = v[k];
+      for (int k = 0; k < 5; ++k) s.stat[tid >> 5][k] = st[k];
+  }
+  __syncthreads();
+  if (tid == 0) {
+    float* sp = g.stat_partial + (int64_t)((POL ? 0 : g.NC) + c) * 8;
+#pragma unroll
+    for (int k = 0; k < 5; ++k) {
+      float t = 0.0f;
+      for (int w = 0; w < S / 32; ++w) t += s.stat[w][k];
+      sp[k] = t;
     }
   }
 }
@@ -412,6 +486,7 @@ struct PpoLoop {
   int64_t N;
   int minibatch, nmb, epochs;
   float* params;
+  float* pt;               // transposed hidden-layer matrices (PpoArgs::params_t)
   float* m;
   float* v;
   double* sq;              // [gridDim.x]
@@ -550,7 +625,9 @@ __global__ void __launch_bounds__(kPpoNT, 1) ppo_persistent_kernel(PpoLoop L) {
         const float vp = L.beta2 * L.v[p] + (1.0f - L.beta2) * gp * gp;
         L.m[p] = mp;
         L.v[p] = vp;
-        L.params[p] -= step_size * mp / (sqrtf(vp) * inv_sqrt_bc2 + L.eps);
+        const float np = L.params[p] - step_size * mp / (sqrtf(vp) * inv_sqrt_bc2 + L.eps);
+        L.params[p] = np;
+        store_transposed<D, H, A>(L.pt, p, np);
       }
       if (blockIdx.x == 0 && tid == 0) {
         L.acc[6] = norm;
@@ -658,7 +735,8 @@ struct AdamArgs {
   float beta1, beta2, step_size, inv_sqrt_bc2, eps, max_norm;
 };
 
-__global__ void ppo_adam_kernel(float* __restrict__ params, float* __restrict__ m,
+template <int D, int H, int A>
+__global__ void ppo_adam_kernel(float* __restrict__ params, float* __restrict__ pt, float* __restrict__ m,
                                 float* __restrict__ v, const float* __restrict__ grad,
                                 const double* __restrict__ norm_p, int64_t P, AdamArgs a) {
   const double norm = *norm_p;
@@ -670,7 +748,9 @@ __global__ void ppo_adam_kernel(float* __restrict__ params, float* __restrict__ 
     const float vp = a.beta2 * v[p] + (1.0f - a.beta2) * gp * gp;
     m[p] = mp;
     v[p] = vp;
-    params[p] -= a.step_size * mp / (sqrtf(vp) * a.inv_sqrt_bc2 + a.eps);
+    const float np = params[p] - a.step_size * mp / (sqrtf(vp) * a.inv_sqrt_bc2 + a.eps);
+    params[p] = np;
+    store_transposed<D, H, A>(pt, p, np);
   }
 }
 
@@ -706,7 +786,7 @@ Feistel make_feistel(uint64_t n, uint64_t seed, uint32_t epoch, uint32_t iterati
 struct PpoPlan {
   int64_t P, N;
   int nmb, NC, slices_per_cta, nsq, steps;
-  int64_t off_advstat, off_partial, off_stat, off_grad, off_sq, off_acc, off_bar, off_bc, total;
+  int64_t off_advstat, off_partial, off_stat, off_grad, off_pt, off_sq, off_acc, off_bar, off_bc, total;
 };
 
 static int64_t align256(int64_t x) { return (x + 255) / 256 * 256; }
@@ -726,6 +806,7 @@ static PpoPlan ppo_plan(const pe_net& net, const pe_ppo_config& cfg, int64_t N) 
   p.off_partial = o; o = align256(o + (int64_t)p.NC * p.P * 4);
   p.off_stat = o; o = align256(o + (int64_t)2 * p.NC * 8 * 4);
   p.off_grad = o; o = align256(o + p.P * 4);
+  p.off_pt = o; o = align256(o + p.P * 4);
   p.off_sq = o; o = align256(o + (int64_t)(p.nsq > 2 * p.NC ? p.nsq : 2 * p.NC) * 8);
   p.off_acc = o; o = align256(o + 8 * 8 + 16);
   p.off_bar = o; o = align256(o + 16);
@@ -742,7 +823,7 @@ pe_status launch_advstats(const float* adv, int64_t N, int M, int nmb, int epoch
   for (int ep = 0; ep < epochs; ++ep) perms.f[ep] = make_feistel((uint64_t)N, seed, ep, iteration);
   {
     ProfScope ps(PE_PROF_PPO_OTHER, st);
-    ppo_advstats_kernel<<<dim3(nmb, epochs), 256, 0, st>>>(adv, N, M, nmb, perms, out);
+    ppo_advstats_kernel<<<dim3(nmb, epochs), 1024, 0, st>>>(adv, N, M, nmb, perms, out);
   }
   PE_CHECK_LAUNCH("ppo_advstats_kernel");
   return PE_OK;
@@ -762,6 +843,7 @@ static pe_status ppo_run(const pe_net& net, float* params, float* m, float* v, i
   float* partial = reinterpret_cast<float*>(ws + pl.off_partial);
   float* stat_partial = reinterpret_cast<float*>(ws + pl.off_stat);
   float* grad = reinterpret_cast<float*>(ws + pl.off_grad);
+  float* pt = reinterpret_cast<float*>(ws + pl.off_pt);
   double* sq = reinterpret_cast<double*>(ws + pl.off_sq);
   double* acc = reinterpret_cast<double*>(ws + pl.off_acc);
   double* norm = acc + 8;
@@ -774,6 +856,11 @@ static pe_status ppo_run(const pe_net& net, float* params, float* m, float* v, i
     ppo_advstats_kernel<<<dim3(pl.nmb, cfg.epochs), 256, 0, st>>>(adv, N, cfg.minibatch, pl.nmb, perms, advstat);
   }
   PE_CHECK_LAUNCH("ppo_advstats_kernel");
+  {
+    ProfScope ps(PE_PROF_PPO_OTHER, st);
+    ppo_transpose_kernel<D, H, A><<<ceil_div(pl.P, 256), 256, 0, st>>>(params, pt);
+  }
+  PE_CHECK_LAUNCH("ppo_transpose_kernel");
   using Smem = PpoSmem<D, H, A>;
   auto kern = ppo_grad_kernel<D, H, A>;
   const int bytes = (int)sizeof(Smem);
@@ -806,6 +893,8 @@ static pe_status ppo_run(const pe_net& net, float* params, float* m, float* v, i
     L.g.adv = adv;
     L.g.ret = ret;
     L.g.params = params;
+    L.g.params_t = pt;
+    L.pt = pt;
     L.g.clip = cfg.clip;
     L.g.vf_coef = cfg.vf_coef;
     L.g.ent_coef = cfg.ent_coef;
@@ -852,6 +941,7 @@ static pe_status ppo_run(const pe_net& net, float* params, float* m, float* v, i
         g.adv = adv;
         g.ret = ret;
         g.params = params;
+        g.params_t = pt;
         g.perm = perms.f[ep];
         g.start = start;
         g.cnt = cnt;
@@ -900,7 +990,7 @@ static pe_status ppo_run(const pe_net& net, float* params, float* m, float* v, i
         a.max_norm = cfg.max_grad_norm;
         {
           ProfScope ps(PE_PROF_PPO_ADAM, st);
-          ppo_adam_kernel<<<(int)((pl.P + 255) / 256), 256, 0, st>>>(params, m, v, grad, norm, pl.P, a);
+          ppo_adam_kernel<D, H, A><<<(int)((pl.P + 255) / 256), 256, 0, st>>>(params, pt, m, v, grad, norm, pl.P, a);
         }
         PE_CHECK_LAUNCH("ppo_adam_kernel");
       }
