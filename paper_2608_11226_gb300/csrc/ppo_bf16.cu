@@ -320,17 +320,18 @@ __global__ void assemble_kernel(AssembleArgs a) {
   }
 }
 
-__global__ void sumsq_kernel(const float* __restrict__ g, int64_t P, double* __restrict__ sq) {
-  __shared__ double red[32];
-  double s = 0.0;
+// fp32 sums of squares over 256 fixed blocks (fixed order: deterministic)
+__global__ void sumsq_kernel(const float* __restrict__ g, int64_t P, float* __restrict__ sq) {
+  __shared__ float red[32];
+  float s = 0.0f;
   for (int64_t p = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; p < P; p += (int64_t)gridDim.x * blockDim.x)
-    s += (double)g[p] * (double)g[p];
+    s = fmaf(g[p], g[p], s);
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
   if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = s;
   __syncthreads();
   if (threadIdx.x == 0) {
-    double t = 0.0;
+    float t = 0.0f;
     for (int w = 0; w < (int)(blockDim.x >> 5); ++w) t += red[w];
     sq[blockIdx.x] = t;
   }
@@ -341,7 +342,7 @@ struct AdamBf16Args {
   float* m;
   float* v;
   const float* grad;
-  const double* sq;
+  const float* sq;
   int nsq;
   int64_t P;
   float beta1, beta2, step_size, inv_sqrt_bc2, eps, max_norm, vf_coef, ent_coef, inv_cnt;
@@ -350,17 +351,17 @@ struct AdamBf16Args {
 };
 
 __global__ void adam_bf16_kernel(AdamBf16Args a) {
-  __shared__ double s_norm;
+  __shared__ float s_norm;
   if (threadIdx.x < 32) {
-    double t = 0.0;
+    float t = 0.0f;
     for (int b = threadIdx.x; b < a.nsq; b += 32) t += a.sq[b];
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
-    if (threadIdx.x == 0) s_norm = sqrt(t);
+    if (threadIdx.x == 0) s_norm = sqrtf(t);
   }
   __syncthreads();
-  const double norm = s_norm;
-  const float coef = (float)fmin(1.0, (double)a.max_norm / (norm + 1e-6));
+  const float norm = s_norm;
+  const float coef = fminf(1.0f, a.max_norm / (norm + 1e-6f));
   for (int64_t p = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; p < a.P; p += (int64_t)gridDim.x * blockDim.x) {
     const float gp = a.grad[p] * coef;
     const float mp = a.beta1 * a.m[p] + (1.0f - a.beta1) * gp;
@@ -479,7 +480,7 @@ pe_status ppo_update_bf16(const pe_net& net, float* params, float* m, float* v, 
   float* w3g[2] = {reinterpret_cast<float*>(at(pl.o_w3g[0])), reinterpret_cast<float*>(at(pl.o_w3g[1]))};
   float* lossp = reinterpret_cast<float*>(at(pl.o_loss));
   float* grad = reinterpret_cast<float*>(at(pl.o_grad));
-  double* sq = reinterpret_cast<double*>(at(pl.o_sq));
+  float* sq = reinterpret_cast<float*>(at(pl.o_sq));
   double* acc = reinterpret_cast<double*>(at(pl.o_acc));
   int32_t* err = reinterpret_cast<int32_t*>(acc + 8);
   double* stat5 = reinterpret_cast<double*>(at(pl.o_stat5));

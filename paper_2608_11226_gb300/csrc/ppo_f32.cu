@@ -20,6 +20,8 @@
 #include <cmath>
 #include <vector>
 
+#include <cstddef>
+
 #include "mlp_f32.cuh"
 
 namespace pe {
@@ -34,15 +36,17 @@ struct FeistelSet {
   Feistel f[kPpoMaxEpochs];
 };
 
-// deterministic block reduction of a double (fixed shuffle tree + fixed order)
-__device__ __forceinline__ double block_sum_d(double v, double* red) {
+// Reductions are fp32 with a fixed order (per-thread sequential sums, a
+// fixed shuffle tree, then warps in order): deterministic, and off the FP64
+// pipe, which on this part runs a few operations per SM per clock.
+__device__ __forceinline__ float block_sum_f(float v, float* red) {
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
   const int w = threadIdx.x >> 5, nw = blockDim.x >> 5;
   __syncthreads();
   if ((threadIdx.x & 31) == 0) red[w] = v;
   __syncthreads();
-  double t = 0.0;
+  float t = 0.0f;
   for (int i = 0; i < nw; ++i) t += red[i];
   return t;
 }
@@ -50,26 +54,75 @@ __device__ __forceinline__ double block_sum_d(double v, double* red) {
 // advantage mean and 1/(std + 1e-8) (unbiased std) of every minibatch
 __global__ void ppo_advstats_kernel(const float* __restrict__ adv, int64_t N, int M, int nmb,
                                     FeistelSet perms, float2* __restrict__ out) {
-  __shared__ double red[32];
+  __shared__ float red[32];
   const int mb = blockIdx.x, ep = blockIdx.y;
   const Feistel& f = perms.f[ep];
   const int64_t start = (int64_t)mb * M;
   const int cnt = (int)(N - start < (int64_t)M ? N - start : (int64_t)M);
-  double s = 0.0;
-  for (int j = threadIdx.x; j < cnt; j += blockDim.x) s += (double)__ldg(adv + feistel_index(f, start + j));
-  const double mean = block_sum_d(s, red) / (double)cnt;
-  double q = 0.0;
+  float s = 0.0f;
+  for (int j = threadIdx.x; j < cnt; j += blockDim.x) s += __ldg(adv + feistel_index(f, start + j));
+  const float mean = block_sum_f(s, red) / (float)cnt;
+  float q = 0.0f;
   for (int j = threadIdx.x; j < cnt; j += blockDim.x) {
-    const double a = (double)__ldg(adv + feistel_index(f, start + j)) - mean;
-    q += a * a;
+    const float a = __ldg(adv + feistel_index(f, start + j)) - mean;
+    q = fmaf(a, a, q);
   }
-  const double ss = block_sum_d(q, red);
+  const float ss = block_sum_f(q, red);
   if (threadIdx.x == 0) {
     if (cnt > 1) {
-      const double sd = sqrt(ss / (double)(cnt - 1));
-      out[ep * nmb + mb] = make_float2((float)mean, (float)(1.0 / (sd + 1e-8)));
+      const float sd = sqrtf(ss / (float)(cnt - 1));
+      out[ep * nmb + mb] = make_float2(mean, 1.0f / (sd + 1e-8f));
     } else {
       out[ep * nmb + mb] = make_float2(0.0f, 1.0f);  // a 1-sample minibatch is not normalised
+    }
+  }
+}
+
+// Dense-layer register tiles for the 64-sample slices: a thread owns RT
+// sample rows x 4 neurons; a warp covers 4 row groups x 8 neuron groups, so
+// each of its float4 loads (inputs and weights) is a single 64- or 128-byte
+// shared-memory wavefront.
+template <int TE, int N, int RT>
+__device__ __forceinline__ bool dense_job(int j, int& eg, int& ng) {
+  constexpr int EG = TE / RT, NG = N / 4, BE = EG / 4;  // BE: 4-row-group blocks along the slice
+  static_assert(EG % 4 == 0 && NG % 8 == 0, "dense tile layout");
+  const int wb = j >> 5, lane = j & 31;
+  eg = (wb % BE) * 4 + (lane & 3);
+  ng = (wb / BE) * 8 + (lane >> 2);
+  return ng < NG;
+}
+
+// outT[n][e] = tanh(b[n] + sum_k inT[k][e] WT[k][n])
+template <int TE, int K, int N, int LD, int RT>
+__device__ __forceinline__ void dense_fwd_w(const float* __restrict__ inT, const float* __restrict__ WT,
+                                            const float* __restrict__ bias, float* __restrict__ outT) {
+  constexpr int JOBS = (TE / RT) * (N / 4);
+  for (int j = threadIdx.x; j < JOBS; j += blockDim.x) {
+    int eg, ng;
+    if (!dense_job<TE, N, RT>(j, eg, ng)) continue;
+    float acc[RT][4];
+#pragma unroll
+    for (int r = 0; r < RT; ++r)
+#pragma unroll
+      for (int c = 0; c < 4; ++c) acc[r][c] = 0.0f;
+#pragma unroll 8
+    for (int k = 0; k < K; ++k) {
+      float xv[RT];
+      load_rt<RT>(inT + k * LD + eg * RT, xv);
+      const float4 w = *reinterpret_cast<const float4*>(WT + k * N + ng * 4);
+      const float wv[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+      for (int r = 0; r < RT; ++r)
+#pragma unroll
+        for (int c = 0; c < 4; ++c) acc[r][c] = fmaf(xv[r], wv[c], acc[r][c]);
+    }
+#pragma unroll
+    for (int c = 0; c < 4; ++c) {
+      const float bb = bias[ng * 4 + c];
+      float o[RT];
+#pragma unroll
+      for (int r = 0; r < RT; ++r) o[r] = tanhf(acc[r][c] + bb);
+      store_rt<RT>(outT + (ng * 4 + c) * LD + eg * RT, o);
     }
   }
 }
@@ -79,9 +132,10 @@ __global__ void ppo_advstats_kernel(const float* __restrict__ adv, int64_t N, in
 template <int TE, int K, int N, int LD, int RT>
 __device__ __forceinline__ void dense_bwd_inplace(const float* __restrict__ inT, const float* __restrict__ W,
                                                   float* hT) {
-  constexpr int EG = TE / RT, NG = N / 4;
-  for (int j = threadIdx.x; j < EG * NG; j += blockDim.x) {
-    const int eg = j % EG, ng = j / EG;
+  constexpr int JOBS = (TE / RT) * (N / 4);
+  for (int j = threadIdx.x; j < JOBS; j += blockDim.x) {
+    int eg, ng;
+    if (!dense_job<TE, N, RT>(j, eg, ng)) continue;
     float acc[RT][4];
 #pragma unroll
     for (int r = 0; r < RT; ++r)
@@ -197,7 +251,7 @@ struct PpoArgs {
   const float* adv;
   const float* ret;
   const float* params;
-  const float* params_t;  // W1, W2, V1, V2 stored transposed ([in][out]) at their own offsets
+  const float* img;       // [2][RoleImage::SIZE] policy and value weight images
   Feistel perm;
   int64_t start;
   int cnt;
@@ -207,33 +261,53 @@ struct PpoArgs {
   float* stat_partial;  // [2*NC][8]
   float* grad_out;      // [P] reduced gradient (persistent kernel)
   int NC, slices_per_cta;
-  int64_t P;
+  int64_t P, PS;  // parameters; row stride of the partial-sum matrix
 };
 
-// Transposed copy of an updated parameter, for the hidden-layer matrices.
+// Per-role weight image: the prefix of PpoSmem (w1t, w2t, w2, w3, b1, b2,
+// b3[8]) as it sits in shared memory, kept up to date by the Adam phase so
+// that a gradient CTA loads its weights as one contiguous float4 copy.
+// Image 0 is the policy network, image 1 the value network (its head is row
+// 0 of w3 and b3[0]).
 template <int D, int H, int A>
-__device__ __forceinline__ void store_transposed(float* pt, int64_t p, float val) {
+struct RoleImage {
+  static constexpr int64_t W1T = 0, W2T = W1T + (int64_t)D * H, W2 = W2T + (int64_t)H * H,
+                           W3 = W2 + (int64_t)H * H, B1 = W3 + (int64_t)A * H, B2 = B1 + H, B3 = B2 + H,
+                           SIZE = B3 + 8;
+  static_assert(SIZE % 4 == 0, "role image is copied as float4");
+};
+
+template <int D, int H, int A>
+__device__ __forceinline__ void store_image(float* img, int64_t p, float val) {
+  using I = RoleImage<D, H, A>;
   const MlpLayout L = mlp_layout(D, H, A);
-  if (p < L.b1) {
-    const int64_t q = p - L.w1;
-    pt[L.w1 + (q % D) * H + q / D] = val;
-  } else if (p >= L.w2 && p < L.b2) {
-    const int64_t q = p - L.w2;
-    pt[L.w2 + (q % H) * H + q / H] = val;
-  } else if (p >= L.v1 && p < L.c1) {
-    const int64_t q = p - L.v1;
-    pt[L.v1 + (q % D) * H + q / D] = val;
-  } else if (p >= L.v2 && p < L.c2) {
-    const int64_t q = p - L.v2;
-    pt[L.v2 + (q % H) * H + q / H] = val;
+  const bool pol = p < L.v1;
+  float* m = img + (pol ? 0 : I::SIZE);
+  const int64_t w1 = pol ? L.w1 : L.v1, b1 = pol ? L.b1 : L.c1, w2 = pol ? L.w2 : L.v2,
+                b2 = pol ? L.b2 : L.c2, w3 = pol ? L.w3 : L.v3, b3 = pol ? L.b3 : L.c3;
+  if (p < b1) {
+    const int64_t q = p - w1;                       // W1[n][k], n = q / D, k = q % D
+    m[I::W1T + (q % D) * H + q / D] = val;
+  } else if (p < w2) {
+    m[I::B1 + (p - b1)] = val;
+  } else if (p < b2) {
+    const int64_t q = p - w2;                       // W2[n][k], n = q / H, k = q % H
+    m[I::W2T + (q % H) * H + q / H] = val;
+    m[I::W2 + q] = val;
+  } else if (p < w3) {
+    m[I::B2 + (p - b2)] = val;
+  } else if (p < b3) {
+    m[I::W3 + (p - w3)] = val;
+  } else {
+    m[I::B3 + (p - b3)] = val;
   }
 }
 
 template <int D, int H, int A>
-__global__ void ppo_transpose_kernel(const float* __restrict__ params, float* __restrict__ pt) {
+__global__ void ppo_image_kernel(const float* __restrict__ params, float* __restrict__ img) {
   const int64_t P = mlp_layout(D, H, A).total;
   for (int64_t p = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; p < P; p += (int64_t)gridDim.x * blockDim.x)
-    store_transposed<D, H, A>(pt, p, params[p]);
+    store_image<D, H, A>(img, p, params[p]);
 }
 
 // One role (policy or value network) of the minibatch gradient over this
@@ -250,19 +324,26 @@ __device__ __forceinline__ void ppo_role(PpoSmem<D, H, A>& s, const PpoArgs& g, 
   const int64_t oW2 = POL ? Lp.w2 : Lp.v2, oB2 = POL ? Lp.b2 : Lp.c2;
   const int64_t oW3 = POL ? Lp.w3 : Lp.v3, oB3 = POL ? Lp.b3 : Lp.c3;
   const int tid = threadIdx.x;
-  // parameters are read through L2 (not the non-coherent L1 path): inside the
-  // persistent update other CTAs rewrite them between minibatches
-  for (int i = tid; i < H * D; i += blockDim.x) s.w1t[i] = __ldcg(g.params_t + oW1 + i);
-  for (int i = tid; i < H * H; i += blockDim.x) {
-    s.w2t[i] = __ldcg(g.params_t + oW2 + i);
-    s.w2[i] = __ldcg(g.params + oW2 + i);
+  // the role's weight image, read through L2 (not the non-coherent L1 path):
+  // inside the persistent update other CTAs rewrite it between minibatches.
+  // Four float4 loads per thread are in flight before they are stored.
+  {
+    using I = RoleImage<D, H, A>;
+    using Sm = PpoSmem<D, H, A>;
+    static_assert(offsetof(Sm, b3) == sizeof(float) * (size_t)I::B3, "image matches shared memory");
+    const float4* src = reinterpret_cast<const float4*>(g.img + (POL ? 0 : I::SIZE));
+    float4* dst = reinterpret_cast<float4*>(s.w1t);
+    constexpr int N4 = (int)(I::SIZE / 4), U = 4;
+    for (int i0 = tid; i0 < N4; i0 += U * kPpoNT) {
+      float4 v[U];
+#pragma unroll
+      for (int u = 0; u < U; ++u)
+        if (i0 + u * kPpoNT < N4) v[u] = __ldcg(src + i0 + u * kPpoNT);
+#pragma unroll
+      for (int u = 0; u < U; ++u)
+        if (i0 + u * kPpoNT < N4) dst[i0 + u * kPpoNT] = v[u];
+    }
   }
-  for (int i = tid; i < H; i += blockDim.x) {
-    s.b1[i] = __ldcg(g.params + oB1 + i);
-    s.b2[i] = __ldcg(g.params + oB2 + i);
-  }
-  for (int i = tid; i < NA * H; i += blockDim.x) s.w3[i] = __ldcg(g.params + oW3 + i);
-  for (int i = tid; i < NA; i += blockDim.x) s.b3[i] = __ldcg(g.params + oB3 + i);
   const float2 as = *g.advstat;
 
   WGradAcc<H, H, kPpoNT> g2;
@@ -312,9 +393,9 @@ __device__ __forceinline__ void ppo_role(PpoSmem<D, H, A>& s, const PpoArgs& g, 
     }
     __syncthreads();
     // forward
-    dense_tanh_t<S, D, H, LD, kPpoRT>(s.xt, s.w1t, s.b1, s.h1t);
+    dense_fwd_w<S, D, H, LD, kPpoRT>(s.xt, s.w1t, s.b1, s.h1t);
     __syncthreads();
-    dense_tanh_t<S, H, H, LD, kPpoRT>(s.h1t, s.w2t, s.b2, s.h2t);
+    dense_fwd_w<S, H, H, LD, kPpoRT>(s.h1t, s.w2t, s.b2, s.h2t);
     __syncthreads();
     // head: 4 interleaved K-parts per output in adjacent lanes, shuffle-combined
     {
@@ -422,7 +503,7 @@ __device__ __forceinline__ void ppo_role(PpoSmem<D, H, A>& s, const PpoArgs& g, 
     }
   }
   // partial gradient row of this CTA (its network's slice of the parameter vector)
-  float* row = g.partial + (int64_t)c * g.P;
+  float* row = g.partial + (int64_t)c * g.PS;
   g1.store(row + oW1);
   g2.store(row + oW2);
 #pragma unroll
@@ -486,14 +567,14 @@ struct PpoLoop {
   int64_t N;
   int minibatch, nmb, epochs;
   float* params;
-  float* pt;               // transposed hidden-layer matrices (PpoArgs::params_t)
+  float* img;              // role weight images (PpoArgs::img), rewritten by the Adam phase
   float* m;
   float* v;
-  double* sq;              // [gridDim.x]
+  float* sq;               // [gridDim.x] per-CTA sums of squares
   double* acc;             // [8] running statistics
   unsigned int* bar;       // [2]: arrival count, generation
   int32_t* err;
-  double* bc;              // [2 * steps]: step_size, 1/sqrt(bc2) per Adam step
+  const float* bc;         // [2 * steps]: step_size, 1/sqrt(bc2) per Adam step
   float beta1, beta2, eps, max_norm;
 };
 
@@ -531,14 +612,13 @@ __global__ void __launch_bounds__(kPpoNT, 1) ppo_persistent_kernel(PpoLoop L) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   PpoSmem<D, H, A>& s = *reinterpret_cast<PpoSmem<D, H, A>*>(smem_raw);
   __shared__ int s_ok;
-  __shared__ double s_part[4][128];
-  __shared__ double s_red[kPpoNT / 32];
-  __shared__ double s_norm;
+  __shared__ float s_red[kPpoNT / 32];
+  __shared__ float s_norm;
   const int NC = L.g.NC, tid = threadIdx.x;
   const int64_t P = L.g.P;
-  const int64_t per = (P + gridDim.x - 1) / gridDim.x;
+  const int64_t PS = L.g.PS;
+  const int64_t per = ((P + gridDim.x - 1) / gridDim.x + 3) / 4 * 4;
   const int64_t p0 = (int64_t)blockIdx.x * per, p1 = p0 + per < P ? p0 + per : P;
-  const int pl = tid & 127, rg = tid >> 7;  // 4 row groups x 128 parameter lanes
   int step = 0;
   for (int ep = 0; ep < L.epochs; ++ep) {
     for (int mb = 0; mb < L.nmb; ++mb, ++step) {
@@ -559,26 +639,48 @@ __global__ void __launch_bounds__(kPpoNT, 1) ppo_persistent_kernel(PpoLoop L) {
         if (tid == 0) atomicExch(L.err, 1);
         return;
       }
-      // phase 2: grad[p] = sum_c partial[c][p] in row order (4 row groups,
-      // combined in group order), and this CTA's sum of squares
-      double q = 0.0;
-      for (int64_t pb = p0; pb < p1; pb += 128) {
-        const int64_t p = pb + pl;
-        double gs = 0.0;
-        if (p < p1) {
-#pragma unroll 4
-          for (int c = rg; c < NC; c += 4) gs += (double)__ldcg(g.partial + (int64_t)c * P + p);
+      // phase 2: grad[p] = sum_c partial[c][p] in a fixed order (row group
+      // rg = c % 8 summed in row order, then the groups in order), and this
+      // CTA's sum of squares.  64 float4 columns x 8 row groups per pass; the
+      // dead h1 slice buffer holds the group sums.
+      float q = 0.0f;
+      {
+        float* part = s.h1t;
+        const int c4 = tid & 63, rg = tid >> 6;
+        for (int64_t pb = p0; pb < p1; pb += 256) {
+          const int64_t p = pb + 4 * c4;
+          float4 acc4 = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+          if (p < p1) {
+#pragma unroll
+            for (int h = 0; h < 8; h += 4) {
+              float4 v[4];
+#pragma unroll
+              for (int u = 0; u < 4; ++u)
+                if (rg + 8 * (h + u) < NC)
+                  v[u] = __ldcg(reinterpret_cast<const float4*>(g.partial + (int64_t)(rg + 8 * (h + u)) * PS + p));
+#pragma unroll
+              for (int u = 0; u < 4; ++u)
+                if (rg + 8 * (h + u) < NC) {
+                  acc4.x += v[u].x;
+                  acc4.y += v[u].y;
+                  acc4.z += v[u].z;
+                  acc4.w += v[u].w;
+                }
+            }
+          }
+          *reinterpret_cast<float4*>(part + rg * 256 + 4 * c4) = acc4;
+          __syncthreads();
+          if (tid < 256 && pb + tid < p1) {
+            float gs = 0.0f;
+#pragma unroll
+            for (int r = 0; r < 8; ++r) gs += part[r * 256 + tid];
+            L.g.grad_out[pb + tid] = gs;
+            q = fmaf(gs, gs, q);
+          }
+          __syncthreads();
         }
-        s_part[rg][pl] = gs;
-        __syncthreads();
-        if (rg == 0 && p < p1) {
-          const float gf = (float)(((s_part[0][pl] + s_part[1][pl]) + s_part[2][pl]) + s_part[3][pl]);
-          L.g.grad_out[p] = gf;
-          q += (double)gf * (double)gf;
-        }
-        __syncthreads();
       }
-      const double qb = block_sum_d(q, s_red);
+      const float qb = block_sum_f(q, s_red);
       if (tid == 0) L.sq[blockIdx.x] = qb;
       if (blockIdx.x == 0 && tid < 32) {
         double v[5] = {0, 0, 0, 0, 0};
@@ -609,16 +711,16 @@ __global__ void __launch_bounds__(kPpoNT, 1) ppo_persistent_kernel(PpoLoop L) {
       }
       // phase 3: global norm (fixed order), clip factor, Adam on this slice
       if (tid < 32) {
-        double t = 0.0;
+        float t = 0.0f;
         for (int b = tid; b < (int)gridDim.x; b += 32) t += __ldcg(L.sq + b);
 #pragma unroll
         for (int o = 16; o > 0; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
-        if (tid == 0) s_norm = sqrt(t);
+        if (tid == 0) s_norm = sqrtf(t);
       }
       __syncthreads();
-      const double norm = s_norm;
-      const float coef = (float)fmin(1.0, (double)L.max_norm / (norm + 1e-6));
-      const float step_size = (float)L.bc[2 * step], inv_sqrt_bc2 = (float)L.bc[2 * step + 1];
+      const float norm = s_norm;
+      const float coef = fminf(1.0f, L.max_norm / (norm + 1e-6f));
+      const float step_size = L.bc[2 * step], inv_sqrt_bc2 = L.bc[2 * step + 1];
       for (int64_t p = p0 + tid; p < p1; p += blockDim.x) {
         const float gp = L.g.grad_out[p] * coef;
         const float mp = L.beta1 * L.m[p] + (1.0f - L.beta1) * gp;
@@ -627,7 +729,7 @@ __global__ void __launch_bounds__(kPpoNT, 1) ppo_persistent_kernel(PpoLoop L) {
         L.v[p] = vp;
         const float np = L.params[p] - step_size * mp / (sqrtf(vp) * inv_sqrt_bc2 + L.eps);
         L.params[p] = np;
-        store_transposed<D, H, A>(L.pt, p, np);
+        store_image<D, H, A>(L.img, p, np);
       }
       if (blockIdx.x == 0 && tid == 0) {
         L.acc[6] = norm;
@@ -652,33 +754,32 @@ struct ReduceArgs {
   const float* partial;
   const float* stat_partial;  // [2*NC][8]
   int NC;
-  int64_t P;
+  int64_t P, PS;
   float* grad;
-  double* sq;             // [gridDim.x]
+  float* sq;              // [gridDim.x]
   unsigned int* ticket;   // zeroed before the first launch; the last block re-zeroes it
-  double* norm;           // [1] out
+  float* norm;            // [1] out
   double* acc;            // [8] running statistics
   float vf_coef, ent_coef, inv_cnt;
 };
 
 __global__ void __launch_bounds__(kRedP * kRedG) ppo_reduce_kernel(ReduceArgs a) {
-  __shared__ double part[kRedG][kRedP];
-  __shared__ double red[kRedG];
+  __shared__ float part[kRedG][kRedP];
+  __shared__ float red[kRedG];
   __shared__ bool last;
   const int lp = threadIdx.x % kRedP, cg = threadIdx.x / kRedP;
   const int64_t p = (int64_t)blockIdx.x * kRedP + lp;
-  double s = 0.0;
+  float s = 0.0f;
   if (p < a.P)
-    for (int c = cg; c < a.NC; c += kRedG) s += (double)__ldg(a.partial + (int64_t)c * a.P + p);
+    for (int c = cg; c < a.NC; c += kRedG) s += __ldg(a.partial + (int64_t)c * a.PS + p);
   part[cg][lp] = s;
   __syncthreads();
   if (cg == 0) {
-    double g = 0.0;
+    float g = 0.0f;
 #pragma unroll
     for (int k = 0; k < kRedG; ++k) g += part[k][lp];
-    const float gf = (float)g;
-    if (p < a.P) a.grad[p] = gf;
-    double q = p < a.P ? (double)gf * (double)gf : 0.0;
+    if (p < a.P) a.grad[p] = g;
+    float q = p < a.P ? g * g : 0.0f;
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) q += __shfl_xor_sync(0xffffffffu, q, o);
     if (lp == 0) {
@@ -692,8 +793,8 @@ __global__ void __launch_bounds__(kRedP * kRedG) ppo_reduce_kernel(ReduceArgs a)
   if (!last) return;
   __threadfence();
   // last block: global norm (fixed order: strided partial sums, then warp tree)
-  double q = 0.0;
-  for (int b = threadIdx.x; b < (int)gridDim.x; b += blockDim.x) q += *((volatile double*)a.sq + b);
+  float q = 0.0f;
+  for (int b = threadIdx.x; b < (int)gridDim.x; b += blockDim.x) q += *((volatile float*)a.sq + b);
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) q += __shfl_xor_sync(0xffffffffu, q, o);
   if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = q;
@@ -713,9 +814,9 @@ __global__ void __launch_bounds__(kRedP * kRedG) ppo_reduce_kernel(ReduceArgs a)
 #pragma unroll
       for (int o = 16; o > 0; o >>= 1) v[k] += __shfl_xor_sync(0xffffffffu, v[k], o);
     if (threadIdx.x == 0) {
-      double t = 0.0;
+      float t = 0.0f;
       for (int k = 0; k < kRedG; ++k) t += red[k];
-      const double norm = sqrt(t);
+      const float norm = sqrtf(t);
       *a.norm = norm;
       const double ic = a.inv_cnt;
       a.acc[0] += v[0] * ic;
@@ -736,11 +837,11 @@ struct AdamArgs {
 };
 
 template <int D, int H, int A>
-__global__ void ppo_adam_kernel(float* __restrict__ params, float* __restrict__ pt, float* __restrict__ m,
+__global__ void ppo_adam_kernel(float* __restrict__ params, float* __restrict__ img, float* __restrict__ m,
                                 float* __restrict__ v, const float* __restrict__ grad,
-                                const double* __restrict__ norm_p, int64_t P, AdamArgs a) {
-  const double norm = *norm_p;
-  const float coef = (float)fmin(1.0, (double)a.max_norm / (norm + 1e-6));
+                                const float* __restrict__ norm_p, int64_t P, AdamArgs a) {
+  const float norm = *norm_p;
+  const float coef = fminf(1.0f, a.max_norm / (norm + 1e-6f));
   for (int64_t p = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; p < P;
        p += (int64_t)gridDim.x * blockDim.x) {
     const float gp = grad[p] * coef;
@@ -750,7 +851,7 @@ __global__ void ppo_adam_kernel(float* __restrict__ params, float* __restrict__ 
     v[p] = vp;
     const float np = params[p] - a.step_size * mp / (sqrtf(vp) * a.inv_sqrt_bc2 + a.eps);
     params[p] = np;
-    store_transposed<D, H, A>(pt, p, np);
+    store_image<D, H, A>(img, p, np);
   }
 }
 
@@ -786,14 +887,21 @@ Feistel make_feistel(uint64_t n, uint64_t seed, uint32_t epoch, uint32_t iterati
 struct PpoPlan {
   int64_t P, N;
   int nmb, NC, slices_per_cta, nsq, steps;
-  int64_t off_advstat, off_partial, off_stat, off_grad, off_pt, off_sq, off_acc, off_bar, off_bc, total;
+  int64_t PS;  // row stride of the partial-sum matrix (P rounded up to 4)
+  int64_t off_advstat, off_partial, off_stat, off_grad, off_img, off_sq, off_acc, off_bar, off_bc, total;
 };
 
 static int64_t align256(int64_t x) { return (x + 255) / 256 * 256; }
 
+static int64_t img_floats(const pe_net& net) {
+  const int64_t D = net.obs_dim, H = net.hidden, A = net.n_actions;
+  return D * H + 2 * H * H + A * H + 2 * H + 8;
+}
+
 static PpoPlan ppo_plan(const pe_net& net, const pe_ppo_config& cfg, int64_t N) {
   PpoPlan p;
   p.P = mlp_layout(net.obs_dim, net.hidden, net.n_actions).total;
+  p.PS = (p.P + 3) / 4 * 4;
   p.N = N;
   p.nmb = (int)((N + cfg.minibatch - 1) / cfg.minibatch);
   const int slices = (cfg.minibatch + kPpoS - 1) / kPpoS;
@@ -803,14 +911,14 @@ static PpoPlan ppo_plan(const pe_net& net, const pe_ppo_config& cfg, int64_t N) 
   p.steps = cfg.epochs * p.nmb;
   int64_t o = 0;
   p.off_advstat = o; o = align256(o + (int64_t)cfg.epochs * p.nmb * 8);
-  p.off_partial = o; o = align256(o + (int64_t)p.NC * p.P * 4);
+  p.off_partial = o; o = align256(o + (int64_t)p.NC * p.PS * 4);
   p.off_stat = o; o = align256(o + (int64_t)2 * p.NC * 8 * 4);
   p.off_grad = o; o = align256(o + p.P * 4);
-  p.off_pt = o; o = align256(o + p.P * 4);
+  p.off_img = o; o = align256(o + 2 * img_floats(net) * 4);
   p.off_sq = o; o = align256(o + (int64_t)(p.nsq > 2 * p.NC ? p.nsq : 2 * p.NC) * 8);
   p.off_acc = o; o = align256(o + 8 * 8 + 16);
   p.off_bar = o; o = align256(o + 16);
-  p.off_bc = o; o = align256(o + (int64_t)p.steps * 16);
+  p.off_bc = o; o = align256(o + (int64_t)p.steps * 8);
   p.total = o;
   return p;
 }
@@ -843,10 +951,10 @@ static pe_status ppo_run(const pe_net& net, float* params, float* m, float* v, i
   float* partial = reinterpret_cast<float*>(ws + pl.off_partial);
   float* stat_partial = reinterpret_cast<float*>(ws + pl.off_stat);
   float* grad = reinterpret_cast<float*>(ws + pl.off_grad);
-  float* pt = reinterpret_cast<float*>(ws + pl.off_pt);
-  double* sq = reinterpret_cast<double*>(ws + pl.off_sq);
+  float* img = reinterpret_cast<float*>(ws + pl.off_img);
+  float* sq = reinterpret_cast<float*>(ws + pl.off_sq);
   double* acc = reinterpret_cast<double*>(ws + pl.off_acc);
-  double* norm = acc + 8;
+  float* norm = reinterpret_cast<float*>(acc + 8);
   unsigned int* ticket = reinterpret_cast<unsigned int*>(acc + 9);
   PE_TRY_CUDA(cudaMemsetAsync(acc, 0, 8 * sizeof(double) + 16, st));
   FeistelSet perms{};
@@ -858,9 +966,9 @@ static pe_status ppo_run(const pe_net& net, float* params, float* m, float* v, i
   PE_CHECK_LAUNCH("ppo_advstats_kernel");
   {
     ProfScope ps(PE_PROF_PPO_OTHER, st);
-    ppo_transpose_kernel<D, H, A><<<ceil_div(pl.P, 256), 256, 0, st>>>(params, pt);
+    ppo_image_kernel<D, H, A><<<ceil_div(pl.P, 256), 256, 0, st>>>(params, img);
   }
-  PE_CHECK_LAUNCH("ppo_transpose_kernel");
+  PE_CHECK_LAUNCH("ppo_image_kernel");
   using Smem = PpoSmem<D, H, A>;
   auto kern = ppo_grad_kernel<D, H, A>;
   const int bytes = (int)sizeof(Smem);
@@ -878,14 +986,14 @@ static pe_status ppo_run(const pe_net& net, float* params, float* m, float* v, i
   PE_TRY_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, pk, kPpoNT, bytes));
   PE_TRY_CUDA(cudaDeviceGetAttribute(&coop, cudaDevAttrCooperativeLaunch, dev));
   if (coop && per_sm * sms >= 2 * pl.NC) {
-    std::vector<double> bc(2 * (size_t)pl.steps);
+    std::vector<float> bc(2 * (size_t)pl.steps);
     for (int k = 0; k < pl.steps; ++k) {
       const double tt = (double)(adam_t + k + 1);
-      bc[2 * k] = cfg.lr / (1.0 - std::pow((double)cfg.beta1, tt));
-      bc[2 * k + 1] = 1.0 / std::sqrt(1.0 - std::pow((double)cfg.beta2, tt));
+      bc[2 * k] = (float)(cfg.lr / (1.0 - std::pow((double)cfg.beta1, tt)));
+      bc[2 * k + 1] = (float)(1.0 / std::sqrt(1.0 - std::pow((double)cfg.beta2, tt)));
     }
-    double* bc_dev = reinterpret_cast<double*>(ws + pl.off_bc);
-    PE_TRY_CUDA(cudaMemcpyAsync(bc_dev, bc.data(), bc.size() * sizeof(double), cudaMemcpyHostToDevice, st));
+    float* bc_dev = reinterpret_cast<float*>(ws + pl.off_bc);
+    PE_TRY_CUDA(cudaMemcpyAsync(bc_dev, bc.data(), bc.size() * sizeof(float), cudaMemcpyHostToDevice, st));
     PpoLoop L;
     L.g.obs = obs;
     L.g.act = act;
@@ -893,8 +1001,8 @@ static pe_status ppo_run(const pe_net& net, float* params, float* m, float* v, i
     L.g.adv = adv;
     L.g.ret = ret;
     L.g.params = params;
-    L.g.params_t = pt;
-    L.pt = pt;
+    L.g.img = img;
+    L.img = img;
     L.g.clip = cfg.clip;
     L.g.vf_coef = cfg.vf_coef;
     L.g.ent_coef = cfg.ent_coef;
@@ -904,6 +1012,7 @@ static pe_status ppo_run(const pe_net& net, float* params, float* m, float* v, i
     L.g.NC = pl.NC;
     L.g.slices_per_cta = pl.slices_per_cta;
     L.g.P = pl.P;
+    L.g.PS = pl.PS;
     L.advstat = advstat;
     L.perms = perms;
     L.N = N;
@@ -941,7 +1050,7 @@ static pe_status ppo_run(const pe_net& net, float* params, float* m, float* v, i
         g.adv = adv;
         g.ret = ret;
         g.params = params;
-        g.params_t = pt;
+        g.img = img;
         g.perm = perms.f[ep];
         g.start = start;
         g.cnt = cnt;
@@ -954,6 +1063,7 @@ static pe_status ppo_run(const pe_net& net, float* params, float* m, float* v, i
         g.NC = pl.NC;
         g.slices_per_cta = pl.slices_per_cta;
         g.P = pl.P;
+        g.PS = pl.PS;
         g.advstat = advstat + (int64_t)ep * pl.nmb + mb;
         {
           ProfScope ps(PE_PROF_PPO_GRAD, st);
@@ -967,6 +1077,7 @@ static pe_status ppo_run(const pe_net& net, float* params, float* m, float* v, i
           ra.stat_partial = stat_partial;
           ra.NC = pl.NC;
           ra.P = pl.P;
+          ra.PS = pl.PS;
           ra.grad = grad;
           ra.sq = sq;
           ra.ticket = ticket;
@@ -990,7 +1101,7 @@ static pe_status ppo_run(const pe_net& net, float* params, float* m, float* v, i
         a.max_norm = cfg.max_grad_norm;
         {
           ProfScope ps(PE_PROF_PPO_ADAM, st);
-          ppo_adam_kernel<D, H, A><<<(int)((pl.P + 255) / 256), 256, 0, st>>>(params, pt, m, v, grad, norm, pl.P, a);
+          ppo_adam_kernel<D, H, A><<<(int)((pl.P + 255) / 256), 256, 0, st>>>(params, img, m, v, grad, norm, pl.P, a);
         }
         PE_CHECK_LAUNCH("ppo_adam_kernel");
       }
