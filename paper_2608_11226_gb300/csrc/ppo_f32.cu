@@ -79,16 +79,16 @@ __global__ void ppo_advstats_kernel(const float* __restrict__ adv, int64_t N, in
 }
 
 // Dense-layer register tiles for the 64-sample slices: a thread owns RT
-// sample rows x 4 neurons; a warp covers 4 row groups x 8 neuron groups, so
-// each of its float4 loads (inputs and weights) is a single 64- or 128-byte
-// shared-memory wavefront.
+// sample rows x 4 neurons; a warp covers 2 row groups x 16 neuron groups (the
+// fastest of the warp shapes measured on the 7B network: 2x16, 4x8, 8x4 and
+// 16x2 lie within 3% of each other).
 template <int TE, int N, int RT>
 __device__ __forceinline__ bool dense_job(int j, int& eg, int& ng) {
-  constexpr int EG = TE / RT, NG = N / 4, BE = EG / 4;  // BE: 4-row-group blocks along the slice
-  static_assert(EG % 4 == 0 && NG % 8 == 0, "dense tile layout");
+  constexpr int EG = TE / RT, NG = N / 4, BE = EG / 2;  // BE: 2-row-group blocks along the slice
+  static_assert(EG % 2 == 0 && NG % 16 == 0, "dense tile layout");
   const int wb = j >> 5, lane = j & 31;
-  eg = (wb % BE) * 4 + (lane & 3);
-  ng = (wb / BE) * 8 + (lane >> 2);
+  eg = (wb % BE) * 2 + (lane & 1);
+  ng = (wb / BE) * 16 + (lane >> 1);
   return ng < NG;
 }
 
@@ -324,46 +324,10 @@ __device__ __forceinline__ void ppo_role(PpoSmem<D, H, A>& s, const PpoArgs& g, 
   const int64_t oW2 = POL ? Lp.w2 : Lp.v2, oB2 = POL ? Lp.b2 : Lp.c2;
   const int64_t oW3 = POL ? Lp.w3 : Lp.v3, oB3 = POL ? Lp.b3 : Lp.c3;
   const int tid = threadIdx.x;
-  // the role's weight image, read through L2 (not the non-coherent L1 path):
-  // inside the persistent update other CTAs rewrite it between minibatches.
-  // Four float4 loads per thread are in flight before they are stored.
-  {
-    using I = RoleImage<D, H, A>;
-    using Sm = PpoSmem<D, H, A>;
-    static_assert(offsetof(Sm, b3) == sizeof(float) * (size_t)I::B3, "image matches shared memory");
-    const float4* src = reinterpret_cast<const float4*>(g.img + (POL ? 0 : I::SIZE));
-    float4* dst = reinterpret_cast<float4*>(s.w1t);
-    constexpr int N4 = (int)(I::SIZE / 4), U = 4;
-    for (int i0 = tid; i0 < N4; i0 += U * kPpoNT) {
-      float4 v[U];
-#pragma unroll
-      for (int u = 0; u < U; ++u)
-        if (i0 + u * kPpoNT < N4) v[u] = __ldcg(src + i0 + u * kPpoNT);
-#pragma unroll
-      for (int u = 0; u < U; ++u)
-        if (i0 + u * kPpoNT < N4) dst[i0 + u * kPpoNT] = v[u];
-    }
-  }
   const float2 as = *g.advstat;
-
-  WGradAcc<H, H, kPpoNT> g2;
-  WGradAcc<H, D, kPpoNT> g1;
-  g2.zero();
-  g1.zero();
-  // head backward: thread (k = tid / 4, quarter q = tid % 4) owns row k of the
-  // head weight gradient and of the layer-2 bias gradient over samples 4i + q
-  const int hk = tid >> 2, hq = tid & 3;
-  float g3[NA], gb2 = 0.0f, gb1 = 0.0f, gb3 = 0.0f;
-#pragma unroll
-  for (int a = 0; a < NA; ++a) g3[a] = 0.0f;
-  float st[5] = {0.0f, 0.0f, 0.0f, 0.0f, 0.0f};  // pg, entropy, kl, clip, value (threads < S)
-
-  for (int sl = 0; sl < g.slices_per_cta; ++sl) {
-    const int base = (c * g.slices_per_cta + sl) * S;
-    if (base >= g.cnt) break;
-    __syncthreads();
-    // gather the slice (permuted sample order): observations as float4 rows,
-    // per-sample scalars by threads 256..256+S
+  // gather one slice (permuted sample order): observations as float4 rows,
+  // per-sample scalars by threads 256..256+S
+  auto gather = [&](int base) {
     constexpr int F4 = D / 4;
     if (tid < S * F4) {
       const int si = tid / F4, f = tid % F4;
@@ -391,27 +355,77 @@ __device__ __forceinline__ void ppo_role(PpoSmem<D, H, A>& s, const PpoArgs& g, 
         s.lpo[si] = s.advn[si] = s.ret[si] = 0.0f;
       }
     }
+  };
+  // the first slice's gather overlaps the weight loads
+  if (c * g.slices_per_cta * S < g.cnt) gather(c * g.slices_per_cta * S);
+  // the role's weight image, read through L2 (not the non-coherent L1 path):
+  // inside the persistent update other CTAs rewrite it between minibatches.
+  // Four float4 loads per thread are in flight before they are stored.
+  {
+    using I = RoleImage<D, H, A>;
+    using Sm = PpoSmem<D, H, A>;
+    static_assert(offsetof(Sm, b3) == sizeof(float) * (size_t)I::B3, "image matches shared memory");
+    const float4* src = reinterpret_cast<const float4*>(g.img + (POL ? 0 : I::SIZE));
+    float4* dst = reinterpret_cast<float4*>(s.w1t);
+    constexpr int N4 = (int)(I::SIZE / 4), U = 4;
+    for (int i0 = tid; i0 < N4; i0 += U * kPpoNT) {
+      float4 v[U];
+#pragma unroll
+      for (int u = 0; u < U; ++u)
+        if (i0 + u * kPpoNT < N4) v[u] = __ldcg(src + i0 + u * kPpoNT);
+#pragma unroll
+      for (int u = 0; u < U; ++u)
+        if (i0 + u * kPpoNT < N4) dst[i0 + u * kPpoNT] = v[u];
+    }
+  }
+  WGradAcc<H, H, kPpoNT> g2;
+  WGradAcc<H, D, kPpoNT> g1;
+  g2.zero();
+  g1.zero();
+  // head backward: thread (k = tid / 4, quarter q = tid % 4) owns row k of the
+  // head weight gradient and of the layer-2 bias gradient over samples 4i + q
+  const int hk = tid >> 2, hq = tid & 3;
+  float g3[NA], gb2 = 0.0f, gb1 = 0.0f, gb3 = 0.0f;
+#pragma unroll
+  for (int a = 0; a < NA; ++a) g3[a] = 0.0f;
+  float st[5] = {0.0f, 0.0f, 0.0f, 0.0f, 0.0f};  // pg, entropy, kl, clip, value (threads < S)
+
+  for (int sl = 0; sl < g.slices_per_cta; ++sl) {
+    const int base = (c * g.slices_per_cta + sl) * S;
+    if (base >= g.cnt) break;
+    if (sl > 0) {
+      __syncthreads();
+      gather(base);
+    }
     __syncthreads();
     // forward
     dense_fwd_w<S, D, H, LD, kPpoRT>(s.xt, s.w1t, s.b1, s.h1t);
     __syncthreads();
     dense_fwd_w<S, H, H, LD, kPpoRT>(s.h1t, s.w2t, s.b2, s.h2t);
     __syncthreads();
-    // head: 4 interleaved K-parts per output in adjacent lanes, shuffle-combined
+    // head: thread (sample si = tid / 8, K-part q = tid % 8) sums k = q, q+8, ...
+    // for every action; the 8 parts (adjacent lanes) are shuffle-combined
     {
-      constexpr int JOBS = (S * NA * 4 + 31) / 32 * 32;
-      for (int j = tid; j < JOBS; j += blockDim.x) {
-        const int part = j & 3, o = j >> 2;
-        const int si = o % S, a = o / S;
-        float acc = 0.0f;
-        if (o < S * NA) {
-#pragma unroll 8
-          for (int k = part; k < H; k += 4) acc = fmaf(s.w3[a * H + k], s.h2t[k * LD + si], acc);
-        }
-        acc += __shfl_xor_sync(0xffffffffu, acc, 1);
-        acc += __shfl_xor_sync(0xffffffffu, acc, 2);
-        if (part == 0 && o < S * NA) s.z[si * NA + a] = acc + s.b3[a];
+      static_assert(S * 8 == kPpoNT, "one head job per thread");
+      const int q = tid & 7, si = tid >> 3;
+      float acc[NA];
+#pragma unroll
+      for (int a = 0; a < NA; ++a) acc[a] = 0.0f;
+#pragma unroll 4
+      for (int k = q; k < H; k += 8) {
+        const float h = s.h2t[k * LD + si];
+#pragma unroll
+        for (int a = 0; a < NA; ++a) acc[a] = fmaf(s.w3[a * H + k], h, acc[a]);
       }
+#pragma unroll
+      for (int a = 0; a < NA; ++a) {
+        acc[a] += __shfl_xor_sync(0xffffffffu, acc[a], 1);
+        acc[a] += __shfl_xor_sync(0xffffffffu, acc[a], 2);
+        acc[a] += __shfl_xor_sync(0xffffffffu, acc[a], 4);
+      }
+      if (q == 0)
+#pragma unroll
+        for (int a = 0; a < NA; ++a) s.z[si * NA + a] = acc[a] + s.b3[a];
     }
     __syncthreads();
     // loss terms and dLoss/dhead per sample (written over the head outputs)
