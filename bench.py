@@ -17,6 +17,7 @@ divided by the slowest rank's time.
 
 --impl reference times the CPU oracle on a bounded sample of the same
 workload (the paper ships no GPU implementation to compare against).
+--ncu-case NAME runs one small case of a hot kernel, sized for ncu captures.
 """
 from __future__ import annotations
 
@@ -55,6 +56,8 @@ def parse():
     ap.add_argument("--r72b-horizon", type=int, default=1024)
     ap.add_argument("--r72b-ppo-minibatches", type=int, default=16,
                     help="72B PPO minibatch steps of 65,536 samples timed (0: skip)")
+    ap.add_argument("--ncu-case", choices=["ppo7b", "ppo72", "gae", "mlp72", "fleet"], default=None,
+                    help="run one small named case of a hot kernel (for ncu captures) and exit")
     ap.add_argument("--gae-large", type=int, nargs=2, default=[2048, 262144], metavar=("T", "E"),
                     help="GAE roofline size (Stress: 2048 x 262144); T=0 skips it")
     return ap.parse_args()
@@ -122,6 +125,19 @@ def load_traffic(kernel: str):
         return None
     for line in open(path):
         if line.strip().startswith("traffic_bytes_per_launch:"):
+            v = line.split(":", 1)[1].strip()
+            return None if v in ("", "null") else float(v)
+    return None
+
+
+def load_traffic_per_unit(kernel: str, key: str):
+    """dram bytes per unit of work (e.g. per env-step) from the committed ncu
+    summary, for kernels whose traffic grows with the size of the launch."""
+    path = os.path.join(ROOT, "profiles", f"{kernel}.md")
+    if not os.path.exists(path):
+        return None
+    for line in open(path):
+        if line.strip().startswith(key + ":"):
             v = line.split(":", 1)[1].strip()
             return None if v in ("", "null") else float(v)
     return None
@@ -256,9 +272,10 @@ def run_ours(args, world, rank, local):
     peaks = json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json"))) if os.path.exists(
         os.path.join(ROOT, "MEASURED_PEAKS.json")) else {"hbm_gbs": 6800.0}
     hbm = float(peaks.get("hbm_gbs", 6800.0))
+    # inputs just written by the rollout sit in L2 at this size: no DRAM traffic figure
     gae_roof = {"kernel": "gae_kernel", "bound": "hbm", "achieved": gae_gbs, "peak": hbm,
                 "unit": "GB/s", "frac": gae_gbs / hbm if gae_gbs else None,
-                "traffic": load_traffic("gae_kernel")}
+                "traffic": None}
 
     # ---- end to end through host buffers: model state uploaded from pinned
     # host memory every step, parameters + statistics + counters read back
@@ -436,7 +453,7 @@ def run_72b(args, world, peaks):
             "roofline_gae": {"kernel": f"gae_kernel ({T} x {E})", "bound": "hbm", "achieved": gae_gbs,
                              "peak": hbm, "unit": "GB/s", "frac": gae_gbs / hbm if gae_gbs else None,
                              "avg_launch_ms": gms / gn if gn else None,
-                             "traffic": load_traffic("gae_kernel")},
+                             "traffic": gae_traffic(T * E)},
             "ppo_update": ppo72}
 
 
@@ -495,6 +512,13 @@ def run_72b_ppo(args, world, peaks, wl, buf, adv, ret):
             "stats": st}
 
 
+def gae_traffic(env_steps: int):
+    """DRAM bytes of one GAE launch larger than L2, scaled from the committed
+    capture's bytes per env-step."""
+    b = load_traffic_per_unit("gae_kernel", "traffic_bytes_per_env_step")
+    return None if b is None else b * env_steps
+
+
 def run_gae_large(args, world, peaks):
     """GAE alone at the Stress size (2,048 x 262,144 env-steps, 9.1 GB of
     algorithmic traffic), on seeded device-resident inputs."""
@@ -524,7 +548,7 @@ def run_gae_large(args, world, peaks):
     torch.cuda.empty_cache()
     return {"kernel": f"gae_kernel ({T} x {E})", "bound": "hbm", "achieved": gbs, "peak": hbm,
             "unit": "GB/s", "frac": gbs / hbm, "avg_launch_ms": ms,
-            "env_steps_per_s": T * E * world / (ms / 1e3), "traffic": load_traffic("gae_kernel")}
+            "env_steps_per_s": T * E * world / (ms / 1e3), "traffic": gae_traffic(T * E)}
 
 
 # --------------------------------------------------------------------------- CPU oracle
@@ -593,8 +617,80 @@ def run_reference(args, world, rank):
     print(json.dumps(out), flush=True)
 
 
+def run_ncu_case(name: str):
+    """Small cases of the hot kernels, sized for ncu captures (a few GB on the
+    device at most, inputs larger than L2 where DRAM figures matter); each
+    runs its kernel a few times and exits."""
+    from paper_2608_11226_gb300 import build, pe
+    from paper_2608_11226_gb300 import workloads as W
+    build.build()
+    pe.lib()
+    if name in ("ppo7b", "ppo72"):
+        # rollout (32 or 16 steps), GAE, then 3 PPO updates of one epoch (16 minibatch steps each)
+        wl = W.make_7b() if name == "ppo7b" else W.make_72b(n_envs=65536)
+        spec, net = wl.env, wl.net
+        T = 32 if name == "ppo7b" else 16
+        mb = 8192 if name == "ppo7b" else 65536
+        env = pe.Env(spec, torch.from_numpy(wl.trace), torch.from_numpy(wl.phase))
+        buf = pe.alloc_rollout(spec, net, T)
+        params = torch.from_numpy(W.init_params(net, seed=0)).cuda()
+        pe.rollout(env, net, params, T, 0, buf, lam=1.0)
+        adv = torch.empty(T, spec.n_envs, device="cuda")
+        ret = torch.empty_like(adv)
+        pe.gae(buf["reward"], buf["value"], buf["done"], buf["last_value"], 0.99, 0.95, adv, ret)
+        ppo = W.PPOSpec(epochs=1, minibatch=mb, ent_coef=wl.ppo.ent_coef)
+        m = torch.zeros_like(params)
+        v = torch.zeros_like(params)
+        st = torch.zeros(8, device="cuda")
+        ws = pe.alloc_workspace(pe.ppo_workspace_bytes(net, ppo, buf["act"].numel()))
+        steps = (buf["act"].numel() + mb - 1) // mb
+        for it in range(3):
+            pe.ppo_update(net, ppo, params, m, v, it * steps, buf["obs"], buf["act"], buf["logp"], adv, ret,
+                          st, ws, seed=7, iteration=it)
+        env.close()
+    elif name == "gae":
+        T, E = 2048, 16384  # 570 MB of algorithmic traffic per launch
+        g = torch.Generator(device="cuda").manual_seed(0)
+        r = torch.randn(T, E, device="cuda", generator=g)
+        v = torch.randn(T, E, device="cuda", generator=g)
+        d = (torch.rand(T, E, device="cuda", generator=g) < 0.002).to(torch.uint8)
+        lv = torch.randn(E, device="cuda", generator=g)
+        adv = torch.empty(T, E, device="cuda")
+        ret = torch.empty_like(adv)
+        for _ in range(3):
+            pe.gae(r, v, d, lv, 0.99, 0.95, adv, ret)
+    elif name == "mlp72":
+        # two 72B rollouts of 8 steps over 65,536 envs: 8 policy + 2 value launches each
+        wl = W.make_72b(n_envs=65536)
+        spec, net = wl.env, wl.net
+        T = 8
+        env = pe.Env(spec, torch.from_numpy(wl.trace), torch.from_numpy(wl.phase))
+        buf = pe.alloc_rollout(spec, net, T)
+        params = torch.from_numpy(W.init_params(net, seed=0)).cuda()
+        ws = pe.alloc_workspace(pe.rollout_workspace_bytes(env, net))
+        for it in range(2):
+            pe.rollout(env, net, params, T, it, buf, lam=1.0, workspace=ws)
+        pe.device_check()
+        env.close()
+    elif name == "fleet":
+        wl = W.make_fleet(n_compositions=20000)
+        tr = torch.from_numpy(wl.traces).cuda()
+        jg = torch.from_numpy(wl.job_of_gpu).cuda()
+        off = torch.from_numpy(wl.offsets).cuda()
+        cnt = torch.empty(off.shape[0], len(wl.windows), dtype=torch.int32, device="cuda")
+        pk = torch.empty_like(cnt)
+        ws = pe.alloc_workspace(pe.fleet_workspace_bytes(wl.n_jobs, tr.shape[1], wl.horizon))
+        for _ in range(2):
+            pe.fleet_windows(tr, jg, wl.n_jobs, off, wl.horizon, wl.windows, wl.budget_q, cnt, pk, ws)
+    torch.cuda.synchronize()
+    print(json.dumps({"ncu_case": name, "ok": True}), flush=True)
+
+
 def main():
     args = parse()
+    if args.ncu_case:
+        run_ncu_case(args.ncu_case)
+        return
     if args.impl == "reference":
         world = int(os.environ.get("WORLD_SIZE", "1"))
         rank = int(os.environ.get("RANK", "0"))
