@@ -49,6 +49,8 @@ def parse():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--fleet-n", type=int, default=1_000_000)
     ap.add_argument("--fleet-steps", type=int, default=3)
+    ap.add_argument("--stagger-stride", type=int, default=1,
+                    help="candidate offset grid of the greedy staggered schedule (0: skip)")
     ap.add_argument("--cpu-envs", type=int, default=48, help="envs in the oracle CPU sample")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--r72b-steps", type=int, default=2, help="timed 72B rollouts (0: skip)")
@@ -365,6 +367,7 @@ def run_fleet(args, world):
     composed = N * H
     c = counts.cpu().numpy()
     p = peaks.cpu().numpy()
+    stagger = run_stagger(args, world, fw, traces, job, p) if args.stagger_stride > 0 else None
     return {"metric": "fleet window-samples/s", "value": ws_per_call * world * args.fleet_steps / (ms / 1e3),
             "unit": "window-samples/s", "ms_per_call": ms / args.fleet_steps,
             "config": {"workload": "fleet: 16 traces x 380,000 samples (2x72B@4, 2x14B@2, 4x7B@1), "
@@ -376,7 +379,49 @@ def run_fleet(args, world):
             "violation_fraction_mean": [float(c[:, i].mean() / (H - w + 1)) for i, w in enumerate(windows)],
             "peak_fraction_of_nameplate_max": [float(p[:, i].max() / (64.0 * w) / W.FLEET_NAMEPLATE_W)
                                                for i, w in enumerate(windows)],
-            "traffic": load_traffic("fleet_windows_kernel")}
+            "traffic": load_traffic("fleet_windows_kernel"),
+            "strategies": stagger}
+
+
+def run_stagger(args, world, fw, traces, job, peaks_random):
+    """Sec. 8 fleet operating strategies on the same traces: naive aligned
+    starts (composition 0), random starts (the other compositions) and the
+    greedy phase-staggered schedule (pe_fleet_stagger over every
+    stride-th offset, 30 s window), as 30 s peaks in kW and fractions of the
+    6.4 kW nameplate; the greedy's time is reported as candidate
+    window-samples/s."""
+    from paper_2608_11226_gb300 import pe
+    from paper_2608_11226_gb300 import workloads as W
+    G, L = fw.traces.shape
+    H, J, st, w = fw.horizon, fw.n_jobs, args.stagger_stride, 60
+    off = torch.empty(J, dtype=torch.int32, device="cuda")
+    pk = torch.empty(J, dtype=torch.int32, device="cuda")
+    ws = torch.empty(pe.fleet_stagger_workspace_bytes(J, L, H, st), dtype=torch.uint8, device="cuda")
+    pe.fleet_stagger(traces, job, J, H, w, st, off, pk, ws)
+    torch.cuda.synchronize()
+    barrier(world)
+    a = torch.cuda.Event(enable_timing=True)
+    b = torch.cuda.Event(enable_timing=True)
+    a.record()
+    pe.fleet_stagger(traces, job, J, H, w, st, off, pk, ws)
+    b.record()
+    torch.cuda.synchronize()
+    ms = max_over_ranks(a.elapsed_time(b), world)
+    ncand = (L + st - 1) // st
+    cand_ws = J * ncand * (H - w + 1)
+    kw = lambda v: float(v) / (64.0 * w) / 1e3  # noqa: E731  (peak window sum -> mean kW over the window)
+    name = W.FLEET_NAMEPLATE_W / 1e3
+    rnd = peaks_random[1:, 1] if peaks_random.shape[0] > 1 else peaks_random[:, 1]
+    stag = kw(pk[-1].item())
+    return {"metric": "staggered-schedule candidate window-samples/s",
+            "value": cand_ws * world / (ms / 1e3), "unit": "window-samples/s", "ms_per_call": ms,
+            "config": {"stride": st, "window": w, "candidates_per_job": ncand, "jobs": J},
+            "offsets": [int(x) for x in off.cpu()],
+            "peak_30s_kw": {"naive_aligned": kw(peaks_random[0, 1]), "random_median": kw(np.median(rnd)),
+                            "random_max": kw(rnd.max()), "phase_staggered": stag},
+            "provisioning_fraction": {"naive_aligned": kw(peaks_random[0, 1]) / name,
+                                      "random_median": kw(np.median(rnd)) / name,
+                                      "phase_staggered": stag / name}}
 
 
 def run_72b(args, world, peaks):

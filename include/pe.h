@@ -243,6 +243,27 @@ pe_status pe_fleet_windows(const float* traces, int32_t G, int32_t L, const int3
                            int32_t* counts, int32_t* peaks, void* workspace,
                            int64_t workspace_bytes, void* stream);
 
+/* Phase-staggered fleet schedule (Sec. 8, Table 9 "Phase-staggered"): a
+ * greedy scheduler places the jobs one at a time in index order 0..J-1.  Job
+ * j takes the start offset o from the grid {0, stride, 2 stride, ...} below L
+ * that minimises the peak w-sample window sum of the partial fleet of jobs
+ * 0..j (jobs 0..j-1 at their chosen offsets; composition and windows as in
+ * pe_fleet_windows, t in [w-1, H)); equal peaks go to the lowest offset.
+ *  traces [G][L] fp32 watts, job_of_gpu [G] in [0, J) (device memory);
+ *  w in [1, 992] (60 = the 30 s window); stride >= 1 (1 = every offset).
+ *  offsets: [J] int32 out, the chosen start offsets; peaks: [J] int32 out,
+ *  the partial fleet's peak window sum (1/64 W x samples) once job j is
+ *  placed (both device memory).
+ *  workspace: >= pe_fleet_stagger_workspace_bytes(J, L, H, stride) bytes.
+ * Like pe_fleet_windows, the call waits for the device-side trace check
+ * before the J stages; the stages themselves run without host round trips.
+ * Errors: PE_EINVAL (sizes, pointers, job map), PE_EOVERFLOW (bad sample or
+ * an int32 window sum out of range), PE_ECUDA. */
+int64_t pe_fleet_stagger_workspace_bytes(int32_t J, int32_t L, int32_t H, int32_t stride);
+pe_status pe_fleet_stagger(const float* traces, int32_t G, int32_t L, const int32_t* job_of_gpu,
+                           int32_t J, int32_t H, int32_t w, int32_t stride, int32_t* offsets,
+                           int32_t* peaks, void* workspace, int64_t workspace_bytes, void* stream);
+
 /* pe_fleet_windows for callers that cannot allocate device memory -- code
  * inside a host process whose device memory belongs to another allocator,
  * or a control loop that cannot afford an allocation's synchronisation.

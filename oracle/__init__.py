@@ -85,6 +85,7 @@ def lib():
                                        vp, vp, u64, u32, i64, vp]),
             "or_fleet_windows": (i32, [i32, i32, vp, vp, i32, vp, i64, i32, vp, i32, i64,
                                        vp, vp]),
+            "or_fleet_stagger": (i32, [i32, i32, vp, vp, i32, i32, i32, i32, vp, vp]),
         }
         for name, (res, args) in sig.items():
             fn = getattr(L, name)
@@ -267,3 +268,16 @@ def fleet_windows(traces, job_of_gpu, n_jobs: int, offsets, horizon: int, window
     if rc != 0:
         raise ValueError("oracle fleet windows rejected its inputs")
     return counts, peaks
+
+
+def fleet_stagger(traces, job_of_gpu, n_jobs: int, horizon: int, w: int, stride: int = 1):
+    """Greedy phase-staggered schedule (Sec. 8): (offsets[J], peaks[J])."""
+    traces = np.ascontiguousarray(traces, np.float32)
+    G, L = traces.shape
+    offsets = np.zeros(n_jobs, np.int32)
+    peaks = np.zeros(n_jobs, np.int32)
+    rc = lib().or_fleet_stagger(G, L, _p(traces), _p(np.ascontiguousarray(job_of_gpu, np.int32)),
+                                n_jobs, horizon, w, stride, _p(offsets), _p(peaks))
+    if rc != 0:
+        raise ValueError("oracle fleet stagger rejected its inputs")
+    return offsets, peaks

@@ -814,3 +814,50 @@ int32_t or_fleet_windows(int32_t G, int32_t L, const float* traces, const int32_
   free(q);
   return 0;
 }
+
+/* ------------------------------------------------------------------------
+ * Phase-staggered fleet schedule (Sec. 8): a greedy scheduler places the
+ * jobs one at a time, in index order.  Job j takes the start offset o from
+ * the candidate grid {0, s, 2s, ...} below L that minimises the peak w-sample
+ * window sum of the partial fleet made of jobs 0..j (the earlier jobs at the
+ * offsets already chosen), over t in [w-1, H); among equal peaks the lowest
+ * offset wins.  offsets[j] gets the choice and peaks[j] the partial fleet's
+ * peak once job j is placed.  Returns 1 on a bad job map.
+ * ---------------------------------------------------------------------- */
+int32_t or_fleet_stagger(int32_t G, int32_t L, const float* traces, const int32_t* job_of_gpu,
+                         int32_t J, int32_t H, int32_t w, int32_t stride, int32_t* offsets,
+                         int32_t* peaks) {
+  for (int32_t g = 0; g < G; ++g)
+    if (job_of_gpu[g] < 0 || job_of_gpu[g] >= J) return 1;
+  /* per-job power series q_j(t) = sum over the job's GPUs of rint(64 x_g(t)) */
+  int64_t* qj = (int64_t*)calloc((size_t)J * (size_t)L, sizeof(int64_t));
+  for (int32_t g = 0; g < G; ++g)
+    for (int32_t t = 0; t < L; ++t)
+      qj[(int64_t)job_of_gpu[g] * L + t] += (int64_t)rintf(traces[(int64_t)g * L + t] * 64.0f);
+  int64_t* placed = (int64_t*)calloc((size_t)(H > 0 ? H : 1), sizeof(int64_t));
+  int64_t* series = (int64_t*)malloc(sizeof(int64_t) * (size_t)(H > 0 ? H : 1));
+  for (int32_t j = 0; j < J; ++j) {
+    int64_t best_peak = -1;
+    int32_t best_o = 0;
+    for (int64_t o = 0; o < L; o += stride) {
+      for (int32_t t = 0; t < H; ++t) series[t] = placed[t] + qj[(int64_t)j * L + (int32_t)(((int64_t)t + o) % L)];
+      int64_t S = 0, peak = 0;
+      for (int32_t t = 0; t < H; ++t) {
+        S += series[t];
+        if (t >= w) S -= series[t - w];
+        if (t >= w - 1 && S > peak) peak = S;
+      }
+      if (best_peak < 0 || peak < best_peak) {
+        best_peak = peak;
+        best_o = (int32_t)o;
+      }
+    }
+    offsets[j] = best_o;
+    peaks[j] = (int32_t)best_peak;
+    for (int32_t t = 0; t < H; ++t) placed[t] += qj[(int64_t)j * L + (int32_t)(((int64_t)t + best_o) % L)];
+  }
+  free(series);
+  free(placed);
+  free(qj);
+  return 0;
+}

@@ -110,6 +110,9 @@ int32_t or_fleet_windows(int32_t G, int32_t L, const float* traces, const int32_
                          int32_t J, const int32_t* offsets, int64_t N, int32_t H,
                          const int32_t* windows, int32_t W, int64_t budget_q,
                          int32_t* counts, int32_t* peaks);
+int32_t or_fleet_stagger(int32_t G, int32_t L, const float* traces, const int32_t* job_of_gpu,
+                         int32_t J, int32_t H, int32_t w, int32_t stride, int32_t* offsets,
+                         int32_t* peaks);
 
 #ifdef __cplusplus
 }

@@ -89,6 +89,10 @@ pe_status ppo_update_bf16(const pe_net& net, float* params, float* m, float* v, 
                           const float* ret, int64_t N, const pe_ppo_config& cfg, float* stats, void* ws,
                           cudaStream_t st);
 int64_t fleet_ws_bytes(int J, int L, int H);
+int64_t fleet_stagger_ws_bytes(int J, int L, int H, int stride);
+pe_status fleet_stagger_launch(const float* traces, int G, int L, const int32_t* job_of_gpu, int J, int H,
+                               int w, int stride, int32_t* offsets_out, int32_t* peaks_out, void* workspace,
+                               cudaStream_t st);
 int64_t rollout_bf16_ws_bytes(const pe_net& net, int64_t E);
 pe_status rollout_bf16(const EnvDev& env, const pe_net& net, const float* params, int T, uint32_t it,
                        float lambda, int det, const pe_rollout_buf& buf, void* ws, cudaStream_t st);
@@ -521,6 +525,27 @@ pe_status pe_fleet_windows(const float* traces, int32_t G, int32_t L, const int3
   if (workspace_bytes < fleet_ws_bytes(J, L, H)) return fail(PE_EINVAL, "workspace too small");
   return fleet_launch(traces, G, L, job_of_gpu, J, offsets, N, H, windows, W, budget_q, counts,
                       peaks, workspace, reinterpret_cast<cudaStream_t>(stream));
+}
+
+int64_t pe_fleet_stagger_workspace_bytes(int32_t J, int32_t L, int32_t H, int32_t stride) {
+  if (J < 1 || J > 32 || L < 1 || H < 1 || stride < 1) return -1;
+  return fleet_stagger_ws_bytes(J, L, H, stride);
+}
+
+pe_status pe_fleet_stagger(const float* traces, int32_t G, int32_t L, const int32_t* job_of_gpu,
+                           int32_t J, int32_t H, int32_t w, int32_t stride, int32_t* offsets,
+                           int32_t* peaks, void* workspace, int64_t workspace_bytes, void* stream) {
+  clear_error();
+  if (G < 1 || G > 64) return fail(PE_EINVAL, "G must be in [1, 64]");
+  if (J < 1 || J > 32 || J > G) return fail(PE_EINVAL, "J must be in [1, min(32, G)]");
+  if (L < 1 || H < 1) return fail(PE_EINVAL, "L >= 1 and H >= 1 required");
+  if ((int64_t)L + H > (int64_t)INT32_MAX) return fail(PE_EINVAL, "L + H too large");
+  if (w < 1 || w > 992) return fail(PE_EINVAL, "window %d outside [1, 992]", w);
+  if (stride < 1) return fail(PE_EINVAL, "stride must be >= 1");
+  if (!traces || !job_of_gpu || !offsets || !peaks || !workspace) return fail(PE_EINVAL, "null argument");
+  if (workspace_bytes < fleet_stagger_ws_bytes(J, L, H, stride)) return fail(PE_EINVAL, "workspace too small");
+  return fleet_stagger_launch(traces, G, L, job_of_gpu, J, H, w, stride, offsets, peaks, workspace,
+                              reinterpret_cast<cudaStream_t>(stream));
 }
 
 }  // extern "C"

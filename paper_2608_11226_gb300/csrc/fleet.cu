@@ -252,12 +252,12 @@ int64_t fleet_ws_bytes(int J, int L, int H) {
   return prex + tot + 256 + 256;
 }
 
-pe_status fleet_launch(const float* traces, int G, int L, const int32_t* job_of_gpu, int J,
-                       const int32_t* offsets, int64_t N, int H, const int32_t* windows, int W,
-                       int64_t budget_q, int32_t* counts, int32_t* peaks, void* workspace,
-                       cudaStream_t st) {
+// Per-job prefix sums (PREX) and validation of the traces, job map and
+// offsets; returns the per-job maxima (for the int32 range checks).
+static pe_status fleet_prepare(const float* traces, int G, int L, const int32_t* job_of_gpu, int J,
+                               const int32_t* offsets, int64_t N, int H, void* workspace, FleetWs& ws,
+                               int64_t& sum_max, cudaStream_t st) {
   char* base = reinterpret_cast<char*>(workspace);
-  FleetWs ws;
   ws.Lp = fleet_lp(L, H);
   ws.nchunk = fleet_nchunk(L, H);
   const int64_t prex_bytes = ((int64_t)J * ws.Lp * 4 + 255) / 256 * 256;
@@ -286,8 +286,19 @@ pe_status fleet_launch(const float* traces, int G, int L, const int32_t* job_of_
   if (flag & 1) return fail(PE_EOVERFLOW, "fleet trace holds a sample that is not finite or outside [0, %g] W", (double)kFleetMaxWatts);
   if (flag & 2) return fail(PE_EINVAL, "job_of_gpu entry outside [0, J)");
   if (flag & 4) return fail(PE_EINVAL, "fleet offset outside [0, L)");
-  int64_t sum_max = 0;
+  sum_max = 0;
   for (int j = 0; j < J; ++j) sum_max += host[j];
+  return PE_OK;
+}
+
+pe_status fleet_launch(const float* traces, int G, int L, const int32_t* job_of_gpu, int J,
+                       const int32_t* offsets, int64_t N, int H, const int32_t* windows, int W,
+                       int64_t budget_q, int32_t* counts, int32_t* peaks, void* workspace,
+                       cudaStream_t st) {
+  FleetWs ws;
+  int64_t sum_max = 0;
+  pe_status s = fleet_prepare(traces, G, L, job_of_gpu, J, offsets, N, H, workspace, ws, sum_max, st);
+  if (s != PE_OK) return s;
   FleetWindows win{};
   for (int k = 0; k < W; ++k) {
     const int64_t w = windows[k];
@@ -307,6 +318,108 @@ pe_status fleet_launch(const float* traces, int G, int L, const int32_t* job_of_
     default: fleet_windows_kernel<4><<<grid_n, 32 * kFleetWarps, 0, st>>>(ws.prex, J, Lx, offsets, N, H, win, counts, peaks); break;
   }
   PE_CHECK_LAUNCH("fleet_windows_kernel");
+  return PE_OK;
+}
+
+// ---------------------------------------------------------------------------
+// Phase-staggered schedule (Sec. 8): jobs placed greedily in index order.
+// Stage j composes jobs 0..j with the earlier offsets fixed and job j at
+// every candidate c * stride; the windows kernel (first j + 1 jobs of the
+// prefix array) gives each candidate's peak, and a one-block argmin keeps
+// the lowest candidate among equal peaks.  The chosen offsets never leave
+// the device between stages.
+// ---------------------------------------------------------------------------
+__global__ void stagger_candidates_kernel(int32_t* __restrict__ cand, int64_t ncand, int j, int stride,
+                                          const int32_t* __restrict__ chosen) {
+  const int64_t total = ncand * (j + 1);
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < total; i += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t c = i / (j + 1);
+    const int k = (int)(i % (j + 1));
+    cand[i] = k < j ? chosen[k] : (int32_t)(c * stride);
+  }
+}
+
+__global__ void __launch_bounds__(1024) stagger_argmin_kernel(const int32_t* __restrict__ peaks, int64_t ncand,
+                                                              int stride, int j, int32_t* __restrict__ chosen,
+                                                              int32_t* __restrict__ chosen_peak) {
+  __shared__ int32_t sp[32];
+  __shared__ int64_t sc[32];
+  int32_t bp = INT_MAX;
+  int64_t bc = ncand;
+  for (int64_t c = threadIdx.x; c < ncand; c += blockDim.x) {
+    const int32_t p = peaks[c];
+    if (p < bp) {  // ascending scan: the first (lowest) candidate of a tie stays
+      bp = p;
+      bc = c;
+    }
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const int32_t op = __shfl_xor_sync(0xffffffffu, bp, o);
+    const int64_t oc = __shfl_xor_sync(0xffffffffu, bc, o);
+    if (op < bp || (op == bp && oc < bc)) {
+      bp = op;
+      bc = oc;
+    }
+  }
+  if ((threadIdx.x & 31) == 0) {
+    sp[threadIdx.x >> 5] = bp;
+    sc[threadIdx.x >> 5] = bc;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    for (int w = 1; w < (int)(blockDim.x >> 5); ++w)
+      if (sp[w] < bp || (sp[w] == bp && sc[w] < bc)) {
+        bp = sp[w];
+        bc = sc[w];
+      }
+    chosen[j] = (int32_t)(bc * stride);
+    chosen_peak[j] = bp;
+  }
+}
+
+static int64_t stagger_ncand(int L, int stride) { return ((int64_t)L + stride - 1) / stride; }
+
+int64_t fleet_stagger_ws_bytes(int J, int L, int H, int stride) {
+  const int64_t nc = stagger_ncand(L, stride);
+  const int64_t cand = (nc * J * 4 + 255) / 256 * 256;
+  const int64_t outs = (nc * 4 + 255) / 256 * 256;
+  return fleet_ws_bytes(J, L, H) + cand + 2 * outs;
+}
+
+pe_status fleet_stagger_launch(const float* traces, int G, int L, const int32_t* job_of_gpu, int J, int H,
+                               int w, int stride, int32_t* offsets_out, int32_t* peaks_out, void* workspace,
+                               cudaStream_t st) {
+  FleetWs ws;
+  int64_t sum_max = 0;
+  pe_status s = fleet_prepare(traces, G, L, job_of_gpu, J, nullptr, 0, H, workspace, ws, sum_max, st);
+  if (s != PE_OK) return s;
+  if (sum_max * w >= (int64_t)INT_MAX) return fail(PE_EOVERFLOW, "window %d: composed window sum may exceed int32", w);
+  const int64_t nc = stagger_ncand(L, stride);
+  char* base = reinterpret_cast<char*>(workspace) + fleet_ws_bytes(J, L, H);
+  int32_t* cand = reinterpret_cast<int32_t*>(base);
+  int32_t* cnt = reinterpret_cast<int32_t*>(base + (nc * J * 4 + 255) / 256 * 256);
+  int32_t* pk = cnt + (nc * 4 + 255) / 256 * 64;
+  FleetWindows win{};
+  win.w[0] = w;
+  win.bw[0] = INT_MAX;  // counts unused
+  const int grid_n = (int)((nc + kFleetWarps - 1) / kFleetWarps);
+  for (int j = 0; j < J; ++j) {
+    {
+      ProfScope ps(PE_PROF_FLEET_PREP, st);
+      stagger_candidates_kernel<<<(int)std::min<int64_t>(ceil_div(nc * (j + 1), 256), 4096), 256, 0, st>>>(
+          cand, nc, j, stride, offsets_out);
+    }
+    {
+      ProfScope ps(PE_PROF_FLEET_WINDOWS, st);
+      fleet_windows_kernel<1><<<grid_n, 32 * kFleetWarps, 0, st>>>(ws.prex, j + 1, ws.Lp, cand, nc, H, win, cnt, pk);
+    }
+    {
+      ProfScope ps(PE_PROF_FLEET_PREP, st);
+      stagger_argmin_kernel<<<1, 1024, 0, st>>>(pk, nc, stride, j, offsets_out, peaks_out);
+    }
+    PE_CHECK_LAUNCH("fleet stagger kernels");
+  }
   return PE_OK;
 }
 

@@ -69,6 +69,7 @@ EXPORTS = (
     "pe_param_count", "pe_rollout_workspace_bytes", "pe_rollout", "pe_value_workspace_bytes",
     "pe_value", "pe_device_check", "pe_gae", "pe_ppo_workspace_bytes",
     "pe_ppo_update", "pe_fleet_workspace_bytes", "pe_fleet_windows", "pe_fleet_windows_noalloc",
+    "pe_fleet_stagger_workspace_bytes", "pe_fleet_stagger",
     "pe_profile_enable",
     "pe_profile_read", "pe_profile_kind_name", "pe_last_error")
 
@@ -98,6 +99,8 @@ def lib():
             "pe_ppo_update": (i32, [vp, vp, vp, vp, i64, vp, vp, vp, vp, vp, i64, vp, vp, vp,
                                     i64, vp]),
             "pe_fleet_workspace_bytes": (i64, [i32, i32, i32]),
+            "pe_fleet_stagger_workspace_bytes": (i64, [i32, i32, i32, i32]),
+            "pe_fleet_stagger": (i32, [vp, i32, i32, vp, i32, i32, i32, i32, vp, vp, vp, i64, vp]),
             "pe_fleet_windows": (i32, [vp, i32, i32, vp, i32, vp, i64, i32, vp, i32, i64, vp,
                                        vp, vp, i64, vp]),
             "pe_fleet_windows_noalloc": (i32, [vp, i32, i32, vp, i32, vp, i64, i32, vp, i32, i64,
@@ -290,6 +293,18 @@ def fleet_windows(traces, job_of_gpu, J: int, offsets, H: int, windows: Sequence
     _check(lib().pe_fleet_windows(_ptr(traces), G, L, _ptr(job_of_gpu), J, _ptr(offsets), N, H,
                                   w, len(windows), budget_q, _ptr(counts), _ptr(peaks),
                                   _ptr(workspace), workspace.numel(), _stream(stream)))
+
+
+def fleet_stagger_workspace_bytes(J: int, L: int, H: int, stride: int) -> int:
+    return int(lib().pe_fleet_stagger_workspace_bytes(J, L, H, stride))
+
+
+def fleet_stagger(traces, job_of_gpu, J: int, H: int, w: int, stride: int, offsets, peaks, workspace,
+                  stream=None):
+    """Greedy phase-staggered start offsets (offsets[J]) and stage peaks (peaks[J])."""
+    G, L = traces.shape
+    _check(lib().pe_fleet_stagger(_ptr(traces), G, L, _ptr(job_of_gpu), J, H, w, stride, _ptr(offsets),
+                                  _ptr(peaks), _ptr(workspace), workspace.numel(), _stream(stream)))
 
 
 FLEET_NOALLOC_SCRATCH_BYTES = 4 * 1024 * 1024

@@ -154,6 +154,66 @@ def test_fleet_parity_full_size_sampled():
         assert p[:, wi].max() <= per
 
 
+# ------------------------------------------------------------ fleet stagger
+def _stagger_gpu(traces, job, J, H, w, stride):
+    tr = torch.from_numpy(np.ascontiguousarray(traces, np.float32)).cuda()
+    jg = torch.from_numpy(np.ascontiguousarray(job, np.int32)).cuda()
+    off = torch.full((J,), -1, dtype=torch.int32, device="cuda")
+    pk = torch.full((J,), -1, dtype=torch.int32, device="cuda")
+    ws = torch.empty(pe.fleet_stagger_workspace_bytes(J, tr.shape[1], H, max(stride, 1)), dtype=torch.uint8,
+                     device="cuda")
+    pe.fleet_stagger(tr, jg, J, H, w, stride, off, pk, ws)
+    torch.cuda.synchronize()
+    return cpu(off), cpu(pk)
+
+
+@pytest.mark.parametrize("L,H,w,stride", [(500, 500, 60, 1), (997, 800, 20, 7), (300, 1000, 1, 4)])
+def test_fleet_stagger_bit_exact(L, H, w, stride):
+    """Greedy staggered offsets and stage peaks equal the oracle's exactly
+    (ragged candidate grids, horizons shorter and longer than the period)."""
+    fw = W.make_fleet(n_compositions=1, length=L, seed=3)
+    g_off, g_pk = _stagger_gpu(fw.traces, fw.job_of_gpu, fw.n_jobs, H, w, stride)
+    o_off, o_pk = O.fleet_stagger(fw.traces, fw.job_of_gpu, fw.n_jobs, H, w, stride)
+    assert np.array_equal(g_off, o_off) and np.array_equal(g_pk, o_pk), (g_off, o_off, g_pk, o_pk)
+
+
+def test_fleet_stagger_full_size_sampled():
+    """The 16-GPU, 380,000-sample fleet with every offset a candidate: each
+    stage's peak is re-evaluated by the oracle at the chosen offsets, and a
+    seeded sample of other candidates (plus offset 0) is never better, nor
+    equal at a lower offset."""
+    fw = W.make_fleet(n_compositions=1)
+    L = fw.traces.shape[1]
+    g_off, g_pk = _stagger_gpu(fw.traces, fw.job_of_gpu, fw.n_jobs, L, 60, 1)
+    rng = np.random.default_rng(5)
+    for j in range(fw.n_jobs):
+        sel = fw.job_of_gpu <= j
+        tr, jb = fw.traces[sel], fw.job_of_gpu[sel]
+        cands = [int(g_off[j])] + [0] + [int(c) for c in rng.integers(0, L, 12)]
+        rows = np.tile(g_off[: j + 1], (len(cands), 1)).astype(np.int32)
+        rows[:, j] = cands
+        _, pk = O.fleet_windows(tr, jb, j + 1, rows, L, [60], 0)
+        assert pk[0, 0] == g_pk[j], (j, pk[0, 0], g_pk[j])
+        for c, p in zip(cands[1:], pk[1:, 0]):
+            assert p > g_pk[j] or (p == g_pk[j] and c >= g_off[j]), (j, c, p, g_off[j], g_pk[j])
+
+
+def test_fleet_stagger_rejects_bad_arguments():
+    fw = W.make_fleet(n_compositions=1, length=200)
+    assert pe.fleet_stagger_workspace_bytes(fw.n_jobs, 200, 200, 0) == -1
+    with pytest.raises(pe.PEError) as e:
+        _stagger_gpu(fw.traces, fw.job_of_gpu, fw.n_jobs, 200, 60, 0)
+    assert e.value.status == pe.PE_EINVAL
+    with pytest.raises(pe.PEError) as e:
+        _stagger_gpu(fw.traces, fw.job_of_gpu, fw.n_jobs, 200, 993, 1)
+    assert e.value.status == pe.PE_EINVAL
+    bad = fw.job_of_gpu.copy()
+    bad[3] = fw.n_jobs
+    with pytest.raises(pe.PEError) as e:
+        _stagger_gpu(fw.traces, bad, fw.n_jobs, 200, 60, 1)
+    assert e.value.status == pe.PE_EINVAL
+
+
 def test_fleet_rejects_bad_offsets_and_traces():
     fw = W.make_fleet(n_compositions=4, length=700)
     fw.offsets[2, 3] = 700

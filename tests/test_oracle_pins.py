@@ -543,3 +543,59 @@ def test_fleet_constant_hand_counted():
     for Bq, want in ((1279, [100, 41]), (1280, [0, 0])):
         c, p = O.fleet_windows(traces, [0, 1], 2, off, 100, [1, 60], Bq)
         assert c.tolist() == [want, want] and p.tolist() == [[1280, 76800]] * 2
+
+
+# ------------------------------------------------------------ fleet stagger
+def _np_window_peak(series, w):
+    c = np.concatenate([[0], np.cumsum(series, dtype=np.int64)])
+    S = c[w:] - c[:-w]          # S[t - w + 1] = sum of series[t-w+1 .. t]
+    return int(S.max())
+
+
+def test_fleet_stagger_square_waves_closed_form():
+    """Two identical square waves (h samples at a, h at b): the greedy puts
+    the second one in anti-phase, offset h, where the 1-sample peak drops
+    from 2a to a + b; the first job ties everywhere and takes offset 0.
+    With a full-period window every offset ties, so both offsets are 0."""
+    h, a, b, L = 5, 300.0, 100.0, 40
+    x = np.array(([a] * h + [b] * h) * (L // (2 * h)), np.float32)
+    traces = np.stack([x, x])
+    off, pk = O.fleet_stagger(traces, [0, 1], 2, L, 1, 1)
+    assert off.tolist() == [0, h]
+    assert pk.tolist() == [int(64 * a), int(64 * (a + b))]
+    off, pk = O.fleet_stagger(traces, [0, 1], 2, L, 2 * h, 1)
+    assert off.tolist() == [0, 0]
+    assert pk[1] == 2 * h * int(64 * (a + b))  # each job gives h(a + b) per full-period window
+
+
+def test_fleet_stagger_matches_brute_force():
+    """Every stage's choice against an independent numpy search over the
+    candidate grid (np.roll for the circular shift, cumulative sums for the
+    windows), on a random 5-GPU, 3-job fleet."""
+    rng = np.random.default_rng(11)
+    G, L, H, w, stride = 5, 47, 47, 6, 3
+    traces = rng.uniform(50, 400, size=(G, L)).astype(np.float32)
+    job = np.array([0, 0, 1, 2, 2], np.int32)
+    off, pk = O.fleet_stagger(traces, job, 3, H, w, stride)
+    q = np.rint(traces.astype(np.float32) * np.float32(64)).astype(np.int64)
+    qj = np.stack([q[job == j].sum(0) for j in range(3)])
+    placed = np.zeros(H, np.int64)
+    for j in range(3):
+        cands = list(range(0, L, stride))
+        peaks = [_np_window_peak(placed + np.roll(qj[j], -o)[:H], w) for o in cands]
+        best = int(np.argmin(peaks))          # argmin returns the first (lowest offset) minimum
+        assert off[j] == cands[best] and pk[j] == peaks[best], (j, off[j], cands[best])
+        placed += np.roll(qj[j], -off[j])[:H]
+
+
+def test_fleet_stagger_invariants():
+    """Stage peaks never fall (each job adds nonnegative power), and the
+    second job's choice is no worse than starting it with the first job."""
+    wl = W.make_fleet(n_compositions=1, length=600)
+    off, pk = O.fleet_stagger(wl.traces, wl.job_of_gpu, wl.n_jobs, 600, 60, 7)
+    assert np.all(np.diff(pk) >= 0)
+    sel = np.isin(wl.job_of_gpu, [0, 1])
+    _, aligned = O.fleet_windows(wl.traces[sel], wl.job_of_gpu[sel], 2,
+                                 np.array([[off[0], off[0]]], np.int32), 600, [60], 0)
+    assert pk[1] <= aligned[0, 0]
+    assert np.all(off % 7 == 0) and np.all(off < 600)
