@@ -49,6 +49,8 @@ def parse():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--fleet-n", type=int, default=1_000_000)
     ap.add_argument("--fleet-steps", type=int, default=3)
+    ap.add_argument("--no-eval", dest="eval", action="store_false",
+                    help="skip the evaluation replay (baseline rules, ledger) and the rule-rollout timing")
     ap.add_argument("--stagger-stride", type=int, default=1,
                     help="candidate offset grid of the greedy staggered schedule (0: skip)")
     ap.add_argument("--cpu-envs", type=int, default=48, help="envs in the oracle CPU sample")
@@ -308,6 +310,7 @@ def run_ours(args, world, rank, local):
 
     # ---- fleet accounting
     fleet = run_fleet(args, world) if args.fleet_n > 0 else None
+    evaluation = run_evaluation(args, world, tr, peaks) if args.eval else None
     r72b = run_72b(args, world, peaks) if args.r72b_steps > 0 else None
     gae_large = run_gae_large(args, world, peaks) if args.gae_large[0] > 0 else None
 
@@ -322,12 +325,85 @@ def run_ours(args, world, rank, local):
                       "l2": "flushed between timed steps (256 MB write)"},
            "roofline": roof, "gae_roofline": gae_roof, "kernels": kernels,
            "gpu_launches": launches, "clocks": clk, "e2e": e2e, "fleet": fleet, "rollout_72b": r72b,
-           "gae_roofline_stress_size": gae_large,
+           "gae_roofline_stress_size": gae_large, "evaluation": evaluation,
            "ppo_stats_last": [float(x) for x in tr.stats.cpu()]}
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         out["cpu_baseline"] = cpu_baseline(args.cpu_envs)
     if rank == 0:
         print(json.dumps(out), flush=True)
+
+
+KWH_PER_Q_SAMPLE = 0.5 / 64.0 / 3.6e6   # one sample of 1/64 W held 0.5 s, in kWh
+PRICE_PER_KWH = 0.08                     # Sec. 4.4 / 9.1
+CO2_KG_PER_KWH = 0.25                    # New York grid intensity, Sec. 4.4
+
+
+def run_evaluation(args, world, tr, peaks):
+    """Sec. 4.4 evaluation replay of the 7B trace: consecutive 500-step
+    episodes covering the trace (119 envs), run under the random policy, the
+    threshold heuristic (90% / 70% of the cap), the hysteresis rule (512 /
+    510 / 525 W at a 561 W budget, scaled to this budget) and the bench's
+    trained network acting deterministically; per arm the violation rates and
+    the energy ledger (kWh, $ at 0.08/kWh, kg CO2 at 0.25 kg/kWh, Wh per
+    1,000 tokens).  Then the rule rollout's throughput on the 72B env
+    (65,536 envs x 1,024 steps)."""
+    from paper_2608_11226_gb300 import pe
+    from paper_2608_11226_gb300 import workloads as W
+    base = W.make_7b(seed=tr.seed)
+    L = base.trace.shape[-1]
+    offs = W.replay_offsets(L, base.env.episode_len)
+    E, T = len(offs), base.env.episode_len
+    wl = W.make_7b(n_envs=E, seed=tr.seed)
+    spec, net = wl.env, wl.net
+    B = spec.budget_q
+    arms = {"random": W.random_rule(), "threshold_90_70": W.threshold_rule(B),
+            "hysteresis_512_510_525": W.hysteresis_rule(B), "learned_deterministic": None}
+    out = {}
+    for name, rule in arms.items():
+        env = pe.Env(spec, torch.from_numpy(wl.trace), torch.from_numpy(wl.phase))
+        pe.set_offsets(env, torch.from_numpy(offs).cuda())
+        if rule is None:
+            buf = pe.alloc_rollout(spec, net, T)
+            pe.rollout(env, net, tr.params, T, 0, buf, deterministic=True)
+        else:
+            buf = pe.alloc_rule_rollout(spec, T)
+            pe.rollout_rule(env, rule, T, 0, buf)
+        torch.cuda.synchronize()
+        viol = buf["viol"].sum(0).cpu().numpy()
+        tok = float(buf["tokens"].double().sum())
+        kwh = float(buf["energy_q"].sum()) * KWH_PER_Q_SAMPLE
+        out[name] = {"violation_rate_0.5s": float(viol[0]) / (E * T), "violation_rate_30s": float(viol[1]) / (E * T),
+                     "tokens": tok, "energy_kwh": kwh, "cost_usd": kwh * PRICE_PER_KWH,
+                     "co2_kg": kwh * CO2_KG_PER_KWH, "wh_per_1k_tokens": 1e3 * kwh * 1e3 / tok if tok else None}
+        env.close()
+    # throughput of the rule rollout at the 72B size
+    w72 = W.make_72b(seed=0)
+    env = pe.Env(w72.env, torch.from_numpy(w72.trace), torch.from_numpy(w72.phase))
+    T72 = 1024
+    buf = pe.alloc_rule_rollout(w72.env, T72)
+    rule = W.hysteresis_rule(w72.env.budget_q)
+    pe.rollout_rule(env, rule, T72, 0, buf)
+    torch.cuda.synchronize()
+    barrier(world)
+    a = torch.cuda.Event(enable_timing=True)
+    b = torch.cuda.Event(enable_timing=True)
+    a.record()
+    for it in range(2):
+        pe.rollout_rule(env, rule, T72, it + 1, buf)
+    b.record()
+    torch.cuda.synchronize()
+    ms = max_over_ranks(a.elapsed_time(b), world) / 2
+    n = w72.env.n_envs * T72
+    hbm = float(peaks.get("hbm_gbs", 6800.0))
+    gbs = 6.0 * n / (ms / 1e3) / 1e9  # act 1 + reward 4 + done 1 bytes written per env-step
+    env.close()
+    return {"arms": out, "config": {"workload": f"7b evaluation replay: {E} consecutive {T}-step episodes "
+                                                "covering the 60,000-sample trace", "n_envs": E, "horizon": T},
+            "rule_rollout_72b": {"metric": "rule-policy env-steps/s (hysteresis, 72B env)",
+                                 "value": n * world / (ms / 1e3), "unit": "env-steps/s", "ms_per_rollout": ms,
+                                 "roofline": {"kernel": "rule_rollout_kernel", "bound": "hbm", "achieved": gbs,
+                                              "peak": hbm, "unit": "GB/s", "frac": gbs / hbm,
+                                              "note": "6 B of buffer writes per env-step; latency-bound"}}}
 
 
 def run_fleet(args, world):

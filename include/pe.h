@@ -179,6 +179,46 @@ pe_status pe_rollout(pe_env* env, const pe_net* net, const float* params, int32_
                      uint32_t iteration, float lambda, int32_t flags, const pe_rollout_buf* buf,
                      void* workspace, int64_t workspace_bytes, void* stream);
 
+/* Episodes that start at given trace offsets (the evaluation replay of
+ * Sec. 4.4 walks a trace in consecutive 500-step episodes): every env starts
+ * a new episode at offsets[e], with its 60-sample history warm-started at
+ * the default level as at any episode start.
+ *  offsets: [E] int32 device memory, each in [60, L - episode_len].
+ * The call waits for the device-side range check.
+ * Errors: PE_EINVAL (null argument, an offset out of range; the envs with
+ * valid offsets are reset), PE_ECUDA. */
+pe_status pe_env_set_offsets(pe_env* env, const int32_t* offsets, void* stream);
+
+/* Baseline rule policies of the evaluation, in place of the network
+ * (Sec. 4.4: random policy and the threshold heuristic that lowers the group
+ * size above 90% of the cap and raises it below 70%; Sec. 4.5: the
+ * hysteresis rule that drops a level when the 30 s mean exceeds 512 W and
+ * climbs when the 30 s mean is below 510 W and the 10 s mean below 525 W, at
+ * a 561 W budget).  "Lower" and "raise" move G for the inc/dec actuator
+ * (actions 1 and 2) and the level index otherwise (clamped to the table).
+ * Thresholds are integers in 1/64 W, so decisions are exact:
+ *  RANDOM:     a = floor(u * A / 2^32), u = Philox(key = seed, ctr = (e, t, iteration, 0)).out[0];
+ *  THRESHOLD:  lower if the latest cluster sample q > hi_q, raise if q < lo_q, else hold;
+ *  HYSTERESIS: lower if S30 > 60 drop30_q; raise if S30 < 60 climb30_q and
+ *              S10 < 20 climb10_q (Eq. 1 window sums), else hold. */
+#define PE_RULE_RANDOM 1
+#define PE_RULE_THRESHOLD 2
+#define PE_RULE_HYSTERESIS 3
+typedef struct pe_rule {
+  int32_t kind;
+  int32_t hi_q, lo_q;                      /* THRESHOLD, 1/64 W */
+  int32_t drop30_q, climb30_q, climb10_q;  /* HYSTERESIS, window means in 1/64 W */
+} pe_rule;
+
+/* horizon steps of every env under a rule policy, with the same step,
+ * episode-end and counter semantics as pe_rollout.  buf: act, reward, done,
+ * viol, tokens, excess and energy_q are required; obs and obs_last are
+ * optional (NULL skips them; fp32, or bf16 when obs_bf16 != 0); logp, value
+ * and last_value are not touched.
+ * Errors: PE_EINVAL (unknown rule, null field, horizon < 1, unsupported env), PE_ECUDA. */
+pe_status pe_rollout_rule(pe_env* env, const pe_rule* rule, int32_t horizon, uint32_t iteration,
+                          float lambda, int32_t obs_bf16, const pe_rollout_buf* buf, void* stream);
+
 /* Value network on n observations (fp32, or bf16 for a BF16 network).
  * workspace: >= pe_value_workspace_bytes(net) bytes (0 for fp32); for a BF16
  * network the workspace must be 256-byte and obs 16-byte aligned. */

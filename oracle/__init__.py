@@ -70,6 +70,9 @@ def lib():
             "or_env_state_size": (i32, []),
             "or_actuator_scale": (C.c_float, [vp, i32, i32]),
             "or_env_init": (i32, [vp, vp, vp, vp, i32, vp]),
+            "or_env_set_offsets": (i32, [vp, vp, vp, vp, i32, vp]),
+            "or_rollout_rule": (i32, [vp, vp, vp, vp, vp, i32, vp, i32, u32, f64, vp, vp, vp, vp,
+                                      vp, vp, vp]),
             "or_env_obs": (None, [vp, vp, vp, vp, vp]),
             "or_mlp_forward": (None, [i32, i32, i32, i32, vp, i64, vp, vp, vp]),
             "or_rollout": (i32, [vp, vp, vp, vp, i32, i32, vp, i32, vp, i32, u32, f64, i32,
@@ -143,6 +146,15 @@ def actuator_scale(spec, level: int, channel: int = 0) -> float:
     return lib().or_actuator_scale(C.byref(cfg), level, channel)
 
 
+class OrRule(C.Structure):
+    _fields_ = [("kind", C.c_int32), ("hi_q", C.c_int32), ("lo_q", C.c_int32),
+                ("drop30_q", C.c_int32), ("climb30_q", C.c_int32), ("climb10_q", C.c_int32)]
+
+
+def or_rule(rule) -> OrRule:
+    return OrRule(rule.kind, rule.hi_q, rule.lo_q, rule.drop30_q, rule.climb30_q, rule.climb10_q)
+
+
 class OracleEnv:
     """A subset of a workload's envs, stepped by the oracle."""
 
@@ -187,6 +199,29 @@ class OracleEnv:
                          _p(out["act_own"]), _p(out["logp"]), _p(out["reward"]), _p(out["done"]),
                          _p(out["viol"]), _p(out["tokens"]), _p(out["excess"]),
                          _p(out["energy_q"]))
+        return out
+
+
+    def set_offsets(self, offsets) -> None:
+        """Start a new episode of every env at the given trace offsets."""
+        off = np.ascontiguousarray(offsets, np.int32)
+        if lib().or_env_set_offsets(C.byref(self.cfg), _p(self.trace), _p(self.phase), _p(off),
+                                    self.n, _p(self.state)) != 0:
+            raise ValueError("oracle rejected an episode offset")
+
+    def rollout_rule(self, rule, T: int, iteration: int, lam: float = 1.0) -> Dict[str, np.ndarray]:
+        """T steps under a baseline rule policy (workloads.RuleSpec)."""
+        n = self.n
+        out = dict(act=np.zeros((T, n), np.uint8), reward=np.zeros((T, n), np.float64),
+                   done=np.zeros((T, n), np.uint8), viol=np.zeros((n, 2), np.int32),
+                   tokens=np.zeros(n, np.float64), excess=np.zeros(n, np.float64),
+                   energy_q=np.zeros(n, np.int64))
+        r = or_rule(rule)
+        if lib().or_rollout_rule(C.byref(self.cfg), _p(self.trace), _p(self.phase), C.byref(r),
+                                 _p(self.env_ids), n, _p(self.state), T, iteration, lam,
+                                 _p(out["act"]), _p(out["reward"]), _p(out["done"]), _p(out["viol"]),
+                                 _p(out["tokens"]), _p(out["excess"]), _p(out["energy_q"])) != 0:
+            raise ValueError("oracle rejected the rule")
         return out
 
 

@@ -150,11 +150,8 @@ static int32_t qc_back(const or_env_cfg* cfg, const float* trace, const uint8_t*
 
 /* Sec. 4.1: episodes start at a randomised offset; the history window is
  * warm-started at the default setting (Sec. 4.5 warm start). */
-static void env_reset(const or_env_cfg* cfg, const float* trace, const uint8_t* phase,
-                      or_env_state* st, uint32_t e, uint32_t t, uint32_t it, uint32_t purpose) {
-  uint32_t u = draw_u32(cfg->seed, e, t, it, purpose);
-  uint32_t span = (uint32_t)(cfg->trace_len - cfg->episode_len - OR_W_LONG + 1);
-  int32_t o = OR_W_LONG + (int32_t)(((uint64_t)u * (uint64_t)span) >> 32);
+static void env_reset_at(const or_env_cfg* cfg, const float* trace, const uint8_t* phase,
+                         or_env_state* st, int32_t o) {
   st->pos = o;
   st->k = 0;
   st->level = cfg->level_init;
@@ -173,6 +170,24 @@ static void env_reset(const or_env_cfg* cfg, const float* trace, const uint8_t* 
       if (i <= OR_W_SHORT) st->s_short[c] += q;
     }
   }
+}
+
+static void env_reset(const or_env_cfg* cfg, const float* trace, const uint8_t* phase,
+                      or_env_state* st, uint32_t e, uint32_t t, uint32_t it, uint32_t purpose) {
+  uint32_t u = draw_u32(cfg->seed, e, t, it, purpose);
+  uint32_t span = (uint32_t)(cfg->trace_len - cfg->episode_len - OR_W_LONG + 1);
+  env_reset_at(cfg, trace, phase, st, OR_W_LONG + (int32_t)(((uint64_t)u * (uint64_t)span) >> 32));
+}
+
+/* Episodes that start at given offsets (the evaluation replay of Sec. 4.4
+ * walks the trace in consecutive 500-step episodes); each offset must leave
+ * the 60-sample history and one full episode inside the trace. */
+int32_t or_env_set_offsets(const or_env_cfg* cfg, const float* trace, const uint8_t* phase,
+                           const int32_t* offsets, int32_t n, or_env_state* states) {
+  for (int32_t i = 0; i < n; ++i)
+    if (offsets[i] < OR_W_LONG || offsets[i] > cfg->trace_len - cfg->episode_len) return 1;
+  for (int32_t i = 0; i < n; ++i) env_reset_at(cfg, trace, phase, &states[i], offsets[i]);
+  return 0;
 }
 
 int32_t or_env_init(const or_env_cfg* cfg, const float* trace, const uint8_t* phase,
@@ -511,6 +526,79 @@ int32_t or_rollout(const or_env_cfg* cfg, const float* trace, const uint8_t* pha
     energy_q[i] = en;
   }
   free(x); free(h1); free(h2); free(z); free(f); free(P);
+  return 0;
+}
+
+/* ------------------------------------------------------------------------
+ * Baseline policies of the evaluation (Sec. 4.4 random policy and threshold
+ * heuristic, Sec. 4.5 hysteresis rule), decided from the state before each
+ * step.  "Lower" and "raise" move the actuator one level: the group size G
+ * for the inc/dec actuator (actions 1 and 2; the env keeps G inside
+ * [g_min, g_max]), the level index otherwise (clamped to the table).
+ *  random:     a = floor(u32 * A / 2^32), u32 the step's action draw;
+ *  threshold:  lower if the latest cluster sample q > hi_q, raise if q < lo_q;
+ *  hysteresis: lower if S30 > 60 drop30_q; raise if S30 < 60 climb30_q and
+ *              S10 < 20 climb10_q (window sums of Eq. 1 in 1/64 W).
+ * ---------------------------------------------------------------------- */
+static int32_t rule_action(const or_env_cfg* cfg, const float* trace, const uint8_t* phase,
+                           const or_env_state* st, const or_rule* r, uint32_t e, uint32_t t,
+                           uint32_t it) {
+  const int32_t incdec = cfg->actuator_kind == OR_ACT_INCDEC;
+  const int32_t hold = incdec ? 0 : st->level;
+  const int32_t lower = incdec ? 1 : (st->level > 0 ? st->level - 1 : 0);
+  const int32_t raise = incdec ? 2 : (st->level < cfg->n_levels - 1 ? st->level + 1 : cfg->n_levels - 1);
+  if (r->kind == OR_RULE_RANDOM) {
+    const uint32_t u = draw_u32(cfg->seed, e, t, it, OR_PURPOSE_ACTION);
+    return (int32_t)(((uint64_t)u * (uint64_t)cfg->n_actions) >> 32);
+  }
+  if (r->kind == OR_RULE_THRESHOLD) {
+    const int32_t q = qc_back(cfg, trace, phase, st, 0);
+    if (q > r->hi_q) return lower;
+    if (q < r->lo_q) return raise;
+    return hold;
+  }
+  int64_t s10 = 0, s30 = 0;
+  for (int32_t c = 0; c < cfg->n_channels; ++c) {
+    s10 += st->s_short[c];
+    s30 += st->s_long[c];
+  }
+  if (s30 > (int64_t)OR_W_LONG * r->drop30_q) return lower;
+  if (s30 < (int64_t)OR_W_LONG * r->climb30_q && s10 < (int64_t)OR_W_SHORT * r->climb10_q) return raise;
+  return hold;
+}
+
+int32_t or_rollout_rule(const or_env_cfg* cfg, const float* trace, const uint8_t* phase,
+                        const or_rule* rule, const int32_t* env_ids, int32_t n,
+                        or_env_state* states, int32_t T, uint32_t iteration, double lambda,
+                        uint8_t* act, double* reward, uint8_t* done, int32_t* viol,
+                        double* tokens, double* excess, int64_t* energy_q) {
+  if (rule->kind < OR_RULE_RANDOM || rule->kind > OR_RULE_HYSTERESIS) return 1;
+  for (int32_t i = 0; i < n; ++i) {
+    or_env_state* st = &states[i];
+    const uint32_t e = (uint32_t)env_ids[i];
+    int32_t v1 = 0, v60 = 0;
+    double tok = 0.0, exc = 0.0;
+    int64_t en = 0;
+    for (int32_t t = 0; t < T; ++t) {
+      const int64_t row = (int64_t)t * n + i;
+      const int32_t a = rule_action(cfg, trace, phase, st, rule, e, (uint32_t)t, iteration);
+      act[row] = (uint8_t)a;
+      or_step_out so = env_step(cfg, trace, phase, st, a, lambda);
+      reward[row] = so.reward;
+      done[row] = (uint8_t)so.done;
+      v1 += so.v1;
+      v60 += so.v60;
+      tok += so.tokens;
+      exc += so.excess;
+      en += so.q;
+      if (so.done) env_reset(cfg, trace, phase, st, e, (uint32_t)t, iteration, OR_PURPOSE_RESET);
+    }
+    viol[2 * i] = v1;
+    viol[2 * i + 1] = v60;
+    tokens[i] = tok;
+    excess[i] = exc;
+    energy_q[i] = en;
+  }
   return 0;
 }
 

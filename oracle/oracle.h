@@ -57,6 +57,14 @@ typedef struct {
   int32_t s_long[OR_MAX_CH];       /* 30 s window sum (60 samples), per channel */
 } or_env_state;
 
+enum { OR_RULE_RANDOM = 1, OR_RULE_THRESHOLD = 2, OR_RULE_HYSTERESIS = 3 };
+
+typedef struct {
+  int32_t kind;
+  int32_t hi_q, lo_q;                      /* threshold rule, 1/64 W */
+  int32_t drop30_q, climb30_q, climb10_q;  /* hysteresis rule, 1/64 W (window means) */
+} or_rule;
+
 typedef struct {
   int32_t epochs, minibatch;
   double lr, clip, vf_coef, ent_coef, max_grad_norm, beta1, beta2, eps;
@@ -85,6 +93,13 @@ int32_t or_rollout(const or_env_cfg* cfg, const float* trace, const uint8_t* pha
                    const uint8_t* forced, float* obs, float* obs_last, uint8_t* act_own,
                    double* logp_taken, double* reward, uint8_t* done, int32_t* viol,
                    double* tokens, double* excess, int64_t* energy_q);
+int32_t or_env_set_offsets(const or_env_cfg* cfg, const float* trace, const uint8_t* phase,
+                           const int32_t* offsets, int32_t n, or_env_state* states);
+int32_t or_rollout_rule(const or_env_cfg* cfg, const float* trace, const uint8_t* phase,
+                        const or_rule* rule, const int32_t* env_ids, int32_t n,
+                        or_env_state* states, int32_t T, uint32_t iteration, double lambda,
+                        uint8_t* act, double* reward, uint8_t* done, int32_t* viol,
+                        double* tokens, double* excess, int64_t* energy_q);
 void or_gae(int32_t T, int32_t E, const float* r, const float* v, const uint8_t* done,
             const float* last_v, double gamma, double lam, double* adv, double* ret);
 double or_ppo_minibatch_grad(int32_t D, int32_t H, int32_t A, const double* params, int64_t M,

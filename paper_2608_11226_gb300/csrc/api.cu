@@ -89,6 +89,14 @@ pe_status ppo_update_bf16(const pe_net& net, float* params, float* m, float* v, 
                           const float* ret, int64_t N, const pe_ppo_config& cfg, float* stats, void* ws,
                           cudaStream_t st);
 int64_t fleet_ws_bytes(int J, int L, int H);
+struct RuleArgs {
+  int32_t kind, hi_q, lo_q, drop30_q, climb30_q, climb10_q;
+  int32_t T, obs_bf16;
+  uint32_t it;
+  float lambda;
+};
+pe_status rule_rollout(const EnvDev& env, const RuleArgs& r, const pe_rollout_buf& buf, cudaStream_t st);
+pe_status env_set_offsets(const EnvDev& env, const int32_t* offsets, int32_t* flag, cudaStream_t st);
 int64_t fleet_stagger_ws_bytes(int J, int L, int H, int stride);
 pe_status fleet_stagger_launch(const float* traces, int G, int L, const int32_t* job_of_gpu, int J, int H,
                                int w, int stride, int32_t* offsets_out, int32_t* peaks_out, void* workspace,
@@ -145,6 +153,7 @@ struct pe_env {
   pe_env_config cfg;
   EnvDev dev;
   int device;
+  int32_t* flag;  // device word for set-up checks (episode offsets)
 };
 
 extern "C" {
@@ -292,18 +301,21 @@ pe_status pe_env_create(const pe_env_config* cfg, const float* trace, const uint
   int32_t* st = nullptr;
   uint8_t* ring = nullptr;
   int32_t* sums = nullptr;
+  int32_t* flag = nullptr;
   if (e1 == cudaSuccess) e1 = cudaMalloc(&dtrace, sizeof(float) * h.size());
   if (e1 == cudaSuccess) e1 = cudaMalloc(&dphase, ph.size());
   if (e1 == cudaSuccess) e1 = cudaMalloc(&st, sizeof(int32_t) * kStN * (size_t)E);
   if (e1 == cudaSuccess) e1 = cudaMalloc(&ring, (size_t)kRing * E);
   if (e1 == cudaSuccess) e1 = cudaMalloc(&sums, sizeof(int32_t) * 8 * (size_t)E);
+  if (e1 == cudaSuccess) e1 = cudaMalloc(&flag, sizeof(int32_t));
   if (e1 != cudaSuccess) {
-    cudaFree(dtrace); cudaFree(dphase); cudaFree(st); cudaFree(ring); cudaFree(sums);
+    cudaFree(dtrace); cudaFree(dphase); cudaFree(st); cudaFree(ring); cudaFree(sums); cudaFree(flag);
     delete env;
     return e1 == cudaErrorMemoryAllocation ? fail(PE_ENOMEM, "device allocation failed")
                                            : cuda_fail(e1, "pe_env_create");
   }
   d.trace = dtrace; d.phase = dphase; d.st = st; d.ring = ring; d.sums = sums;
+  env->flag = flag;
   PE_TRY_CUDA(cudaMemcpy(dtrace, h.data(), sizeof(float) * h.size(), cudaMemcpyHostToDevice));
   PE_TRY_CUDA(cudaMemcpy(dphase, ph.data(), ph.size(), cudaMemcpyHostToDevice));
   launch_env_init(d);  // one-time set-up, not profiled
@@ -321,6 +333,7 @@ pe_status pe_env_destroy(pe_env* env) {
   cudaFree(env->dev.st);
   cudaFree(env->dev.ring);
   cudaFree(env->dev.sums);
+  cudaFree(env->flag);
   delete env;
   return PE_OK;
 }
@@ -371,6 +384,26 @@ static pe_status check_net(const pe_net* net) {
   if (net->obs_dim < 1 || net->hidden < 4 || net->n_actions < 1 || (net->dtype != PE_F32 && net->dtype != PE_BF16))
     return fail(PE_EINVAL, "invalid network description");
   return PE_OK;
+}
+
+pe_status pe_env_set_offsets(pe_env* env, const int32_t* offsets, void* stream) {
+  clear_error();
+  if (!env || !offsets) return fail(PE_EINVAL, "null argument");
+  return env_set_offsets(env->dev, offsets, env->flag, reinterpret_cast<cudaStream_t>(stream));
+}
+
+pe_status pe_rollout_rule(pe_env* env, const pe_rule* rule, int32_t horizon, uint32_t iteration, float lambda,
+                          int32_t obs_bf16, const pe_rollout_buf* buf, void* stream) {
+  clear_error();
+  if (!env || !rule || !buf) return fail(PE_EINVAL, "null argument");
+  if (rule->kind < PE_RULE_RANDOM || rule->kind > PE_RULE_HYSTERESIS) return fail(PE_EINVAL, "unknown rule kind %d", rule->kind);
+  if (horizon < 1) return fail(PE_EINVAL, "horizon must be >= 1");
+  if ((int64_t)horizon * env->dev.E > (int64_t)INT32_MAX) return fail(PE_EINVAL, "horizon * n_envs too large");
+  if (!buf->act || !buf->reward || !buf->done || !buf->viol || !buf->tokens || !buf->excess || !buf->energy_q)
+    return fail(PE_EINVAL, "null rollout buffer field");
+  RuleArgs r{rule->kind, rule->hi_q, rule->lo_q, rule->drop30_q, rule->climb30_q, rule->climb10_q,
+             horizon, obs_bf16 ? 1 : 0, iteration, lambda};
+  return rule_rollout(env->dev, r, *buf, reinterpret_cast<cudaStream_t>(stream));
 }
 
 int64_t pe_rollout_workspace_bytes(const pe_env* env, const pe_net* net) {

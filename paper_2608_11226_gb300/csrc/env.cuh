@@ -117,13 +117,9 @@ __device__ void rebuild_history(const EnvDev& env, Acc& a) {
   }
 }
 
-// new episode (Sec. 4.1: random offset; Sec. 4.5: warm start at the default level)
+// new episode at trace offset o (Sec. 4.5: warm start at the default level)
 template <int C, class Acc>
-__device__ void env_reset(const EnvDev& env, Acc& a, uint32_t eg, uint32_t t, uint32_t it,
-                          uint32_t purpose) {
-  const uint32_t u = draw32(env.seed, eg, t, it, purpose);
-  const uint32_t span = (uint32_t)(env.L - env.ep_len - kWLong + 1);
-  const int o = kWLong + (int)__umulhi(u, span);
+__device__ void env_reset_at(const EnvDev& env, Acc& a, int o) {
   a.pos() = o;
   a.k() = 0;
   a.level() = env.level_init;
@@ -132,6 +128,15 @@ __device__ void env_reset(const EnvDev& env, Acc& a, uint32_t eg, uint32_t t, ui
   a.til() = 0;
   for (int i = 0; i < kRing; ++i) a.set_level_at(i, env.level_init);
   rebuild_history<C>(env, a);
+}
+
+// new episode at a random offset (Sec. 4.1)
+template <int C, class Acc>
+__device__ void env_reset(const EnvDev& env, Acc& a, uint32_t eg, uint32_t t, uint32_t it,
+                          uint32_t purpose) {
+  const uint32_t u = draw32(env.seed, eg, t, it, purpose);
+  const uint32_t span = (uint32_t)(env.L - env.ep_len - kWLong + 1);
+  env_reset_at<C>(env, a, kWLong + (int)__umulhi(u, span));
 }
 
 template <int C, class Acc>

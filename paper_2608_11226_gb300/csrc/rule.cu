@@ -1,0 +1,145 @@
+// Baseline rule policies of the evaluation (Sec. 4.4 random policy and
+// threshold heuristic, Sec. 4.5 hysteresis rule) and explicit episode starts
+// for the full-trace replay.
+//
+// A rule rollout needs no network, so one thread runs one env through the
+// whole horizon in registers (its level ring in global memory): decide from
+// the state before the step, step (actuator, Eqs. 1-3, reward), record the
+// action, reward and done flag, and the per-call counters.
+#include <cuda_bf16.h>
+
+#include "env.cuh"
+
+namespace pe {
+
+// host-side twin declared in api.cu
+struct RuleArgs {
+  int32_t kind, hi_q, lo_q, drop30_q, climb30_q, climb10_q;
+  int32_t T, obs_bf16;
+  uint32_t it;
+  float lambda;
+};
+
+// lower / raise move one level: G for the inc/dec actuator (actions 1 and 2;
+// the env keeps G in [g_min, g_max]), the level index otherwise (clamped)
+template <int C>
+__device__ __forceinline__ int rule_action(const EnvDev& env, RegAcc<C>& a, const RuleArgs& r, uint32_t e,
+                                           uint32_t t) {
+  const bool incdec = env.act_kind == PE_ACT_INCDEC;
+  const int lvl = a.level();
+  const int hold = incdec ? 0 : lvl;
+  const int lower = incdec ? 1 : (lvl > 0 ? lvl - 1 : 0);
+  const int raise = incdec ? 2 : (lvl < env.n_levels - 1 ? lvl + 1 : env.n_levels - 1);
+  if (r.kind == PE_RULE_RANDOM) return (int)__umulhi(draw32(env.seed, e, t, r.it, kDrawAction), (uint32_t)env.A);
+  if (r.kind == PE_RULE_THRESHOLD) {
+    const int32_t q = Qcl<C>(env, a, 0);  // latest actuated cluster sample
+    return q > r.hi_q ? lower : (q < r.lo_q ? raise : hold);
+  }
+  int64_t s10 = 0, s30 = 0;
+#pragma unroll
+  for (int c = 0; c < C; ++c) {
+    s10 += a.ss(c);
+    s30 += a.sl(c);
+  }
+  if (s30 > (int64_t)kWLong * r.drop30_q) return lower;
+  return (s30 < (int64_t)kWLong * r.climb30_q && s10 < (int64_t)kWShort * r.climb10_q) ? raise : hold;
+}
+
+template <int C, int OBS, int D>
+__device__ __forceinline__ void write_obs(const EnvDev& env, RegAcc<C>& a, void* dst, int bf16) {
+  if (bf16) {
+    __nv_bfloat16* o = reinterpret_cast<__nv_bfloat16*>(dst);
+#pragma unroll 1
+    for (int f = 0; f < D; ++f) o[f] = __float2bfloat16_rn(feature<C, OBS>(env, a, f));
+  } else {
+    float* o = reinterpret_cast<float*>(dst);
+#pragma unroll 1
+    for (int f = 0; f < D; ++f) o[f] = feature<C, OBS>(env, a, f);
+  }
+}
+
+template <int C, int OBS, int D>
+__global__ void __launch_bounds__(128) rule_rollout_kernel(EnvDev env, RuleArgs r, pe_rollout_buf buf) {
+  const int e = blockIdx.x * blockDim.x + threadIdx.x;
+  if (e >= env.E) return;
+  RegAcc<C> acc = load_reg<C>(env, e);
+  const size_t ob = r.obs_bf16 ? 2 : 4;
+  int32_t v1 = 0, v60 = 0;
+  float tok = 0.0f, exc = 0.0f;
+  int64_t en = 0;
+  for (int t = 0; t < r.T; ++t) {
+    const int64_t row = (int64_t)t * env.E + e;
+    if (buf.obs) write_obs<C, OBS, D>(env, acc, reinterpret_cast<char*>(buf.obs) + row * D * ob, r.obs_bf16);
+    const int act = rule_action<C>(env, acc, r, (uint32_t)e, (uint32_t)t);
+    const StepOut so = env_step<C>(env, acc, act, r.lambda);
+    buf.act[row] = (uint8_t)act;
+    buf.reward[row] = so.reward;
+    buf.done[row] = (uint8_t)so.done;
+    v1 += so.v1;
+    v60 += so.v60;
+    tok += so.tokens;
+    exc += so.excess;
+    en += so.q;
+    if (so.done) env_reset<C>(env, acc, (uint32_t)e, (uint32_t)t, r.it, kDrawReset);
+  }
+  if (buf.obs_last) write_obs<C, OBS, D>(env, acc, reinterpret_cast<char*>(buf.obs_last) + (int64_t)e * D * ob, r.obs_bf16);
+  buf.viol[2 * e] = v1;
+  buf.viol[2 * e + 1] = v60;
+  buf.tokens[e] = tok;
+  buf.excess[e] = exc;
+  buf.energy_q[e] = en;
+  store_reg<C>(env, e, acc);
+}
+
+// every env starts a new episode at offsets[e]; offsets outside
+// [60, L - episode_len] set *flag and leave that env unchanged
+template <int C>
+__global__ void env_offsets_kernel(EnvDev env, const int32_t* __restrict__ offsets, int32_t* __restrict__ flag) {
+  const int e = blockIdx.x * blockDim.x + threadIdx.x;
+  if (e >= env.E) return;
+  const int o = offsets[e];
+  if (o < kWLong || o > env.L - env.ep_len) {
+    atomicOr(flag, 1);
+    return;
+  }
+  RegAcc<C> a;
+  a.ring = env.ring + (int64_t)e * kRing;
+  env_reset_at<C>(env, a, o);
+  store_reg<C>(env, e, a);
+}
+
+pe_status rule_rollout(const EnvDev& env, const RuleArgs& r, const pe_rollout_buf& buf, cudaStream_t st) {
+  const int grid = ceil_div(env.E, 128);
+  ProfScope ps(PE_PROF_ROLLOUT, st);
+  if (env.C == 1 && env.obs_kind == PE_OBS_TINY8)
+    rule_rollout_kernel<1, PE_OBS_TINY8, 8><<<grid, 128, 0, st>>>(env, r, buf);
+  else if (env.C == 1 && env.obs_kind == PE_OBS_7B16)
+    rule_rollout_kernel<1, PE_OBS_7B16, 16><<<grid, 128, 0, st>>>(env, r, buf);
+  else if (env.C == 4 && env.obs_kind == PE_OBS_OCC32)
+    rule_rollout_kernel<4, PE_OBS_OCC32, 32><<<grid, 128, 0, st>>>(env, r, buf);
+  else if (env.C == 4 && env.obs_kind == PE_OBS_OCC64)
+    rule_rollout_kernel<4, PE_OBS_OCC64, 64><<<grid, 128, 0, st>>>(env, r, buf);
+  else
+    return fail(PE_EINVAL, "rule rollout: unsupported env (C=%d, obs kind %d)", env.C, env.obs_kind);
+  PE_CHECK_LAUNCH("rule_rollout_kernel");
+  return PE_OK;
+}
+
+pe_status env_set_offsets(const EnvDev& env, const int32_t* offsets, int32_t* flag, cudaStream_t st) {
+  const int grid = ceil_div(env.E, 128);
+  PE_TRY_CUDA(cudaMemsetAsync(flag, 0, sizeof(int32_t), st));
+  switch (env.C) {
+    case 1: env_offsets_kernel<1><<<grid, 128, 0, st>>>(env, offsets, flag); break;
+    case 2: env_offsets_kernel<2><<<grid, 128, 0, st>>>(env, offsets, flag); break;
+    case 3: env_offsets_kernel<3><<<grid, 128, 0, st>>>(env, offsets, flag); break;
+    default: env_offsets_kernel<4><<<grid, 128, 0, st>>>(env, offsets, flag); break;
+  }
+  PE_CHECK_LAUNCH("env_offsets_kernel");
+  int32_t h = 0;
+  PE_TRY_CUDA(cudaMemcpyAsync(&h, flag, sizeof(int32_t), cudaMemcpyDeviceToHost, st));
+  PE_TRY_CUDA(cudaStreamSynchronize(st));
+  if (h) return fail(PE_EINVAL, "episode offset outside [60, L - episode_len]");
+  return PE_OK;
+}
+
+}  // namespace pe

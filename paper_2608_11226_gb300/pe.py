@@ -57,6 +57,10 @@ class RolloutBuf(C.Structure):
         "tokens", "excess", "energy_q")]
 
 
+class Rule(C.Structure):
+    _fields_ = [(n, C.c_int32) for n in ("kind", "hi_q", "lo_q", "drop30_q", "climb30_q", "climb10_q")]
+
+
 class PPOConfig(C.Structure):
     _fields_ = [("epochs", C.c_int32), ("minibatch", C.c_int32)] + [
         (n, C.c_float) for n in ("lr", "clip", "vf_coef", "ent_coef", "max_grad_norm",
@@ -69,7 +73,7 @@ EXPORTS = (
     "pe_param_count", "pe_rollout_workspace_bytes", "pe_rollout", "pe_value_workspace_bytes",
     "pe_value", "pe_device_check", "pe_gae", "pe_ppo_workspace_bytes",
     "pe_ppo_update", "pe_fleet_workspace_bytes", "pe_fleet_windows", "pe_fleet_windows_noalloc",
-    "pe_fleet_stagger_workspace_bytes", "pe_fleet_stagger",
+    "pe_fleet_stagger_workspace_bytes", "pe_fleet_stagger", "pe_env_set_offsets", "pe_rollout_rule",
     "pe_profile_enable",
     "pe_profile_read", "pe_profile_kind_name", "pe_last_error")
 
@@ -100,6 +104,8 @@ def lib():
                                     i64, vp]),
             "pe_fleet_workspace_bytes": (i64, [i32, i32, i32]),
             "pe_fleet_stagger_workspace_bytes": (i64, [i32, i32, i32, i32]),
+            "pe_env_set_offsets": (i32, [vp, vp, vp]),
+            "pe_rollout_rule": (i32, [vp, vp, i32, u32, C.c_float, i32, vp, vp]),
             "pe_fleet_stagger": (i32, [vp, i32, i32, vp, i32, i32, i32, i32, vp, vp, vp, i64, vp]),
             "pe_fleet_windows": (i32, [vp, i32, i32, vp, i32, vp, i64, i32, vp, i32, i64, vp,
                                        vp, vp, i64, vp]),
@@ -230,6 +236,38 @@ def rollout(env: Env, net: W.NetSpec, params: torch.Tensor, T: int, iteration: i
     _check(lib().pe_rollout(env._h, C.byref(net_desc(net)), _ptr(params), T, iteration, lam,
                             PE_ROLLOUT_DETERMINISTIC if deterministic else 0, C.byref(rb),
                             _ptr(workspace), nbytes, _stream(stream)))
+
+
+def set_offsets(env: Env, offsets: torch.Tensor, stream=None):
+    """Start a new episode of every env at offsets[e] (int32 device tensor)."""
+    _check(lib().pe_env_set_offsets(env._h, _ptr(offsets), _stream(stream)))
+
+
+def alloc_rule_rollout(spec: W.EnvSpec, T: int, obs: bool = False, obs_bf16: bool = False,
+                       device="cuda") -> Dict[str, torch.Tensor]:
+    """Buffers of a rule-policy rollout (observations only if asked for)."""
+    E, D = spec.n_envs, spec.obs_dim
+    kw = dict(device=device)
+    odt = torch.bfloat16 if obs_bf16 else torch.float32
+    return dict(
+        obs=torch.empty((T, E, D), dtype=odt, **kw) if obs else None,
+        obs_last=torch.empty((E, D), dtype=odt, **kw) if obs else None,
+        act=torch.empty((T, E), dtype=torch.uint8, **kw), logp=None, value=None, last_value=None,
+        reward=torch.empty((T, E), **kw), done=torch.empty((T, E), dtype=torch.uint8, **kw),
+        viol=torch.empty((E, 2), dtype=torch.int32, **kw), tokens=torch.empty(E, **kw),
+        excess=torch.empty(E, **kw), energy_q=torch.empty(E, dtype=torch.int64, **kw))
+
+
+def rollout_rule(env: Env, rule: W.RuleSpec, T: int, iteration: int, buf: Dict[str, torch.Tensor],
+                 lam: float = 1.0, stream=None):
+    """T steps of every env under a baseline rule policy (no network)."""
+    rb = RolloutBuf(*[(b.data_ptr() if (b := buf[k]) is not None else None) for k in (
+        "obs", "obs_last", "act", "logp", "value", "last_value", "reward", "done", "viol",
+        "tokens", "excess", "energy_q")])
+    obs_bf16 = buf["obs"] is not None and buf["obs"].dtype == torch.bfloat16
+    r = Rule(rule.kind, rule.hi_q, rule.lo_q, rule.drop30_q, rule.climb30_q, rule.climb10_q)
+    _check(lib().pe_rollout_rule(env._h, C.byref(r), T, iteration, lam, int(obs_bf16), C.byref(rb),
+                                 _stream(stream)))
 
 
 def value_workspace_bytes(net: W.NetSpec) -> int:

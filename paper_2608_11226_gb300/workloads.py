@@ -398,3 +398,45 @@ def make_fleet(n_compositions: int = 1_000_000, length: int = 380000, seed: int 
     off = fleet_offsets(n_compositions, J, length, seed)
     return FleetWorkload(traces, job, J, off, length, np.asarray(windows, np.int32),
                          budget_q(0.5 * FLEET_NAMEPLATE_W))
+
+
+# ---------------------------------------------------------------------------
+# Baseline rule policies of the evaluation (Sec. 4.4 random policy and
+# threshold heuristic, Sec. 4.5 hysteresis rule) as integer thresholds in
+# 1/64 W, taken as fractions of the env's quantised budget.  The hysteresis
+# thresholds keep the paper's ratios to its 561 W budget (512, 510, 525 W).
+# ---------------------------------------------------------------------------
+RULE_RANDOM, RULE_THRESHOLD, RULE_HYSTERESIS = 1, 2, 3
+
+
+@dataclasses.dataclass
+class RuleSpec:
+    kind: int
+    hi_q: int = 0
+    lo_q: int = 0
+    drop30_q: int = 0
+    climb30_q: int = 0
+    climb10_q: int = 0
+
+
+def random_rule() -> RuleSpec:
+    return RuleSpec(RULE_RANDOM)
+
+
+def threshold_rule(budget_q: int, hi: float = 0.9, lo: float = 0.7) -> RuleSpec:
+    return RuleSpec(RULE_THRESHOLD, hi_q=int(round(hi * budget_q)), lo_q=int(round(lo * budget_q)))
+
+
+def hysteresis_rule(budget_q: int, drop30: float = 512.0 / 561.0, climb30: float = 510.0 / 561.0,
+                    climb10: float = 525.0 / 561.0) -> RuleSpec:
+    return RuleSpec(RULE_HYSTERESIS, drop30_q=int(round(drop30 * budget_q)),
+                    climb30_q=int(round(climb30 * budget_q)), climb10_q=int(round(climb10 * budget_q)))
+
+
+def replay_offsets(trace_len: int, episode_len: int, n: int = -1) -> np.ndarray:
+    """Consecutive episode starts covering a trace (Sec. 4.4 full-trace
+    replay in episode_len-step episodes), after the 60-sample history."""
+    k = (trace_len - 60) // episode_len
+    if n >= 0:
+        k = min(k, n)
+    return (60 + episode_len * np.arange(k)).astype(np.int32)

@@ -39,7 +39,10 @@ class BruteEnv:
         seed = s.seed
         u = int(self.philox([self.e, t, it, purpose], [seed & 0xFFFFFFFF, seed >> 32])[0])
         span = self.L - s.episode_len - W_LONG + 1
-        o = W_LONG + ((u * span) >> 32)
+        self.reset_at(W_LONG + ((u * span) >> 32))
+
+    def reset_at(self, o):
+        s = self.s
         self.pos, self.k = o, 0
         self.level = self.prev = s.level_init
         self.b, self.til = s.b_init, 0

@@ -495,3 +495,86 @@ def test_ppo_bf16_ragged_epochs_72b():
     dp, dref = gp - params, P - params
     assert np.linalg.norm(dp - dref) <= 0.1 * np.linalg.norm(dref), np.linalg.norm(dp - dref) / np.linalg.norm(dref)
     assert abs(gs[1] - st[1]) <= 2e-2 * abs(st[1])
+
+
+# ------------------------------------------------------- baseline rule policies
+def _rule_for(kind, preset, B):
+    if kind == 1:
+        return W.random_rule()
+    if preset == "tiny":  # thresholds between the tiny levels
+        return W.threshold_rule(B, 1.1, 0.98) if kind == 2 else W.hysteresis_rule(B, 1.1, 0.98, 1.05)
+    return W.threshold_rule(B) if kind == 2 else W.hysteresis_rule(B)
+
+
+@pytest.mark.parametrize("preset", ["tiny", "7b", "72b"])
+@pytest.mark.parametrize("kind", [1, 2, 3])
+def test_rule_rollout_parity(preset, kind):
+    """Rule-policy rollouts from explicit episode starts, two calls in a row
+    (state carried across calls, episode boundaries crossed): actions, done
+    flags, violation counts and energy bit-exact; rewards, tokens and excess
+    within 1e-5; the final observation bit-exact."""
+    E = 64
+    wl = {"tiny": W.make_tiny, "7b": W.make_7b, "72b": W.make_72b}[preset](n_envs=E)
+    spec = wl.env
+    rule = _rule_for(kind, preset, spec.budget_q)
+    offs = W.replay_offsets(wl.trace.shape[-1], spec.episode_len)
+    offs = np.resize(offs, E).astype(np.int32)
+    env = pe.Env(spec, torch.from_numpy(wl.trace), torch.from_numpy(wl.phase))
+    pe.set_offsets(env, torch.from_numpy(offs).cuda())
+    oenv = O.OracleEnv(spec, wl.trace, wl.phase, range(E))
+    oenv.set_offsets(offs)
+    bf16 = preset == "72b"
+    for it, T in ((0, 300), (1, 450)):
+        buf = pe.alloc_rule_rollout(spec, T, obs=True, obs_bf16=bf16)
+        pe.rollout_rule(env, rule, T, it, buf, lam=0.5)
+        torch.cuda.synchronize()
+        ref = oenv.rollout_rule(rule, T, it, lam=0.5)
+        assert np.array_equal(cpu(buf["act"]), ref["act"])
+        assert np.array_equal(cpu(buf["done"]), ref["done"])
+        assert np.array_equal(cpu(buf["viol"]), ref["viol"])
+        assert np.array_equal(cpu(buf["energy_q"]), ref["energy_q"])
+        assert rel_err(cpu(buf["reward"]), ref["reward"]) <= TOL
+        assert rel_err(cpu(buf["tokens"]), ref["tokens"]) <= TOL
+        assert rel_err(cpu(buf["excess"]), ref["excess"]) <= TOL
+        o_last = oenv.obs()
+        g_last = cpu(buf["obs_last"].float())
+        if bf16:
+            o_last = torch.from_numpy(o_last).to(torch.bfloat16).float().numpy()
+        assert np.array_equal(g_last, o_last)
+    env.close()
+
+
+def test_rule_rollout_full_size_sampled():
+    """The 72B env at full size (65,536 envs x 1,024 steps) under the
+    hysteresis rule from the random initial offsets; the oracle replays a
+    seeded sample of envs."""
+    wl = W.make_72b()
+    spec = wl.env
+    E, T = spec.n_envs, 1024
+    rule = W.hysteresis_rule(spec.budget_q)
+    env = pe.Env(spec, torch.from_numpy(wl.trace), torch.from_numpy(wl.phase))
+    buf = pe.alloc_rule_rollout(spec, T)
+    pe.rollout_rule(env, rule, T, 2, buf, lam=1.0)
+    torch.cuda.synchronize()
+    ids = np.random.default_rng(9).choice(E, 24, replace=False)
+    oenv = O.OracleEnv(spec, wl.trace, wl.phase, ids)
+    ref = oenv.rollout_rule(rule, T, 2, lam=1.0)
+    ids_t = torch.from_numpy(ids).cuda()
+    assert np.array_equal(cpu(buf["act"][:, ids_t]), ref["act"])
+    assert np.array_equal(cpu(buf["viol"][ids_t]), ref["viol"])
+    assert np.array_equal(cpu(buf["energy_q"][ids_t]), ref["energy_q"])
+    assert rel_err(cpu(buf["reward"][:, ids_t]), ref["reward"]) <= TOL
+    env.close()
+
+
+def test_set_offsets_rejects_out_of_range():
+    wl = W.make_tiny(n_envs=4)
+    env = pe.Env(wl.env, torch.from_numpy(wl.trace), torch.from_numpy(wl.phase))
+    bad = torch.tensor([60, 100, wl.trace.shape[-1] - wl.env.episode_len + 1, 70], dtype=torch.int32).cuda()
+    with pytest.raises(pe.PEError) as e:
+        pe.set_offsets(env, bad)
+    assert e.value.status == pe.PE_EINVAL
+    with pytest.raises(pe.PEError) as e:
+        pe.rollout_rule(env, W.RuleSpec(7), 10, 0, pe.alloc_rule_rollout(wl.env, 10))
+    assert e.value.status == pe.PE_EINVAL
+    env.close()

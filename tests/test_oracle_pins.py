@@ -599,3 +599,90 @@ def test_fleet_stagger_invariants():
                                  np.array([[off[0], off[0]]], np.int32), 600, [60], 0)
     assert pk[1] <= aligned[0, 0]
     assert np.all(off % 7 == 0) and np.all(off < 600)
+
+
+# ------------------------------------------------------- baseline rule policies
+def _brute_rule(b, rule, e, t, it):
+    """The Sec. 4.4 / 4.5 baseline rules, decided on the brute-force env's
+    history (window sums recomputed sample by sample)."""
+    s = b.s
+    incdec = s.actuator_kind == 1
+    hold = 0 if incdec else b.level
+    lower = 1 if incdec else max(b.level - 1, 0)
+    up = 2 if incdec else min(b.level + 1, s.n_levels - 1)
+    if rule.kind == W.RULE_RANDOM:
+        u = int(O.philox4x32_10([e, t, it, 0], [s.seed & 0xFFFFFFFF, s.seed >> 32])[0])
+        return (u * s.n_actions) >> 32
+    if rule.kind == W.RULE_THRESHOLD:
+        q = b.Q(0)
+        return lower if q > rule.hi_q else (up if q < rule.lo_q else hold)
+    s30, s10 = b.S(60), b.S(20)
+    if s30 > 60 * rule.drop30_q:
+        return lower
+    return up if (s30 < 60 * rule.climb30_q and s10 < 20 * rule.climb10_q) else hold
+
+
+@pytest.mark.parametrize("preset", ["tiny", "7b", "72b"])
+@pytest.mark.parametrize("kind", [1, 2, 3])
+def test_rule_rollout_matches_bruteforce(preset, kind):
+    """Baseline-policy rollouts from explicit episode starts (the evaluation
+    replay), across an episode boundary, against the brute-force env driven
+    by the same rules."""
+    wl = {"tiny": W.make_tiny, "7b": W.make_7b, "72b": W.make_72b}[preset](n_envs=2)
+    spec = wl.env
+    B = spec.budget_q
+    rule = {1: W.random_rule(), 2: W.threshold_rule(B), 3: W.hysteresis_rule(B)}[kind]
+    # the tiny trace sits above 0.9 B at every level: thresholds between its
+    # levels make both rules move in both directions
+    if preset == "tiny" and kind == 2:
+        rule = W.threshold_rule(B, 1.1, 0.98)
+    if preset == "tiny" and kind == 3:
+        rule = W.hysteresis_rule(B, 1.1, 0.98, 1.05)
+    if preset == "7b" and kind == 3:  # the 7B 30 s mean stays above 512/561 of B
+        rule = W.hysteresis_rule(B, 1.08, 1.0, 1.05)
+    offs = W.replay_offsets(wl.trace.shape[-1], spec.episode_len, 2)
+    env = O.OracleEnv(spec, wl.trace, wl.phase, [0, 1])
+    env.set_offsets(offs)
+    T = spec.episode_len + 30
+    out = env.rollout_rule(rule, T, 3, lam=0.5)
+    for i in range(2):
+        b = BruteEnv(spec, wl.trace.astype(np.float32), wl.phase, i, O.philox4x32_10)
+        b.reset_at(int(offs[i]))
+        v = [0, 0]
+        en = 0
+        for t in range(T):
+            a = _brute_rule(b, rule, i, t, 3)
+            assert out["act"][t, i] == a, (t, i)
+            st = b.step(a, 0.5, t, 3)
+            assert out["done"][t, i] == st["done"]
+            assert abs(out["reward"][t, i] - st["r"]) <= 1e-12 * max(1.0, abs(st["r"]))
+            v[0] += st["v1"]
+            v[1] += st["v60"]
+            en += st["q"]
+        assert list(out["viol"][i]) == v and out["energy_q"][i] == en
+    acts = np.bincount(out["act"].ravel(), minlength=spec.n_actions)
+    assert (acts > 0).sum() >= (2 if kind != 1 else spec.n_actions // 2)
+
+
+def test_threshold_rule_constant_trace_hand_counted():
+    """A flat 7B trace at 1.2 B watts (above 0.9 B at every group size): the
+    threshold rule lowers G every step, from 4 to the floor 3 after one
+    step, so the energy is one sample at s(4) and the rest at s(3); a flat
+    trace at 0.5 B raises G every step up to G_max = 8."""
+    wl = W.make_7b(n_envs=1)
+    spec = wl.env
+    L = wl.trace.shape[-1]
+    for frac, act, levels in ((1.2, 1, [4, 3]), (0.5, 2, [4, 5, 6, 7, 8])):
+        x = np.float32(frac * spec.budget_q / 64.0)
+        trace = np.full_like(wl.trace, x)
+        phase = np.zeros_like(wl.phase)
+        env = O.OracleEnv(spec, trace, phase, [0])
+        env.set_offsets([100])
+        T = 12
+        out = env.rollout_rule(W.threshold_rule(spec.budget_q), T, 0)
+        assert np.all(out["act"][:, 0] == act)
+        # G in effect at each step: the first action already moves G once
+        g = levels[1:] + [levels[-1]] * (T - len(levels) + 1)
+        q = [int(np.rint(np.float32(x * O.actuator_scale(spec, G)) * np.float32(64))) for G in g[:T]]
+        assert out["energy_q"][0] == sum(q)
+    del L
