@@ -550,6 +550,16 @@ def run_72b(args, world, peaks):
     gae_gbs = 17.0 * T * E / (gms / gn / 1e3) / 1e9 if gn else None
     hbm = float(peaks.get("hbm_gbs", 6800.0))
     ppo72 = run_72b_ppo(args, world, peaks, wl, buf, adv, ret) if args.r72b_ppo_minibatches > 0 else None
+    # the Eq. 7 outer loop: lambda fed back from each rollout's 30 s violation rate (target 8%)
+    lam_dev = torch.tensor([1.0], device="cuda")
+    rate_dev = torch.zeros(1, device="cuda")
+    dual = []
+    for it in range(3):
+        lam_h = float(lam_dev.item())
+        pe.rollout(env, net, params, T, 10 + it, buf, lam=lam_h, workspace=ws)
+        pe.dual_ascent(buf["viol"], T, lam_dev, rate_dev, target=0.08)
+        dual.append({"lambda_in": lam_h, "violation_rate_30s": float(rate_dev.item()),
+                     "lambda_out": float(lam_dev.item())})
     del adv, ret
     pms, pn = prof["mlp_policy_tc"]
     vms, vn = prof["mlp_value_tc"]
@@ -575,7 +585,7 @@ def run_72b(args, world, peaks):
                              "peak": hbm, "unit": "GB/s", "frac": gae_gbs / hbm if gae_gbs else None,
                              "avg_launch_ms": gms / gn if gn else None,
                              "traffic": gae_traffic(T * E)},
-            "ppo_update": ppo72}
+            "ppo_update": ppo72, "dual_ascent_eq7": dual}
 
 
 def run_72b_ppo(args, world, peaks, wl, buf, adv, ret):

@@ -219,6 +219,21 @@ typedef struct pe_rule {
 pe_status pe_rollout_rule(pe_env* env, const pe_rule* rule, int32_t horizon, uint32_t iteration,
                           float lambda, int32_t obs_bf16, const pe_rollout_buf* buf, void* stream);
 
+/* Dual ascent on the Lagrange multiplier of the Eq. 6 reward (Eq. 7,
+ * Sec. 4.5; the G3 design of Sec. 4.2), from a rollout's violation counts:
+ *   v = sum_e viol[e][w] / (n_envs * steps)   (w: 1 = instantaneous, 60 = 30 s window)
+ *   multiplicative (additive = 0, Eq. 7): lambda <- clip(lambda exp(eta (v - target) / target), lo, hi)
+ *   additive (additive = 1, G3):          lambda <- clip(lambda + eta (v - target) / target, lo, hi)
+ *  viol: [n_envs][2] int32 device (pe_rollout_buf.viol); steps: the rollout's horizon;
+ *  lambda: device float, read and updated in place; rate: device float out (v), or NULL.
+ * The paper's Eq. 7 settings are eta = 0.5, [lo, hi] = [1e-3, 2]; its G3 run used a target of 8%.
+ * pe_rollout takes lambda by value, so a caller that feeds the update back reads 4 bytes per
+ * iteration.
+ * Errors: PE_EINVAL (null pointer, sizes, window not 1 or 60, target outside (0, 1), bounds), PE_ECUDA. */
+pe_status pe_dual_ascent(const int32_t* viol, int32_t n_envs, int64_t steps, int32_t window, int32_t additive,
+                         float target, float eta, float lambda_min, float lambda_max, float* lambda, float* rate,
+                         void* stream);
+
 /* Value network on n observations (fp32, or bf16 for a BF16 network).
  * workspace: >= pe_value_workspace_bytes(net) bytes (0 for fp32); for a BF16
  * network the workspace must be 256-byte and obs 16-byte aligned. */

@@ -89,6 +89,7 @@ def lib():
             "or_fleet_windows": (i32, [i32, i32, vp, vp, i32, vp, i64, i32, vp, i32, i64,
                                        vp, vp]),
             "or_fleet_stagger": (i32, [i32, i32, vp, vp, i32, i32, i32, i32, vp, vp]),
+            "or_dual_ascent": (f64, [vp, i32, i64, i32, i32, f64, f64, f64, f64, f64, vp]),
         }
         for name, (res, args) in sig.items():
             fn = getattr(L, name)
@@ -316,3 +317,13 @@ def fleet_stagger(traces, job_of_gpu, n_jobs: int, horizon: int, w: int, stride:
     if rc != 0:
         raise ValueError("oracle fleet stagger rejected its inputs")
     return offsets, peaks
+
+
+def dual_ascent(viol, steps: int, lam: float, target: float = 0.08, eta: float = 0.5, lo: float = 1e-3,
+                hi: float = 2.0, window: int = 60, additive: bool = False):
+    """Eq. 7 (or the additive G3 form): (new lambda, observed violation rate)."""
+    viol = np.ascontiguousarray(viol, np.int32).reshape(-1, 2)
+    rate = np.zeros(1, np.float64)
+    new = lib().or_dual_ascent(_p(viol), viol.shape[0], steps, window, int(additive), lam, target, eta,
+                               lo, hi, _p(rate))
+    return float(new), float(rate[0])

@@ -949,3 +949,26 @@ int32_t or_fleet_stagger(int32_t G, int32_t L, const float* traces, const int32_
   free(qj);
   return 0;
 }
+
+/* ------------------------------------------------------------------------
+ * Dual ascent on the Lagrange multiplier of Eq. 6 (Eq. 7, Sec. 4.5; the G3
+ * design of Sec. 4.2): with the observed violation rate v = (violating
+ * steps) / (env-steps) over the last rollout (window = 1: instantaneous,
+ * 60: the 30 s window of Eq. 2) and target delta,
+ *   multiplicative (Eq. 7): lambda <- clip(lambda exp(eta (v - delta) / delta), lo, hi)
+ *   additive (G3):          lambda <- clip(lambda + eta (v - delta) / delta, lo, hi)
+ * viol is [E][2] (instantaneous, 30 s) as the rollout writes it.
+ * Returns the new lambda; *rate gets v.
+ * ---------------------------------------------------------------------- */
+double or_dual_ascent(const int32_t* viol, int32_t E, int64_t steps, int32_t window, int32_t additive,
+                      double lambda, double target, double eta, double lo, double hi, double* rate) {
+  int64_t n = 0;
+  for (int32_t e = 0; e < E; ++e) n += viol[2 * e + (window == 1 ? 0 : 1)];
+  const double v = (double)n / ((double)E * (double)steps);
+  const double gap = (v - target) / target;
+  double l = additive ? lambda + eta * gap : lambda * exp(eta * gap);
+  if (l < lo) l = lo;
+  if (l > hi) l = hi;
+  if (rate) *rate = v;
+  return l;
+}

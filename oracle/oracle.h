@@ -100,6 +100,8 @@ int32_t or_rollout_rule(const or_env_cfg* cfg, const float* trace, const uint8_t
                         or_env_state* states, int32_t T, uint32_t iteration, double lambda,
                         uint8_t* act, double* reward, uint8_t* done, int32_t* viol,
                         double* tokens, double* excess, int64_t* energy_q);
+double or_dual_ascent(const int32_t* viol, int32_t E, int64_t steps, int32_t window, int32_t additive,
+                      double lambda, double target, double eta, double lo, double hi, double* rate);
 void or_gae(int32_t T, int32_t E, const float* r, const float* v, const uint8_t* done,
             const float* last_v, double gamma, double lam, double* adv, double* ret);
 double or_ppo_minibatch_grad(int32_t D, int32_t H, int32_t A, const double* params, int64_t M,

@@ -97,6 +97,8 @@ struct RuleArgs {
 };
 pe_status rule_rollout(const EnvDev& env, const RuleArgs& r, const pe_rollout_buf& buf, cudaStream_t st);
 pe_status env_set_offsets(const EnvDev& env, const int32_t* offsets, int32_t* flag, cudaStream_t st);
+pe_status dual_ascent(const int32_t* viol, int E, int64_t steps, int window, int additive, float target,
+                      float eta, float lo, float hi, float* lambda, float* rate, cudaStream_t st);
 int64_t fleet_stagger_ws_bytes(int J, int L, int H, int stride);
 pe_status fleet_stagger_launch(const float* traces, int G, int L, const int32_t* job_of_gpu, int J, int H,
                                int w, int stride, int32_t* offsets_out, int32_t* peaks_out, void* workspace,
@@ -404,6 +406,20 @@ pe_status pe_rollout_rule(pe_env* env, const pe_rule* rule, int32_t horizon, uin
   RuleArgs r{rule->kind, rule->hi_q, rule->lo_q, rule->drop30_q, rule->climb30_q, rule->climb10_q,
              horizon, obs_bf16 ? 1 : 0, iteration, lambda};
   return rule_rollout(env->dev, r, *buf, reinterpret_cast<cudaStream_t>(stream));
+}
+
+pe_status pe_dual_ascent(const int32_t* viol, int32_t n_envs, int64_t steps, int32_t window, int32_t additive,
+                         float target, float eta, float lambda_min, float lambda_max, float* lambda, float* rate,
+                         void* stream) {
+  clear_error();
+  if (!viol || !lambda) return fail(PE_EINVAL, "null argument");
+  if (n_envs < 1 || steps < 1) return fail(PE_EINVAL, "n_envs >= 1 and steps >= 1 required");
+  if (window != 1 && window != 60) return fail(PE_EINVAL, "window must be 1 or 60");
+  if (!(target > 0.0f && target < 1.0f)) return fail(PE_EINVAL, "target must be in (0, 1)");
+  if (!(lambda_min >= 0.0f && lambda_max >= lambda_min) || !std::isfinite(eta) || !std::isfinite(lambda_max))
+    return fail(PE_EINVAL, "need 0 <= lambda_min <= lambda_max and a finite eta");
+  return dual_ascent(viol, n_envs, steps, window, additive ? 1 : 0, target, eta, lambda_min, lambda_max, lambda,
+                     rate, reinterpret_cast<cudaStream_t>(stream));
 }
 
 int64_t pe_rollout_workspace_bytes(const pe_env* env, const pe_net* net) {

@@ -142,4 +142,42 @@ pe_status env_set_offsets(const EnvDev& env, const int32_t* offsets, int32_t* fl
   return PE_OK;
 }
 
+// Dual ascent on the Eq. 6 multiplier (Eq. 7; the additive G3 form with the
+// same relative gap): one block sums the rollout's violation counts exactly
+// (int64), then one thread updates lambda in place.  The scalar update runs
+// in fp64 (a handful of operations).
+__global__ void __launch_bounds__(1024) dual_ascent_kernel(const int32_t* __restrict__ viol, int E, int64_t steps,
+                                                           int col, int additive, float target, float eta, float lo,
+                                                           float hi, float* __restrict__ lambda,
+                                                           float* __restrict__ rate) {
+  __shared__ long long red[32];
+  long long n = 0;
+  for (int e = threadIdx.x; e < E; e += blockDim.x) n += viol[2 * e + col];
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) n += __shfl_xor_sync(0xffffffffu, n, o);
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = n;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    long long t = 0;
+    for (int w = 0; w < (int)(blockDim.x >> 5); ++w) t += red[w];
+    const double v = (double)t / ((double)E * (double)steps);
+    const double gap = (v - (double)target) / (double)target;
+    double l = additive ? (double)*lambda + (double)eta * gap : (double)*lambda * exp((double)eta * gap);
+    l = l < (double)lo ? (double)lo : (l > (double)hi ? (double)hi : l);
+    *lambda = (float)l;
+    if (rate) *rate = (float)v;
+  }
+}
+
+pe_status dual_ascent(const int32_t* viol, int E, int64_t steps, int window, int additive, float target,
+                      float eta, float lo, float hi, float* lambda, float* rate, cudaStream_t st) {
+  {
+    ProfScope ps(PE_PROF_PPO_OTHER, st);
+    dual_ascent_kernel<<<1, 1024, 0, st>>>(viol, E, steps, window == 1 ? 0 : 1, additive, target, eta, lo, hi,
+                                           lambda, rate);
+  }
+  PE_CHECK_LAUNCH("dual_ascent_kernel");
+  return PE_OK;
+}
+
 }  // namespace pe

@@ -74,6 +74,7 @@ EXPORTS = (
     "pe_value", "pe_device_check", "pe_gae", "pe_ppo_workspace_bytes",
     "pe_ppo_update", "pe_fleet_workspace_bytes", "pe_fleet_windows", "pe_fleet_windows_noalloc",
     "pe_fleet_stagger_workspace_bytes", "pe_fleet_stagger", "pe_env_set_offsets", "pe_rollout_rule",
+    "pe_dual_ascent",
     "pe_profile_enable",
     "pe_profile_read", "pe_profile_kind_name", "pe_last_error")
 
@@ -105,6 +106,8 @@ def lib():
             "pe_fleet_workspace_bytes": (i64, [i32, i32, i32]),
             "pe_fleet_stagger_workspace_bytes": (i64, [i32, i32, i32, i32]),
             "pe_env_set_offsets": (i32, [vp, vp, vp]),
+            "pe_dual_ascent": (i32, [vp, i32, i64, i32, i32, C.c_float, C.c_float, C.c_float, C.c_float,
+                                     vp, vp, vp]),
             "pe_rollout_rule": (i32, [vp, vp, i32, u32, C.c_float, i32, vp, vp]),
             "pe_fleet_stagger": (i32, [vp, i32, i32, vp, i32, i32, i32, i32, vp, vp, vp, i64, vp]),
             "pe_fleet_windows": (i32, [vp, i32, i32, vp, i32, vp, i64, i32, vp, i32, i64, vp,
@@ -268,6 +271,14 @@ def rollout_rule(env: Env, rule: W.RuleSpec, T: int, iteration: int, buf: Dict[s
     r = Rule(rule.kind, rule.hi_q, rule.lo_q, rule.drop30_q, rule.climb30_q, rule.climb10_q)
     _check(lib().pe_rollout_rule(env._h, C.byref(r), T, iteration, lam, int(obs_bf16), C.byref(rb),
                                  _stream(stream)))
+
+
+def dual_ascent(viol: torch.Tensor, steps: int, lam: torch.Tensor, rate: Optional[torch.Tensor] = None,
+                target: float = 0.08, eta: float = 0.5, lo: float = 1e-3, hi: float = 2.0, window: int = 60,
+                additive: bool = False, stream=None):
+    """Eq. 7 update of the device scalar lam (float32) from a rollout's viol counts."""
+    _check(lib().pe_dual_ascent(_ptr(viol), viol.shape[0], steps, window, int(additive), target, eta, lo, hi,
+                                _ptr(lam), _ptr(rate), _stream(stream)))
 
 
 def value_workspace_bytes(net: W.NetSpec) -> int:

@@ -578,3 +578,30 @@ def test_set_offsets_rejects_out_of_range():
         pe.rollout_rule(env, W.RuleSpec(7), 10, 0, pe.alloc_rule_rollout(wl.env, 10))
     assert e.value.status == pe.PE_EINVAL
     env.close()
+
+
+# ------------------------------------------------------------- dual ascent
+def test_dual_ascent_parity_in_a_lagrange_loop():
+    """Three 72B rollouts with the Eq. 6 reward, lambda fed back through
+    Eq. 7 on the device after each: the observed rates and multipliers
+    match the oracle's update applied to the same counts (fp32 lambda)."""
+    wl = W.make_72b(n_envs=256)
+    spec = wl.env
+    env = pe.Env(spec, torch.from_numpy(wl.trace), torch.from_numpy(wl.phase))
+    T = 200
+    buf = pe.alloc_rule_rollout(spec, T)
+    lam = torch.tensor([1.0], device="cuda")
+    rate = torch.zeros(1, device="cuda")
+    lam_host = 1.0
+    for it, (add, tgt) in enumerate(((False, 0.08), (False, 0.02), (True, 0.3))):
+        pe.rollout_rule(env, W.random_rule(), T, it, buf, lam=lam_host)
+        pe.dual_ascent(buf["viol"], T, lam, rate, target=tgt, additive=add, hi=2.0 if not add else 20.0)
+        torch.cuda.synchronize()
+        o_lam, o_rate = O.dual_ascent(cpu(buf["viol"]), T, lam_host, target=tgt, additive=add,
+                                      hi=2.0 if not add else 20.0)
+        assert abs(float(rate.item()) - o_rate) <= 1e-7 * max(o_rate, 1e-3)
+        assert abs(float(lam.item()) - o_lam) <= 2e-7 * abs(o_lam)
+        lam_host = float(lam.item())
+    with pytest.raises(pe.PEError):
+        pe.dual_ascent(buf["viol"], T, lam, rate, window=30)
+    env.close()

@@ -686,3 +686,27 @@ def test_threshold_rule_constant_trace_hand_counted():
         q = [int(np.rint(np.float32(x * O.actuator_scale(spec, G)) * np.float32(64))) for G in g[:T]]
         assert out["energy_q"][0] == sum(q)
     del L
+
+
+# ------------------------------------------------------------- dual ascent
+def test_dual_ascent_eq7_closed_form():
+    """Eq. 7: on target the multiplier stays; at twice the target it grows by
+    e^eta; at zero violations it shrinks by e^-eta; the clip bounds hold;
+    the additive form moves by eta times the relative gap."""
+    E, T = 10, 100
+    viol = np.zeros((E, 2), np.int32)
+    viol[:, 1] = 8                     # 80 of 1000 env-steps: the 8% target exactly
+    lam, v = O.dual_ascent(viol, T, 1.0)
+    assert v == pytest.approx(0.08) and lam == pytest.approx(1.0, rel=1e-15)
+    viol[:, 1] = 16
+    lam, v = O.dual_ascent(viol, T, 1.0)
+    assert lam == pytest.approx(math.exp(0.5), rel=1e-15)
+    viol[:, 1] = 0
+    lam, _ = O.dual_ascent(viol, T, 1.0)
+    assert lam == pytest.approx(math.exp(-0.5), rel=1e-15)
+    viol[:, 1] = 100                   # every step violates
+    assert O.dual_ascent(viol, T, 1.9)[0] == 2.0
+    assert O.dual_ascent(np.zeros((E, 2)), T, 1e-3)[0] == 1e-3
+    viol[:, 0] = 4                     # the instantaneous count: half the target
+    lam, v = O.dual_ascent(viol, T, 3.0, window=1, additive=True, hi=20.0)
+    assert v == pytest.approx(0.04) and lam == pytest.approx(3.0 - 0.25, rel=1e-15)
