@@ -92,8 +92,8 @@ __device__ __forceinline__ bool dense_job(int j, int& eg, int& ng) {
   return ng < NG;
 }
 
-// outT[n][e] = tanh(b[n] + sum_k inT[k][e] WT[k][n])
-template <int TE, int K, int N, int LD, int RT>
+// outT[n][e] = tanh(b[n] + sum_k inT[k][e] WT[k][n]); WT rows are LDW floats apart
+template <int TE, int K, int N, int LD, int RT, int LDW = N>
 __device__ __forceinline__ void dense_fwd_w(const float* __restrict__ inT, const float* __restrict__ WT,
                                             const float* __restrict__ bias, float* __restrict__ outT) {
   constexpr int JOBS = (TE / RT) * (N / 4);
@@ -109,7 +109,7 @@ __device__ __forceinline__ void dense_fwd_w(const float* __restrict__ inT, const
     for (int k = 0; k < K; ++k) {
       float xv[RT];
       load_rt<RT>(inT + k * LD + eg * RT, xv);
-      const float4 w = *reinterpret_cast<const float4*>(WT + k * N + ng * 4);
+      const float4 w = *reinterpret_cast<const float4*>(WT + k * LDW + ng * 4);
       const float wv[4] = {w.x, w.y, w.z, w.w};
 #pragma unroll
       for (int r = 0; r < RT; ++r)
@@ -127,38 +127,50 @@ __device__ __forceinline__ void dense_fwd_w(const float* __restrict__ inT, const
   }
 }
 
-// back through a tanh layer, in place: hT[n][e] <- (sum_k inT[k][e] W[k][n]) * (1 - hT[n][e]^2).
-// Each thread reads hT only at the elements it writes.
-template <int TE, int K, int N, int LD, int RT>
-__device__ __forceinline__ void dense_bwd_inplace(const float* __restrict__ inT, const float* __restrict__ W,
-                                                  float* hT) {
-  constexpr int JOBS = (TE / RT) * (N / 4);
+// back through a tanh layer, in place, from the transposed weights:
+//   hT[k][e] <- (sum_n inT[n][e] W[n][k]) * (1 - hT[k][e]^2),  W[n][k] = WT[k][n]
+// A thread owns RT = 4 samples x 4 outputs k; per 4 n it loads a 4x4 block of
+// WT (rows k, columns n..n+3) and of inT and does 64 FMAs.  A warp covers 16
+// sample groups x 2 output groups, so its WT loads touch two rows (4 rows
+// apart, different banks with the padded stride) and are broadcasts.
+template <int TE, int K, int N, int LD, int LDW>
+__device__ __forceinline__ void dense_bwd_wt(const float* __restrict__ inT, const float* __restrict__ WT,
+                                             float* hT) {
+  constexpr int RT = 4, EG = TE / RT, NG = N / 4, JOBS = EG * NG;
+  static_assert(K % 4 == 0 && EG == 16, "backward tile layout");
   for (int j = threadIdx.x; j < JOBS; j += blockDim.x) {
-    int eg, ng;
-    if (!dense_job<TE, N, RT>(j, eg, ng)) continue;
+    const int eg = j % EG, kg = j / EG;
     float acc[RT][4];
 #pragma unroll
     for (int r = 0; r < RT; ++r)
 #pragma unroll
       for (int c = 0; c < 4; ++c) acc[r][c] = 0.0f;
-#pragma unroll 8
-    for (int k = 0; k < K; ++k) {
-      float xv[RT];
-      load_rt<RT>(inT + k * LD + eg * RT, xv);
-      const float4 w = *reinterpret_cast<const float4*>(W + k * N + ng * 4);
-      const float wv[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll 2
+    for (int n = 0; n < K; n += 4) {
+      float4 w[4], d[4];
 #pragma unroll
-      for (int r = 0; r < RT; ++r)
+      for (int c = 0; c < 4; ++c) w[c] = *reinterpret_cast<const float4*>(WT + (kg * 4 + c) * LDW + n);
 #pragma unroll
-        for (int c = 0; c < 4; ++c) acc[r][c] = fmaf(xv[r], wv[c], acc[r][c]);
+      for (int q = 0; q < 4; ++q) d[q] = *reinterpret_cast<const float4*>(inT + (n + q) * LD + eg * RT);
+#pragma unroll
+      for (int c = 0; c < 4; ++c) {
+        const float wc[4] = {w[c].x, w[c].y, w[c].z, w[c].w};
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          acc[0][c] = fmaf(d[q].x, wc[q], acc[0][c]);
+          acc[1][c] = fmaf(d[q].y, wc[q], acc[1][c]);
+          acc[2][c] = fmaf(d[q].z, wc[q], acc[2][c]);
+          acc[3][c] = fmaf(d[q].w, wc[q], acc[3][c]);
+        }
+      }
     }
 #pragma unroll
     for (int c = 0; c < 4; ++c) {
       float h[RT], o[RT];
-      load_rt<RT>(hT + (ng * 4 + c) * LD + eg * RT, h);
+      load_rt<RT>(hT + (kg * 4 + c) * LD + eg * RT, h);
 #pragma unroll
       for (int r = 0; r < RT; ++r) o[r] = acc[r][c] * (1.0f - h[r] * h[r]);
-      store_rt<RT>(hT + (ng * 4 + c) * LD + eg * RT, o);
+      store_rt<RT>(hT + (kg * 4 + c) * LD + eg * RT, o);
     }
   }
 }
@@ -216,6 +228,22 @@ struct WGradAcc {
       }
     }
   }
+  // dst (+)= acc in shared memory (the first slice stores)
+  __device__ __forceinline__ void add_to(float* dst, bool first) const {
+#pragma unroll
+    for (int q = 0; q < PER; ++q) {
+      int mg, ng;
+      if (job(q, mg, ng)) {
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+#pragma unroll
+          for (int j = 0; j < 4; ++j) {
+            float* d = dst + (mg + i * MG) * N + ng + j * NG;
+            *d = first ? acc[q][i][j] : *d + acc[q][i][j];
+          }
+      }
+    }
+  }
   __device__ __forceinline__ void store(float* __restrict__ dst) const {
 #pragma unroll
     for (int q = 0; q < PER; ++q) {
@@ -231,12 +259,18 @@ struct WGradAcc {
 };
 
 // Shared memory of one gradient CTA: the role's weights (W1 and W2
-// transposed for the forward pass, W2 as stored for the backward pass) and
-// one 64-sample slice of feature-major activations.  h2t holds h2, then the
+// transposed, w2t rows padded to H + 4 floats so that rows 4 apart fall in
+// different banks; the backward pass reads W2 from the same copy), the
+// CTA's accumulated weight gradients of both hidden layers, and one
+// 64-sample slice of feature-major activations.  h2t holds h2, then the
 // layer-2 pre-activation gradient; h1t holds h1, then the layer-1 one.
+template <int H>
+__host__ __device__ constexpr int w2t_ld() { return H + 4; }
+
 template <int D, int H, int A>
 struct PpoSmem {
-  float w1t[D * H], w2t[H * H], w2[H * H], w3[A * H], b1[H], b2[H], b3[8];
+  float w1t[D * H], w2t[H * w2t_ld<H>()], w3[A * H], b1[H], b2[H], b3[8];
+  float gw2[H * H], gw1[H * D];
   float xt[D * kPpoLD], h1t[H * kPpoLD], h2t[H * kPpoLD];
   float z[kPpoS * A];
   float lpo[kPpoS], advn[kPpoS], ret[kPpoS];
@@ -264,16 +298,16 @@ struct PpoArgs {
   int64_t P, PS;  // parameters; row stride of the partial-sum matrix
 };
 
-// Per-role weight image: the prefix of PpoSmem (w1t, w2t, w2, w3, b1, b2,
-// b3[8]) as it sits in shared memory, kept up to date by the Adam phase so
-// that a gradient CTA loads its weights as one contiguous float4 copy.
+// Per-role weight image: the prefix of PpoSmem (w1t, padded w2t, w3, b1,
+// b2, b3[8]) as it sits in shared memory, kept up to date by the Adam phase
+// so that a gradient CTA loads its weights as one contiguous float4 copy.
 // Image 0 is the policy network, image 1 the value network (its head is row
-// 0 of w3 and b3[0]).
+// 0 of w3 and b3[0]).  The padding floats of w2t stay zero.
 template <int D, int H, int A>
 struct RoleImage {
-  static constexpr int64_t W1T = 0, W2T = W1T + (int64_t)D * H, W2 = W2T + (int64_t)H * H,
-                           W3 = W2 + (int64_t)H * H, B1 = W3 + (int64_t)A * H, B2 = B1 + H, B3 = B2 + H,
-                           SIZE = B3 + 8;
+  static constexpr int64_t LDW = w2t_ld<H>();
+  static constexpr int64_t W1T = 0, W2T = W1T + (int64_t)D * H, W3 = W2T + (int64_t)H * LDW,
+                           B1 = W3 + (int64_t)A * H, B2 = B1 + H, B3 = B2 + H, SIZE = B3 + 8;
   static_assert(SIZE % 4 == 0, "role image is copied as float4");
 };
 
@@ -292,8 +326,7 @@ __device__ __forceinline__ void store_image(float* img, int64_t p, float val) {
     m[I::B1 + (p - b1)] = val;
   } else if (p < b2) {
     const int64_t q = p - w2;                       // W2[n][k], n = q / H, k = q % H
-    m[I::W2T + (q % H) * H + q / H] = val;
-    m[I::W2 + q] = val;
+    m[I::W2T + (q % H) * I::LDW + q / H] = val;
   } else if (p < w3) {
     m[I::B2 + (p - b2)] = val;
   } else if (p < b3) {
@@ -378,10 +411,9 @@ __device__ __forceinline__ void ppo_role(PpoSmem<D, H, A>& s, const PpoArgs& g, 
         if (i0 + u * kPpoNT < N4) dst[i0 + u * kPpoNT] = v[u];
     }
   }
-  WGradAcc<H, H, kPpoNT> g2;
-  WGradAcc<H, D, kPpoNT> g1;
-  g2.zero();
-  g1.zero();
+  // weight-gradient tiles live in registers only during their phase; each
+  // slice adds them into the CTA's shared-memory accumulators gw2 / gw1
+  int nsl = 0;
   // head backward: thread (k = tid / 4, quarter q = tid % 4) owns row k of the
   // head weight gradient and of the layer-2 bias gradient over samples 4i + q
   const int hk = tid >> 2, hq = tid & 3;
@@ -401,7 +433,7 @@ __device__ __forceinline__ void ppo_role(PpoSmem<D, H, A>& s, const PpoArgs& g, 
     // forward
     dense_fwd_w<S, D, H, LD, kPpoRT>(s.xt, s.w1t, s.b1, s.h1t);
     __syncthreads();
-    dense_fwd_w<S, H, H, LD, kPpoRT>(s.h1t, s.w2t, s.b2, s.h2t);
+    dense_fwd_w<S, H, H, LD, kPpoRT, w2t_ld<H>()>(s.h1t, s.w2t, s.b2, s.h2t);
     __syncthreads();
     // head: thread (sample si = tid / 8, K-part q = tid % 8) sums k = q, q+8, ...
     // for every action; the 8 parts (adjacent lanes) are shuffle-combined
@@ -502,24 +534,38 @@ __device__ __forceinline__ void ppo_role(PpoSmem<D, H, A>& s, const PpoArgs& g, 
     }
     __syncthreads();
     // layer-2 weight gradient
-    g2.template add<S, LD>(s.h2t, s.h1t);
+    {
+      WGradAcc<H, H, kPpoNT> g2;
+      g2.zero();
+      g2.template add<S, LD>(s.h2t, s.h1t);
+      g2.add_to(s.gw2, nsl == 0);
+    }
     __syncthreads();
     // back into layer 1 (in place over h1)
-    dense_bwd_inplace<S, H, H, LD, kPpoRT>(s.h2t, s.w2, s.h1t);
+    dense_bwd_wt<S, H, H, LD, w2t_ld<H>()>(s.h2t, s.w2t, s.h1t);
     __syncthreads();
     // layer-1 weight and bias gradients (the bias by the warps the tiles leave idle)
-    g1.template add<S, LD>(s.h1t, s.xt);
+    {
+      WGradAcc<H, D, kPpoNT> g1;
+      g1.zero();
+      g1.template add<S, LD>(s.h1t, s.xt);
+      g1.add_to(s.gw1, nsl == 0);
+    }
     if (tid >= kPpoNT - H) {
       const int n = tid - (kPpoNT - H), lane = tid & 31;
       float acc = 0.0f;
       for (int i = 0; i < S; ++i) acc += s.h1t[n * LD + ((i + lane) & (S - 1))];
       gb1 += acc;
     }
+    ++nsl;
   }
   // partial gradient row of this CTA (its network's slice of the parameter vector)
   float* row = g.partial + (int64_t)c * g.PS;
-  g1.store(row + oW1);
-  g2.store(row + oW2);
+  // the accumulated hidden-layer weight gradients, coalesced (zero if the
+  // CTA's slices held no sample)
+  __syncthreads();
+  for (int i = tid; i < H * H; i += blockDim.x) row[oW2 + i] = nsl ? s.gw2[i] : 0.0f;
+  for (int i = tid; i < H * D; i += blockDim.x) row[oW1 + i] = nsl ? s.gw1[i] : 0.0f;
 #pragma unroll
   for (int a = 0; a < NA; ++a) {
     g3[a] += __shfl_xor_sync(0xffffffffu, g3[a], 1);
@@ -909,7 +955,7 @@ static int64_t align256(int64_t x) { return (x + 255) / 256 * 256; }
 
 static int64_t img_floats(const pe_net& net) {
   const int64_t D = net.obs_dim, H = net.hidden, A = net.n_actions;
-  return D * H + 2 * H * H + A * H + 2 * H + 8;
+  return D * H + H * (H + 4) + A * H + 2 * H + 8;
 }
 
 static PpoPlan ppo_plan(const pe_net& net, const pe_ppo_config& cfg, int64_t N) {
@@ -980,6 +1026,7 @@ static pe_status ppo_run(const pe_net& net, float* params, float* m, float* v, i
   PE_CHECK_LAUNCH("ppo_advstats_kernel");
   {
     ProfScope ps(PE_PROF_PPO_OTHER, st);
+    PE_TRY_CUDA(cudaMemsetAsync(img, 0, 2 * img_floats(net) * sizeof(float), st));  // zero the w2t padding
     ppo_image_kernel<D, H, A><<<ceil_div(pl.P, 256), 256, 0, st>>>(params, img);
   }
   PE_CHECK_LAUNCH("ppo_image_kernel");
