@@ -228,8 +228,8 @@ struct WGradAcc {
       }
     }
   }
-  // dst (+)= acc in shared memory (the first slice stores)
-  __device__ __forceinline__ void add_to(float* dst, bool first) const {
+  // dst (+)= acc in shared memory, rows ld floats apart (the first slice stores)
+  __device__ __forceinline__ void add_to(float* dst, int ld, bool first) const {
 #pragma unroll
     for (int q = 0; q < PER; ++q) {
       int mg, ng;
@@ -238,7 +238,7 @@ struct WGradAcc {
         for (int i = 0; i < 4; ++i)
 #pragma unroll
           for (int j = 0; j < 4; ++j) {
-            float* d = dst + (mg + i * MG) * N + ng + j * NG;
+            float* d = dst + (mg + i * MG) * ld + ng + j * NG;
             *d = first ? acc[q][i][j] : *d + acc[q][i][j];
           }
       }
@@ -270,7 +270,7 @@ __host__ __device__ constexpr int w2t_ld() { return H + 4; }
 template <int D, int H, int A>
 struct PpoSmem {
   float w1t[D * H], w2t[H * w2t_ld<H>()], w3[A * H], b1[H], b2[H], b3[8];
-  float gw2[H * H], gw1[H * D];
+  float gw2[H * w2t_ld<H>()], gw1[H * D];  // gw2 rows padded like w2t (conflict-free adds)
   float xt[D * kPpoLD], h1t[H * kPpoLD], h2t[H * kPpoLD];
   float z[kPpoS * A];
   float lpo[kPpoS], advn[kPpoS], ret[kPpoS];
@@ -538,7 +538,7 @@ __device__ __forceinline__ void ppo_role(PpoSmem<D, H, A>& s, const PpoArgs& g, 
       WGradAcc<H, H, kPpoNT> g2;
       g2.zero();
       g2.template add<S, LD>(s.h2t, s.h1t);
-      g2.add_to(s.gw2, nsl == 0);
+      g2.add_to(s.gw2, w2t_ld<H>(), nsl == 0);
     }
     __syncthreads();
     // back into layer 1 (in place over h1)
@@ -549,7 +549,7 @@ __device__ __forceinline__ void ppo_role(PpoSmem<D, H, A>& s, const PpoArgs& g, 
       WGradAcc<H, D, kPpoNT> g1;
       g1.zero();
       g1.template add<S, LD>(s.h1t, s.xt);
-      g1.add_to(s.gw1, nsl == 0);
+      g1.add_to(s.gw1, D, nsl == 0);
     }
     if (tid >= kPpoNT - H) {
       const int n = tid - (kPpoNT - H), lane = tid & 31;
@@ -564,7 +564,7 @@ __device__ __forceinline__ void ppo_role(PpoSmem<D, H, A>& s, const PpoArgs& g, 
   // the accumulated hidden-layer weight gradients, coalesced (zero if the
   // CTA's slices held no sample)
   __syncthreads();
-  for (int i = tid; i < H * H; i += blockDim.x) row[oW2 + i] = nsl ? s.gw2[i] : 0.0f;
+  for (int i = tid; i < H * H; i += blockDim.x) row[oW2 + i] = nsl ? s.gw2[(i / H) * w2t_ld<H>() + i % H] : 0.0f;
   for (int i = tid; i < H * D; i += blockDim.x) row[oW1 + i] = nsl ? s.gw1[i] : 0.0f;
 #pragma unroll
   for (int a = 0; a < NA; ++a) {
