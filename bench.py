@@ -585,7 +585,41 @@ def run_72b(args, world, peaks):
                              "peak": hbm, "unit": "GB/s", "frac": gae_gbs / hbm if gae_gbs else None,
                              "avg_launch_ms": gms / gn if gn else None,
                              "traffic": gae_traffic(T * E)},
-            "ppo_update": ppo72, "dual_ascent_eq7": dual}
+            "ppo_update": ppo72, "dual_ascent_eq7": dual,
+            "cadence": run_72b_cadence(args, world)}
+
+
+def run_72b_cadence(args, world):
+    """The 72B env at the Sec. 4.5 batch cadence (a step is one generation
+    batch of 24-42 samples): 65,536 envs x 64 batch steps on the tcgen05
+    policy; reports batch-steps/s and the trace samples consumed per second."""
+    from paper_2608_11226_gb300 import pe
+    from paper_2608_11226_gb300 import workloads as W
+    wl = W.make_72b_cadence(n_envs=args.r72b_envs)
+    spec, net = wl.env, wl.net
+    T = 64
+    env = pe.Env(spec, torch.from_numpy(wl.trace), torch.from_numpy(wl.phase))
+    buf = pe.alloc_rollout(spec, net, T)
+    params = torch.from_numpy(W.init_params(net, seed=0)).cuda()
+    ws = pe.alloc_workspace(pe.rollout_workspace_bytes(env, net))
+    pe.rollout(env, net, params, T, 0, buf, lam=1.0, workspace=ws)
+    torch.cuda.synchronize()
+    barrier(world)
+    a = torch.cuda.Event(enable_timing=True)
+    b = torch.cuda.Event(enable_timing=True)
+    a.record()
+    pe.rollout(env, net, params, T, 1, buf, lam=1.0, workspace=ws)
+    b.record()
+    torch.cuda.synchronize()
+    pe.device_check()
+    ms = max_over_ranks(a.elapsed_time(b), world)
+    samples = int(buf["samples"].sum())
+    env.close()
+    return {"metric": "72B batch-cadence rollout steps/s", "value": spec.n_envs * T * world / (ms / 1e3),
+            "unit": "batch-steps/s", "samples_per_s": samples * world / (ms / 1e3), "ms_per_rollout": ms,
+            "mean_samples_per_step": samples / (spec.n_envs * T),
+            "config": {"workload": f"72b cadence: {spec.n_envs} envs x {T} batch steps of 24-42 samples, "
+                                   "40-batch episodes, MLP 32-256-256 bf16"}}
 
 
 def run_72b_ppo(args, world, peaks, wl, buf, adv, ret):

@@ -95,6 +95,16 @@ typedef struct pe_env_config {
   float level_scale[PE_MAX_LEVELS][PE_MAX_CHANNELS];
   float level_tokens[PE_MAX_LEVELS];
   uint64_t seed;            /* Philox4x32-10 key */
+  /* Batch-boundary cadence (Sec. 4.5, Sec. 6.5): samples one step consumes
+   * at each level, in [1, 1024]; all zero: one sample per step.  With a
+   * table, a step is one generation batch: the windows, violations (Eq. 2)
+   * and excess (Eq. 3) advance sample by sample, tokens and excess are
+   * summed over the batch, and the Eq. 6 reward takes the batch's largest
+   * 30 s excess as its peak term; the Eq. 5 feature d_{k-1}/20 becomes the
+   * batch just completed, level_samples[level] x 0.5 s / 20 s.  Episodes
+   * are episode_len batches, drawn so that episode_len x max(level_samples)
+   * samples fit in the trace. */
+  int32_t level_samples[PE_MAX_LEVELS];
 } pe_env_config;
 
 /* Policy/value network: two separate tanh MLPs obs_dim -> hidden -> hidden
@@ -125,6 +135,9 @@ typedef struct pe_rollout_buf {
   float* tokens;      /* [E]    generated tokens of this call */
   float* excess;      /* [E]    integrated excess of this call, W*s (Eq. 3) */
   int64_t* energy_q;  /* [E]    sum of actuated cluster power over the call, 1/64 W per sample */
+  int64_t* samples;   /* [E]    trace samples consumed this call (optional, NULL skips); with a
+                       *        cadence table the violation counts are per sample, so rates
+                       *        divide by this count */
 } pe_rollout_buf;
 
 /* PPO configuration (Sec. 4.2 / 4.5; SB3 defaults where the paper is silent) */

@@ -43,7 +43,8 @@ class EnvCfg(C.Structure):
         ("r_ok", C.c_double), ("r_viol", C.c_double), ("bonus_coef", C.c_double),
         ("level_scale", (C.c_float * MAX_CH) * MAX_LEVELS),
         ("level_tokens", C.c_double * MAX_LEVELS),
-        ("seed", C.c_uint64)]
+        ("seed", C.c_uint64),
+        ("level_samples", C.c_int32 * MAX_LEVELS)]
 
 
 class PPOCfg(C.Structure):
@@ -72,11 +73,11 @@ def lib():
             "or_env_init": (i32, [vp, vp, vp, vp, i32, vp]),
             "or_env_set_offsets": (i32, [vp, vp, vp, vp, i32, vp]),
             "or_rollout_rule": (i32, [vp, vp, vp, vp, vp, i32, vp, i32, u32, f64, vp, vp, vp, vp,
-                                      vp, vp, vp]),
+                                      vp, vp, vp, vp]),
             "or_env_obs": (None, [vp, vp, vp, vp, vp]),
             "or_mlp_forward": (None, [i32, i32, i32, i32, vp, i64, vp, vp, vp]),
             "or_rollout": (i32, [vp, vp, vp, vp, i32, i32, vp, i32, vp, i32, u32, f64, i32,
-                                 vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp]),
+                                 vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp]),
             "or_gae": (None, [i32, i32, vp, vp, vp, vp, f64, f64, vp, vp]),
             "or_ppo_minibatch_grad": (f64, [i32, i32, i32, vp, i64, vp, vp, vp, vp, vp,
                                             f64, f64, f64, vp, vp]),
@@ -139,6 +140,8 @@ def env_cfg(spec) -> EnvCfg:
     for l, v in enumerate(spec.level_tokens):
         c.level_tokens[l] = float(v)
     c.seed = int(spec.seed)
+    for l, v in enumerate(getattr(spec, "level_samples", None) or []):
+        c.level_samples[l] = int(v)
     return c
 
 
@@ -192,14 +195,15 @@ class OracleEnv:
             act_own=np.zeros((T, n), np.uint8), logp=np.zeros((T, n), np.float64),
             reward=np.zeros((T, n), np.float64), done=np.zeros((T, n), np.uint8),
             viol=np.zeros((n, 2), np.int32), tokens=np.zeros(n, np.float64),
-            excess=np.zeros(n, np.float64), energy_q=np.zeros(n, np.int64))
+            excess=np.zeros(n, np.float64), energy_q=np.zeros(n, np.int64),
+            samples=np.zeros(n, np.int64))
         f = None if forced is None else np.ascontiguousarray(forced, np.uint8)
         lib().or_rollout(C.byref(self.cfg), _p(self.trace), _p(self.phase), _p(params), hidden,
                          int(bf16), _p(self.env_ids), n, _p(self.state), T, iteration, lam,
                          int(deterministic), _p(f), _p(out["obs"]), _p(out["obs_last"]),
                          _p(out["act_own"]), _p(out["logp"]), _p(out["reward"]), _p(out["done"]),
                          _p(out["viol"]), _p(out["tokens"]), _p(out["excess"]),
-                         _p(out["energy_q"]))
+                         _p(out["energy_q"]), _p(out["samples"]))
         return out
 
 
@@ -216,12 +220,13 @@ class OracleEnv:
         out = dict(act=np.zeros((T, n), np.uint8), reward=np.zeros((T, n), np.float64),
                    done=np.zeros((T, n), np.uint8), viol=np.zeros((n, 2), np.int32),
                    tokens=np.zeros(n, np.float64), excess=np.zeros(n, np.float64),
-                   energy_q=np.zeros(n, np.int64))
+                   energy_q=np.zeros(n, np.int64), samples=np.zeros(n, np.int64))
         r = or_rule(rule)
         if lib().or_rollout_rule(C.byref(self.cfg), _p(self.trace), _p(self.phase), C.byref(r),
                                  _p(self.env_ids), n, _p(self.state), T, iteration, lam,
                                  _p(out["act"]), _p(out["reward"]), _p(out["done"]), _p(out["viol"]),
-                                 _p(out["tokens"]), _p(out["excess"]), _p(out["energy_q"])) != 0:
+                                 _p(out["tokens"]), _p(out["excess"]), _p(out["energy_q"]),
+                                 _p(out["samples"])) != 0:
             raise ValueError("oracle rejected the rule")
         return out
 

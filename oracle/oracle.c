@@ -148,6 +148,29 @@ static int32_t qc_back(const or_env_cfg* cfg, const float* trace, const uint8_t*
   return s;
 }
 
+/* Batch-boundary cadence (Sec. 4.5): with a level table, one step is one
+ * generation batch and consumes level_samples[level] samples; without one,
+ * a step is one sample. */
+static int32_t cadence_on(const or_env_cfg* cfg) {
+  for (int32_t l = 0; l < OR_MAX_LEVELS; ++l)
+    if (cfg->level_samples[l] > 0) return 1;
+  return 0;
+}
+
+static int32_t step_samples(const or_env_cfg* cfg, int32_t level) {
+  return cfg->level_samples[level] > 0 ? cfg->level_samples[level] : 1;
+}
+
+static int32_t max_step_samples(const or_env_cfg* cfg) {
+  int32_t m = 1;
+  for (int32_t l = 0; l < OR_MAX_LEVELS; ++l)
+    if (cfg->level_samples[l] > m) m = cfg->level_samples[l];
+  return m;
+}
+
+/* samples one episode may span */
+static int32_t episode_span(const or_env_cfg* cfg) { return cfg->episode_len * max_step_samples(cfg); }
+
 /* Sec. 4.1: episodes start at a randomised offset; the history window is
  * warm-started at the default setting (Sec. 4.5 warm start). */
 static void env_reset_at(const or_env_cfg* cfg, const float* trace, const uint8_t* phase,
@@ -175,7 +198,7 @@ static void env_reset_at(const or_env_cfg* cfg, const float* trace, const uint8_
 static void env_reset(const or_env_cfg* cfg, const float* trace, const uint8_t* phase,
                       or_env_state* st, uint32_t e, uint32_t t, uint32_t it, uint32_t purpose) {
   uint32_t u = draw_u32(cfg->seed, e, t, it, purpose);
-  uint32_t span = (uint32_t)(cfg->trace_len - cfg->episode_len - OR_W_LONG + 1);
+  uint32_t span = (uint32_t)(cfg->trace_len - episode_span(cfg) - OR_W_LONG + 1);
   env_reset_at(cfg, trace, phase, st, OR_W_LONG + (int32_t)(((uint64_t)u * (uint64_t)span) >> 32));
 }
 
@@ -185,14 +208,14 @@ static void env_reset(const or_env_cfg* cfg, const float* trace, const uint8_t* 
 int32_t or_env_set_offsets(const or_env_cfg* cfg, const float* trace, const uint8_t* phase,
                            const int32_t* offsets, int32_t n, or_env_state* states) {
   for (int32_t i = 0; i < n; ++i)
-    if (offsets[i] < OR_W_LONG || offsets[i] > cfg->trace_len - cfg->episode_len) return 1;
+    if (offsets[i] < OR_W_LONG || offsets[i] > cfg->trace_len - episode_span(cfg)) return 1;
   for (int32_t i = 0; i < n; ++i) env_reset_at(cfg, trace, phase, &states[i], offsets[i]);
   return 0;
 }
 
 int32_t or_env_init(const or_env_cfg* cfg, const float* trace, const uint8_t* phase,
                     const int32_t* env_ids, int32_t n, or_env_state* states) {
-  if (cfg->trace_len < cfg->episode_len + OR_W_LONG) return 1;
+  if (cfg->trace_len < episode_span(cfg) + OR_W_LONG) return 1;
   for (int32_t i = 0; i < n; ++i)
     env_reset(cfg, trace, phase, &states[i], (uint32_t)env_ids[i], 0u, 0u, OR_PURPOSE_INIT);
   return 0;
@@ -233,7 +256,9 @@ void or_env_obs(const or_env_cfg* cfg, const float* trace, const uint8_t* phase,
       break;
     case OR_OBS_OCC32:
     case OR_OBS_OCC64: {
-      float d = ratio(st->til, 40); /* d / 20 s with d = til * 0.5 s */
+      /* d / 20 s: per-sample steps use the time since the last level change,
+       * the batch cadence the duration of the batch just completed */
+      float d = cadence_on(cfg) ? ratio(step_samples(cfg, st->level), 40) : ratio(st->til, 40);
       f[0] = ratio(Q0, B);
       f[1] = ratio(S20, OR_W_SHORT * B);
       f[2] = ratio(S60, OR_W_LONG * B);
@@ -286,7 +311,8 @@ static double token_rate_max(const or_env_cfg* cfg) {
 
 typedef struct {
   double reward, tokens, excess;
-  int32_t v1, v60, q, done;
+  int32_t v1, v60, done, samples;
+  int64_t q;
 } or_step_out;
 
 /* One environment step: apply the action (Sec. 4.1 action set, G >= 3 floor
@@ -312,35 +338,53 @@ static or_step_out env_step(const or_env_cfg* cfg, const float* trace, const uin
   st->prev_level = st->level;
   st->level = new_level;
 
-  const int32_t p = st->pos;
-  st->ring[p & (OR_RING - 1)] = (uint8_t)new_level;
-  int32_t Q = 0;
-  int64_t S60 = 0;
-  for (int32_t c = 0; c < cfg->n_channels; ++c) {
-    int32_t qin = q_of(cfg, trace, phase, c, p, new_level);
-    int32_t p20 = p - OR_W_SHORT, p60 = p - OR_W_LONG;
-    int32_t q20 = q_of(cfg, trace, phase, c, p20, st->ring[p20 & (OR_RING - 1)]);
-    int32_t q60 = q_of(cfg, trace, phase, c, p60, st->ring[p60 & (OR_RING - 1)]);
-    st->s_short[c] += qin - q20;
-    st->s_long[c] += qin - q60;
-    Q += qin;
-    S60 += st->s_long[c];
-  }
+  /* consume the step's samples: windows (Eq. 1), violations (Eq. 2) and
+   * excess (Eq. 3) per sample; tokens and excess summed over the step; the
+   * Eq. 6 peak term takes the step's largest 30 s excess */
   const int64_t B = cfg->budget_q;
-  o.q = Q;
-  o.v1 = Q > B;
-  o.v60 = S60 > (int64_t)OR_W_LONG * B;
-  double excess_w = o.v60 ? (double)(S60 - (int64_t)OR_W_LONG * B) / (64.0 * OR_W_LONG) : 0.0;
-  o.excess = excess_w * OR_DT;
-  double rate = token_rate(cfg, new_level, st->b);
-  o.tokens = phase[p] == 0 ? rate : 0.0;
-  if (cfg->reward_kind == OR_REWARD_LAGRANGE) {
-    o.reward = o.tokens / 1000.0 - lambda * o.excess - 2.0 * lambda * excess_w;
-  } else {
-    int32_t viol = cfg->reward_window == 1 ? o.v1 : o.v60;
-    o.reward = (viol ? cfg->r_viol : cfg->r_ok) + cfg->bonus_coef * rate / token_rate_max(cfg);
+  const int32_t ns = step_samples(cfg, new_level);
+  const double rate = token_rate(cfg, new_level, st->b);
+  o.q = 0;
+  o.v1 = 0;
+  o.v60 = 0;
+  o.tokens = 0.0;
+  o.excess = 0.0;
+  double peak_w = 0.0, fixed = 0.0;
+  for (int32_t i = 0; i < ns; ++i) {
+    const int32_t p = st->pos;
+    st->ring[p & (OR_RING - 1)] = (uint8_t)new_level;
+    int32_t Q = 0;
+    int64_t S60 = 0;
+    for (int32_t c = 0; c < cfg->n_channels; ++c) {
+      int32_t qin = q_of(cfg, trace, phase, c, p, new_level);
+      int32_t p20 = p - OR_W_SHORT, p60 = p - OR_W_LONG;
+      int32_t q20 = q_of(cfg, trace, phase, c, p20, st->ring[p20 & (OR_RING - 1)]);
+      int32_t q60 = q_of(cfg, trace, phase, c, p60, st->ring[p60 & (OR_RING - 1)]);
+      st->s_short[c] += qin - q20;
+      st->s_long[c] += qin - q60;
+      Q += qin;
+      S60 += st->s_long[c];
+    }
+    const int32_t v1 = Q > B, v60 = S60 > (int64_t)OR_W_LONG * B;
+    const double excess_w = v60 ? (double)(S60 - (int64_t)OR_W_LONG * B) / (64.0 * OR_W_LONG) : 0.0;
+    const double tok = phase[p] == 0 ? rate : 0.0;
+    o.q += Q;
+    o.v1 += v1;
+    o.v60 += v60;
+    o.excess += excess_w * OR_DT;
+    o.tokens += tok;
+    if (excess_w > peak_w) peak_w = excess_w;
+    if (cfg->reward_kind != OR_REWARD_LAGRANGE) {
+      int32_t viol = cfg->reward_window == 1 ? v1 : v60;
+      fixed += (viol ? cfg->r_viol : cfg->r_ok) + cfg->bonus_coef * rate / token_rate_max(cfg);
+    }
+    st->pos = p + 1;
   }
-  st->pos = p + 1;
+  o.samples = ns;
+  if (cfg->reward_kind == OR_REWARD_LAGRANGE)
+    o.reward = o.tokens / 1000.0 - lambda * o.excess - 2.0 * lambda * peak_w;
+  else
+    o.reward = fixed;
   st->k += 1;
   o.done = st->k == cfg->episode_len;
   return o;
@@ -461,7 +505,7 @@ int32_t or_rollout(const or_env_cfg* cfg, const float* trace, const uint8_t* pha
                    double lambda, int32_t deterministic, const uint8_t* forced, float* obs,
                    float* obs_last, uint8_t* act_own, double* logp_taken, double* reward,
                    uint8_t* done, int32_t* viol, double* tokens, double* excess,
-                   int64_t* energy_q) {
+                   int64_t* energy_q, int64_t* samples) {
   const int32_t D = cfg->obs_kind == OR_OBS_TINY8   ? 8
                     : cfg->obs_kind == OR_OBS_7B16  ? 16
                     : cfg->obs_kind == OR_OBS_OCC32 ? 32
@@ -478,7 +522,7 @@ int32_t or_rollout(const or_env_cfg* cfg, const float* trace, const uint8_t* pha
     const uint32_t e = (uint32_t)env_ids[i];
     int32_t v1 = 0, v60 = 0;
     double tok = 0.0, exc = 0.0;
-    int64_t en = 0;
+    int64_t en = 0, smp = 0;
     for (int32_t t = 0; t < T; ++t) {
       const int64_t row = (int64_t)t * n + i;
       or_env_obs(cfg, trace, phase, st, f);
@@ -515,6 +559,7 @@ int32_t or_rollout(const or_env_cfg* cfg, const float* trace, const uint8_t* pha
       tok += so.tokens;
       exc += so.excess;
       en += so.q;
+      smp += so.samples;
       if (so.done) env_reset(cfg, trace, phase, st, e, (uint32_t)t, iteration, OR_PURPOSE_RESET);
     }
     or_env_obs(cfg, trace, phase, st, f);
@@ -524,6 +569,7 @@ int32_t or_rollout(const or_env_cfg* cfg, const float* trace, const uint8_t* pha
     tokens[i] = tok;
     excess[i] = exc;
     energy_q[i] = en;
+    if (samples) samples[i] = smp;
   }
   free(x); free(h1); free(h2); free(z); free(f); free(P);
   return 0;
@@ -571,14 +617,14 @@ int32_t or_rollout_rule(const or_env_cfg* cfg, const float* trace, const uint8_t
                         const or_rule* rule, const int32_t* env_ids, int32_t n,
                         or_env_state* states, int32_t T, uint32_t iteration, double lambda,
                         uint8_t* act, double* reward, uint8_t* done, int32_t* viol,
-                        double* tokens, double* excess, int64_t* energy_q) {
+                        double* tokens, double* excess, int64_t* energy_q, int64_t* samples) {
   if (rule->kind < OR_RULE_RANDOM || rule->kind > OR_RULE_HYSTERESIS) return 1;
   for (int32_t i = 0; i < n; ++i) {
     or_env_state* st = &states[i];
     const uint32_t e = (uint32_t)env_ids[i];
     int32_t v1 = 0, v60 = 0;
     double tok = 0.0, exc = 0.0;
-    int64_t en = 0;
+    int64_t en = 0, smp = 0;
     for (int32_t t = 0; t < T; ++t) {
       const int64_t row = (int64_t)t * n + i;
       const int32_t a = rule_action(cfg, trace, phase, st, rule, e, (uint32_t)t, iteration);
@@ -591,6 +637,7 @@ int32_t or_rollout_rule(const or_env_cfg* cfg, const float* trace, const uint8_t
       tok += so.tokens;
       exc += so.excess;
       en += so.q;
+      smp += so.samples;
       if (so.done) env_reset(cfg, trace, phase, st, e, (uint32_t)t, iteration, OR_PURPOSE_RESET);
     }
     viol[2 * i] = v1;
@@ -598,6 +645,7 @@ int32_t or_rollout_rule(const or_env_cfg* cfg, const float* trace, const uint8_t
     tokens[i] = tok;
     excess[i] = exc;
     energy_q[i] = en;
+    if (samples) samples[i] = smp;
   }
   return 0;
 }

@@ -212,8 +212,14 @@ static pe_status check_env_config(const pe_env_config* c) {
   if (c->n_envs < 1) return fail(PE_EINVAL, "n_envs must be >= 1");
   if (c->n_channels < 1 || c->n_channels > PE_MAX_CHANNELS) return fail(PE_EINVAL, "n_channels must be in [1, 4]");
   if (c->episode_len < 1) return fail(PE_EINVAL, "episode_len must be >= 1");
-  if ((int64_t)c->trace_len < (int64_t)c->episode_len + kWLong)
-    return fail(PE_EINVAL, "trace_len (%d) must be >= episode_len + 60", c->trace_len);
+  int32_t nmax = 1;
+  for (int l = 0; l < PE_MAX_LEVELS; ++l) {
+    if (c->level_samples[l] < 0 || c->level_samples[l] > 1024)
+      return fail(PE_EINVAL, "level_samples[%d] outside [0, 1024]", l);
+    if (c->level_samples[l] > nmax) nmax = c->level_samples[l];
+  }
+  if ((int64_t)c->trace_len < (int64_t)c->episode_len * nmax + kWLong)
+    return fail(PE_EINVAL, "trace_len (%d) must be >= episode_len x max(level_samples) + 60", c->trace_len);
   if (obs_width(c->obs_kind) < 0) return fail(PE_EINVAL, "unknown obs_kind %d", c->obs_kind);
   if (c->n_levels < 1 || c->n_levels > PE_MAX_LEVELS) return fail(PE_EINVAL, "n_levels must be in [1, 32]");
   if (c->level_init < 0 || c->level_init >= c->n_levels) return fail(PE_EINVAL, "level_init out of range");
@@ -276,6 +282,14 @@ pe_status pe_env_create(const pe_env_config* cfg, const float* trace, const uint
         d.scale[l][c] = cfg->level_scale[l][c];
     }
   for (int l = 0; l < PE_MAX_LEVELS; ++l) d.tokens[l] = cfg->level_tokens[l];
+  int32_t nmax = 1;
+  d.cadence = 0;
+  for (int l = 0; l < PE_MAX_LEVELS; ++l) {
+    d.ns[l] = cfg->level_samples[l] > 0 ? cfg->level_samples[l] : 1;
+    if (cfg->level_samples[l] > 0) d.cadence = 1;
+    if (d.ns[l] > nmax) nmax = d.ns[l];
+  }
+  d.span = cfg->episode_len * nmax;
   double rmax = 0.0;
   if (cfg->actuator_kind == PE_ACT_INCDEC) {
     for (int l = cfg->g_min; l <= cfg->g_max; ++l)

@@ -24,6 +24,9 @@ struct EnvDev {
   float r_ok, r_viol, bonus_coef, inv_rate_max;
   float scale[PE_MAX_LEVELS][PE_MAX_CHANNELS];  // actuator table (INCDEC formula pre-evaluated)
   float tokens[PE_MAX_LEVELS];
+  int32_t ns[PE_MAX_LEVELS];  // samples per step at each level (1 without a cadence table)
+  int32_t cadence;            // a cadence table is set
+  int32_t span;               // samples one episode may span: ep_len * max ns
   uint64_t seed;
   const float* trace;    // [C][L]
   const uint8_t* phase;  // [L]
@@ -135,7 +138,7 @@ template <int C, class Acc>
 __device__ void env_reset(const EnvDev& env, Acc& a, uint32_t eg, uint32_t t, uint32_t it,
                           uint32_t purpose) {
   const uint32_t u = draw32(env.seed, eg, t, it, purpose);
-  const uint32_t span = (uint32_t)(env.L - env.ep_len - kWLong + 1);
+  const uint32_t span = (uint32_t)(env.L - env.span - kWLong + 1);
   env_reset_at<C>(env, a, kWLong + (int)__umulhi(u, span));
 }
 
@@ -194,7 +197,7 @@ __device__ __forceinline__ float feature(const EnvDev& env, Acc& a, int f) {
     case 4: return ratio_i((int64_t)Qcl<C>(env, a, 0) - Qcl<C>(env, a, 10), B);
     case 5: return ratio_i(a.level() + 1, env.n_levels);
     case 6: return ratio_i(a.prev() + 1, env.n_levels);
-    case 7: return fminf(ratio_i(a.til(), 40), 1.0f);
+    case 7: return fminf(env.cadence ? ratio_i(env.ns[a.level()], 40) : ratio_i(a.til(), 40), 1.0f);
     default: break;
   }
   if (OBS == PE_OBS_OCC32) {
@@ -223,7 +226,7 @@ __device__ __forceinline__ float feature(const EnvDev& env, Acc& a, int f) {
 
 struct StepOut {
   float reward, tokens, excess;
-  int32_t q, v1, v60, done;
+  int32_t q, v1, v60, done, samples;
 };
 
 // Apply action act and consume one sample (Sec. 4.1 actuator and action set
@@ -242,39 +245,55 @@ __device__ __forceinline__ StepOut env_step(const EnvDev& env, Acc& a, int act, 
   a.til() = (nl != a.level()) ? 0 : a.til() + 1;
   a.prev() = a.level();
   a.level() = nl;
-  const int p = a.pos();
-  const int ph = __ldg(env.phase + p);
-  int32_t Q = 0;
-  int64_t S60 = 0;
-#pragma unroll
-  for (int c = 0; c < C; ++c) {
-    const int32_t qin = quant64(__ldg(env.trace + (int64_t)c * env.L + p), actuator_scale(env, nl, c, ph));
-    const int32_t q20 = a.q_at(env, c, p - kWShort);
-    const int32_t q60 = a.q_at(env, c, p - kWLong);
-    a.ss(c) += qin - q20;
-    a.sl(c) += qin - q60;
-    a.push(c, p, qin);
-    Q += qin;
-    S60 += a.sl(c);
-  }
-  a.set_level_at(p, nl);  // after the window updates: slot p & 63 held position p - 64
+  // consume the step's samples (one, or a generation batch with a cadence
+  // table): windows, violations and excess per sample; tokens and excess
+  // summed; the Eq. 6 peak term is the batch's largest 30 s excess
   const int64_t B60 = (int64_t)kWLong * env.budget_q;
-  StepOut o;
-  o.q = Q;
-  o.v1 = Q > env.budget_q;
-  o.v60 = S60 > B60;
-  const float exc_w = o.v60 ? __fdiv_rn(__ll2float_rn(S60 - B60), 3840.0f) : 0.0f;  // watts over B
-  o.excess = exc_w * 0.5f;                                                            // Eq. 3, W*s
   float rate = env.tokens[nl];
   if (env.act_kind == PE_ACT_INCDEC) rate = __fdiv_rn(rate * (float)a.b(), (float)env.b_init);
-  o.tokens = ph == 0 ? rate : 0.0f;
-  if (env.reward_kind == PE_REWARD_LAGRANGE) {
-    o.reward = o.tokens / 1000.0f - lambda * o.excess - 2.0f * lambda * exc_w;  // Eq. 6
-  } else {
-    const int viol = env.reward_window == 1 ? o.v1 : o.v60;
-    o.reward = (viol ? env.r_viol : env.r_ok) + env.bonus_coef * rate * env.inv_rate_max;
+  StepOut o;
+  o.q = 0;
+  o.v1 = 0;
+  o.v60 = 0;
+  o.tokens = 0.0f;
+  o.excess = 0.0f;
+  float peak_w = 0.0f, fixed = 0.0f;
+  const int n = env.ns[nl];
+  for (int i = 0; i < n; ++i) {
+    const int p = a.pos();
+    const int ph = __ldg(env.phase + p);
+    int32_t Q = 0;
+    int64_t S60 = 0;
+#pragma unroll
+    for (int c = 0; c < C; ++c) {
+      const int32_t qin = quant64(__ldg(env.trace + (int64_t)c * env.L + p), actuator_scale(env, nl, c, ph));
+      const int32_t q20 = a.q_at(env, c, p - kWShort);
+      const int32_t q60 = a.q_at(env, c, p - kWLong);
+      a.ss(c) += qin - q20;
+      a.sl(c) += qin - q60;
+      a.push(c, p, qin);
+      Q += qin;
+      S60 += a.sl(c);
+    }
+    a.set_level_at(p, nl);  // after the window updates: slot p & 63 held position p - 64
+    const int v1 = Q > env.budget_q, v60 = S60 > B60;
+    const float exc_w = v60 ? __fdiv_rn(__ll2float_rn(S60 - B60), 3840.0f) : 0.0f;  // watts over B
+    o.q += Q;
+    o.v1 += v1;
+    o.v60 += v60;
+    o.excess += exc_w * 0.5f;                                                         // Eq. 3, W*s
+    o.tokens += ph == 0 ? rate : 0.0f;
+    peak_w = fmaxf(peak_w, exc_w);
+    if (env.reward_kind != PE_REWARD_LAGRANGE) {
+      const int viol = env.reward_window == 1 ? v1 : v60;
+      fixed += (viol ? env.r_viol : env.r_ok) + env.bonus_coef * rate * env.inv_rate_max;
+    }
+    a.pos() = p + 1;
   }
-  a.pos() = p + 1;
+  o.samples = n;
+  o.reward = env.reward_kind == PE_REWARD_LAGRANGE
+                 ? o.tokens / 1000.0f - lambda * o.excess - 2.0f * lambda * peak_w  // Eq. 6
+                 : fixed;
   a.k() += 1;
   o.done = a.k() == env.ep_len;
   return o;

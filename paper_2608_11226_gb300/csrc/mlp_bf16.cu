@@ -618,12 +618,14 @@ __global__ void __launch_bounds__(128) env_actobs_kernel(EnvDev env, ActArgs a, 
       buf.tokens[e] = so.tokens;
       buf.excess[e] = so.excess;
       buf.energy_q[e] = so.q;
+      if (buf.samples) buf.samples[e] = so.samples;
     } else {
       buf.viol[2 * e] += so.v1;
       buf.viol[2 * e + 1] += so.v60;
       buf.tokens[e] += so.tokens;
       buf.excess[e] += so.excess;
       buf.energy_q[e] += so.q;
+      if (buf.samples) buf.samples[e] += so.samples;
     }
     if (so.done) env_reset<C>(env, acc, (uint32_t)e, (uint32_t)a.t, a.it, kDrawReset);
   }

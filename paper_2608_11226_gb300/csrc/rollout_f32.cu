@@ -40,7 +40,7 @@ __global__ void __launch_bounds__(TE / 4 * H / 4)
 
   float* obs_out = reinterpret_cast<float*>(buf.obs);
   int32_t v1 = 0, v60 = 0;
-  int64_t energy = 0;
+  int64_t energy = 0, smp = 0;
   float tok = 0.0f, exc = 0.0f;
   const int tid = threadIdx.x;
 
@@ -84,6 +84,7 @@ __global__ void __launch_bounds__(TE / 4 * H / 4)
       v1 += so.v1;
       v60 += so.v60;
       energy += so.q;
+      smp += so.samples;
       tok += so.tokens;
       exc += so.excess;
       if (so.done) env_reset<C>(env, acc, eg, (uint32_t)t, it, kDrawReset);
@@ -97,6 +98,7 @@ __global__ void __launch_bounds__(TE / 4 * H / 4)
     buf.tokens[g] = tok;
     buf.excess[g] = exc;
     buf.energy_q[g] = energy;
+    if (buf.samples) buf.samples[g] = smp;
   }
   store_tile<TE, C>(env, s.env, e0, ne);
 }

@@ -66,7 +66,7 @@ __global__ void __launch_bounds__(128) rule_rollout_kernel(EnvDev env, RuleArgs 
   const size_t ob = r.obs_bf16 ? 2 : 4;
   int32_t v1 = 0, v60 = 0;
   float tok = 0.0f, exc = 0.0f;
-  int64_t en = 0;
+  int64_t en = 0, smp = 0;
   for (int t = 0; t < r.T; ++t) {
     const int64_t row = (int64_t)t * env.E + e;
     if (buf.obs) write_obs<C, OBS, D>(env, acc, reinterpret_cast<char*>(buf.obs) + row * D * ob, r.obs_bf16);
@@ -80,6 +80,7 @@ __global__ void __launch_bounds__(128) rule_rollout_kernel(EnvDev env, RuleArgs 
     tok += so.tokens;
     exc += so.excess;
     en += so.q;
+    smp += so.samples;
     if (so.done) env_reset<C>(env, acc, (uint32_t)e, (uint32_t)t, r.it, kDrawReset);
   }
   if (buf.obs_last) write_obs<C, OBS, D>(env, acc, reinterpret_cast<char*>(buf.obs_last) + (int64_t)e * D * ob, r.obs_bf16);
@@ -88,6 +89,7 @@ __global__ void __launch_bounds__(128) rule_rollout_kernel(EnvDev env, RuleArgs 
   buf.tokens[e] = tok;
   buf.excess[e] = exc;
   buf.energy_q[e] = en;
+  if (buf.samples) buf.samples[e] = smp;
   store_reg<C>(env, e, acc);
 }
 
@@ -98,7 +100,7 @@ __global__ void env_offsets_kernel(EnvDev env, const int32_t* __restrict__ offse
   const int e = blockIdx.x * blockDim.x + threadIdx.x;
   if (e >= env.E) return;
   const int o = offsets[e];
-  if (o < kWLong || o > env.L - env.ep_len) {
+  if (o < kWLong || o > env.L - env.span) {
     atomicOr(flag, 1);
     return;
   }
@@ -138,7 +140,7 @@ pe_status env_set_offsets(const EnvDev& env, const int32_t* offsets, int32_t* fl
   int32_t h = 0;
   PE_TRY_CUDA(cudaMemcpyAsync(&h, flag, sizeof(int32_t), cudaMemcpyDeviceToHost, st));
   PE_TRY_CUDA(cudaStreamSynchronize(st));
-  if (h) return fail(PE_EINVAL, "episode offset outside [60, L - episode_len]");
+  if (h) return fail(PE_EINVAL, "episode offset outside [60, L - episode_len x max(level_samples)]");
   return PE_OK;
 }
 

@@ -43,7 +43,8 @@ class EnvConfig(C.Structure):
         ("r_ok", C.c_float), ("r_viol", C.c_float), ("bonus_coef", C.c_float),
         ("level_scale", (C.c_float * MAX_CH) * MAX_LEVELS),
         ("level_tokens", C.c_float * MAX_LEVELS),
-        ("seed", C.c_uint64)]
+        ("seed", C.c_uint64),
+        ("level_samples", C.c_int32 * MAX_LEVELS)]
 
 
 class Net(C.Structure):
@@ -51,10 +52,12 @@ class Net(C.Structure):
                 ("dtype", C.c_int32)]
 
 
+ROLLOUT_FIELDS = ("obs", "obs_last", "act", "logp", "value", "last_value", "reward", "done", "viol",
+                  "tokens", "excess", "energy_q", "samples")
+
+
 class RolloutBuf(C.Structure):
-    _fields_ = [(n, C.c_void_p) for n in (
-        "obs", "obs_last", "act", "logp", "value", "last_value", "reward", "done", "viol",
-        "tokens", "excess", "energy_q")]
+    _fields_ = [(n, C.c_void_p) for n in ROLLOUT_FIELDS]
 
 
 class Rule(C.Structure):
@@ -154,6 +157,8 @@ def env_config(spec: W.EnvSpec) -> EnvConfig:
     for l, v in enumerate(spec.level_tokens):
         c.level_tokens[l] = float(v)
     c.seed = int(spec.seed)
+    for l, v in enumerate(spec.level_samples or []):
+        c.level_samples[l] = int(v)
     return c
 
 
@@ -212,13 +217,12 @@ def alloc_rollout(spec: W.EnvSpec, net: W.NetSpec, T: int, device="cuda") -> Dic
         value=torch.empty((T, E), **kw), last_value=torch.empty(E, **kw),
         reward=torch.empty((T, E), **kw), done=torch.empty((T, E), dtype=torch.uint8, **kw),
         viol=torch.empty((E, 2), dtype=torch.int32, **kw), tokens=torch.empty(E, **kw),
-        excess=torch.empty(E, **kw), energy_q=torch.empty(E, dtype=torch.int64, **kw))
+        excess=torch.empty(E, **kw), energy_q=torch.empty(E, dtype=torch.int64, **kw),
+        samples=torch.empty(E, dtype=torch.int64, **kw))
 
 
-def _rollout_buf(b: Dict[str, torch.Tensor]) -> RolloutBuf:
-    return RolloutBuf(*[b[k].data_ptr() for k in (
-        "obs", "obs_last", "act", "logp", "value", "last_value", "reward", "done", "viol",
-        "tokens", "excess", "energy_q")])
+def _rollout_buf(b: Dict[str, Optional[torch.Tensor]]) -> RolloutBuf:
+    return RolloutBuf(*[(b[k].data_ptr() if b.get(k) is not None else None) for k in ROLLOUT_FIELDS])
 
 
 def rollout_workspace_bytes(env: Env, net: W.NetSpec) -> int:
@@ -258,15 +262,14 @@ def alloc_rule_rollout(spec: W.EnvSpec, T: int, obs: bool = False, obs_bf16: boo
         act=torch.empty((T, E), dtype=torch.uint8, **kw), logp=None, value=None, last_value=None,
         reward=torch.empty((T, E), **kw), done=torch.empty((T, E), dtype=torch.uint8, **kw),
         viol=torch.empty((E, 2), dtype=torch.int32, **kw), tokens=torch.empty(E, **kw),
-        excess=torch.empty(E, **kw), energy_q=torch.empty(E, dtype=torch.int64, **kw))
+        excess=torch.empty(E, **kw), energy_q=torch.empty(E, dtype=torch.int64, **kw),
+        samples=torch.empty(E, dtype=torch.int64, **kw))
 
 
 def rollout_rule(env: Env, rule: W.RuleSpec, T: int, iteration: int, buf: Dict[str, torch.Tensor],
                  lam: float = 1.0, stream=None):
     """T steps of every env under a baseline rule policy (no network)."""
-    rb = RolloutBuf(*[(b.data_ptr() if (b := buf[k]) is not None else None) for k in (
-        "obs", "obs_last", "act", "logp", "value", "last_value", "reward", "done", "viol",
-        "tokens", "excess", "energy_q")])
+    rb = _rollout_buf(buf)
     obs_bf16 = buf["obs"] is not None and buf["obs"].dtype == torch.bfloat16
     r = Rule(rule.kind, rule.hi_q, rule.lo_q, rule.drop30_q, rule.climb30_q, rule.climb10_q)
     _check(lib().pe_rollout_rule(env._h, C.byref(r), T, iteration, lam, int(obs_bf16), C.byref(rb),

@@ -75,6 +75,8 @@ class EnvSpec:
     r_viol: float
     bonus_coef: float
     seed: int
+    # batch-boundary cadence (Sec. 4.5): samples a step consumes at each level; None: one
+    level_samples: Optional[List[int]] = None
 
     @property
     def obs_dim(self) -> int:
@@ -375,6 +377,17 @@ def make_72b(n_envs: int = 65536, seed: int = 0) -> Workload:
 def make_stress(n_envs: int = 262144, seed: int = 0, horizon: int = 2048) -> Workload:
     return _occ_workload("stress", n_envs, 380000, OBS_OCC64, 512, horizon, seed,
                          PPOSpec(epochs=4, minibatch=65536, ent_coef=0.01))
+
+
+def make_72b_cadence(n_envs: int = 65536, seed: int = 0) -> Workload:
+    """The 72B workload at the Sec. 4.5 / 6.5 decision cadence: one step is
+    one generation batch lasting 12 s (level 0) to 21 s (level 15), i.e. 24
+    to 42 half-second samples; an episode is 40 batches (about the 600 s of
+    the paper's episodes)."""
+    wl = make_72b(n_envs=n_envs, seed=seed)
+    wl.env.level_samples = [24 + (18 * l) // 15 for l in range(wl.env.n_levels)]
+    wl.env.episode_len = 40
+    return wl
 
 
 PRESETS = {"tiny": make_tiny, "7b": make_7b, "72b": make_72b, "stress": make_stress}

@@ -38,8 +38,16 @@ class BruteEnv:
         s = self.s
         seed = s.seed
         u = int(self.philox([self.e, t, it, purpose], [seed & 0xFFFFFFFF, seed >> 32])[0])
-        span = self.L - s.episode_len - W_LONG + 1
+        span = self.L - s.episode_len * self.nmax() - W_LONG + 1
         self.reset_at(W_LONG + ((u * span) >> 32))
+
+    def nsamp(self, level):
+        ls = self.s.level_samples
+        return ls[level] if ls and ls[level] > 0 else 1
+
+    def nmax(self):
+        ls = self.s.level_samples
+        return max([1] + [v for v in (ls or [])])
 
     def reset_at(self, o):
         s = self.s
@@ -73,7 +81,9 @@ class BruteEnv:
                   _f32ratio(self.b - s.b_min, s.b_max - s.b_min), _f32ratio(S20, 20 * B),
                   _f32ratio(Q0 - self.Q(10), B), np.float32(0)]
         else:
-            d = _f32ratio(self.til, 40)
+            # d / 20 s: time since the last level change, or with a cadence table
+            # the duration of the batch just completed
+            d = _f32ratio(self.nsamp(self.level), 40) if self.s.level_samples else _f32ratio(self.til, 40)
             f = [_f32ratio(Q0, B), _f32ratio(S20, 20 * B), _f32ratio(S60, 60 * B),
                  _f32ratio(60 * B - S60, 60 * B), _f32ratio(Q0 - self.Q(10), B),
                  _f32ratio(self.level + 1, s.n_levels), _f32ratio(self.prev + 1, s.n_levels),
@@ -120,22 +130,34 @@ class BruteEnv:
             new = a
         self.til = 0 if new != self.level else self.til + 1
         self.prev, self.level = self.level, new
-        p = self.pos
-        self.hist[p] = [self.q(c, p, new) for c in range(self.C)]
-        self.pos += 1
+        # one step consumes nsamp(level) samples (one without a cadence table)
+        v1 = v60 = qsum = 0
+        tokens = excess = peak_w = fixed = 0.0
+        for _ in range(self.nsamp(new)):
+            p = self.pos
+            self.hist[p] = [self.q(c, p, new) for c in range(self.C)]
+            self.pos += 1
+            Q = self.Q(0)
+            S60 = self.S(W_LONG)
+            a1, a60 = int(Q > B), int(S60 > 60 * B)
+            exc_w = (S60 - 60 * B) / 3840.0 if a60 else 0.0
+            tok = self.rate(new, self.b) if self.phase[p] == 0 else 0.0
+            v1 += a1
+            v60 += a60
+            qsum += Q
+            tokens += tok
+            excess += exc_w * 0.5
+            peak_w = max(peak_w, exc_w)
+            viol = a1 if s.reward_window == 1 else a60
+            fixed += (s.r_viol if viol else s.r_ok) + s.bonus_coef * self.rate(new, self.b) / self.rate_max()
         self.k += 1
-        Q = self.Q(0)
-        S60 = self.S(W_LONG)
-        v1, v60 = int(Q > B), int(S60 > 60 * B)
-        exc_w = (S60 - 60 * B) / 3840.0 if v60 else 0.0
-        tokens = self.rate(new, self.b) if self.phase[p] == 0 else 0.0
         if s.reward_kind == 1:
-            r = tokens / 1000.0 - lam * exc_w * 0.5 - 2.0 * lam * exc_w
+            r = tokens / 1000.0 - lam * excess - 2.0 * lam * peak_w
         else:
-            viol = v1 if s.reward_window == 1 else v60
-            r = (s.r_viol if viol else s.r_ok) + s.bonus_coef * self.rate(new, self.b) / self.rate_max()
+            r = fixed
         done = self.k == s.episode_len
-        out = dict(r=r, done=int(done), v1=v1, v60=v60, q=Q, tokens=tokens, excess=exc_w * 0.5)
+        out = dict(r=r, done=int(done), v1=v1, v60=v60, q=qsum, tokens=tokens, excess=excess,
+                   samples=self.nsamp(new))
         if done:
             self.reset(t, it, 1)
         return out

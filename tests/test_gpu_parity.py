@@ -259,6 +259,7 @@ def _rollout_case(wl, T, iters, sample_envs=None, det=False, lam=1.0):
         assert np.array_equal(g["done"], o["done"])
         assert np.array_equal(g["viol"], o["viol"])
         assert np.array_equal(g["energy_q"], o["energy_q"])
+        assert np.array_equal(g["samples"], o["samples"])
         assert rel_err(g["reward"], o["reward"]) <= TOL
         assert rel_err(g["tokens"], o["tokens"]) <= TOL
         assert rel_err(g["excess"], o["excess"]) <= TOL
@@ -277,6 +278,37 @@ def _rollout_case(wl, T, iters, sample_envs=None, det=False, lam=1.0):
 
 def test_rollout_parity_tiny_full():
     _rollout_case(W.make_tiny(), 128, iters=5)   # 640 steps: crosses an episode boundary
+
+
+def test_rollout_parity_tiny_cadence():
+    """The fused fp32 rollout with a cadence table (2, 3 or 5 samples per
+    step by level) across an episode boundary."""
+    wl = W.make_tiny(n_envs=40)
+    wl.env.level_samples = [2, 3, 5]
+    _rollout_case(wl, 300, iters=2)
+
+
+def test_rollout_parity_72b_cadence():
+    """The 72B env at the Sec. 4.5 batch cadence (24-42 samples per step,
+    40-batch episodes) on the tcgen05 path, crossing episode boundaries."""
+    _rollout_case(W.make_72b_cadence(n_envs=128), 30, iters=3, lam=0.7)
+
+
+def test_rule_rollout_parity_72b_cadence():
+    wl = W.make_72b_cadence(n_envs=64)
+    spec = wl.env
+    rule = W.hysteresis_rule(spec.budget_q)
+    env = pe.Env(spec, torch.from_numpy(wl.trace), torch.from_numpy(wl.phase))
+    oenv = O.OracleEnv(spec, wl.trace, wl.phase, range(64))
+    for it, T in ((0, 25), (1, 35)):
+        buf = pe.alloc_rule_rollout(spec, T)
+        pe.rollout_rule(env, rule, T, it, buf, lam=0.5)
+        torch.cuda.synchronize()
+        ref = oenv.rollout_rule(rule, T, it, lam=0.5)
+        for k in ("act", "done", "viol", "energy_q", "samples"):
+            assert np.array_equal(cpu(buf[k]), ref[k]), k
+        assert rel_err(cpu(buf["reward"]), ref["reward"]) <= TOL
+    env.close()
 
 
 def test_rollout_parity_tiny_ragged_tile():

@@ -73,7 +73,7 @@ def _brute_compare(wl, n_envs, T, iters=1, seed_actions=0):
         out = env.rollout(params, wl.net.hidden, wl.net.dtype == 1, T, it, lam=0.7, forced=forced)
         for i, b in enumerate(brutes):
             v1 = v60 = 0
-            en = 0
+            en = smp = 0
             tok = exc = 0.0
             for t in range(T):
                 o = b.obs()
@@ -81,13 +81,22 @@ def _brute_compare(wl, n_envs, T, iters=1, seed_actions=0):
                 st = b.step(int(forced[t, i]), 0.7, t, it)
                 assert out["done"][t, i] == st["done"]
                 assert abs(out["reward"][t, i] - st["r"]) <= 1e-12 * max(1.0, abs(st["r"]))
-                v1 += st["v1"]; v60 += st["v60"]; en += st["q"]
+                v1 += st["v1"]; v60 += st["v60"]; en += st["q"]; smp += st["samples"]
                 tok += st["tokens"]; exc += st["excess"]
             assert np.array_equal(out["obs_last"][i], b.obs())
             assert list(out["viol"][i]) == [v1, v60]
             assert out["energy_q"][i] == en
+            assert out["samples"][i] == smp
             assert abs(out["tokens"][i] - tok) <= 1e-9 * max(1.0, tok)
             assert abs(out["excess"][i] - exc) <= 1e-9 * max(1.0, exc)
+
+
+def test_env_72b_cadence_matches_bruteforce():
+    """Batch-boundary cadence (Sec. 4.5): a step consumes 24-42 samples by
+    level, the Eq. 6 reward sums the batch with its peak 30 s excess, and
+    episodes of 40 batches; two iterations cross an episode boundary."""
+    wl = W.make_72b_cadence(n_envs=2)
+    _brute_compare(wl, 2, 45, iters=2)
 
 
 def test_env_tiny_matches_bruteforce():
