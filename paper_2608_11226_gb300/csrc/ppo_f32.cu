@@ -20,9 +20,7 @@
 #include <cmath>
 #include <vector>
 
-#include <cooperative_groups.h>
 #include <cstddef>
-#include <cstdlib>
 
 #include "mlp_f32.cuh"
 
@@ -348,10 +346,7 @@ __global__ void ppo_image_kernel(const float* __restrict__ params, float* __rest
 // One role (policy or value network) of the minibatch gradient over this
 // CTA's slices: forward, loss, backward; weight-gradient partials in
 // registers, written as this CTA's row of the partial-sum matrix.
-// CLR > 0: the CTA is one of CLR same-role CTAs of a thread-block cluster;
-// the cluster sums its members' gradients over distributed shared memory
-// (in rank order) and writes one partial-sum row per cluster (row c / CLR).
-template <int D, int H, int A, bool POL, int CLR = 0>
+template <int D, int H, int A, bool POL>
 __device__ __forceinline__ void ppo_role(PpoSmem<D, H, A>& s, const PpoArgs& g, int c) {
   constexpr int NA = POL ? A : 1;
   constexpr int S = kPpoS, LD = kPpoLD;
@@ -564,6 +559,13 @@ __device__ __forceinline__ void ppo_role(PpoSmem<D, H, A>& s, const PpoArgs& g, 
     }
     ++nsl;
   }
+  // partial gradient row of this CTA (its network's slice of the parameter vector)
+  float* row = g.partial + (int64_t)c * g.PS;
+  // the accumulated hidden-layer weight gradients, coalesced (zero if the
+  // CTA's slices held no sample)
+  __syncthreads();
+  for (int i = tid; i < H * H; i += blockDim.x) row[oW2 + i] = nsl ? s.gw2[(i / H) * w2t_ld<H>() + i % H] : 0.0f;
+  for (int i = tid; i < H * D; i += blockDim.x) row[oW1 + i] = nsl ? s.gw1[i] : 0.0f;
 #pragma unroll
   for (int a = 0; a < NA; ++a) {
     g3[a] += __shfl_xor_sync(0xffffffffu, g3[a], 1);
@@ -571,61 +573,13 @@ __device__ __forceinline__ void ppo_role(PpoSmem<D, H, A>& s, const PpoArgs& g, 
   }
   gb2 += __shfl_xor_sync(0xffffffffu, gb2, 1);
   gb2 += __shfl_xor_sync(0xffffffffu, gb2, 2);
-  __syncthreads();
-  if constexpr (CLR > 0) {
-    // every gradient of the role in shared memory: gw2, gw1, and the small
-    // ones in the dead h2 buffer as [b1 | b2 | W3 | b3]
-    float* sm = s.h2t;
-    if (nsl == 0) {
-      for (int i = tid; i < H * w2t_ld<H>(); i += blockDim.x) s.gw2[i] = 0.0f;
-      for (int i = tid; i < H * D; i += blockDim.x) s.gw1[i] = 0.0f;
-    }
-    if (hq == 0 && hk < H) {
+  if (hq == 0 && hk < H) {
 #pragma unroll
-      for (int a = 0; a < NA; ++a) sm[2 * H + a * H + hk] = g3[a];
-      sm[H + hk] = gb2;
-    }
-    if (tid >= kPpoNT - H) sm[tid - (kPpoNT - H)] = gb1;
-    if (tid < NA) sm[2 * H + NA * H + tid] = gb3;
-    namespace cg = cooperative_groups;
-    cg::cluster_group cl = cg::this_cluster();
-    cl.sync();
-    // this rank's share of the role's parameters (canonical order W1 b1 W2 b2
-    // W3 b3 from oW1), summed over the cluster's CTAs in rank order
-    constexpr int PR = H * D + H + H * H + H + NA * H + NA;
-    constexpr int CH = (PR + CLR - 1) / CLR;
-    const int rank = (int)cl.block_rank();
-    float* out = g.partial + (int64_t)(c / CLR) * g.PS + oW1;
-    const int p1 = (rank + 1) * CH < PR ? (rank + 1) * CH : PR;
-    for (int p = rank * CH + tid; p < p1; p += blockDim.x) {
-      const float* loc;
-      if (p < H * D) loc = s.gw1 + p;
-      else if (p < H * D + H) loc = sm + (p - H * D);
-      else if (p < H * D + H + H * H) {
-        const int q = p - (H * D + H);
-        loc = s.gw2 + (q / H) * w2t_ld<H>() + q % H;
-      } else if (p < H * D + 2 * H + H * H) loc = sm + H + (p - (H * D + H + H * H));
-      else loc = sm + 2 * H + (p - (H * D + 2 * H + H * H));  // W3 then b3, contiguous
-      float v = 0.0f;
-#pragma unroll
-      for (int r = 0; r < CLR; ++r) v += *cl.map_shared_rank(loc, r);
-      out[p] = v;
-    }
-    cl.sync();  // no member overwrites its gradients before every rank has read them
-  } else {
-    // partial gradient row of this CTA (its network's slice of the parameter vector),
-    // zero where the CTA's slices held no sample
-    float* row = g.partial + (int64_t)c * g.PS;
-    for (int i = tid; i < H * H; i += blockDim.x) row[oW2 + i] = nsl ? s.gw2[(i / H) * w2t_ld<H>() + i % H] : 0.0f;
-    for (int i = tid; i < H * D; i += blockDim.x) row[oW1 + i] = nsl ? s.gw1[i] : 0.0f;
-    if (hq == 0 && hk < H) {
-#pragma unroll
-      for (int a = 0; a < NA; ++a) row[oW3 + (int64_t)a * H + hk] = g3[a];
-      row[oB2 + hk] = gb2;
-    }
-    if (tid >= kPpoNT - H) row[oB1 + tid - (kPpoNT - H)] = gb1;
-    if (tid < NA) row[oB3 + tid] = gb3;
+    for (int a = 0; a < NA; ++a) row[oW3 + (int64_t)a * H + hk] = g3[a];
+    row[oB2 + hk] = gb2;
   }
+  if (tid >= kPpoNT - H) row[oB1 + tid - (kPpoNT - H)] = gb1;
+  if (tid < NA) row[oB3 + tid] = gb3;
   // statistics of the CTA's samples (held by threads < S), fixed shuffle tree
   if (tid < S) {
 #pragma unroll
@@ -713,7 +667,7 @@ __device__ __forceinline__ bool grid_barrier(unsigned int* bar, int* s_ok) {
   return *s_ok != 0;
 }
 
-template <int D, int H, int A, int CLR = 0>
+template <int D, int H, int A>
 __global__ void __launch_bounds__(kPpoNT, 1) ppo_persistent_kernel(PpoLoop L) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   PpoSmem<D, H, A>& s = *reinterpret_cast<PpoSmem<D, H, A>*>(smem_raw);
@@ -721,7 +675,6 @@ __global__ void __launch_bounds__(kPpoNT, 1) ppo_persistent_kernel(PpoLoop L) {
   __shared__ float s_red[kPpoNT / 32];
   __shared__ float s_norm;
   const int NC = L.g.NC, tid = threadIdx.x;
-  const int NR = CLR > 0 ? NC / CLR : NC;  // rows of the partial-sum matrix
   const int64_t P = L.g.P;
   const int64_t PS = L.g.PS;
   const int64_t per = ((P + gridDim.x - 1) / gridDim.x + 3) / 4 * 4;
@@ -739,9 +692,9 @@ __global__ void __launch_bounds__(kPpoNT, 1) ppo_persistent_kernel(PpoLoop L) {
       g.advstat = L.advstat + (int64_t)ep * L.nmb + mb;
       // phase 1: gradient partials of this CTA's role and samples
       if ((int)blockIdx.x < NC)
-        ppo_role<D, H, A, true, CLR>(s, g, blockIdx.x);
+        ppo_role<D, H, A, true>(s, g, blockIdx.x);
       else
-        ppo_role<D, H, A, false, CLR>(s, g, blockIdx.x - NC);
+        ppo_role<D, H, A, false>(s, g, blockIdx.x - NC);
       if (!grid_barrier(L.bar, &s_ok)) {
         if (tid == 0) atomicExch(L.err, 1);
         return;
@@ -763,11 +716,11 @@ __global__ void __launch_bounds__(kPpoNT, 1) ppo_persistent_kernel(PpoLoop L) {
               float4 v[4];
 #pragma unroll
               for (int u = 0; u < 4; ++u)
-                if (rg + 8 * (h + u) < NR)
+                if (rg + 8 * (h + u) < NC)
                   v[u] = __ldcg(reinterpret_cast<const float4*>(g.partial + (int64_t)(rg + 8 * (h + u)) * PS + p));
 #pragma unroll
               for (int u = 0; u < 4; ++u)
-                if (rg + 8 * (h + u) < NR) {
+                if (rg + 8 * (h + u) < NC) {
                   acc4.x += v[u].x;
                   acc4.y += v[u].y;
                   acc4.z += v[u].z;
@@ -1140,37 +1093,7 @@ static pe_status ppo_run(const pe_net& net, float* params, float* m, float* v, i
     L.eps = cfg.eps;
     L.max_norm = cfg.max_grad_norm;
     void* kargs[] = {&L};
-    // first choice: clusters of 8 same-role CTAs that pre-reduce their
-    // gradients in distributed shared memory (8x fewer partial rows); if the
-    // device cannot co-schedule them, the plain cooperative launch
-    bool launched = false;
-    constexpr int kClr = 8;
-    static const bool no_cluster = std::getenv("PE_PPO_NO_CLUSTER") != nullptr;  // forces the plain launch
-    if (pl.NC % kClr == 0 && !no_cluster) {
-      auto pkc = ppo_persistent_kernel<D, H, A, kClr>;
-      cudaLaunchConfig_t lc = {};
-      cudaLaunchAttribute at[2];
-      at[0].id = cudaLaunchAttributeClusterDimension;
-      at[0].val.clusterDim.x = kClr;
-      at[0].val.clusterDim.y = 1;
-      at[0].val.clusterDim.z = 1;
-      at[1].id = cudaLaunchAttributeCooperative;
-      at[1].val.cooperative = 1;
-      lc.gridDim = dim3(2 * pl.NC);
-      lc.blockDim = dim3(kPpoNT);
-      lc.dynamicSmemBytes = (size_t)bytes;
-      lc.stream = st;
-      lc.attrs = at;
-      lc.numAttrs = 2;
-      int ncl = 0;
-      if (cudaFuncSetAttribute(pkc, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes) == cudaSuccess &&
-          cudaOccupancyMaxActiveClusters(&ncl, pkc, &lc) == cudaSuccess && ncl * kClr >= 2 * pl.NC) {
-        ProfScope ps(PE_PROF_PPO_GRAD, st);
-        launched = cudaLaunchKernelEx(&lc, pkc, L) == cudaSuccess;
-      }
-      if (!launched) (void)cudaGetLastError();  // clear a refused cluster launch; fall back below
-    }
-    if (!launched) {
+    {
       ProfScope ps(PE_PROF_PPO_GRAD, st);
       PE_TRY_CUDA(cudaLaunchCooperativeKernel((void*)pk, dim3(2 * pl.NC), dim3(kPpoNT), kargs, (size_t)bytes, st));
     }

@@ -6,7 +6,6 @@ that near-zero entries do not fail a pure relative test; sampled actions
 agree on >= 99.9% of steps under teacher forcing (the oracle steps with the
 GPU's actions, so one flipped sample cannot cascade).
 """
-import os
 import numpy as np
 import pytest
 import torch
@@ -638,18 +637,3 @@ def test_dual_ascent_parity_in_a_lagrange_loop():
     with pytest.raises(pe.PEError):
         pe.dual_ascent(buf["viol"], T, lam, rate, window=30)
     env.close()
-
-
-def test_ppo_plain_cooperative_path():
-    """The update without thread-block clusters (PE_PPO_NO_CLUSTER: the plain
-    cooperative launch, one partial-sum row per CTA) in a fresh process, on
-    the single-step and ragged cases of the clustered path."""
-    import subprocess
-    import sys
-    code = ("import sys; sys.path.insert(0, '.'); import pytest; "
-            "sys.exit(pytest.main(['-q', '-x', '-m', 'gpu', 'tests/test_gpu_parity.py', "
-            "'-k', 'ppo_single_step_parity or ppo_ragged_minibatches or ppo_7b_first_steps']))")
-    env = dict(os.environ, PE_PPO_NO_CLUSTER="1")
-    r = subprocess.run([sys.executable, "-c", code], env=env, capture_output=True, text=True,
-                       cwd=os.path.dirname(os.path.dirname(os.path.abspath(__file__))))
-    assert r.returncode == 0, r.stdout[-2000:] + r.stderr[-2000:]
