@@ -586,7 +586,8 @@ def run_72b(args, world, peaks):
                              "avg_launch_ms": gms / gn if gn else None,
                              "traffic": gae_traffic(T * E)},
             "ppo_update": ppo72, "dual_ascent_eq7": dual,
-            "cadence": run_72b_cadence(args, world)}
+            "cadence": run_72b_cadence(args, world),
+            "mixed_families": run_72b_mixed(args, world)}
 
 
 def run_72b_cadence(args, world):
@@ -620,6 +621,40 @@ def run_72b_cadence(args, world):
             "mean_samples_per_step": samples / (spec.n_envs * T),
             "config": {"workload": f"72b cadence: {spec.n_envs} envs x {T} batch steps of 24-42 samples, "
                                    "40-batch episodes, MLP 32-256-256 bf16"}}
+
+
+def run_72b_mixed(args, world):
+    """Domain randomisation (Sec. 4.2 G2): the 72B env drawing every episode
+    from a 72B-, 14B- or 7B-shaped trace family (own channel count and
+    budget), 65,536 envs x 1,024 steps on the tcgen05 policy."""
+    from paper_2608_11226_gb300 import pe
+    from paper_2608_11226_gb300 import workloads as W
+    wl = W.make_72b_mixed(n_envs=args.r72b_envs)
+    spec, net = wl.env, wl.net
+    T = args.r72b_horizon
+    env = pe.Env(spec, torch.from_numpy(wl.trace), torch.from_numpy(wl.phase))
+    buf = pe.alloc_rollout(spec, net, T)
+    params = torch.from_numpy(W.init_params(net, seed=0)).cuda()
+    ws = pe.alloc_workspace(pe.rollout_workspace_bytes(env, net))
+    pe.rollout(env, net, params, T, 0, buf, lam=1.0, workspace=ws)
+    torch.cuda.synchronize()
+    barrier(world)
+    a = torch.cuda.Event(enable_timing=True)
+    b = torch.cuda.Event(enable_timing=True)
+    a.record()
+    pe.rollout(env, net, params, T, 1, buf, lam=1.0, workspace=ws)
+    b.record()
+    torch.cuda.synchronize()
+    pe.device_check()
+    ms = max_over_ranks(a.elapsed_time(b), world)
+    v = buf["viol"].sum(0).cpu().numpy()
+    n = spec.n_envs * T
+    env.close()
+    return {"metric": "72B mixed-family rollout env-steps/s", "value": n * world / (ms / 1e3),
+            "unit": "env-steps/s", "ms_per_rollout": ms,
+            "violation_rate_30s": float(v[1]) / n,
+            "config": {"workload": f"72b mixed families: {spec.n_envs} envs x {T} steps, episodes drawn from "
+                                   "72B-/14B-/7B-shaped traces (4/2/1 GPUs, own budgets), MLP 32-256-256 bf16"}}
 
 
 def run_72b_ppo(args, world, peaks, wl, buf, adv, ret):

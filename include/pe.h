@@ -49,6 +49,7 @@ typedef int32_t pe_status;
 #define PE_ESTATE 6     /* object in the wrong state */
 
 #define PE_MAX_LEVELS 32
+#define PE_MAX_FAMILIES 4
 #define PE_MAX_CHANNELS 4
 
 /* actuator kinds */
@@ -105,6 +106,18 @@ typedef struct pe_env_config {
    * are episode_len batches, drawn so that episode_len x max(level_samples)
    * samples fit in the trace. */
   int32_t level_samples[PE_MAX_LEVELS];
+  /* Domain randomisation (Sec. 4.2, design G2): n_families in [2, 4] trace
+   * families, 0 or 1 for the single trace.  Every episode start draws its
+   * family f = floor(w1 * n_families / 2^32) from word 1 of the episode's
+   * Philox draw (word 0 keeps choosing the offset, now inside family f).
+   * Family f has fam_len[f] samples, fam_channels[f] <= n_channels GPUs and
+   * the budget fam_budget_q[f] (1/64 W), which normalises its state and
+   * decides its violations (the cap-relative state of G2).  With families,
+   * pe_env_create's trace is family-major [f][n_channels][fam_len[f]]
+   * (channels at or above fam_channels[f] are ignored) and its phase array
+   * [f][fam_len[f]]; trace_len and budget_q are then unused. */
+  int32_t n_families;
+  int32_t fam_len[PE_MAX_FAMILIES], fam_channels[PE_MAX_FAMILIES], fam_budget_q[PE_MAX_FAMILIES];
 } pe_env_config;
 
 /* Policy/value network: two separate tanh MLPs obs_dim -> hidden -> hidden

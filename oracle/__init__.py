@@ -44,7 +44,9 @@ class EnvCfg(C.Structure):
         ("level_scale", (C.c_float * MAX_CH) * MAX_LEVELS),
         ("level_tokens", C.c_double * MAX_LEVELS),
         ("seed", C.c_uint64),
-        ("level_samples", C.c_int32 * MAX_LEVELS)]
+        ("level_samples", C.c_int32 * MAX_LEVELS),
+        ("n_families", C.c_int32), ("fam_len", C.c_int32 * 4), ("fam_channels", C.c_int32 * 4),
+        ("fam_budget_q", C.c_int32 * 4)]
 
 
 class PPOCfg(C.Structure):
@@ -142,6 +144,11 @@ def env_cfg(spec) -> EnvCfg:
     c.seed = int(spec.seed)
     for l, v in enumerate(getattr(spec, "level_samples", None) or []):
         c.level_samples[l] = int(v)
+    c.n_families = int(getattr(spec, "n_families", 0) or 0)
+    for f in range(c.n_families):
+        c.fam_len[f] = int(spec.fam_len[f])
+        c.fam_channels[f] = int(spec.fam_channels[f])
+        c.fam_budget_q[f] = int(spec.fam_budget_q[f])
     return c
 
 

@@ -47,11 +47,15 @@ void or_philox4x32_10(const uint32_t ctr[4], const uint32_t key[2], uint32_t out
   out[0] = c0; out[1] = c1; out[2] = c2; out[3] = c3;
 }
 
-static uint32_t draw_u32(uint64_t seed, uint32_t a, uint32_t b, uint32_t c, uint32_t d) {
+static void draw_4(uint64_t seed, uint32_t a, uint32_t b, uint32_t c, uint32_t d, uint32_t out[4]) {
   uint32_t ctr[4] = {a, b, c, d};
   uint32_t key[2] = {(uint32_t)seed, (uint32_t)(seed >> 32)};
-  uint32_t out[4];
   or_philox4x32_10(ctr, key, out);
+}
+
+static uint32_t draw_u32(uint64_t seed, uint32_t a, uint32_t b, uint32_t c, uint32_t d) {
+  uint32_t out[4];
+  draw_4(seed, a, b, c, d, out);
   return out[0];
 }
 
@@ -171,6 +175,27 @@ static int32_t max_step_samples(const or_env_cfg* cfg) {
 /* samples one episode may span */
 static int32_t episode_span(const or_env_cfg* cfg) { return cfg->episode_len * max_step_samples(cfg); }
 
+/* The env as one trace family sees it (domain randomisation, Sec. 4.2 G2):
+ * the family's length, channel count and budget, and its slices of the
+ * family-major trace and phase buffers.  One family: the env itself. */
+static void fam_view(const or_env_cfg* cfg, const float* trace, const uint8_t* phase, int32_t f,
+                     or_env_cfg* cf, const float** tr, const uint8_t** ph) {
+  *cf = *cfg;
+  *tr = trace;
+  *ph = phase;
+  if (cfg->n_families <= 1) return;
+  int64_t to = 0, po = 0;
+  for (int32_t g = 0; g < f; ++g) {
+    to += (int64_t)cfg->n_channels * cfg->fam_len[g];
+    po += cfg->fam_len[g];
+  }
+  cf->trace_len = cfg->fam_len[f];
+  cf->n_channels = cfg->fam_channels[f];
+  cf->budget_q = cfg->fam_budget_q[f];
+  *tr = trace + to;
+  *ph = phase + po;
+}
+
 /* Sec. 4.1: episodes start at a randomised offset; the history window is
  * warm-started at the default setting (Sec. 4.5 warm start). */
 static void env_reset_at(const or_env_cfg* cfg, const float* trace, const uint8_t* phase,
@@ -195,11 +220,20 @@ static void env_reset_at(const or_env_cfg* cfg, const float* trace, const uint8_
   }
 }
 
+/* word 1 of the episode draw picks the trace family (G2 domain
+ * randomisation), word 0 the offset inside that family's trace */
 static void env_reset(const or_env_cfg* cfg, const float* trace, const uint8_t* phase,
                       or_env_state* st, uint32_t e, uint32_t t, uint32_t it, uint32_t purpose) {
-  uint32_t u = draw_u32(cfg->seed, e, t, it, purpose);
-  uint32_t span = (uint32_t)(cfg->trace_len - episode_span(cfg) - OR_W_LONG + 1);
-  env_reset_at(cfg, trace, phase, st, OR_W_LONG + (int32_t)(((uint64_t)u * (uint64_t)span) >> 32));
+  uint32_t w[4];
+  draw_4(cfg->seed, e, t, it, purpose, w);
+  const int32_t f = cfg->n_families > 1 ? (int32_t)(((uint64_t)w[1] * (uint64_t)cfg->n_families) >> 32) : 0;
+  or_env_cfg cf;
+  const float* tr;
+  const uint8_t* ph;
+  fam_view(cfg, trace, phase, f, &cf, &tr, &ph);
+  uint32_t span = (uint32_t)(cf.trace_len - episode_span(&cf) - OR_W_LONG + 1);
+  env_reset_at(&cf, tr, ph, st, OR_W_LONG + (int32_t)(((uint64_t)w[0] * (uint64_t)span) >> 32));
+  st->fam = f;
 }
 
 /* Episodes that start at given offsets (the evaluation replay of Sec. 4.4
@@ -207,15 +241,31 @@ static void env_reset(const or_env_cfg* cfg, const float* trace, const uint8_t* 
  * the 60-sample history and one full episode inside the trace. */
 int32_t or_env_set_offsets(const or_env_cfg* cfg, const float* trace, const uint8_t* phase,
                            const int32_t* offsets, int32_t n, or_env_state* states) {
-  for (int32_t i = 0; i < n; ++i)
-    if (offsets[i] < OR_W_LONG || offsets[i] > cfg->trace_len - episode_span(cfg)) return 1;
-  for (int32_t i = 0; i < n; ++i) env_reset_at(cfg, trace, phase, &states[i], offsets[i]);
+  for (int32_t i = 0; i < n; ++i) {
+    or_env_cfg cf;
+    const float* tr;
+    const uint8_t* ph;
+    fam_view(cfg, trace, phase, states[i].fam, &cf, &tr, &ph);
+    if (offsets[i] < OR_W_LONG || offsets[i] > cf.trace_len - episode_span(&cf)) return 1;
+  }
+  for (int32_t i = 0; i < n; ++i) {
+    or_env_cfg cf;
+    const float* tr;
+    const uint8_t* ph;
+    fam_view(cfg, trace, phase, states[i].fam, &cf, &tr, &ph);
+    env_reset_at(&cf, tr, ph, &states[i], offsets[i]);
+  }
   return 0;
 }
 
 int32_t or_env_init(const or_env_cfg* cfg, const float* trace, const uint8_t* phase,
                     const int32_t* env_ids, int32_t n, or_env_state* states) {
-  if (cfg->trace_len < episode_span(cfg) + OR_W_LONG) return 1;
+  if (cfg->n_families > 1) {
+    for (int32_t f = 0; f < cfg->n_families; ++f)
+      if (cfg->fam_len[f] < episode_span(cfg) + OR_W_LONG) return 1;
+  } else if (cfg->trace_len < episode_span(cfg) + OR_W_LONG) {
+    return 1;
+  }
   for (int32_t i = 0; i < n; ++i)
     env_reset(cfg, trace, phase, &states[i], (uint32_t)env_ids[i], 0u, 0u, OR_PURPOSE_INIT);
   return 0;
@@ -226,8 +276,8 @@ static float ratio(int64_t num, int64_t den) { return (float)num / (float)den; }
 /* Observation vectors: Sec. 4.1 (TINY8), the 7B state of the workload
  * (last 8 samples, 30 s mean, budget slack), Eq. 5 (OCC32 / OCC64 core),
  * all normalised by the budget B. */
-void or_env_obs(const or_env_cfg* cfg, const float* trace, const uint8_t* phase,
-                const or_env_state* st, float* f) {
+static void env_obs_view(const or_env_cfg* cfg, const float* trace, const uint8_t* phase,
+                         const or_env_state* st, float* f) {
   const int64_t B = cfg->budget_q;
   const int32_t C = cfg->n_channels;
   int64_t S20 = 0, S60 = 0;
@@ -289,6 +339,15 @@ void or_env_obs(const or_env_cfg* cfg, const float* trace, const uint8_t* phase,
     default:
       break;
   }
+}
+
+void or_env_obs(const or_env_cfg* cfg, const float* trace, const uint8_t* phase,
+                const or_env_state* st, float* f) {
+  or_env_cfg cf;
+  const float* tr;
+  const uint8_t* ph;
+  fam_view(cfg, trace, phase, st->fam, &cf, &tr, &ph);
+  env_obs_view(&cf, tr, ph, st, f);
 }
 
 static double token_rate(const or_env_cfg* cfg, int32_t level, int32_t b) {
@@ -525,7 +584,11 @@ int32_t or_rollout(const or_env_cfg* cfg, const float* trace, const uint8_t* pha
     int64_t en = 0, smp = 0;
     for (int32_t t = 0; t < T; ++t) {
       const int64_t row = (int64_t)t * n + i;
-      or_env_obs(cfg, trace, phase, st, f);
+      or_env_cfg cf;
+      const float* tr;
+      const uint8_t* ph;
+      fam_view(cfg, trace, phase, st->fam, &cf, &tr, &ph);
+      env_obs_view(&cf, tr, ph, st, f);
       memcpy(obs + row * D, f, sizeof(float) * (size_t)D);
       obs_to_double(D, f, x, bf16);
       policy_fwd(D, H, A, P, x, h1, h2, z, bf16);
@@ -551,7 +614,7 @@ int32_t or_rollout(const or_env_cfg* cfg, const float* trace, const uint8_t* pha
       int32_t a = forced ? (int32_t)forced[row] : own;
       act_own[row] = (uint8_t)own;
       logp_taken[row] = z[a] - m - log(S);
-      or_step_out so = env_step(cfg, trace, phase, st, a, lambda);
+      or_step_out so = env_step(&cf, tr, ph, st, a, lambda);
       reward[row] = so.reward;
       done[row] = (uint8_t)so.done;
       v1 += so.v1;
@@ -627,9 +690,13 @@ int32_t or_rollout_rule(const or_env_cfg* cfg, const float* trace, const uint8_t
     int64_t en = 0, smp = 0;
     for (int32_t t = 0; t < T; ++t) {
       const int64_t row = (int64_t)t * n + i;
-      const int32_t a = rule_action(cfg, trace, phase, st, rule, e, (uint32_t)t, iteration);
+      or_env_cfg cf;
+      const float* tr;
+      const uint8_t* ph;
+      fam_view(cfg, trace, phase, st->fam, &cf, &tr, &ph);
+      const int32_t a = rule_action(&cf, tr, ph, st, rule, e, (uint32_t)t, iteration);
       act[row] = (uint8_t)a;
-      or_step_out so = env_step(cfg, trace, phase, st, a, lambda);
+      or_step_out so = env_step(&cf, tr, ph, st, a, lambda);
       reward[row] = so.reward;
       done[row] = (uint8_t)so.done;
       v1 += so.v1;

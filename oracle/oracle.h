@@ -27,6 +27,7 @@
 #define OR_MAX_LEVELS 32
 #define OR_MAX_CH 4
 #define OR_RING 64
+#define OR_MAX_FAM 4
 
 enum { OR_ACT_SET_LEVEL = 0, OR_ACT_INCDEC = 1 };
 enum { OR_OBS_TINY8 = 0, OR_OBS_7B16 = 1, OR_OBS_OCC32 = 2, OR_OBS_OCC64 = 3 };
@@ -46,6 +47,13 @@ typedef struct {
   /* batch-boundary cadence (Sec. 4.5): samples one step consumes at each
    * level; all zero: one sample per step */
   int32_t level_samples[OR_MAX_LEVELS];
+  /* domain randomisation (Sec. 4.2, design G2): n_families trace families;
+   * family f has fam_len[f] samples, fam_channels[f] GPUs (<= n_channels)
+   * and budget fam_budget_q[f].  The trace buffer is family-major
+   * [f][n_channels][fam_len[f]] and the phase buffer [f][fam_len[f]].
+   * 0 or 1 family: the single trace of trace_len / n_channels / budget_q. */
+  int32_t n_families;
+  int32_t fam_len[OR_MAX_FAM], fam_channels[OR_MAX_FAM], fam_budget_q[OR_MAX_FAM];
 } or_env_cfg;
 
 typedef struct {
@@ -58,6 +66,7 @@ typedef struct {
   uint8_t ring[OR_RING];           /* level used for the sample at position p, at p & 63 */
   int32_t s_short[OR_MAX_CH];      /* 10 s window sum (20 samples), per channel */
   int32_t s_long[OR_MAX_CH];       /* 30 s window sum (60 samples), per channel */
+  int32_t fam;                     /* trace family of the current episode */
 } or_env_state;
 
 enum { OR_RULE_RANDOM = 1, OR_RULE_THRESHOLD = 2, OR_RULE_HYSTERESIS = 3 };

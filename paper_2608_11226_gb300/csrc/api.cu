@@ -218,8 +218,17 @@ static pe_status check_env_config(const pe_env_config* c) {
       return fail(PE_EINVAL, "level_samples[%d] outside [0, 1024]", l);
     if (c->level_samples[l] > nmax) nmax = c->level_samples[l];
   }
-  if ((int64_t)c->trace_len < (int64_t)c->episode_len * nmax + kWLong)
-    return fail(PE_EINVAL, "trace_len (%d) must be >= episode_len x max(level_samples) + 60", c->trace_len);
+  if (c->n_families < 0 || c->n_families > PE_MAX_FAMILIES) return fail(PE_EINVAL, "n_families must be in [0, 4]");
+  const int nf = c->n_families > 1 ? c->n_families : 1;
+  for (int f = 0; f < nf; ++f) {
+    const int64_t L = c->n_families > 1 ? c->fam_len[f] : c->trace_len;
+    const int32_t ch = c->n_families > 1 ? c->fam_channels[f] : c->n_channels;
+    const int64_t B = c->n_families > 1 ? c->fam_budget_q[f] : c->budget_q;
+    if (L < (int64_t)c->episode_len * nmax + kWLong)
+      return fail(PE_EINVAL, "trace length (%lld) must be >= episode_len x max(level_samples) + 60", (long long)L);
+    if (ch < 1 || ch > c->n_channels) return fail(PE_EINVAL, "family channel count outside [1, n_channels]");
+    if (B < 1 || B * kWLong * PE_MAX_CHANNELS >= INT32_MAX) return fail(PE_EINVAL, "budget_q out of range");
+  }
   if (obs_width(c->obs_kind) < 0) return fail(PE_EINVAL, "unknown obs_kind %d", c->obs_kind);
   if (c->n_levels < 1 || c->n_levels > PE_MAX_LEVELS) return fail(PE_EINVAL, "n_levels must be in [1, 32]");
   if (c->level_init < 0 || c->level_init >= c->n_levels) return fail(PE_EINVAL, "level_init out of range");
@@ -239,8 +248,7 @@ static pe_status check_env_config(const pe_env_config* c) {
   }
   if (c->obs_kind == PE_OBS_7B16 && c->actuator_kind != PE_ACT_INCDEC)
     return fail(PE_EINVAL, "7B16 observations need the inc/dec actuator");
-  if (c->budget_q < 1 || (int64_t)c->budget_q * kWLong * PE_MAX_CHANNELS >= INT32_MAX)
-    return fail(PE_EINVAL, "budget_q out of range");
+  (void)0;  // budgets checked per trace family above
   if (c->reward_kind != PE_REWARD_FIXED && c->reward_kind != PE_REWARD_LAGRANGE)
     return fail(PE_EINVAL, "unknown reward_kind");
   if (c->reward_window != 1 && c->reward_window != kWLong) return fail(PE_EINVAL, "reward_window must be 1 or 60");
@@ -255,21 +263,40 @@ pe_status pe_env_create(const pe_env_config* cfg, const float* trace, const uint
   pe_status s = check_env_config(cfg);
   if (s != PE_OK) return s;
   const int C = cfg->n_channels, L = cfg->trace_len, E = cfg->n_envs;
+  // trace families (one: the single [C][L] trace)
+  const int F = cfg->n_families > 1 ? cfg->n_families : 1;
+  int32_t fL[PE_MAX_FAMILIES], fC[PE_MAX_FAMILIES], fB[PE_MAX_FAMILIES];
+  int64_t ftoff[PE_MAX_FAMILIES], fpoff[PE_MAX_FAMILIES], tot_t = 0, tot_p = 0;
+  for (int f = 0; f < F; ++f) {
+    fL[f] = cfg->n_families > 1 ? cfg->fam_len[f] : L;
+    fC[f] = cfg->n_families > 1 ? cfg->fam_channels[f] : C;
+    fB[f] = cfg->n_families > 1 ? cfg->fam_budget_q[f] : cfg->budget_q;
+    ftoff[f] = tot_t;
+    fpoff[f] = tot_p;
+    tot_t += (int64_t)C * fL[f];
+    tot_p += fL[f];
+  }
   // host copies for validation (trace and phase may live in host or device memory)
-  std::vector<float> h((size_t)C * L);
-  std::vector<uint8_t> ph((size_t)L);
+  std::vector<float> h((size_t)tot_t);
+  std::vector<uint8_t> ph((size_t)tot_p);
   PE_TRY_CUDA(cudaMemcpy(h.data(), trace, sizeof(float) * h.size(), cudaMemcpyDefault));
   PE_TRY_CUDA(cudaMemcpy(ph.data(), phase, ph.size(), cudaMemcpyDefault));
-  for (int i = 0; i < L; ++i)
-    if (ph[i] > 7) return fail(PE_EINVAL, "phase label %d at %d outside [0, 7]", (int)ph[i], i);
+  for (int64_t i = 0; i < tot_p; ++i)
+    if (ph[i] > 7) return fail(PE_EINVAL, "phase label %d at %lld outside [0, 7]", (int)ph[i], (long long)i);
   pe_env* env = new pe_env();
   env->cfg = *cfg;
   EnvDev& d = env->dev;
   memset(&d, 0, sizeof(d));
-  d.E = E; d.C = C; d.L = L; d.A = cfg->n_actions; d.obs_kind = cfg->obs_kind;
+  d.E = E; d.C = C; d.L = fL[0]; d.A = cfg->n_actions; d.obs_kind = cfg->obs_kind;
   d.act_kind = cfg->actuator_kind; d.n_levels = cfg->n_levels; d.level_init = cfg->level_init;
   d.g_min = cfg->g_min; d.g_max = cfg->g_max; d.b_min = cfg->b_min; d.b_max = cfg->b_max;
-  d.b_init = cfg->b_init; d.ep_len = cfg->episode_len; d.budget_q = cfg->budget_q;
+  d.b_init = cfg->b_init; d.ep_len = cfg->episode_len; d.budget_q = fB[0];
+  d.F = F;
+  for (int f = 0; f < F; ++f) {
+    d.fL[f] = fL[f];
+    d.fC[f] = fC[f];
+    d.fB[f] = fB[f];
+  }
   d.phase_mask = cfg->scale_phase_mask; d.reward_kind = cfg->reward_kind;
   d.reward_window = cfg->reward_window; d.r_ok = cfg->r_ok; d.r_viol = cfg->r_viol;
   d.bonus_coef = cfg->bonus_coef; d.seed = cfg->seed;
@@ -304,10 +331,13 @@ pe_status pe_env_create(const pe_env_config* cfg, const float* trace, const uint
     float smax = 1.0f;
     for (int l = 0; l < cfg->n_levels; ++l) smax = fmaxf(smax, d.scale[l][c]);
     if (!(smax >= 0.0f) || !std::isfinite(smax)) { delete env; return fail(PE_EINVAL, "actuator scale not finite"); }
-    for (int i = 0; i < L; ++i) {
-      const float x = h[(size_t)c * L + i];
-      if (!std::isfinite(x) || x < 0.0f) { delete env; return fail(PE_EOVERFLOW, "trace sample (%d, %d) is not a finite non-negative power", c, i); }
-      qmax = fmax(qmax, (double)x * smax * 64.0);
+    for (int f = 0; f < F; ++f) {
+      if (c >= fC[f]) continue;  // channels a family does not have are never read
+      for (int i = 0; i < fL[f]; ++i) {
+        const float x = h[(size_t)(ftoff[f] + (int64_t)c * fL[f] + i)];
+        if (!std::isfinite(x) || x < 0.0f) { delete env; return fail(PE_EOVERFLOW, "trace sample (%d, %d) of family %d is not a finite non-negative power", c, i, f); }
+        qmax = fmax(qmax, (double)x * smax * 64.0);
+      }
     }
   }
   if (qmax * C * kWLong >= 2147483000.0) { delete env; return fail(PE_EOVERFLOW, "trace too large for the 1/64 W fixed point"); }
@@ -330,7 +360,11 @@ pe_status pe_env_create(const pe_env_config* cfg, const float* trace, const uint
     return e1 == cudaErrorMemoryAllocation ? fail(PE_ENOMEM, "device allocation failed")
                                            : cuda_fail(e1, "pe_env_create");
   }
-  d.trace = dtrace; d.phase = dphase; d.st = st; d.ring = ring; d.sums = sums;
+  for (int f = 0; f < F; ++f) {
+    d.ftrace[f] = dtrace + ftoff[f];
+    d.fphase[f] = dphase + fpoff[f];
+  }
+  d.st = st; d.ring = ring; d.sums = sums;
   env->flag = flag;
   PE_TRY_CUDA(cudaMemcpy(dtrace, h.data(), sizeof(float) * h.size(), cudaMemcpyHostToDevice));
   PE_TRY_CUDA(cudaMemcpy(dphase, ph.data(), ph.size(), cudaMemcpyHostToDevice));
@@ -344,8 +378,8 @@ pe_status pe_env_create(const pe_env_config* cfg, const float* trace, const uint
 pe_status pe_env_destroy(pe_env* env) {
   clear_error();
   if (!env) return PE_OK;
-  cudaFree((void*)env->dev.trace);
-  cudaFree((void*)env->dev.phase);
+  cudaFree((void*)env->dev.ftrace[0]);
+  cudaFree((void*)env->dev.fphase[0]);
   cudaFree(env->dev.st);
   cudaFree(env->dev.ring);
   cudaFree(env->dev.sums);

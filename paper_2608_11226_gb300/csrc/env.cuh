@@ -28,20 +28,40 @@ struct EnvDev {
   int32_t cadence;            // a cadence table is set
   int32_t span;               // samples one episode may span: ep_len * max ns
   uint64_t seed;
-  const float* trace;    // [C][L]
-  const uint8_t* phase;  // [L]
+  // trace families (domain randomisation, Sec. 4.2 G2; one family without
+  // it): family f has a [C][fL[f]] trace (channels >= fC[f] are zero), a
+  // [fL[f]] phase array and the budget fB[f] in 1/64 W
+  int32_t F;
+  const float* ftrace[PE_MAX_FAMILIES];
+  const uint8_t* fphase[PE_MAX_FAMILIES];
+  int32_t fL[PE_MAX_FAMILIES], fC[PE_MAX_FAMILIES], fB[PE_MAX_FAMILIES];
   // persistent env state, SoA
-  int32_t* st;     // [6][E]: pos, k, level, prev, b, til
+  int32_t* st;     // [7][E]: pos, k, level, prev, b, til, family
   uint8_t* ring;   // [E][64]: level used for the sample at position p (slot p & 63)
   int32_t* sums;   // [E][8]: s_short[4], s_long[4] (per channel)
 };
 
-enum { kStPos = 0, kStK, kStLevel, kStPrev, kStB, kStTil, kStN };
+enum { kStPos = 0, kStK, kStLevel, kStPrev, kStB, kStTil, kStFam, kStN };
+
+// one trace family's view (selected with constant indices: the EnvDev
+// arrays stay in kernel parameter space)
+struct Fam {
+  const float* trace;
+  const uint8_t* phase;
+  int32_t L, C, B;
+};
+
+__device__ __forceinline__ Fam fam_of(const EnvDev& env, int f) {
+  if (f == 1) return Fam{env.ftrace[1], env.fphase[1], env.fL[1], env.fC[1], env.fB[1]};
+  if (f == 2) return Fam{env.ftrace[2], env.fphase[2], env.fL[2], env.fC[2], env.fB[2]};
+  if (f == 3) return Fam{env.ftrace[3], env.fphase[3], env.fL[3], env.fC[3], env.fB[3]};
+  return Fam{env.ftrace[0], env.fphase[0], env.fL[0], env.fC[0], env.fB[0]};
+}
 
 // Per-tile env state staged in shared memory for the whole horizon.
 template <int TE, int C>
 struct EnvTile {
-  int32_t pos[TE], k[TE], level[TE], prev[TE], b[TE], til[TE];
+  int32_t pos[TE], k[TE], level[TE], prev[TE], b[TE], til[TE], fam[TE];
   int32_t s_short[TE][4], s_long[TE][4];
   int32_t q[TE][C][kRing];  // actuated per-channel samples of positions p-64..p-1, slot p & 63
   uint8_t ring[TE][kRing];  // level of each of those samples
@@ -51,9 +71,9 @@ __device__ __forceinline__ float actuator_scale(const EnvDev& env, int level, in
   return ((env.phase_mask >> ph) & 1) ? env.scale[level][c] : 1.0f;
 }
 
-__device__ __forceinline__ int32_t sample_q(const EnvDev& env, int c, int pos, int level) {
-  const float x = __ldg(env.trace + (int64_t)c * env.L + pos);
-  return quant64(x, actuator_scale(env, level, c, __ldg(env.phase + pos)));
+__device__ __forceinline__ int32_t sample_q(const EnvDev& env, const Fam& fm, int c, int pos, int level) {
+  const float x = __ldg(fm.trace + (int64_t)c * fm.L + pos);
+  return quant64(x, actuator_scale(env, level, c, __ldg(fm.phase + pos)));
 }
 
 // ---------------------------------------------------------------------------
@@ -74,6 +94,7 @@ struct TileAcc {
   __device__ int32_t& prev() { return s.prev[e]; }
   __device__ int32_t& b() { return s.b[e]; }
   __device__ int32_t& til() { return s.til[e]; }
+  __device__ int32_t& fam() { return s.fam[e]; }
   __device__ int32_t& ss(int c) { return s.s_short[e][c]; }
   __device__ int32_t& sl(int c) { return s.s_long[e][c]; }
   __device__ uint8_t level_at(int p) const { return s.ring[e][p & (kRing - 1)]; }
@@ -85,9 +106,10 @@ struct TileAcc {
 
 template <int C>
 struct RegAcc {
-  int32_t pos_, k_, level_, prev_, b_, til_;
+  int32_t pos_, k_, level_, prev_, b_, til_, fam_;
   int32_t ss_[C], sl_[C];
   uint8_t* ring;  // global [64]
+  __device__ int32_t& fam() { return fam_; }
   __device__ int32_t& pos() { return pos_; }
   __device__ int32_t& k() { return k_; }
   __device__ int32_t& level() { return level_; }
@@ -98,7 +120,9 @@ struct RegAcc {
   __device__ int32_t& sl(int c) { return sl_[c]; }
   __device__ uint8_t level_at(int p) const { return ring[p & (kRing - 1)]; }
   __device__ void set_level_at(int p, int l) { ring[p & (kRing - 1)] = (uint8_t)l; }
-  __device__ int32_t q_at(const EnvDev& env, int c, int p) const { return sample_q(env, c, p, level_at(p)); }
+  __device__ int32_t q_at(const EnvDev& env, int c, int p) const {
+    return sample_q(env, fam_of(env, fam_), c, p, level_at(p));
+  }
   __device__ void push(int, int, int32_t) {}
 };
 
@@ -110,7 +134,7 @@ __device__ void rebuild_history(const EnvDev& env, Acc& a) {
     int32_t ss = 0, sl = 0;
     for (int i = 1; i <= kWLong; ++i) {
       const int pp = p - i;
-      const int32_t q = sample_q(env, c, pp, a.level_at(pp));
+      const int32_t q = sample_q(env, fam_of(env, a.fam()), c, pp, a.level_at(pp));
       a.push(c, pp, q);
       sl += q;
       if (i <= kWShort) ss += q;
@@ -133,13 +157,16 @@ __device__ void env_reset_at(const EnvDev& env, Acc& a, int o) {
   rebuild_history<C>(env, a);
 }
 
-// new episode at a random offset (Sec. 4.1)
+// new episode at a random offset (Sec. 4.1); with several trace families,
+// word 1 of the draw picks the episode's family (Sec. 4.2 G2) and word 0
+// the offset inside that family's trace
 template <int C, class Acc>
 __device__ void env_reset(const EnvDev& env, Acc& a, uint32_t eg, uint32_t t, uint32_t it,
                           uint32_t purpose) {
-  const uint32_t u = draw32(env.seed, eg, t, it, purpose);
-  const uint32_t span = (uint32_t)(env.L - env.span - kWLong + 1);
-  env_reset_at<C>(env, a, kWLong + (int)__umulhi(u, span));
+  const u32x4 w = philox10(u32x4{eg, t, it, purpose}, (uint32_t)env.seed, (uint32_t)(env.seed >> 32));
+  a.fam() = env.F > 1 ? (int)__umulhi(w.y, (uint32_t)env.F) : 0;
+  const uint32_t span = (uint32_t)(fam_of(env, a.fam()).L - env.span - kWLong + 1);
+  env_reset_at<C>(env, a, kWLong + (int)__umulhi(w.x, span));
 }
 
 template <int C, class Acc>
@@ -162,11 +189,12 @@ __device__ __forceinline__ int32_t Qcl(const EnvDev& env, Acc& a, int i) {
 //   OCC32/OCC64: Eq. 5 eight-vector, then per-channel recent samples and means
 template <int C, int OBS, class Acc>
 __device__ __forceinline__ float feature(const EnvDev& env, Acc& a, int f) {
-  const int64_t B = env.budget_q;
+  const Fam fm = fam_of(env, a.fam());
+  const int64_t B = fm.B;
   if (OBS == PE_OBS_TINY8) {
     if (f < 5) return ratio_i(Qcl<C>(env, a, 4 - f), B);
     if (f == 5) return ratio_i(B - Qcl<C>(env, a, 0), B);
-    if (f == 6) return (float)__ldg(env.phase + a.pos() - 1);
+    if (f == 6) return (float)__ldg(fm.phase + a.pos() - 1);
     return ratio_i(a.level(), env.n_levels - 1);
   }
   int64_t S20 = 0, S60 = 0;
@@ -180,7 +208,7 @@ __device__ __forceinline__ float feature(const EnvDev& env, Acc& a, int f) {
     switch (f) {
       case 8: return ratio_i(S60, kWLong * B);
       case 9: return ratio_i(kWLong * B - S60, kWLong * B);
-      case 10: return (float)__ldg(env.phase + a.pos() - 1);
+      case 10: return (float)__ldg(fm.phase + a.pos() - 1);
       case 11: return ratio_i(a.level() - env.g_min, env.g_max - env.g_min);
       case 12: return ratio_i(a.b() - env.b_min, env.b_max - env.b_min);
       case 13: return ratio_i(S20, kWShort * B);
@@ -203,25 +231,25 @@ __device__ __forceinline__ float feature(const EnvDev& env, Acc& a, int f) {
   if (OBS == PE_OBS_OCC32) {
     if (f < 24) {
       const int c = (f - 8) >> 2, i = (f - 8) & 3;
-      return c < C ? ratio_i((int64_t)C * Qc<C>(env, a, c, 3 - i), B) : 0.0f;
+      return c < fm.C ? ratio_i((int64_t)fm.C * Qc<C>(env, a, c, 3 - i), B) : 0.0f;
     }
     if (f < 28) {
       const int c = f - 24;
-      return c < C ? ratio_i((int64_t)C * a.sl(c), kWLong * B) : 0.0f;
+      return c < fm.C ? ratio_i((int64_t)fm.C * a.sl(c), kWLong * B) : 0.0f;
     }
     return 0.0f;
   }
   // OCC64
   if (f < 56) {
     const int c = (f - 8) / 12, i = (f - 8) % 12;
-    return c < C ? ratio_i((int64_t)C * Qc<C>(env, a, c, 11 - i), B) : 0.0f;
+    return c < fm.C ? ratio_i((int64_t)fm.C * Qc<C>(env, a, c, 11 - i), B) : 0.0f;
   }
   if (f < 60) {
     const int c = f - 56;
-    return c < C ? ratio_i((int64_t)C * a.ss(c), kWShort * B) : 0.0f;
+    return c < fm.C ? ratio_i((int64_t)fm.C * a.ss(c), kWShort * B) : 0.0f;
   }
   const int c = f - 60;
-  return c < C ? ratio_i((int64_t)C * a.sl(c), kWLong * B) : 0.0f;
+  return c < fm.C ? ratio_i((int64_t)fm.C * a.sl(c), kWLong * B) : 0.0f;
 }
 
 struct StepOut {
@@ -248,7 +276,8 @@ __device__ __forceinline__ StepOut env_step(const EnvDev& env, Acc& a, int act, 
   // consume the step's samples (one, or a generation batch with a cadence
   // table): windows, violations and excess per sample; tokens and excess
   // summed; the Eq. 6 peak term is the batch's largest 30 s excess
-  const int64_t B60 = (int64_t)kWLong * env.budget_q;
+  const Fam fm = fam_of(env, a.fam());
+  const int64_t B60 = (int64_t)kWLong * fm.B;
   float rate = env.tokens[nl];
   if (env.act_kind == PE_ACT_INCDEC) rate = __fdiv_rn(rate * (float)a.b(), (float)env.b_init);
   StepOut o;
@@ -261,12 +290,12 @@ __device__ __forceinline__ StepOut env_step(const EnvDev& env, Acc& a, int act, 
   const int n = env.ns[nl];
   for (int i = 0; i < n; ++i) {
     const int p = a.pos();
-    const int ph = __ldg(env.phase + p);
+    const int ph = __ldg(fm.phase + p);
     int32_t Q = 0;
     int64_t S60 = 0;
 #pragma unroll
     for (int c = 0; c < C; ++c) {
-      const int32_t qin = quant64(__ldg(env.trace + (int64_t)c * env.L + p), actuator_scale(env, nl, c, ph));
+      const int32_t qin = quant64(__ldg(fm.trace + (int64_t)c * fm.L + p), actuator_scale(env, nl, c, ph));
       const int32_t q20 = a.q_at(env, c, p - kWShort);
       const int32_t q60 = a.q_at(env, c, p - kWLong);
       a.ss(c) += qin - q20;
@@ -276,7 +305,7 @@ __device__ __forceinline__ StepOut env_step(const EnvDev& env, Acc& a, int act, 
       S60 += a.sl(c);
     }
     a.set_level_at(p, nl);  // after the window updates: slot p & 63 held position p - 64
-    const int v1 = Q > env.budget_q, v60 = S60 > B60;
+    const int v1 = Q > fm.B, v60 = S60 > B60;
     const float exc_w = v60 ? __fdiv_rn(__ll2float_rn(S60 - B60), 3840.0f) : 0.0f;  // watts over B
     o.q += Q;
     o.v1 += v1;
@@ -309,6 +338,7 @@ __device__ void load_tile(const EnvDev& env, EnvTile<TE, C>& s, int e0, int ne) 
     s.prev[e] = env.st[kStPrev * env.E + g];
     s.b[e] = env.st[kStB * env.E + g];
     s.til[e] = env.st[kStTil * env.E + g];
+    s.fam[e] = env.st[kStFam * env.E + g];
     for (int i = 0; i < kRing; ++i) s.ring[e][i] = env.ring[(int64_t)g * kRing + i];
     TileAcc<TE, C> a{s, e};
     rebuild_history<C>(env, a);
@@ -325,6 +355,7 @@ __device__ void store_tile(const EnvDev& env, const EnvTile<TE, C>& s, int e0, i
     env.st[kStPrev * env.E + g] = s.prev[e];
     env.st[kStB * env.E + g] = s.b[e];
     env.st[kStTil * env.E + g] = s.til[e];
+    env.st[kStFam * env.E + g] = s.fam[e];
     for (int i = 0; i < kRing; ++i) env.ring[(int64_t)g * kRing + i] = s.ring[e][i];
     for (int c = 0; c < 4; ++c) {
       env.sums[(int64_t)g * 8 + c] = c < C ? s.s_short[e][c] : 0;
@@ -343,6 +374,7 @@ __device__ __forceinline__ RegAcc<C> load_reg(const EnvDev& env, int g) {
   a.prev_ = env.st[kStPrev * env.E + g];
   a.b_ = env.st[kStB * env.E + g];
   a.til_ = env.st[kStTil * env.E + g];
+  a.fam_ = env.st[kStFam * env.E + g];
   a.ring = env.ring + (int64_t)g * kRing;
 #pragma unroll
   for (int c = 0; c < C; ++c) {
@@ -360,6 +392,7 @@ __device__ __forceinline__ void store_reg(const EnvDev& env, int g, const RegAcc
   env.st[kStPrev * env.E + g] = a.prev_;
   env.st[kStB * env.E + g] = a.b_;
   env.st[kStTil * env.E + g] = a.til_;
+  env.st[kStFam * env.E + g] = a.fam_;
 #pragma unroll
   for (int c = 0; c < 4; ++c) {
     env.sums[(int64_t)g * 8 + c] = c < C ? a.ss_[c] : 0;

@@ -100,12 +100,14 @@ __global__ void env_offsets_kernel(EnvDev env, const int32_t* __restrict__ offse
   const int e = blockIdx.x * blockDim.x + threadIdx.x;
   if (e >= env.E) return;
   const int o = offsets[e];
-  if (o < kWLong || o > env.L - env.span) {
+  const int fam = env.st[kStFam * env.E + e];
+  if (o < kWLong || o > fam_of(env, fam).L - env.span) {
     atomicOr(flag, 1);
     return;
   }
   RegAcc<C> a;
   a.ring = env.ring + (int64_t)e * kRing;
+  a.fam() = fam;  // the env keeps its episode's trace family
   env_reset_at<C>(env, a, o);
   store_reg<C>(env, e, a);
 }

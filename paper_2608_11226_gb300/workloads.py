@@ -77,6 +77,12 @@ class EnvSpec:
     seed: int
     # batch-boundary cadence (Sec. 4.5): samples a step consumes at each level; None: one
     level_samples: Optional[List[int]] = None
+    # domain randomisation (Sec. 4.2 G2): trace families drawn per episode; the trace and
+    # phase arrays are then family-major concatenations ([f][n_channels][fam_len[f]])
+    n_families: int = 0
+    fam_len: Optional[List[int]] = None
+    fam_channels: Optional[List[int]] = None
+    fam_budget_q: Optional[List[int]] = None
 
     @property
     def obs_dim(self) -> int:
@@ -388,6 +394,39 @@ def make_72b_cadence(n_envs: int = 65536, seed: int = 0) -> Workload:
     wl.env.level_samples = [24 + (18 * l) // 15 for l in range(wl.env.n_levels)]
     wl.env.episode_len = 40
     return wl
+
+
+def make_72b_mixed(n_envs: int = 65536, seed: int = 0) -> Workload:
+    """Domain randomisation (Sec. 4.2, design G2): the 72B controller's env
+    drawing each episode from one of three trace families (a 4-GPU
+    72B-shaped trace, a 2-GPU 14B-shaped pair anti-correlated at -0.13 as in
+    Sec. 6.3, and a 1-GPU 7B-shaped trace), each with its own budget (its
+    mean cluster power at the default level / 0.888) so that the
+    cap-relative state of G2 transfers across scales."""
+    base = make_72b(n_envs=n_envs, seed=seed)
+    t72, p72 = base.trace, base.phase
+    ft, fj = fleet_traces(seed + 1, length=15000)
+    t14 = ft[fj == 2]                      # a 2-GPU 14B-shaped job of the fleet mix
+    p14 = np.zeros(t14.shape[1], np.uint8)
+    t7, p7 = trace_7b(seed + 2, length=20000)
+    scale = base.env.level_scale
+    fams = [(t72, p72), (t14, p14), (np.asarray(t7, np.float32).reshape(1, -1), p7)]
+    C = base.env.n_channels
+    traces, phases, lens, chans, budgets = [], [], [], [], []
+    for tr, ph in fams:
+        c, L = tr.shape
+        pad = np.zeros((C, L), np.float32)
+        pad[:c] = tr
+        traces.append(pad.ravel())
+        phases.append(np.asarray(ph, np.uint8))
+        lens.append(L)
+        chans.append(c)
+        mean_cluster = float(tr.astype(np.float64).sum(axis=0).mean()) * scale[7][0]
+        budgets.append(budget_q(mean_cluster / 0.888))
+    env = dataclasses.replace(base.env, n_families=3, fam_len=lens, fam_channels=chans, fam_budget_q=budgets,
+                              trace_len=lens[0], budget_q=budgets[0])
+    return Workload("72b_mixed", env, base.net, base.ppo, base.horizon, np.concatenate(traces),
+                    np.concatenate(phases))
 
 
 PRESETS = {"tiny": make_tiny, "7b": make_7b, "72b": make_72b, "stress": make_stress}

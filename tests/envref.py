@@ -19,8 +19,19 @@ def _f32ratio(num, den):
 
 class BruteEnv:
     def __init__(self, spec, trace, phase, env_id, philox):
-        self.s, self.trace, self.phase, self.e, self.philox = spec, trace, phase, env_id, philox
-        self.C, self.L = trace.shape
+        self.s, self.e, self.philox = spec, env_id, philox
+        # trace families (domain randomisation): family-major [f][n_channels][L_f] buffers;
+        # one family: the [C][L] trace itself
+        if getattr(spec, "n_families", 0) > 1:
+            self.fams, to, po = [], 0, 0
+            for L, c, B in zip(spec.fam_len, spec.fam_channels, spec.fam_budget_q):
+                tr = np.asarray(trace[to:to + spec.n_channels * L], np.float32).reshape(spec.n_channels, L)[:c]
+                self.fams.append((tr, phase[po:po + L], B))
+                to += spec.n_channels * L
+                po += L
+        else:
+            self.fams = [(trace, phase, spec.budget_q)]
+        self.use_family(0)
         self.reset(0, 0, 2)
 
     def scale(self, level, c):
@@ -34,10 +45,17 @@ class BruteEnv:
         sc = self.scale(level, c) if (self.s.scale_phase_mask >> int(self.phase[pos])) & 1 else np.float32(1.0)
         return int(np.rint(np.float32(np.float32(x * sc) * np.float32(64.0))))
 
+    def use_family(self, f):
+        self.fam = f
+        self.trace, self.phase, self.B = self.fams[f]
+        self.C, self.L = self.trace.shape
+
     def reset(self, t, it, purpose):
         s = self.s
         seed = s.seed
-        u = int(self.philox([self.e, t, it, purpose], [seed & 0xFFFFFFFF, seed >> 32])[0])
+        w = self.philox([self.e, t, it, purpose], [seed & 0xFFFFFFFF, seed >> 32])
+        u, v = int(w[0]), int(w[1])
+        self.use_family((v * len(self.fams)) >> 32 if len(self.fams) > 1 else 0)
         span = self.L - s.episode_len * self.nmax() - W_LONG + 1
         self.reset_at(W_LONG + ((u * span) >> 32))
 
@@ -68,7 +86,7 @@ class BruteEnv:
         return sum(v[c] for v in vals) if c is not None else sum(sum(v) for v in vals)
 
     def obs(self):
-        s, B, C = self.s, self.s.budget_q, self.C
+        s, B, C = self.s, self.B, self.C
         S20, S60, Q0 = self.S(W_SHORT), self.S(W_LONG), self.Q(0)
         ph = np.float32(self.phase[self.pos - 1])
         if s.obs_kind == 0:
@@ -115,7 +133,7 @@ class BruteEnv:
         return max(self.rate(l, s.b_init) for l in range(s.n_levels))
 
     def step(self, a, lam, t, it):
-        s, B = self.s, self.s.budget_q
+        s, B = self.s, self.B
         new = self.level
         if s.actuator_kind == ACT_INCDEC:
             if a == 1:

@@ -293,6 +293,36 @@ def test_rollout_parity_72b_cadence():
     _rollout_case(W.make_72b_cadence(n_envs=128), 30, iters=3, lam=0.7)
 
 
+def test_rollout_parity_72b_mixed_families():
+    """Domain randomisation (Sec. 4.2 G2): the 72B env drawing each episode
+    from a 4-GPU 72B-, a 2-GPU 14B- or a 1-GPU 7B-shaped trace family with
+    its own budget, on the tcgen05 path across episode boundaries."""
+    _rollout_case(W.make_72b_mixed(n_envs=128), 400, iters=3, lam=0.7)
+
+
+def test_rule_rollout_parity_mixed_families_with_offsets():
+    """Rule rollouts on the mixed env, before and after explicit episode
+    starts (which keep each env's family)."""
+    wl = W.make_72b_mixed(n_envs=64)
+    spec = wl.env
+    rule = W.threshold_rule(spec.budget_q)
+    env = pe.Env(spec, torch.from_numpy(wl.trace), torch.from_numpy(wl.phase))
+    oenv = O.OracleEnv(spec, wl.trace, wl.phase, range(64))
+    for it, T in ((0, 300), (1, 200)):
+        buf = pe.alloc_rule_rollout(spec, T)
+        pe.rollout_rule(env, rule, T, it, buf, lam=0.5)
+        torch.cuda.synchronize()
+        ref = oenv.rollout_rule(rule, T, it, lam=0.5)
+        for k in ("act", "done", "viol", "energy_q"):
+            assert np.array_equal(cpu(buf[k]), ref[k]), k
+        if it == 0:
+            offs = np.full(64, 100, np.int32)
+            pe.set_offsets(env, torch.from_numpy(offs).cuda())
+            oenv.set_offsets(offs)
+    assert np.array_equal(cpu(buf["energy_q"]), ref["energy_q"])
+    env.close()
+
+
 def test_rule_rollout_parity_72b_cadence():
     wl = W.make_72b_cadence(n_envs=64)
     spec = wl.env

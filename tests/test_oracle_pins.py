@@ -99,6 +99,24 @@ def test_env_72b_cadence_matches_bruteforce():
     _brute_compare(wl, 2, 45, iters=2)
 
 
+def test_env_mixed_families_matches_bruteforce():
+    """Domain randomisation (Sec. 4.2 G2): each episode draws its trace
+    family (4-GPU 72B-, 2-GPU 14B- or 1-GPU 7B-shaped, each with its own
+    budget) from word 1 of the episode draw and its offset from word 0; the
+    oracle's per-family view matches the brute-force env across episode
+    boundaries, and more than one family is visited."""
+    wl = W.make_72b_mixed(n_envs=4)
+    _brute_compare(wl, 4, 520, iters=2)
+    seen = set()
+    for e in range(4):
+        b = BruteEnv(wl.env, wl.trace, wl.phase, e, O.philox4x32_10)
+        seen.add(b.fam)
+        for t in range(3):
+            b.reset(t, 0, 1)
+            seen.add(b.fam)
+    assert len(seen) == 3
+
+
 def test_env_tiny_matches_bruteforce():
     _brute_compare(W.make_tiny(n_envs=3), 3, 620, iters=2)
 
