@@ -167,12 +167,21 @@ def barrier(world):
 
 
 def max_over_ranks(x: float, world: int) -> float:
+    """The slowest rank's time (replicas report the whole job's throughput
+    against it); NCCL reduces on the device, gloo on the host."""
     if world == 1:
         return x
     import torch.distributed as dist
-    t = torch.tensor([x], dtype=torch.float64, device="cuda")
+    dev = "cuda" if dist.get_backend() == "nccl" else "cpu"
+    t = torch.tensor([x], dtype=torch.float64, device=dev)
     dist.all_reduce(t, op=dist.ReduceOp.MAX)
     return float(t.item())
+
+
+def job_value(units_per_rank: float, world: int, max_ms: float) -> float:
+    """Whole-job throughput of weak-scaled replicas: every rank's units over
+    the slowest rank's time."""
+    return units_per_rank * world / (max_ms / 1e3)
 
 
 # --------------------------------------------------------------------------- our path
@@ -250,7 +259,7 @@ def run_ours(args, world, rank, local):
     total_ms = max_over_ranks(total_ms, world)
     ms_step = total_ms / args.steps
     env_steps = tr.E * tr.T
-    value = env_steps * world * args.steps / (total_ms / 1e3)
+    value = job_value(env_steps * args.steps, world, total_ms)
     launches = sum(n for _, n in prof.values())
     # ---- dominant kernel roofline (fp32 FFMA bound)
     gms, gn = prof["ppo_grad"]
