@@ -318,7 +318,7 @@ def run_ours(args, world, rank, local):
            "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h}
 
     # ---- fleet accounting
-    fleet = run_fleet(args, world) if args.fleet_n > 0 else None
+    fleet = run_fleet(args, world, tr) if args.fleet_n > 0 else None
     evaluation = run_evaluation(args, world, tr, peaks) if args.eval else None
     r72b = run_72b(args, world, peaks) if args.r72b_steps > 0 else None
     gae_large = run_gae_large(args, world, peaks) if args.gae_large[0] > 0 else None
@@ -415,7 +415,7 @@ def run_evaluation(args, world, tr, peaks):
                                               "note": "6 B of buffer writes per env-step; latency-bound"}}}
 
 
-def run_fleet(args, world):
+def run_fleet(args, world, tr=None):
     from paper_2608_11226_gb300 import pe
     from paper_2608_11226_gb300 import workloads as W
     fw = W.make_fleet(n_compositions=args.fleet_n)
@@ -452,7 +452,7 @@ def run_fleet(args, world):
     composed = N * H
     c = counts.cpu().numpy()
     p = peaks.cpu().numpy()
-    stagger = run_stagger(args, world, fw, traces, job, p) if args.stagger_stride > 0 else None
+    stagger = run_stagger(args, world, fw, traces, job, p, tr) if args.stagger_stride > 0 else None
     return {"metric": "fleet window-samples/s", "value": ws_per_call * world * args.fleet_steps / (ms / 1e3),
             "unit": "window-samples/s", "ms_per_call": ms / args.fleet_steps,
             "config": {"workload": "fleet: 16 traces x 380,000 samples (2x72B@4, 2x14B@2, 4x7B@1), "
@@ -468,7 +468,42 @@ def run_fleet(args, world):
             "strategies": stagger}
 
 
-def run_stagger(args, world, fw, traces, job, peaks_random):
+def controlled_7b_traces(fw, tr):
+    """Sec. 8 "job control": each single-GPU 7B job of the fleet replayed
+    through the 7B env under the bench's trained controller, deterministic,
+    in consecutive 500-step episodes (Sec. 4.4 replay); its actuated power
+    (1/64 W, exact as watts) replaces the raw trace.  The controller's budget
+    for a job keeps the 7B study's ratio of budget to full-timeline mean
+    power (314.6 / 314.9 W, Sec. 6.1)."""
+    import dataclasses
+    from paper_2608_11226_gb300 import pe
+    from paper_2608_11226_gb300 import workloads as W
+    base = W.make_7b(seed=tr.seed)
+    L = fw.traces.shape[1]
+    T = base.env.episode_len
+    offs = W.replay_offsets(L, T)
+    out = fw.traces.copy()
+    jobs7 = [j for j, (kind, gpus) in enumerate(W.FLEET_JOBS) if kind == "7B" and gpus == 1]
+    for j in jobs7:
+        g = int(np.nonzero(fw.job_of_gpu == j)[0][0])
+        x = fw.traces[g]
+        spec = dataclasses.replace(base.env, n_envs=len(offs), trace_len=L,
+                                   budget_q=W.budget_q(float(x.astype(np.float64).mean()) * 314.6 / 314.9))
+        env = pe.Env(spec, torch.from_numpy(np.ascontiguousarray(x.reshape(1, L))),
+                     torch.zeros(L, dtype=torch.uint8))
+        pe.set_offsets(env, torch.from_numpy(offs).cuda())
+        buf = pe.alloc_rollout(spec, base.net, T)
+        pe.rollout(env, base.net, tr.params, T, 0, buf, deterministic=True)
+        q = buf["q"].cpu().numpy()
+        series = x.copy()
+        for k, o in enumerate(offs):
+            series[o:o + T] = q[:, k].astype(np.float32) / np.float32(64.0)
+        out[g] = series
+        env.close()
+    return out
+
+
+def run_stagger(args, world, fw, traces, job, peaks_random, tr=None):
     """Sec. 8 fleet operating strategies on the same traces: naive aligned
     starts (composition 0), random starts (the other compositions) and the
     greedy phase-staggered schedule (pe_fleet_stagger over every
@@ -498,15 +533,24 @@ def run_stagger(args, world, fw, traces, job, peaks_random):
     name = W.FLEET_NAMEPLATE_W / 1e3
     rnd = peaks_random[1:, 1] if peaks_random.shape[0] > 1 else peaks_random[:, 1]
     stag = kw(pk[-1].item())
+    ctl = None
+    if tr is not None:  # staggering combined with job-level control of the 7B jobs
+        ctl_traces = torch.from_numpy(controlled_7b_traces(fw, tr)).cuda()
+        pk2 = torch.empty_like(pk)
+        off2 = torch.empty_like(off)
+        pe.fleet_stagger(ctl_traces, job, J, H, w, st, off2, pk2, ws)
+        ctl = kw(pk2[-1].item())
     return {"metric": "staggered-schedule candidate window-samples/s",
             "value": cand_ws * world / (ms / 1e3), "unit": "window-samples/s", "ms_per_call": ms,
             "config": {"stride": st, "window": w, "candidates_per_job": ncand, "jobs": J},
             "offsets": [int(x) for x in off.cpu()],
             "peak_30s_kw": {"naive_aligned": kw(peaks_random[0, 1]), "random_median": kw(np.median(rnd)),
-                            "random_max": kw(rnd.max()), "phase_staggered": stag},
+                            "random_max": kw(rnd.max()), "phase_staggered": stag,
+                            "staggered_with_job_control": ctl},
             "provisioning_fraction": {"naive_aligned": kw(peaks_random[0, 1]) / name,
                                       "random_median": kw(np.median(rnd)) / name,
-                                      "phase_staggered": stag / name}}
+                                      "phase_staggered": stag / name,
+                                      "staggered_with_job_control": ctl / name if ctl else None}}
 
 
 def run_72b(args, world, peaks):

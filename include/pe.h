@@ -151,6 +151,8 @@ typedef struct pe_rollout_buf {
   int64_t* samples;   /* [E]    trace samples consumed this call (optional, NULL skips); with a
                        *        cadence table the violation counts are per sample, so rates
                        *        divide by this count */
+  int32_t* q;         /* [T][E] actuated cluster power of step t, 1/64 W (summed over the
+                       *        batch's samples with a cadence table); optional, NULL skips */
 } pe_rollout_buf;
 
 /* PPO configuration (Sec. 4.2 / 4.5; SB3 defaults where the paper is silent) */

@@ -75,11 +75,11 @@ def lib():
             "or_env_init": (i32, [vp, vp, vp, vp, i32, vp]),
             "or_env_set_offsets": (i32, [vp, vp, vp, vp, i32, vp]),
             "or_rollout_rule": (i32, [vp, vp, vp, vp, vp, i32, vp, i32, u32, f64, vp, vp, vp, vp,
-                                      vp, vp, vp, vp]),
+                                      vp, vp, vp, vp, vp]),
             "or_env_obs": (None, [vp, vp, vp, vp, vp]),
             "or_mlp_forward": (None, [i32, i32, i32, i32, vp, i64, vp, vp, vp]),
             "or_rollout": (i32, [vp, vp, vp, vp, i32, i32, vp, i32, vp, i32, u32, f64, i32,
-                                 vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp]),
+                                 vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp]),
             "or_gae": (None, [i32, i32, vp, vp, vp, vp, f64, f64, vp, vp]),
             "or_ppo_minibatch_grad": (f64, [i32, i32, i32, vp, i64, vp, vp, vp, vp, vp,
                                             f64, f64, f64, vp, vp]),
@@ -203,14 +203,14 @@ class OracleEnv:
             reward=np.zeros((T, n), np.float64), done=np.zeros((T, n), np.uint8),
             viol=np.zeros((n, 2), np.int32), tokens=np.zeros(n, np.float64),
             excess=np.zeros(n, np.float64), energy_q=np.zeros(n, np.int64),
-            samples=np.zeros(n, np.int64))
+            samples=np.zeros(n, np.int64), q=np.zeros((T, n), np.int32))
         f = None if forced is None else np.ascontiguousarray(forced, np.uint8)
         lib().or_rollout(C.byref(self.cfg), _p(self.trace), _p(self.phase), _p(params), hidden,
                          int(bf16), _p(self.env_ids), n, _p(self.state), T, iteration, lam,
                          int(deterministic), _p(f), _p(out["obs"]), _p(out["obs_last"]),
                          _p(out["act_own"]), _p(out["logp"]), _p(out["reward"]), _p(out["done"]),
                          _p(out["viol"]), _p(out["tokens"]), _p(out["excess"]),
-                         _p(out["energy_q"]), _p(out["samples"]))
+                         _p(out["energy_q"]), _p(out["samples"]), _p(out["q"]))
         return out
 
 
@@ -227,13 +227,14 @@ class OracleEnv:
         out = dict(act=np.zeros((T, n), np.uint8), reward=np.zeros((T, n), np.float64),
                    done=np.zeros((T, n), np.uint8), viol=np.zeros((n, 2), np.int32),
                    tokens=np.zeros(n, np.float64), excess=np.zeros(n, np.float64),
-                   energy_q=np.zeros(n, np.int64), samples=np.zeros(n, np.int64))
+                   energy_q=np.zeros(n, np.int64), samples=np.zeros(n, np.int64),
+                   q=np.zeros((T, n), np.int32))
         r = or_rule(rule)
         if lib().or_rollout_rule(C.byref(self.cfg), _p(self.trace), _p(self.phase), C.byref(r),
                                  _p(self.env_ids), n, _p(self.state), T, iteration, lam,
                                  _p(out["act"]), _p(out["reward"]), _p(out["done"]), _p(out["viol"]),
                                  _p(out["tokens"]), _p(out["excess"]), _p(out["energy_q"]),
-                                 _p(out["samples"])) != 0:
+                                 _p(out["samples"]), _p(out["q"])) != 0:
             raise ValueError("oracle rejected the rule")
         return out
 

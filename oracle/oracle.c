@@ -564,7 +564,7 @@ int32_t or_rollout(const or_env_cfg* cfg, const float* trace, const uint8_t* pha
                    double lambda, int32_t deterministic, const uint8_t* forced, float* obs,
                    float* obs_last, uint8_t* act_own, double* logp_taken, double* reward,
                    uint8_t* done, int32_t* viol, double* tokens, double* excess,
-                   int64_t* energy_q, int64_t* samples) {
+                   int64_t* energy_q, int64_t* samples, int32_t* qout) {
   const int32_t D = cfg->obs_kind == OR_OBS_TINY8   ? 8
                     : cfg->obs_kind == OR_OBS_7B16  ? 16
                     : cfg->obs_kind == OR_OBS_OCC32 ? 32
@@ -617,6 +617,7 @@ int32_t or_rollout(const or_env_cfg* cfg, const float* trace, const uint8_t* pha
       or_step_out so = env_step(&cf, tr, ph, st, a, lambda);
       reward[row] = so.reward;
       done[row] = (uint8_t)so.done;
+      if (qout) qout[row] = (int32_t)so.q;
       v1 += so.v1;
       v60 += so.v60;
       tok += so.tokens;
@@ -680,7 +681,8 @@ int32_t or_rollout_rule(const or_env_cfg* cfg, const float* trace, const uint8_t
                         const or_rule* rule, const int32_t* env_ids, int32_t n,
                         or_env_state* states, int32_t T, uint32_t iteration, double lambda,
                         uint8_t* act, double* reward, uint8_t* done, int32_t* viol,
-                        double* tokens, double* excess, int64_t* energy_q, int64_t* samples) {
+                        double* tokens, double* excess, int64_t* energy_q, int64_t* samples,
+                        int32_t* qout) {
   if (rule->kind < OR_RULE_RANDOM || rule->kind > OR_RULE_HYSTERESIS) return 1;
   for (int32_t i = 0; i < n; ++i) {
     or_env_state* st = &states[i];
@@ -699,6 +701,7 @@ int32_t or_rollout_rule(const or_env_cfg* cfg, const float* trace, const uint8_t
       or_step_out so = env_step(&cf, tr, ph, st, a, lambda);
       reward[row] = so.reward;
       done[row] = (uint8_t)so.done;
+      if (qout) qout[row] = (int32_t)so.q;
       v1 += so.v1;
       v60 += so.v60;
       tok += so.tokens;

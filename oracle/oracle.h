@@ -104,14 +104,16 @@ int32_t or_rollout(const or_env_cfg* cfg, const float* trace, const uint8_t* pha
                    int32_t T, uint32_t iteration, double lambda, int32_t deterministic,
                    const uint8_t* forced, float* obs, float* obs_last, uint8_t* act_own,
                    double* logp_taken, double* reward, uint8_t* done, int32_t* viol,
-                   double* tokens, double* excess, int64_t* energy_q, int64_t* samples);
+                   double* tokens, double* excess, int64_t* energy_q, int64_t* samples,
+                   int32_t* qout);
 int32_t or_env_set_offsets(const or_env_cfg* cfg, const float* trace, const uint8_t* phase,
                            const int32_t* offsets, int32_t n, or_env_state* states);
 int32_t or_rollout_rule(const or_env_cfg* cfg, const float* trace, const uint8_t* phase,
                         const or_rule* rule, const int32_t* env_ids, int32_t n,
                         or_env_state* states, int32_t T, uint32_t iteration, double lambda,
                         uint8_t* act, double* reward, uint8_t* done, int32_t* viol,
-                        double* tokens, double* excess, int64_t* energy_q, int64_t* samples);
+                        double* tokens, double* excess, int64_t* energy_q, int64_t* samples,
+                        int32_t* qout);
 double or_dual_ascent(const int32_t* viol, int32_t E, int64_t steps, int32_t window, int32_t additive,
                       double lambda, double target, double eta, double lo, double hi, double* rate);
 void or_gae(int32_t T, int32_t E, const float* r, const float* v, const uint8_t* done,

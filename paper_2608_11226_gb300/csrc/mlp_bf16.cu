@@ -612,6 +612,7 @@ __global__ void __launch_bounds__(128) env_actobs_kernel(EnvDev env, ActArgs a, 
     buf.logp[row] = lp;
     buf.reward[row] = so.reward;
     buf.done[row] = (uint8_t)so.done;
+    if (buf.q) buf.q[row] = so.q;
     if (a.t == 0) {
       buf.viol[2 * e] = so.v1;
       buf.viol[2 * e + 1] = so.v60;

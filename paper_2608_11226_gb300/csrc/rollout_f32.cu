@@ -81,6 +81,7 @@ __global__ void __launch_bounds__(TE / 4 * H / 4)
       buf.logp[row] = lp;
       buf.reward[row] = so.reward;
       buf.done[row] = (uint8_t)so.done;
+      if (buf.q) buf.q[row] = so.q;
       v1 += so.v1;
       v60 += so.v60;
       energy += so.q;

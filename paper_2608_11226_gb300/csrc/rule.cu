@@ -75,6 +75,7 @@ __global__ void __launch_bounds__(128) rule_rollout_kernel(EnvDev env, RuleArgs 
     buf.act[row] = (uint8_t)act;
     buf.reward[row] = so.reward;
     buf.done[row] = (uint8_t)so.done;
+    if (buf.q) buf.q[row] = so.q;
     v1 += so.v1;
     v60 += so.v60;
     tok += so.tokens;

@@ -55,7 +55,7 @@ class Net(C.Structure):
 
 
 ROLLOUT_FIELDS = ("obs", "obs_last", "act", "logp", "value", "last_value", "reward", "done", "viol",
-                  "tokens", "excess", "energy_q", "samples")
+                  "tokens", "excess", "energy_q", "samples", "q")
 
 
 class RolloutBuf(C.Structure):
@@ -225,7 +225,7 @@ def alloc_rollout(spec: W.EnvSpec, net: W.NetSpec, T: int, device="cuda") -> Dic
         reward=torch.empty((T, E), **kw), done=torch.empty((T, E), dtype=torch.uint8, **kw),
         viol=torch.empty((E, 2), dtype=torch.int32, **kw), tokens=torch.empty(E, **kw),
         excess=torch.empty(E, **kw), energy_q=torch.empty(E, dtype=torch.int64, **kw),
-        samples=torch.empty(E, dtype=torch.int64, **kw))
+        samples=torch.empty(E, dtype=torch.int64, **kw), q=torch.empty((T, E), dtype=torch.int32, **kw))
 
 
 def _rollout_buf(b: Dict[str, Optional[torch.Tensor]]) -> RolloutBuf:
@@ -270,7 +270,7 @@ def alloc_rule_rollout(spec: W.EnvSpec, T: int, obs: bool = False, obs_bf16: boo
         reward=torch.empty((T, E), **kw), done=torch.empty((T, E), dtype=torch.uint8, **kw),
         viol=torch.empty((E, 2), dtype=torch.int32, **kw), tokens=torch.empty(E, **kw),
         excess=torch.empty(E, **kw), energy_q=torch.empty(E, dtype=torch.int64, **kw),
-        samples=torch.empty(E, dtype=torch.int64, **kw))
+        samples=torch.empty(E, dtype=torch.int64, **kw), q=torch.empty((T, E), dtype=torch.int32, **kw))
 
 
 def rollout_rule(env: Env, rule: W.RuleSpec, T: int, iteration: int, buf: Dict[str, torch.Tensor],

@@ -245,7 +245,7 @@ def _rollout_case(wl, T, iters, sample_envs=None, det=False, lam=1.0):
         pe.device_check()
         g = {}
         for k, v in buf.items():
-            sel = v[:, ids_d] if v.dim() >= 2 and k in ("obs", "act", "logp", "value", "reward", "done") else v[ids_d]
+            sel = v[:, ids_d] if v.dim() >= 2 and k in ("obs", "act", "logp", "value", "reward", "done", "q") else v[ids_d]
             g[k] = cpu(sel.float() if sel.dtype == torch.bfloat16 else sel)
         forced = g["act"]
         o = ora.rollout(params, net.hidden, bf16, T, it, lam=lam, deterministic=det, forced=forced)
@@ -259,6 +259,7 @@ def _rollout_case(wl, T, iters, sample_envs=None, det=False, lam=1.0):
         assert np.array_equal(g["viol"], o["viol"])
         assert np.array_equal(g["energy_q"], o["energy_q"])
         assert np.array_equal(g["samples"], o["samples"])
+        assert np.array_equal(g["q"], o["q"])
         assert rel_err(g["reward"], o["reward"]) <= TOL
         assert rel_err(g["tokens"], o["tokens"]) <= TOL
         assert rel_err(g["excess"], o["excess"]) <= TOL
@@ -334,7 +335,7 @@ def test_rule_rollout_parity_72b_cadence():
         pe.rollout_rule(env, rule, T, it, buf, lam=0.5)
         torch.cuda.synchronize()
         ref = oenv.rollout_rule(rule, T, it, lam=0.5)
-        for k in ("act", "done", "viol", "energy_q", "samples"):
+        for k in ("act", "done", "viol", "energy_q", "samples", "q"):
             assert np.array_equal(cpu(buf[k]), ref[k]), k
         assert rel_err(cpu(buf["reward"]), ref["reward"]) <= TOL
     env.close()

@@ -79,7 +79,7 @@ def _brute_compare(wl, n_envs, T, iters=1, seed_actions=0):
                 o = b.obs()
                 assert np.array_equal(out["obs"][t, i], o), (it, t, i)
                 st = b.step(int(forced[t, i]), 0.7, t, it)
-                assert out["done"][t, i] == st["done"]
+                assert out["done"][t, i] == st["done"] and out["q"][t, i] == st["q"]
                 assert abs(out["reward"][t, i] - st["r"]) <= 1e-12 * max(1.0, abs(st["r"]))
                 v1 += st["v1"]; v60 += st["v60"]; en += st["q"]; smp += st["samples"]
                 tok += st["tokens"]; exc += st["excess"]
