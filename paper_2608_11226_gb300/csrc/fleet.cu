@@ -243,6 +243,86 @@ __global__ void __launch_bounds__(32 * kFleetWarps)
   }
 }
 
+// The same walk for fleets of at most 8 jobs: the J stream pointers live
+// in registers (no shared-memory pointer reloads), and each iteration
+// issues the loads of two 32-sample blocks before using either.
+constexpr int kFleetJMax = 8;
+
+template <int NW>
+__global__ void __launch_bounds__(32 * kFleetWarps)
+    fleet_windows_j8_kernel(const uint32_t* __restrict__ prex, int J, int64_t Lp,
+                            const int32_t* __restrict__ offsets, int64_t N, int H, FleetWindows win,
+                            int32_t* __restrict__ counts, int32_t* __restrict__ peaks) {
+  __shared__ uint32_t ring_all[kFleetWarps][kFleetRing];
+  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+  const int64_t n = (int64_t)blockIdx.x * kFleetWarps + wid;
+  if (n >= N) return;  // the whole warp leaves together; no block-wide barrier follows
+  uint32_t* ring = ring_all[wid];
+  // every lane holds all J stream bases (t = 0 at index 1 + o_j); lane j also
+  // loads pre(-1)'s term PREX[j][o_j]
+  const uint32_t* bp[kFleetJMax];
+  uint32_t pre_m1 = 0;
+#pragma unroll
+  for (int j = 0; j < kFleetJMax; ++j) {
+    bp[j] = prex;
+    if (j < J) {
+      const int32_t o = __ldg(offsets + n * J + j);
+      bp[j] = prex + (int64_t)j * Lp + o + 1;
+      if (lane == j) pre_m1 = __ldg(bp[j] - 1);
+    }
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) pre_m1 += __shfl_xor_sync(0xffffffffu, pre_m1, o);
+  if (lane == 0) ring[kFleetRing - 1] = pre_m1;
+  __syncwarp();
+  int32_t cnt[NW], pk[NW];
+#pragma unroll
+  for (int k = 0; k < NW; ++k) cnt[k] = pk[k] = 0;
+  for (int t0 = 0; t0 < H; t0 += 64) {
+    const int ta = t0 + lane, tb = t0 + 32 + lane;
+    uint32_t pa = 0, pb = 0;
+#pragma unroll
+    for (int j = 0; j < kFleetJMax; ++j) {
+      if (j < J) {
+        if (ta < H) pa += __ldg(bp[j] + ta);
+        if (tb < H) pb += __ldg(bp[j] + tb);
+      }
+    }
+#pragma unroll
+    for (int half = 0; half < 2; ++half) {
+      const int t = half ? tb : ta;
+      const uint32_t pre = half ? pb : pa;
+      ring[t & (kFleetRing - 1)] = pre;
+      __syncwarp();
+      if (t < H) {
+#pragma unroll
+        for (int k = 0; k < NW; ++k) {
+          const int w = win.w[k];
+          if (t >= w - 1) {
+            const int32_t S = (int32_t)(pre - ring[(t - w) & (kFleetRing - 1)]);
+            cnt[k] += S > win.bw[k];
+            pk[k] = max(pk[k], S);
+          }
+        }
+      }
+      __syncwarp();
+    }
+  }
+#pragma unroll
+  for (int k = 0; k < NW; ++k) {
+    int32_t c = cnt[k], p = pk[k];
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      c += __shfl_xor_sync(0xffffffffu, c, o);
+      p = max(p, __shfl_xor_sync(0xffffffffu, p, o));
+    }
+    if (lane == 0) {
+      counts[n * NW + k] = c;
+      peaks[n * NW + k] = p;
+    }
+  }
+}
+
 static int64_t fleet_lp(int L, int H) { return (((int64_t)L + H + 1) + 3) / 4 * 4; }
 static int fleet_nchunk(int L, int H) { return (int)((((int64_t)L + H) + kFleetChunk - 1) / kFleetChunk); }
 
@@ -311,11 +391,20 @@ pe_status fleet_launch(const float* traces, int G, int L, const int32_t* job_of_
   const int grid_n = (int)((N + kFleetWarps - 1) / kFleetWarps);
   const int64_t Lx = ws.Lp;
   ProfScope ps(PE_PROF_FLEET_WINDOWS, st);
-  switch (W) {
-    case 1: fleet_windows_kernel<1><<<grid_n, 32 * kFleetWarps, 0, st>>>(ws.prex, J, Lx, offsets, N, H, win, counts, peaks); break;
-    case 2: fleet_windows_kernel<2><<<grid_n, 32 * kFleetWarps, 0, st>>>(ws.prex, J, Lx, offsets, N, H, win, counts, peaks); break;
-    case 3: fleet_windows_kernel<3><<<grid_n, 32 * kFleetWarps, 0, st>>>(ws.prex, J, Lx, offsets, N, H, win, counts, peaks); break;
-    default: fleet_windows_kernel<4><<<grid_n, 32 * kFleetWarps, 0, st>>>(ws.prex, J, Lx, offsets, N, H, win, counts, peaks); break;
+  if (J <= kFleetJMax) {
+    switch (W) {
+      case 1: fleet_windows_j8_kernel<1><<<grid_n, 32 * kFleetWarps, 0, st>>>(ws.prex, J, Lx, offsets, N, H, win, counts, peaks); break;
+      case 2: fleet_windows_j8_kernel<2><<<grid_n, 32 * kFleetWarps, 0, st>>>(ws.prex, J, Lx, offsets, N, H, win, counts, peaks); break;
+      case 3: fleet_windows_j8_kernel<3><<<grid_n, 32 * kFleetWarps, 0, st>>>(ws.prex, J, Lx, offsets, N, H, win, counts, peaks); break;
+      default: fleet_windows_j8_kernel<4><<<grid_n, 32 * kFleetWarps, 0, st>>>(ws.prex, J, Lx, offsets, N, H, win, counts, peaks); break;
+    }
+  } else {
+    switch (W) {
+      case 1: fleet_windows_kernel<1><<<grid_n, 32 * kFleetWarps, 0, st>>>(ws.prex, J, Lx, offsets, N, H, win, counts, peaks); break;
+      case 2: fleet_windows_kernel<2><<<grid_n, 32 * kFleetWarps, 0, st>>>(ws.prex, J, Lx, offsets, N, H, win, counts, peaks); break;
+      case 3: fleet_windows_kernel<3><<<grid_n, 32 * kFleetWarps, 0, st>>>(ws.prex, J, Lx, offsets, N, H, win, counts, peaks); break;
+      default: fleet_windows_kernel<4><<<grid_n, 32 * kFleetWarps, 0, st>>>(ws.prex, J, Lx, offsets, N, H, win, counts, peaks); break;
+    }
   }
   PE_CHECK_LAUNCH("fleet_windows_kernel");
   return PE_OK;
@@ -412,7 +501,10 @@ pe_status fleet_stagger_launch(const float* traces, int G, int L, const int32_t*
     }
     {
       ProfScope ps(PE_PROF_FLEET_WINDOWS, st);
-      fleet_windows_kernel<1><<<grid_n, 32 * kFleetWarps, 0, st>>>(ws.prex, j + 1, ws.Lp, cand, nc, H, win, cnt, pk);
+      if (j + 1 <= kFleetJMax)
+        fleet_windows_j8_kernel<1><<<grid_n, 32 * kFleetWarps, 0, st>>>(ws.prex, j + 1, ws.Lp, cand, nc, H, win, cnt, pk);
+      else
+        fleet_windows_kernel<1><<<grid_n, 32 * kFleetWarps, 0, st>>>(ws.prex, j + 1, ws.Lp, cand, nc, H, win, cnt, pk);
     }
     {
       ProfScope ps(PE_PROF_FLEET_PREP, st);
