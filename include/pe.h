@@ -313,7 +313,11 @@ pe_status pe_ppo_update(const pe_net* net, float* params, float* adam_m, float* 
  *  traces: [G][L] fp32 watts; job_of_gpu: [G] in [0, J); offsets: [N][J] in [0, L)
  *  (all device memory); windows: [W] HOST array, W in [1, 4], each w in [1, 992];
  *  counts, peaks: [N][W] int32 (device).
- *  workspace: >= pe_fleet_workspace_bytes(J, L, H) bytes.
+ *  workspace: pe_fleet_workspace_bytes(J, L, H) bytes.  For J <= 8 that size
+ *  holds four copies of the per-job prefix sums, each shifted by one sample,
+ *  so that the counts use 16-byte loads; a smaller workspace, down to the one
+ *  copy of J * (L + H + 128) words plus 1 KiB, gives the same results through
+ *  4-byte loads.
  * The call validates the traces on the device and waits for that check
  * (one small device-to-host read on `stream`) before launching the counts.
  * Errors: PE_EINVAL (sizes, pointers, job map or offsets out of range),
@@ -353,9 +357,10 @@ pe_status pe_fleet_stagger(const float* traces, int32_t G, int32_t L, const int3
  * The paper has no counterpart: this is a deployment convenience.
  * Same arguments and results as pe_fleet_windows without the workspace: the
  * scratch is one file-scope device array of PE_FLEET_NOALLOC_SCRATCH_BYTES
- * (4 MiB, held by every GPU that loads the library until exit).  Requests
- * needing more (pe_fleet_workspace_bytes(J, L, H), about J * (L + H) * 4
- * bytes) return PE_EINVAL with that limit in the message, before any launch.  The call allocates nothing (no
+ * (4 MiB, held by every GPU that loads the library until exit); the 16-byte
+ * path runs when its four prefix copies fit.  Requests whose single copy
+ * (about J * (L + H + 128) * 4 bytes) does not fit return PE_EINVAL with
+ * that limit in the message, before any launch.  The call allocates nothing (no
  * cudaMalloc, no allocating library routine).  Its first call on a device
  * looks up the array's device address (cudaGetSymbolAddress) with that
  * device current; make that first call before any stream capture.  All

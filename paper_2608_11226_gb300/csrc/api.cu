@@ -89,6 +89,7 @@ pe_status ppo_update_bf16(const pe_net& net, float* params, float* m, float* v, 
                           const float* ret, int64_t N, const pe_ppo_config& cfg, float* stats, void* ws,
                           cudaStream_t st);
 int64_t fleet_ws_bytes(int J, int L, int H);
+int64_t fleet_ws_min_bytes(int J, int L, int H);
 struct RuleArgs {
   int32_t kind, hi_q, lo_q, drop30_q, climb30_q, climb10_q;
   int32_t T, obs_bf16;
@@ -113,7 +114,7 @@ pe_status device_check(cudaStream_t st);
 pe_status fleet_launch(const float* traces, int G, int L, const int32_t* job_of_gpu, int J,
                        const int32_t* offsets, int64_t N, int H, const int32_t* windows, int W,
                        int64_t budget_q, int32_t* counts, int32_t* peaks, void* workspace,
-                       cudaStream_t st);
+                       int64_t workspace_bytes, cudaStream_t st);
 
 static int obs_width(int kind) {
   switch (kind) {
@@ -619,9 +620,9 @@ pe_status pe_fleet_windows(const float* traces, int32_t G, int32_t L, const int3
   if (budget_q < 0) return fail(PE_EINVAL, "budget_q must be >= 0");
   if (!traces || !job_of_gpu || !workspace || (N > 0 && (!offsets || !counts || !peaks)))
     return fail(PE_EINVAL, "null argument");
-  if (workspace_bytes < fleet_ws_bytes(J, L, H)) return fail(PE_EINVAL, "workspace too small");
+  if (workspace_bytes < fleet_ws_min_bytes(J, L, H)) return fail(PE_EINVAL, "workspace too small");
   return fleet_launch(traces, G, L, job_of_gpu, J, offsets, N, H, windows, W, budget_q, counts,
-                      peaks, workspace, reinterpret_cast<cudaStream_t>(stream));
+                      peaks, workspace, workspace_bytes, reinterpret_cast<cudaStream_t>(stream));
 }
 
 int64_t pe_fleet_stagger_workspace_bytes(int32_t J, int32_t L, int32_t H, int32_t stride) {

@@ -323,24 +323,147 @@ __global__ void __launch_bounds__(32 * kFleetWarps)
   }
 }
 
-static int64_t fleet_lp(int L, int H) { return (((int64_t)L + H + 1) + 3) / 4 * 4; }
+// Fleets of at most 8 jobs with 16-byte loads.  The workspace holds four
+// copies of the prefix array, copy c shifted left by c samples
+// (X_c[j][x] = PREX[j][x + c], zero past the end), so that for any offset the
+// stream of job j starts 16-byte aligned in copy (o_j + 1) & 3.  Each lane
+// composes 4 consecutive samples per load; one warp iteration covers 128.
+// The 1024-slot ring keeps its size: windows of 128 samples or more read it
+// before the block's prefixes are written (their starts all precede the
+// block), shorter windows after (their starts lie at most 127 back).
+template <bool EDGE, int NW>
+__device__ __forceinline__ void fleet_block4(const uint32_t* ring, int T, int H, const uint4& pre,
+                                             const FleetWindows& win, bool long_windows,
+                                             int32_t (&cnt)[NW], int32_t (&pk)[NW]) {
+  const uint32_t pv[4] = {pre.x, pre.y, pre.z, pre.w};
+#pragma unroll
+  for (int k = 0; k < NW; ++k) {
+    const int w = win.w[k];
+    if ((w >= 128) != long_windows) continue;
+    uint32_t old[4];
+    if ((w & 3) == 0) {
+      const uint4 o4 = *reinterpret_cast<const uint4*>(ring + ((T - w) & (kFleetRing - 1)));
+      old[0] = o4.x; old[1] = o4.y; old[2] = o4.z; old[3] = o4.w;
+    } else {
+#pragma unroll
+      for (int i = 0; i < 4; ++i) old[i] = ring[(T + i - w) & (kFleetRing - 1)];
+    }
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const int32_t S = (int32_t)(pv[i] - old[i]);
+      const bool in = !EDGE || (T + i < H && T + i >= w - 1);
+      cnt[k] += (in && S > win.bw[k]);
+      if (in) pk[k] = max(pk[k], S);
+    }
+  }
+}
+
+template <int NW>
+__global__ void __launch_bounds__(32 * kFleetWarps)
+    fleet_windows_v4_kernel(const uint32_t* __restrict__ prex4, int J, int64_t Lp, int64_t cs,
+                            const int32_t* __restrict__ offsets, int64_t N, int H, FleetWindows win,
+                            int wmax, int32_t* __restrict__ counts, int32_t* __restrict__ peaks) {
+  __shared__ __align__(16) uint32_t ring_all[kFleetWarps][kFleetRing];
+  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+  const int64_t n = (int64_t)blockIdx.x * kFleetWarps + wid;
+  if (n >= N) return;  // the whole warp leaves together; no block-wide barrier follows
+  uint32_t* ring = ring_all[wid];
+  const uint4* bp[kFleetJMax];
+  uint32_t pre_m1 = 0;
+#pragma unroll
+  for (int j = 0; j < kFleetJMax; ++j) {
+    bp[j] = reinterpret_cast<const uint4*>(prex4);
+    if (j < J) {
+      const int32_t o = __ldg(offsets + n * J + j);
+      const int s = o + 1, c = s & 3;
+      bp[j] = reinterpret_cast<const uint4*>(prex4 + c * cs + (int64_t)j * Lp + (s - c));
+      if (lane == j) pre_m1 = __ldg(prex4 + (int64_t)j * Lp + o);
+    }
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) pre_m1 += __shfl_xor_sync(0xffffffffu, pre_m1, o);
+  if (lane == 0) ring[kFleetRing - 1] = pre_m1;
+  __syncwarp();
+  int32_t cnt[NW], pk[NW];
+#pragma unroll
+  for (int k = 0; k < NW; ++k) cnt[k] = pk[k] = 0;
+  for (int t0 = 0; t0 < H; t0 += 128) {
+    const int T = t0 + 4 * lane;
+    uint4 pre = make_uint4(0u, 0u, 0u, 0u);
+#pragma unroll
+    for (int j = 0; j < kFleetJMax; ++j) {
+      if (j < J) {
+        const uint4 v = __ldg(bp[j] + (t0 >> 2) + lane);
+        pre.x += v.x; pre.y += v.y; pre.z += v.z; pre.w += v.w;
+      }
+    }
+    const bool edge = t0 < wmax - 1 || t0 + 128 > H;
+    if (edge) fleet_block4<true, NW>(ring, T, H, pre, win, true, cnt, pk);
+    else fleet_block4<false, NW>(ring, T, H, pre, win, true, cnt, pk);
+    __syncwarp();
+    *reinterpret_cast<uint4*>(ring + (T & (kFleetRing - 1))) = pre;
+    __syncwarp();
+    if (edge) fleet_block4<true, NW>(ring, T, H, pre, win, false, cnt, pk);
+    else fleet_block4<false, NW>(ring, T, H, pre, win, false, cnt, pk);
+  }
+#pragma unroll
+  for (int k = 0; k < NW; ++k) {
+    int32_t c = cnt[k], p = pk[k];
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      c += __shfl_xor_sync(0xffffffffu, c, o);
+      p = max(p, __shfl_xor_sync(0xffffffffu, p, o));
+    }
+    if (lane == 0) {
+      counts[n * NW + k] = c;
+      peaks[n * NW + k] = p;
+    }
+  }
+}
+
+// copies 1..3 of the prefix array for the 16-byte path (copy 0 is PREX,
+// copy c starts cs = J * Lp words after copy c - 1); entries past PREX's last
+// index (L + H) are zero in every copy
+__global__ void fleet_shift_copies_kernel(uint32_t* __restrict__ prex4, int J, int64_t Lp, int64_t last) {
+  const int64_t total = (int64_t)J * Lp;
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < total; i += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t x = i % Lp;
+    const uint32_t* row = prex4 + (i - x);
+    if (x > last) prex4[i] = 0u;
+#pragma unroll
+    for (int c = 1; c < 4; ++c) prex4[c * total + i] = x + c <= last ? row[x + c] : 0u;
+  }
+}
+
+// row stride: PREX[j][0 .. L + H] plus the 127 words a 128-sample block of
+// the 16-byte path may read past a stream's end, rounded to 16 bytes
+static int64_t fleet_lp(int L, int H) { return (((int64_t)L + H + 1 + 127) + 3) / 4 * 4; }
+static int fleet_ncopy(int J, int64_t workspace_bytes, int L, int H);
 static int fleet_nchunk(int L, int H) { return (int)((((int64_t)L + H) + kFleetChunk - 1) / kFleetChunk); }
 
-int64_t fleet_ws_bytes(int J, int L, int H) {
-  const int64_t prex = ((int64_t)J * fleet_lp(L, H) * 4 + 255) / 256 * 256;
+static int64_t fleet_bytes(int J, int L, int H, int ncopy) {
+  const int64_t prex = ((int64_t)ncopy * J * fleet_lp(L, H) * 4 + 255) / 256 * 256;
   const int64_t tot = ((int64_t)J * fleet_nchunk(L, H) * 4 + 255) / 256 * 256;
   return prex + tot + 256 + 256;
+}
+
+// the least workspace (one prefix copy, 4-byte loads) and the workspace of
+// the 16-byte path (four shifted copies; fleets of at most 8 jobs)
+int64_t fleet_ws_min_bytes(int J, int L, int H) { return fleet_bytes(J, L, H, 1); }
+int64_t fleet_ws_bytes(int J, int L, int H) { return fleet_bytes(J, L, H, J <= kFleetJMax ? 4 : 1); }
+static int fleet_ncopy(int J, int64_t workspace_bytes, int L, int H) {
+  return J <= kFleetJMax && workspace_bytes >= fleet_bytes(J, L, H, 4) ? 4 : 1;
 }
 
 // Per-job prefix sums (PREX) and validation of the traces, job map and
 // offsets; returns the per-job maxima (for the int32 range checks).
 static pe_status fleet_prepare(const float* traces, int G, int L, const int32_t* job_of_gpu, int J,
-                               const int32_t* offsets, int64_t N, int H, void* workspace, FleetWs& ws,
-                               int64_t& sum_max, cudaStream_t st) {
+                               const int32_t* offsets, int64_t N, int H, void* workspace, int ncopy,
+                               FleetWs& ws, int64_t& sum_max, cudaStream_t st) {
   char* base = reinterpret_cast<char*>(workspace);
   ws.Lp = fleet_lp(L, H);
   ws.nchunk = fleet_nchunk(L, H);
-  const int64_t prex_bytes = ((int64_t)J * ws.Lp * 4 + 255) / 256 * 256;
+  const int64_t prex_bytes = ((int64_t)ncopy * J * ws.Lp * 4 + 255) / 256 * 256;
   const int64_t tot_bytes = ((int64_t)J * ws.nchunk * 4 + 255) / 256 * 256;
   ws.prex = reinterpret_cast<uint32_t*>(base);
   ws.totals = reinterpret_cast<uint32_t*>(base + prex_bytes);
@@ -353,6 +476,9 @@ static pe_status fleet_prepare(const float* traces, int G, int L, const int32_t*
     fleet_chunk_sums_kernel<<<grid, 256, 0, st>>>(traces, G, L, H, job_of_gpu, J, ws);
     fleet_chunk_scan_kernel<<<J, 32, 0, st>>>(ws);
     fleet_prefix_kernel<<<grid, 256, 0, st>>>(traces, G, L, H, job_of_gpu, J, ws);
+    if (ncopy == 4)
+      fleet_shift_copies_kernel<<<(int)std::min<int64_t>(ceil_div((int64_t)J * ws.Lp, 256), 4096), 256, 0, st>>>(
+          ws.prex, J, ws.Lp, (int64_t)L + H);
     if (N > 0)
       fleet_check_offsets_kernel<<<(int)std::min<int64_t>(ceil_div(N * J, 256), 4096), 256, 0, st>>>(
           offsets, N * J, L, ws.flag);
@@ -374,24 +500,35 @@ static pe_status fleet_prepare(const float* traces, int G, int L, const int32_t*
 pe_status fleet_launch(const float* traces, int G, int L, const int32_t* job_of_gpu, int J,
                        const int32_t* offsets, int64_t N, int H, const int32_t* windows, int W,
                        int64_t budget_q, int32_t* counts, int32_t* peaks, void* workspace,
-                       cudaStream_t st) {
+                       int64_t workspace_bytes, cudaStream_t st) {
   FleetWs ws;
   int64_t sum_max = 0;
-  pe_status s = fleet_prepare(traces, G, L, job_of_gpu, J, offsets, N, H, workspace, ws, sum_max, st);
+  const int ncopy = fleet_ncopy(J, workspace_bytes, L, H);
+  pe_status s = fleet_prepare(traces, G, L, job_of_gpu, J, offsets, N, H, workspace, ncopy, ws, sum_max, st);
   if (s != PE_OK) return s;
   FleetWindows win{};
+  int wmax = 0;
   for (int k = 0; k < W; ++k) {
     const int64_t w = windows[k];
     if (sum_max * w >= (int64_t)INT_MAX || budget_q * w >= (int64_t)INT_MAX)
       return fail(PE_EOVERFLOW, "window %d: composed window sum may exceed int32", (int)w);
     win.w[k] = (int32_t)w;
     win.bw[k] = (int32_t)(budget_q * w);
+    wmax = std::max(wmax, (int)w);
   }
   if (N == 0) return PE_OK;
   const int grid_n = (int)((N + kFleetWarps - 1) / kFleetWarps);
   const int64_t Lx = ws.Lp;
   ProfScope ps(PE_PROF_FLEET_WINDOWS, st);
-  if (J <= kFleetJMax) {
+  const int64_t cs = (int64_t)J * Lx;
+  if (ncopy == 4) {
+    switch (W) {
+      case 1: fleet_windows_v4_kernel<1><<<grid_n, 32 * kFleetWarps, 0, st>>>(ws.prex, J, Lx, cs, offsets, N, H, win, wmax, counts, peaks); break;
+      case 2: fleet_windows_v4_kernel<2><<<grid_n, 32 * kFleetWarps, 0, st>>>(ws.prex, J, Lx, cs, offsets, N, H, win, wmax, counts, peaks); break;
+      case 3: fleet_windows_v4_kernel<3><<<grid_n, 32 * kFleetWarps, 0, st>>>(ws.prex, J, Lx, cs, offsets, N, H, win, wmax, counts, peaks); break;
+      default: fleet_windows_v4_kernel<4><<<grid_n, 32 * kFleetWarps, 0, st>>>(ws.prex, J, Lx, cs, offsets, N, H, win, wmax, counts, peaks); break;
+    }
+  } else if (J <= kFleetJMax) {
     switch (W) {
       case 1: fleet_windows_j8_kernel<1><<<grid_n, 32 * kFleetWarps, 0, st>>>(ws.prex, J, Lx, offsets, N, H, win, counts, peaks); break;
       case 2: fleet_windows_j8_kernel<2><<<grid_n, 32 * kFleetWarps, 0, st>>>(ws.prex, J, Lx, offsets, N, H, win, counts, peaks); break;
@@ -481,7 +618,8 @@ pe_status fleet_stagger_launch(const float* traces, int G, int L, const int32_t*
                                cudaStream_t st) {
   FleetWs ws;
   int64_t sum_max = 0;
-  pe_status s = fleet_prepare(traces, G, L, job_of_gpu, J, nullptr, 0, H, workspace, ws, sum_max, st);
+  const int ncopy = J <= kFleetJMax ? 4 : 1;  // the stagger workspace always holds the copies
+  pe_status s = fleet_prepare(traces, G, L, job_of_gpu, J, nullptr, 0, H, workspace, ncopy, ws, sum_max, st);
   if (s != PE_OK) return s;
   if (sum_max * w >= (int64_t)INT_MAX) return fail(PE_EOVERFLOW, "window %d: composed window sum may exceed int32", w);
   const int64_t nc = stagger_ncand(L, stride);
@@ -501,8 +639,9 @@ pe_status fleet_stagger_launch(const float* traces, int G, int L, const int32_t*
     }
     {
       ProfScope ps(PE_PROF_FLEET_WINDOWS, st);
-      if (j + 1 <= kFleetJMax)
-        fleet_windows_j8_kernel<1><<<grid_n, 32 * kFleetWarps, 0, st>>>(ws.prex, j + 1, ws.Lp, cand, nc, H, win, cnt, pk);
+      if (ncopy == 4)
+        fleet_windows_v4_kernel<1><<<grid_n, 32 * kFleetWarps, 0, st>>>(ws.prex, j + 1, ws.Lp, (int64_t)J * ws.Lp, cand,
+                                                                          nc, H, win, w, cnt, pk);
       else
         fleet_windows_kernel<1><<<grid_n, 32 * kFleetWarps, 0, st>>>(ws.prex, j + 1, ws.Lp, cand, nc, H, win, cnt, pk);
     }

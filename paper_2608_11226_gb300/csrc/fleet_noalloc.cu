@@ -20,7 +20,7 @@
 
 namespace pe {
 
-int64_t fleet_ws_bytes(int J, int L, int H);
+int64_t fleet_ws_min_bytes(int J, int L, int H);
 
 static __device__ __align__(256) unsigned char g_fleet_scratch[PE_FLEET_NOALLOC_SCRATCH_BYTES];
 
@@ -54,10 +54,10 @@ extern "C" pe_status pe_fleet_windows_noalloc(const float* traces, int32_t G, in
   using namespace pe;
   clear_error();
   if (J < 1 || J > 32 || L < 1 || H < 0) return fail(PE_EINVAL, "J must be in [1, 32], L >= 1, H >= 0");
-  const int64_t need = fleet_ws_bytes(J, L, H);
+  const int64_t need = fleet_ws_min_bytes(J, L, H);
   if (need > (int64_t)PE_FLEET_NOALLOC_SCRATCH_BYTES)
     return fail(PE_EINVAL,
-                "fleet scratch of %lld bytes (pe_fleet_workspace_bytes) exceeds the fixed %lld-byte "
+                "fleet scratch of %lld bytes (one prefix copy) exceeds the fixed %lld-byte "
                 "static scratch of pe_fleet_windows_noalloc; use pe_fleet_windows with a workspace",
                 (long long)need, (long long)PE_FLEET_NOALLOC_SCRATCH_BYTES);
   void* scratch = nullptr;

@@ -99,14 +99,17 @@ def test_gae_empty_is_noop():
 
 
 # ---------------------------------------------------------------------- fleet
-def _fleet_gpu(fw, windows):
+def _fleet_gpu(fw, windows, ws_short=0):
+    """ws_short > 0 passes a workspace that many bytes short of
+    pe_fleet_workspace_bytes: for J <= 8 that drops the shifted prefix copies
+    and the call takes its 4-byte-load path."""
     traces = torch.from_numpy(fw.traces).cuda()
     job = torch.from_numpy(fw.job_of_gpu).cuda()
     off = torch.from_numpy(fw.offsets).cuda()
     N = fw.offsets.shape[0]
     counts = torch.empty((N, len(windows)), dtype=torch.int32, device="cuda")
     peaks = torch.empty_like(counts)
-    ws = torch.empty(pe.fleet_workspace_bytes(fw.n_jobs, fw.traces.shape[1], fw.horizon),
+    ws = torch.empty(pe.fleet_workspace_bytes(fw.n_jobs, fw.traces.shape[1], fw.horizon) - ws_short,
                      dtype=torch.uint8, device="cuda")
     pe.fleet_windows(traces, job, fw.n_jobs, off, fw.horizon, windows, fw.budget_q, counts, peaks, ws)
     torch.cuda.synchronize()
@@ -121,14 +124,45 @@ def test_fleet_parity_small_bit_exact():
     assert np.array_equal(c, oc) and np.array_equal(p, op)
 
 
-@pytest.mark.parametrize("H", [1, 31, 599, 600, 2500])
-def test_fleet_parity_horizons(H):
+@pytest.mark.parametrize("H", [1, 31, 127, 128, 129, 599, 600, 2500])
+@pytest.mark.parametrize("path", ["copies", "one_copy"])
+def test_fleet_parity_horizons(H, path):
     fw = W.make_fleet(n_compositions=9, length=2500, windows=(1, 60, 600))
     fw.horizon = H
-    c, p = _fleet_gpu(fw, [1, 7, 60, 600])
-    oc, op = O.fleet_windows(fw.traces, fw.job_of_gpu, fw.n_jobs, fw.offsets, H,
-                             [1, 7, 60, 600], fw.budget_q)
+    windows = [1, 7, 60, 600]
+    c, p = _fleet_gpu(fw, windows, ws_short=1 if path == "one_copy" else 0)
+    oc, op = O.fleet_windows(fw.traces, fw.job_of_gpu, fw.n_jobs, fw.offsets, H, windows, fw.budget_q)
     assert np.array_equal(c, oc) and np.array_equal(p, op)
+
+
+@pytest.mark.parametrize("windows", [[1, 2, 3, 5], [127, 128, 129, 992], [4, 124, 132, 991]])
+def test_fleet_parity_window_alignments(windows):
+    """Windows on and off the 4-sample and 128-sample block boundaries of the
+    16-byte path, including the largest window; offsets at both trace ends."""
+    fw = W.make_fleet(n_compositions=11, length=3000, windows=(1, 60, 600))
+    fw.offsets[0, :] = 0
+    fw.offsets[1, :] = fw.traces.shape[1] - 1
+    fw.offsets[2, :] = np.arange(fw.n_jobs) % 4
+    for short in (0, 1):
+        c, p = _fleet_gpu(fw, windows, ws_short=short)
+        oc, op = O.fleet_windows(fw.traces, fw.job_of_gpu, fw.n_jobs, fw.offsets, fw.horizon, windows,
+                                 fw.budget_q)
+        assert np.array_equal(c, oc) and np.array_equal(p, op)
+
+
+def test_fleet_parity_more_than_eight_jobs():
+    """Twelve jobs over the sixteen traces: the path for fleets of more than
+    eight jobs (one prefix copy, stream bases in shared memory)."""
+    fw = W.make_fleet(n_compositions=13, length=1800, windows=(1, 60, 600))
+    fw.job_of_gpu = (np.arange(fw.traces.shape[0]) % 12).astype(np.int32)
+    fw.n_jobs = 12
+    fw.offsets = np.random.default_rng(4).integers(0, 1800, (13, 12)).astype(np.int32)
+    fw.budget_q = fw.budget_q // 2
+    c, p = _fleet_gpu(fw, [1, 60, 600])
+    oc, op = O.fleet_windows(fw.traces, fw.job_of_gpu, fw.n_jobs, fw.offsets, fw.horizon, [1, 60, 600],
+                             fw.budget_q)
+    assert np.array_equal(c, oc) and np.array_equal(p, op)
+    assert c.sum() > 0
 
 
 def test_fleet_parity_full_size_sampled():
