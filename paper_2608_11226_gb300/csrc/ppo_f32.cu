@@ -612,6 +612,38 @@ __global__ void __launch_bounds__(kPpoNT) ppo_grad_kernel(PpoArgs g) {
     ppo_role<D, H, A, false>(s, g, blockIdx.x - g.NC);
 }
 
+// Running minibatch statistics from the per-CTA partials, by one whole warp:
+// lane c sums rows c, c + 32, ... in fp32, a fixed xor tree combines the
+// lanes, and lane 0 adds the minibatch means to the fp64 running sums
+// (pg loss, value loss, entropy, approximate KL, clip fraction, total loss).
+// The partials are read through L2: inside the persistent update other CTAs
+// wrote them.
+__device__ __forceinline__ void fold_stats(const float* stat_partial, int NC, float inv_cnt, float vf_coef,
+                                           float ent_coef, double* acc) {
+  const int lane = threadIdx.x & 31;
+  float v[5] = {0.0f, 0.0f, 0.0f, 0.0f, 0.0f};
+  for (int c = lane; c < NC; c += 32) {
+    v[0] += __ldcg(stat_partial + c * 8 + 0);
+    v[1] += __ldcg(stat_partial + c * 8 + 1);
+    v[2] += __ldcg(stat_partial + c * 8 + 2);
+    v[3] += __ldcg(stat_partial + c * 8 + 3);
+    v[4] += __ldcg(stat_partial + (NC + c) * 8 + 4);
+  }
+#pragma unroll
+  for (int k = 0; k < 5; ++k)
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v[k] += __shfl_xor_sync(0xffffffffu, v[k], o);
+  if (lane == 0) {
+    const double ic = inv_cnt;
+    acc[0] += (double)v[0] * ic;
+    acc[1] += (double)v[4] * ic;
+    acc[2] += (double)v[1] * ic;
+    acc[3] += (double)v[2] * ic;
+    acc[4] += (double)v[3] * ic;
+    acc[5] += (double)v[0] * ic + (double)vf_coef * v[4] * ic - (double)ent_coef * v[1] * ic;
+  }
+}
+
 // ---------------------------------------------------------------------------
 // Persistent form of the whole update: one cooperative launch runs every
 // minibatch step as three phases separated by grid barriers -- gradient
@@ -742,40 +774,21 @@ __global__ void __launch_bounds__(kPpoNT, 1) ppo_persistent_kernel(PpoLoop L) {
       }
       const float qb = block_sum_f(q, s_red);
       if (tid == 0) L.sq[blockIdx.x] = qb;
-      if (blockIdx.x == 0 && tid < 32) {
-        double v[5] = {0, 0, 0, 0, 0};
-        for (int c = tid; c < NC; c += 32) {
-          v[0] += __ldcg(g.stat_partial + c * 8 + 0);
-          v[1] += __ldcg(g.stat_partial + c * 8 + 1);
-          v[2] += __ldcg(g.stat_partial + c * 8 + 2);
-          v[3] += __ldcg(g.stat_partial + c * 8 + 3);
-          v[4] += __ldcg(g.stat_partial + (NC + c) * 8 + 4);
-        }
-#pragma unroll
-        for (int k = 0; k < 5; ++k)
-#pragma unroll
-          for (int o = 16; o > 0; o >>= 1) v[k] += __shfl_xor_sync(0xffffffffu, v[k], o);
-        if (tid == 0) {
-          const double ic = g.inv_cnt;
-          L.acc[0] += v[0] * ic;
-          L.acc[1] += v[4] * ic;
-          L.acc[2] += v[1] * ic;
-          L.acc[3] += v[2] * ic;
-          L.acc[4] += v[3] * ic;
-          L.acc[5] += v[0] * ic + g.vf_coef * v[4] * ic - g.ent_coef * v[1] * ic;
-        }
-      }
       if (!grid_barrier(L.bar, &s_ok)) {
         if (tid == 0) atomicExch(L.err, 1);
         return;
       }
-      // phase 3: global norm (fixed order), clip factor, Adam on this slice
+      // phase 3: global norm (fixed order), clip factor, Adam on this slice.
+      // The last CTA, whose parameter slice is the shortest, also folds the
+      // minibatch statistics (its warp 1), off the barrier-bound path.
       if (tid < 32) {
         float t = 0.0f;
         for (int b = tid; b < (int)gridDim.x; b += 32) t += __ldcg(L.sq + b);
 #pragma unroll
         for (int o = 16; o > 0; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
         if (tid == 0) s_norm = sqrtf(t);
+      } else if (tid < 64 && blockIdx.x == gridDim.x - 1) {
+        fold_stats(g.stat_partial, NC, g.inv_cnt, g.vf_coef, g.ent_coef, L.acc);
       }
       __syncthreads();
       const float norm = s_norm;
@@ -860,31 +873,12 @@ __global__ void __launch_bounds__(kRedP * kRedG) ppo_reduce_kernel(ReduceArgs a)
   if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = q;
   __syncthreads();
   if (threadIdx.x < 32) {
-    // minibatch statistics: lane c sums rows c, c+32, ... of the stat partials
-    double v[5] = {0, 0, 0, 0, 0};
-    for (int c = threadIdx.x; c < a.NC; c += 32) {
-      v[0] += a.stat_partial[c * 8 + 0];
-      v[1] += a.stat_partial[c * 8 + 1];
-      v[2] += a.stat_partial[c * 8 + 2];
-      v[3] += a.stat_partial[c * 8 + 3];
-      v[4] += a.stat_partial[(a.NC + c) * 8 + 4];
-    }
-#pragma unroll
-    for (int k = 0; k < 5; ++k)
-#pragma unroll
-      for (int o = 16; o > 0; o >>= 1) v[k] += __shfl_xor_sync(0xffffffffu, v[k], o);
+    fold_stats(a.stat_partial, a.NC, a.inv_cnt, a.vf_coef, a.ent_coef, a.acc);
     if (threadIdx.x == 0) {
       float t = 0.0f;
       for (int k = 0; k < kRedG; ++k) t += red[k];
       const float norm = sqrtf(t);
       *a.norm = norm;
-      const double ic = a.inv_cnt;
-      a.acc[0] += v[0] * ic;
-      a.acc[1] += v[4] * ic;
-      a.acc[2] += v[1] * ic;
-      a.acc[3] += v[2] * ic;
-      a.acc[4] += v[3] * ic;
-      a.acc[5] += v[0] * ic + a.vf_coef * v[4] * ic - a.ent_coef * v[1] * ic;
       a.acc[6] = norm;
       a.acc[7] += 1.0;
       *a.ticket = 0u;
