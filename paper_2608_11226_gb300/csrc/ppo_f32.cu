@@ -31,6 +31,7 @@ constexpr int kPpoLD = kPpoS + 4;   // row stride of feature-major activations
 constexpr int kPpoNT = 512;         // threads per gradient CTA
 constexpr int kPpoRT = 4;           // sample rows per thread tile in the dense layers
 constexpr int kPpoMaxEpochs = 16;
+constexpr int kPpoMaxNC = 128;      // CTAs per network: above half the SMs of any GB300
 
 struct FeistelSet {
   Feistel f[kPpoMaxEpochs];
@@ -92,14 +93,15 @@ __device__ __forceinline__ bool dense_job(int j, int& eg, int& ng) {
   return ng < NG;
 }
 
-// outT[n][e] = tanh(b[n] + sum_k inT[k][e] WT[k][n]); WT rows are LDW floats apart
+// outT[n][e] = tanh(b[n] + sum_k inT[k][e] WT[k][n]) for samples e < SV (a
+// multiple of RT; later rows are left as they are); WT rows are LDW floats apart
 template <int TE, int K, int N, int LD, int RT, int LDW = N>
 __device__ __forceinline__ void dense_fwd_w(const float* __restrict__ inT, const float* __restrict__ WT,
-                                            const float* __restrict__ bias, float* __restrict__ outT) {
+                                            const float* __restrict__ bias, float* __restrict__ outT, int SV) {
   constexpr int JOBS = (TE / RT) * (N / 4);
   for (int j = threadIdx.x; j < JOBS; j += blockDim.x) {
     int eg, ng;
-    if (!dense_job<TE, N, RT>(j, eg, ng)) continue;
+    if (!dense_job<TE, N, RT>(j, eg, ng) || eg * RT >= SV) continue;
     float acc[RT][4];
 #pragma unroll
     for (int r = 0; r < RT; ++r)
@@ -135,11 +137,12 @@ __device__ __forceinline__ void dense_fwd_w(const float* __restrict__ inT, const
 // apart, different banks with the padded stride) and are broadcasts.
 template <int TE, int K, int N, int LD, int LDW>
 __device__ __forceinline__ void dense_bwd_wt(const float* __restrict__ inT, const float* __restrict__ WT,
-                                             float* hT) {
+                                             float* hT, int SV) {
   constexpr int RT = 4, EG = TE / RT, NG = N / 4, JOBS = EG * NG;
   static_assert(K % 4 == 0 && EG == 16, "backward tile layout");
   for (int j = threadIdx.x; j < JOBS; j += blockDim.x) {
     const int eg = j % EG, kg = j / EG;
+    if (eg * RT >= SV) continue;  // samples past the slice's valid rows
     float acc[RT][4];
 #pragma unroll
     for (int r = 0; r < RT; ++r)
@@ -200,14 +203,15 @@ struct WGradAcc {
 #pragma unroll
         for (int j = 0; j < 4; ++j) acc[q][i][j] = 0.0f;
   }
+  // over samples s < SV (a multiple of 4, at most S)
   template <int S, int LD>
-  __device__ __forceinline__ void add(const float* __restrict__ aT, const float* __restrict__ bT) {
+  __device__ __forceinline__ void add(const float* __restrict__ aT, const float* __restrict__ bT, int SV) {
 #pragma unroll
     for (int q = 0; q < PER; ++q) {
       int mg, ng;
       if (job(q, mg, ng)) {
 #pragma unroll 2
-        for (int s = 0; s < S; s += 4) {
+        for (int s = 0; s < SV; s += 4) {
           float4 a[4], b[4];
 #pragma unroll
           for (int i = 0; i < 4; ++i) a[i] = *reinterpret_cast<const float4*>(aT + (mg + i * MG) * LD + s);
@@ -294,7 +298,8 @@ struct PpoArgs {
   float* partial;       // [NC][P]
   float* stat_partial;  // [2*NC][8]
   float* grad_out;      // [P] reduced gradient (persistent kernel)
-  int NC, slices_per_cta;
+  int NC;       // CTAs per network
+  int per_cta;  // minibatch samples per CTA, ceil(cnt / NC): CTA c takes [c * per_cta, (c + 1) * per_cta)
   int64_t P, PS;  // parameters; row stride of the partial-sum matrix
 };
 
@@ -358,14 +363,15 @@ __device__ __forceinline__ void ppo_role(PpoSmem<D, H, A>& s, const PpoArgs& g, 
   const int64_t oW3 = POL ? Lp.w3 : Lp.v3, oB3 = POL ? Lp.b3 : Lp.c3;
   const int tid = threadIdx.x;
   const float2 as = *g.advstat;
-  // gather one slice (permuted sample order): observations as float4 rows,
-  // per-sample scalars by threads 256..256+S
-  auto gather = [&](int base) {
+  // gather one slice (permuted sample order) of nv <= S samples:
+  // observations as float4 rows, per-sample scalars by threads 256..256+S;
+  // rows past nv are zero and marked invalid
+  auto gather = [&](int base, int nv) {
     constexpr int F4 = D / 4;
     if (tid < S * F4) {
       const int si = tid / F4, f = tid % F4;
       float4 v = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
-      if (base + si < g.cnt) {
+      if (si < nv) {
         const uint32_t idx = feistel_index(g.perm, g.start + base + si);
         v = __ldg(reinterpret_cast<const float4*>(g.obs + (int64_t)idx * D) + f);
       }
@@ -375,7 +381,7 @@ __device__ __forceinline__ void ppo_role(PpoSmem<D, H, A>& s, const PpoArgs& g, 
       s.xt[(4 * f + 3) * LD + si] = v.w;
     } else if (tid >= 256 && tid < 256 + S) {
       const int si = tid - 256;
-      const int ok = base + si < g.cnt;
+      const int ok = si < nv;
       s.valid[si] = ok;
       if (ok) {
         const uint32_t idx = feistel_index(g.perm, g.start + base + si);
@@ -389,8 +395,10 @@ __device__ __forceinline__ void ppo_role(PpoSmem<D, H, A>& s, const PpoArgs& g, 
       }
     }
   };
+  // this CTA's samples [c0, c1) of the minibatch, in slices of S
+  const int c0 = c * g.per_cta, c1 = min(c0 + g.per_cta, g.cnt);
   // the first slice's gather overlaps the weight loads
-  if (c * g.slices_per_cta * S < g.cnt) gather(c * g.slices_per_cta * S);
+  if (c0 < c1) gather(c0, min(S, c1 - c0));
   // the role's weight image, read through L2 (not the non-coherent L1 path):
   // inside the persistent update other CTAs rewrite it between minibatches.
   // Four float4 loads per thread are in flight before they are stored.
@@ -422,24 +430,27 @@ __device__ __forceinline__ void ppo_role(PpoSmem<D, H, A>& s, const PpoArgs& g, 
   for (int a = 0; a < NA; ++a) g3[a] = 0.0f;
   float st[5] = {0.0f, 0.0f, 0.0f, 0.0f, 0.0f};  // pg, entropy, kl, clip, value (threads < S)
 
-  for (int sl = 0; sl < g.slices_per_cta; ++sl) {
-    const int base = (c * g.slices_per_cta + sl) * S;
-    if (base >= g.cnt) break;
-    if (sl > 0) {
+  for (int base = c0; base < c1; base += S) {
+    // nv valid samples; the tiles cover the first SV rows (nv rounded up to
+    // 8: whole 4-row groups, both groups of a warp).  Rows in [nv, SV) are
+    // zero-input samples whose loss gradient is zero.
+    const int nv = min(S, c1 - base), SV = min(S, (nv + 7) & ~7);
+    if (base > c0) {
       __syncthreads();
-      gather(base);
+      gather(base, nv);
     }
     __syncthreads();
     // forward
-    dense_fwd_w<S, D, H, LD, kPpoRT>(s.xt, s.w1t, s.b1, s.h1t);
+    dense_fwd_w<S, D, H, LD, kPpoRT>(s.xt, s.w1t, s.b1, s.h1t, SV);
     __syncthreads();
-    dense_fwd_w<S, H, H, LD, kPpoRT, w2t_ld<H>()>(s.h1t, s.w2t, s.b2, s.h2t);
+    dense_fwd_w<S, H, H, LD, kPpoRT, w2t_ld<H>()>(s.h1t, s.w2t, s.b2, s.h2t, SV);
     __syncthreads();
     // head: thread (sample si = tid / 8, K-part q = tid % 8) sums k = q, q+8, ...
     // for every action; the 8 parts (adjacent lanes) are shuffle-combined
     {
       static_assert(S * 8 == kPpoNT, "one head job per thread");
       const int q = tid & 7, si = tid >> 3;
+      if (si < SV) {  // warp-uniform: a warp covers 4 samples and SV is a multiple of 8
       float acc[NA];
 #pragma unroll
       for (int a = 0; a < NA; ++a) acc[a] = 0.0f;
@@ -458,6 +469,7 @@ __device__ __forceinline__ void ppo_role(PpoSmem<D, H, A>& s, const PpoArgs& g, 
       if (q == 0)
 #pragma unroll
         for (int a = 0; a < NA; ++a) s.z[si * NA + a] = acc[a] + s.b3[a];
+      }
     }
     __syncthreads();
     // loss terms and dLoss/dhead per sample (written over the head outputs)
@@ -512,7 +524,7 @@ __device__ __forceinline__ void ppo_role(PpoSmem<D, H, A>& s, const PpoArgs& g, 
 #pragma unroll
       for (int a = 0; a < NA; ++a) w3k[a] = s.w3[a * H + hk];
 #pragma unroll 4
-      for (int i = 0; i < S / 4; ++i) {
+      for (int i = 0; i < SV / 4; ++i) {
         const int si = 4 * i + hq;
         const float h = s.h2t[hk * LD + si];
         float d = 0.0f;
@@ -537,24 +549,27 @@ __device__ __forceinline__ void ppo_role(PpoSmem<D, H, A>& s, const PpoArgs& g, 
     {
       WGradAcc<H, H, kPpoNT> g2;
       g2.zero();
-      g2.template add<S, LD>(s.h2t, s.h1t);
+      g2.template add<S, LD>(s.h2t, s.h1t, SV);
       g2.add_to(s.gw2, w2t_ld<H>(), nsl == 0);
     }
     __syncthreads();
     // back into layer 1 (in place over h1)
-    dense_bwd_wt<S, H, H, LD, w2t_ld<H>()>(s.h2t, s.w2t, s.h1t);
+    dense_bwd_wt<S, H, H, LD, w2t_ld<H>()>(s.h2t, s.w2t, s.h1t, SV);
     __syncthreads();
     // layer-1 weight and bias gradients (the bias by the warps the tiles leave idle)
     {
       WGradAcc<H, D, kPpoNT> g1;
       g1.zero();
-      g1.template add<S, LD>(s.h1t, s.xt);
+      g1.template add<S, LD>(s.h1t, s.xt, SV);
       g1.add_to(s.gw1, D, nsl == 0);
     }
     if (tid >= kPpoNT - H) {
       const int n = tid - (kPpoNT - H), lane = tid & 31;
       float acc = 0.0f;
-      for (int i = 0; i < S; ++i) acc += s.h1t[n * LD + ((i + lane) & (S - 1))];
+      for (int i = 0; i < S; ++i) {
+        const int e = (i + lane) & (S - 1);
+        if (e < SV) acc += s.h1t[n * LD + e];
+      }
       gb1 += acc;
     }
     ++nsl;
@@ -564,7 +579,16 @@ __device__ __forceinline__ void ppo_role(PpoSmem<D, H, A>& s, const PpoArgs& g, 
   // the accumulated hidden-layer weight gradients, coalesced (zero if the
   // CTA's slices held no sample)
   __syncthreads();
-  for (int i = tid; i < H * H; i += blockDim.x) row[oW2 + i] = nsl ? s.gw2[(i / H) * w2t_ld<H>() + i % H] : 0.0f;
+  {
+#pragma unroll 8
+    for (int u = 0; u < (H * H + kPpoNT - 1) / kPpoNT; ++u) {
+      const int i = tid + u * kPpoNT;
+      if (i < H * H) {
+        const float v = s.gw2[(i / H) * w2t_ld<H>() + i % H];
+        row[oW2 + i] = nsl ? v : 0.0f;
+      }
+    }
+  }
   for (int i = tid; i < H * D; i += blockDim.x) row[oW1 + i] = nsl ? s.gw1[i] : 0.0f;
 #pragma unroll
   for (int a = 0; a < NA; ++a) {
@@ -721,6 +745,7 @@ __global__ void __launch_bounds__(kPpoNT, 1) ppo_persistent_kernel(PpoLoop L) {
       g.start = start;
       g.cnt = cnt;
       g.inv_cnt = 1.0f / (float)cnt;
+      g.per_cta = (cnt + NC - 1) / NC;
       g.advstat = L.advstat + (int64_t)ep * L.nmb + mb;
       // phase 1: gradient partials of this CTA's role and samples
       if ((int)blockIdx.x < NC)
@@ -743,8 +768,7 @@ __global__ void __launch_bounds__(kPpoNT, 1) ppo_persistent_kernel(PpoLoop L) {
           const int64_t p = pb + 4 * c4;
           float4 acc4 = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
           if (p < p1) {
-#pragma unroll
-            for (int h = 0; h < 8; h += 4) {
+            for (int h = 0; 8 * h < NC; h += 4) {
               float4 v[4];
 #pragma unroll
               for (int u = 0; u < 4; ++u)
@@ -940,7 +964,7 @@ Feistel make_feistel(uint64_t n, uint64_t seed, uint32_t epoch, uint32_t iterati
 
 struct PpoPlan {
   int64_t P, N;
-  int nmb, NC, slices_per_cta, nsq, steps;
+  int nmb, NC, nsq, steps;  // NC: the most CTAs per network a launch may use (workspace bound)
   int64_t PS;  // row stride of the partial-sum matrix (P rounded up to 4)
   int64_t off_advstat, off_partial, off_stat, off_grad, off_img, off_sq, off_acc, off_bar, off_bc, total;
 };
@@ -958,9 +982,8 @@ static PpoPlan ppo_plan(const pe_net& net, const pe_ppo_config& cfg, int64_t N) 
   p.PS = (p.P + 3) / 4 * 4;
   p.N = N;
   p.nmb = (int)((N + cfg.minibatch - 1) / cfg.minibatch);
-  const int slices = (cfg.minibatch + kPpoS - 1) / kPpoS;
-  p.NC = slices < 64 ? slices : 64;
-  p.slices_per_cta = (slices + p.NC - 1) / p.NC;
+  const int ncap = (cfg.minibatch + 7) / 8;  // at least 8 samples per CTA
+  p.NC = ncap < kPpoMaxNC ? ncap : kPpoMaxNC;
   p.nsq = (int)((p.P + kRedP - 1) / kRedP);
   p.steps = cfg.epochs * p.nmb;
   int64_t o = 0;
@@ -1040,7 +1063,9 @@ static pe_status ppo_run(const pe_net& net, float* params, float* m, float* v, i
   int per_sm = 0, coop = 0;
   PE_TRY_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, pk, kPpoNT, bytes));
   PE_TRY_CUDA(cudaDeviceGetAttribute(&coop, cudaDevAttrCooperativeLaunch, dev));
-  if (coop && per_sm * sms >= 2 * pl.NC) {
+  // one CTA per SM for each network: as many CTAs as the GPU holds at once
+  const int nc = std::min(pl.NC, per_sm * sms / 2);
+  if (coop && nc >= 1) {
     std::vector<float> bc(2 * (size_t)pl.steps);
     for (int k = 0; k < pl.steps; ++k) {
       const double tt = (double)(adam_t + k + 1);
@@ -1064,8 +1089,7 @@ static pe_status ppo_run(const pe_net& net, float* params, float* m, float* v, i
     L.g.partial = partial;
     L.g.stat_partial = stat_partial;
     L.g.grad_out = grad;
-    L.g.NC = pl.NC;
-    L.g.slices_per_cta = pl.slices_per_cta;
+    L.g.NC = nc;
     L.g.P = pl.P;
     L.g.PS = pl.PS;
     L.advstat = advstat;
@@ -1089,10 +1113,11 @@ static pe_status ppo_run(const pe_net& net, float* params, float* m, float* v, i
     void* kargs[] = {&L};
     {
       ProfScope ps(PE_PROF_PPO_GRAD, st);
-      PE_TRY_CUDA(cudaLaunchCooperativeKernel((void*)pk, dim3(2 * pl.NC), dim3(kPpoNT), kargs, (size_t)bytes, st));
+      PE_TRY_CUDA(cudaLaunchCooperativeKernel((void*)pk, dim3(2 * nc), dim3(kPpoNT), kargs, (size_t)bytes, st));
     }
     PE_CHECK_LAUNCH("ppo_persistent_kernel");
   } else {
+    const int ncf = std::min(pl.NC, 64);
     int64_t t = adam_t;
     for (int ep = 0; ep < cfg.epochs; ++ep) {
       for (int mb = 0; mb < pl.nmb; ++mb) {
@@ -1115,14 +1140,14 @@ static pe_status ppo_run(const pe_net& net, float* params, float* m, float* v, i
         g.inv_cnt = 1.0f / (float)cnt;
         g.partial = partial;
         g.stat_partial = stat_partial;
-        g.NC = pl.NC;
-        g.slices_per_cta = pl.slices_per_cta;
+        g.NC = ncf;
+        g.per_cta = (cnt + ncf - 1) / ncf;
         g.P = pl.P;
         g.PS = pl.PS;
         g.advstat = advstat + (int64_t)ep * pl.nmb + mb;
         {
           ProfScope ps(PE_PROF_PPO_GRAD, st);
-          kern<<<2 * pl.NC, kPpoNT, bytes, st>>>(g);
+          kern<<<2 * ncf, kPpoNT, bytes, st>>>(g);
         }
         PE_CHECK_LAUNCH("ppo_grad_kernel");
         {
@@ -1130,7 +1155,7 @@ static pe_status ppo_run(const pe_net& net, float* params, float* m, float* v, i
           ReduceArgs ra;
           ra.partial = partial;
           ra.stat_partial = stat_partial;
-          ra.NC = pl.NC;
+          ra.NC = ncf;
           ra.P = pl.P;
           ra.PS = pl.PS;
           ra.grad = grad;
