@@ -688,33 +688,32 @@ struct PpoLoop {
   float* v;
   float* sq;               // [gridDim.x] per-CTA sums of squares
   double* acc;             // [8] running statistics
-  unsigned int* bar;       // [2]: arrival count, generation
+  unsigned int* bar;       // monotonic arrival count, zeroed before the launch
   int32_t* err;
   const float* bc;         // [2 * steps]: step_size, 1/sqrt(bc2) per Adam step
   float beta1, beta2, eps, max_norm;
 };
 
+// Grid barrier on a monotonic arrival counter (zeroed before the launch):
+// the k-th barrier's arrivals are numbered k*G .. k*G + G - 1 (no CTA can
+// arrive at barrier k + 1 before all have arrived at k), so each CTA waits
+// for the counter to reach (k + 1) * G; the last arrival releases everyone
+// with its own atomic, and nothing is reset.  The wait is bounded.
 __device__ __forceinline__ bool grid_barrier(unsigned int* bar, int* s_ok) {
   __syncthreads();
   if (threadIdx.x == 0) {
-    volatile unsigned int* gen = bar + 1;
-    const unsigned int g0 = *gen;
     __threadfence();
-    const unsigned int arrived = atomicAdd(bar, 1u) + 1u;
+    const unsigned int old = atomicAdd(bar, 1u);
+    const unsigned int target = (old / gridDim.x + 1u) * gridDim.x;
+    volatile unsigned int* vb = bar;
     bool ok = true;
-    if (arrived == gridDim.x) {
-      atomicExch(bar, 0u);
-      __threadfence();
-      atomicAdd(bar + 1, 1u);
-    } else {
-      const long long t0 = clock64();
-      while (*gen == g0) {
-        if (clock64() - t0 > 4000000000LL) {  // about 2 s at the maximum SM clock
-          ok = false;
-          break;
-        }
-        __nanosleep(64);
+    const long long t0 = clock64();
+    while ((int)(*vb - target) < 0) {
+      if (clock64() - t0 > 4000000000LL) {  // about 2 s at the maximum SM clock
+        ok = false;
+        break;
       }
+      __nanosleep(32);
     }
     __threadfence();
     *s_ok = ok;
