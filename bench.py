@@ -572,7 +572,8 @@ def run_72b(args, world, peaks):
     for k in range(pe.PE_PROF_KINDS):
         pe.profile_read(k)
     barrier(world)
-    pe.profile_enable(True)
+    # whole rollouts timed with the per-launch event profiler off (its event
+    # pairs around ~2,050 launches would add to the rollout's time) ...
     stream = torch.cuda.current_stream()
     a = torch.cuda.Event(enable_timing=True)
     b = torch.cuda.Event(enable_timing=True)
@@ -581,9 +582,14 @@ def run_72b(args, world, peaks):
         pe.rollout(env, net, params, T, it + 1, buf, lam=1.0, workspace=ws)
     b.record(stream)
     torch.cuda.synchronize()
-    pe.profile_enable(False)
     pe.device_check()
     ms = max_over_ranks(a.elapsed_time(b), world) / args.r72b_steps
+    # ... and one more rollout with it on, for the per-kernel device times
+    pe.profile_enable(True)
+    pe.rollout(env, net, params, T, args.r72b_steps + 1, buf, lam=1.0, workspace=ws)
+    torch.cuda.synchronize()
+    pe.profile_enable(False)
+    pe.device_check()
     prof = {pe.profile_kind_name(k): pe.profile_read(k) for k in range(pe.PE_PROF_KINDS)}
     D, H, A = net.obs_dim, net.hidden, net.n_actions
     pol_flop = 2.0 * E * (D * H + H * H + H * A)          # one policy launch (E rows)
@@ -618,15 +624,14 @@ def run_72b(args, world, peaks):
     vms, vn = prof["mlp_value_tc"]
     peak = float(peaks.get("bf16_tflops_sustained", 1728.9))
     pol = pol_flop / (pms / pn / 1e3) / 1e12 if pn else None
-    val = val_flop * args.r72b_steps / (vms / 1e3) / 1e12 if vn else None
+    val = val_flop / (vms / 1e3) / 1e12 if vn else None
     env.close()
     return {"metric": "72B rollout env-steps/s", "value": E * T * world / (ms / 1e3),
             "unit": "env-steps/s", "ms_per_rollout": ms,
             "config": {"workload": f"72b: {E} envs x {T} steps, 4-channel 22,000-sample trace, "
                                    "16 levels, MLP 32-256-256 bf16 (tcgen05), value on all T*E obs",
                        "n_envs": E, "horizon": T},
-            "kernels": {k: {"ms_per_rollout": v[0] / args.r72b_steps,
-                            "launches_per_rollout": v[1] / args.r72b_steps} for k, v in prof.items() if v[1]},
+            "kernels": {k: {"ms_per_rollout": v[0], "launches_per_rollout": v[1]} for k, v in prof.items() if v[1]},
             "roofline_policy_mlp": {"kernel": f"mlp_bf16_kernel (policy, {E} rows)", "bound": "tensor",
                                     "achieved": pol, "peak": peak, "unit": "TFLOP/s",
                                     "frac": pol / peak if pol else None,
@@ -738,7 +743,8 @@ def run_72b_ppo(args, world, peaks, wl, buf, adv, ret):
     for k in range(pe.PE_PROF_KINDS):
         pe.profile_read(k)
     barrier(world)
-    pe.profile_enable(True)
+    # timed with the per-launch event profiler off, then one more update with
+    # it on for the per-kernel device times
     stream = torch.cuda.current_stream()
     e0 = torch.cuda.Event(enable_timing=True)
     e1 = torch.cuda.Event(enable_timing=True)
@@ -746,14 +752,17 @@ def run_72b_ppo(args, world, peaks, wl, buf, adv, ret):
     pe.ppo_update(net, ppo, params, m, v, 1, obs, act, lpo, a_, r_, stats, ws, seed=7, iteration=1)
     e1.record(stream)
     torch.cuda.synchronize()
-    pe.profile_enable(False)
     ms = max_over_ranks(e0.elapsed_time(e1), world)
+    st = [float(x) for x in stats.cpu()]
+    pe.profile_enable(True)
+    pe.ppo_update(net, ppo, params, m, v, 2, obs, act, lpo, a_, r_, stats, ws, seed=7, iteration=2)
+    torch.cuda.synchronize()
+    pe.profile_enable(False)
     prof = {pe.profile_kind_name(k): pe.profile_read(k) for k in range(pe.PE_PROF_KINDS)}
     steps = (n + mb - 1) // mb
     fl = ppo_flops_per_sample(net.obs_dim, net.hidden, net.n_actions) * n
     peak = float(peaks.get("bf16_tflops_sustained", 1728.9))
     ach = fl / (ms / 1e3) / 1e12
-    st = [float(x) for x in stats.cpu()]
     del ws
     return {"metric": "72B PPO update samples/s", "value": n * world / (ms / 1e3), "unit": "samples/s",
             "ms_per_minibatch_step": ms / steps, "minibatch": mb, "steps": steps,

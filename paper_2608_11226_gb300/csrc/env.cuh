@@ -99,8 +99,9 @@ struct TileAcc {
   __device__ int32_t& sl(int c) { return s.s_long[e][c]; }
   __device__ uint8_t level_at(int p) const { return s.ring[e][p & (kRing - 1)]; }
   __device__ void set_level_at(int p, int l) { s.ring[e][p & (kRing - 1)] = (uint8_t)l; }
-  // actuated sample of channel c at a recent position p (p in [pos-64, pos))
-  __device__ int32_t q_at(const EnvDev&, int c, int p) const { return s.q[e][c][p & (kRing - 1)]; }
+  // actuated sample of channel c at a recent position p (p in [pos-64, pos));
+  // fm is the env's family view (unused: the tile caches the samples)
+  __device__ int32_t q_at(const EnvDev&, const Fam&, int c, int p) const { return s.q[e][c][p & (kRing - 1)]; }
   __device__ void push(int c, int p, int32_t q) { s.q[e][c][p & (kRing - 1)] = q; }
 };
 
@@ -120,8 +121,9 @@ struct RegAcc {
   __device__ int32_t& sl(int c) { return sl_[c]; }
   __device__ uint8_t level_at(int p) const { return ring[p & (kRing - 1)]; }
   __device__ void set_level_at(int p, int l) { ring[p & (kRing - 1)] = (uint8_t)l; }
-  __device__ int32_t q_at(const EnvDev& env, int c, int p) const {
-    return sample_q(env, fam_of(env, fam_), c, p, level_at(p));
+  // recomputed from the trace of the env's family (view fm) and the level ring
+  __device__ int32_t q_at(const EnvDev& env, const Fam& fm, int c, int p) const {
+    return sample_q(env, fm, c, p, level_at(p));
   }
   __device__ void push(int, int, int32_t) {}
 };
@@ -130,11 +132,12 @@ struct RegAcc {
 template <int C, class Acc>
 __device__ void rebuild_history(const EnvDev& env, Acc& a) {
   const int p = a.pos();
+  const Fam fm = fam_of(env, a.fam());
   for (int c = 0; c < C; ++c) {
     int32_t ss = 0, sl = 0;
     for (int i = 1; i <= kWLong; ++i) {
       const int pp = p - i;
-      const int32_t q = sample_q(env, fam_of(env, a.fam()), c, pp, a.level_at(pp));
+      const int32_t q = sample_q(env, fm, c, pp, a.level_at(pp));
       a.push(c, pp, q);
       sl += q;
       if (i <= kWShort) ss += q;
@@ -170,15 +173,15 @@ __device__ void env_reset(const EnvDev& env, Acc& a, uint32_t eg, uint32_t t, ui
 }
 
 template <int C, class Acc>
-__device__ __forceinline__ int32_t Qc(const EnvDev& env, Acc& a, int c, int i) {
-  return a.q_at(env, c, a.pos() - 1 - i);
+__device__ __forceinline__ int32_t Qc(const EnvDev& env, Acc& a, const Fam& fm, int c, int i) {
+  return a.q_at(env, fm, c, a.pos() - 1 - i);
 }
 
 template <int C, class Acc>
-__device__ __forceinline__ int32_t Qcl(const EnvDev& env, Acc& a, int i) {
+__device__ __forceinline__ int32_t Qcl(const EnvDev& env, Acc& a, const Fam& fm, int i) {
   int32_t v = 0;
 #pragma unroll
-  for (int c = 0; c < C; ++c) v += Qc<C>(env, a, c, i);
+  for (int c = 0; c < C; ++c) v += Qc<C>(env, a, fm, c, i);
   return v;
 }
 
@@ -187,13 +190,14 @@ __device__ __forceinline__ int32_t Qcl(const EnvDev& env, Acc& a, int i) {
 //   TINY8 (Sec. 4.1): 5 latest samples, headroom, phase, level
 //   7B16: 8 latest samples, 30 s mean, 30 s slack, phase, G, b, 10 s mean, 5 s slope, 0
 //   OCC32/OCC64: Eq. 5 eight-vector, then per-channel recent samples and means
+//   fm: the env's family view, fam_of(env, a.fam()), taken once per step by
+//   callers that write a whole observation
 template <int C, int OBS, class Acc>
-__device__ __forceinline__ float feature(const EnvDev& env, Acc& a, int f) {
-  const Fam fm = fam_of(env, a.fam());
+__device__ __forceinline__ float feature(const EnvDev& env, Acc& a, const Fam& fm, int f) {
   const int64_t B = fm.B;
   if (OBS == PE_OBS_TINY8) {
-    if (f < 5) return ratio_i(Qcl<C>(env, a, 4 - f), B);
-    if (f == 5) return ratio_i(B - Qcl<C>(env, a, 0), B);
+    if (f < 5) return ratio_i(Qcl<C>(env, a, fm, 4 - f), B);
+    if (f == 5) return ratio_i(B - Qcl<C>(env, a, fm, 0), B);
     if (f == 6) return (float)__ldg(fm.phase + a.pos() - 1);
     return ratio_i(a.level(), env.n_levels - 1);
   }
@@ -204,7 +208,7 @@ __device__ __forceinline__ float feature(const EnvDev& env, Acc& a, int f) {
     S60 += a.sl(c);
   }
   if (OBS == PE_OBS_7B16) {
-    if (f < 8) return ratio_i(Qcl<C>(env, a, 7 - f), B);
+    if (f < 8) return ratio_i(Qcl<C>(env, a, fm, 7 - f), B);
     switch (f) {
       case 8: return ratio_i(S60, kWLong * B);
       case 9: return ratio_i(kWLong * B - S60, kWLong * B);
@@ -212,17 +216,17 @@ __device__ __forceinline__ float feature(const EnvDev& env, Acc& a, int f) {
       case 11: return ratio_i(a.level() - env.g_min, env.g_max - env.g_min);
       case 12: return ratio_i(a.b() - env.b_min, env.b_max - env.b_min);
       case 13: return ratio_i(S20, kWShort * B);
-      case 14: return ratio_i((int64_t)Qcl<C>(env, a, 0) - Qcl<C>(env, a, 10), B);
+      case 14: return ratio_i((int64_t)Qcl<C>(env, a, fm, 0) - Qcl<C>(env, a, fm, 10), B);
       default: return 0.0f;
     }
   }
   // OCC32 / OCC64 (Eq. 5 core)
   switch (f) {
-    case 0: return ratio_i(Qcl<C>(env, a, 0), B);
+    case 0: return ratio_i(Qcl<C>(env, a, fm, 0), B);
     case 1: return ratio_i(S20, kWShort * B);
     case 2: return ratio_i(S60, kWLong * B);
     case 3: return ratio_i(kWLong * B - S60, kWLong * B);
-    case 4: return ratio_i((int64_t)Qcl<C>(env, a, 0) - Qcl<C>(env, a, 10), B);
+    case 4: return ratio_i((int64_t)Qcl<C>(env, a, fm, 0) - Qcl<C>(env, a, fm, 10), B);
     case 5: return ratio_i(a.level() + 1, env.n_levels);
     case 6: return ratio_i(a.prev() + 1, env.n_levels);
     case 7: return fminf(env.cadence ? ratio_i(env.ns[a.level()], 40) : ratio_i(a.til(), 40), 1.0f);
@@ -231,7 +235,7 @@ __device__ __forceinline__ float feature(const EnvDev& env, Acc& a, int f) {
   if (OBS == PE_OBS_OCC32) {
     if (f < 24) {
       const int c = (f - 8) >> 2, i = (f - 8) & 3;
-      return c < fm.C ? ratio_i((int64_t)fm.C * Qc<C>(env, a, c, 3 - i), B) : 0.0f;
+      return c < fm.C ? ratio_i((int64_t)fm.C * Qc<C>(env, a, fm, c, 3 - i), B) : 0.0f;
     }
     if (f < 28) {
       const int c = f - 24;
@@ -242,7 +246,7 @@ __device__ __forceinline__ float feature(const EnvDev& env, Acc& a, int f) {
   // OCC64
   if (f < 56) {
     const int c = (f - 8) / 12, i = (f - 8) % 12;
-    return c < fm.C ? ratio_i((int64_t)fm.C * Qc<C>(env, a, c, 11 - i), B) : 0.0f;
+    return c < fm.C ? ratio_i((int64_t)fm.C * Qc<C>(env, a, fm, c, 11 - i), B) : 0.0f;
   }
   if (f < 60) {
     const int c = f - 56;
@@ -250,6 +254,11 @@ __device__ __forceinline__ float feature(const EnvDev& env, Acc& a, int f) {
   }
   const int c = f - 60;
   return c < fm.C ? ratio_i((int64_t)fm.C * a.sl(c), kWLong * B) : 0.0f;
+}
+
+template <int C, int OBS, class Acc>
+__device__ __forceinline__ float feature(const EnvDev& env, Acc& a, int f) {
+  return feature<C, OBS>(env, a, fam_of(env, a.fam()), f);
 }
 
 struct StepOut {
@@ -296,8 +305,8 @@ __device__ __forceinline__ StepOut env_step(const EnvDev& env, Acc& a, int act, 
 #pragma unroll
     for (int c = 0; c < C; ++c) {
       const int32_t qin = quant64(__ldg(fm.trace + (int64_t)c * fm.L + p), actuator_scale(env, nl, c, ph));
-      const int32_t q20 = a.q_at(env, c, p - kWShort);
-      const int32_t q60 = a.q_at(env, c, p - kWLong);
+      const int32_t q20 = a.q_at(env, fm, c, p - kWShort);
+      const int32_t q60 = a.q_at(env, fm, c, p - kWLong);
       a.ss(c) += qin - q20;
       a.sl(c) += qin - q60;
       a.push(c, p, qin);

@@ -32,7 +32,7 @@ __device__ __forceinline__ int rule_action(const EnvDev& env, RegAcc<C>& a, cons
   const int raise = incdec ? 2 : (lvl < env.n_levels - 1 ? lvl + 1 : env.n_levels - 1);
   if (r.kind == PE_RULE_RANDOM) return (int)__umulhi(draw32(env.seed, e, t, r.it, kDrawAction), (uint32_t)env.A);
   if (r.kind == PE_RULE_THRESHOLD) {
-    const int32_t q = Qcl<C>(env, a, 0);  // latest actuated cluster sample
+    const int32_t q = Qcl<C>(env, a, fam_of(env, a.fam()), 0);  // latest actuated cluster sample
     return q > r.hi_q ? lower : (q < r.lo_q ? raise : hold);
   }
   int64_t s10 = 0, s30 = 0;
@@ -47,14 +47,15 @@ __device__ __forceinline__ int rule_action(const EnvDev& env, RegAcc<C>& a, cons
 
 template <int C, int OBS, int D>
 __device__ __forceinline__ void write_obs(const EnvDev& env, RegAcc<C>& a, void* dst, int bf16) {
+  const Fam fm = fam_of(env, a.fam());
   if (bf16) {
     __nv_bfloat16* o = reinterpret_cast<__nv_bfloat16*>(dst);
 #pragma unroll 1
-    for (int f = 0; f < D; ++f) o[f] = __float2bfloat16_rn(feature<C, OBS>(env, a, f));
+    for (int f = 0; f < D; ++f) o[f] = __float2bfloat16_rn(feature<C, OBS>(env, a, fm, f));
   } else {
     float* o = reinterpret_cast<float*>(dst);
 #pragma unroll 1
-    for (int f = 0; f < D; ++f) o[f] = feature<C, OBS>(env, a, f);
+    for (int f = 0; f < D; ++f) o[f] = feature<C, OBS>(env, a, fm, f);
   }
 }
 
