@@ -248,9 +248,20 @@ __global__ void __launch_bounds__(32 * kFleetWarps)
 // issues the loads of two 32-sample blocks before using either.
 constexpr int kFleetJMax = 8;
 
+// prefix-array row of each composed stream (stream k reads row r[k]): the
+// identity for a fleet, {partial fleet, candidate job} for the stagger
+struct StreamRows {
+  int32_t r[kFleetJMax];
+};
+static StreamRows identity_rows() {
+  StreamRows m;
+  for (int k = 0; k < kFleetJMax; ++k) m.r[k] = k;
+  return m;
+}
+
 template <int NW>
 __global__ void __launch_bounds__(32 * kFleetWarps)
-    fleet_windows_j8_kernel(const uint32_t* __restrict__ prex, int J, int64_t Lp,
+    fleet_windows_j8_kernel(const uint32_t* __restrict__ prex, int J, int64_t Lp, StreamRows rows,
                             const int32_t* __restrict__ offsets, int64_t N, int H, FleetWindows win,
                             int32_t* __restrict__ counts, int32_t* __restrict__ peaks) {
   __shared__ uint32_t ring_all[kFleetWarps][kFleetRing];
@@ -267,7 +278,7 @@ __global__ void __launch_bounds__(32 * kFleetWarps)
     bp[j] = prex;
     if (j < J) {
       const int32_t o = __ldg(offsets + n * J + j);
-      bp[j] = prex + (int64_t)j * Lp + o + 1;
+      bp[j] = prex + (int64_t)rows.r[j] * Lp + o + 1;
       if (lane == j) pre_m1 = __ldg(bp[j] - 1);
     }
   }
@@ -360,7 +371,7 @@ __device__ __forceinline__ void fleet_block4(const uint32_t* ring, int T, int H,
 
 template <int NW>
 __global__ void __launch_bounds__(32 * kFleetWarps)
-    fleet_windows_v4_kernel(const uint32_t* __restrict__ prex4, int J, int64_t Lp, int64_t cs,
+    fleet_windows_v4_kernel(const uint32_t* __restrict__ prex4, int J, int64_t Lp, int64_t cs, StreamRows rows,
                             const int32_t* __restrict__ offsets, int64_t N, int H, FleetWindows win,
                             int wmax, int32_t* __restrict__ counts, int32_t* __restrict__ peaks) {
   __shared__ __align__(16) uint32_t ring_all[kFleetWarps][kFleetRing];
@@ -376,8 +387,8 @@ __global__ void __launch_bounds__(32 * kFleetWarps)
     if (j < J) {
       const int32_t o = __ldg(offsets + n * J + j);
       const int s = o + 1, c = s & 3;
-      bp[j] = reinterpret_cast<const uint4*>(prex4 + c * cs + (int64_t)j * Lp + (s - c));
-      if (lane == j) pre_m1 = __ldg(prex4 + (int64_t)j * Lp + o);
+      bp[j] = reinterpret_cast<const uint4*>(prex4 + c * cs + (int64_t)rows.r[j] * Lp + (s - c));
+      if (lane == j) pre_m1 = __ldg(prex4 + (int64_t)rows.r[j] * Lp + o);
     }
   }
 #pragma unroll
@@ -421,17 +432,18 @@ __global__ void __launch_bounds__(32 * kFleetWarps)
   }
 }
 
-// copies 1..3 of the prefix array for the 16-byte path (copy 0 is PREX,
-// copy c starts cs = J * Lp words after copy c - 1); entries past PREX's last
-// index (L + H) are zero in every copy
-__global__ void fleet_shift_copies_kernel(uint32_t* __restrict__ prex4, int J, int64_t Lp, int64_t last) {
-  const int64_t total = (int64_t)J * Lp;
+// copies 1..3 of nrows prefix rows for the 16-byte path (copy 0 is the rows
+// themselves, copy c starts cs words after copy c - 1); entries past a row's
+// last index are zero in every copy
+__global__ void fleet_shift_copies_kernel(uint32_t* __restrict__ rows0, int nrows, int64_t Lp, int64_t cs,
+                                          int64_t last) {
+  const int64_t total = (int64_t)nrows * Lp;
   for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < total; i += (int64_t)gridDim.x * blockDim.x) {
     const int64_t x = i % Lp;
-    const uint32_t* row = prex4 + (i - x);
-    if (x > last) prex4[i] = 0u;
+    const uint32_t* row = rows0 + (i - x);
+    if (x > last) rows0[i] = 0u;
 #pragma unroll
-    for (int c = 1; c < 4; ++c) prex4[c * total + i] = x + c <= last ? row[x + c] : 0u;
+    for (int c = 1; c < 4; ++c) rows0[c * cs + i] = x + c <= last ? row[x + c] : 0u;
   }
 }
 
@@ -441,8 +453,9 @@ static int64_t fleet_lp(int L, int H) { return (((int64_t)L + H + 1 + 127) + 3) 
 static int fleet_ncopy(int J, int64_t workspace_bytes, int L, int H);
 static int fleet_nchunk(int L, int H) { return (int)((((int64_t)L + H) + kFleetChunk - 1) / kFleetChunk); }
 
-static int64_t fleet_bytes(int J, int L, int H, int ncopy) {
-  const int64_t prex = ((int64_t)ncopy * J * fleet_lp(L, H) * 4 + 255) / 256 * 256;
+// rows = J job rows plus `extra` working rows, in each of ncopy copies
+static int64_t fleet_bytes(int J, int L, int H, int ncopy, int extra = 0) {
+  const int64_t prex = ((int64_t)ncopy * (J + extra) * fleet_lp(L, H) * 4 + 255) / 256 * 256;
   const int64_t tot = ((int64_t)J * fleet_nchunk(L, H) * 4 + 255) / 256 * 256;
   return prex + tot + 256 + 256;
 }
@@ -459,11 +472,11 @@ static int fleet_ncopy(int J, int64_t workspace_bytes, int L, int H) {
 // offsets; returns the per-job maxima (for the int32 range checks).
 static pe_status fleet_prepare(const float* traces, int G, int L, const int32_t* job_of_gpu, int J,
                                const int32_t* offsets, int64_t N, int H, void* workspace, int ncopy,
-                               FleetWs& ws, int64_t& sum_max, cudaStream_t st) {
+                               int extra, FleetWs& ws, int64_t& sum_max, cudaStream_t st) {
   char* base = reinterpret_cast<char*>(workspace);
   ws.Lp = fleet_lp(L, H);
   ws.nchunk = fleet_nchunk(L, H);
-  const int64_t prex_bytes = ((int64_t)ncopy * J * ws.Lp * 4 + 255) / 256 * 256;
+  const int64_t prex_bytes = ((int64_t)ncopy * (J + extra) * ws.Lp * 4 + 255) / 256 * 256;
   const int64_t tot_bytes = ((int64_t)J * ws.nchunk * 4 + 255) / 256 * 256;
   ws.prex = reinterpret_cast<uint32_t*>(base);
   ws.totals = reinterpret_cast<uint32_t*>(base + prex_bytes);
@@ -478,7 +491,7 @@ static pe_status fleet_prepare(const float* traces, int G, int L, const int32_t*
     fleet_prefix_kernel<<<grid, 256, 0, st>>>(traces, G, L, H, job_of_gpu, J, ws);
     if (ncopy == 4)
       fleet_shift_copies_kernel<<<(int)std::min<int64_t>(ceil_div((int64_t)J * ws.Lp, 256), 4096), 256, 0, st>>>(
-          ws.prex, J, ws.Lp, (int64_t)L + H);
+          ws.prex, J, ws.Lp, (int64_t)(J + extra) * ws.Lp, (int64_t)L + H);
     if (N > 0)
       fleet_check_offsets_kernel<<<(int)std::min<int64_t>(ceil_div(N * J, 256), 4096), 256, 0, st>>>(
           offsets, N * J, L, ws.flag);
@@ -504,7 +517,7 @@ pe_status fleet_launch(const float* traces, int G, int L, const int32_t* job_of_
   FleetWs ws;
   int64_t sum_max = 0;
   const int ncopy = fleet_ncopy(J, workspace_bytes, L, H);
-  pe_status s = fleet_prepare(traces, G, L, job_of_gpu, J, offsets, N, H, workspace, ncopy, ws, sum_max, st);
+  pe_status s = fleet_prepare(traces, G, L, job_of_gpu, J, offsets, N, H, workspace, ncopy, 0, ws, sum_max, st);
   if (s != PE_OK) return s;
   FleetWindows win{};
   int wmax = 0;
@@ -521,19 +534,20 @@ pe_status fleet_launch(const float* traces, int G, int L, const int32_t* job_of_
   const int64_t Lx = ws.Lp;
   ProfScope ps(PE_PROF_FLEET_WINDOWS, st);
   const int64_t cs = (int64_t)J * Lx;
+  const StreamRows id = identity_rows();
   if (ncopy == 4) {
     switch (W) {
-      case 1: fleet_windows_v4_kernel<1><<<grid_n, 32 * kFleetWarps, 0, st>>>(ws.prex, J, Lx, cs, offsets, N, H, win, wmax, counts, peaks); break;
-      case 2: fleet_windows_v4_kernel<2><<<grid_n, 32 * kFleetWarps, 0, st>>>(ws.prex, J, Lx, cs, offsets, N, H, win, wmax, counts, peaks); break;
-      case 3: fleet_windows_v4_kernel<3><<<grid_n, 32 * kFleetWarps, 0, st>>>(ws.prex, J, Lx, cs, offsets, N, H, win, wmax, counts, peaks); break;
-      default: fleet_windows_v4_kernel<4><<<grid_n, 32 * kFleetWarps, 0, st>>>(ws.prex, J, Lx, cs, offsets, N, H, win, wmax, counts, peaks); break;
+      case 1: fleet_windows_v4_kernel<1><<<grid_n, 32 * kFleetWarps, 0, st>>>(ws.prex, J, Lx, cs, id, offsets, N, H, win, wmax, counts, peaks); break;
+      case 2: fleet_windows_v4_kernel<2><<<grid_n, 32 * kFleetWarps, 0, st>>>(ws.prex, J, Lx, cs, id, offsets, N, H, win, wmax, counts, peaks); break;
+      case 3: fleet_windows_v4_kernel<3><<<grid_n, 32 * kFleetWarps, 0, st>>>(ws.prex, J, Lx, cs, id, offsets, N, H, win, wmax, counts, peaks); break;
+      default: fleet_windows_v4_kernel<4><<<grid_n, 32 * kFleetWarps, 0, st>>>(ws.prex, J, Lx, cs, id, offsets, N, H, win, wmax, counts, peaks); break;
     }
   } else if (J <= kFleetJMax) {
     switch (W) {
-      case 1: fleet_windows_j8_kernel<1><<<grid_n, 32 * kFleetWarps, 0, st>>>(ws.prex, J, Lx, offsets, N, H, win, counts, peaks); break;
-      case 2: fleet_windows_j8_kernel<2><<<grid_n, 32 * kFleetWarps, 0, st>>>(ws.prex, J, Lx, offsets, N, H, win, counts, peaks); break;
-      case 3: fleet_windows_j8_kernel<3><<<grid_n, 32 * kFleetWarps, 0, st>>>(ws.prex, J, Lx, offsets, N, H, win, counts, peaks); break;
-      default: fleet_windows_j8_kernel<4><<<grid_n, 32 * kFleetWarps, 0, st>>>(ws.prex, J, Lx, offsets, N, H, win, counts, peaks); break;
+      case 1: fleet_windows_j8_kernel<1><<<grid_n, 32 * kFleetWarps, 0, st>>>(ws.prex, J, Lx, id, offsets, N, H, win, counts, peaks); break;
+      case 2: fleet_windows_j8_kernel<2><<<grid_n, 32 * kFleetWarps, 0, st>>>(ws.prex, J, Lx, id, offsets, N, H, win, counts, peaks); break;
+      case 3: fleet_windows_j8_kernel<3><<<grid_n, 32 * kFleetWarps, 0, st>>>(ws.prex, J, Lx, id, offsets, N, H, win, counts, peaks); break;
+      default: fleet_windows_j8_kernel<4><<<grid_n, 32 * kFleetWarps, 0, st>>>(ws.prex, J, Lx, id, offsets, N, H, win, counts, peaks); break;
     }
   } else {
     switch (W) {
@@ -555,14 +569,25 @@ pe_status fleet_launch(const float* traces, int G, int L, const int32_t* job_of_
 // the lowest candidate among equal peaks.  The chosen offsets never leave
 // the device between stages.
 // ---------------------------------------------------------------------------
-__global__ void stagger_candidates_kernel(int32_t* __restrict__ cand, int64_t ncand, int j, int stride,
-                                          const int32_t* __restrict__ chosen) {
-  const int64_t total = ncand * (j + 1);
+// candidate c's stream offsets: (0 for the partial-fleet row, c * stride)
+// from the second stage on, (c * stride) alone for the first job
+__global__ void stagger_candidates_kernel(int32_t* __restrict__ cand, int64_t ncand, int per, int stride) {
+  const int64_t total = ncand * per;
   for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < total; i += (int64_t)gridDim.x * blockDim.x) {
-    const int64_t c = i / (j + 1);
-    const int k = (int)(i % (j + 1));
-    cand[i] = k < j ? chosen[k] : (int32_t)(c * stride);
+    const int64_t c = i / per;
+    cand[i] = (int)(i % per) == per - 1 ? (int32_t)(c * stride) : 0;
   }
+}
+
+// partial-fleet row R[y] = sum over the placed jobs k < j of PREX[k][o_k + y]
+// for y in [0, H] (zero past H): stage j adds job j - 1 at its chosen
+// offset (stage 1 starts from zero).  With offset 0, R composes like a job.
+__global__ void stagger_compose_kernel(uint32_t* __restrict__ R, const uint32_t* __restrict__ prex, int64_t Lp,
+                                       int jprev, const int32_t* __restrict__ chosen, int H) {
+  const int32_t o = chosen[jprev];
+  const uint32_t* src = prex + (int64_t)jprev * Lp + o;
+  for (int64_t y = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; y < Lp; y += (int64_t)gridDim.x * blockDim.x)
+    R[y] = y <= H ? (jprev > 0 ? R[y] : 0u) + src[y] : 0u;
 }
 
 __global__ void __launch_bounds__(1024) stagger_argmin_kernel(const int32_t* __restrict__ peaks, int64_t ncand,
@@ -606,11 +631,15 @@ __global__ void __launch_bounds__(1024) stagger_argmin_kernel(const int32_t* __r
 
 static int64_t stagger_ncand(int L, int stride) { return ((int64_t)L + stride - 1) / stride; }
 
+// four prefix copies of the J job rows and the partial-fleet row, then two
+// candidate offsets and a peak and count per candidate
+static int64_t stagger_prefix_bytes(int J, int L, int H) { return fleet_bytes(J, L, H, 4, 1); }
+
 int64_t fleet_stagger_ws_bytes(int J, int L, int H, int stride) {
   const int64_t nc = stagger_ncand(L, stride);
-  const int64_t cand = (nc * J * 4 + 255) / 256 * 256;
+  const int64_t cand = (nc * 2 * 4 + 255) / 256 * 256;
   const int64_t outs = (nc * 4 + 255) / 256 * 256;
-  return fleet_ws_bytes(J, L, H) + cand + 2 * outs;
+  return stagger_prefix_bytes(J, L, H) + cand + 2 * outs;
 }
 
 pe_status fleet_stagger_launch(const float* traces, int G, int L, const int32_t* job_of_gpu, int J, int H,
@@ -618,32 +647,44 @@ pe_status fleet_stagger_launch(const float* traces, int G, int L, const int32_t*
                                cudaStream_t st) {
   FleetWs ws;
   int64_t sum_max = 0;
-  const int ncopy = J <= kFleetJMax ? 4 : 1;  // the stagger workspace always holds the copies
-  pe_status s = fleet_prepare(traces, G, L, job_of_gpu, J, nullptr, 0, H, workspace, ncopy, ws, sum_max, st);
+  // job rows 0..J-1 and the partial-fleet row J, in four shifted copies
+  pe_status s = fleet_prepare(traces, G, L, job_of_gpu, J, nullptr, 0, H, workspace, 4, 1, ws, sum_max, st);
   if (s != PE_OK) return s;
   if (sum_max * w >= (int64_t)INT_MAX) return fail(PE_EOVERFLOW, "window %d: composed window sum may exceed int32", w);
   const int64_t nc = stagger_ncand(L, stride);
-  char* base = reinterpret_cast<char*>(workspace) + fleet_ws_bytes(J, L, H);
+  char* base = reinterpret_cast<char*>(workspace) + stagger_prefix_bytes(J, L, H);
   int32_t* cand = reinterpret_cast<int32_t*>(base);
-  int32_t* cnt = reinterpret_cast<int32_t*>(base + (nc * J * 4 + 255) / 256 * 256);
+  int32_t* cnt = reinterpret_cast<int32_t*>(base + (nc * 2 * 4 + 255) / 256 * 256);
   int32_t* pk = cnt + (nc * 4 + 255) / 256 * 64;
+  const int64_t cs = (int64_t)(J + 1) * ws.Lp;
+  uint32_t* R = ws.prex + (int64_t)J * ws.Lp;
   FleetWindows win{};
   win.w[0] = w;
   win.bw[0] = INT_MAX;  // counts unused
   const int grid_n = (int)((nc + kFleetWarps - 1) / kFleetWarps);
   for (int j = 0; j < J; ++j) {
+    // stage j composes two streams: the partial fleet of jobs 0..j-1 (row J,
+    // offset 0) and job j at each candidate; the first stage has job 0 alone
+    const int per = j == 0 ? 1 : 2;
+    StreamRows rows = identity_rows();
+    if (j > 0) {
+      rows.r[0] = J;
+      rows.r[1] = j;
+    }
     {
       ProfScope ps(PE_PROF_FLEET_PREP, st);
-      stagger_candidates_kernel<<<(int)std::min<int64_t>(ceil_div(nc * (j + 1), 256), 4096), 256, 0, st>>>(
-          cand, nc, j, stride, offsets_out);
+      if (j > 0) {
+        const int gb = (int)std::min<int64_t>(ceil_div(ws.Lp, 256), 4096);
+        stagger_compose_kernel<<<gb, 256, 0, st>>>(R, ws.prex, ws.Lp, j - 1, offsets_out, H);
+        fleet_shift_copies_kernel<<<gb, 256, 0, st>>>(R, 1, ws.Lp, cs, (int64_t)H);
+      }
+      stagger_candidates_kernel<<<(int)std::min<int64_t>(ceil_div(nc * per, 256), 4096), 256, 0, st>>>(
+          cand, nc, per, stride);
     }
     {
       ProfScope ps(PE_PROF_FLEET_WINDOWS, st);
-      if (ncopy == 4)
-        fleet_windows_v4_kernel<1><<<grid_n, 32 * kFleetWarps, 0, st>>>(ws.prex, j + 1, ws.Lp, (int64_t)J * ws.Lp, cand,
-                                                                          nc, H, win, w, cnt, pk);
-      else
-        fleet_windows_kernel<1><<<grid_n, 32 * kFleetWarps, 0, st>>>(ws.prex, j + 1, ws.Lp, cand, nc, H, win, cnt, pk);
+      fleet_windows_v4_kernel<1><<<grid_n, 32 * kFleetWarps, 0, st>>>(ws.prex, per, ws.Lp, cs, rows, cand, nc, H,
+                                                                        win, w, cnt, pk);
     }
     {
       ProfScope ps(PE_PROF_FLEET_PREP, st);
