@@ -66,36 +66,39 @@ __device__ __forceinline__ void store_rt(float* p, const float (&v)[RT]) {
 }
 
 // outT[n][e] = tanh(b[n] + sum_k inT[k][e] * WT[k][n]) for TE rows; each
-// thread owns an RT-row x 4-neuron register tile.  LD is the row stride (in
-// floats) of inT and outT.
+// thread owns an RT-row x 4-neuron register tile, accumulated as neuron pairs
+// with the packed two-lane FMA (__ffma2_rn: two round-to-nearest fused
+// multiply-adds, the same results as fmaf, in one instruction) and the row
+// value broadcast to both lanes.  LD is the row stride (in floats) of inT
+// and outT.
 template <int TE, int K, int N, int LD = TE, int RT = 4>
 __device__ __forceinline__ void dense_tanh_t(const float* __restrict__ inT, const float* __restrict__ WT,
                                              const float* __restrict__ bias, float* __restrict__ outT) {
   constexpr int EG = TE / RT, NG = N / 4;
   for (int j = threadIdx.x; j < EG * NG; j += blockDim.x) {
     const int eg = j % EG, ng = j / EG;
-    float acc[RT][4];
+    float2 acc2[RT][2];
 #pragma unroll
-    for (int r = 0; r < RT; ++r)
-#pragma unroll
-      for (int c = 0; c < 4; ++c) acc[r][c] = 0.0f;
+    for (int r = 0; r < RT; ++r) acc2[r][0] = acc2[r][1] = make_float2(0.0f, 0.0f);
 #pragma unroll 8
     for (int k = 0; k < K; ++k) {
       float xv[RT];
       load_rt<RT>(inT + k * LD + eg * RT, xv);
       const float4 w = *reinterpret_cast<const float4*>(WT + k * N + ng * 4);
-      const float wv[4] = {w.x, w.y, w.z, w.w};
+      const float2 w01 = make_float2(w.x, w.y), w23 = make_float2(w.z, w.w);
 #pragma unroll
-      for (int r = 0; r < RT; ++r)
-#pragma unroll
-        for (int c = 0; c < 4; ++c) acc[r][c] = fmaf(xv[r], wv[c], acc[r][c]);
+      for (int r = 0; r < RT; ++r) {
+        const float2 xx = make_float2(xv[r], xv[r]);
+        acc2[r][0] = __ffma2_rn(xx, w01, acc2[r][0]);
+        acc2[r][1] = __ffma2_rn(xx, w23, acc2[r][1]);
+      }
     }
 #pragma unroll
     for (int c = 0; c < 4; ++c) {
       const float bb = bias[ng * 4 + c];
       float o[RT];
 #pragma unroll
-      for (int r = 0; r < RT; ++r) o[r] = tanhf(acc[r][c] + bb);
+      for (int r = 0; r < RT; ++r) o[r] = tanhf(((c & 1) ? acc2[r][c >> 1].y : acc2[r][c >> 1].x) + bb);
       store_rt<RT>(outT + (ng * 4 + c) * LD + eg * RT, o);
     }
   }

@@ -94,7 +94,10 @@ __device__ __forceinline__ bool dense_job(int j, int& eg, int& ng) {
 }
 
 // outT[n][e] = tanh(b[n] + sum_k inT[k][e] WT[k][n]) for samples e < SV (a
-// multiple of RT; later rows are left as they are); WT rows are LDW floats apart
+// multiple of RT; later rows are left as they are); WT rows are LDW floats apart.
+// Neuron pairs accumulate with the packed two-lane FMA (__ffma2_rn: two
+// round-to-nearest fused multiply-adds, the same results as fmaf, in one
+// instruction), the sample value broadcast to both lanes.
 template <int TE, int K, int N, int LD, int RT, int LDW = N>
 __device__ __forceinline__ void dense_fwd_w(const float* __restrict__ inT, const float* __restrict__ WT,
                                             const float* __restrict__ bias, float* __restrict__ outT, int SV) {
@@ -102,28 +105,28 @@ __device__ __forceinline__ void dense_fwd_w(const float* __restrict__ inT, const
   for (int j = threadIdx.x; j < JOBS; j += blockDim.x) {
     int eg, ng;
     if (!dense_job<TE, N, RT>(j, eg, ng) || eg * RT >= SV) continue;
-    float acc[RT][4];
+    float2 acc2[RT][2];
 #pragma unroll
-    for (int r = 0; r < RT; ++r)
-#pragma unroll
-      for (int c = 0; c < 4; ++c) acc[r][c] = 0.0f;
+    for (int r = 0; r < RT; ++r) acc2[r][0] = acc2[r][1] = make_float2(0.0f, 0.0f);
 #pragma unroll 8
     for (int k = 0; k < K; ++k) {
       float xv[RT];
       load_rt<RT>(inT + k * LD + eg * RT, xv);
       const float4 w = *reinterpret_cast<const float4*>(WT + k * LDW + ng * 4);
-      const float wv[4] = {w.x, w.y, w.z, w.w};
+      const float2 w01 = make_float2(w.x, w.y), w23 = make_float2(w.z, w.w);
 #pragma unroll
-      for (int r = 0; r < RT; ++r)
-#pragma unroll
-        for (int c = 0; c < 4; ++c) acc[r][c] = fmaf(xv[r], wv[c], acc[r][c]);
+      for (int r = 0; r < RT; ++r) {
+        const float2 xx = make_float2(xv[r], xv[r]);
+        acc2[r][0] = __ffma2_rn(xx, w01, acc2[r][0]);
+        acc2[r][1] = __ffma2_rn(xx, w23, acc2[r][1]);
+      }
     }
 #pragma unroll
     for (int c = 0; c < 4; ++c) {
       const float bb = bias[ng * 4 + c];
       float o[RT];
 #pragma unroll
-      for (int r = 0; r < RT; ++r) o[r] = tanhf(acc[r][c] + bb);
+      for (int r = 0; r < RT; ++r) o[r] = tanhf(((c & 1) ? acc2[r][c >> 1].y : acc2[r][c >> 1].x) + bb);
       store_rt<RT>(outT + (ng * 4 + c) * LD + eg * RT, o);
     }
   }
@@ -132,7 +135,8 @@ __device__ __forceinline__ void dense_fwd_w(const float* __restrict__ inT, const
 // back through a tanh layer, in place, from the transposed weights:
 //   hT[k][e] <- (sum_n inT[n][e] W[n][k]) * (1 - hT[k][e]^2),  W[n][k] = WT[k][n]
 // A thread owns RT = 4 samples x 4 outputs k; per 4 n it loads a 4x4 block of
-// WT (rows k, columns n..n+3) and of inT and does 64 FMAs.  A warp covers 16
+// WT (rows k, columns n..n+3) and of inT and does 64 FMAs as 32 packed
+// two-lane FMAs over sample pairs (the weight broadcast to both lanes).  A warp covers 16
 // sample groups x 2 output groups, so its WT loads touch two rows (4 rows
 // apart, different banks with the padded stride) and are broadcasts.
 template <int TE, int K, int N, int LD, int LDW>
@@ -143,11 +147,9 @@ __device__ __forceinline__ void dense_bwd_wt(const float* __restrict__ inT, cons
   for (int j = threadIdx.x; j < JOBS; j += blockDim.x) {
     const int eg = j % EG, kg = j / EG;
     if (eg * RT >= SV) continue;  // samples past the slice's valid rows
-    float acc[RT][4];
+    float2 acc2[2][4];  // acc2[rp][c] = (acc[2 rp][c], acc[2 rp + 1][c])
 #pragma unroll
-    for (int r = 0; r < RT; ++r)
-#pragma unroll
-      for (int c = 0; c < 4; ++c) acc[r][c] = 0.0f;
+    for (int c = 0; c < 4; ++c) acc2[0][c] = acc2[1][c] = make_float2(0.0f, 0.0f);
 #pragma unroll 2
     for (int n = 0; n < K; n += 4) {
       float4 w[4], d[4];
@@ -160,10 +162,9 @@ __device__ __forceinline__ void dense_bwd_wt(const float* __restrict__ inT, cons
         const float wc[4] = {w[c].x, w[c].y, w[c].z, w[c].w};
 #pragma unroll
         for (int q = 0; q < 4; ++q) {
-          acc[0][c] = fmaf(d[q].x, wc[q], acc[0][c]);
-          acc[1][c] = fmaf(d[q].y, wc[q], acc[1][c]);
-          acc[2][c] = fmaf(d[q].z, wc[q], acc[2][c]);
-          acc[3][c] = fmaf(d[q].w, wc[q], acc[3][c]);
+          const float2 ww = make_float2(wc[q], wc[q]);
+          acc2[0][c] = __ffma2_rn(make_float2(d[q].x, d[q].y), ww, acc2[0][c]);
+          acc2[1][c] = __ffma2_rn(make_float2(d[q].z, d[q].w), ww, acc2[1][c]);
         }
       }
     }
@@ -171,8 +172,9 @@ __device__ __forceinline__ void dense_bwd_wt(const float* __restrict__ inT, cons
     for (int c = 0; c < 4; ++c) {
       float h[RT], o[RT];
       load_rt<RT>(hT + (kg * 4 + c) * LD + eg * RT, h);
+      const float a4[4] = {acc2[0][c].x, acc2[0][c].y, acc2[1][c].x, acc2[1][c].y};
 #pragma unroll
-      for (int r = 0; r < RT; ++r) o[r] = acc[r][c] * (1.0f - h[r] * h[r]);
+      for (int r = 0; r < RT; ++r) o[r] = a4[r] * (1.0f - h[r] * h[r]);
       store_rt<RT>(hT + (kg * 4 + c) * LD + eg * RT, o);
     }
   }
