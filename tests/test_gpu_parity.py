@@ -563,6 +563,29 @@ def test_ppo_7b_first_steps():
     assert rel_err(gm, m) <= TOL and rel_err(gp, P) <= TOL
 
 
+@pytest.mark.parametrize("n", [60, 1000, 4999, 8192])
+def test_ppo_7b_single_step_partitions(n):
+    """One step over n samples of the 7B networks.  The update gives each CTA
+    ceil(n / NC) consecutive samples (NC = 76 per network on 152 SMs, fewer
+    for small n), in slices of up to 64 whose tiles stop at the valid rows
+    rounded up to 8: n = 60 (8-sample shares, the last one short), 1000
+    (14-sample shares, the last CTAs empty), 4999 (a 2-sample second slice)
+    and 8192 (the bench's 64 + 44)."""
+    wl = W.make_7b(n_envs=512)
+    params, buf, adv, ret = _ppo_inputs(wl, 64, seed=4)
+    D = wl.net.obs_dim
+    sub = {"obs": buf["obs"].reshape(-1, D)[:n].contiguous(), "act": buf["act"].reshape(-1)[:n].contiguous(),
+           "logp": buf["logp"].reshape(-1)[:n].contiguous()}
+    a_, r_ = adv.reshape(-1)[:n].contiguous(), ret.reshape(-1)[:n].contiguous()
+    ppo = W.PPOSpec(epochs=1, minibatch=n)
+    gp, gm, gv, gs = _run_ppo(wl, ppo, params, sub, a_, r_)
+    P, m, v, t, st = _oracle_ppo(wl, ppo, params, sub, a_, r_)
+    assert t == 1 and gs[7] == 1
+    assert rel_err(gm, m) <= TOL and rel_err(gp, P) <= TOL
+    for k in (1, 2, 6):   # value loss, entropy, grad norm
+        assert abs(gs[k] - st[k]) <= TOL * max(abs(st[k]), 1e-3), (k, gs[k], st[k])
+
+
 # ------------------------------------------------------------------ bf16 PPO
 @pytest.mark.parametrize("preset,E,T", [("72b", 64, 64), ("stress", 32, 64)])
 def test_ppo_bf16_single_step(preset, E, T):
