@@ -247,6 +247,22 @@ typedef struct pe_rule {
 pe_status pe_rollout_rule(pe_env* env, const pe_rule* rule, int32_t horizon, uint32_t iteration,
                           float lambda, int32_t obs_bf16, const pe_rollout_buf* buf, void* stream);
 
+/* Teacher-forced rollout (replay of a given action sequence): env e takes
+ * action actions[t][e] at step t and steps exactly as in pe_rollout (actuator,
+ * Eqs. 1-3, reward, episode ends and resets drawn from `iteration`), with no
+ * network: replaying the actions a pe_rollout call took, from the same env
+ * state, reproduces its observations, rewards, done flags and counters.  It
+ * serves recorded controllers, constant schedules and parity checks in which
+ * one flipped sample must not change the rest of a trajectory.
+ *  actions: [horizon][E] uint8 device memory, each in [0, A); checked on the
+ *  device first (the call waits for the check; nothing runs on a bad value).
+ *  buf: as pe_rollout_rule (act receives a copy of the actions; obs/obs_last
+ *  optional, fp32 or bf16 by obs_bf16; logp, value, last_value untouched).
+ * Errors: PE_EINVAL (null argument or field, horizon < 1, an action outside
+ * [0, A), unsupported env), PE_ECUDA. */
+pe_status pe_rollout_replay(pe_env* env, const uint8_t* actions, int32_t horizon, uint32_t iteration,
+                            float lambda, int32_t obs_bf16, const pe_rollout_buf* buf, void* stream);
+
 /* Dual ascent on the Lagrange multiplier of the Eq. 6 reward (Eq. 7,
  * Sec. 4.5; the G3 design of Sec. 4.2), from a rollout's violation counts:
  *   v = sum_e viol[e][w] / (n_envs * steps)   (w: 1 = instantaneous, 60 = 30 s window)

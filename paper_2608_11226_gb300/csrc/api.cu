@@ -95,8 +95,11 @@ struct RuleArgs {
   int32_t T, obs_bf16;
   uint32_t it;
   float lambda;
+  const uint8_t* forced;
 };
+constexpr int32_t kRuleReplay = 4;
 pe_status rule_rollout(const EnvDev& env, const RuleArgs& r, const pe_rollout_buf& buf, cudaStream_t st);
+pe_status replay_check(const uint8_t* act, int64_t n, int A, int32_t* flag, cudaStream_t st);
 pe_status env_set_offsets(const EnvDev& env, const int32_t* offsets, int32_t* flag, cudaStream_t st);
 pe_status dual_ascent(const int32_t* viol, int E, int64_t steps, int window, int additive, float target,
                       float eta, float lo, float hi, float* lambda, float* rate, cudaStream_t st);
@@ -453,8 +456,23 @@ pe_status pe_rollout_rule(pe_env* env, const pe_rule* rule, int32_t horizon, uin
   if (!buf->act || !buf->reward || !buf->done || !buf->viol || !buf->tokens || !buf->excess || !buf->energy_q)
     return fail(PE_EINVAL, "null rollout buffer field");
   RuleArgs r{rule->kind, rule->hi_q, rule->lo_q, rule->drop30_q, rule->climb30_q, rule->climb10_q,
-             horizon, obs_bf16 ? 1 : 0, iteration, lambda};
+             horizon, obs_bf16 ? 1 : 0, iteration, lambda, nullptr};
   return rule_rollout(env->dev, r, *buf, reinterpret_cast<cudaStream_t>(stream));
+}
+
+pe_status pe_rollout_replay(pe_env* env, const uint8_t* actions, int32_t horizon, uint32_t iteration, float lambda,
+                            int32_t obs_bf16, const pe_rollout_buf* buf, void* stream) {
+  clear_error();
+  if (!env || !actions || !buf) return fail(PE_EINVAL, "null argument");
+  if (horizon < 1) return fail(PE_EINVAL, "horizon must be >= 1");
+  if ((int64_t)horizon * env->dev.E > (int64_t)INT32_MAX) return fail(PE_EINVAL, "horizon * n_envs too large");
+  if (!buf->act || !buf->reward || !buf->done || !buf->viol || !buf->tokens || !buf->excess || !buf->energy_q)
+    return fail(PE_EINVAL, "null rollout buffer field");
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  pe_status s = replay_check(actions, (int64_t)horizon * env->dev.E, env->dev.A, env->flag, st);
+  if (s != PE_OK) return s;
+  RuleArgs r{kRuleReplay, 0, 0, 0, 0, 0, horizon, obs_bf16 ? 1 : 0, iteration, lambda, actions};
+  return rule_rollout(env->dev, r, *buf, st);
 }
 
 pe_status pe_dual_ascent(const int32_t* viol, int32_t n_envs, int64_t steps, int32_t window, int32_t additive,

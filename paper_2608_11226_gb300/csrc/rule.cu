@@ -18,13 +18,18 @@ struct RuleArgs {
   int32_t T, obs_bf16;
   uint32_t it;
   float lambda;
+  const uint8_t* forced;  // [T][E] actions of a replay (kind kRuleReplay)
 };
+
+// a replay (teacher-forced rollout): env e takes action forced[t][e] at step t
+constexpr int32_t kRuleReplay = 4;
 
 // lower / raise move one level: G for the inc/dec actuator (actions 1 and 2;
 // the env keeps G in [g_min, g_max]), the level index otherwise (clamped)
 template <int C>
 __device__ __forceinline__ int rule_action(const EnvDev& env, RegAcc<C>& a, const RuleArgs& r, uint32_t e,
                                            uint32_t t) {
+  if (r.kind == kRuleReplay) return r.forced[(int64_t)t * env.E + e];
   const bool incdec = env.act_kind == PE_ACT_INCDEC;
   const int lvl = a.level();
   const int hold = incdec ? 0 : lvl;
@@ -112,6 +117,25 @@ __global__ void env_offsets_kernel(EnvDev env, const int32_t* __restrict__ offse
   a.fam() = fam;  // the env keeps its episode's trace family
   env_reset_at<C>(env, a, o);
   store_reg<C>(env, e, a);
+}
+
+// a replay's actions must lie in [0, A)
+__global__ void replay_check_kernel(const uint8_t* __restrict__ act, int64_t n, int A, int32_t* __restrict__ flag) {
+  int bad = 0;
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x)
+    bad |= act[i] >= A;
+  if (__any_sync(0xffffffffu, bad) && (threadIdx.x & 31) == 0) atomicOr(flag, 1);
+}
+
+pe_status replay_check(const uint8_t* act, int64_t n, int A, int32_t* flag, cudaStream_t st) {
+  PE_TRY_CUDA(cudaMemsetAsync(flag, 0, sizeof(int32_t), st));
+  replay_check_kernel<<<(int)std::min<int64_t>(ceil_div(n, 256), 4096), 256, 0, st>>>(act, n, A, flag);
+  PE_CHECK_LAUNCH("replay_check_kernel");
+  int32_t host = 0;
+  PE_TRY_CUDA(cudaMemcpyAsync(&host, flag, sizeof(int32_t), cudaMemcpyDeviceToHost, st));
+  PE_TRY_CUDA(cudaStreamSynchronize(st));
+  if (host) return fail(PE_EINVAL, "replay action outside [0, A)");
+  return PE_OK;
 }
 
 pe_status rule_rollout(const EnvDev& env, const RuleArgs& r, const pe_rollout_buf& buf, cudaStream_t st) {

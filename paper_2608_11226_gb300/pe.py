@@ -78,7 +78,7 @@ EXPORTS = (
     "pe_param_count", "pe_rollout_workspace_bytes", "pe_rollout", "pe_value_workspace_bytes",
     "pe_value", "pe_device_check", "pe_gae", "pe_ppo_workspace_bytes",
     "pe_ppo_update", "pe_fleet_workspace_bytes", "pe_fleet_windows", "pe_fleet_windows_noalloc",
-    "pe_fleet_stagger_workspace_bytes", "pe_fleet_stagger", "pe_env_set_offsets", "pe_rollout_rule",
+    "pe_fleet_stagger_workspace_bytes", "pe_fleet_stagger", "pe_env_set_offsets", "pe_rollout_rule", "pe_rollout_replay",
     "pe_dual_ascent",
     "pe_profile_enable",
     "pe_profile_read", "pe_profile_kind_name", "pe_last_error")
@@ -114,6 +114,7 @@ def lib():
             "pe_dual_ascent": (i32, [vp, i32, i64, i32, i32, C.c_float, C.c_float, C.c_float, C.c_float,
                                      vp, vp, vp]),
             "pe_rollout_rule": (i32, [vp, vp, i32, u32, C.c_float, i32, vp, vp]),
+            "pe_rollout_replay": (i32, [vp, vp, i32, u32, C.c_float, i32, vp, vp]),
             "pe_fleet_stagger": (i32, [vp, i32, i32, vp, i32, i32, i32, i32, vp, vp, vp, i64, vp]),
             "pe_fleet_windows": (i32, [vp, i32, i32, vp, i32, vp, i64, i32, vp, i32, i64, vp,
                                        vp, vp, i64, vp]),
@@ -281,6 +282,17 @@ def rollout_rule(env: Env, rule: W.RuleSpec, T: int, iteration: int, buf: Dict[s
     r = Rule(rule.kind, rule.hi_q, rule.lo_q, rule.drop30_q, rule.climb30_q, rule.climb10_q)
     _check(lib().pe_rollout_rule(env._h, C.byref(r), T, iteration, lam, int(obs_bf16), C.byref(rb),
                                  _stream(stream)))
+
+
+def rollout_replay(env: Env, actions: torch.Tensor, T: int, iteration: int, buf: Dict[str, torch.Tensor],
+                   lam: float = 1.0, stream=None):
+    """Teacher-forced rollout: env e takes actions[t][e] (uint8, device, [T][E]) at step t."""
+    if actions.dtype != torch.uint8 or actions.numel() != T * env.spec.n_envs or not actions.is_contiguous():
+        raise ValueError("actions must be a contiguous uint8 tensor of T x n_envs")
+    rb = _rollout_buf(buf)
+    obs_bf16 = buf["obs"] is not None and buf["obs"].dtype == torch.bfloat16
+    _check(lib().pe_rollout_replay(env._h, _ptr(actions), T, iteration, lam, int(obs_bf16), C.byref(rb),
+                                   _stream(stream)))
 
 
 def dual_ascent(viol: torch.Tensor, steps: int, lam: torch.Tensor, rate: Optional[torch.Tensor] = None,

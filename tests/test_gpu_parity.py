@@ -664,6 +664,82 @@ def test_rule_rollout_parity(preset, kind):
     env.close()
 
 
+@pytest.mark.parametrize("preset", ["tiny", "7b", "72b"])
+def test_replay_rollout_parity(preset):
+    """Teacher-forced rollouts (pe_rollout_replay) of seeded random actions,
+    two calls in a row crossing episode ends, against the oracle stepping
+    with the same forced actions: observations (bf16 after RNE for the 72B
+    env), done flags, violation counts, energy and per-step power bit-exact;
+    rewards, tokens and excess within 1e-5."""
+    E = 64
+    wl = {"tiny": W.make_tiny, "7b": W.make_7b, "72b": W.make_72b}[preset](n_envs=E)
+    spec, net = wl.env, wl.net
+    bf16 = preset == "72b"
+    params = W.init_params(net, seed=2, bias_scale=0.05)
+    env = pe.Env(spec, torch.from_numpy(wl.trace), torch.from_numpy(wl.phase))
+    oenv = O.OracleEnv(spec, wl.trace, wl.phase, range(E))
+    rng = np.random.default_rng(9)
+    for it, T in ((0, 300), (1, 450)):
+        acts = rng.integers(0, spec.n_actions, (T, E)).astype(np.uint8)
+        buf = pe.alloc_rule_rollout(spec, T, obs=True, obs_bf16=bf16)
+        pe.rollout_replay(env, torch.from_numpy(acts).cuda(), T, it, buf, lam=0.5)
+        torch.cuda.synchronize()
+        ref = oenv.rollout(params, net.hidden, bf16, T, it, lam=0.5, forced=acts)
+        want_obs, want_last = ref["obs"], ref["obs_last"]
+        if bf16:
+            want_obs = torch.from_numpy(want_obs).to(torch.bfloat16).float().numpy()
+            want_last = torch.from_numpy(want_last).to(torch.bfloat16).float().numpy()
+        assert np.array_equal(cpu(buf["act"]), acts)
+        assert np.array_equal(cpu(buf["obs"].float()), want_obs)
+        assert np.array_equal(cpu(buf["obs_last"].float()), want_last)
+        assert np.array_equal(cpu(buf["done"]), ref["done"])
+        assert ref["done"].any() or it == 0
+        assert np.array_equal(cpu(buf["viol"]), ref["viol"])
+        assert np.array_equal(cpu(buf["energy_q"]), ref["energy_q"])
+        assert np.array_equal(cpu(buf["samples"]), ref["samples"])
+        assert np.array_equal(cpu(buf["q"]), ref["q"])
+        assert rel_err(cpu(buf["reward"]), ref["reward"]) <= TOL
+        assert rel_err(cpu(buf["tokens"]), ref["tokens"]) <= TOL
+        assert rel_err(cpu(buf["excess"]), ref["excess"]) <= TOL
+    env.close()
+
+
+def test_replay_reproduces_policy_rollout():
+    """Replaying the actions a 7B policy rollout took, from the same saved env
+    state, reproduces that rollout's observations, rewards, done flags,
+    counters and final state bit for bit (the same env step on both paths)."""
+    wl = W.make_7b(n_envs=256)
+    spec, net = wl.env, wl.net
+    T = 600
+    env = pe.Env(spec, torch.from_numpy(wl.trace), torch.from_numpy(wl.phase))
+    snap = env.save()
+    p_dev = torch.from_numpy(W.init_params(net, seed=3, bias_scale=0.05)).cuda()
+    buf = pe.alloc_rollout(spec, net, T)
+    pe.rollout(env, net, p_dev, T, 4, buf, lam=0.7)
+    after = env.save()
+    env.load(snap)
+    rb = pe.alloc_rule_rollout(spec, T, obs=True)
+    pe.rollout_replay(env, buf["act"].contiguous(), T, 4, rb, lam=0.7)
+    torch.cuda.synchronize()
+    for k in ("obs", "obs_last", "act", "reward", "done", "viol", "tokens", "excess", "energy_q", "samples", "q"):
+        assert torch.equal(buf[k], rb[k]), k
+    assert env.save() == after
+    env.close()
+
+
+def test_replay_rejects_bad_actions():
+    wl = W.make_tiny(n_envs=8)
+    spec = wl.env
+    env = pe.Env(spec, torch.from_numpy(wl.trace), torch.from_numpy(wl.phase))
+    acts = torch.zeros((5, 8), dtype=torch.uint8, device="cuda")
+    acts[3, 2] = spec.n_actions
+    buf = pe.alloc_rule_rollout(spec, 5)
+    with pytest.raises(pe.PEError) as e:
+        pe.rollout_replay(env, acts, 5, 0, buf)
+    assert e.value.status == pe.PE_EINVAL and "outside" in str(e.value)
+    env.close()
+
+
 def test_rule_rollout_full_size_sampled():
     """The 72B env at full size (65,536 envs x 1,024 steps) under the
     hysteresis rule from the random initial offsets; the oracle replays a
