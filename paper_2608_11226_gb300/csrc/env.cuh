@@ -256,6 +256,78 @@ __device__ __forceinline__ float feature(const EnvDev& env, Acc& a, const Fam& f
   return c < fm.C ? ratio_i((int64_t)fm.C * a.sl(c), kWLong * B) : 0.0f;
 }
 
+// All D features of an Eq. 5 observation (OCC32 / OCC64) for an env whose
+// samples are recomputed from the trace (RegAcc): the actuated samples the
+// features read -- positions pos-1 .. pos-NB and pos-11, every channel -- are
+// fetched once, with all their loads independent, instead of per feature.
+// The arithmetic is feature()'s, so the results are the same bits.
+template <int C, int OBS, int D>
+__device__ __forceinline__ void features_eq5(const EnvDev& env, RegAcc<C>& a, const Fam& fm, float (&o)[D]) {
+  static_assert(OBS == PE_OBS_OCC32 || OBS == PE_OBS_OCC64, "Eq. 5 observations");
+  constexpr int NB = OBS == PE_OBS_OCC32 ? 4 : 12;  // recent samples per channel
+  constexpr int NP = NB > 10 ? NB : NB + 1;          // back positions read, pos-11 included
+  const int p0 = a.pos() - 1;
+  uint8_t lv[NP], ph[NP];
+  float x[C][NP];
+#pragma unroll
+  for (int i = 0; i < NP; ++i) {
+    const int pp = p0 - (i < NB ? i : 10);
+    lv[i] = a.level_at(pp);
+    ph[i] = __ldg(fm.phase + pp);
+#pragma unroll
+    for (int c = 0; c < C; ++c) x[c][i] = __ldg(fm.trace + (int64_t)c * fm.L + pp);
+  }
+  int32_t q[C][NP];
+#pragma unroll
+  for (int i = 0; i < NP; ++i)
+#pragma unroll
+    for (int c = 0; c < C; ++c) q[c][i] = quant64(x[c][i], actuator_scale(env, lv[i], c, ph[i]));
+  const int i10 = NB > 10 ? 10 : NB;
+  int32_t Q0 = 0, Q10 = 0;
+#pragma unroll
+  for (int c = 0; c < C; ++c) {
+    Q0 += q[c][0];
+    Q10 += q[c][i10];
+  }
+  const int64_t B = fm.B;
+  int64_t S20 = 0, S60 = 0;
+#pragma unroll
+  for (int c = 0; c < C; ++c) {
+    S20 += a.ss(c);
+    S60 += a.sl(c);
+  }
+  o[0] = ratio_i(Q0, B);
+  o[1] = ratio_i(S20, kWShort * B);
+  o[2] = ratio_i(S60, kWLong * B);
+  o[3] = ratio_i(kWLong * B - S60, kWLong * B);
+  o[4] = ratio_i((int64_t)Q0 - Q10, B);
+  o[5] = ratio_i(a.level() + 1, env.n_levels);
+  o[6] = ratio_i(a.prev() + 1, env.n_levels);
+  o[7] = fminf(env.cadence ? ratio_i(env.ns[a.level()], 40) : ratio_i(a.til(), 40), 1.0f);
+  if (OBS == PE_OBS_OCC32) {
+#pragma unroll
+    for (int f = 8; f < 24; ++f) {
+      const int c = (f - 8) >> 2, i = (f - 8) & 3;
+      o[f] = c < fm.C ? ratio_i((int64_t)fm.C * q[c][3 - i], B) : 0.0f;
+    }
+#pragma unroll
+    for (int c = 0; c < 4; ++c) o[24 + c] = c < fm.C ? ratio_i((int64_t)fm.C * a.sl(c), kWLong * B) : 0.0f;
+#pragma unroll
+    for (int f = 28; f < D; ++f) o[f] = 0.0f;
+  } else {
+#pragma unroll
+    for (int f = 8; f < 56; ++f) {
+      const int c = (f - 8) / 12, i = (f - 8) % 12;
+      o[f] = c < fm.C ? ratio_i((int64_t)fm.C * q[c][11 - i], B) : 0.0f;
+    }
+#pragma unroll
+    for (int c = 0; c < 4; ++c) {
+      o[56 + c] = c < fm.C ? ratio_i((int64_t)fm.C * a.ss(c), kWShort * B) : 0.0f;
+      o[60 + c] = c < fm.C ? ratio_i((int64_t)fm.C * a.sl(c), kWLong * B) : 0.0f;
+    }
+  }
+}
+
 template <int C, int OBS, class Acc>
 __device__ __forceinline__ float feature(const EnvDev& env, Acc& a, int f) {
   return feature<C, OBS>(env, a, fam_of(env, a.fam()), f);

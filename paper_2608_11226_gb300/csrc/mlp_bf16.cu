@@ -635,12 +635,13 @@ __global__ void __launch_bounds__(128) env_actobs_kernel(EnvDev env, ActArgs a, 
                            ? reinterpret_cast<__nv_bfloat16*>(buf.obs) + ((int64_t)(a.t + 1) * env.E + e) * D
                            : reinterpret_cast<__nv_bfloat16*>(buf.obs_last) + (int64_t)e * D;
   const Fam fm = fam_of(env, acc.fam());
-#pragma unroll 1
+  float o[D];
+  features_eq5<C, OBS, D>(env, acc, fm, o);
+#pragma unroll
   for (int f0 = 0; f0 < D; f0 += 8) {
     uint32_t p[4];
 #pragma unroll
-    for (int i = 0; i < 4; ++i)
-      p[i] = tc::pack_bf16(feature<C, OBS>(env, acc, fm, f0 + 2 * i), feature<C, OBS>(env, acc, fm, f0 + 2 * i + 1));
+    for (int i = 0; i < 4; ++i) p[i] = tc::pack_bf16(o[f0 + 2 * i], o[f0 + 2 * i + 1]);
     *reinterpret_cast<uint4*>(dst + f0) = make_uint4(p[0], p[1], p[2], p[3]);
   }
   store_reg<C>(env, e, acc);

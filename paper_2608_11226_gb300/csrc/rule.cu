@@ -53,6 +53,20 @@ __device__ __forceinline__ int rule_action(const EnvDev& env, RegAcc<C>& a, cons
 template <int C, int OBS, int D>
 __device__ __forceinline__ void write_obs(const EnvDev& env, RegAcc<C>& a, void* dst, int bf16) {
   const Fam fm = fam_of(env, a.fam());
+  if constexpr (OBS == PE_OBS_OCC32 || OBS == PE_OBS_OCC64) {
+    float v[D];
+    features_eq5<C, OBS, D>(env, a, fm, v);
+    if (bf16) {
+      __nv_bfloat16* o = reinterpret_cast<__nv_bfloat16*>(dst);
+#pragma unroll
+      for (int f = 0; f < D; ++f) o[f] = __float2bfloat16_rn(v[f]);
+    } else {
+      float* o = reinterpret_cast<float*>(dst);
+#pragma unroll
+      for (int f = 0; f < D; ++f) o[f] = v[f];
+    }
+    return;
+  }
   if (bf16) {
     __nv_bfloat16* o = reinterpret_cast<__nv_bfloat16*>(dst);
 #pragma unroll 1
