@@ -23,6 +23,7 @@
 #include <cstddef>
 
 #include "mlp_f32.cuh"
+#include "tc.cuh"
 
 namespace pe {
 
@@ -282,6 +283,7 @@ struct PpoSmem {
   float lpo[kPpoS], advn[kPpoS], ret[kPpoS];
   int32_t act[kPpoS], valid[kPpoS];
   float stat[kPpoS / 32][8];
+  uint64_t bar_w;  // mbarrier of the weight-image bulk copy (one phase per minibatch step)
 };
 
 struct PpoArgs {
@@ -300,6 +302,8 @@ struct PpoArgs {
   float* partial;       // [NC][P]
   float* stat_partial;  // [2*NC][8]
   float* grad_out;      // [P] reduced gradient (persistent kernel)
+  int32_t* err;  // set when a bounded wait gives up (reported as stats[7] = -1)
+  uint32_t wphase;  // parity of this step's weight-image mbarrier phase
   int NC;       // CTAs per network
   int per_cta;  // minibatch samples per CTA, ceil(cnt / NC): CTA c takes [c * per_cta, (c + 1) * per_cta)
   int64_t P, PS;  // parameters; row stride of the partial-sum matrix
@@ -401,26 +405,25 @@ __device__ __forceinline__ void ppo_role(PpoSmem<D, H, A>& s, const PpoArgs& g, 
   const int c0 = c * g.per_cta, c1 = min(c0 + g.per_cta, g.cnt);
   // the first slice's gather overlaps the weight loads
   if (c0 < c1) gather(c0, min(S, c1 - c0));
-  // the role's weight image, read through L2 (not the non-coherent L1 path):
-  // inside the persistent update other CTAs rewrite it between minibatches.
-  // Four float4 loads per thread are in flight before they are stored.
+  // the role's weight image, one bulk copy into shared memory completed on
+  // an mbarrier (its bytes all in flight at once).  Inside the persistent
+  // update other CTAs rewrite the image between minibatches with ordinary
+  // stores, made visible to this CTA by the grid barrier; the proxy fences
+  // order those writes, and this CTA's earlier reads of the weights, before
+  // the copy.  Every thread waits, bounded, before the first slice.
   {
     using I = RoleImage<D, H, A>;
     using Sm = PpoSmem<D, H, A>;
     static_assert(offsetof(Sm, b3) == sizeof(float) * (size_t)I::B3, "image matches shared memory");
-    const float4* src = reinterpret_cast<const float4*>(g.img + (POL ? 0 : I::SIZE));
-    float4* dst = reinterpret_cast<float4*>(s.w1t);
-    constexpr int N4 = (int)(I::SIZE / 4), U = 4;
-    for (int i0 = tid; i0 < N4; i0 += U * kPpoNT) {
-      float4 v[U];
-#pragma unroll
-      for (int u = 0; u < U; ++u)
-        if (i0 + u * kPpoNT < N4) v[u] = __ldcg(src + i0 + u * kPpoNT);
-#pragma unroll
-      for (int u = 0; u < U; ++u)
-        if (i0 + u * kPpoNT < N4) dst[i0 + u * kPpoNT] = v[u];
+    static_assert((I::SIZE * sizeof(float)) % 16 == 0, "bulk copy size");
+    if (tid == 0) {
+      asm volatile("fence.proxy.async.global;" ::: "memory");
+      tc::fence_async_smem();
+      tc::mbar_expect_tx(&s.bar_w, (uint32_t)(I::SIZE * sizeof(float)));
+      tc::bulk_g2s(s.w1t, g.img + (POL ? 0 : I::SIZE), (uint32_t)(I::SIZE * sizeof(float)), &s.bar_w);
     }
   }
+  if (!tc::mbar_wait(&s.bar_w, g.wphase)) atomicExch(g.err, 1);
   // weight-gradient tiles live in registers only during their phase; each
   // slice adds them into the CTA's shared-memory accumulators gw2 / gw1
   int nsl = 0;
@@ -632,6 +635,11 @@ template <int D, int H, int A>
 __global__ void __launch_bounds__(kPpoNT) ppo_grad_kernel(PpoArgs g) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   PpoSmem<D, H, A>& s = *reinterpret_cast<PpoSmem<D, H, A>*>(smem_raw);
+  if (threadIdx.x == 0) {
+    tc::mbar_init(&s.bar_w, 1);
+    tc::fence_mbar_init();
+  }
+  __syncthreads();
   if ((int)blockIdx.x < g.NC)
     ppo_role<D, H, A, true>(s, g, blockIdx.x);
   else
@@ -736,6 +744,11 @@ __global__ void __launch_bounds__(kPpoNT, 1) ppo_persistent_kernel(PpoLoop L) {
   const int64_t PS = L.g.PS;
   const int64_t per = ((P + gridDim.x - 1) / gridDim.x + 3) / 4 * 4;
   const int64_t p0 = (int64_t)blockIdx.x * per, p1 = p0 + per < P ? p0 + per : P;
+  if (tid == 0) {
+    tc::mbar_init(&s.bar_w, 1);
+    tc::fence_mbar_init();
+  }
+  __syncthreads();
   int step = 0;
   for (int ep = 0; ep < L.epochs; ++ep) {
     for (int mb = 0; mb < L.nmb; ++mb, ++step) {
@@ -747,6 +760,7 @@ __global__ void __launch_bounds__(kPpoNT, 1) ppo_persistent_kernel(PpoLoop L) {
       g.cnt = cnt;
       g.inv_cnt = 1.0f / (float)cnt;
       g.per_cta = (cnt + NC - 1) / NC;
+      g.wphase = (uint32_t)(step & 1);
       g.advstat = L.advstat + (int64_t)ep * L.nmb + mb;
       // phase 1: gradient partials of this CTA's role and samples
       if ((int)blockIdx.x < NC)
@@ -1091,6 +1105,8 @@ static pe_status ppo_run(const pe_net& net, float* params, float* m, float* v, i
     L.g.stat_partial = stat_partial;
     L.g.grad_out = grad;
     L.g.NC = nc;
+    L.g.err = bar_err;
+    L.g.wphase = 0;
     L.g.P = pl.P;
     L.g.PS = pl.PS;
     L.advstat = advstat;
@@ -1143,6 +1159,8 @@ static pe_status ppo_run(const pe_net& net, float* params, float* m, float* v, i
         g.stat_partial = stat_partial;
         g.NC = ncf;
         g.per_cta = (cnt + ncf - 1) / ncf;
+        g.err = bar_err;
+        g.wphase = 0;  // a fresh mbarrier in every launch
         g.P = pl.P;
         g.PS = pl.PS;
         g.advstat = advstat + (int64_t)ep * pl.nmb + mb;
