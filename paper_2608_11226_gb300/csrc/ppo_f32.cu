@@ -181,86 +181,61 @@ __device__ __forceinline__ void dense_bwd_wt(const float* __restrict__ inT, cons
   }
 }
 
-// acc[m][n] += sum_s aT[m][s] bT[n][s].  Each thread owns 4x4 tiles whose rows
-// and columns are interleaved (m = mg + i*M/4, n = ng + j*N/4); a warp covers
-// WM x WN (mg, ng) pairs, so one float4 load of the warp touches WM (or WN)
-// distinct rows in distinct shared-memory bank groups: one wavefront each.
+// dst[m][n] (+)= sum_s aT[m][s] bT[n][s] (weight gradients).  Each thread owns
+// 4x4 tiles whose rows and columns are interleaved (m = mg + i*M/4,
+// n = ng + j*N/4); a warp covers WM x WN (mg, ng) pairs, so one float4 load of
+// the warp touches WM (or WN) distinct rows in distinct shared-memory bank
+// groups: one wavefront each.
 template <int M, int N, int NT>
 struct WGradAcc {
   static constexpr int MG = M / 4, NG = N / 4;
   static constexpr int WN = NG < 4 ? NG : 4, WM = 32 / WN;
   static constexpr int TM = (MG + WM - 1) / WM, TN = NG / WN;
   static constexpr int NWARP = NT / 32, WT = TM * TN, PER = (WT + NWARP - 1) / NWARP;
-  float acc[PER][4][4];
   __device__ __forceinline__ bool job(int q, int& mg, int& ng) const {
     const int wt = (int)(threadIdx.x >> 5) + q * NWARP, lane = threadIdx.x & 31;
     mg = (wt / TN) * WM + lane / WN;
     ng = (wt % TN) * WN + lane % WN;
     return wt < WT && mg < MG;
   }
-  __device__ __forceinline__ void zero() {
-#pragma unroll
-    for (int q = 0; q < PER; ++q)
+  // dst (+)= sum_s aT[m][s] bT[n][s] over s < SV, one 4x4 tile at a time (16
+  // packed accumulators live), even and odd samples in the two lanes of a
+  // packed two-lane FMA and added at the end; rows of dst ld floats apart
+  template <int S, int LD>
+  __device__ __forceinline__ void accumulate(const float* __restrict__ aT, const float* __restrict__ bT, int SV,
+                                             float* dst, int ld, bool first) const {
+#pragma unroll 1
+    for (int q = 0; q < PER; ++q) {
+      int mg, ng;
+      if (!job(q, mg, ng)) continue;
+      float2 v2[4][4];
 #pragma unroll
       for (int i = 0; i < 4; ++i)
 #pragma unroll
-        for (int j = 0; j < 4; ++j) acc[q][i][j] = 0.0f;
-  }
-  // over samples s < SV (a multiple of 4, at most S)
-  template <int S, int LD>
-  __device__ __forceinline__ void add(const float* __restrict__ aT, const float* __restrict__ bT, int SV) {
-#pragma unroll
-    for (int q = 0; q < PER; ++q) {
-      int mg, ng;
-      if (job(q, mg, ng)) {
+        for (int j = 0; j < 4; ++j) v2[i][j] = make_float2(0.0f, 0.0f);
 #pragma unroll 2
-        for (int s = 0; s < SV; s += 4) {
-          float4 a[4], b[4];
+      for (int s = 0; s < SV; s += 4) {
+        float4 a[4], b[4];
 #pragma unroll
-          for (int i = 0; i < 4; ++i) a[i] = *reinterpret_cast<const float4*>(aT + (mg + i * MG) * LD + s);
+        for (int i = 0; i < 4; ++i) a[i] = *reinterpret_cast<const float4*>(aT + (mg + i * MG) * LD + s);
 #pragma unroll
-          for (int j = 0; j < 4; ++j) b[j] = *reinterpret_cast<const float4*>(bT + (ng + j * NG) * LD + s);
-#pragma unroll
-          for (int i = 0; i < 4; ++i)
-#pragma unroll
-            for (int j = 0; j < 4; ++j) {
-              float v = acc[q][i][j];
-              v = fmaf(a[i].x, b[j].x, v);
-              v = fmaf(a[i].y, b[j].y, v);
-              v = fmaf(a[i].z, b[j].z, v);
-              v = fmaf(a[i].w, b[j].w, v);
-              acc[q][i][j] = v;
-            }
-        }
-      }
-    }
-  }
-  // dst (+)= acc in shared memory, rows ld floats apart (the first slice stores)
-  __device__ __forceinline__ void add_to(float* dst, int ld, bool first) const {
-#pragma unroll
-    for (int q = 0; q < PER; ++q) {
-      int mg, ng;
-      if (job(q, mg, ng)) {
+        for (int j = 0; j < 4; ++j) b[j] = *reinterpret_cast<const float4*>(bT + (ng + j * NG) * LD + s);
 #pragma unroll
         for (int i = 0; i < 4; ++i)
 #pragma unroll
           for (int j = 0; j < 4; ++j) {
-            float* d = dst + (mg + i * MG) * ld + ng + j * NG;
-            *d = first ? acc[q][i][j] : *d + acc[q][i][j];
+            v2[i][j] = __ffma2_rn(make_float2(a[i].x, a[i].y), make_float2(b[j].x, b[j].y), v2[i][j]);
+            v2[i][j] = __ffma2_rn(make_float2(a[i].z, a[i].w), make_float2(b[j].z, b[j].w), v2[i][j]);
           }
       }
-    }
-  }
-  __device__ __forceinline__ void store(float* __restrict__ dst) const {
 #pragma unroll
-    for (int q = 0; q < PER; ++q) {
-      int mg, ng;
-      if (job(q, mg, ng)) {
+      for (int i = 0; i < 4; ++i)
 #pragma unroll
-        for (int i = 0; i < 4; ++i)
-#pragma unroll
-          for (int j = 0; j < 4; ++j) dst[(int64_t)(mg + i * MG) * N + ng + j * NG] = acc[q][i][j];
-      }
+        for (int j = 0; j < 4; ++j) {
+          float* d = dst + (mg + i * MG) * ld + ng + j * NG;
+          const float v = v2[i][j].x + v2[i][j].y;
+          *d = first ? v : *d + v;
+        }
     }
   }
 };
@@ -553,9 +528,7 @@ __device__ __forceinline__ void ppo_role(PpoSmem<D, H, A>& s, const PpoArgs& g, 
     // layer-2 weight gradient
     {
       WGradAcc<H, H, kPpoNT> g2;
-      g2.zero();
-      g2.template add<S, LD>(s.h2t, s.h1t, SV);
-      g2.add_to(s.gw2, w2t_ld<H>(), nsl == 0);
+      g2.template accumulate<S, LD>(s.h2t, s.h1t, SV, s.gw2, w2t_ld<H>(), nsl == 0);
     }
     __syncthreads();
     // back into layer 1 (in place over h1)
@@ -564,9 +537,7 @@ __device__ __forceinline__ void ppo_role(PpoSmem<D, H, A>& s, const PpoArgs& g, 
     // layer-1 weight and bias gradients (the bias by the warps the tiles leave idle)
     {
       WGradAcc<H, D, kPpoNT> g1;
-      g1.zero();
-      g1.template add<S, LD>(s.h1t, s.xt, SV);
-      g1.add_to(s.gw1, D, nsl == 0);
+      g1.template accumulate<S, LD>(s.h1t, s.xt, SV, s.gw1, D, nsl == 0);
     }
     if (tid >= kPpoNT - H) {
       const int n = tid - (kPpoNT - H), lane = tid & 31;
