@@ -211,6 +211,17 @@ def test_fleet_stagger_bit_exact(L, H, w, stride):
     assert np.array_equal(g_off, o_off) and np.array_equal(g_pk, o_pk), (g_off, o_off, g_pk, o_pk)
 
 
+def test_fleet_stagger_twelve_jobs_bit_exact():
+    """Twelve jobs over the sixteen traces (more than the eight streams of one
+    composed load): every stage composes the partial-fleet row with one
+    candidate job, so the stage count, not the stream count, grows."""
+    fw = W.make_fleet(n_compositions=1, length=900, seed=5)
+    job = (np.arange(fw.traces.shape[0]) % 12).astype(np.int32)
+    g_off, g_pk = _stagger_gpu(fw.traces, job, 12, 700, 60, 3)
+    o_off, o_pk = O.fleet_stagger(fw.traces, job, 12, 700, 60, 3)
+    assert np.array_equal(g_off, o_off) and np.array_equal(g_pk, o_pk), (g_off, o_off, g_pk, o_pk)
+
+
 def test_fleet_stagger_full_size_sampled():
     """The 16-GPU, 380,000-sample fleet with every offset a candidate: each
     stage's peak is re-evaluated by the oracle at the chosen offsets, and a
