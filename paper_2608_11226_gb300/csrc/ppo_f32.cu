@@ -376,10 +376,6 @@ __device__ __forceinline__ void ppo_role(PpoSmem<D, H, A>& s, const PpoArgs& g, 
       }
     }
   };
-  // this CTA's samples [c0, c1) of the minibatch, in slices of S
-  const int c0 = c * g.per_cta, c1 = min(c0 + g.per_cta, g.cnt);
-  // the first slice's gather overlaps the weight loads
-  if (c0 < c1) gather(c0, min(S, c1 - c0));
   // the role's weight image, one bulk copy into shared memory completed on
   // an mbarrier (its bytes all in flight at once).  Inside the persistent
   // update other CTAs rewrite the image between minibatches with ordinary
@@ -398,6 +394,10 @@ __device__ __forceinline__ void ppo_role(PpoSmem<D, H, A>& s, const PpoArgs& g, 
       tc::bulk_g2s(s.w1t, g.img + (POL ? 0 : I::SIZE), (uint32_t)(I::SIZE * sizeof(float)), &s.bar_w);
     }
   }
+  // this CTA's samples [c0, c1) of the minibatch, in slices of S
+  const int c0 = c * g.per_cta, c1 = min(c0 + g.per_cta, g.cnt);
+  // the first slice's gather overlaps the weight copy, issued above
+  if (c0 < c1) gather(c0, min(S, c1 - c0));
   if (!tc::mbar_wait(&s.bar_w, g.wphase)) atomicExch(g.err, 1);
   // weight-gradient tiles live in registers only during their phase; each
   // slice adds them into the CTA's shared-memory accumulators gw2 / gw1
