@@ -263,6 +263,21 @@ pe_status pe_rollout_rule(pe_env* env, const pe_rule* rule, int32_t horizon, uin
 pe_status pe_rollout_replay(pe_env* env, const uint8_t* actions, int32_t horizon, uint32_t iteration,
                             float lambda, int32_t obs_bf16, const pe_rollout_buf* buf, void* stream);
 
+/* Self-test of the library's bounded waits (failure detection without a GPU
+ * fault): every spin-wait in the kernels gives up after a clock64 budget,
+ * records an error word and returns, so the context stays usable.  This call
+ * runs the same waits with budget limit_cycles (in SM clock cycles):
+ *  mode 0: the persistent update's grid barrier, 2 CTAs, one of which never
+ *          arrives -> the wait runs out -> PE_ETIMEOUT;
+ *  mode 1: the same barrier with both CTAs arriving -> PE_OK;
+ *  mode 2: an mbarrier wait (as in the tensor-core kernels) that nothing
+ *          completes -> PE_ETIMEOUT.
+ *  workspace: >= 16 bytes of device memory.  The call waits for the result.
+ * Errors: PE_EINVAL (mode outside [0, 2], limit_cycles outside [1e3, 8e9],
+ * null workspace), PE_ETIMEOUT (a wait gave up, as modes 0 and 2 intend),
+ * PE_ECUDA. */
+pe_status pe_wait_selftest(int32_t mode, int64_t limit_cycles, void* workspace, void* stream);
+
 /* Dual ascent on the Lagrange multiplier of the Eq. 6 reward (Eq. 7,
  * Sec. 4.5; the G3 design of Sec. 4.2), from a rollout's violation counts:
  *   v = sum_e viol[e][w] / (n_envs * steps)   (w: 1 = instantaneous, 60 = 30 s window)

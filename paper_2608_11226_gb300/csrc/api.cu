@@ -100,6 +100,7 @@ struct RuleArgs {
 constexpr int32_t kRuleReplay = 4;
 pe_status rule_rollout(const EnvDev& env, const RuleArgs& r, const pe_rollout_buf& buf, cudaStream_t st);
 pe_status replay_check(const uint8_t* act, int64_t n, int A, int32_t* flag, cudaStream_t st);
+pe_status wait_selftest(int mode, int64_t limit_cycles, void* ws, cudaStream_t st);
 pe_status env_set_offsets(const EnvDev& env, const int32_t* offsets, int32_t* flag, cudaStream_t st);
 pe_status dual_ascent(const int32_t* viol, int E, int64_t steps, int window, int additive, float target,
                       float eta, float lo, float hi, float* lambda, float* rate, cudaStream_t st);
@@ -458,6 +459,14 @@ pe_status pe_rollout_rule(pe_env* env, const pe_rule* rule, int32_t horizon, uin
   RuleArgs r{rule->kind, rule->hi_q, rule->lo_q, rule->drop30_q, rule->climb30_q, rule->climb10_q,
              horizon, obs_bf16 ? 1 : 0, iteration, lambda, nullptr};
   return rule_rollout(env->dev, r, *buf, reinterpret_cast<cudaStream_t>(stream));
+}
+
+pe_status pe_wait_selftest(int32_t mode, int64_t limit_cycles, void* workspace, void* stream) {
+  clear_error();
+  if (mode < 0 || mode > 2) return fail(PE_EINVAL, "mode must be 0, 1 or 2");
+  if (limit_cycles < 1000 || limit_cycles > 8000000000LL) return fail(PE_EINVAL, "limit_cycles outside [1e3, 8e9]");
+  if (!workspace) return fail(PE_EINVAL, "null workspace");
+  return wait_selftest(mode, limit_cycles, workspace, reinterpret_cast<cudaStream_t>(stream));
 }
 
 pe_status pe_rollout_replay(pe_env* env, const uint8_t* actions, int32_t horizon, uint32_t iteration, float lambda,

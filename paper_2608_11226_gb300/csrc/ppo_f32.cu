@@ -680,7 +680,7 @@ struct PpoLoop {
 // arrive at barrier k + 1 before all have arrived at k), so each CTA waits
 // for the counter to reach (k + 1) * G; the last arrival releases everyone
 // with its own atomic, and nothing is reset.  The wait is bounded.
-__device__ __forceinline__ bool grid_barrier(unsigned int* bar, int* s_ok) {
+__device__ __forceinline__ bool grid_barrier(unsigned int* bar, int* s_ok, long long limit = 4000000000LL) {
   __syncthreads();
   if (threadIdx.x == 0) {
     __threadfence();
@@ -690,7 +690,7 @@ __device__ __forceinline__ bool grid_barrier(unsigned int* bar, int* s_ok) {
     bool ok = true;
     const long long t0 = clock64();
     while ((int)(*vb - target) < 0) {
-      if (clock64() - t0 > 4000000000LL) {  // about 2 s at the maximum SM clock
+      if (clock64() - t0 > limit) {  // by default about 2 s at the maximum SM clock
         ok = false;
         break;
       }
@@ -701,6 +701,44 @@ __device__ __forceinline__ bool grid_barrier(unsigned int* bar, int* s_ok) {
   }
   __syncthreads();
   return *s_ok != 0;
+}
+
+// Self-test of the bounded waits (mode 0: the grid barrier with CTA 1 never
+// arriving; mode 1: the same barrier with every CTA arriving; mode 2: an
+// mbarrier nothing arrives at).  A wait that gives up sets *err.
+__global__ void wait_selftest_kernel(unsigned int* bar, int32_t* err, int mode, long long limit) {
+  __shared__ int s_ok;
+  __shared__ uint64_t mb;
+  if (mode == 2) {
+    if (threadIdx.x == 0) {
+      tc::mbar_init(&mb, 1);
+      tc::fence_mbar_init();
+    }
+    __syncthreads();
+    if (!tc::mbar_wait(&mb, 0, limit) && threadIdx.x == 0) atomicExch(err, 1);
+    return;
+  }
+  if (mode == 0 && blockIdx.x == 1) return;  // this CTA never reaches the barrier
+  if (!grid_barrier(bar, &s_ok, limit) && threadIdx.x == 0) atomicExch(err, 1);
+}
+
+pe_status wait_selftest(int mode, int64_t limit_cycles, void* ws, cudaStream_t st) {
+  unsigned int* bar = reinterpret_cast<unsigned int*>(ws);
+  int32_t* err = reinterpret_cast<int32_t*>(reinterpret_cast<char*>(ws) + 8);
+  PE_TRY_CUDA(cudaMemsetAsync(ws, 0, 16, st));
+  long long limit = (long long)limit_cycles;
+  if (mode == 2) {
+    wait_selftest_kernel<<<1, 32, 0, st>>>(bar, err, mode, limit);
+  } else {
+    void* args[] = {&bar, &err, &mode, &limit};
+    PE_TRY_CUDA(cudaLaunchCooperativeKernel((void*)wait_selftest_kernel, dim3(2), dim3(32), args, 0, st));
+  }
+  PE_CHECK_LAUNCH("wait_selftest_kernel");
+  int32_t host = 0;
+  PE_TRY_CUDA(cudaMemcpyAsync(&host, err, sizeof(int32_t), cudaMemcpyDeviceToHost, st));
+  PE_TRY_CUDA(cudaStreamSynchronize(st));
+  if (host) return fail(PE_ETIMEOUT, "bounded wait gave up (self-test mode %d)", mode);
+  return PE_OK;
 }
 
 template <int D, int H, int A>

@@ -78,7 +78,7 @@ EXPORTS = (
     "pe_param_count", "pe_rollout_workspace_bytes", "pe_rollout", "pe_value_workspace_bytes",
     "pe_value", "pe_device_check", "pe_gae", "pe_ppo_workspace_bytes",
     "pe_ppo_update", "pe_fleet_workspace_bytes", "pe_fleet_windows", "pe_fleet_windows_noalloc",
-    "pe_fleet_stagger_workspace_bytes", "pe_fleet_stagger", "pe_env_set_offsets", "pe_rollout_rule", "pe_rollout_replay",
+    "pe_fleet_stagger_workspace_bytes", "pe_fleet_stagger", "pe_env_set_offsets", "pe_rollout_rule", "pe_rollout_replay", "pe_wait_selftest",
     "pe_dual_ascent",
     "pe_profile_enable",
     "pe_profile_read", "pe_profile_kind_name", "pe_last_error")
@@ -115,6 +115,7 @@ def lib():
                                      vp, vp, vp]),
             "pe_rollout_rule": (i32, [vp, vp, i32, u32, C.c_float, i32, vp, vp]),
             "pe_rollout_replay": (i32, [vp, vp, i32, u32, C.c_float, i32, vp, vp]),
+            "pe_wait_selftest": (i32, [i32, C.c_int64, vp, vp]),
             "pe_fleet_stagger": (i32, [vp, i32, i32, vp, i32, i32, i32, i32, vp, vp, vp, i64, vp]),
             "pe_fleet_windows": (i32, [vp, i32, i32, vp, i32, vp, i64, i32, vp, i32, i64, vp,
                                        vp, vp, i64, vp]),
@@ -293,6 +294,12 @@ def rollout_replay(env: Env, actions: torch.Tensor, T: int, iteration: int, buf:
     obs_bf16 = buf["obs"] is not None and buf["obs"].dtype == torch.bfloat16
     _check(lib().pe_rollout_replay(env._h, _ptr(actions), T, iteration, lam, int(obs_bf16), C.byref(rb),
                                    _stream(stream)))
+
+
+def wait_selftest(mode: int, limit_cycles: int, workspace: torch.Tensor, stream=None):
+    """Run one of the library's bounded waits with a short budget (see pe.h);
+    raises PEError with PE_ETIMEOUT when the wait gives up."""
+    _check(lib().pe_wait_selftest(mode, int(limit_cycles), _ptr(workspace), _stream(stream)))
 
 
 def dual_ascent(viol: torch.Tensor, steps: int, lam: torch.Tensor, rate: Optional[torch.Tensor] = None,

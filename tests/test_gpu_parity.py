@@ -93,6 +93,28 @@ def test_gae_parity_vector_paths(T, E):
     assert rel_err(cpu(ret[:, ci]), rr) <= TOL
 
 
+def test_bounded_waits_give_up_and_leave_the_context_usable():
+    """Failure detection without a GPU fault: the grid barrier of the
+    persistent update with one CTA that never arrives, and an mbarrier that
+    nothing completes, both give up after their budget (about 0.1 s here)
+    and report PE_ETIMEOUT; the barrier with every CTA arriving passes; the
+    context stays usable for a real call afterwards."""
+    ws = torch.zeros(16, dtype=torch.uint8, device="cuda")
+    pe.wait_selftest(1, 200_000_000, ws)
+    for mode in (0, 2):
+        with pytest.raises(pe.PEError) as e:
+            pe.wait_selftest(mode, 200_000_000, ws)
+        assert e.value.status == pe.PE_ETIMEOUT
+    pe.device_check()
+    r = torch.ones(4, 8, device="cuda")
+    adv = torch.empty_like(r)
+    ret = torch.empty_like(r)
+    pe.gae(r, torch.zeros_like(r), torch.zeros(4, 8, dtype=torch.uint8, device="cuda"),
+           torch.zeros(8, device="cuda"), 0.5, 1.0, adv, ret)
+    torch.cuda.synchronize()
+    assert torch.allclose(adv[0], torch.full((8,), 1.875, device="cuda"))
+
+
 def test_gae_empty_is_noop():
     z = torch.empty(0, 5, device="cuda")
     pe.gae(z, z, z.to(torch.uint8), torch.empty(5, device="cuda"), 0.99, 0.95, z, z)
