@@ -494,6 +494,57 @@ def test_env_checkpoint_roundtrip():
         assert torch.equal(ba[k], bb[k]), k
 
 
+def test_training_resume_is_bit_exact():
+    """Checkpoint/resume of training: two Tiny iterations (rollout, GAE, PPO
+    update) run straight equal one iteration, a save of the env state,
+    parameters and Adam moments, a restore into fresh objects, and the second
+    iteration -- every buffer and statistic bit for bit (the draws are
+    counter-based on (seed, iteration, env, step), the reductions fixed-order)."""
+    wl = W.make_tiny(n_envs=64)
+    spec, net, T = wl.env, wl.net, 128
+    ppo = W.PPOSpec(epochs=2, minibatch=2048)
+    N = spec.n_envs * T
+
+    def iteration(env, p, m, v, adam_t, it):
+        buf = pe.alloc_rollout(spec, net, T)
+        pe.rollout(env, net, p, T, it, buf)
+        adv = torch.empty(T, spec.n_envs, device="cuda")
+        ret = torch.empty_like(adv)
+        pe.gae(buf["reward"], buf["value"], buf["done"], buf["last_value"], ppo.gamma, ppo.lam, adv, ret)
+        stats = torch.zeros(8, device="cuda")
+        ws = torch.empty(pe.ppo_workspace_bytes(net, ppo, N), dtype=torch.uint8, device="cuda")
+        pe.ppo_update(net, ppo, p, m, v, adam_t, buf["obs"], buf["act"], buf["logp"], adv, ret, stats, ws,
+                      seed=11, iteration=it)
+        torch.cuda.synchronize()
+        return buf, stats, adam_t + ppo.epochs * ((N + ppo.minibatch - 1) // ppo.minibatch)
+
+    def fresh():
+        env = pe.Env(spec, torch.from_numpy(wl.trace), torch.from_numpy(wl.phase))
+        p = torch.from_numpy(W.init_params(net, seed=5, bias_scale=0.05)).cuda()
+        return env, p, torch.zeros_like(p), torch.zeros_like(p)
+
+    env_a, pa, ma, va = fresh()
+    _, _, ta = iteration(env_a, pa, ma, va, 0, 0)
+    buf_a, st_a, _ = iteration(env_a, pa, ma, va, ta, 1)
+
+    env_b, pb, mb, vb = fresh()
+    _, _, tb = iteration(env_b, pb, mb, vb, 0, 0)
+    ckpt = (env_b.save(), pb.cpu(), mb.cpu(), vb.cpu(), tb)
+    env_b.close()
+    env_c, pc, mc, vc = fresh()
+    env_c.load(ckpt[0])
+    pc.copy_(ckpt[1]); mc.copy_(ckpt[2]); vc.copy_(ckpt[3])
+    buf_c, st_c, _ = iteration(env_c, pc, mc, vc, ckpt[4], 1)
+
+    for k in buf_a:
+        if buf_a[k] is not None:
+            assert torch.equal(buf_a[k], buf_c[k]), k
+    assert torch.equal(pa, pc) and torch.equal(ma, mc) and torch.equal(va, vc)
+    assert torch.equal(st_a, st_c)
+    env_a.close()
+    env_c.close()
+
+
 def test_env_rejects_bad_trace():
     wl = W.make_tiny(n_envs=4)
     tr = wl.trace.copy()
