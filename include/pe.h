@@ -383,19 +383,28 @@ pe_status pe_fleet_stagger(const float* traces, int32_t G, int32_t L, const int3
                            int32_t* peaks, void* workspace, int64_t workspace_bytes, void* stream);
 
 /* pe_fleet_windows for callers that cannot allocate device memory -- code
- * inside a host process whose device memory belongs to another allocator,
- * or a control loop that cannot afford an allocation's synchronisation.
+ * inside a host process whose device memory belongs to another allocator
+ * (a framework's caching allocator, a service with a fixed memory budget),
+ * or a control loop that must not add allocations to its timeline.
  * The paper has no counterpart: this is a deployment convenience.
  * Same arguments and results as pe_fleet_windows without the workspace: the
  * scratch is one file-scope device array of PE_FLEET_NOALLOC_SCRATCH_BYTES
- * (4 MiB, held by every GPU that loads the library until exit); the 16-byte
- * path runs when its four prefix copies fit.  Requests whose single copy
- * (about J * (L + H + 128) * 4 bytes) does not fit return PE_EINVAL with
- * that limit in the message, before any launch.  The call allocates nothing (no
- * cudaMalloc, no allocating library routine).  Its first call on a device
- * looks up the array's device address (cudaGetSymbolAddress) with that
- * device current; make that first call before any stream capture.  All
- * calls share the array: calls that overlap on the GPU race. */
+ * (4 MiB); the 16-byte path runs when its four prefix copies fit.  Requests
+ * whose single copy (about J * (L + H + 128) * 4 bytes) does not fit return
+ * PE_EINVAL with that limit in the message, before any launch.
+ * Set-up: the first call on a device, with that device current, looks up
+ * the array's device address (cudaGetSymbolAddress).  Under lazy module
+ * loading, the CUDA default, that lookup is also when the driver loads the
+ * array's module and reserves the 4 MiB on the device, once; the device
+ * then holds it until the process exits.  Make that first call at set-up
+ * time, before any stream capture.  The address is looked up again only if
+ * the device's context changed (after cudaDeviceReset).
+ * The calls allocate nothing (no cudaMalloc, no cudaFree, no allocating
+ * library routine).  Like pe_fleet_windows, every call waits on `stream`
+ * for the device-side validation read before it launches the counts, so it
+ * returns only once the preparation kernels have finished.  All calls share
+ * the array, which keeps the last call's contents: calls that overlap on the
+ * GPU (other streams, other host threads) race. */
 #define PE_FLEET_NOALLOC_SCRATCH_BYTES (4 * 1024 * 1024)
 pe_status pe_fleet_windows_noalloc(const float* traces, int32_t G, int32_t L,
                                    const int32_t* job_of_gpu, int32_t J, const int32_t* offsets,

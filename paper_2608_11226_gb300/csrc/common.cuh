@@ -127,6 +127,24 @@ __device__ __forceinline__ float bf16r(float x) {
   return __uint_as_float(u & 0xFFFF0000u);
 }
 
+// Approximate KL term of one sample, (rho - 1) - log rho with
+// rho = exp(x) (Schulman's k3 estimator), without the cancellation of the
+// literal fp32 form: for |x| < 1/8 the Taylor series of e^x - 1 - x,
+//   x^2/2 (1 + x/3 (1 + x/4 (1 + x/5 (1 + x/6 (1 + x/7))))),
+// whose first dropped term is below 2e-8 of the sum; above that the direct
+// form, whose cancellation costs less than a few ulps there.
+__device__ __forceinline__ float kl_term(float x) {
+  if (fabsf(x) < 0.125f) {
+    float t = fmaf(x, 1.0f / 7.0f, 1.0f);
+    t = fmaf(x * (1.0f / 6.0f), t, 1.0f);
+    t = fmaf(x * (1.0f / 5.0f), t, 1.0f);
+    t = fmaf(x * (1.0f / 4.0f), t, 1.0f);
+    t = fmaf(x * (1.0f / 3.0f), t, 1.0f);
+    return 0.5f * x * x * t;
+  }
+  return expm1f(x) - x;
+}
+
 inline int ceil_div(int64_t a, int64_t b) { return (int)((a + b - 1) / b); }
 
 // launch profiling: brackets a launch with CUDA events when enabled

@@ -204,7 +204,7 @@ __global__ void __launch_bounds__(kLossThreads) ppo_bf16_loss_kernel(LossArgs g)
     const float s1 = rho * an, s2 = rc * an;
     v[0] = -fminf(s1, s2);
     v[1] = Hs;
-    v[2] = (rho - 1.0f) - logr;
+    v[2] = kl_term(logr);
     v[3] = fabsf(rho - 1.0f) > g.clip ? 1.0f : 0.0f;
     const float dlp = (s1 <= s2 ? -an : 0.0f) * rho * g.inv_cnt;
     uint32_t pk[kHead / 2];

@@ -2,20 +2,26 @@
 // surrogate, squared-error value loss, entropy bonus, global-norm gradient
 // clipping and Adam).
 //
-// Per minibatch three launches:
-//   1. ppo_grad_kernel: 2*NC CTAs, the first NC differentiate the policy
-//      network, the other NC the value network (their gradients are
-//      independent).  A CTA walks its share of the minibatch in slices of 32
-//      permuted samples (Feistel order), runs forward and backward with the
-//      activations feature-major in shared memory, and keeps its weight
-//      gradient tiles in registers across slices; it writes one fp32 partial
-//      gradient row.
-//   2. ppo_reduce_kernel: fixed-order sum of the NC partial rows (in fp64),
-//      per-block sums of squares for the global norm.  Deterministic.
-//   3. ppo_adam_kernel: global norm, clip factor, Adam step; accumulates the
-//      minibatch statistics.
-// The per-minibatch advantage mean/std (which depend only on the
-// permutation) are computed for all minibatches up front.
+// The update runs as one cooperative launch (ppo_persistent_kernel) of one
+// CTA per SM: NC policy-role CTAs and NC value-role CTAs (their gradients are
+// independent).  Every minibatch step is three phases behind bounded grid
+// barriers:
+//   1. gradient: each CTA takes ceil(cnt / NC) consecutive samples of the
+//      minibatch (Feistel order) in slices of 64, runs forward and backward
+//      with the activations feature-major in shared memory (4x4 register
+//      tiles, packed two-lane FMA), adds the hidden-layer weight gradients of
+//      every slice into shared-memory accumulators, and writes one fp32
+//      partial gradient row; its weights arrive as one bulk copy of a
+//      per-role image laid out like shared memory;
+//   2. reduce: a fixed-order fp32 sum of the NC partial rows of each network
+//      and per-CTA sums of squares (deterministic);
+//   3. Adam: global norm in a fixed order, clip factor, Adam step on each
+//      CTA's slice of the parameters, which also rewrites the role images.
+// The three-launch loop (ppo_grad_kernel, ppo_reduce_kernel,
+// ppo_adam_kernel) computes the same sums and is the fallback when the
+// cooperative launch is not available.  The per-minibatch advantage
+// mean/std (which depend only on the permutation) are computed for all
+// minibatches up front.
 #include <algorithm>
 #include <cmath>
 #include <vector>
@@ -333,7 +339,7 @@ __global__ void ppo_image_kernel(const float* __restrict__ params, float* __rest
 // CTA's slices: forward, loss, backward; weight-gradient partials in
 // registers, written as this CTA's row of the partial-sum matrix.
 template <int D, int H, int A, bool POL>
-__device__ __forceinline__ void ppo_role(PpoSmem<D, H, A>& s, const PpoArgs& g, int c) {
+__device__ __forceinline__ bool ppo_role(PpoSmem<D, H, A>& s, const PpoArgs& g, int c) {
   constexpr int NA = POL ? A : 1;
   constexpr int S = kPpoS, LD = kPpoLD;
   static_assert(D % 4 == 0 && H % 32 == 0 && S * (D / 4) <= 256 && 256 + S <= kPpoNT && 4 * H <= kPpoNT,
@@ -398,7 +404,17 @@ __device__ __forceinline__ void ppo_role(PpoSmem<D, H, A>& s, const PpoArgs& g, 
   const int c0 = c * g.per_cta, c1 = min(c0 + g.per_cta, g.cnt);
   // the first slice's gather overlaps the weight copy, issued above
   if (c0 < c1) gather(c0, min(S, c1 - c0));
-  if (!tc::mbar_wait(&s.bar_w, g.wphase)) atomicExch(g.err, 1);
+  // A wait that gives up (in any thread) stops the whole CTA: thread 0
+  // records the error, waits once more (bounded) so that the copy into this
+  // CTA's shared memory is no longer in flight, and the role returns false.
+  if (!__syncthreads_and(tc::mbar_wait(&s.bar_w, g.wphase))) {
+    if (tid == 0) {
+      atomicExch(g.err, 1);
+      (void)tc::mbar_wait(&s.bar_w, g.wphase);
+    }
+    __syncthreads();
+    return false;
+  }
   // weight-gradient tiles live in registers only during their phase; each
   // slice adds them into the CTA's shared-memory accumulators gw2 / gw1
   int nsl = 0;
@@ -485,7 +501,7 @@ __device__ __forceinline__ void ppo_role(PpoSmem<D, H, A>& s, const PpoArgs& g, 
         const float s1 = rho * an, s2 = rc * an;
         st[0] += -fminf(s1, s2);
         st[1] += Hs;
-        st[2] += (rho - 1.0f) - logr;
+        st[2] += kl_term(logr);
         st[3] += fabsf(rho - 1.0f) > g.clip ? 1.0f : 0.0f;
         const float dlp = (s1 <= s2 ? -an : 0.0f) * rho * g.inv_cnt;
 #pragma unroll
@@ -600,6 +616,7 @@ __device__ __forceinline__ void ppo_role(PpoSmem<D, H, A>& s, const PpoArgs& g, 
       sp[k] = t;
     }
   }
+  return true;
 }
 
 template <int D, int H, int A>
@@ -612,9 +629,9 @@ __global__ void __launch_bounds__(kPpoNT) ppo_grad_kernel(PpoArgs g) {
   }
   __syncthreads();
   if ((int)blockIdx.x < g.NC)
-    ppo_role<D, H, A, true>(s, g, blockIdx.x);
+    (void)ppo_role<D, H, A, true>(s, g, blockIdx.x);
   else
-    ppo_role<D, H, A, false>(s, g, blockIdx.x - g.NC);
+    (void)ppo_role<D, H, A, false>(s, g, blockIdx.x - g.NC);
 }
 
 // Running minibatch statistics from the per-CTA partials, by one whole warp:
@@ -772,10 +789,11 @@ __global__ void __launch_bounds__(kPpoNT, 1) ppo_persistent_kernel(PpoLoop L) {
       g.wphase = (uint32_t)(step & 1);
       g.advstat = L.advstat + (int64_t)ep * L.nmb + mb;
       // phase 1: gradient partials of this CTA's role and samples
-      if ((int)blockIdx.x < NC)
-        ppo_role<D, H, A, true>(s, g, blockIdx.x);
-      else
-        ppo_role<D, H, A, false>(s, g, blockIdx.x - NC);
+      // a role whose weight copy timed out has recorded the error; the CTA
+      // stops, and the others give up at their next (bounded) barrier
+      const bool role_ok = (int)blockIdx.x < NC ? ppo_role<D, H, A, true>(s, g, blockIdx.x)
+                                                : ppo_role<D, H, A, false>(s, g, blockIdx.x - NC);
+      if (!role_ok) return;
       if (!grid_barrier(L.bar, &s_ok)) {
         if (tid == 0) atomicExch(L.err, 1);
         return;

@@ -507,6 +507,122 @@ def test_ppo_grad_norm_clip():
     assert np.linalg.norm(m / 0.1) == pytest.approx(1e-3 * n / (n + 1e-6), rel=1e-9)
 
 
+class _RoundF32(torch.autograd.Function):
+    """fp32 rounding in the forward pass, identity in the backward pass."""
+
+    @staticmethod
+    def forward(ctx, t):
+        return t.float().double()
+
+    @staticmethod
+    def backward(ctx, g):
+        return g
+
+
+def _torch_loss_of(net, p, obs, act, lpo, adv, ret, clip, vf, ent, bf16):
+    """The SB3 PPO loss of one minibatch as a function of the fp64 parameter
+    tensor p, written independently of the oracle.  bf16 networks see their
+    fp32-cast masters with the weights rounded to bf16 (straight-through, so
+    the gradient of the rounded weights reaches the masters) and the same
+    rounding points as _torch_ppo_loss_bf16."""
+    D, H, A = net.obs_dim, net.hidden, net.n_actions
+    sizes = [H * D, H, H * H, H, A * H, A, H * D, H, H * H, H, H, 1]
+    W1, b1, W2, b2, W3, b3, V1, c1, V2, c2, V3, c3 = torch.split(p, sizes)
+    x = torch.tensor(obs, dtype=torch.float64)
+    if bf16:
+        x = _rb(x)
+        wr = lambda w: _RoundFwd.apply(_RoundF32.apply(w))
+        br = _RoundF32.apply
+
+        def fwd(Wa, ba, Wb, bb, Wc, bc, out):
+            h1 = _TanhRound.apply(_RoundBwd.apply(x @ wr(Wa.view(H, D)).T + br(ba)))
+            h2 = _TanhRound.apply(_RoundBwd.apply(h1 @ wr(Wb.view(H, H)).T + br(bb)))
+            return _RoundBwd.apply(h2 @ wr(Wc.view(out, H)).T) + br(bc)
+    else:
+        def fwd(Wa, ba, Wb, bb, Wc, bc, out):
+            return torch.tanh(torch.tanh(x @ Wa.view(H, D).T + ba) @ Wb.view(H, H).T + bb) @ Wc.view(out, H).T + bc
+    z = fwd(W1, b1, W2, b2, W3, b3, A)
+    V = fwd(V1, c1, V2, c2, V3, c3, 1)[:, 0]
+    logp_all = torch.log_softmax(z, -1)
+    lp = logp_all[torch.arange(len(act)), torch.tensor(act, dtype=torch.long)]
+    a = torch.tensor(adv, dtype=torch.float64)
+    a = (a - a.mean()) / (a.std() + 1e-8)
+    logr = lp - torch.tensor(lpo, dtype=torch.float64)
+    rho = torch.exp(logr)
+    pg = -torch.min(rho * a, torch.clamp(rho, 1 - clip, 1 + clip) * a).mean()
+    vl = ((torch.tensor(ret, dtype=torch.float64) - V) ** 2).mean()
+    H_ = -(logp_all.exp() * logp_all).sum(-1).mean()
+    with torch.no_grad():
+        kl = ((rho - 1) - logr).mean().item()
+        cf = ((rho - 1).abs() > clip).double().mean().item()
+    return pg + vf * vl - ent * H_, (pg.item(), vl.item(), H_.item(), kl, cf)
+
+
+def _torch_ppo_update(net, ppo, params, m0, v0, t0, batch, seed, iteration):
+    """The whole update loop in torch: per epoch the oracle's Feistel order
+    (any permutation is valid; the loop must gather every per-sample array
+    through the same index), ragged last minibatch, autograd gradient,
+    torch.nn.utils.clip_grad_norm_, torch.optim.Adam resumed from (m0, v0,
+    t0).  Returns params, moments, per-step statistics means and step count."""
+    obs, act, lpo, adv, ret = batch
+    N = len(act)
+    p = torch.tensor(np.asarray(params, np.float64), requires_grad=True)
+    opt = torch.optim.Adam([p], lr=ppo.lr, betas=(ppo.beta1, ppo.beta2), eps=ppo.eps)
+    if t0:
+        opt.state[p] = {"step": torch.tensor(float(t0), dtype=torch.float64),
+                        "exp_avg": torch.tensor(m0, dtype=torch.float64),
+                        "exp_avg_sq": torch.tensor(v0, dtype=torch.float64)}
+    acc = np.zeros(5)
+    steps = 0
+    for ep in range(ppo.epochs):
+        perm = O.feistel_perm(N, O.perm_keys(seed, ep, iteration))
+        for start in range(0, N, ppo.minibatch):
+            idx = perm[start:start + ppo.minibatch]
+            opt.zero_grad()
+            loss, st = _torch_loss_of(net, p, obs[idx], act[idx], lpo[idx], adv[idx], ret[idx], ppo.clip,
+                                      ppo.vf_coef, ppo.ent_coef, net.dtype == 1)
+            loss.backward()
+            torch.nn.utils.clip_grad_norm_([p], ppo.max_grad_norm)
+            opt.step()
+            acc += st
+            steps += 1
+    s = opt.state[p]
+    return p.detach().numpy(), s["exp_avg"].numpy(), s["exp_avg_sq"].numpy(), acc / steps, steps
+
+
+@pytest.mark.parametrize("bf16", [0, 1])
+def test_ppo_update_loop_matches_torch_autograd_clip_and_adam(bf16):
+    """or_ppo_update_ex over 2 epochs x 3 minibatches (40, 40 and a ragged
+    20), resumed from nonzero Adam moments at step 3, against an independent
+    torch loop (autograd, clip_grad_norm_, optim.Adam): parameters, both
+    moments, the step count and the statistics.  A frozen bias correction,
+    moments dropped between minibatches, a gather that takes one array through
+    a different index, or a ragged tail normalised over the full minibatch
+    size each fail this."""
+    net = W.NetSpec(6, 16 if bf16 else 8, 4, bf16)
+    params = W.init_params(net, seed=8, bias_scale=0.1).astype(np.float64)
+    N = 100
+    obs, act, lpo, adv, ret = _ppo_batch(net, N, seed=5)
+    adv = (adv + 0.7).astype(np.float32)   # a nonzero mean, so normalisation matters
+    ppo = W.PPOSpec(epochs=2, minibatch=40, lr=3e-3, ent_coef=0.01, max_grad_norm=0.5)
+    rng = np.random.default_rng(3)
+    m0 = 1e-3 * rng.standard_normal(params.size)
+    v0 = 1e-5 * rng.random(params.size)
+    P, m, v, t, st = O.ppo_update(net, ppo, params, m0, v0, 3, obs, act, lpo, adv, ret, seed=11, iteration=4)
+    tp, tm, tv, tst, steps = _torch_ppo_update(net, ppo, params, m0, v0, 3, (obs, act, lpo, adv, ret), 11, 4)
+    assert t == 3 + 6 and steps == 6 and st[7] == 6
+    assert np.allclose(P, tp, rtol=1e-9, atol=1e-12)
+    assert np.allclose(m, tm, rtol=1e-9, atol=1e-14)
+    assert np.allclose(v, tv, rtol=1e-9, atol=1e-16)
+    # statistics: pg, value loss, entropy, approx KL, clip fraction (means over the steps)
+    for k, want in zip((0, 1, 2, 3, 4), tst):
+        assert st[k] == pytest.approx(want, rel=1e-9, abs=1e-12), k
+    # the steps moved the policy: the later minibatches see rho != 1
+    assert st[3] > 0.0
+    # and the parameters moved by about lr per step
+    assert 0.5 * 3e-3 < np.abs(P - params).max() <= 6 * 3e-3 * (1 + 1e-6)
+
+
 # ---------------------------------------------------------------------- fleet
 def _brute_fleet(traces, job, J, offsets, H, windows, Bq):
     q = np.rint(traces.astype(np.float32) * np.float32(64)).astype(np.int64)

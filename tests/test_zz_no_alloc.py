@@ -1,13 +1,15 @@
 """pe_fleet_windows_noalloc: the fleet window counts for callers that cannot
 allocate device memory (their device memory belongs to another allocator,
-or their control loop cannot afford an allocation's synchronisation).  It
-must give exactly the results of pe_fleet_windows with a caller workspace,
-call after call, although every call reuses the same fixed scratch array
-that keeps the previous call's contents.  Collected last on purpose."""
+or their control loop must not add allocations to its timeline).  It must
+give exactly the results of pe_fleet_windows with a caller workspace, and of
+the CPU oracle, call after call, although every call reuses the same fixed
+scratch array that keeps the previous call's contents.  Collected last on
+purpose."""
 import numpy as np
 import pytest
 import torch
 
+import oracle as O
 from paper_2608_11226_gb300 import pe
 from paper_2608_11226_gb300 import workloads as W
 
@@ -39,14 +41,20 @@ def _with_workspace(fw, dev, windows):
     return counts.cpu().numpy(), peaks.cpu().numpy()
 
 
-def _noalloc(fw, dev, windows):
+def _noalloc(fw, dev, windows, stream=None):
     N = fw.offsets.shape[0]
     counts = torch.full((N, len(windows)), -7, dtype=torch.int32, device="cuda")
     peaks = torch.full_like(counts, -7)
+    torch.cuda.synchronize()
     pe.fleet_windows_noalloc(dev[0], dev[1], fw.n_jobs, dev[2], fw.horizon, windows, fw.budget_q,
-                             counts, peaks)
+                             counts, peaks, stream=stream)
     torch.cuda.synchronize()
     return counts.cpu().numpy(), peaks.cpu().numpy()
+
+
+def _oracle(fw, windows):
+    return O.fleet_windows(fw.traces, fw.job_of_gpu, fw.n_jobs, fw.offsets, fw.horizon, windows,
+                           fw.budget_q)
 
 
 def test_noalloc_matches_workspace_entry_point_two_calls_in_a_row():
@@ -57,6 +65,60 @@ def test_noalloc_matches_workspace_entry_point_two_calls_in_a_row():
         c_ref, p_ref = _with_workspace(fw, dev, windows)
         c, p = _noalloc(fw, dev, windows)
         assert np.array_equal(c, c_ref) and np.array_equal(p, p_ref)
+        if n < 100:
+            oc, op = _oracle(fw, windows)
+            assert np.array_equal(c, oc) and np.array_equal(p, op)
+
+
+def _fits(length):
+    """Whether a fleet of trace length `length` (H = L) fits the static
+    scratch: the entry point rejects an oversized request on the host, before
+    touching any device buffer."""
+    fw = W.make_fleet(n_compositions=1, length=1000, seed=0)
+    tr = torch.zeros((fw.traces.shape[0], length), dtype=torch.float32, device="cuda")
+    job = torch.from_numpy(fw.job_of_gpu).cuda()
+    off = torch.zeros((1, fw.n_jobs), dtype=torch.int32, device="cuda")
+    c = torch.zeros((1, 1), dtype=torch.int32, device="cuda")
+    try:
+        # N = 0: nothing is counted even when the request fits
+        pe.fleet_windows_noalloc(tr, job, fw.n_jobs, off[:0], length, [1], fw.budget_q, c, c)
+        return True
+    except pe.PEError as e:
+        assert e.status == pe.PE_EINVAL and "static scratch" in str(e)
+        return False
+
+
+def test_noalloc_just_under_its_limit_and_on_a_side_stream():
+    """The largest fleet that fits (one prefix copy filling the array up to
+    its last words, where the maxima and the flag sit), on a non-default
+    stream, against the workspace entry point and the oracle."""
+    lo, hi = 2000, 200000
+    assert _fits(lo) and not _fits(hi)
+    while hi - lo > 1:
+        mid = (lo + hi) // 2
+        lo, hi = (mid, hi) if _fits(mid) else (lo, mid)
+    fw, dev = _inputs(6, lo, 11)
+    windows = [1, 60, 600]
+    side = torch.cuda.Stream()
+    c, p = _noalloc(fw, dev, windows, stream=side)
+    c_ref, p_ref = _with_workspace(fw, dev, windows)
+    oc, op = _oracle(fw, windows)
+    assert np.array_equal(c, c_ref) and np.array_equal(p, p_ref)
+    assert np.array_equal(c, oc) and np.array_equal(p, op)
+    # a second call in a row on the default stream, after the near-full one
+    fw2, dev2 = _inputs(40, 3000, 12)
+    c2, p2 = _noalloc(fw2, dev2, windows)
+    oc2, op2 = _oracle(fw2, windows)
+    assert np.array_equal(c2, oc2) and np.array_equal(p2, op2)
+
+
+def test_noalloc_zero_compositions_is_a_noop():
+    fw, dev = _inputs(1, 3000, 2)
+    counts = torch.full((1, 3), -7, dtype=torch.int32, device="cuda")
+    pe.fleet_windows_noalloc(dev[0], dev[1], fw.n_jobs, dev[2][:0], fw.horizon, [1, 60, 600],
+                             fw.budget_q, counts, counts)
+    torch.cuda.synchronize()
+    assert (counts.cpu().numpy() == -7).all()
 
 
 def test_noalloc_rejects_requests_beyond_its_scratch():
