@@ -64,6 +64,14 @@ def parse():
                     help="run one small named case of a hot kernel (for ncu captures) and exit")
     ap.add_argument("--gae-large", type=int, nargs=2, default=[2048, 262144], metavar=("T", "E"),
                     help="GAE roofline size (Stress: 2048 x 262144); T=0 skips it")
+    ap.add_argument("--stress", type=int, nargs=2, default=[262144, 2048], metavar=("E", "T"),
+                    help="Stress iteration size (envs, horizon); E=0 skips the leg")
+    ap.add_argument("--stress-fleet-n", type=int, default=1_000_000,
+                    help="fleet compositions recomputed inside each Stress iteration")
+    ap.add_argument("--no-cpu-table", dest="cpu_table", action="store_false",
+                    help="skip the per-configuration oracle table (1 core and all host cores)")
+    ap.add_argument("--no-roofs", dest="roofs", action="store_false",
+                    help="skip the FP32 / INT32 / L2 roof microbenchmarks")
     return ap.parse_args()
 
 
@@ -184,6 +192,35 @@ def job_value(units_per_rank: float, world: int, max_ms: float) -> float:
     return units_per_rank * world / (max_ms / 1e3)
 
 
+# --------------------------------------------------------------------------- measured roofs
+def measure_roofs(local: int):
+    """FP32 FMA (scalar and packed two-lane), INT32 add and L2-read roofs of
+    this GPU, each the best of 3 timed throughput loops (pe_roof_probe),
+    with the SM clock sampled while they run."""
+    from paper_2608_11226_gb300 import pe
+    buf = torch.zeros(8 * 1024 * 1024, dtype=torch.float32, device="cuda")  # 32 MB: L2-resident
+    clocks = ClockSampler(local)
+    clocks.start()
+    out = {}
+    for name, kind, reps, unit, scale in (("fp32_ffma", pe.PE_ROOF_FFMA, 200000, "TFLOP/s", 1e12),
+                                          ("fp32_ffma2", pe.PE_ROOF_FFMA2, 100000, "TFLOP/s", 1e12),
+                                          ("int32_add", pe.PE_ROOF_IADD, 100000, "Tops/s", 1e12),
+                                          ("l2_read", pe.PE_ROOF_L2, 20, "GB/s", 1e9)):
+        best = 0.0
+        for _ in range(3):
+            ms, units = pe.roof_probe(kind, buf, reps)
+            best = max(best, units / (ms / 1e3) / scale)
+        out[name] = {"value": best, "unit": unit}
+    clk = clocks.stop()
+    out["fp32_fma_peak_tflops"] = max(out["fp32_ffma"]["value"], out["fp32_ffma2"]["value"])
+    out["clocks"] = clk
+    out["how"] = ("pe_roof_probe: 8 CTAs x 256 threads per SM, 8 independent chains per thread "
+                  "(FFMA / packed FFMA2 / IADD), or 16-byte L2-only loads over a 32 MB buffer; "
+                  "best of 3 launches timed with CUDA events")
+    del buf
+    return out
+
+
 # --------------------------------------------------------------------------- our path
 class Trainer:
     """State of one 7B PPO training replica on the device."""
@@ -227,6 +264,7 @@ def run_ours(args, world, rank, local):
     from paper_2608_11226_gb300 import workloads as W
     build.build()
     pe.lib()
+    roofs = measure_roofs(local) if args.roofs else None
     tr = Trainer(seed=rank)
     flush = torch.empty(64 * 1024 * 1024, dtype=torch.float32, device="cuda")  # 256 MB > L2
     for _ in range(args.warmup):
@@ -268,12 +306,19 @@ def run_ours(args, world, rank, local):
     samples_per_launch = (tr.E * tr.T * tr.wl.ppo.epochs) if gn == args.steps else tr.wl.ppo.minibatch
     kname = "ppo_persistent_kernel" if gn == args.steps else "ppo_grad_kernel"
     fl_launch = ppo_flops_per_sample(net.obs_dim, net.hidden, net.n_actions) * samples_per_launch
-    peak_tflops = N_SM * FP32_LANES_PER_SM * 2 * SM_MAX_MHZ * 1e6 / 1e12
+    derived_tflops = N_SM * FP32_LANES_PER_SM * 2 * SM_MAX_MHZ * 1e6 / 1e12
+    if roofs:
+        peak_tflops = roofs["fp32_fma_peak_tflops"]
+        src = ("measured: pe_roof_probe FP32 FMA throughput loop (best of scalar FFMA and packed "
+               f"FFMA2) in this run; derived figure {derived_tflops:.1f} TFLOP/s at 2070 MHz")
+    else:
+        peak_tflops = derived_tflops
+        src = "derived: 152 SMs x 128 FP32 lanes x 2 FLOP x 2070 MHz"
     ach = fl_launch / (gms / gn / 1e3) / 1e12 if gn else None
     roof = {"kernel": kname, "bound": "alu", "achieved": ach, "peak": peak_tflops,
             "unit": "TFLOP/s", "frac": (ach / peak_tflops) if ach else None,
             "traffic": load_traffic(kname),
-            "peak_source": "derived: 152 SMs x 128 FP32 lanes x 2 FLOP x 2070 MHz",
+            "peak_source": src, "frac_of_derived": (ach / derived_tflops) if ach else None,
             "avg_launch_ms": gms / gn if gn else None, "launches": gn,
             "flop_per_launch": fl_launch}
     kernels = {k: {"ms_per_step": ms / args.steps, "launches_per_step": n / args.steps,
@@ -317,11 +362,16 @@ def run_ours(args, world, rank, local):
     e2e = {"value": env_steps * world * e2e_steps / e2e_s, "unit": "env-steps/s",
            "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h}
 
+    ppo_stats_last = [float(x) for x in tr.stats.cpu()]
     # ---- fleet accounting
-    fleet = run_fleet(args, world, tr) if args.fleet_n > 0 else None
+    fleet = run_fleet(args, world, tr, roofs) if args.fleet_n > 0 else None
     evaluation = run_evaluation(args, world, tr, peaks) if args.eval else None
     r72b = run_72b(args, world, peaks) if args.r72b_steps > 0 else None
     gae_large = run_gae_large(args, world, peaks) if args.gae_large[0] > 0 else None
+    tiny = run_tiny(args, world)
+    del tr
+    torch.cuda.empty_cache()
+    stress = run_stress(args, world, peaks, local) if args.stress[0] > 0 else None
 
     out = {"metric": METRIC, "value": value, "unit": "env-steps/s", "n_gpus": world,
            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_step,
@@ -335,9 +385,12 @@ def run_ours(args, world, rank, local):
            "roofline": roof, "gae_roofline": gae_roof, "kernels": kernels,
            "gpu_launches": launches, "clocks": clk, "e2e": e2e, "fleet": fleet, "rollout_72b": r72b,
            "gae_roofline_stress_size": gae_large, "evaluation": evaluation,
-           "ppo_stats_last": [float(x) for x in tr.stats.cpu()]}
+           "stress_iteration": stress, "tiny_iteration": tiny, "measured_roofs": roofs,
+           "ppo_stats_last": ppo_stats_last}
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         out["cpu_baseline"] = cpu_baseline(args.cpu_envs)
+    if rank == 0 and world == 1 and args.cpu_table:
+        out["per_config"] = per_config_table(out)
     if rank == 0:
         print(json.dumps(out), flush=True)
 
@@ -415,7 +468,7 @@ def run_evaluation(args, world, tr, peaks):
                                               "note": "6 B of buffer writes per env-step; latency-bound"}}}
 
 
-def run_fleet(args, world, tr=None):
+def run_fleet(args, world, tr=None, roofs=None):
     from paper_2608_11226_gb300 import pe
     from paper_2608_11226_gb300 import workloads as W
     fw = W.make_fleet(n_compositions=args.fleet_n)
@@ -461,6 +514,13 @@ def run_fleet(args, world, tr=None):
             "kernel_ms_per_launch": wms / wn if wn else None,
             "composed_samples_per_s": composed / (wms / wn / 1e3) if wn else None,
             "logical_l2_gbs": 4.0 * fw.n_jobs * composed / (wms / wn / 1e3) / 1e9 if wn else None,
+            "roofline": ({"kernel": "fleet_windows_v4_kernel", "bound": "l2",
+                          "achieved": 4.0 * fw.n_jobs * composed / (wms / wn / 1e3) / 1e9,
+                          "peak": roofs["l2_read"]["value"], "unit": "GB/s",
+                          "frac": 4.0 * fw.n_jobs * composed / (wms / wn / 1e3) / 1e9 / roofs["l2_read"]["value"],
+                          "note": "logical bytes: 4 B per job per composed sample, against the measured "
+                                  "L2-read roof (32 MB resident buffer)"}
+                         if (wn and roofs) else None),
             "violation_fraction_mean": [float(c[:, i].mean() / (H - w + 1)) for i, w in enumerate(windows)],
             "peak_fraction_of_nameplate_max": [float(p[:, i].max() / (64.0 * w) / W.FLEET_NAMEPLATE_W)
                                                for i, w in enumerate(windows)],
@@ -772,6 +832,169 @@ def run_72b_ppo(args, world, peaks, wl, buf, adv, ret):
                          "achieved": ach, "peak": peak, "unit": "TFLOP/s", "frac": ach / peak,
                          "flop_per_sample": ppo_flops_per_sample(net.obs_dim, net.hidden, net.n_actions)},
             "stats": st}
+
+
+def run_tiny(args, world):
+    """One PPO iteration of the Tiny workload (64 envs x 128 steps, fp32
+    8-64-64, PPO 4 epochs over one minibatch of the whole rollout), 10 timed
+    iterations after 3 warm-up ones."""
+    from paper_2608_11226_gb300 import pe
+    from paper_2608_11226_gb300 import workloads as W
+    wl = W.make_tiny()
+    spec, net = wl.env, wl.net
+    T, E = wl.horizon, spec.n_envs
+    env = pe.Env(spec, torch.from_numpy(wl.trace), torch.from_numpy(wl.phase))
+    buf = pe.alloc_rollout(spec, net, T)
+    params = torch.from_numpy(W.init_params(net, seed=0)).cuda()
+    m = torch.zeros_like(params)
+    v = torch.zeros_like(params)
+    adv = torch.empty(T, E, device="cuda")
+    ret = torch.empty_like(adv)
+    stats = torch.zeros(8, device="cuda")
+    ppo = W.PPOSpec(epochs=4, minibatch=T * E)
+    ws = pe.alloc_workspace(pe.ppo_workspace_bytes(net, ppo, T * E))
+
+    def it(k):
+        pe.rollout(env, net, params, T, k, buf)
+        pe.gae(buf["reward"], buf["value"], buf["done"], buf["last_value"], 0.99, 0.95, adv, ret)
+        pe.ppo_update(net, ppo, params, m, v, 4 * k, buf["obs"], buf["act"], buf["logp"], adv, ret, stats,
+                      ws, seed=7, iteration=k)
+    for k in range(3):
+        it(k)
+    torch.cuda.synchronize()
+    barrier(world)
+    stream = torch.cuda.current_stream()
+    a = torch.cuda.Event(enable_timing=True)
+    b = torch.cuda.Event(enable_timing=True)
+    a.record(stream)
+    for k in range(3, 13):
+        it(k)
+    b.record(stream)
+    torch.cuda.synchronize()
+    ms = max_over_ranks(a.elapsed_time(b), world) / 10
+    env.close()
+    return {"metric": "Tiny PPO iteration env-steps/s", "value": T * E * world / (ms / 1e3),
+            "unit": "env-steps/s", "ms_per_iteration": ms,
+            "config": {"workload": "tiny: 64 envs x 128 steps, 4,000-sample trace, 3 actions, MLP 8-64-64 "
+                                   "fp32, GAE, PPO 4 epochs x one 8,192-sample minibatch"}}
+
+
+def run_stress(args, world, peaks, local):
+    """One full iteration of the Stress configuration, timed once after a
+    short warm-up of each kernel: the rollout of 262,144 envs x 2,048 steps
+    over a 4 x 380,000-sample trace (bf16 64-512-512 policy on the tcgen05
+    tensor cores with streamed weights, then the value network on every
+    observation), GAE, the full PPO update (4 epochs x minibatch 65,536 =
+    32,768 minibatch steps), and the fleet windows recomputed at
+    --stress-fleet-n compositions.  Reports env-steps/s of the iteration,
+    the phase times and the bf16 FLOP rate of the update against the
+    measured sustained peak."""
+    from paper_2608_11226_gb300 import pe
+    from paper_2608_11226_gb300 import workloads as W
+    E, T = args.stress
+    wl = W.make_stress(n_envs=E, horizon=T)
+    spec, net, ppo = wl.env, wl.net, wl.ppo
+    env = pe.Env(spec, torch.from_numpy(wl.trace), torch.from_numpy(wl.phase))
+    buf = pe.alloc_rollout(spec, net, T)
+    buf["q"] = None
+    N = T * E
+    params = torch.from_numpy(W.init_params(net, seed=0)).cuda()
+    m = torch.zeros_like(params)
+    v = torch.zeros_like(params)
+    adv = torch.empty(T, E, device="cuda")
+    ret = torch.empty_like(adv)
+    stats = torch.zeros(8, device="cuda")
+    rws = pe.alloc_workspace(pe.rollout_workspace_bytes(env, net))
+    pws = pe.alloc_workspace(pe.ppo_workspace_bytes(net, ppo, N))
+    fw = W.make_fleet(n_compositions=args.stress_fleet_n)
+    ftr = torch.from_numpy(fw.traces).cuda()
+    fjob = torch.from_numpy(fw.job_of_gpu).cuda()
+    foff = torch.from_numpy(fw.offsets).cuda()
+    fcnt = torch.empty((foff.shape[0], 3), dtype=torch.int32, device="cuda")
+    fpk = torch.empty_like(fcnt)
+    fws = pe.alloc_workspace(pe.fleet_workspace_bytes(fw.n_jobs, ftr.shape[1], fw.horizon))
+    # warm-up: a 4-step rollout, GAE, 2 minibatch steps of the update, one fleet call
+    pe.rollout(env, net, params, 4, 0, buf, lam=1.0, workspace=rws)
+    pe.gae(buf["reward"], buf["value"], buf["done"], buf["last_value"], 0.99, 0.95, adv, ret)
+    wppo = W.PPOSpec(epochs=1, minibatch=ppo.minibatch, ent_coef=ppo.ent_coef)
+    nw = 2 * ppo.minibatch
+    pe.ppo_update(net, wppo, params.clone(), m.clone(), v.clone(), 0, buf["obs"].view(-1, net.obs_dim)[:nw],
+                  buf["act"].view(-1)[:nw], buf["logp"].view(-1)[:nw], adv.view(-1)[:nw], ret.view(-1)[:nw],
+                  stats, pws, seed=7, iteration=0)
+    pe.fleet_windows(ftr, fjob, fw.n_jobs, foff, fw.horizon, [1, 60, 600], fw.budget_q, fcnt, fpk, fws)
+    torch.cuda.synchronize()
+    pe.device_check()
+    barrier(world)
+    clocks = ClockSampler(local)
+    clocks.start()
+    stream = torch.cuda.current_stream()
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(5)]
+    ev[0].record(stream)
+    pe.rollout(env, net, params, T, 1, buf, lam=1.0, workspace=rws)
+    ev[1].record(stream)
+    pe.gae(buf["reward"], buf["value"], buf["done"], buf["last_value"], 0.99, 0.95, adv, ret)
+    ev[2].record(stream)
+    pe.ppo_update(net, ppo, params, m, v, 0, buf["obs"], buf["act"], buf["logp"], adv, ret, stats, pws,
+                  seed=7, iteration=1)
+    ev[3].record(stream)
+    pe.fleet_windows(ftr, fjob, fw.n_jobs, foff, fw.horizon, [1, 60, 600], fw.budget_q, fcnt, fpk, fws)
+    ev[4].record(stream)
+    torch.cuda.synchronize()
+    clk = clocks.stop()
+    pe.device_check()
+    ph = [ev[i].elapsed_time(ev[i + 1]) for i in range(4)]
+    total = max_over_ranks(sum(ph), world)
+    D, H, A = net.obs_dim, net.hidden, net.n_actions
+    steps = ppo.epochs * ((N + ppo.minibatch - 1) // ppo.minibatch)
+    ppo_flop = ppo_flops_per_sample(D, H, A) * N * ppo.epochs
+    roll_flop = 2.0 * N * (D * H + H * H + H * A) + 2.0 * (N + E) * (D * H + H * H + H)
+    peak = float(peaks.get("bf16_tflops_sustained", 1725.0))
+    ppo_tf = ppo_flop / (ph[2] / 1e3) / 1e12
+    roll_tf = roll_flop / (ph[0] / 1e3) / 1e12
+    st = [float(x) for x in stats.cpu()]
+    out = {"metric": "Stress PPO iteration env-steps/s", "value": N * world / (total / 1e3), "unit": "env-steps/s",
+           "ms_per_iteration": total,
+           "phases_ms": {"rollout": ph[0], "gae": ph[1], "ppo_update": ph[2], "fleet_windows": ph[3]},
+           "config": {"workload": f"stress: {E} envs x {T} steps over a 4 x 380,000-sample 72B-shaped trace, "
+                                  "16 levels, MLP 64-512-512 bf16 (tcgen05, streamed weights), GAE, PPO 4 epochs x "
+                                  f"minibatch 65,536 ({steps} minibatch steps), fleet windows at "
+                                  f"{foff.shape[0]} compositions", "n_envs": E, "horizon": T,
+                      "timed": "one iteration after a short warm-up of each kernel; inputs larger than L2"},
+           "roofline": {"kernel": "bf16 PPO update (all its kernels)", "bound": "tensor", "achieved": ppo_tf,
+                        "peak": peak, "unit": "TFLOP/s", "frac": ppo_tf / peak,
+                        "flop": ppo_flop, "peak_source": "MEASURED_PEAKS.json bf16_tflops_sustained"},
+           "roofline_rollout_mlp": {"kernel": "rollout (policy + value MLP on tcgen05, env step)", "bound": "tensor",
+                                    "achieved": roll_tf, "peak": peak, "unit": "TFLOP/s", "frac": roll_tf / peak},
+           "gae_gbs": 17.0 * N / (ph[1] / 1e3) / 1e9,
+           "fleet_window_samples_per_s": sum(foff.shape[0] * (fw.horizon - w + 1) for w in (1, 60, 600)) / (ph[3] / 1e3),
+           "ppo_stats": st, "clocks": clk}
+    env.close()
+    del buf, adv, ret, pws, rws
+    torch.cuda.empty_cache()
+    return out
+
+
+def per_config_table(out):
+    """Per configuration: the GPU figure of this run, its roofline fraction,
+    and the CPU oracle on 1 core and on all host cores (process-sharded,
+    bounded samples; "extrapolated" where the sample is smaller than the
+    configuration)."""
+    from oracle import cpu_rate
+    cpu = cpu_rate.rates()
+    r72 = out.get("rollout_72b") or {}
+    gpu = {
+        "tiny": ((out.get("tiny_iteration") or {}).get("value"), None, "PPO iteration env-steps/s"),
+        "7b": (out["value"], (out.get("roofline") or {}).get("frac"), "PPO iteration env-steps/s"),
+        "72b": (r72.get("value"), (r72.get("roofline_policy_mlp") or {}).get("frac"),
+                "rollout env-steps/s (policy MLP tensor fraction)"),
+        "stress": ((out.get("stress_iteration") or {}).get("value"),
+                   ((out.get("stress_iteration") or {}).get("roofline") or {}).get("frac"),
+                   "PPO iteration env-steps/s (update tensor fraction)"),
+        "fleet": ((out.get("fleet") or {}).get("value"),
+                  ((out.get("fleet") or {}).get("roofline") or {}).get("frac"),
+                  "window-samples/s (logical L2 fraction)"),
+    }
+    return {k: {"gpu": gpu[k][0], "gpu_metric": gpu[k][2], "roofline_frac": gpu[k][1], **cpu[k]} for k in cpu}
 
 
 def gae_traffic(env_steps: int):

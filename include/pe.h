@@ -433,6 +433,27 @@ pe_status pe_profile_enable(int32_t on);
 pe_status pe_profile_read(int32_t kind, double* total_ms, int64_t* launches);
 const char* pe_profile_kind_name(int32_t kind);
 
+/* Measured roofs for the roofline fractions of the kernels that neither HBM
+ * nor the tensor cores bound (measurement support; the paper has no
+ * counterpart).  One warm-up and one timed launch of a throughput loop over
+ * 8 CTAs of 256 threads per SM, timed with CUDA events on `stream`; the call
+ * waits for the result.
+ *  kind 0 (PE_ROOF_FFMA):  scalar fp32 FMA, units = FLOPs (2 per FMA), reps = loop trips;
+ *  kind 1 (PE_ROOF_FFMA2): packed two-lane fp32 FMA, units = FLOPs;
+ *  kind 2 (PE_ROOF_IADD):  int32 adds, units = adds;
+ *  kind 3 (PE_ROOF_L2):    16-byte loads cached in L2 only over buf[4096, bytes),
+ *                          reps passes, units = bytes (pick a buffer L2 holds).
+ *  buf: >= 64 KiB of device memory, 16-byte aligned (its first 4 KiB are
+ *  scratch words the loops keep alive and never write in practice).
+ *  ms: host out, device time of the timed launch; units: host out.
+ * Errors: PE_EINVAL (kind, sizes, alignment), PE_ECUDA. */
+#define PE_ROOF_FFMA 0
+#define PE_ROOF_FFMA2 1
+#define PE_ROOF_IADD 2
+#define PE_ROOF_L2 3
+pe_status pe_roof_probe(int32_t kind, void* buf, int64_t bytes, int64_t reps, double* ms, double* units,
+                        void* stream);
+
 /* Synchronise `stream`, then report device-side errors of earlier launches:
  * PE_ETIMEOUT if a bounded tensor-core wait gave up (the flag is cleared). */
 pe_status pe_device_check(void* stream);

@@ -79,7 +79,7 @@ EXPORTS = (
     "pe_value", "pe_device_check", "pe_gae", "pe_ppo_workspace_bytes",
     "pe_ppo_update", "pe_fleet_workspace_bytes", "pe_fleet_windows", "pe_fleet_windows_noalloc",
     "pe_fleet_stagger_workspace_bytes", "pe_fleet_stagger", "pe_env_set_offsets", "pe_rollout_rule", "pe_rollout_replay", "pe_wait_selftest",
-    "pe_dual_ascent",
+    "pe_dual_ascent", "pe_roof_probe",
     "pe_profile_enable",
     "pe_profile_read", "pe_profile_kind_name", "pe_last_error")
 
@@ -121,6 +121,7 @@ def lib():
                                        vp, vp, i64, vp]),
             "pe_fleet_windows_noalloc": (i32, [vp, i32, i32, vp, i32, vp, i64, i32, vp, i32, i64,
                                                vp, vp, vp]),
+            "pe_roof_probe": (i32, [i32, vp, i64, i64, C.POINTER(C.c_double), C.POINTER(C.c_double), vp]),
             "pe_profile_enable": (i32, [i32]),
             "pe_profile_read": (i32, [i32, C.POINTER(C.c_double), C.POINTER(C.c_int64)]),
             "pe_profile_kind_name": (C.c_char_p, [i32]),
@@ -383,6 +384,17 @@ def fleet_stagger(traces, job_of_gpu, J: int, H: int, w: int, stride: int, offse
     G, L = traces.shape
     _check(lib().pe_fleet_stagger(_ptr(traces), G, L, _ptr(job_of_gpu), J, H, w, stride, _ptr(offsets),
                                   _ptr(peaks), _ptr(workspace), workspace.numel(), _stream(stream)))
+
+
+PE_ROOF_FFMA, PE_ROOF_FFMA2, PE_ROOF_IADD, PE_ROOF_L2 = 0, 1, 2, 3
+
+
+def roof_probe(kind: int, buf, reps: int, stream=None):
+    """(device ms, units) of one timed throughput loop (pe_roof_probe)."""
+    ms, units = C.c_double(0.0), C.c_double(0.0)
+    _check(lib().pe_roof_probe(kind, _ptr(buf), buf.numel() * buf.element_size(), reps, C.byref(ms),
+                               C.byref(units), _stream(stream)))
+    return ms.value, units.value
 
 
 FLEET_NOALLOC_SCRATCH_BYTES = 4 * 1024 * 1024

@@ -592,6 +592,37 @@ def _oracle_ppo(wl, ppo, params, buf, adv, ret, iteration=0, max_steps=-1):
                         max_steps)
 
 
+def assert_stats(gs, st, min_cnt, tol=TOL):
+    """All eight update statistics.  [1] value loss, [2] entropy, [5] total
+    loss, [6] last gradient norm: relative.  [0] the clipped surrogate is a
+    mean of terms whose normalised advantages sum to zero, so its error is
+    measured against max(|pg|, 1).  [3] approximate KL, a mean of about
+    (log rho)^2 / 2: relative, plus an absolute floor for the log-ratio noise
+    e of the two forward passes (fp32 against fp64 accumulation), which adds
+    about mean(|log rho| e) + mean(e^2): 1e-9 for fp32 networks, and
+    1e-3 sqrt(2 KL) + 1e-6 for bf16 networks, where a bf16 rounding flip of a
+    hidden activation moves a logit by up to about 1e-3.  [4] clip fraction:
+    the GPU decides |rho - 1| > clip in fp32, the oracle in fp64, so a sample
+    within rounding of the boundary may count on one side only; at most one
+    such sample per minibatch step.  [7] step count: exact."""
+    assert gs[7] == st[7]
+    for k in (1, 2, 5, 6):
+        assert abs(gs[k] - st[k]) <= tol * max(abs(st[k]), 1e-3), (k, gs[k], st[k])
+    assert abs(gs[0] - st[0]) <= tol * max(abs(st[0]), 1.0), (0, gs[0], st[0])
+    floor = 1e-9 if tol <= TOL else 1e-3 * np.sqrt(2.0 * abs(st[3])) + 1e-6
+    assert abs(gs[3] - st[3]) <= tol * abs(st[3]) + floor, (3, gs[3], st[3])
+    assert abs(gs[4] - st[4]) <= 1.0 / min_cnt + 1e-7, (4, gs[4], st[4])
+
+
+def assert_update_fp32(gp, gm, gv, P, m, v):
+    """fp32 update after several steps: parameters and Adam's first moment
+    within the benchmark spec's 1e-5 (rms-floored relative); the second moment is
+    quadratic in the gradient, so twice that."""
+    assert rel_err(gm, m) <= TOL, rel_err(gm, m)
+    assert rel_err(gv, v) <= 2 * TOL, rel_err(gv, v)
+    assert rel_err(gp, P) <= TOL, rel_err(gp, P)
+
+
 def test_ppo_single_step_parity():
     """One minibatch step: Adam's first moment after one step is
     (1 - beta1) * the clipped gradient, so it exposes the gradient itself."""
@@ -601,41 +632,60 @@ def test_ppo_single_step_parity():
     gp, gm, gv, gs = _run_ppo(wl, ppo, params, buf, adv, ret)
     P, m, v, t, st = _oracle_ppo(wl, ppo, params, buf, adv, ret)
     assert t == 1
-    assert rel_err(gm, m) <= TOL
-    assert rel_err(gv, v) <= 2 * TOL
-    assert rel_err(gp, P) <= TOL
-    for k in (1, 2, 5, 6):   # value loss, entropy, total loss, grad norm
-        assert abs(gs[k] - st[k]) <= TOL * max(abs(st[k]), 1e-3), (k, gs[k], st[k])
-    assert abs(gs[0] - st[0]) <= 1e-5 * max(abs(st[0]), 1.0)   # pg loss is ~0 at rho = 1
+    assert_update_fp32(gp, gm, gv, P, m, v)
+    assert_stats(gs, st, 8192)
+    # first step: the policy is the rollout's, rho = 1 on both sides
+    assert abs(gs[3]) < 1e-9 and gs[4] == 0.0 and st[4] == 0.0
 
 
-def test_ppo_ragged_minibatches():
-    """3 steps over minibatches of 3000, 3000 and 2192 samples."""
+@pytest.mark.parametrize("clip", [0.2, 0.01])
+def test_ppo_ragged_minibatches(clip):
+    """3 steps over minibatches of 3000, 3000 and 2192 samples; the small clip
+    range makes the later steps clip a share of their samples."""
     wl = W.make_tiny()
     params, buf, adv, ret = _ppo_inputs(wl, 128, seed=1)
-    ppo = W.PPOSpec(epochs=1, minibatch=3000)
+    ppo = W.PPOSpec(epochs=1, minibatch=3000, clip=clip)
     gp, gm, gv, gs = _run_ppo(wl, ppo, params, buf, adv, ret, iteration=5)
     P, m, v, t, st = _oracle_ppo(wl, ppo, params, buf, adv, ret, iteration=5)
     assert t == 3 and gs[7] == 3
-    assert rel_err(gp, P) <= 1e-4
-    assert rel_err(gm, m) <= 1e-3
+    assert_update_fp32(gp, gm, gv, P, m, v)
+    assert_stats(gs, st, 2192)
+    assert st[3] > 0.0
 
 
-def test_ppo_full_update_tiny():
+@pytest.mark.parametrize("clip", [0.2, 0.01])
+def test_ppo_full_update_tiny(clip):
     """4 epochs x 4 minibatches (ragged last one: 8192 = 3*2500 + 692)."""
     wl = W.make_tiny()
     params, buf, adv, ret = _ppo_inputs(wl, 128, seed=3)
-    ppo = W.PPOSpec(epochs=4, minibatch=2500)
+    ppo = W.PPOSpec(epochs=4, minibatch=2500, clip=clip)
     gp, gm, gv, gs = _run_ppo(wl, ppo, params, buf, adv, ret, iteration=2)
     P, m, v, t, st = _oracle_ppo(wl, ppo, params, buf, adv, ret, iteration=2)
     assert t == 16 and gs[7] == 16
-    # Adam normalises each step by sqrt(v): a parameter whose gradient is
-    # within rounding of zero can move by up to lr either way, so the
-    # end-of-update comparison is on the parameter vector as a whole
-    dp, dref = gp - params, P - params
-    assert np.linalg.norm(dp - dref) <= 1e-3 * np.linalg.norm(dref)
-    assert rel_err(gp, P) <= 1e-4
-    assert abs(gs[1] - st[1]) <= 1e-4 * abs(st[1])
+    assert_update_fp32(gp, gm, gv, P, m, v)
+    assert_stats(gs, st, 692)
+    if clip < 0.1:
+        assert st[4] > 0.05   # the clip fraction is exercised
+
+
+@pytest.mark.parametrize("clip,lr,ent", [(0.2, 3e-4, 0.0), (0.01, 3e-4, 0.0), (0.2, 3e-3, 0.01)])
+def test_ppo_7b_multi_epoch_persistent(clip, lr, ent):
+    """The 7B networks (16-128-128x5, the persistent update kernel that the
+    benchmark runs for 1,024 steps per launch) over 2 epochs x 3 minibatches
+    (3000, 3000, 2192) of 8,192 samples: from the second step on, every CTA
+    reads the weight images that the previous step's Adam phase rewrote.
+    Parameters, both moments and all statistics against the oracle."""
+    wl = W.make_7b(n_envs=128)
+    params, buf, adv, ret = _ppo_inputs(wl, 64, seed=4)
+    ppo = W.PPOSpec(epochs=2, minibatch=3000, clip=clip, lr=lr, ent_coef=ent)
+    gp, gm, gv, gs = _run_ppo(wl, ppo, params, buf, adv, ret, iteration=1)
+    P, m, v, t, st = _oracle_ppo(wl, ppo, params, buf, adv, ret, iteration=1)
+    assert t == 6 and gs[7] == 6
+    assert_update_fp32(gp, gm, gv, P, m, v)
+    assert_stats(gs, st, 2192)
+    assert st[3] > 0.0
+    if clip < 0.1 or lr > 1e-3:
+        assert st[4] > 0.05
 
 
 def test_ppo_7b_first_steps():
@@ -645,6 +695,7 @@ def test_ppo_7b_first_steps():
     gp, gm, gv, gs = _run_ppo(wl, ppo, params, buf, adv, ret)
     P, m, v, t, st = _oracle_ppo(wl, ppo, params, buf, adv, ret)
     assert rel_err(gm, m) <= TOL and rel_err(gp, P) <= TOL
+    assert_stats(gs, st, 32768)
 
 
 @pytest.mark.parametrize("n", [60, 1000, 4999, 8192])
@@ -666,17 +717,19 @@ def test_ppo_7b_single_step_partitions(n):
     P, m, v, t, st = _oracle_ppo(wl, ppo, params, sub, a_, r_)
     assert t == 1 and gs[7] == 1
     assert rel_err(gm, m) <= TOL and rel_err(gp, P) <= TOL
-    for k in (1, 2, 6):   # value loss, entropy, grad norm
-        assert abs(gs[k] - st[k]) <= TOL * max(abs(st[k]), 1e-3), (k, gs[k], st[k])
+    assert_stats(gs, st, n)
 
 
 # ------------------------------------------------------------------ bf16 PPO
+BF16_TOL = 2e-2
+
+
 @pytest.mark.parametrize("preset,E,T", [("72b", 64, 64), ("stress", 32, 64)])
 def test_ppo_bf16_single_step(preset, E, T):
     """One minibatch over all N = T*E samples of a bf16 network: tensor-core
-    forward over the permuted rows, cuBLASLt backward products, own loss,
-    reduction and Adam.  Adam's first moment after one step is 0.1 x the
-    clipped gradient."""
+    forward over the permuted rows, tensor-core backward, own loss, reduction
+    and Adam.  Adam's first moment after one step is 0.1 x the clipped
+    gradient."""
     wl = W.make_72b(n_envs=E) if preset == "72b" else W.make_stress(n_envs=E, horizon=T)
     params, buf, adv, ret = _ppo_inputs(wl, T, seed=2)
     ppo = W.PPOSpec(epochs=1, minibatch=T * E, ent_coef=0.01)
@@ -684,21 +737,34 @@ def test_ppo_bf16_single_step(preset, E, T):
     P, m, v, t, st = _oracle_ppo(wl, ppo, params, buf, adv, ret, iteration=1)
     assert t == 1 and gs[7] == 1
     assert bf16_ok(gm, m), (np.abs(gm - m).max() / np.abs(m).max())
-    for k in (1, 2, 6):   # value loss, entropy, grad norm
-        assert abs(gs[k] - st[k]) <= 2e-2 * max(abs(st[k]), 1e-3), (k, gs[k], st[k])
+    assert_stats(gs, st, T * E, tol=BF16_TOL)
 
 
-def test_ppo_bf16_ragged_epochs_72b():
-    """2 epochs x 3 minibatches (1500, 1500, 1096) on the 72B network."""
-    wl = W.make_72b(n_envs=64)
-    params, buf, adv, ret = _ppo_inputs(wl, 64, seed=4)
-    ppo = W.PPOSpec(epochs=2, minibatch=1500, ent_coef=0.01)
+@pytest.mark.parametrize("preset,E,mb,clip", [("72b", 64, 1500, 0.2), ("72b", 64, 1500, 0.01),
+                                              ("stress", 32, 900, 0.01)])
+def test_ppo_bf16_ragged_epochs(preset, E, mb, clip):
+    """2 epochs x 3 ragged minibatches of T * E = 64 * E samples (72B: 1500,
+    1500, 1096; Stress: 900, 900, 248).  The oracle emulates the GPU's bf16
+    rounding points, so what remains is fp32 against fp64 accumulation and
+    rare 1-ulp rounding flips: the moments, the parameters and their moves
+    from the start must agree within the benchmark spec's 2e-2 (rms-floored
+    relative; the moves measured 1.4e-2 on the 72B networks, the rest about
+    2e-4), and the first moment also within 1e-3, which a dropped term or a
+    wrongly scaled gradient exceeds."""
+    T = 64
+    wl = W.make_72b(n_envs=E) if preset == "72b" else W.make_stress(n_envs=E, horizon=T)
+    params, buf, adv, ret = _ppo_inputs(wl, T, seed=4)
+    ppo = W.PPOSpec(epochs=2, minibatch=mb, ent_coef=0.01, clip=clip)
     gp, gm, gv, gs = _run_ppo(wl, ppo, params, buf, adv, ret, iteration=3)
     P, m, v, t, st = _oracle_ppo(wl, ppo, params, buf, adv, ret, iteration=3)
     assert t == 6 and gs[7] == 6
-    dp, dref = gp - params, P - params
-    assert np.linalg.norm(dp - dref) <= 0.1 * np.linalg.norm(dref), np.linalg.norm(dp - dref) / np.linalg.norm(dref)
-    assert abs(gs[1] - st[1]) <= 2e-2 * abs(st[1])
+    assert rel_err(gm, m) <= 1e-3, rel_err(gm, m)
+    assert rel_err(gv, v) <= BF16_TOL and rel_err(gp, P) <= BF16_TOL
+    assert rel_err(gp - params, P - params) <= BF16_TOL, rel_err(gp - params, P - params)
+    assert_stats(gs, st, T * E - 2 * mb, tol=BF16_TOL)
+    assert st[3] > 0.0
+    if clip < 0.1:
+        assert st[4] > 0.05
 
 
 # ------------------------------------------------------- baseline rule policies
