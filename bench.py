@@ -369,7 +369,6 @@ def run_ours(args, world, rank, local):
     r72b = run_72b(args, world, peaks) if args.r72b_steps > 0 else None
     gae_large = run_gae_large(args, world, peaks) if args.gae_large[0] > 0 else None
     tiny = run_tiny(args, world)
-    del tr
     torch.cuda.empty_cache()
     stress = run_stress(args, world, peaks, local) if args.stress[0] > 0 else None
 
