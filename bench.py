@@ -777,7 +777,7 @@ def run_72b_mixed(args, world):
 def run_72b_ppo(args, world, peaks, wl, buf, adv, ret):
     """bf16 PPO update of the 72B networks on the first K x 65,536 samples of
     the 72B rollout (one epoch, K minibatch steps): tensor-core forward over
-    the permuted rows, cuBLASLt backward products, own loss/reduction/Adam.
+    the permuted rows, tensor-core backward products, own loss/reduction/Adam.
     Reports samples/s and the whole step's bf16 FLOP rate against the
     measured sustained bf16 peak."""
     from paper_2608_11226_gb300 import pe

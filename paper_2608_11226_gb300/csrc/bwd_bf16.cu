@@ -1,0 +1,562 @@
+// Backward pass of the bf16 policy/value networks (72B: 32-256-256x16,
+// Stress: 64-512-512x16) on the tcgen05 tensor cores, for the PPO update
+// (Sec. 4.2).  With z = W3 h2 + b3, h2 = tanh(W2 h1 + b2), h1 = tanh(W1 x + b1)
+// and dz = dLoss/dz per sample (from the loss kernel), the update needs
+//   da2 = bf16(dz W3 (1 - h2^2)),  da1 = bf16(da2 W2 (1 - h1^2))   (per sample)
+//   dW2 = da2^T h1, db2 = sum da2, dW1 = da1^T x, db1 = sum da1,
+//   dW3 = dz^T h2                                                (over samples)
+// with fp32 accumulation everywhere and bf16 at the rounding points the
+// oracle emulates (dz, da2 and da1 enter the products as bf16).
+//
+// Every per-sample operand lives in global memory as a 128-row "tile image",
+// byte for byte the swizzled shared-memory layout the kernels use (see
+// tc.cuh), so that each operand tile arrives with one bulk copy:
+//   x, h1, h2, da2, da1: K-major over features, 128-byte rows, H/64 blocks
+//   (x: D = 32 in 64-byte rows); dz: 16 bf16 in 32-byte rows.
+// Read with samples as the reduction dimension, the same bytes are the
+// MN-major operands of the weight-gradient products.
+//
+// bwd_data_kernel (one 128-sample tile at a time, persistent):
+//   dh2 = dz W3 (one MMA per 256 columns, K = 16) -> TMEM; epilogue:
+//   da2 = bf16(dh2 (1 - h2^2)) into shared memory (the next A operand) and
+//   its tile image; dh1 = da2 W2 with W2^T streamed through a two-slot ring
+//   of 32 KB stages by a producer warp; epilogue: da1 = bf16(dh1 (1 - h1^2))
+//   to its tile image.
+// wgrad_kernel (split over samples): each CTA owns 128 output rows (one
+//   block of layer outputs o) of one network and one 256-column chunk, and
+//   accumulates over its share of the minibatch, 64 samples per stage:
+//   [dW2 | db2] = da2^T [h1 | 1], and for column chunk 0 also
+//   [dW1 | db1] = da1^T [x | 1] and dW3^T = h2^T dz; it writes its fp32
+//   accumulators as one partial block.  wgrad_reduce_kernel sums the partial
+//   blocks of every output in a fixed order (deterministic) into the
+//   canonical gradient vector.
+#include <algorithm>
+
+#include "mlp_f32.cuh"
+#include "tc.cuh"
+
+namespace pe {
+
+extern __device__ int32_t g_tc_error;
+
+constexpr int kBwRows = 128;            // samples per tile (MMA M of the data products)
+constexpr int kBwStage = 32768;         // one streamed W2^T stage: 256 rows x 64 K, SW128
+constexpr int kBwCompute = 512;         // 16 compute warps
+constexpr int kBwThreads = kBwCompute + 32;  // + the producer warp
+
+// backward weight image of one network: W3^T (H rows x 16, K-major SW32),
+// then the W2^T stages: stage (h, kb) = rows i in [256 h, 256 h + 256) of
+// W2^T, K = o in [64 kb, 64 kb + 64), K-major SW128
+template <int H>
+struct BwdImg {
+  static constexpr int W3T = H * 32;
+  static constexpr int NH = H / 256, KB = H / 64, STAGES = NH * KB;
+  static constexpr int TOTAL = W3T + STAGES * kBwStage;
+  static_assert(W3T % 1024 == 0, "stages start on a swizzle atom");
+};
+
+int64_t bwd_image_bytes(int H) {
+  if (H == 256) return BwdImg<256>::TOTAL;
+  if (H == 512) return BwdImg<512>::TOTAL;
+  return -1;
+}
+
+template <int D, int H>
+__global__ void bwd_image_kernel(const float* __restrict__ params, int A, int value_net, uint8_t* __restrict__ img) {
+  using I = BwdImg<H>;
+  const MlpLayout Lp = mlp_layout(D, H, A);
+  const float* w2 = params + (value_net ? Lp.v2 : Lp.w2);
+  const float* w3 = params + (value_net ? Lp.v3 : Lp.w3);
+  const int nout = value_net ? 1 : A;
+  const int total = H * 16 + H * H;
+  for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < total; i += gridDim.x * blockDim.x) {
+    if (i < H * 16) {
+      const int o = i / 16, a = i % 16;  // W3^T[o][a] = W3[a][o]
+      const float v = a < nout ? w3[(int64_t)a * H + o] : 0.0f;
+      *reinterpret_cast<__nv_bfloat16*>(img + tc::swz_offset<32>(o, a, H)) = __float2bfloat16_rn(v);
+    } else {
+      const int j = i - H * 16, o = j / H, c = j % H;  // W2[o][c] = W2^T[c][o]
+      const int stage = (c / 256) * I::KB + o / 64;
+      *reinterpret_cast<__nv_bfloat16*>(img + I::W3T + stage * kBwStage + tc::swz_offset<128>(c % 256, o % 64, 256)) =
+          __float2bfloat16_rn(w2[j]);
+    }
+  }
+}
+
+template <int H>
+struct BwdSmem {
+  alignas(1024) uint8_t da2[kBwRows * H * 2];  // A operand of dh1 = da2 W2 (K-major SW128)
+  alignas(1024) uint8_t ring[2][kBwStage];
+  alignas(1024) uint8_t w3t[H * 32];           // B operand of dh2 = dz W3 (K-major SW32)
+  alignas(1024) uint8_t dz[kBwRows * 32];      // A operand of dh2 (K-major SW32)
+  uint64_t full[2], empty[2], bar_mma, bar_w;
+  uint32_t tmem_base;
+  int32_t err;
+};
+
+__device__ __forceinline__ void bw_compute_sync() { asm volatile("bar.sync 1, 512;" ::: "memory"); }
+
+// d = bf16(g (1 - h^2)) for 16 columns: g from TMEM, h (bf16) from a tile image
+__device__ __forceinline__ void tanh_grad16(const float (&g)[16], const uint8_t* hrow, uint32_t o0, uint32_t o1,
+                                            bool valid, uint32_t (&pk)[8]) {
+  const uint4 a = *reinterpret_cast<const uint4*>(hrow + o0);
+  const uint4 b = *reinterpret_cast<const uint4*>(hrow + o1);
+  const uint32_t hw[8] = {a.x, a.y, a.z, a.w, b.x, b.y, b.z, b.w};
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    const float h0 = __uint_as_float(hw[i] << 16), h1 = __uint_as_float(hw[i] & 0xFFFF0000u);
+    pk[i] = valid ? tc::pack_bf16(g[2 * i] * (1.0f - h0 * h0), g[2 * i + 1] * (1.0f - h1 * h1)) : 0u;
+  }
+}
+
+struct BwdArgs {
+  const uint8_t* img;   // backward weight image of the network
+  const uint8_t* dz;    // dz tile images (4 KB per tile)
+  const uint8_t* h1;    // h1 tile images
+  const uint8_t* h2;    // h2 tile images
+  uint8_t* da2;         // out: da2 tile images
+  uint8_t* da1;         // out: da1 tile images
+  int64_t n;            // valid samples
+  int32_t* err;
+};
+
+template <int H>
+__global__ void __launch_bounds__(kBwThreads, 1) bwd_data_kernel(BwdArgs g) {
+  using I = BwdImg<H>;
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
+  BwdSmem<H>& s = *reinterpret_cast<BwdSmem<H>*>(base);
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  if (tid == 0) {
+    s.err = 0;
+    for (int i = 0; i < 2; ++i) {
+      tc::mbar_init(&s.full[i], 1);
+      tc::mbar_init(&s.empty[i], 1);
+    }
+    tc::mbar_init(&s.bar_mma, 1);
+    tc::mbar_init(&s.bar_w, 1);
+    tc::fence_mbar_init();
+  }
+  if (warp == 0) tc::tmem_alloc(&s.tmem_base, H);
+  tc::fence_before();
+  __syncthreads();
+  tc::fence_after();
+  const uint32_t tmem = s.tmem_base;
+  const int64_t tiles = (g.n + kBwRows - 1) / kBwRows;
+  const int my_tiles = (int)((tiles - blockIdx.x + gridDim.x - 1) / gridDim.x);
+  if (tid == 0) {
+    tc::mbar_expect_tx(&s.bar_w, (uint32_t)I::W3T);
+    tc::bulk_g2s(s.w3t, g.img, (uint32_t)I::W3T, &s.bar_w);
+  }
+  int last_issued = -1;  // producer: global index of its last issued stage
+  if (warp == kBwCompute / 32) {
+    // producer: the W2^T stages of every tile, in consumption order
+    if (lane == 0) {
+      int gs = 0;
+      for (int t = 0; t < my_tiles; ++t) {
+        for (int st = 0; st < I::STAGES; ++st, ++gs) {
+          const int slot = gs & 1;
+          if (gs >= 2 && !tc::mbar_wait(&s.empty[slot], ((gs - 2) >> 1) & 1)) {
+            atomicExch(&s.err, 1);
+            t = my_tiles;
+            break;
+          }
+          tc::mbar_expect_tx(&s.full[slot], (uint32_t)kBwStage);
+          tc::bulk_g2s(s.ring[slot], g.img + I::W3T + (int64_t)st * kBwStage, (uint32_t)kBwStage, &s.full[slot]);
+          last_issued = gs;
+        }
+      }
+    }
+  } else {
+    if (!tc::mbar_wait(&s.bar_w, 0)) atomicExch(&s.err, 1);
+    const bool issuer = (tid == 32);
+    const uint32_t da2a = tc::smem_u32(s.da2), dza = tc::smem_u32(s.dz), w3a = tc::smem_u32(s.w3t);
+    const uint32_t r0a = tc::smem_u32(s.ring[0]), r1a = tc::smem_u32(s.ring[1]);
+    constexpr uint32_t kIdN = tc::idesc_bf16(kBwRows, 256);
+    uint32_t phase = 0;
+    int gs = 0;
+    const int quad = warp & 3, slice = warp >> 2, row = quad * 32 + lane;
+    const uint32_t lane_addr = tmem + ((uint32_t)(quad * 32) << 16);
+    for (int t = 0; t < my_tiles; ++t) {
+      // every compute thread takes the same decision (a named barrier with an OR)
+      if (tc::bar_any(1, kBwCompute, s.err != 0)) break;
+      const int64_t tile = blockIdx.x + (int64_t)t * gridDim.x;
+      const int nr = (int)(g.n - tile * kBwRows < kBwRows ? g.n - tile * kBwRows : kBwRows);
+      const bool valid = row < nr;
+      // dz tile (4 KB, already in the SW32 layout)
+      if (tid < kBwRows * 2)
+        reinterpret_cast<uint4*>(s.dz)[tid] = __ldg(reinterpret_cast<const uint4*>(g.dz + tile * (kBwRows * 32)) + tid);
+      tc::fence_async_smem();
+      bw_compute_sync();
+      // dh2 (TMEM cols 0..H) = dz W3: one K = 16 MMA per 256 columns
+      if (issuer) {
+        tc::fence_after();
+#pragma unroll
+        for (int h = 0; h < I::NH; ++h)
+          tc::mma_bf16(tmem + h * 256, tc::desc_strided(dza, 16, 256, tc::kLayoutSW32),
+                       tc::desc_strided(w3a + h * 256 * 32, 16, 256, tc::kLayoutSW32), kIdN, 0);
+        tc::mma_commit(&s.bar_mma);
+      }
+      if (!tc::mbar_wait(&s.bar_mma, phase)) atomicExch(&s.err, 1);
+      phase ^= 1;
+      tc::fence_after();
+      // da2 = bf16(dh2 (1 - h2^2)): shared-memory A tile and its tile image
+      {
+        const uint8_t* h2t = g.h2 + tile * (int64_t)(kBwRows * H * 2);
+        uint8_t* outt = g.da2 + tile * (int64_t)(kBwRows * H * 2);
+#pragma unroll 1
+        for (int j = 0; j < H / 4 / 16; ++j) {
+          const int c = slice * (H / 4) + j * 16;
+          float v[16];
+          tc::tmem_ld16(lane_addr + (uint32_t)c, v);
+          const uint32_t o0 = tc::swz_offset<128>(row, c, kBwRows), o1 = tc::swz_offset<128>(row, c + 8, kBwRows);
+          uint32_t pk[8];
+          tanh_grad16(v, h2t, o0, o1, valid, pk);
+          const uint4 lo = make_uint4(pk[0], pk[1], pk[2], pk[3]), hi = make_uint4(pk[4], pk[5], pk[6], pk[7]);
+          *reinterpret_cast<uint4*>(s.da2 + o0) = lo;
+          *reinterpret_cast<uint4*>(s.da2 + o1) = hi;
+          *reinterpret_cast<uint4*>(outt + o0) = lo;
+          *reinterpret_cast<uint4*>(outt + o1) = hi;
+        }
+      }
+      tc::fence_before();
+      tc::fence_async_smem();
+      bw_compute_sync();
+      // dh1 (TMEM cols 0..H) = da2 W2, W2^T streamed: stage (h, kb)
+      if (issuer) {
+        tc::fence_after();
+        for (int h = 0; h < I::NH; ++h)
+          for (int kb = 0; kb < I::KB; ++kb) {
+            const int slot = gs & 1;
+            if (!tc::mbar_wait(&s.full[slot], (gs >> 1) & 1)) atomicExch(&s.err, 1);
+            tc::fence_after();
+            const uint32_t ra = slot ? r1a : r0a;
+#pragma unroll
+            for (int kk = 0; kk < 4; ++kk)
+              tc::mma_bf16(tmem + h * 256, tc::desc_kmajor(da2a + kb * kBwRows * 128 + kk * 32, 1024, tc::kLayoutSW128),
+                           tc::desc_kmajor(ra + kk * 32, 1024, tc::kLayoutSW128), kIdN, (kb | kk) != 0);
+            tc::mma_commit(&s.empty[slot]);
+            ++gs;
+          }
+        tc::mma_commit(&s.bar_mma);
+      }
+      if (!tc::mbar_wait(&s.bar_mma, phase)) atomicExch(&s.err, 1);
+      phase ^= 1;
+      tc::fence_after();
+      // da1 = bf16(dh1 (1 - h1^2)) to its tile image
+      {
+        const uint8_t* h1t = g.h1 + tile * (int64_t)(kBwRows * H * 2);
+        uint8_t* outt = g.da1 + tile * (int64_t)(kBwRows * H * 2);
+#pragma unroll 1
+        for (int j = 0; j < H / 4 / 16; ++j) {
+          const int c = slice * (H / 4) + j * 16;
+          float v[16];
+          tc::tmem_ld16(lane_addr + (uint32_t)c, v);
+          const uint32_t o0 = tc::swz_offset<128>(row, c, kBwRows), o1 = tc::swz_offset<128>(row, c + 8, kBwRows);
+          uint32_t pk[8];
+          tanh_grad16(v, h1t, o0, o1, valid, pk);
+          *reinterpret_cast<uint4*>(outt + o0) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+          *reinterpret_cast<uint4*>(outt + o1) = make_uint4(pk[4], pk[5], pk[6], pk[7]);
+        }
+      }
+      tc::fence_before();
+      bw_compute_sync();
+    }
+  }
+  __syncthreads();
+  // on an error, the producer waits (bounded) for its last copy before the
+  // CTA leaves, so that no bulk copy into this CTA's shared memory is in flight
+  if (s.err && warp == kBwCompute / 32 && lane == 0 && last_issued >= 0)
+    (void)tc::mbar_wait(&s.full[last_issued & 1], (last_issued >> 1) & 1);
+  if (tid == 0 && s.err) {
+    atomicExch(&g_tc_error, 1);
+    if (g.err) atomicExch(g.err, 1);
+  }
+  __syncthreads();
+  if (warp == 0) tc::tmem_dealloc(tmem, H);
+}
+
+// ---------------------------------------------------------------------------
+// weight gradients: split over samples, 64 samples per stage
+// ---------------------------------------------------------------------------
+constexpr int kWgSamples = 64;
+constexpr int kWgThreads = 128;
+// stage layout (bytes): A da2 | A da1 | A h2 (each 2 blocks of 64 features x
+// 64 samples), B h1 (4 blocks: 256 columns), B x (64 samples x D), B dz
+constexpr int kWgA = 2 * kWgSamples * 128;  // 16 KB
+constexpr int kWgDa2 = 0, kWgDa1 = kWgA, kWgH2 = 2 * kWgA, kWgH1 = 3 * kWgA;
+constexpr int kWgX = kWgH1 + 4 * kWgSamples * 128;        // 80 KB
+constexpr int kWgDz = kWgX + kWgSamples * 128;            // x takes at most 8 KB
+constexpr int kWgStageBytes = kWgDz + kWgSamples * 32;    // 90 KB
+constexpr int kWgMaxCols = 256 + 16 + 64 + 16 + 16;       // dW2 | db2 | dW1 | db1 | dW3^T
+
+template <int D>
+struct WgCols {  // TMEM / partial-block column of each product
+  static constexpr int DW2 = 0, DB2 = 256, DW1 = 272, DB1 = 272 + D, DW3 = 288 + D, NC0 = 304 + D;
+};
+
+struct WgSmem {
+  alignas(1024) uint8_t st[2][kWgStageBytes];
+  alignas(1024) uint8_t ones[512];  // 16 samples x 16 columns of bf16 ones (B of the bias sums)
+  uint64_t full[2], empty[2], bar_mma;
+  uint32_t tmem_base;
+  int32_t err;
+};
+
+struct WgNet {
+  const uint8_t *da2, *da1, *h1, *h2, *dz;  // tile images
+};
+
+struct WgArgs {
+  WgNet net[2];
+  const uint8_t* x;   // shared input tile images
+  int64_t n;          // valid samples
+  int nstages;        // ceil(n / 64)
+  int spc;            // stages per CTA
+  int S;              // sample chunks (CTAs per group)
+  float* part;        // [groups * S][128][kWgMaxCols]
+  int32_t* err;
+};
+
+template <int D, int H>
+__global__ void __launch_bounds__(kWgThreads, 1) wgrad_kernel(WgArgs g) {
+  using Cn = WgCols<D>;
+  constexpr int NCH = H / 256, MB = H / 128;
+  constexpr int XB = D * 2;                    // x row bytes (64 or 128)
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
+  WgSmem& s = *reinterpret_cast<WgSmem*>(base);
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int grp = blockIdx.x / g.S, chunk = blockIdx.x % g.S;
+  const int ni = grp / (MB * NCH), mb = (grp / NCH) % MB, nc = grp % NCH;
+  const bool first = nc == 0;  // column chunk 0 also takes dW1, db1, dW3^T
+  const WgNet& nt = g.net[ni];
+  const int k0 = chunk * g.spc, k1 = min(k0 + g.spc, g.nstages);
+  if (tid == 0) {
+    s.err = 0;
+    for (int i = 0; i < 2; ++i) {
+      tc::mbar_init(&s.full[i], 1);
+      tc::mbar_init(&s.empty[i], 1);
+    }
+    tc::mbar_init(&s.bar_mma, 1);
+    tc::fence_mbar_init();
+  }
+  for (int i = tid; i < 512 / 4; i += kWgThreads) reinterpret_cast<uint32_t*>(s.ones)[i] = 0x3F803F80u;
+  if (warp == 0) tc::tmem_alloc(&s.tmem_base, 512);
+  tc::fence_async_smem();
+  tc::fence_before();
+  __syncthreads();
+  tc::fence_after();
+  const uint32_t tmem = s.tmem_base;
+  const int64_t hb = (int64_t)kWgSamples * 128;  // bytes of one 64-sample half of a 128-row block
+  int last_issued = -1;
+  if (warp == 0) {
+    if (lane == 0) {
+      for (int k = k0; k < k1; ++k) {
+        const int j = k - k0, slot = j & 1;
+        if (j >= 2 && !tc::mbar_wait(&s.empty[slot], ((j - 2) >> 1) & 1)) {
+          atomicExch(&s.err, 1);
+          break;
+        }
+        const int64_t tile = k >> 1, half = k & 1;
+        const int64_t tb = tile * (int64_t)(kBwRows * H * 2);  // tile image base of a hidden-width operand
+        uint8_t* d = s.st[slot];
+        const uint32_t bytes = (uint32_t)(2 * hb + 4 * hb + (first ? 4 * hb + kWgSamples * XB + kWgSamples * 32 : 0));
+        tc::mbar_expect_tx(&s.full[slot], bytes);
+        for (int q = 0; q < 2; ++q) {
+          const int64_t off = tb + (int64_t)(2 * mb + q) * kBwRows * 128 + half * hb;
+          tc::bulk_g2s(d + kWgDa2 + q * hb, nt.da2 + off, (uint32_t)hb, &s.full[slot]);
+          if (first) {
+            tc::bulk_g2s(d + kWgDa1 + q * hb, nt.da1 + off, (uint32_t)hb, &s.full[slot]);
+            tc::bulk_g2s(d + kWgH2 + q * hb, nt.h2 + off, (uint32_t)hb, &s.full[slot]);
+          }
+        }
+        for (int q = 0; q < 4; ++q) {
+          const int64_t off = tb + (int64_t)(4 * nc + q) * kBwRows * 128 + half * hb;
+          tc::bulk_g2s(d + kWgH1 + q * hb, nt.h1 + off, (uint32_t)hb, &s.full[slot]);
+        }
+        if (first) {
+          tc::bulk_g2s(d + kWgX, g.x + tile * (int64_t)(kBwRows * XB) + half * kWgSamples * XB,
+                       (uint32_t)(kWgSamples * XB), &s.full[slot]);
+          tc::bulk_g2s(d + kWgDz, nt.dz + tile * (int64_t)(kBwRows * 32) + half * kWgSamples * 32,
+                       (uint32_t)(kWgSamples * 32), &s.full[slot]);
+        }
+        last_issued = j;
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      const uint32_t onea = tc::smem_u32(s.ones);
+      constexpr uint32_t kIdW2 = tc::idesc_bf16_mn(128, 256, 1, 1);
+      constexpr uint32_t kId16 = tc::idesc_bf16_mn(128, 16, 1, 1);
+      constexpr uint32_t kIdD = tc::idesc_bf16_mn(128, D, 1, 1);
+      constexpr uint32_t kXLayout = D == 32 ? tc::kLayoutSW64 : tc::kLayoutSW128;
+      constexpr uint32_t kXAtom = D == 32 ? 512 : 1024;
+      const uint64_t ones = tc::desc_strided(onea, 16, 256, tc::kLayoutSW32);
+      for (int k = k0; k < k1; ++k) {
+        const int j = k - k0, slot = j & 1;
+        if (!tc::mbar_wait(&s.full[slot], (j >> 1) & 1)) {
+          atomicExch(&s.err, 1);
+          break;
+        }
+        tc::fence_after();
+        const uint32_t sa = tc::smem_u32(s.st[slot]);
+#pragma unroll
+        for (int kk = 0; kk < kWgSamples / 16; ++kk) {
+          const uint32_t acc = (j | kk) != 0;
+          const uint64_t a2 = tc::desc_strided(sa + kWgDa2 + kk * 2048, (uint32_t)hb, 1024, tc::kLayoutSW128);
+          tc::mma_bf16(tmem + Cn::DW2, a2, tc::desc_strided(sa + kWgH1 + kk * 2048, (uint32_t)hb, 1024, tc::kLayoutSW128),
+                       kIdW2, acc);
+          if (first) {
+            tc::mma_bf16(tmem + Cn::DB2, a2, ones, kId16, acc);
+            const uint64_t a1 = tc::desc_strided(sa + kWgDa1 + kk * 2048, (uint32_t)hb, 1024, tc::kLayoutSW128);
+            tc::mma_bf16(tmem + Cn::DW1, a1,
+                         tc::desc_strided(sa + kWgX + kk * 16 * XB, 16, kXAtom, kXLayout), kIdD, acc);
+            tc::mma_bf16(tmem + Cn::DB1, a1, ones, kId16, acc);
+            tc::mma_bf16(tmem + Cn::DW3, tc::desc_strided(sa + kWgH2 + kk * 2048, (uint32_t)hb, 1024, tc::kLayoutSW128),
+                         tc::desc_strided(sa + kWgDz + kk * 512, 16, 256, tc::kLayoutSW32), kId16, acc);
+          }
+        }
+        tc::mma_commit(&s.empty[slot]);
+      }
+      tc::mma_commit(&s.bar_mma);
+    }
+  }
+  // epilogue: the accumulators of this CTA's 128 output rows
+  __syncwarp();
+  const bool have = k1 > k0;
+  if (have && !tc::mbar_wait(&s.bar_mma, 0)) atomicExch(&s.err, 1);
+  tc::fence_after();
+  __syncthreads();
+  {
+    const int row = warp * 32 + lane;
+    float* prow = g.part + ((int64_t)blockIdx.x * 128 + row) * kWgMaxCols;
+    const int ncols = first ? Cn::NC0 : 256;
+    const uint32_t lane_addr = tmem + ((uint32_t)(warp * 32) << 16);
+    for (int c = 0; c < ncols; c += 16) {
+      float v[16];
+      tc::tmem_ld16(lane_addr + (uint32_t)c, v);
+#pragma unroll
+      for (int q = 0; q < 4; ++q)
+        *reinterpret_cast<float4*>(prow + c + 4 * q) =
+            (have && !s.err) ? make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3])
+                             : make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+    }
+  }
+  tc::fence_before();
+  __syncthreads();
+  if (s.err && warp == 0 && lane == 0 && last_issued >= 0)
+    (void)tc::mbar_wait(&s.full[last_issued & 1], (last_issued >> 1) & 1);
+  if (tid == 0 && s.err) {
+    atomicExch(&g_tc_error, 1);
+    if (g.err) atomicExch(g.err, 1);
+  }
+  __syncthreads();
+  if (warp == 0) tc::tmem_dealloc(tmem, 512);
+}
+
+// grad <- sum over the S sample chunks of each partial block, in chunk order
+template <int D, int H>
+__global__ void wgrad_reduce_kernel(const float* __restrict__ part, int S, int A, float* __restrict__ grad) {
+  using Cn = WgCols<D>;
+  constexpr int NCH = H / 256, MB = H / 128;
+  const MlpLayout Lp = mlp_layout(D, H, A);
+  const int64_t total = (int64_t)2 * MB * NCH * 128 * kWgMaxCols;
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < total; i += (int64_t)gridDim.x * blockDim.x) {
+    const int col = (int)(i % kWgMaxCols);
+    const int row = (int)((i / kWgMaxCols) % 128);
+    const int grp = (int)(i / ((int64_t)kWgMaxCols * 128));
+    const int ni = grp / (MB * NCH), mb = (grp / NCH) % MB, nc = grp % NCH;
+    const int o = mb * 128 + row;
+    const int nout = ni ? 1 : A;
+    int64_t dst = -1;
+    if (col < 256) {
+      dst = (ni ? Lp.v2 : Lp.w2) + (int64_t)o * H + nc * 256 + col;
+    } else if (nc == 0) {
+      if (col == Cn::DB2) dst = (ni ? Lp.c2 : Lp.b2) + o;
+      else if (col >= Cn::DW1 && col < Cn::DW1 + D) dst = (ni ? Lp.v1 : Lp.w1) + (int64_t)o * D + (col - Cn::DW1);
+      else if (col == Cn::DB1) dst = (ni ? Lp.c1 : Lp.b1) + o;
+      else if (col >= Cn::DW3 && col < Cn::DW3 + nout) dst = (ni ? Lp.v3 : Lp.w3) + (int64_t)(col - Cn::DW3) * H + o;
+    }
+    if (dst < 0) continue;
+    const float* p = part + ((int64_t)grp * S * 128 + row) * kWgMaxCols + col;
+    float acc = 0.0f;
+    for (int k = 0; k < S; ++k) acc += p[(int64_t)k * 128 * kWgMaxCols];
+    grad[dst] = acc;
+  }
+}
+
+// ---------------------------------------------------------------------------
+// host side
+// ---------------------------------------------------------------------------
+// partial blocks for up to kWgMaxCtas CTAs (the launch keeps groups x S below it)
+constexpr int kWgMaxCtas = 256;
+int64_t wgrad_partial_bytes() { return (int64_t)kWgMaxCtas * 128 * kWgMaxCols * 4; }
+
+template <int D, int H>
+static pe_status bwd_launch(const float* params, int A, uint8_t* const img[2], const uint8_t* x,
+                            const uint8_t* const dz[2], const uint8_t* const h1[2], const uint8_t* const h2[2],
+                            uint8_t* const da2[2], uint8_t* const da1[2], int64_t n, float* part, float* grad,
+                            int32_t* err, cudaStream_t st) {
+  int dev = 0, sms = 0;
+  PE_TRY_CUDA(cudaGetDevice(&dev));
+  PE_TRY_CUDA(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
+  {
+    ProfScope ps(PE_PROF_PPO_OTHER, st);
+    for (int ni = 0; ni < 2; ++ni) bwd_image_kernel<D, H><<<128, 256, 0, st>>>(params, A, ni, img[ni]);
+  }
+  PE_CHECK_LAUNCH("bwd_image_kernel");
+  const int64_t tiles = (n + kBwRows - 1) / kBwRows;
+  {
+    auto kern = bwd_data_kernel<H>;
+    const int bytes = (int)sizeof(BwdSmem<H>) + 1024;
+    PE_TRY_CUDA(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes));
+    const int grid = (int)std::min<int64_t>(tiles, sms);
+    ProfScope ps(PE_PROF_PPO_GRAD, st);
+    for (int ni = 0; ni < 2; ++ni) {
+      BwdArgs a{img[ni], dz[ni], h1[ni], h2[ni], da2[ni], da1[ni], n, err};
+      kern<<<grid, kBwThreads, bytes, st>>>(a);
+    }
+  }
+  PE_CHECK_LAUNCH("bwd_data_kernel");
+  {
+    constexpr int groups = 2 * (H / 128) * (H / 256);
+    WgArgs a;
+    for (int ni = 0; ni < 2; ++ni) a.net[ni] = WgNet{da2[ni], da1[ni], h1[ni], h2[ni], dz[ni]};
+    a.x = x;
+    a.n = n;
+    a.nstages = (int)((n + kWgSamples - 1) / kWgSamples);
+    const int s_want = std::max(1, std::min(std::min(sms, kWgMaxCtas) / groups, a.nstages));
+    a.spc = (a.nstages + s_want - 1) / s_want;
+    a.S = (a.nstages + a.spc - 1) / a.spc;
+    a.part = part;
+    a.err = err;
+    auto kern = wgrad_kernel<D, H>;
+    const int bytes = (int)sizeof(WgSmem) + 1024;
+    PE_TRY_CUDA(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes));
+    ProfScope ps(PE_PROF_PPO_GRAD, st);
+    kern<<<groups * a.S, kWgThreads, bytes, st>>>(a);
+    PE_CHECK_LAUNCH("wgrad_kernel");
+    wgrad_reduce_kernel<D, H><<<std::min<int64_t>(4096, ceil_div((int64_t)groups * 128 * kWgMaxCols, 256)), 256, 0, st>>>(
+        part, a.S, A, grad);
+    PE_CHECK_LAUNCH("wgrad_reduce_kernel");
+  }
+  return PE_OK;
+}
+
+// the whole backward of both networks of a bf16 PPO minibatch step: writes
+// every weight and the hidden-layer biases of the gradient vector (the head
+// biases come from the loss kernel's partial sums)
+pe_status bf16_backward(const pe_net& net, const float* params, uint8_t* const img[2], const uint8_t* x,
+                        const uint8_t* const dz[2], const uint8_t* const h1[2], const uint8_t* const h2[2],
+                        uint8_t* const da2[2], uint8_t* const da1[2], int64_t n, float* part, float* grad,
+                        int32_t* err, cudaStream_t st) {
+  if (n <= 0) return PE_OK;
+  if (net.obs_dim == 32 && net.hidden == 256)
+    return bwd_launch<32, 256>(params, net.n_actions, img, x, dz, h1, h2, da2, da1, n, part, grad, err, st);
+  if (net.obs_dim == 64 && net.hidden == 512)
+    return bwd_launch<64, 512>(params, net.n_actions, img, x, dz, h1, h2, da2, da1, n, part, grad, err, st);
+  return fail(PE_EINVAL, "unsupported bf16 network for the backward pass");
+}
+
+}  // namespace pe

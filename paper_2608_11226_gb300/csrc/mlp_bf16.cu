@@ -27,13 +27,17 @@ namespace pe {
 __device__ int32_t g_tc_error = 0;
 
 // optional extras of a forward pass used by the PPO update: rows gathered
-// through an index array, and the bf16 input and hidden activations saved
-// row-major ([n][D], [n][H]) for the backward pass
+// through an index array, and the bf16 input and hidden activations saved for
+// the backward pass as "tile images": tile t (rows 128 t .. 128 t + 127) is
+// stored exactly as the kernel holds it in shared memory (K-major, swizzled:
+// x with 64- or 128-byte rows, h1 and h2 with 128-byte rows in H / 64
+// blocks), all 128 rows written (rows past n hold the finite activations of
+// a zero input), so that the backward kernels bulk-copy them as operands.
 struct MlpSave {
   const uint32_t* gather;  // row r of the tile reads obs row gather[r] (NULL: row r)
-  __nv_bfloat16* x;        // [n][D] or NULL
-  __nv_bfloat16* h1;       // [n][H] or NULL
-  __nv_bfloat16* h2;       // [n][H] or NULL
+  __nv_bfloat16* x;        // tiles of 128 x D, or NULL
+  __nv_bfloat16* h1;       // tiles of 128 x H, or NULL
+  __nv_bfloat16* h2;       // tiles of 128 x H, or NULL
 };
 
 constexpr int kTcRows = 128;     // rows (envs / samples) per tile, the MMA M
@@ -118,21 +122,22 @@ __device__ __forceinline__ void epi_compute(uint32_t tmem, int col0, const float
 
 template <int H>
 __device__ __forceinline__ void epi_store(const uint32_t (&pk)[H / 8], uint8_t* act,
-                                          __nv_bfloat16* gsave, int64_t r0, int nr) {
+                                          __nv_bfloat16* gsave, int64_t tile) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int quad = warp & 3, slice = warp >> 2;
   const int row = quad * 32 + lane;
+  uint8_t* g = gsave ? reinterpret_cast<uint8_t*>(gsave) + tile * (int64_t)(kTcRows * H * 2) : nullptr;
 #pragma unroll
   for (int j = 0; j < H / 64; ++j) {
     const int c = slice * (H / 4) + j * 16;
     const uint4 lo = make_uint4(pk[j * 8 + 0], pk[j * 8 + 1], pk[j * 8 + 2], pk[j * 8 + 3]);
     const uint4 hi = make_uint4(pk[j * 8 + 4], pk[j * 8 + 5], pk[j * 8 + 6], pk[j * 8 + 7]);
-    *reinterpret_cast<uint4*>(act + tc::swz_offset<128>(row, c, kTcRows)) = lo;
-    *reinterpret_cast<uint4*>(act + tc::swz_offset<128>(row, c + 8, kTcRows)) = hi;
-    if (gsave && row < nr) {
-      uint4* g = reinterpret_cast<uint4*>(gsave + (r0 + row) * H + c);
-      g[0] = lo;
-      g[1] = hi;
+    const uint32_t o0 = tc::swz_offset<128>(row, c, kTcRows), o1 = tc::swz_offset<128>(row, c + 8, kTcRows);
+    *reinterpret_cast<uint4*>(act + o0) = lo;
+    *reinterpret_cast<uint4*>(act + o1) = hi;
+    if (g) {
+      *reinterpret_cast<uint4*>(g + o0) = lo;
+      *reinterpret_cast<uint4*>(g + o1) = hi;
     }
   }
 }
@@ -183,7 +188,9 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   constexpr uint32_t kIdH = tc::idesc_bf16(kTcRows, kHeadN);
   uint32_t phase = 0, phase_hi = 0;
   const int64_t tiles = (n + kTcRows - 1) / kTcRows;
-  for (int64_t tile = blockIdx.x; tile < tiles && s.err == 0; tile += gridDim.x) {
+  for (int64_t tile = blockIdx.x; tile < tiles; tile += gridDim.x) {
+    // a wait that gave up stops every thread of the CTA at the same tile
+    if (__syncthreads_or(s.err != 0)) break;
     const int64_t r0 = tile * kTcRows;
     const int nr = (int)(n - r0 < kTcRows ? n - r0 : kTcRows);
     // observation tile -> X (D bf16 per row, swizzled like W1)
@@ -194,9 +201,11 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       if (r < nr) {
         const int64_t src = save.gather ? (int64_t)__ldg(save.gather + r0 + r) : r0 + r;
         v = __ldg(reinterpret_cast<const uint4*>(obs + src * D) + c);
-        if (save.x) *(reinterpret_cast<uint4*>(save.x + (r0 + r) * D) + c) = v;
       }
-      *reinterpret_cast<uint4*>(s.act + tc::swz_offset<I::RB1>(r, c * 8, kTcRows)) = v;
+      const uint32_t off = tc::swz_offset<I::RB1>(r, c * 8, kTcRows);
+      *reinterpret_cast<uint4*>(s.act + off) = v;
+      if (save.x)
+        *reinterpret_cast<uint4*>(reinterpret_cast<uint8_t*>(save.x) + tile * (int64_t)(kTcRows * D * 2) + off) = v;
     }
     tc::fence_async_smem();
     __syncthreads();
@@ -230,7 +239,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     if (!tc::mbar_wait(&s.bar_hi, phase_hi)) atomicExch(&s.err, 1);
     tc::fence_after();
     if (hi_half) epi_compute<H>(tmem, 0, s.b1, pk);
-    epi_store<H>(pk, s.act, save.h1, r0, nr);
+    epi_store<H>(pk, s.act, save.h1, tile);
     phase ^= 1;
     phase_hi ^= 1;
     tc::fence_before();
@@ -261,7 +270,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     if (!tc::mbar_wait(&s.bar_hi, phase_hi)) atomicExch(&s.err, 1);
     tc::fence_after();
     if (hi_half) epi_compute<H>(tmem, 256, s.b2, pk);
-    epi_store<H>(pk, s.act, save.h2, r0, nr);
+    epi_store<H>(pk, s.act, save.h2, tile);
     phase ^= 1;
     phase_hi ^= 1;
     tc::fence_before();
@@ -409,6 +418,7 @@ __global__ void __launch_bounds__(kStreamThreads, 1)
   const int64_t tiles = (n + kTcRows - 1) / kTcRows;
   const int my_tiles = (int)((tiles - blockIdx.x + gridDim.x - 1) / gridDim.x);
 
+  int last_issued = -1;  // producer: global index of its last issued stage
   if (warp == kComputeThreads / 32) {
     // producer: every stage of every tile of this CTA, in consumption order
     if (lane == 0) {
@@ -423,6 +433,7 @@ __global__ void __launch_bounds__(kStreamThreads, 1)
           }
           tc::mbar_expect_tx(&s.full[slot], (uint32_t)I::stage_bytes(st));
           tc::bulk_g2s(s.ring[slot], img + I::stage_off(st), (uint32_t)I::stage_bytes(st), &s.full[slot]);
+          last_issued = gs;
         }
       }
     }
@@ -437,7 +448,8 @@ __global__ void __launch_bounds__(kStreamThreads, 1)
     const int quad = warp & 3, slice = warp >> 2, row = quad * 32 + lane;
     const uint32_t lane_addr = tmem + ((uint32_t)(quad * 32) << 16);
     for (int t = 0; t < my_tiles; ++t) {
-      if (s.err) break;
+      // every compute thread takes the same decision (a named barrier with an OR)
+      if (tc::bar_any(1, kComputeThreads, s.err != 0)) break;
       const int64_t tile = blockIdx.x + (int64_t)t * gridDim.x;
       const int64_t rbase = tile * kTcRows;
       const int nr = (int)(n - rbase < kTcRows ? n - rbase : kTcRows);
@@ -448,9 +460,11 @@ __global__ void __launch_bounds__(kStreamThreads, 1)
         if (r < nr) {
           const int64_t src = save.gather ? (int64_t)__ldg(save.gather + rbase + r) : rbase + r;
           v = __ldg(reinterpret_cast<const uint4*>(obs + src * D) + c);
-          if (save.x) *(reinterpret_cast<uint4*>(save.x + (rbase + r) * D) + c) = v;
         }
-        *reinterpret_cast<uint4*>(s.act + tc::swz_offset<128>(r, c * 8, kTcRows)) = v;
+        const uint32_t off = tc::swz_offset<128>(r, c * 8, kTcRows);
+        *reinterpret_cast<uint4*>(s.act + off) = v;
+        if (save.x)
+          *reinterpret_cast<uint4*>(reinterpret_cast<uint8_t*>(save.x) + tile * (int64_t)(kTcRows * D * 2) + off) = v;
       }
       tc::fence_async_smem();
       compute_sync();
@@ -488,12 +502,13 @@ __global__ void __launch_bounds__(kStreamThreads, 1)
 #pragma unroll
         for (int i = 0; i < 8; ++i)
           p[i] = tc::pack_bf16(tanhf(v[2 * i] + s.b1[c + 2 * i]), tanhf(v[2 * i + 1] + s.b1[c + 2 * i + 1]));
-        *reinterpret_cast<uint4*>(s.act + tc::swz_offset<128>(row, c, kTcRows)) = make_uint4(p[0], p[1], p[2], p[3]);
-        *reinterpret_cast<uint4*>(s.act + tc::swz_offset<128>(row, c + 8, kTcRows)) = make_uint4(p[4], p[5], p[6], p[7]);
-        if (save.h1 && row < nr) {
-          uint4* g = reinterpret_cast<uint4*>(save.h1 + (rbase + row) * H + c);
-          g[0] = make_uint4(p[0], p[1], p[2], p[3]);
-          g[1] = make_uint4(p[4], p[5], p[6], p[7]);
+        const uint32_t o0 = tc::swz_offset<128>(row, c, kTcRows), o1 = tc::swz_offset<128>(row, c + 8, kTcRows);
+        *reinterpret_cast<uint4*>(s.act + o0) = make_uint4(p[0], p[1], p[2], p[3]);
+        *reinterpret_cast<uint4*>(s.act + o1) = make_uint4(p[4], p[5], p[6], p[7]);
+        if (save.h1) {
+          uint8_t* g = reinterpret_cast<uint8_t*>(save.h1) + tile * (int64_t)(kTcRows * H * 2);
+          *reinterpret_cast<uint4*>(g + o0) = make_uint4(p[0], p[1], p[2], p[3]);
+          *reinterpret_cast<uint4*>(g + o1) = make_uint4(p[4], p[5], p[6], p[7]);
         }
       }
       tc::fence_before();
@@ -524,12 +539,13 @@ __global__ void __launch_bounds__(kStreamThreads, 1)
 #pragma unroll
         for (int i = 0; i < 8; ++i)
           p[i] = tc::pack_bf16(tanhf(v[2 * i] + s.b2[c + 2 * i]), tanhf(v[2 * i + 1] + s.b2[c + 2 * i + 1]));
-        *reinterpret_cast<uint4*>(s.act + tc::swz_offset<128>(row, c, kTcRows)) = make_uint4(p[0], p[1], p[2], p[3]);
-        *reinterpret_cast<uint4*>(s.act + tc::swz_offset<128>(row, c + 8, kTcRows)) = make_uint4(p[4], p[5], p[6], p[7]);
-        if (save.h2 && row < nr) {
-          uint4* g = reinterpret_cast<uint4*>(save.h2 + (rbase + row) * H + c);
-          g[0] = make_uint4(p[0], p[1], p[2], p[3]);
-          g[1] = make_uint4(p[4], p[5], p[6], p[7]);
+        const uint32_t o0 = tc::swz_offset<128>(row, c, kTcRows), o1 = tc::swz_offset<128>(row, c + 8, kTcRows);
+        *reinterpret_cast<uint4*>(s.act + o0) = make_uint4(p[0], p[1], p[2], p[3]);
+        *reinterpret_cast<uint4*>(s.act + o1) = make_uint4(p[4], p[5], p[6], p[7]);
+        if (save.h2) {
+          uint8_t* g = reinterpret_cast<uint8_t*>(save.h2) + tile * (int64_t)(kTcRows * H * 2);
+          *reinterpret_cast<uint4*>(g + o0) = make_uint4(p[0], p[1], p[2], p[3]);
+          *reinterpret_cast<uint4*>(g + o1) = make_uint4(p[4], p[5], p[6], p[7]);
         }
       }
       tc::fence_before();
@@ -567,10 +583,15 @@ __global__ void __launch_bounds__(kStreamThreads, 1)
     }
   }
   __syncthreads();
+  // on an error, the producer waits (bounded) for its last copy before the
+  // CTA leaves, so that no bulk copy into this CTA's shared memory is in flight
+  if (s.err && warp == kComputeThreads / 32 && lane == 0 && last_issued >= 0)
+    (void)tc::mbar_wait(&s.full[last_issued & 1], (last_issued >> 1) & 1);
   if (tid == 0 && s.err) {
     atomicExch(&g_tc_error, 1);
     if (err) atomicExch(err, 1);
   }
+  __syncthreads();
   if (warp == 0) tc::tmem_dealloc(tmem, 512);
 }
 

@@ -18,21 +18,31 @@ __device__ __forceinline__ uint32_t smem_u32(const void* p) {
 // XOR-ed with bits [7, 7+b)):
 //   SW128: rows of 128 B (64 bf16), 8-row atoms of 1024 B, b = 3
 //   SW64 : rows of  64 B (32 bf16), 8-row atoms of  512 B, b = 2
+//   SW32 : rows of  32 B (16 bf16), 8-row atoms of  256 B, b = 1
 // Element (r, k) of a tile with R rows and K columns (bf16) lives in K-block
-// kb = k / KB (KB = 64 or 32 elements) at byte
+// kb = k / KB (KB = 64, 32 or 16 elements) at byte
 //   kb * R * RB + r * RB + (((k % KB) / 8) ^ ((r % 8) >> s)) * 16 + (k % 8) * 2
-// with RB the row bytes and s = 0 for SW128, s = 1 for SW64; the atom base must
-// be aligned to the atom size.
-enum : uint32_t { kLayoutSW128 = 2, kLayoutSW64 = 4 };
+// with RB the row bytes and s = 0 for SW128, 1 for SW64, 2 for SW32; the atom
+// base must be aligned to the atom size.
+enum : uint32_t { kLayoutSW128 = 2, kLayoutSW64 = 4, kLayoutSW32 = 6 };
 
 template <int RB>
 __host__ __device__ __forceinline__ uint32_t swz_offset(int r, int k, int R) {
+  static_assert(RB == 128 || RB == 64 || RB == 32, "row bytes of a swizzled layout");
   constexpr int KB = RB / 2;  // bf16 elements per row of a K-block
   const int kb = k / KB, kk = k % KB;
   const int chunk = kk / 8;
-  const int phys = RB == 128 ? (chunk ^ (r & 7)) : (chunk ^ ((r >> 1) & 3));
+  const int phys = RB == 128 ? (chunk ^ (r & 7)) : RB == 64 ? (chunk ^ ((r >> 1) & 3)) : (chunk ^ ((r >> 2) & 1));
   return (uint32_t)(kb * R * RB + r * RB + phys * 16 + (kk % 8) * 2);
 }
+
+// The same bytes serve as an MN-major operand.  A tile stored as above with
+// rows = K (samples) and contiguous elements = M or N (features) is the
+// canonical MN-major swizzled layout: the 128/64/32-byte rows hold 64/32/16
+// consecutive M (or N) elements of one K index, XOR-swizzled within 8-row
+// atoms.  Its descriptor takes two strides: LBO = bytes between atoms that
+// are adjacent along M/N (the next 64/32/16 elements), SBO = bytes between
+// 8-row groups along K.
 
 // tcgen05 shared-memory matrix descriptor, K-major, swizzled:
 // start address >> 4 [0,14), leading-dim byte offset >> 4 [16,30) (unused
@@ -48,9 +58,28 @@ __device__ __forceinline__ uint64_t desc_kmajor(uint32_t saddr, uint32_t sbo_byt
   return d;
 }
 
+// shared-memory matrix descriptor with both byte strides given (MN-major
+// operands, and K-major SW32 tiles): start >> 4 at [0,14), LBO >> 4 at
+// [16,30), SBO >> 4 at [32,46), 0b001 at [46,49), layout type at [61,64)
+__device__ __forceinline__ uint64_t desc_strided(uint32_t saddr, uint32_t lbo_bytes, uint32_t sbo_bytes,
+                                                 uint32_t layout) {
+  uint64_t d = 0;
+  d |= (uint64_t)((saddr >> 4) & 0x3FFFu);
+  d |= (uint64_t)((lbo_bytes >> 4) & 0x3FFFu) << 16;
+  d |= (uint64_t)((sbo_bytes >> 4) & 0x3FFFu) << 32;
+  d |= (uint64_t)1u << 46;
+  d |= (uint64_t)(layout & 7u) << 61;
+  return d;
+}
+
 // instruction descriptor for kind::f16 with bf16 A and B, fp32 D, both K-major
 __host__ __device__ constexpr uint32_t idesc_bf16(int M, int N) {
   return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
+}
+
+// the same with A and/or B MN-major (bits 15 and 16 of the descriptor)
+__host__ __device__ constexpr uint32_t idesc_bf16_mn(int M, int N, int a_mn, int b_mn) {
+  return idesc_bf16(M, N) | ((uint32_t)(a_mn & 1) << 15) | ((uint32_t)(b_mn & 1) << 16);
 }
 
 __device__ __forceinline__ void mma_bf16(uint32_t tmem_d, uint64_t da, uint64_t db, uint32_t idesc,
@@ -99,6 +128,22 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, float (&v)[16]) {
   asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 #pragma unroll
   for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+// named barrier `id` over `nthreads` threads that also ORs a predicate across
+// them: every thread gets the same answer, so a loop can stop uniformly
+__device__ __forceinline__ bool bar_any(int id, int nthreads, bool pred) {
+  uint32_t r;
+  asm volatile(
+      "{\n\t.reg .pred p, q;\n\t"
+      "setp.ne.u32 p, %1, 0;\n\t"
+      "bar.red.or.pred q, %2, %3, p;\n\t"
+      "selp.u32 %0, 1, 0, q;\n\t"
+      "}\n"
+      : "=r"(r)
+      : "r"((uint32_t)pred), "r"(id), "r"(nthreads)
+      : "memory");
+  return r != 0;
 }
 
 // ---------------------------------------------------------------- mbarriers
