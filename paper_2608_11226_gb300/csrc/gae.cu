@@ -9,9 +9,9 @@
 // affine map A_start = alpha + beta * A_end, warp 0 chains the chunk maps
 // through shared memory, and each thread then re-runs its chunk with the
 // right carry-in and streams A and R out.  Longer horizons loop over
-// super-chunks of CL*NW steps from the end.  The launch shape is chosen from
-// the problem size (measured on GB300: 69% of the HBM roofline at
-// 2,048 x 262,144, 54% at 1,024 x 65,536).
+// super-chunks of CL*NW steps from the end.  That time-parallel form serves
+// narrow batches; batches of 32,768 envs or more take the barrier-free
+// per-column kernel below.
 #include <type_traits>
 
 #include "common.cuh"
@@ -128,6 +128,81 @@ __global__ void __launch_bounds__(32 * NW)
 }
 
 
+// Wide batches (E >= 32,768): one thread per V envs walks the whole horizon
+// backwards, A_t = delta_t + gamma lambda (1 - d_t) A_{t+1} in the same
+// order as the recursion, with no barrier and no shared memory.  The loads of
+// the next P steps are kept in flight in a register ring, so each SM holds
+// enough outstanding bytes to cover HBM latency; every warp streams
+// 32 * V consecutive envs of a row (coalesced).
+template <int V, int P>
+__global__ void __launch_bounds__(128)
+    gae_stream_kernel(const float* __restrict__ r, const float* __restrict__ v, const uint8_t* __restrict__ d,
+                      const float* __restrict__ last_v, int T, int E, float gamma, float lam,
+                      float* __restrict__ adv, float* __restrict__ ret) {
+  using FV = typename std::conditional<V == 2, float2, float>::type;
+  using BV = typename std::conditional<V == 2, uchar2, unsigned char>::type;
+  const int e0 = (blockIdx.x * blockDim.x + threadIdx.x) * V;
+  if (e0 >= E) return;
+  const float gl = gamma * lam;
+  FV rb[P], vb[P];
+  BV db[P];
+  auto load = [&](int k, int t) {
+    const int64_t o = (int64_t)t * E + e0;
+    rb[k] = __ldcs(reinterpret_cast<const FV*>(r + o));
+    vb[k] = __ldcs(reinterpret_cast<const FV*>(v + o));
+    db[k] = __ldcs(reinterpret_cast<const BV*>(d + o));
+  };
+#pragma unroll
+  for (int k = 0; k < P; ++k)
+    if (T - 1 - k >= 0) load(k, T - 1 - k);
+  float A[V], vn[V];
+  {
+    const FV q = *reinterpret_cast<const FV*>(last_v + e0);
+    const float* qp = reinterpret_cast<const float*>(&q);
+#pragma unroll
+    for (int u = 0; u < V; ++u) {
+      A[u] = 0.0f;
+      vn[u] = qp[u];
+    }
+  }
+  for (int base = T - 1; base >= 0; base -= P) {
+#pragma unroll
+    for (int k = 0; k < P; ++k) {
+      const int t = base - k;
+      if (t >= 0) {
+        const float* rp = reinterpret_cast<const float*>(&rb[k]);
+        const float* vp = reinterpret_cast<const float*>(&vb[k]);
+        const unsigned char* dp = reinterpret_cast<const unsigned char*>(&db[k]);
+        float ao[V], ro[V];
+#pragma unroll
+        for (int u = 0; u < V; ++u) {
+          const float nt = 1.0f - (float)dp[u];
+          const float delta = rp[u] + gamma * vn[u] * nt - vp[u];
+          A[u] = delta + gl * nt * A[u];
+          ao[u] = A[u];
+          ro[u] = A[u] + vp[u];
+          vn[u] = vp[u];
+        }
+        if (t - P >= 0) load(k, t - P);
+        const int64_t o = (int64_t)t * E + e0;
+        __stcs(reinterpret_cast<FV*>(adv + o), *reinterpret_cast<FV*>(ao));
+        __stcs(reinterpret_cast<FV*>(ret + o), *reinterpret_cast<FV*>(ro));
+      }
+    }
+  }
+}
+
+template <int V, int P>
+static pe_status gae_stream_run(const float* r, const float* v, const uint8_t* d, const float* last_v, int T,
+                                int E, float gamma, float lam, float* adv, float* ret, cudaStream_t st) {
+  {
+    ProfScope ps(PE_PROF_GAE, st);
+    gae_stream_kernel<V, P><<<ceil_div(E / V, 128), 128, 0, st>>>(r, v, d, last_v, T, E, gamma, lam, adv, ret);
+  }
+  PE_CHECK_LAUNCH("gae_stream_kernel");
+  return PE_OK;
+}
+
 template <int CL, int NW, int V>
 static pe_status gae_run(const float* r, const float* v, const uint8_t* d, const float* last_v, int T,
                          int E, float gamma, float lam, float* adv, float* ret, cudaStream_t st) {
@@ -151,6 +226,8 @@ pe_status gae_launch(const float* r, const float* v, const uint8_t* d, const flo
                                       reinterpret_cast<uintptr_t>(adv) | reinterpret_cast<uintptr_t>(ret) |
                                       reinterpret_cast<uintptr_t>(last_v)) % 8 == 0) &&
                    reinterpret_cast<uintptr_t>(d) % 2 == 0;
+  if (E >= 131072 && al2) return gae_stream_run<2, 12>(r, v, d, last_v, T, E, gamma, lam, adv, ret, st);
+  if (E >= 32768) return gae_stream_run<1, 16>(r, v, d, last_v, T, E, gamma, lam, adv, ret, st);
   if (n >= ((int64_t)1 << 28) && al4) return gae_run<4, 8, 4>(r, v, d, last_v, T, E, gamma, lam, adv, ret, st);
   if (E >= 16384 && al2) return gae_run<4, 16, 2>(r, v, d, last_v, T, E, gamma, lam, adv, ret, st);
   return gae_run<8, 32, 1>(r, v, d, last_v, T, E, gamma, lam, adv, ret, st);

@@ -71,11 +71,15 @@ def test_gae_parity(T, E):
     assert rel_err(cpu(ret), rr) <= TOL
 
 
-@pytest.mark.parametrize("T,E", [(64, 16384), (2048, 131072)])
+@pytest.mark.parametrize("T,E", [(64, 16384), (2048, 131072), (1024, 65536), (37, 32771), (300, 131074),
+                                 (5, 262144)])
 def test_gae_parity_vector_paths(T, E):
-    """The 2- and 4-env-per-thread vector kernels (chosen for E >= 16,384 and
-    T*E >= 2^28); envs are independent, so the oracle checks sampled columns
-    including both ends of a 128-env CTA span."""
+    """The wide-batch kernels: the 2-env-per-thread chunked kernel
+    (16,384 <= E < 32,768) and the per-column streaming kernel (E >= 32,768;
+    2 envs per thread from 131,072 when aligned, else 1), with ragged CTA
+    spans (32,771 and 131,074 envs), horizons shorter than, equal to and not a
+    multiple of its 16- or 12-step load ring.  Envs are independent, so the
+    oracle checks sampled columns including both ends of a CTA span."""
     g = torch.Generator(device="cuda").manual_seed(E)
     r = torch.randn(T, E, device="cuda", generator=g)
     v = torch.randn(T, E, device="cuda", generator=g)
@@ -86,7 +90,7 @@ def test_gae_parity_vector_paths(T, E):
     pe.gae(r, v, d, lv, 0.99, 0.95, adv, ret)
     torch.cuda.synchronize()
     rng = np.random.default_rng(T)
-    cols = np.unique(np.concatenate([[0, 1, 127, 128, E - 1], rng.choice(E, 59, replace=False)]))
+    cols = np.unique(np.concatenate([[0, 1, 127, 128, 255, 256, E - 2, E - 1], rng.choice(E, 59, replace=False)]))
     ci = torch.from_numpy(cols).cuda()
     ra, rr = O.gae(cpu(r[:, ci]), cpu(v[:, ci]), cpu(d[:, ci]), cpu(lv[ci]), 0.99, 0.95)
     assert rel_err(cpu(adv[:, ci]), ra) <= TOL
