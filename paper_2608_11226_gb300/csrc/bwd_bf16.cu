@@ -62,8 +62,11 @@ int64_t bwd_image_bytes(int H) {
 }
 
 template <int D, int H>
-__global__ void bwd_image_kernel(const float* __restrict__ params, int A, int value_net, uint8_t* __restrict__ img) {
+__global__ void bwd_image_kernel(const float* __restrict__ params, int A, uint8_t* __restrict__ img0,
+                                 uint8_t* __restrict__ img1) {
   using I = BwdImg<H>;
+  const int value_net = (int)blockIdx.y;  // y = 0 policy, 1 value
+  uint8_t* img = value_net ? img1 : img0;
   const MlpLayout Lp = mlp_layout(D, H, A);
   const float* w2 = params + (value_net ? Lp.v2 : Lp.w2);
   const float* w3 = params + (value_net ? Lp.v3 : Lp.w3);
@@ -96,11 +99,10 @@ struct BwdSmem {
 
 __device__ __forceinline__ void bw_compute_sync() { asm volatile("bar.sync 1, 512;" ::: "memory"); }
 
-// d = bf16(g (1 - h^2)) for 16 columns: g from TMEM, h (bf16) from a tile image
-__device__ __forceinline__ void tanh_grad16(const float (&g)[16], const uint8_t* hrow, uint32_t o0, uint32_t o1,
-                                            bool valid, uint32_t (&pk)[8]) {
-  const uint4 a = *reinterpret_cast<const uint4*>(hrow + o0);
-  const uint4 b = *reinterpret_cast<const uint4*>(hrow + o1);
+// d = bf16(g (1 - h^2)) for 16 columns: g from TMEM, h as 16 packed bf16
+__device__ __forceinline__ void tanh_grad16(const float (&g)[16], const uint4 (&h)[2], bool valid,
+                                            uint32_t (&pk)[8]) {
+  const uint4 a = h[0], b = h[1];
   const uint32_t hw[8] = {a.x, a.y, a.z, a.w, b.x, b.y, b.z, b.w};
 #pragma unroll
   for (int i = 0; i < 8; ++i) {
@@ -121,7 +123,7 @@ struct BwdArgs {
 };
 
 template <int H>
-__global__ void __launch_bounds__(kBwThreads, 1) bwd_data_kernel(BwdArgs g) {
+__global__ void __maxnreg__(120) bwd_data_kernel(BwdArgs g) {
   using I = BwdImg<H>;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
@@ -177,15 +179,39 @@ __global__ void __launch_bounds__(kBwThreads, 1) bwd_data_kernel(BwdArgs g) {
     int gs = 0;
     const int quad = warp & 3, slice = warp >> 2, row = quad * 32 + lane;
     const uint32_t lane_addr = tmem + ((uint32_t)(quad * 32) << 16);
+    // Loads run ahead of their use: the next tile's dz chunk is fetched while
+    // this tile runs, and each epilogue fetches its first PF activation
+    // chunks (h2, then h1; 32 bytes per 16 columns) before it waits for its
+    // MMAs, then refills the slot it just used, so global latency overlaps
+    // the tensor core instead of stalling the epilogue.
+    constexpr int NJ = H / 4 / 16;              // 16-column chunks per thread
+    constexpr int PF = NJ < 4 ? NJ : 4;         // chunks in flight
+    const int tile0 = blockIdx.x;
+    uint4 dzv = make_uint4(0, 0, 0, 0);
+    if (tid < kBwRows * 2 && my_tiles > 0)
+      dzv = __ldg(reinterpret_cast<const uint4*>(g.dz + (int64_t)tile0 * (kBwRows * 32)) + tid);
+    auto hload = [&](const uint8_t* ht, int j, uint4 (&dst)[2]) {
+      const int c = slice * (H / 4) + j * 16;
+      dst[0] = __ldg(reinterpret_cast<const uint4*>(ht + tc::swz_offset<128>(row, c, kBwRows)));
+      dst[1] = __ldg(reinterpret_cast<const uint4*>(ht + tc::swz_offset<128>(row, c + 8, kBwRows)));
+    };
     for (int t = 0; t < my_tiles; ++t) {
       // every compute thread takes the same decision (a named barrier with an OR)
       if (tc::bar_any(1, kBwCompute, s.err != 0)) break;
       const int64_t tile = blockIdx.x + (int64_t)t * gridDim.x;
       const int nr = (int)(g.n - tile * kBwRows < kBwRows ? g.n - tile * kBwRows : kBwRows);
       const bool valid = row < nr;
-      // dz tile (4 KB, already in the SW32 layout)
-      if (tid < kBwRows * 2)
-        reinterpret_cast<uint4*>(s.dz)[tid] = __ldg(reinterpret_cast<const uint4*>(g.dz + tile * (kBwRows * 32)) + tid);
+      const uint8_t* h2t = g.h2 + tile * (int64_t)(kBwRows * H * 2);
+      const uint8_t* h1t = g.h1 + tile * (int64_t)(kBwRows * H * 2);
+      uint4 hb[PF][2];
+#pragma unroll
+      for (int j = 0; j < PF; ++j) hload(h2t, j, hb[j]);
+      // dz tile (4 KB, already in the SW32 layout), then the next tile's
+      if (tid < kBwRows * 2) {
+        reinterpret_cast<uint4*>(s.dz)[tid] = dzv;
+        if (t + 1 < my_tiles)
+          dzv = __ldg(reinterpret_cast<const uint4*>(g.dz + (tile + gridDim.x) * (kBwRows * 32)) + tid);
+      }
       tc::fence_async_smem();
       bw_compute_sync();
       // dh2 (TMEM cols 0..H) = dz W3: one K = 16 MMA per 256 columns
@@ -202,16 +228,16 @@ __global__ void __launch_bounds__(kBwThreads, 1) bwd_data_kernel(BwdArgs g) {
       tc::fence_after();
       // da2 = bf16(dh2 (1 - h2^2)): shared-memory A tile and its tile image
       {
-        const uint8_t* h2t = g.h2 + tile * (int64_t)(kBwRows * H * 2);
         uint8_t* outt = g.da2 + tile * (int64_t)(kBwRows * H * 2);
-#pragma unroll 1
-        for (int j = 0; j < H / 4 / 16; ++j) {
+#pragma unroll
+        for (int j = 0; j < NJ; ++j) {
           const int c = slice * (H / 4) + j * 16;
           float v[16];
           tc::tmem_ld16(lane_addr + (uint32_t)c, v);
           const uint32_t o0 = tc::swz_offset<128>(row, c, kBwRows), o1 = tc::swz_offset<128>(row, c + 8, kBwRows);
           uint32_t pk[8];
-          tanh_grad16(v, h2t, o0, o1, valid, pk);
+          tanh_grad16(v, hb[j % PF], valid, pk);
+          if (j + PF < NJ) hload(h2t, j + PF, hb[j % PF]);
           const uint4 lo = make_uint4(pk[0], pk[1], pk[2], pk[3]), hi = make_uint4(pk[4], pk[5], pk[6], pk[7]);
           *reinterpret_cast<uint4*>(s.da2 + o0) = lo;
           *reinterpret_cast<uint4*>(s.da2 + o1) = hi;
@@ -219,6 +245,9 @@ __global__ void __launch_bounds__(kBwThreads, 1) bwd_data_kernel(BwdArgs g) {
           *reinterpret_cast<uint4*>(outt + o1) = hi;
         }
       }
+      // the h1 chunks of the second epilogue, in flight during the dh1 MMAs
+#pragma unroll
+      for (int j = 0; j < PF; ++j) hload(h1t, j, hb[j]);
       tc::fence_before();
       tc::fence_async_smem();
       bw_compute_sync();
@@ -245,16 +274,16 @@ __global__ void __launch_bounds__(kBwThreads, 1) bwd_data_kernel(BwdArgs g) {
       tc::fence_after();
       // da1 = bf16(dh1 (1 - h1^2)) to its tile image
       {
-        const uint8_t* h1t = g.h1 + tile * (int64_t)(kBwRows * H * 2);
         uint8_t* outt = g.da1 + tile * (int64_t)(kBwRows * H * 2);
-#pragma unroll 1
-        for (int j = 0; j < H / 4 / 16; ++j) {
+#pragma unroll
+        for (int j = 0; j < NJ; ++j) {
           const int c = slice * (H / 4) + j * 16;
           float v[16];
           tc::tmem_ld16(lane_addr + (uint32_t)c, v);
           const uint32_t o0 = tc::swz_offset<128>(row, c, kBwRows), o1 = tc::swz_offset<128>(row, c + 8, kBwRows);
           uint32_t pk[8];
-          tanh_grad16(v, h1t, o0, o1, valid, pk);
+          tanh_grad16(v, hb[j % PF], valid, pk);
+          if (j + PF < NJ) hload(h1t, j + PF, hb[j % PF]);
           *reinterpret_cast<uint4*>(outt + o0) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
           *reinterpret_cast<uint4*>(outt + o1) = make_uint4(pk[4], pk[5], pk[6], pk[7]);
         }
@@ -503,7 +532,7 @@ static pe_status bwd_launch(const float* params, int A, uint8_t* const img[2], c
   PE_TRY_CUDA(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
   {
     ProfScope ps(PE_PROF_PPO_OTHER, st);
-    for (int ni = 0; ni < 2; ++ni) bwd_image_kernel<D, H><<<128, 256, 0, st>>>(params, A, ni, img[ni]);
+    bwd_image_kernel<D, H><<<dim3(128, 2), 256, 0, st>>>(params, A, img[0], img[1]);
   }
   PE_CHECK_LAUNCH("bwd_image_kernel");
   const int64_t tiles = (n + kBwRows - 1) / kBwRows;

@@ -133,14 +133,17 @@ __global__ void __launch_bounds__(32 * NW)
 // order as the recursion, with no barrier and no shared memory.  The loads of
 // the next P steps are kept in flight in a register ring, so each SM holds
 // enough outstanding bytes to cover HBM latency; every warp streams
-// 32 * V consecutive envs of a row (coalesced).
+// 32 * V consecutive envs of a row (coalesced).  V grows with E so that all
+// threads are resident in one wave (about 14 warps per SM; a second, partly
+// filled wave cost a sixth of the bandwidth), and P shrinks as V grows so
+// that each SM keeps about 64 KB of loads in flight.
 template <int V, int P>
 __global__ void __launch_bounds__(128)
     gae_stream_kernel(const float* __restrict__ r, const float* __restrict__ v, const uint8_t* __restrict__ d,
                       const float* __restrict__ last_v, int T, int E, float gamma, float lam,
                       float* __restrict__ adv, float* __restrict__ ret) {
-  using FV = typename std::conditional<V == 2, float2, float>::type;
-  using BV = typename std::conditional<V == 2, uchar2, unsigned char>::type;
+  using FV = typename std::conditional<V == 4, float4, typename std::conditional<V == 2, float2, float>::type>::type;
+  using BV = typename std::conditional<V == 4, uchar4, typename std::conditional<V == 2, uchar2, unsigned char>::type>::type;
   const int e0 = (blockIdx.x * blockDim.x + threadIdx.x) * V;
   if (e0 >= E) return;
   const float gl = gamma * lam;
@@ -226,8 +229,10 @@ pe_status gae_launch(const float* r, const float* v, const uint8_t* d, const flo
                                       reinterpret_cast<uintptr_t>(adv) | reinterpret_cast<uintptr_t>(ret) |
                                       reinterpret_cast<uintptr_t>(last_v)) % 8 == 0) &&
                    reinterpret_cast<uintptr_t>(d) % 2 == 0;
-  if (E >= 131072 && al2) return gae_stream_run<2, 12>(r, v, d, last_v, T, E, gamma, lam, adv, ret, st);
-  if (E >= 32768) return gae_stream_run<1, 16>(r, v, d, last_v, T, E, gamma, lam, adv, ret, st);
+  if (E >= 196608 && al4) return gae_stream_run<4, 8>(r, v, d, last_v, T, E, gamma, lam, adv, ret, st);
+  if (E >= 98304 && al2) return gae_stream_run<2, 8>(r, v, d, last_v, T, E, gamma, lam, adv, ret, st);
+  if (E >= 49152) return gae_stream_run<1, 16>(r, v, d, last_v, T, E, gamma, lam, adv, ret, st);
+  if (E >= 32768) return gae_stream_run<1, 32>(r, v, d, last_v, T, E, gamma, lam, adv, ret, st);
   if (n >= ((int64_t)1 << 28) && al4) return gae_run<4, 8, 4>(r, v, d, last_v, T, E, gamma, lam, adv, ret, st);
   if (E >= 16384 && al2) return gae_run<4, 16, 2>(r, v, d, last_v, T, E, gamma, lam, adv, ret, st);
   return gae_run<8, 32, 1>(r, v, d, last_v, T, E, gamma, lam, adv, ret, st);

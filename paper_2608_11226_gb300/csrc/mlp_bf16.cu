@@ -62,9 +62,12 @@ struct Img {
 // (policy: W1 W2 W3 of A rows; value: V1 V2 V3 of 1 row), rows >= nout of the
 // head are zero.
 template <int D, int H>
-__global__ void weight_image_kernel(const float* __restrict__ params, int A, int value_net,
-                                    uint8_t* __restrict__ img) {
+__global__ void weight_image_kernel(const float* __restrict__ params, int A, int value_first,
+                                    uint8_t* __restrict__ img0, int64_t img_stride) {
   using I = Img<D, H>;
+  // blockIdx.y selects the network: value_first + y (0 policy, 1 value)
+  const int value_net = value_first + (int)blockIdx.y;
+  uint8_t* img = img0 + blockIdx.y * img_stride;
   const MlpLayout Lp = mlp_layout(D, H, A);
   const float* w1 = params + (value_net ? Lp.v1 : Lp.w1);
   const float* w2 = params + (value_net ? Lp.v2 : Lp.w2);
@@ -188,27 +191,43 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   constexpr uint32_t kIdH = tc::idesc_bf16(kTcRows, kHeadN);
   uint32_t phase = 0, phase_hi = 0;
   const int64_t tiles = (n + kTcRows - 1) / kTcRows;
+  // Observation tiles are fetched one tile ahead: each thread holds its
+  // 16-byte chunk(s) of the next tile in registers while the current tile's
+  // layers run, so the global load latency is off the critical path.
+  constexpr int CPR = D / 8;                         // 16-byte chunks per row
+  constexpr int XCH = kTcRows * CPR / kTcThreads;    // chunks per thread
+  static_assert(kTcRows * CPR % kTcThreads == 0, "observation chunks per thread");
+  uint4 xv[XCH];
+  auto fetch_x = [&](int64_t tl) {
+#pragma unroll
+    for (int q = 0; q < XCH; ++q) {
+      const int i = tid + q * kTcThreads, r = i / CPR, c = i % CPR;
+      const int64_t row = tl * kTcRows + r;
+      xv[q] = make_uint4(0, 0, 0, 0);
+      if (tl < tiles && row < n) {
+        const int64_t src = save.gather ? (int64_t)__ldg(save.gather + row) : row;
+        xv[q] = __ldg(reinterpret_cast<const uint4*>(obs + src * D) + c);
+      }
+    }
+  };
+  fetch_x(blockIdx.x);
   for (int64_t tile = blockIdx.x; tile < tiles; tile += gridDim.x) {
     // a wait that gave up stops every thread of the CTA at the same tile
     if (__syncthreads_or(s.err != 0)) break;
     const int64_t r0 = tile * kTcRows;
     const int nr = (int)(n - r0 < kTcRows ? n - r0 : kTcRows);
     // observation tile -> X (D bf16 per row, swizzled like W1)
-    constexpr int CPR = D / 8;  // 16-byte chunks per row
-    for (int i = tid; i < kTcRows * CPR; i += blockDim.x) {
-      const int r = i / CPR, c = i % CPR;
-      uint4 v = make_uint4(0, 0, 0, 0);
-      if (r < nr) {
-        const int64_t src = save.gather ? (int64_t)__ldg(save.gather + r0 + r) : r0 + r;
-        v = __ldg(reinterpret_cast<const uint4*>(obs + src * D) + c);
-      }
+#pragma unroll
+    for (int q = 0; q < XCH; ++q) {
+      const int i = tid + q * kTcThreads, r = i / CPR, c = i % CPR;
       const uint32_t off = tc::swz_offset<I::RB1>(r, c * 8, kTcRows);
-      *reinterpret_cast<uint4*>(s.act + off) = v;
+      *reinterpret_cast<uint4*>(s.act + off) = xv[q];
       if (save.x)
-        *reinterpret_cast<uint4*>(reinterpret_cast<uint8_t*>(save.x) + tile * (int64_t)(kTcRows * D * 2) + off) = v;
+        *reinterpret_cast<uint4*>(reinterpret_cast<uint8_t*>(save.x) + tile * (int64_t)(kTcRows * D * 2) + off) = xv[q];
     }
     tc::fence_async_smem();
     __syncthreads();
+    fetch_x(tile + gridDim.x);
     // Each layer's N = H outputs are issued as two halves of H/2 columns with
     // separate commits, so that the warps of the first column half run their
     // epilogue while the tensor core computes the second half.
@@ -342,9 +361,11 @@ struct ImgS {
 };
 
 template <int D, int H>
-__global__ void weight_image_stream_kernel(const float* __restrict__ params, int A, int value_net,
-                                           uint8_t* __restrict__ img) {
+__global__ void weight_image_stream_kernel(const float* __restrict__ params, int A, int value_first,
+                                           uint8_t* __restrict__ img0, int64_t img_stride) {
   using I = ImgS<D, H>;
+  const int value_net = value_first + (int)blockIdx.y;
+  uint8_t* img = img0 + blockIdx.y * img_stride;
   const MlpLayout Lp = mlp_layout(D, H, A);
   const float* w1 = params + (value_net ? Lp.v1 : Lp.w1);
   const float* w2 = params + (value_net ? Lp.v2 : Lp.w2);
@@ -720,11 +741,11 @@ static pe_status make_images(const float* params, int A, uint8_t* ws, cudaStream
   const int64_t img = NetKind<D, H>::kImgPad;
   ProfScope ps(PE_PROF_VALUE, st);
   if constexpr (NetKind<D, H>::kStream) {
-    if (policy) weight_image_stream_kernel<D, H><<<128, 256, 0, st>>>(params, A, 0, ws);
-    weight_image_stream_kernel<D, H><<<128, 256, 0, st>>>(params, A, 1, ws + img);
+    weight_image_stream_kernel<D, H><<<dim3(128, policy ? 2 : 1), 256, 0, st>>>(params, A, policy ? 0 : 1,
+                                                                                policy ? ws : ws + img, img);
   } else {
-    if (policy) weight_image_kernel<D, H><<<64, 256, 0, st>>>(params, A, 0, ws);
-    weight_image_kernel<D, H><<<64, 256, 0, st>>>(params, A, 1, ws + img);
+    weight_image_kernel<D, H><<<dim3(64, policy ? 2 : 1), 256, 0, st>>>(params, A, policy ? 0 : 1,
+                                                                        policy ? ws : ws + img, img);
   }
   PE_CHECK_LAUNCH("weight_image_kernel");
   return PE_OK;
