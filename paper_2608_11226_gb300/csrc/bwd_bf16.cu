@@ -123,7 +123,7 @@ struct BwdArgs {
 };
 
 template <int H>
-__global__ void __maxnreg__(120) bwd_data_kernel(BwdArgs g) {
+__global__ void __launch_bounds__(kBwThreads, 1) bwd_data_kernel(BwdArgs g) {
   using I = BwdImg<H>;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
@@ -185,7 +185,7 @@ __global__ void __maxnreg__(120) bwd_data_kernel(BwdArgs g) {
     // MMAs, then refills the slot it just used, so global latency overlaps
     // the tensor core instead of stalling the epilogue.
     constexpr int NJ = H / 4 / 16;              // 16-column chunks per thread
-    constexpr int PF = NJ < 4 ? NJ : 4;         // chunks in flight
+    constexpr int PF = H == 256 ? 4 : 2;        // chunks in flight (within the 96 registers of 17 warps)
     const int tile0 = blockIdx.x;
     uint4 dzv = make_uint4(0, 0, 0, 0);
     if (tid < kBwRows * 2 && my_tiles > 0)

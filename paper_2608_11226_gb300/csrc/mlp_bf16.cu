@@ -9,12 +9,12 @@
 //   - a persistent CTA copies the image into shared memory with one bulk copy
 //     (cp.async.bulk, completion on an mbarrier) and keeps it for all its tiles;
 //   - per layer one thread issues tcgen05.mma (M=128, K=16 per instruction)
-//     into TMEM; eight warps read the fp32 accumulators back (tcgen05.ld),
+//     into TMEM; sixteen warps read the fp32 accumulators back (tcgen05.ld),
 //     add the bias, apply tanh, round to bf16 and write the next layer's A
 //     operand into shared memory in the swizzled layout.
 // Precision: bf16 observations, weights and hidden activations, fp32
-// accumulation, fp32 bias and tanh -- the quantisation points the oracle
-// emulates.
+// accumulation, fp32 bias and the SFU's tanh, rounded to bf16 -- the
+// quantisation points the oracle emulates (with an exact tanh).
 #include <type_traits>
 
 #include "env.cuh"
@@ -119,7 +119,7 @@ __device__ __forceinline__ void epi_compute(uint32_t tmem, int col0, const float
     tc::tmem_ld16(lane_addr + (uint32_t)(col0 + c), v);
 #pragma unroll
     for (int i = 0; i < 8; ++i)
-      pk[j * 8 + i] = tc::pack_bf16(tanhf(v[2 * i] + bias[c + 2 * i]), tanhf(v[2 * i + 1] + bias[c + 2 * i + 1]));
+      pk[j * 8 + i] = tc::tanh_pack2(v[2 * i], v[2 * i + 1], *reinterpret_cast<const float2*>(bias + c + 2 * i));
   }
 }
 
@@ -522,7 +522,7 @@ __global__ void __launch_bounds__(kStreamThreads, 1)
         uint32_t p[8];
 #pragma unroll
         for (int i = 0; i < 8; ++i)
-          p[i] = tc::pack_bf16(tanhf(v[2 * i] + s.b1[c + 2 * i]), tanhf(v[2 * i + 1] + s.b1[c + 2 * i + 1]));
+          p[i] = tc::tanh_pack2(v[2 * i], v[2 * i + 1], *reinterpret_cast<const float2*>(s.b1 + c + 2 * i));
         const uint32_t o0 = tc::swz_offset<128>(row, c, kTcRows), o1 = tc::swz_offset<128>(row, c + 8, kTcRows);
         *reinterpret_cast<uint4*>(s.act + o0) = make_uint4(p[0], p[1], p[2], p[3]);
         *reinterpret_cast<uint4*>(s.act + o1) = make_uint4(p[4], p[5], p[6], p[7]);
@@ -559,7 +559,7 @@ __global__ void __launch_bounds__(kStreamThreads, 1)
         uint32_t p[8];
 #pragma unroll
         for (int i = 0; i < 8; ++i)
-          p[i] = tc::pack_bf16(tanhf(v[2 * i] + s.b2[c + 2 * i]), tanhf(v[2 * i + 1] + s.b2[c + 2 * i + 1]));
+          p[i] = tc::tanh_pack2(v[2 * i], v[2 * i + 1], *reinterpret_cast<const float2*>(s.b2 + c + 2 * i));
         const uint32_t o0 = tc::swz_offset<128>(row, c, kTcRows), o1 = tc::swz_offset<128>(row, c + 8, kTcRows);
         *reinterpret_cast<uint4*>(s.act + o0) = make_uint4(p[0], p[1], p[2], p[3]);
         *reinterpret_cast<uint4*>(s.act + o1) = make_uint4(p[4], p[5], p[6], p[7]);
