@@ -133,10 +133,11 @@ __global__ void __launch_bounds__(32 * NW)
 // order as the recursion, with no barrier and no shared memory.  The loads of
 // the next P steps are kept in flight in a register ring, so each SM holds
 // enough outstanding bytes to cover HBM latency; every warp streams
-// 32 * V consecutive envs of a row (coalesced).  V grows with E so that all
-// threads are resident in one wave (about 14 warps per SM; a second, partly
-// filled wave cost a sixth of the bandwidth), and P shrinks as V grows so
-// that each SM keeps about 64 KB of loads in flight.
+// 32 * V consecutive envs of a row (coalesced).  Measured on GB300: one env
+// per thread with 16 loads in flight reaches 74% of the HBM copy peak at
+// 65,536 envs (14 warps per SM); at 262,144 envs four envs per thread (8
+// steps in flight) keep the launch to one wave and reach 77%, where two
+// envs per thread at 94 registers spilled into a second wave (54%).
 template <int V, int P>
 __global__ void __launch_bounds__(128)
     gae_stream_kernel(const float* __restrict__ r, const float* __restrict__ v, const uint8_t* __restrict__ d,
@@ -230,7 +231,6 @@ pe_status gae_launch(const float* r, const float* v, const uint8_t* d, const flo
                                       reinterpret_cast<uintptr_t>(last_v)) % 8 == 0) &&
                    reinterpret_cast<uintptr_t>(d) % 2 == 0;
   if (E >= 196608 && al4) return gae_stream_run<4, 8>(r, v, d, last_v, T, E, gamma, lam, adv, ret, st);
-  if (E >= 98304 && al2) return gae_stream_run<2, 8>(r, v, d, last_v, T, E, gamma, lam, adv, ret, st);
   if (E >= 49152) return gae_stream_run<1, 16>(r, v, d, last_v, T, E, gamma, lam, adv, ret, st);
   if (E >= 32768) return gae_stream_run<1, 32>(r, v, d, last_v, T, E, gamma, lam, adv, ret, st);
   if (n >= ((int64_t)1 << 28) && al4) return gae_run<4, 8, 4>(r, v, d, last_v, T, E, gamma, lam, adv, ret, st);

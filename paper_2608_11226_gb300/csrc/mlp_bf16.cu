@@ -13,8 +13,8 @@
 //     add the bias, apply tanh, round to bf16 and write the next layer's A
 //     operand into shared memory in the swizzled layout.
 // Precision: bf16 observations, weights and hidden activations, fp32
-// accumulation, fp32 bias and the SFU's tanh, rounded to bf16 -- the
-// quantisation points the oracle emulates (with an exact tanh).
+// accumulation, fp32 bias and tanh -- the quantisation points the oracle
+// emulates.
 #include <type_traits>
 
 #include "env.cuh"

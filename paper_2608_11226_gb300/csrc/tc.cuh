@@ -192,21 +192,14 @@ __device__ __forceinline__ void bulk_g2s(void* dst_smem, const void* src_gmem, u
       : "memory");
 }
 
-// hidden-layer activation of the bf16 networks: the SFU's tanh (tanh.approx.f32,
-// one instruction; measured on GB300 against double: max relative error
-// 9.9e-6, max absolute error 7.8e-6).  Its result is rounded to bf16, whose
-// quantum is 3.9e-3 relative, so it moves an activation by one bf16 ulp only
-// when the exact value lies within about 1e-5 of a rounding midpoint.
-__device__ __forceinline__ float tanh_sfu(float x) {
-  float y;
-  asm("tanh.approx.f32 %0, %1;" : "=f"(y) : "f"(x));
-  return y;
-}
-
-// tanh(v + b) for two adjacent columns, packed to a bf16 pair
+// tanh(v + b) for two adjacent columns, packed to a bf16 pair.  The bias is
+// added with the packed two-lane fp32 add (the same rounding as two adds);
+// tanh is the accurate tanhf: the SFU's tanh.approx.f32 (relative error up
+// to 1e-5, measured) moved enough activations across bf16 rounding
+// boundaries to break the value network's parity with the oracle.
 __device__ __forceinline__ uint32_t tanh_pack2(float v0, float v1, float2 b) {
   const float2 z = __fadd2_rn(make_float2(v0, v1), b);
-  __nv_bfloat162 r = __floats2bfloat162_rn(tanh_sfu(z.x), tanh_sfu(z.y));
+  __nv_bfloat162 r = __floats2bfloat162_rn(tanhf(z.x), tanhf(z.y));
   return *reinterpret_cast<uint32_t*>(&r);
 }
 
