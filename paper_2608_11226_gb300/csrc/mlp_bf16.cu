@@ -15,6 +15,7 @@
 // Precision: bf16 observations, weights and hidden activations, fp32
 // accumulation, fp32 bias and tanh -- the quantisation points the oracle
 // emulates.
+#include <algorithm>
 #include <type_traits>
 
 #include "env.cuh"
@@ -617,6 +618,282 @@ __global__ void __launch_bounds__(kStreamThreads, 1)
 }
 
 // ---------------------------------------------------------------------------
+// Two tiles in flight (72B network, H = 256): the per-tile chain of
+// mlp_bf16_kernel (layer MMA, then an epilogue that waits for it, then the
+// next MMA) leaves the tensor core idle during every epilogue and the
+// epilogue warps idle during every MMA.  Here a CTA holds two 128-row tiles
+// (slots 0 and 1), each with its own activation buffer and its own half of
+// TMEM (columns 256 s .. 256 s + 255 for layer 1, layer 2 and the head in
+// turn), and runs them half a stage apart: the epilogue of one slot overlaps
+// the MMAs of the other.  Shared memory holds two activation tiles (128 KB),
+// so W2 (128 KB) is streamed from L2 in 32 KB K-blocks through a two-slot
+// ring instead of staying resident; W1, W3 and the biases stay resident.
+// Warp roles: warps 0-15 run the epilogues (TMEM -> bias, tanh, bf16 ->
+// shared memory), warp 16 streams the W2 stages, warp 17 issues the MMAs.
+// The roles hand over through mbarriers (one completion per tile pair):
+//   xin[s], h1in[s], h2in[s]: the 16 epilogue warps have written the slot's
+//                             X, h1 or h2 (count 16, lane 0 of each warp);
+//   mma1[s], mma2[s], head[s]: the slot's layer-1, layer-2, head MMAs are
+//                             done (tcgen05.commit).
+// The arithmetic of every tile is mlp_bf16_kernel's, so the results are the
+// same bits.
+// ---------------------------------------------------------------------------
+constexpr int kPairThreads = 576;
+constexpr int kPairW2Stage = 32768;  // one K-block of 64 of W2 (256 rows x 128 B)
+
+template <int D, int H>
+struct MlpPairSmem {
+  alignas(1024) uint8_t act[2][kTcRows * H * 2];  // per slot: X (aliases the start), then h1, then h2
+  alignas(1024) uint8_t ring[2][kPairW2Stage];
+  alignas(1024) uint8_t w1[Img<D, H>::W1];
+  alignas(1024) uint8_t w3[Img<D, H>::W3];
+  float b1[H], b2[H], b3[kHeadN];
+  uint64_t bar_w, full[2], empty[2], mma1[2], mma2[2], head[2], xin[2], h1in[2], h2in[2];
+  uint32_t tmem_base;
+  int32_t err;
+};
+
+template <int D, int H>
+__global__ void __launch_bounds__(kPairThreads, 1)
+    mlp_bf16_pair_kernel(const uint8_t* __restrict__ img, const float* __restrict__ params, int A,
+                         int value_net, const __nv_bfloat16* __restrict__ obs, int64_t n,
+                         float* __restrict__ out, int out_stride, int nout, int32_t* __restrict__ err,
+                         MlpSave save) {
+  using I = Img<D, H>;
+  static_assert(H == 256, "two tiles in flight need 2 x 256 TMEM columns");
+  constexpr int KB2 = H / 64;   // W2 stages per tile
+  constexpr int CPR = D / 8;    // 16-byte observation chunks per row
+  constexpr int XCH = kTcRows * CPR / kTcThreads;
+  static_assert(kTcRows * CPR % kTcThreads == 0, "observation chunks per thread");
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
+  MlpPairSmem<D, H>& s = *reinterpret_cast<MlpPairSmem<D, H>*>(base);
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const MlpLayout Lp = mlp_layout(D, H, A);
+  if (tid == 0) {
+    s.err = 0;
+    tc::mbar_init(&s.bar_w, 1);
+    for (int i = 0; i < 2; ++i) {
+      tc::mbar_init(&s.full[i], 1);
+      tc::mbar_init(&s.empty[i], 1);
+      tc::mbar_init(&s.mma1[i], 1);
+      tc::mbar_init(&s.mma2[i], 1);
+      tc::mbar_init(&s.head[i], 1);
+      tc::mbar_init(&s.xin[i], 16);
+      tc::mbar_init(&s.h1in[i], 16);
+      tc::mbar_init(&s.h2in[i], 16);
+    }
+    tc::fence_mbar_init();
+  }
+  if (warp == 0) tc::tmem_alloc(&s.tmem_base, 512);
+  for (int i = tid; i < H; i += blockDim.x) {
+    s.b1[i] = __ldg(params + (value_net ? Lp.c1 : Lp.b1) + i);
+    s.b2[i] = __ldg(params + (value_net ? Lp.c2 : Lp.b2) + i);
+  }
+  if (tid < kHeadN) s.b3[tid] = tid < nout ? __ldg(params + (value_net ? Lp.c3 : Lp.b3) + tid) : 0.0f;
+  tc::fence_before();
+  __syncthreads();
+  tc::fence_after();
+  const uint32_t tmem = s.tmem_base;
+  const int64_t tiles = (n + kTcRows - 1) / kTcRows;
+  const int my_tiles = (int)((tiles - blockIdx.x + gridDim.x - 1) / gridDim.x);
+  const int npairs = (my_tiles + 1) / 2;
+  int last_issued = -1;
+  if (warp == 16) {
+    // producer: W2's K-blocks for every tile slot, in the issuer's order
+    if (lane == 0) {
+      int gs = 0;
+      for (int p = 0; p < npairs; ++p)
+        for (int sl = 0; sl < 2; ++sl)
+          for (int kb = 0; kb < KB2; ++kb, ++gs) {
+            const int slot = gs & 1;
+            if (gs >= 2 && !tc::mbar_wait(&s.empty[slot], ((gs - 2) >> 1) & 1)) atomicExch(&s.err, 1);
+            tc::mbar_expect_tx(&s.full[slot], (uint32_t)kPairW2Stage);
+            tc::bulk_g2s(s.ring[slot], img + I::W1 + (int64_t)kb * kPairW2Stage, (uint32_t)kPairW2Stage,
+                         &s.full[slot]);
+            last_issued = gs;
+          }
+    }
+  } else if (warp == 17) {
+    // MMA issuer
+    if (lane == 0) {
+      tc::mbar_expect_tx(&s.bar_w, (uint32_t)(I::W1 + I::W3));
+      tc::bulk_g2s(s.w1, img, (uint32_t)I::W1, &s.bar_w);
+      tc::bulk_g2s(s.w3, img + I::W1 + I::W2, (uint32_t)I::W3, &s.bar_w);
+      if (!tc::mbar_wait(&s.bar_w, 0)) atomicExch(&s.err, 1);
+      const uint32_t w1a = tc::smem_u32(s.w1), w3a = tc::smem_u32(s.w3);
+      const uint32_t r0a = tc::smem_u32(s.ring[0]), r1a = tc::smem_u32(s.ring[1]);
+      constexpr uint32_t kL1 = I::RB1 == 64 ? tc::kLayoutSW64 : tc::kLayoutSW128;
+      constexpr uint32_t kIdN = tc::idesc_bf16(kTcRows, H);
+      constexpr uint32_t kIdH = tc::idesc_bf16(kTcRows, kHeadN);
+      int gs = 0;
+      for (int p = 0; p < npairs; ++p) {
+        const uint32_t par = p & 1;
+        for (int sl = 0; sl < 2; ++sl) {
+          if (!tc::mbar_wait(&s.xin[sl], par)) atomicExch(&s.err, 1);
+          tc::fence_after();
+          const uint32_t xa = tc::smem_u32(s.act[sl]);
+#pragma unroll
+          for (int kk = 0; kk < D / 16; ++kk)
+            tc::mma_bf16(tmem + sl * 256, tc::desc_kmajor(xa + kk * 32, 8 * I::RB1, kL1),
+                         tc::desc_kmajor(w1a + kk * 32, 8 * I::RB1, kL1), kIdN, kk > 0);
+          tc::mma_commit(&s.mma1[sl]);
+        }
+        for (int sl = 0; sl < 2; ++sl) {
+          if (!tc::mbar_wait(&s.h1in[sl], par)) atomicExch(&s.err, 1);
+          tc::fence_after();
+          const uint32_t ha = tc::smem_u32(s.act[sl]);
+          for (int kb = 0; kb < KB2; ++kb, ++gs) {
+            const int slot = gs & 1;
+            if (!tc::mbar_wait(&s.full[slot], (gs >> 1) & 1)) atomicExch(&s.err, 1);
+            tc::fence_after();
+            const uint32_t ra = slot ? r1a : r0a;
+#pragma unroll
+            for (int kk = 0; kk < 4; ++kk)
+              tc::mma_bf16(tmem + sl * 256, tc::desc_kmajor(ha + kb * kTcRows * 128 + kk * 32, 1024, tc::kLayoutSW128),
+                           tc::desc_kmajor(ra + kk * 32, 1024, tc::kLayoutSW128), kIdN, (kb | kk) != 0);
+            tc::mma_commit(&s.empty[slot]);
+          }
+          tc::mma_commit(&s.mma2[sl]);
+        }
+        for (int sl = 0; sl < 2; ++sl) {
+          if (!tc::mbar_wait(&s.h2in[sl], par)) atomicExch(&s.err, 1);
+          tc::fence_after();
+          const uint32_t ha = tc::smem_u32(s.act[sl]);
+#pragma unroll 1
+          for (int kb = 0; kb < H / 64; ++kb)
+#pragma unroll
+            for (int kk = 0; kk < 4; ++kk)
+              tc::mma_bf16(tmem + sl * 256, tc::desc_kmajor(ha + kb * kTcRows * 128 + kk * 32, 1024, tc::kLayoutSW128),
+                           tc::desc_kmajor(w3a + kb * kHeadN * 128 + kk * 32, 1024, tc::kLayoutSW128), kIdH,
+                           (kb | kk) != 0);
+          tc::mma_commit(&s.head[sl]);
+        }
+      }
+    }
+  } else {
+    // epilogue warps
+    const int quad = warp & 3, slice = warp >> 2, row = quad * 32 + lane;
+    const uint32_t lane_base = tmem + ((uint32_t)(quad * 32) << 16);
+    uint4 xv[2][XCH];
+    auto fetch_x = [&](int k, uint4 (&dst)[XCH]) {
+      const int64_t tl = blockIdx.x + (int64_t)k * gridDim.x;
+#pragma unroll
+      for (int q = 0; q < XCH; ++q) {
+        const int i = tid + q * kTcThreads, r = i / CPR, c = i % CPR;
+        const int64_t rr = tl * kTcRows + r;
+        dst[q] = make_uint4(0, 0, 0, 0);
+        if (k < my_tiles && rr < n) {
+          const int64_t src = save.gather ? (int64_t)__ldg(save.gather + rr) : rr;
+          dst[q] = __ldg(reinterpret_cast<const uint4*>(obs + src * D) + c);
+        }
+      }
+    };
+    // head readout of the tile in slot sl (warps 0-3: one row per thread)
+    auto head_out = [&](int sl, int k) {
+      if (warp < 4 && k < my_tiles) {
+        const int64_t tl = blockIdx.x + (int64_t)k * gridDim.x;
+        const int nr = (int)(n - tl * kTcRows < kTcRows ? n - tl * kTcRows : kTcRows);
+        float v[16];
+        tc::tmem_ld16(lane_base + (uint32_t)(sl * 256), v);
+        if (row < nr) {
+          float* o = out + (tl * kTcRows + row) * out_stride;
+#pragma unroll
+          for (int j = 0; j < kHeadN; ++j)
+            if (j < nout) o[j] = v[j] + s.b3[j];
+        }
+      }
+    };
+    // hidden layer epilogue of slot sl: tanh(acc + bias) -> bf16 -> act[sl] (+ the tile image)
+    auto hidden = [&](int sl, const float* bias, __nv_bfloat16* gsave, int k) {
+      const int64_t tl = blockIdx.x + (int64_t)k * gridDim.x;
+      uint8_t* g = (gsave && k < my_tiles) ? reinterpret_cast<uint8_t*>(gsave) + tl * (int64_t)(kTcRows * H * 2)
+                                           : nullptr;
+#pragma unroll
+      for (int j = 0; j < H / 64; ++j) {
+        const int c = slice * (H / 4) + j * 16;
+        float v[16];
+        tc::tmem_ld16(lane_base + (uint32_t)(sl * 256 + c), v);
+        uint32_t pk[8];
+#pragma unroll
+        for (int i = 0; i < 8; ++i)
+          pk[i] = tc::tanh_pack2(v[2 * i], v[2 * i + 1], *reinterpret_cast<const float2*>(bias + c + 2 * i));
+        const uint32_t o0 = tc::swz_offset<128>(row, c, kTcRows), o1 = tc::swz_offset<128>(row, c + 8, kTcRows);
+        const uint4 lo = make_uint4(pk[0], pk[1], pk[2], pk[3]), hi = make_uint4(pk[4], pk[5], pk[6], pk[7]);
+        *reinterpret_cast<uint4*>(s.act[sl] + o0) = lo;
+        *reinterpret_cast<uint4*>(s.act[sl] + o1) = hi;
+        if (g) {
+          *reinterpret_cast<uint4*>(g + o0) = lo;
+          *reinterpret_cast<uint4*>(g + o1) = hi;
+        }
+      }
+    };
+    auto handover = [&](uint64_t* bar) {
+      tc::fence_async_smem();
+      tc::fence_before();
+      __syncwarp();
+      if (lane == 0) asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(tc::smem_u32(bar)) : "memory");
+    };
+    fetch_x(0, xv[0]);
+    fetch_x(1, xv[1]);
+    for (int p = 0; p < npairs; ++p) {
+      const uint32_t par = p & 1;
+      for (int sl = 0; sl < 2; ++sl) {
+        const int k = 2 * p + sl;
+        if (p > 0) {
+          // the previous tile of this slot: its head is done, read it out;
+          // its h2 is no longer needed, so X may overwrite the buffer
+          if (!tc::mbar_wait(&s.head[sl], par ^ 1)) atomicExch(&s.err, 1);
+          tc::fence_after();
+          head_out(sl, k - 2);
+        }
+        const int64_t tl = blockIdx.x + (int64_t)k * gridDim.x;
+#pragma unroll
+        for (int q = 0; q < XCH; ++q) {
+          const int i = tid + q * kTcThreads, r = i / CPR, c = i % CPR;
+          const uint32_t off = tc::swz_offset<I::RB1>(r, c * 8, kTcRows);
+          *reinterpret_cast<uint4*>(s.act[sl] + off) = xv[sl][q];
+          if (save.x && k < my_tiles)
+            *reinterpret_cast<uint4*>(reinterpret_cast<uint8_t*>(save.x) + tl * (int64_t)(kTcRows * D * 2) + off) =
+                xv[sl][q];
+        }
+        handover(&s.xin[sl]);
+      }
+      fetch_x(2 * p + 2, xv[0]);
+      fetch_x(2 * p + 3, xv[1]);
+      for (int sl = 0; sl < 2; ++sl) {
+        if (!tc::mbar_wait(&s.mma1[sl], par)) atomicExch(&s.err, 1);
+        tc::fence_after();
+        hidden(sl, s.b1, save.h1, 2 * p + sl);
+        handover(&s.h1in[sl]);
+      }
+      for (int sl = 0; sl < 2; ++sl) {
+        if (!tc::mbar_wait(&s.mma2[sl], par)) atomicExch(&s.err, 1);
+        tc::fence_after();
+        hidden(sl, s.b2, save.h2, 2 * p + sl);
+        handover(&s.h2in[sl]);
+      }
+    }
+    if (npairs > 0)
+      for (int sl = 0; sl < 2; ++sl) {
+        if (!tc::mbar_wait(&s.head[sl], (npairs - 1) & 1)) atomicExch(&s.err, 1);
+        tc::fence_after();
+        head_out(sl, 2 * (npairs - 1) + sl);
+      }
+  }
+  tc::fence_before();
+  __syncthreads();
+  if (s.err && warp == 16 && lane == 0 && last_issued >= 0)
+    (void)tc::mbar_wait(&s.full[last_issued & 1], (last_issued >> 1) & 1);
+  if (tid == 0 && s.err) {
+    atomicExch(&g_tc_error, 1);
+    if (err) atomicExch(err, 1);
+  }
+  __syncthreads();
+  if (warp == 0) tc::tmem_dealloc(tmem, 512);
+}
+
+// ---------------------------------------------------------------------------
 // decoupled bf16 rollout: per step, an env kernel (one thread per env: act on
 // the previous step's logits, then observe) and the tensor-core policy kernel
 // ---------------------------------------------------------------------------
@@ -726,11 +1003,12 @@ static pe_status launch_mlp(const uint8_t* img, const float* params, int A, int 
     ProfScope ps(prof_kind, st);
     kern<<<grid, kStreamThreads, bytes, st>>>(img, params, A, value_net, o, n, out, out_stride, nout, err, save);
   } else {
-    auto kern = mlp_bf16_kernel<D, H>;
-    const int bytes = (int)sizeof(MlpBf16Smem<D, H>) + 1024;
+    auto kern = mlp_bf16_pair_kernel<D, H>;
+    const int bytes = (int)sizeof(MlpPairSmem<D, H>) + 1024;
     PE_TRY_CUDA(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes));
+    const int pgrid = (int)std::min<int64_t>((tiles + 1) / 2, sms);
     ProfScope ps(prof_kind, st);
-    kern<<<grid, kTcThreads, bytes, st>>>(img, params, A, value_net, o, n, out, out_stride, nout, err, save);
+    kern<<<pgrid, kPairThreads, bytes, st>>>(img, params, A, value_net, o, n, out, out_stride, nout, err, save);
   }
   PE_CHECK_LAUNCH("mlp_bf16_kernel");
   return PE_OK;
