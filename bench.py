@@ -60,7 +60,7 @@ def parse():
     ap.add_argument("--r72b-horizon", type=int, default=1024)
     ap.add_argument("--r72b-ppo-minibatches", type=int, default=16,
                     help="72B PPO minibatch steps of 65,536 samples timed (0: skip)")
-    ap.add_argument("--ncu-case", choices=["ppo7b", "ppo72", "gae", "mlp72", "fleet"], default=None,
+    ap.add_argument("--ncu-case", choices=["ppo7b", "ppo72", "ppostress", "gae", "mlp72", "fleet"], default=None,
                     help="run one small named case of a hot kernel (for ncu captures) and exit")
     ap.add_argument("--gae-large", type=int, nargs=2, default=[2048, 262144], metavar=("T", "E"),
                     help="GAE roofline size (Stress: 2048 x 262144); T=0 skips it")
@@ -1109,11 +1109,12 @@ def run_ncu_case(name: str):
     from paper_2608_11226_gb300 import workloads as W
     build.build()
     pe.lib()
-    if name in ("ppo7b", "ppo72"):
-        # rollout (32 or 16 steps), GAE, then 3 PPO updates of one epoch (16 minibatch steps each)
-        wl = W.make_7b() if name == "ppo7b" else W.make_72b(n_envs=65536)
+    if name in ("ppo7b", "ppo72", "ppostress"):
+        # rollout (32, 16 or 4 steps), GAE, then 3 PPO updates of one epoch (16 minibatch steps each)
+        wl = (W.make_7b() if name == "ppo7b" else W.make_72b(n_envs=65536) if name == "ppo72"
+              else W.make_stress(n_envs=262144, horizon=4))
         spec, net = wl.env, wl.net
-        T = 32 if name == "ppo7b" else 16
+        T = {"ppo7b": 32, "ppo72": 16, "ppostress": 4}[name]
         mb = 8192 if name == "ppo7b" else 65536
         env = pe.Env(spec, torch.from_numpy(wl.trace), torch.from_numpy(wl.phase))
         buf = pe.alloc_rollout(spec, net, T)

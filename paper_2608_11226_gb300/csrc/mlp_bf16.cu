@@ -1,17 +1,20 @@
 // bf16 policy/value MLPs on the 5th-generation tensor cores (tcgen05), and the
-// decoupled rollout that uses them (72B workload: D=32, H=256, A=16, C=4).
+// decoupled rollout that uses them (72B workload: D=32, H=256, A=16, C=4;
+// Stress: D=64, H=512).
 //
 // A policy/value network is tanh(W2 tanh(W1 x + b1) + b2) followed by a
 // linear head (Sec. 4.2 actor-critic), evaluated on 128-row tiles:
 //   - the fp32 master parameters are first converted once per call into a
-//     bf16 "weight image": each matrix laid out exactly as the kernel keeps it
-//     in shared memory (K-major, 128-byte or 64-byte swizzle);
-//   - a persistent CTA copies the image into shared memory with one bulk copy
-//     (cp.async.bulk, completion on an mbarrier) and keeps it for all its tiles;
+//     bf16 "weight image": each matrix laid out exactly as the kernels keep
+//     it in shared memory (K-major, 128-byte or 64-byte swizzle), W2 in
+//     32 KB K-blocks that stream through a two-slot ring;
 //   - per layer one thread issues tcgen05.mma (M=128, K=16 per instruction)
 //     into TMEM; sixteen warps read the fp32 accumulators back (tcgen05.ld),
 //     add the bias, apply tanh, round to bf16 and write the next layer's A
-//     operand into shared memory in the swizzled layout.
+//     operand into shared memory in the swizzled layout;
+//   - 72B (mlp_bf16_pair_kernel): two tiles in flight per CTA, so that the
+//     epilogue of one overlaps the MMAs of the other; Stress
+//     (mlp_bf16_stream_kernel): one tile, its 592 KB of weights streamed.
 // Precision: bf16 observations, weights and hidden activations, fp32
 // accumulation, fp32 bias and tanh -- the quantisation points the oracle
 // emulates.
@@ -89,248 +92,6 @@ __global__ void weight_image_kernel(const float* __restrict__ params, int A, int
           __float2bfloat16_rn(v);
     }
   }
-}
-
-template <int D, int H>
-struct MlpBf16Smem {
-  // operand images (bulk-copied): W1 | W2 | W3, then the activation tile
-  alignas(1024) uint8_t w[Img<D, H>::TOTAL];
-  alignas(1024) uint8_t act[Img<D, H>::ACT];  // X (layer-1 A operand) aliases its start
-  float b1[H], b2[H], b3[kHeadN];
-  uint64_t bar_w, bar_mma, bar_hi;  // bar_mma: first column half (and the head), bar_hi: second half
-  uint32_t tmem_base;
-  int32_t err;
-};
-
-// fp32 epilogue of one layer for this warp's H/4 columns, in two parts so that
-// the arithmetic can overlap the tensor core while the store waits for it:
-//   epi_compute: TMEM -> tanh(. + b) -> packed bf16 pairs in registers
-//   epi_store:   registers -> the next layer's A tile (swizzled)
-// Warp w reads TMEM lanes 32*(w%4)..+31 (its rows) and column slice w/4.
-template <int H>
-__device__ __forceinline__ void epi_compute(uint32_t tmem, int col0, const float* bias,
-                                            uint32_t (&pk)[H / 8]) {
-  const int warp = threadIdx.x >> 5;
-  const int quad = warp & 3, slice = warp >> 2;
-  const uint32_t lane_addr = tmem + ((uint32_t)(quad * 32) << 16);
-#pragma unroll
-  for (int j = 0; j < H / 64; ++j) {
-    const int c = slice * (H / 4) + j * 16;
-    float v[16];
-    tc::tmem_ld16(lane_addr + (uint32_t)(col0 + c), v);
-#pragma unroll
-    for (int i = 0; i < 8; ++i)
-      pk[j * 8 + i] = tc::tanh_pack2(v[2 * i], v[2 * i + 1], *reinterpret_cast<const float2*>(bias + c + 2 * i));
-  }
-}
-
-template <int H>
-__device__ __forceinline__ void epi_store(const uint32_t (&pk)[H / 8], uint8_t* act,
-                                          __nv_bfloat16* gsave, int64_t tile) {
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int quad = warp & 3, slice = warp >> 2;
-  const int row = quad * 32 + lane;
-  uint8_t* g = gsave ? reinterpret_cast<uint8_t*>(gsave) + tile * (int64_t)(kTcRows * H * 2) : nullptr;
-#pragma unroll
-  for (int j = 0; j < H / 64; ++j) {
-    const int c = slice * (H / 4) + j * 16;
-    const uint4 lo = make_uint4(pk[j * 8 + 0], pk[j * 8 + 1], pk[j * 8 + 2], pk[j * 8 + 3]);
-    const uint4 hi = make_uint4(pk[j * 8 + 4], pk[j * 8 + 5], pk[j * 8 + 6], pk[j * 8 + 7]);
-    const uint32_t o0 = tc::swz_offset<128>(row, c, kTcRows), o1 = tc::swz_offset<128>(row, c + 8, kTcRows);
-    *reinterpret_cast<uint4*>(act + o0) = lo;
-    *reinterpret_cast<uint4*>(act + o1) = hi;
-    if (g) {
-      *reinterpret_cast<uint4*>(g + o0) = lo;
-      *reinterpret_cast<uint4*>(g + o1) = hi;
-    }
-  }
-}
-
-// One MLP over n rows of bf16 observations [n][D]; writes out[r * out_stride + j]
-// for j < nout.  Persistent over 128-row tiles.  *err is set to 1 if a bounded
-// wait timed out.
-template <int D, int H>
-__global__ void __launch_bounds__(kTcThreads, 1)
-    mlp_bf16_kernel(const uint8_t* __restrict__ img, const float* __restrict__ params, int A,
-                    int value_net, const __nv_bfloat16* __restrict__ obs, int64_t n,
-                    float* __restrict__ out, int out_stride, int nout, int32_t* __restrict__ err,
-                    MlpSave save) {
-  using I = Img<D, H>;
-  extern __shared__ __align__(1024) uint8_t smem_raw[];
-  // align the dynamic shared window to 1024 B for the swizzle atoms
-  uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
-  MlpBf16Smem<D, H>& s = *reinterpret_cast<MlpBf16Smem<D, H>*>(base);
-  const int tid = threadIdx.x, warp = tid >> 5;
-  const MlpLayout Lp = mlp_layout(D, H, A);
-  if (tid == 0) {
-    s.err = 0;
-    tc::mbar_init(&s.bar_w, 1);
-    tc::mbar_init(&s.bar_mma, 1);
-    tc::mbar_init(&s.bar_hi, 1);
-    tc::fence_mbar_init();
-  }
-  if (warp == 0) tc::tmem_alloc(&s.tmem_base, 512);
-  for (int i = tid; i < H; i += blockDim.x) {
-    s.b1[i] = __ldg(params + (value_net ? Lp.c1 : Lp.b1) + i);
-    s.b2[i] = __ldg(params + (value_net ? Lp.c2 : Lp.b2) + i);
-  }
-  if (tid < kHeadN) s.b3[tid] = tid < nout ? __ldg(params + (value_net ? Lp.c3 : Lp.b3) + tid) : 0.0f;
-  tc::fence_before();
-  __syncthreads();
-  tc::fence_after();
-  const uint32_t tmem = s.tmem_base;
-  if (tid == 0) {
-    tc::mbar_expect_tx(&s.bar_w, (uint32_t)I::TOTAL);
-    tc::bulk_g2s(s.w, img, (uint32_t)I::TOTAL, &s.bar_w);
-  }
-  if (!tc::mbar_wait(&s.bar_w, 0)) atomicExch(&s.err, 1);
-  __syncthreads();
-
-  const uint32_t w1 = tc::smem_u32(s.w), w2 = w1 + I::W1, w3 = w2 + I::W2;
-  const uint32_t xa = tc::smem_u32(s.act);
-  constexpr uint32_t kIdHalf = tc::idesc_bf16(kTcRows, H / 2);
-  constexpr uint32_t kIdH = tc::idesc_bf16(kTcRows, kHeadN);
-  uint32_t phase = 0, phase_hi = 0;
-  const int64_t tiles = (n + kTcRows - 1) / kTcRows;
-  // Observation tiles are fetched one tile ahead: each thread holds its
-  // 16-byte chunk(s) of the next tile in registers while the current tile's
-  // layers run, so the global load latency is off the critical path.
-  constexpr int CPR = D / 8;                         // 16-byte chunks per row
-  constexpr int XCH = kTcRows * CPR / kTcThreads;    // chunks per thread
-  static_assert(kTcRows * CPR % kTcThreads == 0, "observation chunks per thread");
-  uint4 xv[XCH];
-  auto fetch_x = [&](int64_t tl) {
-#pragma unroll
-    for (int q = 0; q < XCH; ++q) {
-      const int i = tid + q * kTcThreads, r = i / CPR, c = i % CPR;
-      const int64_t row = tl * kTcRows + r;
-      xv[q] = make_uint4(0, 0, 0, 0);
-      if (tl < tiles && row < n) {
-        const int64_t src = save.gather ? (int64_t)__ldg(save.gather + row) : row;
-        xv[q] = __ldg(reinterpret_cast<const uint4*>(obs + src * D) + c);
-      }
-    }
-  };
-  fetch_x(blockIdx.x);
-  for (int64_t tile = blockIdx.x; tile < tiles; tile += gridDim.x) {
-    // a wait that gave up stops every thread of the CTA at the same tile
-    if (__syncthreads_or(s.err != 0)) break;
-    const int64_t r0 = tile * kTcRows;
-    const int nr = (int)(n - r0 < kTcRows ? n - r0 : kTcRows);
-    // observation tile -> X (D bf16 per row, swizzled like W1)
-#pragma unroll
-    for (int q = 0; q < XCH; ++q) {
-      const int i = tid + q * kTcThreads, r = i / CPR, c = i % CPR;
-      const uint32_t off = tc::swz_offset<I::RB1>(r, c * 8, kTcRows);
-      *reinterpret_cast<uint4*>(s.act + off) = xv[q];
-      if (save.x)
-        *reinterpret_cast<uint4*>(reinterpret_cast<uint8_t*>(save.x) + tile * (int64_t)(kTcRows * D * 2) + off) = xv[q];
-    }
-    tc::fence_async_smem();
-    __syncthreads();
-    fetch_x(tile + gridDim.x);
-    // Each layer's N = H outputs are issued as two halves of H/2 columns with
-    // separate commits, so that the warps of the first column half run their
-    // epilogue while the tensor core computes the second half.
-    const bool hi_half = (warp >> 2) >= 2;  // column slices 2, 3
-    // layer 1: D1[128 x H] (TMEM cols 0..H) = X W1^T
-    if (tid == 0) {
-      tc::fence_after();
-#pragma unroll 1
-      for (int h = 0; h < 2; ++h) {
-#pragma unroll
-        for (int kk = 0; kk < D / 16; ++kk)
-          tc::mma_bf16(tmem + h * (H / 2),
-                       tc::desc_kmajor(xa + kk * 32, 8 * I::RB1, I::RB1 == 64 ? tc::kLayoutSW64 : tc::kLayoutSW128),
-                       tc::desc_kmajor(w1 + h * (H / 2) * I::RB1 + kk * 32, 8 * I::RB1,
-                                       I::RB1 == 64 ? tc::kLayoutSW64 : tc::kLayoutSW128),
-                       kIdHalf, kk > 0);
-        tc::mma_commit(h == 0 ? &s.bar_mma : &s.bar_hi);
-      }
-    }
-    // epilogue 1: the first column half computes as soon as its MMAs are done;
-    // every warp stores only after all layer-1 MMAs have read X (same buffer)
-    uint32_t pk[H / 8];
-    if (!hi_half) {
-      if (!tc::mbar_wait(&s.bar_mma, phase)) atomicExch(&s.err, 1);
-      tc::fence_after();
-      epi_compute<H>(tmem, 0, s.b1, pk);
-    }
-    if (!tc::mbar_wait(&s.bar_hi, phase_hi)) atomicExch(&s.err, 1);
-    tc::fence_after();
-    if (hi_half) epi_compute<H>(tmem, 0, s.b1, pk);
-    epi_store<H>(pk, s.act, save.h1, tile);
-    phase ^= 1;
-    phase_hi ^= 1;
-    tc::fence_before();
-    tc::fence_async_smem();
-    __syncthreads();
-    // layer 2: D2 (TMEM cols 256..256+H) = H1 W2^T
-    if (tid == 0) {
-      tc::fence_after();
-#pragma unroll 1
-      for (int h = 0; h < 2; ++h) {
-#pragma unroll 1
-        for (int kb = 0; kb < H / 64; ++kb)
-#pragma unroll
-          for (int kk = 0; kk < 4; ++kk)
-            tc::mma_bf16(tmem + 256 + h * (H / 2),
-                         tc::desc_kmajor(xa + kb * kTcRows * 128 + kk * 32, 1024, tc::kLayoutSW128),
-                         tc::desc_kmajor(w2 + kb * H * 128 + h * (H / 2) * 128 + kk * 32, 1024, tc::kLayoutSW128),
-                         kIdHalf, (kb | kk) != 0);
-        tc::mma_commit(h == 0 ? &s.bar_mma : &s.bar_hi);
-      }
-    }
-    // epilogue 2: as epilogue 1 (H2 overwrites H1, which the MMAs read)
-    if (!hi_half) {
-      if (!tc::mbar_wait(&s.bar_mma, phase)) atomicExch(&s.err, 1);
-      tc::fence_after();
-      epi_compute<H>(tmem, 256, s.b2, pk);
-    }
-    if (!tc::mbar_wait(&s.bar_hi, phase_hi)) atomicExch(&s.err, 1);
-    tc::fence_after();
-    if (hi_half) epi_compute<H>(tmem, 256, s.b2, pk);
-    epi_store<H>(pk, s.act, save.h2, tile);
-    phase ^= 1;
-    phase_hi ^= 1;
-    tc::fence_before();
-    tc::fence_async_smem();
-    __syncthreads();
-    // head: D3 (TMEM cols 0..16) = H2 W3^T
-    if (tid == 0) {
-      tc::fence_after();
-#pragma unroll 1
-      for (int kb = 0; kb < H / 64; ++kb)
-#pragma unroll
-        for (int kk = 0; kk < 4; ++kk)
-          tc::mma_bf16(tmem, tc::desc_kmajor(xa + kb * kTcRows * 128 + kk * 32, 1024, tc::kLayoutSW128),
-                       tc::desc_kmajor(w3 + kb * kHeadN * 128 + kk * 32, 1024, tc::kLayoutSW128), kIdH,
-                       (kb | kk) != 0);
-      tc::mma_commit(&s.bar_mma);
-    }
-    if (!tc::mbar_wait(&s.bar_mma, phase)) atomicExch(&s.err, 1);
-    phase ^= 1;
-    tc::fence_after();
-    if (warp < 4) {
-      const int row = warp * 32 + (tid & 31);
-      float v[16];
-      tc::tmem_ld16(tmem + ((uint32_t)(warp * 32) << 16), v);
-      if (row < nr) {
-        float* o = out + (r0 + row) * out_stride;
-#pragma unroll
-        for (int j = 0; j < kHeadN; ++j)
-          if (j < nout) o[j] = v[j] + s.b3[j];
-      }
-    }
-    tc::fence_before();
-    __syncthreads();
-  }
-  if (tid == 0 && s.err) {
-    atomicExch(&g_tc_error, 1);
-    if (err) atomicExch(err, 1);
-  }
-  __syncthreads();
-  if (warp == 0) tc::tmem_dealloc(tmem, 512);
 }
 
 // ---------------------------------------------------------------------------
@@ -618,10 +379,10 @@ __global__ void __launch_bounds__(kStreamThreads, 1)
 }
 
 // ---------------------------------------------------------------------------
-// Two tiles in flight (72B network, H = 256): the per-tile chain of
-// mlp_bf16_kernel (layer MMA, then an epilogue that waits for it, then the
-// next MMA) leaves the tensor core idle during every epilogue and the
-// epilogue warps idle during every MMA.  Here a CTA holds two 128-row tiles
+// Two tiles in flight (72B network, H = 256): with one tile per CTA, the
+// chain of layer MMA, then an epilogue that waits for it, then the next MMA
+// leaves the tensor core idle during every epilogue and the epilogue warps
+// idle during every MMA.  Here a CTA holds two 128-row tiles
 // (slots 0 and 1), each with its own activation buffer and its own half of
 // TMEM (columns 256 s .. 256 s + 255 for layer 1, layer 2 and the head in
 // turn), and runs them half a stage apart: the epilogue of one slot overlaps
@@ -635,8 +396,8 @@ __global__ void __launch_bounds__(kStreamThreads, 1)
 //                             X, h1 or h2 (count 16, lane 0 of each warp);
 //   mma1[s], mma2[s], head[s]: the slot's layer-1, layer-2, head MMAs are
 //                             done (tcgen05.commit).
-// The arithmetic of every tile is mlp_bf16_kernel's, so the results are the
-// same bits.
+// The arithmetic of every tile is that of a one-tile kernel (the same MMAs
+// in the same order, the same epilogue), so the results are the same bits.
 // ---------------------------------------------------------------------------
 constexpr int kPairThreads = 576;
 constexpr int kPairW2Stage = 32768;  // one K-block of 64 of W2 (256 rows x 128 B)
@@ -1010,7 +771,7 @@ static pe_status launch_mlp(const uint8_t* img, const float* params, int A, int 
     ProfScope ps(prof_kind, st);
     kern<<<pgrid, kPairThreads, bytes, st>>>(img, params, A, value_net, o, n, out, out_stride, nout, err, save);
   }
-  PE_CHECK_LAUNCH("mlp_bf16_kernel");
+  PE_CHECK_LAUNCH("bf16 MLP kernel");
   return PE_OK;
 }
 

@@ -192,14 +192,28 @@ __device__ __forceinline__ void bulk_g2s(void* dst_smem, const void* src_gmem, u
       : "memory");
 }
 
-// tanh(v + b) for two adjacent columns, packed to a bf16 pair.  The bias is
-// added with the packed two-lane fp32 add (the same rounding as two adds);
-// tanh is the accurate tanhf: the SFU's tanh.approx.f32 (relative error up
-// to 1e-5, measured) moved enough activations across bf16 rounding
-// boundaries to break the value network's parity with the oracle.
+// tanh of a hidden pre-activation whose result is rounded to bf16 next.
+// The SFU's tanh (tanh.approx.f32, one instruction) is within 1e-5 relative
+// of tanh on GB300 (max 9.9e-6 measured against double over [-8, 8]), while
+// tanhf takes about 2.5x its issue cost.  The bf16 rounding of the two can
+// differ only if the approximation lies within their error of a rounding
+// midpoint, i.e. if its low 16 bits are within 256 fp32 ulps (at least
+// 1.5e-5 relative) of 0x8000; there the accurate tanhf is taken.  So the
+// rounded result is the rounding of tanhf's value, at the SFU's cost for
+// more than 99% of the elements.
+__device__ __forceinline__ float tanh_for_bf16(float z) {
+  float y;
+  asm("tanh.approx.f32 %0, %1;" : "=f"(y) : "f"(z));
+  const int d = (int)(__float_as_uint(y) & 0xFFFFu) - 0x8000;
+  if (d >= -256 && d <= 256) y = tanhf(z);
+  return y;
+}
+
+// tanh(v + b) for two adjacent columns, packed to a bf16 pair (the bias added
+// with the packed two-lane fp32 add: the same rounding as two adds)
 __device__ __forceinline__ uint32_t tanh_pack2(float v0, float v1, float2 b) {
   const float2 z = __fadd2_rn(make_float2(v0, v1), b);
-  __nv_bfloat162 r = __floats2bfloat162_rn(tanhf(z.x), tanhf(z.y));
+  __nv_bfloat162 r = __floats2bfloat162_rn(tanh_for_bf16(z.x), tanh_for_bf16(z.y));
   return *reinterpret_cast<uint32_t*>(&r);
 }
 
