@@ -282,9 +282,7 @@ __global__ void __launch_bounds__(kStreamThreads, 1)
         float v[16];
         tc::tmem_ld16(lane_addr + (uint32_t)c, v);
         uint32_t p[8];
-#pragma unroll
-        for (int i = 0; i < 8; ++i)
-          p[i] = tc::tanh_pack2(v[2 * i], v[2 * i + 1], *reinterpret_cast<const float2*>(s.b1 + c + 2 * i));
+        tc::tanh16_bf16(v, s.b1 + c, p);
         const uint32_t o0 = tc::swz_offset<128>(row, c, kTcRows), o1 = tc::swz_offset<128>(row, c + 8, kTcRows);
         *reinterpret_cast<uint4*>(s.act + o0) = make_uint4(p[0], p[1], p[2], p[3]);
         *reinterpret_cast<uint4*>(s.act + o1) = make_uint4(p[4], p[5], p[6], p[7]);
@@ -319,9 +317,7 @@ __global__ void __launch_bounds__(kStreamThreads, 1)
         float v[16];
         tc::tmem_ld16(lane_addr + (uint32_t)c, v);
         uint32_t p[8];
-#pragma unroll
-        for (int i = 0; i < 8; ++i)
-          p[i] = tc::tanh_pack2(v[2 * i], v[2 * i + 1], *reinterpret_cast<const float2*>(s.b2 + c + 2 * i));
+        tc::tanh16_bf16(v, s.b2 + c, p);
         const uint32_t o0 = tc::swz_offset<128>(row, c, kTcRows), o1 = tc::swz_offset<128>(row, c + 8, kTcRows);
         *reinterpret_cast<uint4*>(s.act + o0) = make_uint4(p[0], p[1], p[2], p[3]);
         *reinterpret_cast<uint4*>(s.act + o1) = make_uint4(p[4], p[5], p[6], p[7]);
@@ -576,9 +572,7 @@ __global__ void __launch_bounds__(kPairThreads, 1)
         float v[16];
         tc::tmem_ld16(lane_base + (uint32_t)(sl * 256 + c), v);
         uint32_t pk[8];
-#pragma unroll
-        for (int i = 0; i < 8; ++i)
-          pk[i] = tc::tanh_pack2(v[2 * i], v[2 * i + 1], *reinterpret_cast<const float2*>(bias + c + 2 * i));
+        tc::tanh16_bf16(v, bias + c, pk);
         const uint32_t o0 = tc::swz_offset<128>(row, c, kTcRows), o1 = tc::swz_offset<128>(row, c + 8, kTcRows);
         const uint4 lo = make_uint4(pk[0], pk[1], pk[2], pk[3]), hi = make_uint4(pk[4], pk[5], pk[6], pk[7]);
         *reinterpret_cast<uint4*>(s.act[sl] + o0) = lo;
