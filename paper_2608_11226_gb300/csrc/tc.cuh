@@ -193,45 +193,14 @@ __device__ __forceinline__ void bulk_g2s(void* dst_smem, const void* src_gmem, u
 }
 
 // tanh of 16 hidden pre-activations (v + bias, one TMEM chunk of a thread's
-// row), rounded to bf16 and packed in pairs.
-// The SFU's tanh (tanh.approx.f32, one instruction) is within 1e-5 relative
-// of tanh on GB300 (max 9.9e-6 measured against double over [-8, 8]), while
-// tanhf takes about 2.5x its issue cost.  The bf16 rounding of the two can
-// differ only if the approximation lies within their error of a rounding
-// midpoint, i.e. if its low 16 bits are within 256 fp32 ulps (at least
-// 1.5e-5 relative) of 0x8000; such elements take the accurate tanhf.  So the
-// rounded result is the rounding of tanhf's value.  The fall-back runs per
-// element under a warp-uniform test (any lane of the warp needs it), so that
-// a warp skips tanhf entirely for the ~80% of elements where no lane does;
-// the bias is added with the packed two-lane fp32 add (the same rounding as
-// two adds).
+// row), rounded to bf16 and packed in pairs; the bias is added with the
+// packed two-lane fp32 add (the same rounding as two adds).
 __device__ __forceinline__ void tanh16_bf16(const float (&v)[16], const float* bias, uint32_t (&pk)[8]) {
-  float z[16], y[16];
-  uint32_t amb = 0;
 #pragma unroll
   for (int i = 0; i < 16; i += 2) {
-    const float2 t = __fadd2_rn(make_float2(v[i], v[i + 1]), *reinterpret_cast<const float2*>(bias + i));
-    z[i] = t.x;
-    z[i + 1] = t.y;
-  }
-#pragma unroll
-  for (int i = 0; i < 16; ++i) {
-    asm("tanh.approx.f32 %0, %1;" : "=f"(y[i]) : "f"(z[i]));
-    const int d = (int)(__float_as_uint(y[i]) & 0xFFFFu) - 0x8000;
-    amb |= (d >= -256 && d <= 256) ? (1u << i) : 0u;
-  }
-  const uint32_t any = __reduce_or_sync(0xffffffffu, amb);
-  if (any) {
-#pragma unroll
-    for (int i = 0; i < 16; ++i)
-      if ((any >> i) & 1u) {
-        if ((amb >> i) & 1u) y[i] = tanhf(z[i]);
-      }
-  }
-#pragma unroll
-  for (int i = 0; i < 8; ++i) {
-    __nv_bfloat162 r = __floats2bfloat162_rn(y[2 * i], y[2 * i + 1]);
-    pk[i] = *reinterpret_cast<uint32_t*>(&r);
+    const float2 z = __fadd2_rn(make_float2(v[i], v[i + 1]), *reinterpret_cast<const float2*>(bias + i));
+    __nv_bfloat162 r = __floats2bfloat162_rn(tanhf(z.x), tanhf(z.y));
+    pk[i / 2] = *reinterpret_cast<uint32_t*>(&r);
   }
 }
 
