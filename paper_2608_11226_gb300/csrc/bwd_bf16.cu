@@ -201,6 +201,14 @@ __global__ void __launch_bounds__(kBwThreads, 1) bwd_data_kernel(BwdArgs g) {
       const bool valid = row < nr;
       const uint8_t* h2t = g.h2 + tile * (int64_t)(kBwRows * H * 2);
       const uint8_t* h1t = g.h1 + tile * (int64_t)(kBwRows * H * 2);
+      if (t + 1 < my_tiles) {
+        // the next tile's h1/h2 images asked of L2 a tile ahead (128-byte lines)
+        const int64_t nxt = (tile + gridDim.x) * (int64_t)(kBwRows * H * 2);
+        for (int64_t off = (int64_t)tid * 128; off < (int64_t)kBwRows * H * 2; off += (int64_t)kBwCompute * 128) {
+          tc::prefetch_l2(g.h2 + nxt + off);
+          tc::prefetch_l2(g.h1 + nxt + off);
+        }
+      }
       uint4 hb[PF][2];
 #pragma unroll
       for (int j = 0; j < PF; ++j) hload(h2t, j, hb[j]);
@@ -458,10 +466,27 @@ __global__ void __launch_bounds__(kBwPairThreads, 1) bwd_data_pair_kernel(BwdArg
       if (tid < kBwRows * 2 && k < my_tiles)
         dst = __ldg(reinterpret_cast<const uint4*>(g.dz + tile_of(k) * (kBwRows * 32)) + tid);
     };
+    // The h1/h2 tile images of a pair's two tiles (4 x 64 KB) are asked of L2
+    // one pair ahead, one 128-byte line per thread per image, so that the
+    // epilogues' loads hit L2 instead of waiting for HBM.
+    auto prefetch_pair = [&](int p) {
+#pragma unroll
+      for (int sl = 0; sl < 2; ++sl) {
+        const int k = 2 * p + sl;
+        if (k < my_tiles) {
+          const int64_t off = tile_of(k) * (int64_t)(kBwRows * H * 2) + (int64_t)tid * 128;
+          tc::prefetch_l2(g.h2 + off);
+          tc::prefetch_l2(g.h1 + off);
+        }
+      }
+    };
+    static_assert(kBwRows * H * 2 == 512 * 128, "one line per epilogue thread per tile image");
+    prefetch_pair(0);
     fetch_dz(0, dzv[0]);
     fetch_dz(1, dzv[1]);
     for (int p = 0; p < npairs; ++p) {
       const uint32_t par = p & 1;
+      prefetch_pair(p + 1);
       for (int sl = 0; sl < 2; ++sl) {
         if (tid < kBwRows * 2) reinterpret_cast<uint4*>(s.dz[sl])[tid] = dzv[sl];
         handover(&s.dzin[sl]);
@@ -663,13 +688,29 @@ __global__ void __launch_bounds__(kWgThreads, 1) wgrad_kernel(WgArgs g) {
   if (warp == 0) tc::tmem_dealloc(tmem, 512);
 }
 
-// grad <- sum over the S sample chunks of each partial block, in chunk order
+// The rest of the minibatch gradient and its squared norm, in one launch of
+// kWgReduceBlocks blocks (all orders fixed, so the result is deterministic):
+//   - every weight and hidden-bias entry: the sum over the S sample chunks
+//     of its partial blocks, in chunk order;
+//   - block 0 also sums the loss kernel's block partials (lane-strided, then
+//     a fixed shuffle tree): the five minibatch statistics and the head-bias
+//     gradients (from the unrounded dz);
+//   - each block writes the fp32 sum of squares of the entries it wrote
+//     (threads in order of a fixed tree), the Adam kernel sums the blocks.
+constexpr int kWgReduceBlocks = 256;
+constexpr int kLossPartW = 32;  // loss-kernel partial row: pg, ent, kl, clip, vl, db3[16], dc3
+
 template <int D, int H>
-__global__ void wgrad_reduce_kernel(const float* __restrict__ part, int S, int A, float* __restrict__ grad) {
+__global__ void __launch_bounds__(256) wgrad_reduce_kernel(const float* __restrict__ part, int S, int A,
+                                                           float* __restrict__ grad, const float* __restrict__ lossp,
+                                                           int nlb, double* __restrict__ stat5,
+                                                           float* __restrict__ sq) {
   using Cn = WgCols<D>;
   constexpr int NCH = H / 256, MB = H / 128;
+  __shared__ float red[8];
   const MlpLayout Lp = mlp_layout(D, H, A);
   const int64_t total = (int64_t)2 * MB * NCH * 128 * kWgMaxCols;
+  float q = 0.0f;
   for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < total; i += (int64_t)gridDim.x * blockDim.x) {
     const int col = (int)(i % kWgMaxCols);
     const int row = (int)((i / kWgMaxCols) % 128);
@@ -691,8 +732,44 @@ __global__ void wgrad_reduce_kernel(const float* __restrict__ part, int S, int A
     float acc = 0.0f;
     for (int k = 0; k < S; ++k) acc += p[(int64_t)k * 128 * kWgMaxCols];
     grad[dst] = acc;
+    q = fmaf(acc, acc, q);
+  }
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (blockIdx.x == 0) {
+    // warp w: statistic w (w < 5), then head-bias sums j = w - 5 (policy j < A, then the value's)
+    for (int w = warp; w < 5 + A + 1; w += blockDim.x >> 5) {
+      if (w < 5) {
+        double t = 0.0;
+        for (int b = lane; b < nlb; b += 32) t += (double)lossp[(int64_t)b * kLossPartW + w];
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) t += __shfl_xor_sync(0xffffffffu, t, off);
+        if (lane == 0) stat5[w] = t;
+      } else {
+        const int j = w - 5;
+        const int col = j < A ? 5 + j : 21;
+        float t = 0.0f;
+        for (int b = lane; b < nlb; b += 32) t += lossp[(int64_t)b * kLossPartW + col];
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) t += __shfl_xor_sync(0xffffffffu, t, off);
+        if (lane == 0) {
+          grad[j < A ? Lp.b3 + j : Lp.c3] = t;
+          q = fmaf(t, t, q);
+        }
+      }
+    }
+  }
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) q += __shfl_xor_sync(0xffffffffu, q, off);
+  if (lane == 0) red[warp] = q;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    float t = 0.0f;
+    for (int w = 0; w < (int)(blockDim.x >> 5); ++w) t += red[w];
+    sq[blockIdx.x] = t;
   }
 }
+
+int wgrad_reduce_blocks() { return kWgReduceBlocks; }
 
 // ---------------------------------------------------------------------------
 // host side
@@ -705,7 +782,7 @@ template <int D, int H>
 static pe_status bwd_launch(const float* params, int A, uint8_t* const img[2], const uint8_t* x,
                             const uint8_t* const dz[2], const uint8_t* const h1[2], const uint8_t* const h2[2],
                             uint8_t* const da2[2], uint8_t* const da1[2], int64_t n, float* part, float* grad,
-                            int32_t* err, cudaStream_t st) {
+                            const float* lossp, int nlb, double* stat5, float* sq, int32_t* err, cudaStream_t st) {
   int dev = 0, sms = 0;
   PE_TRY_CUDA(cudaGetDevice(&dev));
   PE_TRY_CUDA(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
@@ -755,25 +832,27 @@ static pe_status bwd_launch(const float* params, int A, uint8_t* const img[2], c
     ProfScope ps(PE_PROF_PPO_GRAD, st);
     kern<<<groups * a.S, kWgThreads, bytes, st>>>(a);
     PE_CHECK_LAUNCH("wgrad_kernel");
-    wgrad_reduce_kernel<D, H><<<std::min<int64_t>(4096, ceil_div((int64_t)groups * 128 * kWgMaxCols, 256)), 256, 0, st>>>(
-        part, a.S, A, grad);
+    wgrad_reduce_kernel<D, H><<<kWgReduceBlocks, 256, 0, st>>>(part, a.S, A, grad, lossp, nlb, stat5, sq);
     PE_CHECK_LAUNCH("wgrad_reduce_kernel");
   }
   return PE_OK;
 }
 
 // the whole backward of both networks of a bf16 PPO minibatch step: writes
-// every weight and the hidden-layer biases of the gradient vector (the head
-// biases come from the loss kernel's partial sums)
+// every entry of the gradient vector (the head biases from the loss kernel's
+// partials), the five minibatch statistics, and kWgReduceBlocks partial sums
+// of squares of the gradient
 pe_status bf16_backward(const pe_net& net, const float* params, uint8_t* const img[2], const uint8_t* x,
                         const uint8_t* const dz[2], const uint8_t* const h1[2], const uint8_t* const h2[2],
                         uint8_t* const da2[2], uint8_t* const da1[2], int64_t n, float* part, float* grad,
-                        int32_t* err, cudaStream_t st) {
+                        const float* lossp, int nlb, double* stat5, float* sq, int32_t* err, cudaStream_t st) {
   if (n <= 0) return PE_OK;
   if (net.obs_dim == 32 && net.hidden == 256)
-    return bwd_launch<32, 256>(params, net.n_actions, img, x, dz, h1, h2, da2, da1, n, part, grad, err, st);
+    return bwd_launch<32, 256>(params, net.n_actions, img, x, dz, h1, h2, da2, da1, n, part, grad, lossp, nlb, stat5,
+                               sq, err, st);
   if (net.obs_dim == 64 && net.hidden == 512)
-    return bwd_launch<64, 512>(params, net.n_actions, img, x, dz, h1, h2, da2, da1, n, part, grad, err, st);
+    return bwd_launch<64, 512>(params, net.n_actions, img, x, dz, h1, h2, da2, da1, n, part, grad, lossp, nlb, stat5,
+                               sq, err, st);
   return fail(PE_EINVAL, "unsupported bf16 network for the backward pass");
 }
 

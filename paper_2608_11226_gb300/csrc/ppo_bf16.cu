@@ -14,8 +14,9 @@
 //                products and tanh derivatives (da2, da1), then the weight
 //                and hidden-bias gradients split over samples with a
 //                fixed-order reduction into the canonical gradient vector;
-//   step      -- head-bias and statistics sums, global norm, clip, Adam on
-//                the fp32 master parameters.
+//   step      -- the gradient's squared norm (summed with the weight
+//                gradients' reduction), clip, Adam on the fp32 master
+//                parameters.
 // Rounding points (which the oracle reproduces): dz, da2 and da1 enter the
 // products as bf16; the layer bias gradients sum the rounded values, the head
 // bias gradient the fp32 dz.
@@ -41,7 +42,8 @@ int64_t wgrad_partial_bytes();
 pe_status bf16_backward(const pe_net& net, const float* params, uint8_t* const img[2], const uint8_t* x,
                         const uint8_t* const dz[2], const uint8_t* const h1[2], const uint8_t* const h2[2],
                         uint8_t* const da2[2], uint8_t* const da1[2], int64_t n, float* part, float* grad,
-                        int32_t* err, cudaStream_t st);
+                        const float* lossp, int nlb, double* stat5, float* sq, int32_t* err, cudaStream_t st);
+int wgrad_reduce_blocks();
 
 constexpr int kHead = 16;   // head rows (logits; the value head padded with zero rows)
 constexpr int kTile = 128;  // rows of a tile image
@@ -163,52 +165,6 @@ __global__ void __launch_bounds__(kLossThreads) ppo_bf16_loss_kernel(LossArgs g)
   }
 }
 
-struct HeadArgs {
-  float* grad;
-  const float* lossp;  // [nlb][32]
-  double* stat5;       // [5] minibatch loss statistics out
-  int nlb, A;
-  int64_t ob3[2];
-};
-
-// head-bias gradients (from the unrounded dz) and the minibatch loss
-// statistics: one warp per sum, lane-strided then a fixed shuffle tree
-__global__ void head_assemble_kernel(HeadArgs a) {
-  const int warp = (int)((blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5), lane = threadIdx.x & 31;
-  if (warp < 5) {
-    double s = 0.0;
-    for (int b = lane; b < a.nlb; b += 32) s += (double)a.lossp[(int64_t)b * kPartW + warp];
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
-    if (lane == 0) a.stat5[warp] = s;
-  } else if (warp < 5 + a.A + 1) {
-    const int j = warp - 5;  // policy head bias j < A, then the value head bias
-    const int col = j < a.A ? 5 + j : 21;
-    float s = 0.0f;
-    for (int b = lane; b < a.nlb; b += 32) s += a.lossp[(int64_t)b * kPartW + col];
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
-    if (lane == 0) a.grad[j < a.A ? a.ob3[0] + j : a.ob3[1]] = s;
-  }
-}
-
-// fp32 sums of squares over 256 fixed blocks (fixed order: deterministic)
-__global__ void sumsq_kernel(const float* __restrict__ g, int64_t P, float* __restrict__ sq) {
-  __shared__ float red[32];
-  float s = 0.0f;
-  for (int64_t p = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; p < P; p += (int64_t)gridDim.x * blockDim.x)
-    s = fmaf(g[p], g[p], s);
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
-  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = s;
-  __syncthreads();
-  if (threadIdx.x == 0) {
-    float t = 0.0f;
-    for (int w = 0; w < (int)(blockDim.x >> 5); ++w) t += red[w];
-    sq[blockIdx.x] = t;
-  }
-}
-
 struct AdamBf16Args {
   float* params;
   float* m;
@@ -291,7 +247,7 @@ static Bf16Plan bf16_plan(const pe_net& net, const pe_ppo_config& cfg, int64_t N
   p.rows = (p.mb + kTile - 1) / kTile * kTile;
   p.nmb = (int)((N + cfg.minibatch - 1) / cfg.minibatch);
   p.nlb = (p.rows + kLossThreads - 1) / kLossThreads;
-  p.nsq = 256;
+  p.nsq = wgrad_reduce_blocks();
   p.img = bf16_image_bytes(net);
   p.bimg = al(bwd_image_bytes(p.H));
   const int64_t rows = p.rows, H = p.H;
@@ -355,7 +311,6 @@ pe_status ppo_update_bf16(const pe_net& net, float* params, float* m, float* v, 
   int32_t* err = reinterpret_cast<int32_t*>(acc + 8);
   double* stat5 = reinterpret_cast<double*>(at(pl.o_stat5));
   const int A = pl.A;
-  const MlpLayout Lp = mlp_layout(pl.D, pl.H, A);
   PE_TRY_CUDA(cudaMemsetAsync(acc, 0, 8 * 8 + 8, st));
   pe_status s = launch_advstats(adv, N, cfg.minibatch, pl.nmb, cfg.epochs, cfg.seed, cfg.iteration, advstat, st);
   if (s != PE_OK) return s;
@@ -403,16 +358,8 @@ pe_status ppo_update_bf16(const pe_net& net, float* params, float* m, float* v, 
       }
       PE_CHECK_LAUNCH("ppo_bf16_loss_kernel");
       s = bf16_backward(net, params, bimg, reinterpret_cast<const uint8_t*>(x), dzc, h1c, h2c, da2, da1, cnt, part,
-                        grad, err, st);
+                        grad, lossp, nlb, stat5, sq, err, st);
       if (s != PE_OK) return s;
-      HeadArgs ha;
-      ha.grad = grad;
-      ha.lossp = lossp;
-      ha.stat5 = stat5;
-      ha.nlb = nlb;
-      ha.A = A;
-      ha.ob3[0] = Lp.b3;
-      ha.ob3[1] = Lp.c3;
       t += 1;
       AdamBf16Args ad;
       ad.params = params;
@@ -435,8 +382,6 @@ pe_status ppo_update_bf16(const pe_net& net, float* params, float* m, float* v, 
       ad.acc = acc;
       {
         ProfScope ps(PE_PROF_PPO_ADAM, st);
-        head_assemble_kernel<<<ceil_div((5 + A + 1) * 32, 256), 256, 0, st>>>(ha);
-        sumsq_kernel<<<pl.nsq, 256, 0, st>>>(grad, pl.P, sq);
         adam_bf16_kernel<<<ceil_div(pl.P, 256), 256, 0, st>>>(ad);
       }
       PE_CHECK_LAUNCH("ppo bf16 step kernels");

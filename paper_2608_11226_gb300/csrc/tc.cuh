@@ -146,6 +146,11 @@ __device__ __forceinline__ bool bar_any(int id, int nthreads, bool pred) {
   return r != 0;
 }
 
+// ask L2 to fetch the 128-byte line holding p (no register result, no wait)
+__device__ __forceinline__ void prefetch_l2(const void* p) {
+  asm volatile("prefetch.global.L2 [%0];" ::"l"(p));
+}
+
 // ---------------------------------------------------------------- mbarriers
 __device__ __forceinline__ void mbar_init(uint64_t* b, uint32_t count) {
   asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(b)), "r"(count) : "memory");
