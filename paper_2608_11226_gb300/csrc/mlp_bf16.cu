@@ -681,12 +681,14 @@ __global__ void __launch_bounds__(128) env_actobs_kernel(EnvDev env, ActArgs a, 
     float lp;
     const int act = sample_action<A>(z, r, a.det != 0, &lp);
     const StepOut so = env_step<C>(env, acc, act, a.lambda);
+    // the rollout buffer is not read again during the rollout: streaming
+    // stores (evict first) keep L2 for the env state, the rings and the logits
     const int64_t row = (int64_t)a.t * env.E + e;
-    buf.act[row] = (uint8_t)act;
-    buf.logp[row] = lp;
-    buf.reward[row] = so.reward;
-    buf.done[row] = (uint8_t)so.done;
-    if (buf.q) buf.q[row] = so.q;
+    __stcs(buf.act + row, (uint8_t)act);
+    __stcs(buf.logp + row, lp);
+    __stcs(buf.reward + row, so.reward);
+    __stcs(buf.done + row, (uint8_t)so.done);
+    if (buf.q) __stcs(buf.q + row, so.q);
     if (a.t == 0) {
       buf.viol[2 * e] = so.v1;
       buf.viol[2 * e + 1] = so.v60;
@@ -716,7 +718,7 @@ __global__ void __launch_bounds__(128) env_actobs_kernel(EnvDev env, ActArgs a, 
     uint32_t p[4];
 #pragma unroll
     for (int i = 0; i < 4; ++i) p[i] = tc::pack_bf16(o[f0 + 2 * i], o[f0 + 2 * i + 1]);
-    *reinterpret_cast<uint4*>(dst + f0) = make_uint4(p[0], p[1], p[2], p[3]);
+    __stcs(reinterpret_cast<uint4*>(dst + f0), make_uint4(p[0], p[1], p[2], p[3]));
   }
   store_reg<C>(env, e, acc);
 }
