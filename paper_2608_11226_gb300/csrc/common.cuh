@@ -145,6 +145,28 @@ __device__ __forceinline__ float kl_term(float x) {
   return expm1f(x) - x;
 }
 
+// The PPO loss of a minibatch, taken in the forward pass's head epilogue
+// (Sec. 4.2; SB3's clipped surrogate, squared-error value loss and entropy
+// bonus).  Row r of the minibatch is sample gather[r]; the thread that reads
+// the row's head from TMEM computes the loss terms and dLoss/dhead, writes
+// dz -- rounded to bf16 -- into the dz tile image (16 bf16 per row, 32-byte
+// rows, 32-byte swizzle; rows past the minibatch are zero), and each head
+// warp writes the fixed-order (shuffle tree) sums of its 32 rows as one
+// partial row: columns 0-3 pg loss, entropy, approximate KL, clip indicator
+// and 5..5+A-1 the policy head-bias gradient (policy network), column 4 the
+// value loss and 21 the value head-bias gradient (value network), both from
+// the unrounded dz.
+struct PpoHead {
+  const uint8_t* act;
+  const float* logp_old;
+  const float* adv;
+  const float* ret;
+  const float2* advstat;  // (mean, 1 / (std + 1e-8)) of the minibatch's advantages
+  float clip, vf_coef, ent_coef, inv_cnt;
+  uint8_t* dz;            // dz tile images of this network
+  float* part;            // [tiles * 4][32] partial rows
+};
+
 inline int ceil_div(int64_t a, int64_t b) { return (int)((a + b - 1) / b); }
 
 // launch profiling: brackets a launch with CUDA events when enabled

@@ -42,11 +42,103 @@ struct MlpSave {
   __nv_bfloat16* x;        // tiles of 128 x D, or NULL
   __nv_bfloat16* h1;       // tiles of 128 x H, or NULL
   __nv_bfloat16* h2;       // tiles of 128 x H, or NULL
+  PpoHead loss;            // loss.dz != NULL: the PPO loss replaces the head output
 };
 
 constexpr int kTcRows = 128;     // rows (envs / samples) per tile, the MMA M
 constexpr int kTcThreads = 512;  // 16 warps: 4 TMEM lane quadrants x 4 column slices
 constexpr int kHeadN = 16;       // head width (logits or value padded to 16)
+
+// Head epilogue of a PPO forward pass for row `row` (0..127) of tile `tile`:
+// z[16] are the head accumulators of the row (before the bias).  Called by
+// all 32 lanes of a head warp (warp < 4); rows past n contribute zero.
+__device__ __forceinline__ void ppo_head_row(const PpoHead& L, int value_net, int A, const float* b3,
+                                             const uint32_t* gather, int64_t tile, int row, int64_t n,
+                                             const float (&acc)[16], int warp) {
+  constexpr int kW = 32;
+  const int64_t j = tile * kTcRows + row;
+  const bool valid = j < n;
+  float v[22];
+#pragma unroll
+  for (int k = 0; k < 22; ++k) v[k] = 0.0f;
+  uint32_t pk[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+  if (valid) {
+    const uint32_t i = gather[j];
+    if (!value_net) {
+      const float2 as = *L.advstat;
+      float z[kHeadN];
+#pragma unroll
+      for (int a = 0; a < kHeadN; ++a) z[a] = a < A ? acc[a] + b3[a] : -INFINITY;
+      float m = z[0];
+#pragma unroll
+      for (int a = 1; a < kHeadN; ++a) m = fmaxf(m, z[a]);
+      float se = 0.0f;
+#pragma unroll
+      for (int a = 0; a < kHeadN; ++a) se += a < A ? expf(z[a] - m) : 0.0f;
+      const float lse = m + logf(se);
+      float lp[kHeadN], pr[kHeadN], Hs = 0.0f;
+#pragma unroll
+      for (int a = 0; a < kHeadN; ++a) {
+        lp[a] = a < A ? z[a] - lse : 0.0f;
+        pr[a] = a < A ? expf(lp[a]) : 0.0f;
+        Hs -= pr[a] * lp[a];
+      }
+      const int act = L.act[i];
+      const float an = (L.adv[i] - as.x) * as.y;
+      float lpa = 0.0f;
+#pragma unroll
+      for (int a = 0; a < kHeadN; ++a)
+        if (a == act) lpa = lp[a];
+      const float logr = lpa - L.logp_old[i];
+      const float rho = expf(logr);
+      const float rc = fminf(fmaxf(rho, 1.0f - L.clip), 1.0f + L.clip);
+      const float s1 = rho * an, s2 = rc * an;
+      v[0] = -fminf(s1, s2);
+      v[1] = Hs;
+      v[2] = kl_term(logr);
+      v[3] = fabsf(rho - 1.0f) > L.clip ? 1.0f : 0.0f;
+      const float dlp = (s1 <= s2 ? -an : 0.0f) * rho * L.inv_cnt;
+#pragma unroll
+      for (int a = 0; a < kHeadN; a += 2) {
+        float d0 = 0.0f, d1 = 0.0f;
+        if (a < A) d0 = dlp * ((a == act ? 1.0f : 0.0f) - pr[a]) + L.ent_coef * L.inv_cnt * pr[a] * (lp[a] + Hs);
+        if (a + 1 < A)
+          d1 = dlp * ((a + 1 == act ? 1.0f : 0.0f) - pr[a + 1]) + L.ent_coef * L.inv_cnt * pr[a + 1] * (lp[a + 1] + Hs);
+        v[5 + a] = d0;
+        v[5 + a + 1] = d1;
+        pk[a / 2] = tc::pack_bf16(d0, d1);
+      }
+    } else {
+      const float V = acc[0] + b3[0], R = L.ret[i];
+      v[4] = (R - V) * (R - V);
+      const float dV = L.vf_coef * 2.0f * (V - R) * L.inv_cnt;
+      v[21] = dV;
+      pk[0] = tc::pack_bf16(dV, 0.0f);
+    }
+  }
+  // dz row (zeros past the minibatch): 16-byte chunk c at (c ^ ((row >> 2) & 1)) * 16
+  uint8_t* dzr = L.dz + tile * (int64_t)(kTcRows * 32) + row * 32;
+  const int sw = (row >> 2) & 1;
+  *reinterpret_cast<uint4*>(dzr + (sw << 4)) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+  *reinterpret_cast<uint4*>(dzr + ((1 ^ sw) << 4)) = make_uint4(pk[4], pk[5], pk[6], pk[7]);
+  // this warp's partial row
+#pragma unroll
+  for (int k = 0; k < 22; ++k)
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v[k] += __shfl_xor_sync(0xffffffffu, v[k], o);
+  if ((threadIdx.x & 31) == 0) {
+    float* pr = L.part + (tile * 4 + warp) * kW;
+    if (!value_net) {
+#pragma unroll
+      for (int k = 0; k < 4; ++k) pr[k] = v[k];
+#pragma unroll
+      for (int k = 5; k < 21; ++k) pr[k] = v[k];
+    } else {
+      pr[4] = v[4];
+      pr[21] = v[21];
+    }
+  }
+}
 
 // byte sizes of the weight image parts of one network (D, H)
 template <int D, int H>
@@ -350,7 +442,9 @@ __global__ void __launch_bounds__(kStreamThreads, 1)
       if (warp < 4) {
         float v[16];
         tc::tmem_ld16(lane_addr, v);
-        if (row < nr) {
+        if (save.loss.dz) {
+          ppo_head_row(save.loss, value_net, A, s.b3, save.gather, tile, row, n, v, warp);
+        } else if (row < nr) {
           float* o = out + (rbase + row) * out_stride;
 #pragma unroll
           for (int j = 0; j < kHeadN; ++j)
@@ -553,7 +647,9 @@ __global__ void __launch_bounds__(kPairThreads, 1)
         const int nr = (int)(n - tl * kTcRows < kTcRows ? n - tl * kTcRows : kTcRows);
         float v[16];
         tc::tmem_ld16(lane_base + (uint32_t)(sl * 256), v);
-        if (row < nr) {
+        if (save.loss.dz) {
+          ppo_head_row(save.loss, value_net, A, s.b3, save.gather, tl, row, n, v, warp);
+        } else if (row < nr) {
           float* o = out + (tl * kTcRows + row) * out_stride;
 #pragma unroll
           for (int j = 0; j < kHeadN; ++j)
@@ -881,11 +977,13 @@ pe_status bf16_make_images(const pe_net& net, const float* params, uint8_t* two_
   return fail(PE_EINVAL, "unsupported bf16 network");
 }
 
-pe_status bf16_forward_save(const pe_net& net, const uint8_t* img, const float* params, int value_net,
-                            const void* obs, const uint32_t* gather, int64_t n, float* out, int out_stride,
+pe_status bf16_forward_loss(const pe_net& net, const uint8_t* img, const float* params, int value_net,
+                            const void* obs, const uint32_t* gather, int64_t n, const PpoHead& loss,
                             __nv_bfloat16* x, __nv_bfloat16* h1, __nv_bfloat16* h2, int32_t* err,
                             cudaStream_t st) {
-  const MlpSave sv{gather, x, h1, h2};
+  const MlpSave sv{gather, x, h1, h2, loss};
+  float* out = nullptr;
+  const int out_stride = 0;
   const int nout = value_net ? 1 : net.n_actions;
   if (net.obs_dim == 32 && net.hidden == 256)
     return launch_mlp<32, 256>(img, params, net.n_actions, value_net, obs, n, out, out_stride, nout, err, st,

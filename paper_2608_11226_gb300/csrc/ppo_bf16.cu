@@ -6,10 +6,11 @@
 //                Feistel-permuted rows, saving x, h1, h2 (bf16) as 128-row
 //                tile images (the kernels' swizzled shared-memory layout)
 //                besides the heads;
-//   loss      -- one thread per sample: clipped surrogate, value loss,
-//                entropy; dLoss/dhead in fp32, rounded to bf16 into dz tile
-//                images (zero rows past the minibatch), fixed-order block
-//                partials of the head-bias gradients and the statistics;
+//   loss      -- in the forward kernels' head epilogue, one thread per
+//                sample: clipped surrogate, value loss, entropy; dLoss/dhead
+//                in fp32, rounded to bf16 into dz tile images (zero rows past
+//                the minibatch), fixed-order per-warp partials of the
+//                head-bias gradients and the statistics;
 //   backward  -- on the tensor cores (bwd_bf16.cu): per network the data
 //                products and tanh derivatives (da2, da1), then the weight
 //                and hidden-bias gradients split over samples with a
@@ -31,8 +32,8 @@ namespace pe {
 // defined in mlp_bf16.cu / ppo_f32.cu / bwd_bf16.cu
 int64_t bf16_image_bytes(const pe_net& net);
 pe_status bf16_make_images(const pe_net& net, const float* params, uint8_t* two_images, cudaStream_t st);
-pe_status bf16_forward_save(const pe_net& net, const uint8_t* img, const float* params, int value_net,
-                            const void* obs, const uint32_t* gather, int64_t n, float* out, int out_stride,
+pe_status bf16_forward_loss(const pe_net& net, const uint8_t* img, const float* params, int value_net,
+                            const void* obs, const uint32_t* gather, int64_t n, const PpoHead& loss,
                             __nv_bfloat16* x, __nv_bfloat16* h1, __nv_bfloat16* h2, int32_t* err,
                             cudaStream_t st);
 pe_status launch_advstats(const float* adv, int64_t N, int M, int nmb, int epochs, uint64_t seed,
@@ -56,114 +57,7 @@ __global__ void perm_index_kernel(Feistel f, int64_t start, int cnt, uint32_t* _
   if (j < cnt) idx[j] = feistel_index(f, start + j);
 }
 
-struct LossArgs {
-  const float* zp;  // [cnt][16] policy logits
-  const float* zv;  // [cnt] values
-  const uint32_t* idx;
-  const uint8_t* act;
-  const float* logp_old;
-  const float* adv;
-  const float* ret;
-  const float2* advstat;
-  int cnt, rows, A;  // rows: cnt rounded up to whole tiles
-  float clip, vf_coef, ent_coef, inv_cnt;
-  uint8_t* dzp;  // dz tile images (policy: 16 columns), 32-byte rows, SW32 swizzle
-  uint8_t* dzv;  // (value: column 0)
-  float* part;   // [nblk][32]: pg, ent, kl, clip, vl, db3[16], dc3
-};
-
-constexpr int kLossThreads = 256;
-constexpr int kPartW = 32;
-
-// byte offset of 16-byte chunk c (0: columns 0-7, 1: columns 8-15) of row j
-// of a dz tile image
-__device__ __forceinline__ int64_t dz_chunk(int64_t j, int c) {
-  const int r = (int)(j % kTile);
-  return (j / kTile) * (kTile * 32) + r * 32 + ((c ^ ((r >> 2) & 1)) << 4);
-}
-
-__global__ void __launch_bounds__(kLossThreads) ppo_bf16_loss_kernel(LossArgs g) {
-  __shared__ float red[kLossThreads / 32][kPartW];
-  const int j = blockIdx.x * blockDim.x + threadIdx.x;
-  float v[kPartW];
-#pragma unroll
-  for (int k = 0; k < kPartW; ++k) v[k] = 0.0f;
-  uint32_t pk[kHead / 2] = {0, 0, 0, 0, 0, 0, 0, 0};
-  uint32_t pv = 0;
-  if (j < g.cnt) {
-    const uint32_t i = g.idx[j];
-    const float2 as = *g.advstat;
-    float z[kHead];
-#pragma unroll
-    for (int a = 0; a < kHead; ++a) z[a] = a < g.A ? g.zp[(int64_t)j * kHead + a] : -INFINITY;
-    float m = z[0];
-#pragma unroll
-    for (int a = 1; a < kHead; ++a) m = fmaxf(m, z[a]);
-    float se = 0.0f;
-#pragma unroll
-    for (int a = 0; a < kHead; ++a) se += a < g.A ? expf(z[a] - m) : 0.0f;
-    const float lse = m + logf(se);
-    float lp[kHead], p[kHead], Hs = 0.0f;
-#pragma unroll
-    for (int a = 0; a < kHead; ++a) {
-      lp[a] = a < g.A ? z[a] - lse : 0.0f;
-      p[a] = a < g.A ? expf(lp[a]) : 0.0f;
-      Hs -= p[a] * lp[a];
-    }
-    const int act = g.act[i];
-    const float an = (g.adv[i] - as.x) * as.y;
-    float lpa = 0.0f;
-#pragma unroll
-    for (int a = 0; a < kHead; ++a)
-      if (a == act) lpa = lp[a];
-    const float logr = lpa - g.logp_old[i];
-    const float rho = expf(logr);
-    const float rc = fminf(fmaxf(rho, 1.0f - g.clip), 1.0f + g.clip);
-    const float s1 = rho * an, s2 = rc * an;
-    v[0] = -fminf(s1, s2);
-    v[1] = Hs;
-    v[2] = kl_term(logr);
-    v[3] = fabsf(rho - 1.0f) > g.clip ? 1.0f : 0.0f;
-    const float dlp = (s1 <= s2 ? -an : 0.0f) * rho * g.inv_cnt;
-#pragma unroll
-    for (int a = 0; a < kHead; a += 2) {
-      float d0 = 0.0f, d1 = 0.0f;
-      if (a < g.A) d0 = dlp * ((a == act ? 1.0f : 0.0f) - p[a]) + g.ent_coef * g.inv_cnt * p[a] * (lp[a] + Hs);
-      if (a + 1 < g.A)
-        d1 = dlp * ((a + 1 == act ? 1.0f : 0.0f) - p[a + 1]) + g.ent_coef * g.inv_cnt * p[a + 1] * (lp[a + 1] + Hs);
-      v[5 + a] = d0;
-      v[5 + a + 1] = d1;
-      __nv_bfloat162 b2 = __floats2bfloat162_rn(d0, d1);
-      pk[a / 2] = *reinterpret_cast<uint32_t*>(&b2);
-    }
-    const float V = g.zv[j], R = g.ret[i];
-    v[4] = (R - V) * (R - V);
-    const float dV = g.vf_coef * 2.0f * (V - R) * g.inv_cnt;
-    v[21] = dV;
-    __nv_bfloat162 b2 = __floats2bfloat162_rn(dV, 0.0f);
-    pv = *reinterpret_cast<uint32_t*>(&b2);
-  }
-  if (j < g.rows) {  // rows past the minibatch are written as zeros
-    *reinterpret_cast<uint4*>(g.dzp + dz_chunk(j, 0)) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
-    *reinterpret_cast<uint4*>(g.dzp + dz_chunk(j, 1)) = make_uint4(pk[4], pk[5], pk[6], pk[7]);
-    *reinterpret_cast<uint4*>(g.dzv + dz_chunk(j, 0)) = make_uint4(pv, 0u, 0u, 0u);
-    *reinterpret_cast<uint4*>(g.dzv + dz_chunk(j, 1)) = make_uint4(0u, 0u, 0u, 0u);
-  }
-  // fixed-order block partial sums
-#pragma unroll
-  for (int k = 0; k < kPartW; ++k)
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) v[k] += __shfl_xor_sync(0xffffffffu, v[k], o);
-  if ((threadIdx.x & 31) == 0)
-#pragma unroll
-    for (int k = 0; k < kPartW; ++k) red[threadIdx.x >> 5][k] = v[k];
-  __syncthreads();
-  if (threadIdx.x < kPartW) {
-    float t = 0.0f;
-    for (int w = 0; w < kLossThreads / 32; ++w) t += red[w][threadIdx.x];
-    g.part[(int64_t)blockIdx.x * kPartW + threadIdx.x] = t;
-  }
-}
+constexpr int kPartW = 32;  // partial row of the fused loss: pg, ent, kl, clip, vl, db3[16], dc3
 
 struct AdamBf16Args {
   float* params;
@@ -230,7 +124,7 @@ struct Bf16Plan {
   int64_t P, N;
   int nmb, mb, rows, D, H, A, nlb, nsq;
   int64_t img, bimg;
-  int64_t o_adv, o_idx, o_img, o_bimg, o_x, o_h[4], o_zp, o_zv, o_dz[2], o_da2[2], o_da1[2], o_part, o_loss,
+  int64_t o_adv, o_idx, o_img, o_bimg, o_x, o_h[4], o_dz[2], o_da2[2], o_da1[2], o_part, o_loss,
       o_grad, o_sq, o_acc, o_stat5, total;
 };
 
@@ -246,7 +140,7 @@ static Bf16Plan bf16_plan(const pe_net& net, const pe_ppo_config& cfg, int64_t N
   p.mb = (int)std::min<int64_t>(cfg.minibatch, N);
   p.rows = (p.mb + kTile - 1) / kTile * kTile;
   p.nmb = (int)((N + cfg.minibatch - 1) / cfg.minibatch);
-  p.nlb = (p.rows + kLossThreads - 1) / kLossThreads;
+  p.nlb = p.rows / kTile * 4;  // one partial row per head warp (4 per tile)
   p.nsq = wgrad_reduce_blocks();
   p.img = bf16_image_bytes(net);
   p.bimg = al(bwd_image_bytes(p.H));
@@ -258,8 +152,6 @@ static Bf16Plan bf16_plan(const pe_net& net, const pe_ppo_config& cfg, int64_t N
   p.o_bimg = o; o = al(o + 2 * p.bimg);
   p.o_x = o; o = al(o + rows * p.D * 2);
   for (int i = 0; i < 4; ++i) { p.o_h[i] = o; o = al(o + rows * H * 2); }
-  p.o_zp = o; o = al(o + rows * kHead * 4);
-  p.o_zv = o; o = al(o + rows * 4);
   for (int i = 0; i < 2; ++i) { p.o_dz[i] = o; o = al(o + rows * 32); }
   for (int i = 0; i < 2; ++i) { p.o_da2[i] = o; o = al(o + rows * H * 2); }
   for (int i = 0; i < 2; ++i) { p.o_da1[i] = o; o = al(o + rows * H * 2); }
@@ -295,8 +187,6 @@ pe_status ppo_update_bf16(const pe_net& net, float* params, float* m, float* v, 
   __nv_bfloat16* x = reinterpret_cast<__nv_bfloat16*>(at(pl.o_x));
   __nv_bfloat16* h[4];
   for (int i = 0; i < 4; ++i) h[i] = reinterpret_cast<__nv_bfloat16*>(at(pl.o_h[i]));
-  float* zp = reinterpret_cast<float*>(at(pl.o_zp));
-  float* zv = reinterpret_cast<float*>(at(pl.o_zv));
   uint8_t* const dz[2] = {u8(pl.o_dz[0]), u8(pl.o_dz[1])};
   uint8_t* const da2[2] = {u8(pl.o_da2[0]), u8(pl.o_da2[1])};
   uint8_t* const da1[2] = {u8(pl.o_da1[0]), u8(pl.o_da1[1])};
@@ -328,35 +218,24 @@ pe_status ppo_update_bf16(const pe_net& net, float* params, float* m, float* v, 
       PE_CHECK_LAUNCH("perm_index_kernel");
       s = bf16_make_images(net, params, img, st);
       if (s != PE_OK) return s;
-      s = bf16_forward_save(net, img, params, 0, obs, idx, cnt, zp, kHead, x, h[0], h[1], err, st);
+      PpoHead lh;
+      lh.act = act;
+      lh.logp_old = logp_old;
+      lh.adv = adv;
+      lh.ret = ret;
+      lh.advstat = advstat + (int64_t)ep * pl.nmb + mbi;
+      lh.clip = cfg.clip;
+      lh.vf_coef = cfg.vf_coef;
+      lh.ent_coef = cfg.ent_coef;
+      lh.inv_cnt = 1.0f / (float)cnt;
+      lh.part = lossp;
+      lh.dz = dz[0];
+      s = bf16_forward_loss(net, img, params, 0, obs, idx, cnt, lh, x, h[0], h[1], err, st);
       if (s != PE_OK) return s;
-      s = bf16_forward_save(net, img + pl.img, params, 1, obs, idx, cnt, zv, 1, nullptr, h[2], h[3], err, st);
+      lh.dz = dz[1];
+      s = bf16_forward_loss(net, img + pl.img, params, 1, obs, idx, cnt, lh, nullptr, h[2], h[3], err, st);
       if (s != PE_OK) return s;
-      LossArgs la;
-      la.zp = zp;
-      la.zv = zv;
-      la.idx = idx;
-      la.act = act;
-      la.logp_old = logp_old;
-      la.adv = adv;
-      la.ret = ret;
-      la.advstat = advstat + (int64_t)ep * pl.nmb + mbi;
-      la.cnt = cnt;
-      la.rows = rows;
-      la.A = A;
-      la.clip = cfg.clip;
-      la.vf_coef = cfg.vf_coef;
-      la.ent_coef = cfg.ent_coef;
-      la.inv_cnt = 1.0f / (float)cnt;
-      la.dzp = dz[0];
-      la.dzv = dz[1];
-      la.part = lossp;
-      const int nlb = ceil_div(rows, kLossThreads);
-      {
-        ProfScope ps(PE_PROF_PPO_OTHER, st);
-        ppo_bf16_loss_kernel<<<nlb, kLossThreads, 0, st>>>(la);
-      }
-      PE_CHECK_LAUNCH("ppo_bf16_loss_kernel");
+      const int nlb = rows / kTile * 4;
       s = bf16_backward(net, params, bimg, reinterpret_cast<const uint8_t*>(x), dzc, h1c, h2c, da2, da1, cnt, part,
                         grad, lossp, nlb, stat5, sq, err, st);
       if (s != PE_OK) return s;
