@@ -692,9 +692,10 @@ __global__ void __launch_bounds__(kWgThreads, 1) wgrad_kernel(WgArgs g) {
 // kWgReduceBlocks blocks (all orders fixed, so the result is deterministic):
 //   - every weight and hidden-bias entry: the sum over the S sample chunks
 //     of its partial blocks, in chunk order;
-//   - block 0 also sums the loss kernel's block partials (lane-strided, then
-//     a fixed shuffle tree): the five minibatch statistics and the head-bias
-//     gradients (from the unrounded dz);
+//   - blocks 0 .. 5 + A also sum the loss partial rows, one quantity per
+//     block (the five minibatch statistics, then the head-bias gradients
+//     from the unrounded dz): thread t takes rows t, t + 256, ... in order,
+//     then a fixed shuffle tree and the warps in order;
 //   - each block writes the fp32 sum of squares of the entries it wrote
 //     (threads in order of a fixed tree), the Adam kernel sums the blocks.
 constexpr int kWgReduceBlocks = 256;
@@ -735,26 +736,27 @@ __global__ void __launch_bounds__(256) wgrad_reduce_kernel(const float* __restri
     q = fmaf(acc, acc, q);
   }
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  if (blockIdx.x == 0) {
-    // warp w: statistic w (w < 5), then head-bias sums j = w - 5 (policy j < A, then the value's)
-    for (int w = warp; w < 5 + A + 1; w += blockDim.x >> 5) {
-      if (w < 5) {
-        double t = 0.0;
-        for (int b = lane; b < nlb; b += 32) t += (double)lossp[(int64_t)b * kLossPartW + w];
+  __shared__ double redd[8];
+  const int w = (int)blockIdx.x;  // statistic w (w < 5), then head-bias sum j = w - 5 (policy j < A, then the value's)
+  if (w < 5 + A + 1) {
+    const int col = w < 5 ? w : (w - 5 < A ? 5 + (w - 5) : 21);
+    double t = 0.0;
+#pragma unroll 4
+    for (int b = threadIdx.x; b < nlb; b += blockDim.x) t += (double)lossp[(int64_t)b * kLossPartW + col];
 #pragma unroll
-        for (int off = 16; off > 0; off >>= 1) t += __shfl_xor_sync(0xffffffffu, t, off);
-        if (lane == 0) stat5[w] = t;
+    for (int off = 16; off > 0; off >>= 1) t += __shfl_xor_sync(0xffffffffu, t, off);
+    if (lane == 0) redd[warp] = t;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      double u = 0.0;
+      for (int k = 0; k < (int)(blockDim.x >> 5); ++k) u += redd[k];
+      if (w < 5) {
+        stat5[w] = u;
       } else {
         const int j = w - 5;
-        const int col = j < A ? 5 + j : 21;
-        float t = 0.0f;
-        for (int b = lane; b < nlb; b += 32) t += lossp[(int64_t)b * kLossPartW + col];
-#pragma unroll
-        for (int off = 16; off > 0; off >>= 1) t += __shfl_xor_sync(0xffffffffu, t, off);
-        if (lane == 0) {
-          grad[j < A ? Lp.b3 + j : Lp.c3] = t;
-          q = fmaf(t, t, q);
-        }
+        const float g = (float)u;
+        grad[j < A ? Lp.b3 + j : Lp.c3] = g;
+        q = fmaf(g, g, q);
       }
     }
   }
@@ -764,7 +766,7 @@ __global__ void __launch_bounds__(256) wgrad_reduce_kernel(const float* __restri
   __syncthreads();
   if (threadIdx.x == 0) {
     float t = 0.0f;
-    for (int w = 0; w < (int)(blockDim.x >> 5); ++w) t += red[w];
+    for (int k = 0; k < (int)(blockDim.x >> 5); ++k) t += red[k];
     sq[blockIdx.x] = t;
   }
 }
