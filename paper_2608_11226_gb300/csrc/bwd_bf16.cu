@@ -21,7 +21,9 @@
 //   da2 = bf16(dh2 (1 - h2^2)) into shared memory (the next A operand) and
 //   its tile image; dh1 = da2 W2 with W2^T streamed through a two-slot ring
 //   of 32 KB stages by a producer warp; epilogue: da1 = bf16(dh1 (1 - h1^2))
-//   to its tile image.
+//   to its tile image.  A loader warp brings the tile's h2 image into the da2
+//   buffer with one bulk copy (da2 then overwrites it in place) and, after
+//   the dh1 MMAs, its h1 image, so the epilogues read h from shared memory.
 // wgrad_kernel (split over samples): each CTA owns 128 output rows (one
 //   block of layer outputs o) of one network and one 256-column chunk, and
 //   accumulates over its share of the minibatch, 64 samples per stage:
@@ -40,7 +42,7 @@ namespace pe {
 constexpr int kBwRows = 128;            // samples per tile (MMA M of the data products)
 constexpr int kBwStage = 32768;         // one streamed W2^T stage: 256 rows x 64 K, SW128
 constexpr int kBwCompute = 512;         // 16 compute warps
-constexpr int kBwThreads = kBwCompute + 32;  // + the producer warp
+constexpr int kBwThreads = kBwCompute + 64;  // + the W2^T producer warp and the h loader warp
 
 // backward weight image of one network: W3^T (H rows x 16, K-major SW32),
 // then the W2^T stages: stage (h, kb) = rows i in [256 h, 256 h + 256) of
@@ -86,11 +88,17 @@ __global__ void bwd_image_kernel(const float* __restrict__ params, int A, uint8_
 
 template <int H>
 struct BwdSmem {
-  alignas(1024) uint8_t da2[kBwRows * H * 2];  // A operand of dh1 = da2 W2 (K-major SW128)
+  // A operand of dh1 = da2 W2 (K-major SW128).  Each tile's h2 image arrives
+  // here first and da2 overwrites it in place (da2 is elementwise in h2);
+  // after the dh1 MMAs the h1 image arrives here for the second epilogue.
+  alignas(1024) uint8_t da2[kBwRows * H * 2];
   alignas(1024) uint8_t ring[2][kBwStage];
   alignas(1024) uint8_t w3t[H * 32];           // B operand of dh2 = dz W3 (K-major SW32)
   alignas(1024) uint8_t dz[kBwRows * 32];      // A operand of dh2 (K-major SW32)
   uint64_t full[2], empty[2], bar_mma, bar_w;
+  uint64_t hin;     // an h image landed in da2 (two completions per tile: h2, then h1)
+  uint64_t dh1;     // the tile's dh1 MMAs are done (da2 may be overwritten by h1)
+  uint64_t bfree;   // the 16 compute warps finished reading h1 (the buffer may take the next h2)
   uint32_t tmem_base;
   int32_t err;
 };
@@ -123,6 +131,7 @@ struct BwdArgs {
 template <int H>
 __global__ void __launch_bounds__(kBwThreads, 1) bwd_data_kernel(BwdArgs g) {
   using I = BwdImg<H>;
+  constexpr int kTileBytes = kBwRows * H * 2;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
   BwdSmem<H>& s = *reinterpret_cast<BwdSmem<H>*>(base);
@@ -135,6 +144,9 @@ __global__ void __launch_bounds__(kBwThreads, 1) bwd_data_kernel(BwdArgs g) {
     }
     tc::mbar_init(&s.bar_mma, 1);
     tc::mbar_init(&s.bar_w, 1);
+    tc::mbar_init(&s.hin, 1);
+    tc::mbar_init(&s.dh1, 1);
+    tc::mbar_init(&s.bfree, kBwCompute / 32);
     tc::fence_mbar_init();
   }
   if (warp == 0) tc::tmem_alloc(&s.tmem_base, H);
@@ -149,6 +161,7 @@ __global__ void __launch_bounds__(kBwThreads, 1) bwd_data_kernel(BwdArgs g) {
     tc::bulk_g2s(s.w3t, g.img, (uint32_t)I::W3T, &s.bar_w);
   }
   int last_issued = -1;  // producer: global index of its last issued stage
+  int h_issued = 0;      // loader: h copies issued (the hin phases)
   if (warp == kBwCompute / 32) {
     // producer: the W2^T stages of every tile, in consumption order
     if (lane == 0) {
@@ -167,6 +180,29 @@ __global__ void __launch_bounds__(kBwThreads, 1) bwd_data_kernel(BwdArgs g) {
         }
       }
     }
+  } else if (warp == kBwCompute / 32 + 1) {
+    // loader: per tile, the h2 image into the da2 buffer once the previous
+    // tile's second epilogue has read h1 out of it, then the h1 image once
+    // the dh1 MMAs have read da2
+    if (lane == 0) {
+      for (int t = 0; t < my_tiles; ++t) {
+        const int64_t tile = blockIdx.x + (int64_t)t * gridDim.x;
+        if (t > 0 && !tc::mbar_wait(&s.bfree, (t - 1) & 1)) {
+          atomicExch(&s.err, 1);
+          break;
+        }
+        tc::mbar_expect_tx(&s.hin, (uint32_t)kTileBytes);
+        tc::bulk_g2s(s.da2, g.h2 + tile * (int64_t)kTileBytes, (uint32_t)kTileBytes, &s.hin);
+        ++h_issued;
+        if (!tc::mbar_wait(&s.dh1, t & 1)) {
+          atomicExch(&s.err, 1);
+          break;
+        }
+        tc::mbar_expect_tx(&s.hin, (uint32_t)kTileBytes);
+        tc::bulk_g2s(s.da2, g.h1 + tile * (int64_t)kTileBytes, (uint32_t)kTileBytes, &s.hin);
+        ++h_issued;
+      }
+    }
   } else {
     if (!tc::mbar_wait(&s.bar_w, 0)) atomicExch(&s.err, 1);
     const bool issuer = (tid == 32);
@@ -177,41 +213,46 @@ __global__ void __launch_bounds__(kBwThreads, 1) bwd_data_kernel(BwdArgs g) {
     int gs = 0;
     const int quad = warp & 3, slice = warp >> 2, row = quad * 32 + lane;
     const uint32_t lane_addr = tmem + ((uint32_t)(quad * 32) << 16);
-    // Loads run ahead of their use: the next tile's dz chunk is fetched while
-    // this tile runs, and each epilogue fetches its first PF activation
-    // chunks (h2, then h1; 32 bytes per 16 columns) before it waits for its
-    // MMAs, then refills the slot it just used, so global latency overlaps
-    // the tensor core instead of stalling the epilogue.
-    constexpr int NJ = H / 4 / 16;              // 16-column chunks per thread
-    constexpr int PF = H == 256 ? 4 : 2;        // chunks in flight (within the 96 registers of 17 warps)
+    constexpr int NJ = H / 4 / 16;  // 16-column chunks per thread
+    // d = bf16(TMEM (1 - h^2)) for this thread's chunks, h read from the
+    // shared buffer at the offsets d is written to (in place when sbuf)
+    auto epi = [&](bool valid, uint8_t* outt, bool in_place) {
+#pragma unroll 2
+      for (int j = 0; j < NJ; ++j) {
+        const int c = slice * (H / 4) + j * 16;
+        float v[16];
+        tc::tmem_ld16(lane_addr + (uint32_t)c, v);
+        const uint32_t o0 = tc::swz_offset<128>(row, c, kBwRows), o1 = tc::swz_offset<128>(row, c + 8, kBwRows);
+        const uint4 hb[2] = {*reinterpret_cast<const uint4*>(s.da2 + o0), *reinterpret_cast<const uint4*>(s.da2 + o1)};
+        uint32_t pk[8];
+        tanh_grad16(v, hb, valid, pk);
+        const uint4 lo = make_uint4(pk[0], pk[1], pk[2], pk[3]), hi = make_uint4(pk[4], pk[5], pk[6], pk[7]);
+        if (in_place) {
+          *reinterpret_cast<uint4*>(s.da2 + o0) = lo;
+          *reinterpret_cast<uint4*>(s.da2 + o1) = hi;
+        }
+        *reinterpret_cast<uint4*>(outt + o0) = lo;
+        *reinterpret_cast<uint4*>(outt + o1) = hi;
+      }
+    };
     const int tile0 = blockIdx.x;
     uint4 dzv = make_uint4(0, 0, 0, 0);
     if (tid < kBwRows * 2 && my_tiles > 0)
       dzv = __ldg(reinterpret_cast<const uint4*>(g.dz + (int64_t)tile0 * (kBwRows * 32)) + tid);
-    auto hload = [&](const uint8_t* ht, int j, uint4 (&dst)[2]) {
-      const int c = slice * (H / 4) + j * 16;
-      dst[0] = __ldg(reinterpret_cast<const uint4*>(ht + tc::swz_offset<128>(row, c, kBwRows)));
-      dst[1] = __ldg(reinterpret_cast<const uint4*>(ht + tc::swz_offset<128>(row, c + 8, kBwRows)));
-    };
     for (int t = 0; t < my_tiles; ++t) {
       // every compute thread takes the same decision (a named barrier with an OR)
       if (tc::bar_any(1, kBwCompute, s.err != 0)) break;
       const int64_t tile = blockIdx.x + (int64_t)t * gridDim.x;
       const int nr = (int)(g.n - tile * kBwRows < kBwRows ? g.n - tile * kBwRows : kBwRows);
       const bool valid = row < nr;
-      const uint8_t* h2t = g.h2 + tile * (int64_t)(kBwRows * H * 2);
-      const uint8_t* h1t = g.h1 + tile * (int64_t)(kBwRows * H * 2);
       if (t + 1 < my_tiles) {
         // the next tile's h1/h2 images asked of L2 a tile ahead (128-byte lines)
-        const int64_t nxt = (tile + gridDim.x) * (int64_t)(kBwRows * H * 2);
-        for (int64_t off = (int64_t)tid * 128; off < (int64_t)kBwRows * H * 2; off += (int64_t)kBwCompute * 128) {
+        const int64_t nxt = (tile + gridDim.x) * (int64_t)kTileBytes;
+        for (int64_t off = (int64_t)tid * 128; off < (int64_t)kTileBytes; off += (int64_t)kBwCompute * 128) {
           tc::prefetch_l2(g.h2 + nxt + off);
           tc::prefetch_l2(g.h1 + nxt + off);
         }
       }
-      uint4 hb[PF][2];
-#pragma unroll
-      for (int j = 0; j < PF; ++j) hload(h2t, j, hb[j]);
       // dz tile (4 KB, already in the SW32 layout), then the next tile's
       if (tid < kBwRows * 2) {
         reinterpret_cast<uint4*>(s.dz)[tid] = dzv;
@@ -231,29 +272,10 @@ __global__ void __launch_bounds__(kBwThreads, 1) bwd_data_kernel(BwdArgs g) {
       }
       if (!tc::mbar_wait(&s.bar_mma, phase)) atomicExch(&s.err, 1);
       phase ^= 1;
+      if (!tc::mbar_wait(&s.hin, 0)) atomicExch(&s.err, 1);  // h2 in the buffer
       tc::fence_after();
-      // da2 = bf16(dh2 (1 - h2^2)): shared-memory A tile and its tile image
-      {
-        uint8_t* outt = g.da2 + tile * (int64_t)(kBwRows * H * 2);
-#pragma unroll
-        for (int j = 0; j < NJ; ++j) {
-          const int c = slice * (H / 4) + j * 16;
-          float v[16];
-          tc::tmem_ld16(lane_addr + (uint32_t)c, v);
-          const uint32_t o0 = tc::swz_offset<128>(row, c, kBwRows), o1 = tc::swz_offset<128>(row, c + 8, kBwRows);
-          uint32_t pk[8];
-          tanh_grad16(v, hb[j % PF], valid, pk);
-          if (j + PF < NJ) hload(h2t, j + PF, hb[j % PF]);
-          const uint4 lo = make_uint4(pk[0], pk[1], pk[2], pk[3]), hi = make_uint4(pk[4], pk[5], pk[6], pk[7]);
-          *reinterpret_cast<uint4*>(s.da2 + o0) = lo;
-          *reinterpret_cast<uint4*>(s.da2 + o1) = hi;
-          *reinterpret_cast<uint4*>(outt + o0) = lo;
-          *reinterpret_cast<uint4*>(outt + o1) = hi;
-        }
-      }
-      // the h1 chunks of the second epilogue, in flight during the dh1 MMAs
-#pragma unroll
-      for (int j = 0; j < PF; ++j) hload(h1t, j, hb[j]);
+      // da2 = bf16(dh2 (1 - h2^2)): in place over h2 (the next A operand) and its tile image
+      epi(valid, g.da2 + tile * (int64_t)kTileBytes, true);
       tc::fence_before();
       tc::fence_async_smem();
       bw_compute_sync();
@@ -274,35 +296,28 @@ __global__ void __launch_bounds__(kBwThreads, 1) bwd_data_kernel(BwdArgs g) {
             ++gs;
           }
         tc::mma_commit(&s.bar_mma);
+        tc::mma_commit(&s.dh1);  // the loader may now bring h1 over da2
       }
       if (!tc::mbar_wait(&s.bar_mma, phase)) atomicExch(&s.err, 1);
       phase ^= 1;
+      if (!tc::mbar_wait(&s.hin, 1)) atomicExch(&s.err, 1);  // h1 in the buffer
       tc::fence_after();
       // da1 = bf16(dh1 (1 - h1^2)) to its tile image
-      {
-        uint8_t* outt = g.da1 + tile * (int64_t)(kBwRows * H * 2);
-#pragma unroll
-        for (int j = 0; j < NJ; ++j) {
-          const int c = slice * (H / 4) + j * 16;
-          float v[16];
-          tc::tmem_ld16(lane_addr + (uint32_t)c, v);
-          const uint32_t o0 = tc::swz_offset<128>(row, c, kBwRows), o1 = tc::swz_offset<128>(row, c + 8, kBwRows);
-          uint32_t pk[8];
-          tanh_grad16(v, hb[j % PF], valid, pk);
-          if (j + PF < NJ) hload(h1t, j + PF, hb[j % PF]);
-          *reinterpret_cast<uint4*>(outt + o0) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
-          *reinterpret_cast<uint4*>(outt + o1) = make_uint4(pk[4], pk[5], pk[6], pk[7]);
-        }
-      }
+      epi(valid, g.da1 + tile * (int64_t)kTileBytes, false);
       tc::fence_before();
-      bw_compute_sync();
+      tc::fence_async_smem();
+      __syncwarp();
+      if (lane == 0) asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(tc::smem_u32(&s.bfree)) : "memory");
     }
   }
   __syncthreads();
-  // on an error, the producer waits (bounded) for its last copy before the
-  // CTA leaves, so that no bulk copy into this CTA's shared memory is in flight
+  // on an error, the producer and the loader wait (bounded) for their last
+  // copies before the CTA leaves, so that no bulk copy into this CTA's shared
+  // memory is in flight (at most one h copy is outstanding at a time)
   if (s.err && warp == kBwCompute / 32 && lane == 0 && last_issued >= 0)
     (void)tc::mbar_wait(&s.full[last_issued & 1], (last_issued >> 1) & 1);
+  if (s.err && warp == kBwCompute / 32 + 1 && lane == 0 && h_issued > 0)
+    (void)tc::mbar_wait(&s.hin, (h_issued - 1) & 1);
   if (tid == 0 && s.err && g.err) atomicExch(g.err, 1);
   __syncthreads();
   if (warp == 0) tc::tmem_dealloc(tmem, H);
@@ -317,9 +332,14 @@ __global__ void __launch_bounds__(kBwThreads, 1) bwd_data_kernel(BwdArgs g) {
 // warp 17 issues the MMAs; hand-overs as in the forward pair kernel:
 //   dzin[s], d2in[s]: the 16 epilogue warps wrote the slot's dz / da2;
 //   mma1[s], mma2[s]: the slot's dh2 / dh1 MMAs are done.
+// Warp 18 brings each slot's h2 image into the slot's da2 buffer (da2
+// overwrites it in place) and, once the slot's dh1 MMAs are done, its h1
+// image:
+//   hin[s]: an h image landed (h2, then h1: two completions per tile);
+//   bfree[s]: the 16 epilogue warps have read the slot's h1.
 // The arithmetic of every tile is bwd_data_kernel's: the same bits.
 // ---------------------------------------------------------------------------
-constexpr int kBwPairThreads = 576;
+constexpr int kBwPairThreads = 608;
 
 template <int H>
 struct BwdPairSmem {
@@ -327,7 +347,7 @@ struct BwdPairSmem {
   alignas(1024) uint8_t ring[2][kBwStage];
   alignas(1024) uint8_t w3t[H * 32];
   alignas(1024) uint8_t dz[2][kBwRows * 32];
-  uint64_t bar_w, full[2], empty[2], mma1[2], mma2[2], dzin[2], d2in[2];
+  uint64_t bar_w, full[2], empty[2], mma1[2], mma2[2], dzin[2], d2in[2], hin[2], bfree[2];
   uint32_t tmem_base;
   int32_t err;
 };
@@ -350,6 +370,8 @@ __global__ void __launch_bounds__(kBwPairThreads, 1) bwd_data_pair_kernel(BwdArg
       tc::mbar_init(&s.mma2[i], 1);
       tc::mbar_init(&s.dzin[i], 16);
       tc::mbar_init(&s.d2in[i], 16);
+      tc::mbar_init(&s.hin[i], 1);
+      tc::mbar_init(&s.bfree[i], 16);
     }
     tc::fence_mbar_init();
   }
@@ -361,8 +383,35 @@ __global__ void __launch_bounds__(kBwPairThreads, 1) bwd_data_pair_kernel(BwdArg
   const int64_t tiles = (g.n + kBwRows - 1) / kBwRows;
   const int my_tiles = (int)((tiles - blockIdx.x + gridDim.x - 1) / gridDim.x);
   const int npairs = (my_tiles + 1) / 2;
+  constexpr int kTileBytes = kBwRows * H * 2;
   int last_issued = -1;
-  if (warp == 16) {
+  int h_issued[2] = {0, 0};  // loader: h copies issued per slot (the hin phases)
+  if (warp == 18) {
+    if (lane == 0) {
+      // the slot's h2 image once its previous tile's h1 has been read, an
+      // arrival without bytes for a slot with no tile
+      auto bring = [&](int sl, int k, const uint8_t* src) {
+        const bool vt = k < my_tiles;
+        tc::mbar_expect_tx(&s.hin[sl], vt ? (uint32_t)kTileBytes : 0u);
+        if (vt)
+          tc::bulk_g2s(s.da2[sl], src + ((int64_t)blockIdx.x + (int64_t)k * gridDim.x) * kTileBytes,
+                       (uint32_t)kTileBytes, &s.hin[sl]);
+        ++h_issued[sl];
+      };
+      bool ok = true;
+      for (int p = 0; p < npairs && ok; ++p) {
+        for (int sl = 0; sl < 2 && ok; ++sl) {
+          ok = p == 0 || tc::mbar_wait(&s.bfree[sl], (p - 1) & 1);
+          if (ok) bring(sl, 2 * p + sl, g.h2);
+        }
+        for (int sl = 0; sl < 2 && ok; ++sl) {
+          ok = tc::mbar_wait(&s.mma2[sl], p & 1);
+          if (ok) bring(sl, 2 * p + sl, g.h1);
+        }
+      }
+      if (!ok) atomicExch(&s.err, 1);
+    }
+  } else if (warp == 16) {
     if (lane == 0) {
       int gs = 0;
       for (int p = 0; p < npairs; ++p)
@@ -417,42 +466,38 @@ __global__ void __launch_bounds__(kBwPairThreads, 1) bwd_data_pair_kernel(BwdArg
     const int quad = warp & 3, slice = warp >> 2, row = quad * 32 + lane;
     const uint32_t lane_base = tmem + ((uint32_t)(quad * 32) << 16);
     auto tile_of = [&](int k) { return (int64_t)blockIdx.x + (int64_t)k * gridDim.x; };
-    auto hload = [&](const uint8_t* ht, int j, uint4 (&dst)[2]) {
-      const int c = slice * (H / 4) + j * 16;
-      dst[0] = __ldg(reinterpret_cast<const uint4*>(ht + tc::swz_offset<128>(row, c, kBwRows)));
-      dst[1] = __ldg(reinterpret_cast<const uint4*>(ht + tc::swz_offset<128>(row, c + 8, kBwRows)));
-    };
     auto handover = [&](uint64_t* bar) {
       tc::fence_async_smem();
       tc::fence_before();
       __syncwarp();
       if (lane == 0) asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(tc::smem_u32(bar)) : "memory");
     };
-    // one epilogue: d = bf16(TMEM (1 - h^2)) of slot sl into the tile image (and the da2 buffer)
-    auto epi = [&](int sl, int k, const uint8_t* hsrc, uint8_t* gout, uint8_t* sbuf, uint64_t* mbar, uint32_t par) {
+    // one epilogue: d = bf16(TMEM (1 - h^2)) of slot sl, h read from the
+    // slot's buffer where the loader put it; d to the tile image and, for
+    // da2, in place over h2 (the next A operand)
+    auto epi = [&](int sl, int k, uint8_t* gout, bool in_place, uint64_t* mbar, uint32_t par, uint32_t hpar) {
       const bool vt = k < my_tiles;
       const int64_t tl = tile_of(k);
       const int nr = vt ? (int)(g.n - tl * kBwRows < kBwRows ? g.n - tl * kBwRows : kBwRows) : 0;
       const bool valid = row < nr;
-      const uint8_t* ht = hsrc + (vt ? tl : 0) * (int64_t)(kBwRows * H * 2);
-      uint4 hb[NJ][2];
-#pragma unroll
-      for (int j = 0; j < NJ; ++j) hload(ht, j, hb[j]);
+      if (!tc::mbar_wait(&s.hin[sl], hpar)) atomicExch(&s.err, 1);
       if (!tc::mbar_wait(mbar, par)) atomicExch(&s.err, 1);
       tc::fence_after();
-      uint8_t* outt = vt ? gout + tl * (int64_t)(kBwRows * H * 2) : nullptr;
+      uint8_t* outt = vt ? gout + tl * (int64_t)kTileBytes : nullptr;
+      uint8_t* buf = s.da2[sl];
 #pragma unroll
       for (int j = 0; j < NJ; ++j) {
         const int c = slice * (H / 4) + j * 16;
         float v[16];
         tc::tmem_ld16(lane_base + (uint32_t)(sl * 256 + c), v);
         const uint32_t o0 = tc::swz_offset<128>(row, c, kBwRows), o1 = tc::swz_offset<128>(row, c + 8, kBwRows);
+        const uint4 hb[2] = {*reinterpret_cast<const uint4*>(buf + o0), *reinterpret_cast<const uint4*>(buf + o1)};
         uint32_t pk[8];
-        tanh_grad16(v, hb[j], valid, pk);
+        tanh_grad16(v, hb, valid, pk);
         const uint4 lo = make_uint4(pk[0], pk[1], pk[2], pk[3]), hi = make_uint4(pk[4], pk[5], pk[6], pk[7]);
-        if (sbuf) {
-          *reinterpret_cast<uint4*>(sbuf + o0) = lo;
-          *reinterpret_cast<uint4*>(sbuf + o1) = hi;
+        if (in_place) {
+          *reinterpret_cast<uint4*>(buf + o0) = lo;
+          *reinterpret_cast<uint4*>(buf + o1) = hi;
         }
         if (outt) {
           *reinterpret_cast<uint4*>(outt + o0) = lo;
@@ -468,7 +513,7 @@ __global__ void __launch_bounds__(kBwPairThreads, 1) bwd_data_pair_kernel(BwdArg
     };
     // The h1/h2 tile images of a pair's two tiles (4 x 64 KB) are asked of L2
     // one pair ahead, one 128-byte line per thread per image, so that the
-    // epilogues' loads hit L2 instead of waiting for HBM.
+    // loader's bulk copies read L2 instead of waiting for HBM.
     auto prefetch_pair = [&](int p) {
 #pragma unroll
       for (int sl = 0; sl < 2; ++sl) {
@@ -494,12 +539,12 @@ __global__ void __launch_bounds__(kBwPairThreads, 1) bwd_data_pair_kernel(BwdArg
       fetch_dz(2 * p + 2, dzv[0]);
       fetch_dz(2 * p + 3, dzv[1]);
       for (int sl = 0; sl < 2; ++sl) {
-        epi(sl, 2 * p + sl, g.h2, g.da2, s.da2[sl], &s.mma1[sl], par);
+        epi(sl, 2 * p + sl, g.da2, true, &s.mma1[sl], par, 0);
         handover(&s.d2in[sl]);
       }
       for (int sl = 0; sl < 2; ++sl) {
-        epi(sl, 2 * p + sl, g.h1, g.da1, nullptr, &s.mma2[sl], par);
-        tc::fence_before();
+        epi(sl, 2 * p + sl, g.da1, false, &s.mma2[sl], par, 1);
+        handover(&s.bfree[sl]);
       }
     }
   }
@@ -507,6 +552,9 @@ __global__ void __launch_bounds__(kBwPairThreads, 1) bwd_data_pair_kernel(BwdArg
   __syncthreads();
   if (s.err && warp == 16 && lane == 0 && last_issued >= 0)
     (void)tc::mbar_wait(&s.full[last_issued & 1], (last_issued >> 1) & 1);
+  if (s.err && warp == 18 && lane == 0)
+    for (int sl = 0; sl < 2; ++sl)
+      if (h_issued[sl] > 0) (void)tc::mbar_wait(&s.hin[sl], (h_issued[sl] - 1) & 1);
   if (tid == 0 && s.err && g.err) atomicExch(g.err, 1);
   __syncthreads();
   if (warp == 0) tc::tmem_dealloc(tmem, 512);
@@ -694,21 +742,22 @@ __global__ void __launch_bounds__(kWgThreads, 1) wgrad_kernel(WgArgs g) {
 //     of its partial blocks, in chunk order;
 //   - blocks 0 .. 5 + A also sum the loss partial rows, one quantity per
 //     block (the five minibatch statistics, then the head-bias gradients
-//     from the unrounded dz): thread t takes rows t, t + 256, ... in order,
+//     from the unrounded dz): thread t takes rows t, t + 512, ... in order,
 //     then a fixed shuffle tree and the warps in order;
 //   - each block writes the fp32 sum of squares of the entries it wrote
 //     (threads in order of a fixed tree), the Adam kernel sums the blocks.
 constexpr int kWgReduceBlocks = 256;
+constexpr int kWgReduceThreads = 512;  // 27 warps per SM, eight chunk loads in flight per thread
 constexpr int kLossPartW = 32;  // loss-kernel partial row: pg, ent, kl, clip, vl, db3[16], dc3
 
 template <int D, int H>
-__global__ void __launch_bounds__(256) wgrad_reduce_kernel(const float* __restrict__ part, int S, int A,
+__global__ void __launch_bounds__(kWgReduceThreads) wgrad_reduce_kernel(const float* __restrict__ part, int S, int A,
                                                            float* __restrict__ grad, const float* __restrict__ lossp,
                                                            int nlb, double* __restrict__ stat5,
                                                            float* __restrict__ sq) {
   using Cn = WgCols<D>;
   constexpr int NCH = H / 256, MB = H / 128;
-  __shared__ float red[8];
+  __shared__ float red[kWgReduceThreads / 32];
   const MlpLayout Lp = mlp_layout(D, H, A);
   const int64_t total = (int64_t)2 * MB * NCH * 128 * kWgMaxCols;
   float q = 0.0f;
@@ -731,12 +780,13 @@ __global__ void __launch_bounds__(256) wgrad_reduce_kernel(const float* __restri
     if (dst < 0) continue;
     const float* p = part + ((int64_t)grp * S * 128 + row) * kWgMaxCols + col;
     float acc = 0.0f;
+#pragma unroll 8
     for (int k = 0; k < S; ++k) acc += p[(int64_t)k * 128 * kWgMaxCols];
     grad[dst] = acc;
     q = fmaf(acc, acc, q);
   }
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  __shared__ double redd[8];
+  __shared__ double redd[kWgReduceThreads / 32];
   const int w = (int)blockIdx.x;  // statistic w (w < 5), then head-bias sum j = w - 5 (policy j < A, then the value's)
   if (w < 5 + A + 1) {
     const int col = w < 5 ? w : (w - 5 < A ? 5 + (w - 5) : 21);
@@ -834,7 +884,7 @@ static pe_status bwd_launch(const float* params, int A, uint8_t* const img[2], c
     ProfScope ps(PE_PROF_PPO_GRAD, st);
     kern<<<groups * a.S, kWgThreads, bytes, st>>>(a);
     PE_CHECK_LAUNCH("wgrad_kernel");
-    wgrad_reduce_kernel<D, H><<<kWgReduceBlocks, 256, 0, st>>>(part, a.S, A, grad, lossp, nlb, stat5, sq);
+    wgrad_reduce_kernel<D, H><<<kWgReduceBlocks, kWgReduceThreads, 0, st>>>(part, a.S, A, grad, lossp, nlb, stat5, sq);
     PE_CHECK_LAUNCH("wgrad_reduce_kernel");
   }
   return PE_OK;
