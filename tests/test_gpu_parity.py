@@ -433,12 +433,19 @@ def test_rollout_parity_72b_small():
     _rollout_case(W.make_72b(n_envs=512), 600, iters=1, lam=0.7)
 
 
+def test_rollout_parity_72b_two_chains_ragged():
+    """700 envs run as two stream chains split on a tile boundary (384 +
+    316 envs, the second ending in a ragged tile); every env is replayed,
+    including both sides of the split."""
+    _rollout_case(W.make_72b(n_envs=700), 40, iters=2, lam=0.7)
+
+
 def test_rollout_parity_72b_full_size_sampled():
     """The full 72B workload (65,536 envs x 1,024 steps); the oracle replays
     a seeded sample of envs including both ends and a tile boundary."""
     wl = W.make_72b()
     rng = np.random.default_rng(5)
-    ids = np.unique(np.concatenate([[0, 127, 128, 65535], rng.choice(65536, 12, replace=False)]))
+    ids = np.unique(np.concatenate([[0, 127, 128, 32767, 32768, 65535], rng.choice(65536, 12, replace=False)]))
     _rollout_case(wl, 1024, iters=1, sample_envs=ids)
 
 
