@@ -60,7 +60,8 @@ def parse():
     ap.add_argument("--r72b-horizon", type=int, default=1024)
     ap.add_argument("--r72b-ppo-minibatches", type=int, default=16,
                     help="72B PPO minibatch steps of 65,536 samples timed (0: skip)")
-    ap.add_argument("--ncu-case", choices=["ppo7b", "ppo72", "ppostress", "gae", "mlp72", "fleet"], default=None,
+    ap.add_argument("--ncu-case", choices=["ppo7b", "ppo72", "ppostress", "gae", "gae-chunked", "mlp72", "fleet"],
+                    default=None,
                     help="run one small named case of a hot kernel (for ncu captures) and exit")
     ap.add_argument("--gae-large", type=int, nargs=2, default=[2048, 262144], metavar=("T", "E"),
                     help="GAE roofline size (Stress: 2048 x 262144); T=0 skips it")
@@ -331,7 +332,7 @@ def run_ours(args, world, rank, local):
         os.path.join(ROOT, "MEASURED_PEAKS.json")) else {"hbm_gbs": 6800.0}
     hbm = float(peaks.get("hbm_gbs", 6800.0))
     # inputs just written by the rollout sit in L2 at this size: no DRAM traffic figure
-    gae_roof = {"kernel": "gae_kernel", "bound": "hbm", "achieved": gae_gbs, "peak": hbm,
+    gae_roof = {"kernel": gae_kernel_name(tr.E), "bound": "hbm", "achieved": gae_gbs, "peak": hbm,
                 "unit": "GB/s", "frac": gae_gbs / hbm if gae_gbs else None,
                 "traffic": None}
 
@@ -651,7 +652,7 @@ def run_72b(args, world, peaks):
     pe.device_check()
     prof = {pe.profile_kind_name(k): pe.profile_read(k) for k in range(pe.PE_PROF_KINDS)}
     D, H, A = net.obs_dim, net.hidden, net.n_actions
-    pol_flop = 2.0 * E * (D * H + H * H + H * A)          # one policy launch (E rows)
+    pol_flop_all = 2.0 * T * E * (D * H + H * H + H * A)  # every policy launch of one rollout
     val_flop = 2.0 * (T + 1) * E * (D * H + H * H + H)   # the value launches of one rollout
     # GAE over the 72B rollout buffer (T*E = 67M env-steps, 1.14 GB of algorithmic traffic)
     adv = torch.empty(T, E, device="cuda")
@@ -682,7 +683,10 @@ def run_72b(args, world, peaks):
     pms, pn = prof["mlp_policy_tc"]
     vms, vn = prof["mlp_value_tc"]
     peak = float(peaks.get("bf16_tflops_sustained", 1728.9))
-    pol = pol_flop / (pms / pn / 1e3) / 1e12 if pn else None
+    # the policy runs as two chains of E/2-row launches on two streams: the
+    # sum of the launches' event times counts time shared with the other
+    # chain's env steps, so this figure is a lower bound
+    pol = pol_flop_all / (pms / 1e3) / 1e12 if pn else None
     val = val_flop / (vms / 1e3) / 1e12 if vn else None
     env.close()
     return {"metric": "72B rollout env-steps/s", "value": E * T * world / (ms / 1e3),
@@ -691,17 +695,19 @@ def run_72b(args, world, peaks):
                                    "16 levels, MLP 32-256-256 bf16 (tcgen05), value on all T*E obs",
                        "n_envs": E, "horizon": T},
             "kernels": {k: {"ms_per_rollout": v[0], "launches_per_rollout": v[1]} for k, v in prof.items() if v[1]},
-            "roofline_policy_mlp": {"kernel": f"mlp_bf16_kernel (policy, {E} rows)", "bound": "tensor",
+            "roofline_policy_mlp": {"kernel": f"mlp_bf16_pair_kernel (policy, {pn // max(T, 1)} launches per "
+                                              f"step over {E} rows)", "bound": "tensor",
                                     "achieved": pol, "peak": peak, "unit": "TFLOP/s",
                                     "frac": pol / peak if pol else None,
-                                    "traffic": load_traffic("mlp_bf16_kernel")},
-            "roofline_value_mlp": {"kernel": "mlp_bf16_kernel (value, T*E rows)", "bound": "tensor",
+                                    "avg_launch_ms": pms / pn if pn else None,
+                                    "traffic": load_traffic("mlp_bf16_pair_kernel")},
+            "roofline_value_mlp": {"kernel": "mlp_bf16_pair_kernel (value, T*E rows)", "bound": "tensor",
                                    "achieved": val, "peak": peak, "unit": "TFLOP/s",
                                    "frac": val / peak if val else None},
-            "roofline_gae": {"kernel": f"gae_kernel ({T} x {E})", "bound": "hbm", "achieved": gae_gbs,
+            "roofline_gae": {"kernel": f"{gae_kernel_name(E)} ({T} x {E})", "bound": "hbm", "achieved": gae_gbs,
                              "peak": hbm, "unit": "GB/s", "frac": gae_gbs / hbm if gae_gbs else None,
                              "avg_launch_ms": gms / gn if gn else None,
-                             "traffic": gae_traffic(T * E)},
+                             "traffic": gae_traffic(T * E, E)},
             "ppo_update": ppo72, "dual_ascent_eq7": dual,
             "cadence": run_72b_cadence(args, world),
             "mixed_families": run_72b_mixed(args, world)}
@@ -996,10 +1002,23 @@ def per_config_table(out):
     return {k: {"gpu": gpu[k][0], "gpu_metric": gpu[k][2], "roofline_frac": gpu[k][1], **cpu[k]} for k in cpu}
 
 
-def gae_traffic(env_steps: int):
+def gae_kernel_name(E: int) -> str:
+    """The GAE kernel the library picks for a batch of E envs (its dispatch
+    by width): streamed per env column for wide batches, chunked below."""
+    if E >= 196608 and E % 4 == 0:
+        return "gae_stream_kernel<4, 8>"
+    if E >= 49152:
+        return "gae_stream_kernel<1, 16>"
+    if E >= 32768:
+        return "gae_stream_kernel<1, 32>"
+    return "gae_kernel_v (chunked)"
+
+
+def gae_traffic(env_steps: int, E: int):
     """DRAM bytes of one GAE launch larger than L2, scaled from the committed
-    capture's bytes per env-step."""
-    b = load_traffic_per_unit("gae_kernel", "traffic_bytes_per_env_step")
+    capture's bytes per env-step of the same kernel."""
+    key = "traffic_bytes_per_env_step_v4" if E >= 196608 and E % 4 == 0 else "traffic_bytes_per_env_step_v1"
+    b = load_traffic_per_unit("gae_stream_kernel", key) if E >= 32768 else None
     return None if b is None else b * env_steps
 
 
@@ -1030,9 +1049,9 @@ def run_gae_large(args, world, peaks):
     hbm = float(peaks.get("hbm_gbs", 6800.0))
     del r, v, d, adv, ret
     torch.cuda.empty_cache()
-    return {"kernel": f"gae_kernel ({T} x {E})", "bound": "hbm", "achieved": gbs, "peak": hbm,
+    return {"kernel": f"{gae_kernel_name(E)} ({T} x {E})", "bound": "hbm", "achieved": gbs, "peak": hbm,
             "unit": "GB/s", "frac": gbs / hbm, "avg_launch_ms": ms,
-            "env_steps_per_s": T * E * world / (ms / 1e3), "traffic": gae_traffic(T * E)}
+            "env_steps_per_s": T * E * world / (ms / 1e3), "traffic": gae_traffic(T * E, E)}
 
 
 # --------------------------------------------------------------------------- CPU oracle
@@ -1133,8 +1152,10 @@ def run_ncu_case(name: str):
             pe.ppo_update(net, ppo, params, m, v, it * steps, buf["obs"], buf["act"], buf["logp"], adv, ret,
                           st, ws, seed=7, iteration=it)
         env.close()
-    elif name == "gae":
-        T, E = 2048, 16384  # 570 MB of algorithmic traffic per launch
+    elif name == "gae-chunked":
+        # the chunked kernel of narrower batches: 2,048 x 16,384 (570 MB of
+        # algorithmic traffic, more than L2)
+        T, E = 2048, 16384
         g = torch.Generator(device="cuda").manual_seed(0)
         r = torch.randn(T, E, device="cuda", generator=g)
         v = torch.randn(T, E, device="cuda", generator=g)
@@ -1144,6 +1165,21 @@ def run_ncu_case(name: str):
         ret = torch.empty_like(adv)
         for _ in range(3):
             pe.gae(r, v, d, lv, 0.99, 0.95, adv, ret)
+    elif name == "gae":
+        # the two streamed launch shapes: 1,024 x 65,536 (one env per thread,
+        # the 72B rollout's shape, 1.1 GB of algorithmic traffic) and
+        # 512 x 262,144 (four envs per thread, the Stress width, 2.3 GB)
+        for T, E in ((1024, 65536), (512, 262144)):
+            g = torch.Generator(device="cuda").manual_seed(0)
+            r = torch.randn(T, E, device="cuda", generator=g)
+            v = torch.randn(T, E, device="cuda", generator=g)
+            d = (torch.rand(T, E, device="cuda", generator=g) < 0.002).to(torch.uint8)
+            lv = torch.randn(E, device="cuda", generator=g)
+            adv = torch.empty(T, E, device="cuda")
+            ret = torch.empty_like(adv)
+            for _ in range(3):
+                pe.gae(r, v, d, lv, 0.99, 0.95, adv, ret)
+            del r, v, d, lv, adv, ret
     elif name == "mlp72":
         # two 72B rollouts of 8 steps over 65,536 envs: 8 policy + 2 value launches each
         wl = W.make_72b(n_envs=65536)
