@@ -367,7 +367,7 @@ def run_ours(args, world, rank, local):
     # ---- fleet accounting
     fleet = run_fleet(args, world, tr, roofs) if args.fleet_n > 0 else None
     evaluation = run_evaluation(args, world, tr, peaks) if args.eval else None
-    r72b = run_72b(args, world, peaks) if args.r72b_steps > 0 else None
+    r72b = run_72b(args, world, peaks, local) if args.r72b_steps > 0 else None
     gae_large = run_gae_large(args, world, peaks) if args.gae_large[0] > 0 else None
     tiny = run_tiny(args, world)
     torch.cuda.empty_cache()
@@ -613,7 +613,68 @@ def run_stagger(args, world, fw, traces, job, peaks_random, tr=None):
                                       "staggered_with_job_control": ctl / name if ctl else None}}
 
 
-def run_72b(args, world, peaks):
+def run_72b_iteration(args, world, peaks, local, wl, env, params, buf, rws):
+    """One whole 72B PPO iteration, timed with CUDA events and clock records:
+    the rollout (65,536 envs x 1,024 steps), GAE and the full update (4 epochs
+    x 1,024 minibatch steps of 65,536 samples), as the Stress leg times its
+    iteration."""
+    from paper_2608_11226_gb300 import pe
+    net, ppo = wl.net, wl.ppo
+    T, E = args.r72b_horizon, wl.env.n_envs
+    N = T * E
+    adv = torch.empty(T, E, device="cuda")
+    ret = torch.empty_like(adv)
+    m = torch.zeros_like(params)
+    v = torch.zeros_like(params)
+    stats = torch.zeros(8, device="cuda")
+    pws = pe.alloc_workspace(pe.ppo_workspace_bytes(net, ppo, N))
+    # warm-up of the update at this size: two minibatch steps
+    pe.gae(buf["reward"], buf["value"], buf["done"], buf["last_value"], 0.99, 0.95, adv, ret)
+    nw = 2 * ppo.minibatch
+    wppo = type(ppo)(epochs=1, minibatch=ppo.minibatch, ent_coef=ppo.ent_coef)
+    pe.ppo_update(net, wppo, params.clone(), m.clone(), v.clone(), 0, buf["obs"].view(-1, net.obs_dim)[:nw],
+                  buf["act"].view(-1)[:nw], buf["logp"].view(-1)[:nw], adv.view(-1)[:nw], ret.view(-1)[:nw],
+                  stats, pws, seed=7, iteration=0)
+    torch.cuda.synchronize()
+    barrier(world)
+    clocks = ClockSampler(local)
+    clocks.start()
+    stream = torch.cuda.current_stream()
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
+    ev[0].record(stream)
+    pe.rollout(env, net, params, T, 50, buf, lam=1.0, workspace=rws)
+    ev[1].record(stream)
+    pe.gae(buf["reward"], buf["value"], buf["done"], buf["last_value"], 0.99, 0.95, adv, ret)
+    ev[2].record(stream)
+    pe.ppo_update(net, ppo, params, m, v, 0, buf["obs"], buf["act"], buf["logp"], adv, ret, stats, pws,
+                  seed=7, iteration=1)
+    ev[3].record(stream)
+    torch.cuda.synchronize()
+    clk = clocks.stop()
+    pe.device_check()
+    ph = [ev[i].elapsed_time(ev[i + 1]) for i in range(3)]
+    total = max_over_ranks(sum(ph), world)
+    steps = ppo.epochs * ((N + ppo.minibatch - 1) // ppo.minibatch)
+    D, H, A = net.obs_dim, net.hidden, net.n_actions
+    ppo_flop = ppo_flops_per_sample(D, H, A) * N * ppo.epochs
+    peak = float(peaks.get("bf16_tflops_sustained", 1725.0))
+    ppo_tf = ppo_flop / (ph[2] / 1e3) / 1e12
+    del pws, adv, ret
+    torch.cuda.empty_cache()
+    return {"metric": "72B PPO iteration env-steps/s", "value": N * world / (total / 1e3), "unit": "env-steps/s",
+            "ms_per_iteration": total,
+            "phases_ms": {"rollout": ph[0], "gae": ph[1], "ppo_update": ph[2]},
+            "ppo_ms_per_minibatch_step": ph[2] / steps, "ppo_minibatch_steps": steps,
+            "config": {"workload": f"72b: {E} envs x {T} steps, MLP 32-256-256 bf16 (tcgen05), GAE, "
+                                   f"PPO {ppo.epochs} epochs x minibatch {ppo.minibatch} ({steps} minibatch steps)",
+                       "timed": "one iteration after the rollout and update legs; inputs larger than L2"},
+            "roofline": {"kernel": "bf16 PPO update (all its kernels)", "bound": "tensor", "achieved": ppo_tf,
+                         "peak": peak, "unit": "TFLOP/s", "frac": ppo_tf / peak, "flop": ppo_flop,
+                         "peak_source": "MEASURED_PEAKS.json bf16_tflops_sustained"},
+            "clocks": clk}
+
+
+def run_72b(args, world, peaks, local=0):
     """The 72B workload's rollout (65,536 envs x 1,024 steps, bf16 32-256-256
     policy/value MLPs on the tcgen05 tensor cores, 4 channels, Eq. 6 reward),
     timed the same way; reports env-steps/s and the tensor-core MLP kernel's
@@ -688,6 +749,7 @@ def run_72b(args, world, peaks):
     # chain's env steps, so this figure is a lower bound
     pol = pol_flop_all / (pms / 1e3) / 1e12 if pn else None
     val = val_flop / (vms / 1e3) / 1e12 if vn else None
+    it72 = run_72b_iteration(args, world, peaks, local, wl, env, params, buf, ws)
     env.close()
     return {"metric": "72B rollout env-steps/s", "value": E * T * world / (ms / 1e3),
             "unit": "env-steps/s", "ms_per_rollout": ms,
@@ -709,6 +771,7 @@ def run_72b(args, world, peaks):
                              "avg_launch_ms": gms / gn if gn else None,
                              "traffic": gae_traffic(T * E, E)},
             "ppo_update": ppo72, "dual_ascent_eq7": dual,
+            "iteration": it72,
             "cadence": run_72b_cadence(args, world),
             "mixed_families": run_72b_mixed(args, world)}
 
@@ -990,8 +1053,9 @@ def per_config_table(out):
     gpu = {
         "tiny": ((out.get("tiny_iteration") or {}).get("value"), None, "PPO iteration env-steps/s"),
         "7b": (out["value"], (out.get("roofline") or {}).get("frac"), "PPO iteration env-steps/s"),
-        "72b": (r72.get("value"), (r72.get("roofline_policy_mlp") or {}).get("frac"),
-                "rollout env-steps/s (policy MLP tensor fraction)"),
+        "72b": ((r72.get("iteration") or {}).get("value"),
+                ((r72.get("iteration") or {}).get("roofline") or {}).get("frac"),
+                "PPO iteration env-steps/s (update tensor fraction)"),
         "stress": ((out.get("stress_iteration") or {}).get("value"),
                    ((out.get("stress_iteration") or {}).get("roofline") or {}).get("frac"),
                    "PPO iteration env-steps/s (update tensor fraction)"),
