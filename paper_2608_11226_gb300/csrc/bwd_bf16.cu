@@ -34,26 +34,14 @@
 //   canonical gradient vector.
 #include <algorithm>
 
+#include "bf16_layout.cuh"
 #include "mlp_f32.cuh"
 #include "tc.cuh"
 
 namespace pe {
 
-constexpr int kBwRows = 128;            // samples per tile (MMA M of the data products)
-constexpr int kBwStage = 32768;         // one streamed W2^T stage: 256 rows x 64 K, SW128
 constexpr int kBwCompute = 512;         // 16 compute warps
 constexpr int kBwThreads = kBwCompute + 64;  // + the W2^T producer warp and the h loader warp
-
-// backward weight image of one network: W3^T (H rows x 16, K-major SW32),
-// then the W2^T stages: stage (h, kb) = rows i in [256 h, 256 h + 256) of
-// W2^T, K = o in [64 kb, 64 kb + 64), K-major SW128
-template <int H>
-struct BwdImg {
-  static constexpr int W3T = H * 32;
-  static constexpr int NH = H / 256, KB = H / 64, STAGES = NH * KB;
-  static constexpr int TOTAL = W3T + STAGES * kBwStage;
-  static_assert(W3T % 1024 == 0, "stages start on a swizzle atom");
-};
 
 int64_t bwd_image_bytes(int H) {
   if (H == 256) return BwdImg<256>::TOTAL;
@@ -104,18 +92,6 @@ struct BwdSmem {
 };
 
 __device__ __forceinline__ void bw_compute_sync() { asm volatile("bar.sync 1, 512;" ::: "memory"); }
-
-// d = bf16(g (1 - h^2)) for 16 columns: g from TMEM, h as 16 packed bf16
-__device__ __forceinline__ void tanh_grad16(const float (&g)[16], const uint4 (&h)[2], bool valid,
-                                            uint32_t (&pk)[8]) {
-  const uint4 a = h[0], b = h[1];
-  const uint32_t hw[8] = {a.x, a.y, a.z, a.w, b.x, b.y, b.z, b.w};
-#pragma unroll
-  for (int i = 0; i < 8; ++i) {
-    const float h0 = __uint_as_float(hw[i] << 16), h1 = __uint_as_float(hw[i] & 0xFFFF0000u);
-    pk[i] = valid ? tc::pack_bf16(g[2 * i] * (1.0f - h0 * h0), g[2 * i + 1] * (1.0f - h1 * h1)) : 0u;
-  }
-}
 
 struct BwdArgs {
   const uint8_t* img;   // backward weight image of the network
@@ -831,20 +807,30 @@ constexpr int kWgMaxCtas = 256;
 int64_t wgrad_partial_bytes() { return (int64_t)kWgMaxCtas * 128 * kWgMaxCols * 4; }
 
 template <int D, int H>
-static pe_status bwd_launch(const float* params, int A, uint8_t* const img[2], const uint8_t* x,
-                            const uint8_t* const dz[2], const uint8_t* const h1[2], const uint8_t* const h2[2],
-                            uint8_t* const da2[2], uint8_t* const da1[2], int64_t n, float* part, float* grad,
-                            const float* lossp, int nlb, double* stat5, float* sq, int32_t* err, cudaStream_t st) {
-  int dev = 0, sms = 0;
-  PE_TRY_CUDA(cudaGetDevice(&dev));
-  PE_TRY_CUDA(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
+static pe_status bwd_images(const float* params, int A, uint8_t* const img[2], cudaStream_t st) {
   {
     ProfScope ps(PE_PROF_PPO_OTHER, st);
     bwd_image_kernel<D, H><<<dim3(128, 2), 256, 0, st>>>(params, A, img[0], img[1]);
   }
   PE_CHECK_LAUNCH("bwd_image_kernel");
+  return PE_OK;
+}
+
+template <int D, int H>
+static pe_status bwd_launch(const float* params, int A, uint8_t* const img[2], const uint8_t* x,
+                            const uint8_t* const dz[2], const uint8_t* const h1[2], const uint8_t* const h2[2],
+                            uint8_t* const da2[2], uint8_t* const da1[2], int64_t n, float* part, float* grad,
+                            const float* lossp, int nlb, double* stat5, float* sq, int32_t* err, bool data_done,
+                            cudaStream_t st) {
+  int dev = 0, sms = 0;
+  PE_TRY_CUDA(cudaGetDevice(&dev));
+  PE_TRY_CUDA(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
   const int64_t tiles = (n + kBwRows - 1) / kBwRows;
-  if constexpr (H == 256) {
+  if (data_done) {
+    // the backward images and the data products came with the fused forward-backward kernel
+  } else if constexpr (H == 256) {
+    pe_status s = bwd_images<D, H>(params, A, img, st);
+    if (s != PE_OK) return s;
     auto kern = bwd_data_pair_kernel<H>;
     const int bytes = (int)sizeof(BwdPairSmem<H>) + 1024;
     PE_TRY_CUDA(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes));
@@ -855,6 +841,8 @@ static pe_status bwd_launch(const float* params, int A, uint8_t* const img[2], c
       kern<<<grid, kBwPairThreads, bytes, st>>>(a);
     }
   } else {
+    pe_status s = bwd_images<D, H>(params, A, img, st);
+    if (s != PE_OK) return s;
     auto kern = bwd_data_kernel<H>;
     const int bytes = (int)sizeof(BwdSmem<H>) + 1024;
     PE_TRY_CUDA(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes));
@@ -897,15 +885,22 @@ static pe_status bwd_launch(const float* params, int A, uint8_t* const img[2], c
 pe_status bf16_backward(const pe_net& net, const float* params, uint8_t* const img[2], const uint8_t* x,
                         const uint8_t* const dz[2], const uint8_t* const h1[2], const uint8_t* const h2[2],
                         uint8_t* const da2[2], uint8_t* const da1[2], int64_t n, float* part, float* grad,
-                        const float* lossp, int nlb, double* stat5, float* sq, int32_t* err, cudaStream_t st) {
+                        const float* lossp, int nlb, double* stat5, float* sq, int32_t* err, bool data_done,
+                        cudaStream_t st) {
   if (n <= 0) return PE_OK;
   if (net.obs_dim == 32 && net.hidden == 256)
     return bwd_launch<32, 256>(params, net.n_actions, img, x, dz, h1, h2, da2, da1, n, part, grad, lossp, nlb, stat5,
-                               sq, err, st);
+                               sq, err, data_done, st);
   if (net.obs_dim == 64 && net.hidden == 512)
     return bwd_launch<64, 512>(params, net.n_actions, img, x, dz, h1, h2, da2, da1, n, part, grad, lossp, nlb, stat5,
-                               sq, err, st);
+                               sq, err, data_done, st);
   return fail(PE_EINVAL, "unsupported bf16 network for the backward pass");
+}
+
+pe_status bf16_bwd_images(const pe_net& net, const float* params, uint8_t* const img[2], cudaStream_t st) {
+  if (net.obs_dim == 32 && net.hidden == 256) return bwd_images<32, 256>(params, net.n_actions, img, st);
+  if (net.obs_dim == 64 && net.hidden == 512) return bwd_images<64, 512>(params, net.n_actions, img, st);
+  return fail(PE_EINVAL, "unsupported bf16 network for the backward images");
 }
 
 }  // namespace pe

@@ -15,6 +15,8 @@
 //                products and tanh derivatives (da2, da1), then the weight
 //                and hidden-bias gradients split over samples with a
 //                fixed-order reduction into the canonical gradient vector;
+//                for the 72B networks the forward, the loss and the data
+//                products of a network run as one kernel (fused_bf16.cu);
 //   step      -- the gradient's squared norm (summed with the weight
 //                gradients' reduction), clip, Adam on the fp32 master
 //                parameters.
@@ -43,7 +45,15 @@ int64_t wgrad_partial_bytes();
 pe_status bf16_backward(const pe_net& net, const float* params, uint8_t* const img[2], const uint8_t* x,
                         const uint8_t* const dz[2], const uint8_t* const h1[2], const uint8_t* const h2[2],
                         uint8_t* const da2[2], uint8_t* const da1[2], int64_t n, float* part, float* grad,
-                        const float* lossp, int nlb, double* stat5, float* sq, int32_t* err, cudaStream_t st);
+                        const float* lossp, int nlb, double* stat5, float* sq, int32_t* err, bool data_done,
+                        cudaStream_t st);
+pe_status bf16_bwd_images(const pe_net& net, const float* params, uint8_t* const img[2], cudaStream_t st);
+// defined in fused_bf16.cu
+bool bf16_fused_supported(const pe_net& net);
+pe_status bf16_fused_fwd_bwd(const pe_net& net, const uint8_t* img, const uint8_t* bimg, const float* params,
+                             int value_net, const void* obs, const uint32_t* gather, int64_t n, const PpoHead& loss,
+                             __nv_bfloat16* x, __nv_bfloat16* h1, __nv_bfloat16* h2, uint8_t* da2, uint8_t* da1,
+                             int32_t* err, cudaStream_t st);
 int wgrad_reduce_blocks();
 
 constexpr int kHead = 16;   // head rows (logits; the value head padded with zero rows)
@@ -205,6 +215,7 @@ pe_status ppo_update_bf16(const pe_net& net, float* params, float* m, float* v, 
   pe_status s = launch_advstats(adv, N, cfg.minibatch, pl.nmb, cfg.epochs, cfg.seed, cfg.iteration, advstat, st);
   if (s != PE_OK) return s;
   int64_t t = adam_t;
+  const bool fused = bf16_fused_supported(net);
   for (int ep = 0; ep < cfg.epochs; ++ep) {
     const Feistel f = make_feistel((uint64_t)N, cfg.seed, ep, cfg.iteration);
     for (int mbi = 0; mbi < pl.nmb; ++mbi) {
@@ -229,15 +240,29 @@ pe_status ppo_update_bf16(const pe_net& net, float* params, float* m, float* v, 
       lh.ent_coef = cfg.ent_coef;
       lh.inv_cnt = 1.0f / (float)cnt;
       lh.part = lossp;
-      lh.dz = dz[0];
-      s = bf16_forward_loss(net, img, params, 0, obs, idx, cnt, lh, x, h[0], h[1], err, st);
-      if (s != PE_OK) return s;
-      lh.dz = dz[1];
-      s = bf16_forward_loss(net, img + pl.img, params, 1, obs, idx, cnt, lh, nullptr, h[2], h[3], err, st);
+      if (fused) {
+        // 72B: forward, loss and backward data products of a network in one
+        // kernel (its backward images first)
+        s = bf16_bwd_images(net, params, bimg, st);
+        if (s != PE_OK) return s;
+        lh.dz = dz[0];
+        s = bf16_fused_fwd_bwd(net, img, bimg[0], params, 0, obs, idx, cnt, lh, x, h[0], h[1], da2[0], da1[0], err,
+                               st);
+        if (s != PE_OK) return s;
+        lh.dz = dz[1];
+        s = bf16_fused_fwd_bwd(net, img + pl.img, bimg[1], params, 1, obs, idx, cnt, lh, nullptr, h[2], h[3], da2[1],
+                               da1[1], err, st);
+      } else {
+        lh.dz = dz[0];
+        s = bf16_forward_loss(net, img, params, 0, obs, idx, cnt, lh, x, h[0], h[1], err, st);
+        if (s != PE_OK) return s;
+        lh.dz = dz[1];
+        s = bf16_forward_loss(net, img + pl.img, params, 1, obs, idx, cnt, lh, nullptr, h[2], h[3], err, st);
+      }
       if (s != PE_OK) return s;
       const int nlb = rows / kTile * 4;
       s = bf16_backward(net, params, bimg, reinterpret_cast<const uint8_t*>(x), dzc, h1c, h2c, da2, da1, cnt, part,
-                        grad, lossp, nlb, stat5, sq, err, st);
+                        grad, lossp, nlb, stat5, sq, err, fused, st);
       if (s != PE_OK) return s;
       t += 1;
       AdamBf16Args ad;
