@@ -16,7 +16,9 @@
 // Read with samples as the reduction dimension, the same bytes are the
 // MN-major operands of the weight-gradient products.
 //
-// bwd_data_kernel (one 128-sample tile at a time, persistent):
+// bwd_data_kernel (Stress, H = 512; one 128-sample tile at a time,
+// persistent; the 72B networks compute these products inside the fused
+// forward-backward kernel of fused_bf16.cu):
 //   dh2 = dz W3 (one MMA per 256 columns, K = 16) -> TMEM; epilogue:
 //   da2 = bf16(dh2 (1 - h2^2)) into shared memory (the next A operand) and
 //   its tile image; dh1 = da2 W2 with W2^T streamed through a two-slot ring
@@ -297,243 +299,6 @@ __global__ void __launch_bounds__(kBwThreads, 1) bwd_data_kernel(BwdArgs g) {
   if (tid == 0 && s.err && g.err) atomicExch(g.err, 1);
   __syncthreads();
   if (warp == 0) tc::tmem_dealloc(tmem, H);
-}
-
-// ---------------------------------------------------------------------------
-// Two tiles in flight for the 72B networks (H = 256), as in the forward
-// mlp_bf16_pair_kernel: each CTA holds two 128-sample tiles (slots), each
-// with its own da2 buffer, dz tile and half of TMEM (columns 256 s ..
-// 256 s + 255 for dh2, then dh1), and the epilogue of one slot overlaps the
-// MMAs of the other.  Warps 0-15 run the epilogues, warp 16 streams W2^T,
-// warp 17 issues the MMAs; hand-overs as in the forward pair kernel:
-//   dzin[s], d2in[s]: the 16 epilogue warps wrote the slot's dz / da2;
-//   mma1[s], mma2[s]: the slot's dh2 / dh1 MMAs are done.
-// Warp 18 brings each slot's h2 image into the slot's da2 buffer (da2
-// overwrites it in place) and, once the slot's dh1 MMAs are done, its h1
-// image:
-//   hin[s]: an h image landed (h2, then h1: two completions per tile);
-//   bfree[s]: the 16 epilogue warps have read the slot's h1.
-// The arithmetic of every tile is bwd_data_kernel's: the same bits.
-// ---------------------------------------------------------------------------
-constexpr int kBwPairThreads = 608;
-
-template <int H>
-struct BwdPairSmem {
-  alignas(1024) uint8_t da2[2][kBwRows * H * 2];
-  alignas(1024) uint8_t ring[2][kBwStage];
-  alignas(1024) uint8_t w3t[H * 32];
-  alignas(1024) uint8_t dz[2][kBwRows * 32];
-  uint64_t bar_w, full[2], empty[2], mma1[2], mma2[2], dzin[2], d2in[2], hin[2], bfree[2];
-  uint32_t tmem_base;
-  int32_t err;
-};
-
-template <int H>
-__global__ void __launch_bounds__(kBwPairThreads, 1) bwd_data_pair_kernel(BwdArgs g) {
-  using I = BwdImg<H>;
-  static_assert(H == 256, "two tiles in flight need 2 x 256 TMEM columns");
-  extern __shared__ __align__(1024) uint8_t smem_raw[];
-  uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
-  BwdPairSmem<H>& s = *reinterpret_cast<BwdPairSmem<H>*>(base);
-  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  if (tid == 0) {
-    s.err = 0;
-    tc::mbar_init(&s.bar_w, 1);
-    for (int i = 0; i < 2; ++i) {
-      tc::mbar_init(&s.full[i], 1);
-      tc::mbar_init(&s.empty[i], 1);
-      tc::mbar_init(&s.mma1[i], 1);
-      tc::mbar_init(&s.mma2[i], 1);
-      tc::mbar_init(&s.dzin[i], 16);
-      tc::mbar_init(&s.d2in[i], 16);
-      tc::mbar_init(&s.hin[i], 1);
-      tc::mbar_init(&s.bfree[i], 16);
-    }
-    tc::fence_mbar_init();
-  }
-  if (warp == 0) tc::tmem_alloc(&s.tmem_base, 512);
-  tc::fence_before();
-  __syncthreads();
-  tc::fence_after();
-  const uint32_t tmem = s.tmem_base;
-  const int64_t tiles = (g.n + kBwRows - 1) / kBwRows;
-  const int my_tiles = (int)((tiles - blockIdx.x + gridDim.x - 1) / gridDim.x);
-  const int npairs = (my_tiles + 1) / 2;
-  constexpr int kTileBytes = kBwRows * H * 2;
-  int last_issued = -1;
-  int h_issued[2] = {0, 0};  // loader: h copies issued per slot (the hin phases)
-  if (warp == 18) {
-    if (lane == 0) {
-      // the slot's h2 image once its previous tile's h1 has been read, an
-      // arrival without bytes for a slot with no tile
-      auto bring = [&](int sl, int k, const uint8_t* src) {
-        const bool vt = k < my_tiles;
-        tc::mbar_expect_tx(&s.hin[sl], vt ? (uint32_t)kTileBytes : 0u);
-        if (vt)
-          tc::bulk_g2s(s.da2[sl], src + ((int64_t)blockIdx.x + (int64_t)k * gridDim.x) * kTileBytes,
-                       (uint32_t)kTileBytes, &s.hin[sl]);
-        ++h_issued[sl];
-      };
-      bool ok = true;
-      for (int p = 0; p < npairs && ok; ++p) {
-        for (int sl = 0; sl < 2 && ok; ++sl) {
-          ok = p == 0 || tc::mbar_wait(&s.bfree[sl], (p - 1) & 1);
-          if (ok) bring(sl, 2 * p + sl, g.h2);
-        }
-        for (int sl = 0; sl < 2 && ok; ++sl) {
-          ok = tc::mbar_wait(&s.mma2[sl], p & 1);
-          if (ok) bring(sl, 2 * p + sl, g.h1);
-        }
-      }
-      if (!ok) atomicExch(&s.err, 1);
-    }
-  } else if (warp == 16) {
-    if (lane == 0) {
-      int gs = 0;
-      for (int p = 0; p < npairs; ++p)
-        for (int sl = 0; sl < 2; ++sl)
-          for (int st = 0; st < I::STAGES; ++st, ++gs) {
-            const int slot = gs & 1;
-            if (gs >= 2 && !tc::mbar_wait(&s.empty[slot], ((gs - 2) >> 1) & 1)) atomicExch(&s.err, 1);
-            tc::mbar_expect_tx(&s.full[slot], (uint32_t)kBwStage);
-            tc::bulk_g2s(s.ring[slot], g.img + I::W3T + (int64_t)st * kBwStage, (uint32_t)kBwStage, &s.full[slot]);
-            last_issued = gs;
-          }
-    }
-  } else if (warp == 17) {
-    if (lane == 0) {
-      tc::mbar_expect_tx(&s.bar_w, (uint32_t)I::W3T);
-      tc::bulk_g2s(s.w3t, g.img, (uint32_t)I::W3T, &s.bar_w);
-      if (!tc::mbar_wait(&s.bar_w, 0)) atomicExch(&s.err, 1);
-      const uint32_t w3a = tc::smem_u32(s.w3t);
-      const uint32_t r0a = tc::smem_u32(s.ring[0]), r1a = tc::smem_u32(s.ring[1]);
-      constexpr uint32_t kIdN = tc::idesc_bf16(kBwRows, 256);
-      int gs = 0;
-      for (int p = 0; p < npairs; ++p) {
-        const uint32_t par = p & 1;
-        for (int sl = 0; sl < 2; ++sl) {
-          if (!tc::mbar_wait(&s.dzin[sl], par)) atomicExch(&s.err, 1);
-          tc::fence_after();
-          tc::mma_bf16(tmem + sl * 256, tc::desc_strided(tc::smem_u32(s.dz[sl]), 16, 256, tc::kLayoutSW32),
-                       tc::desc_strided(w3a, 16, 256, tc::kLayoutSW32), kIdN, 0);
-          tc::mma_commit(&s.mma1[sl]);
-        }
-        for (int sl = 0; sl < 2; ++sl) {
-          if (!tc::mbar_wait(&s.d2in[sl], par)) atomicExch(&s.err, 1);
-          tc::fence_after();
-          const uint32_t da2a = tc::smem_u32(s.da2[sl]);
-          for (int kb = 0; kb < I::KB; ++kb, ++gs) {
-            const int slot = gs & 1;
-            if (!tc::mbar_wait(&s.full[slot], (gs >> 1) & 1)) atomicExch(&s.err, 1);
-            tc::fence_after();
-            const uint32_t ra = slot ? r1a : r0a;
-#pragma unroll
-            for (int kk = 0; kk < 4; ++kk)
-              tc::mma_bf16(tmem + sl * 256, tc::desc_kmajor(da2a + kb * kBwRows * 128 + kk * 32, 1024, tc::kLayoutSW128),
-                           tc::desc_kmajor(ra + kk * 32, 1024, tc::kLayoutSW128), kIdN, (kb | kk) != 0);
-            tc::mma_commit(&s.empty[slot]);
-          }
-          tc::mma_commit(&s.mma2[sl]);
-        }
-      }
-    }
-  } else {
-    constexpr int NJ = H / 4 / 16;  // 16-column chunks per thread
-    const int quad = warp & 3, slice = warp >> 2, row = quad * 32 + lane;
-    const uint32_t lane_base = tmem + ((uint32_t)(quad * 32) << 16);
-    auto tile_of = [&](int k) { return (int64_t)blockIdx.x + (int64_t)k * gridDim.x; };
-    auto handover = [&](uint64_t* bar) {
-      tc::fence_async_smem();
-      tc::fence_before();
-      __syncwarp();
-      if (lane == 0) asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(tc::smem_u32(bar)) : "memory");
-    };
-    // one epilogue: d = bf16(TMEM (1 - h^2)) of slot sl, h read from the
-    // slot's buffer where the loader put it; d to the tile image and, for
-    // da2, in place over h2 (the next A operand)
-    auto epi = [&](int sl, int k, uint8_t* gout, bool in_place, uint64_t* mbar, uint32_t par, uint32_t hpar) {
-      const bool vt = k < my_tiles;
-      const int64_t tl = tile_of(k);
-      const int nr = vt ? (int)(g.n - tl * kBwRows < kBwRows ? g.n - tl * kBwRows : kBwRows) : 0;
-      const bool valid = row < nr;
-      if (!tc::mbar_wait(&s.hin[sl], hpar)) atomicExch(&s.err, 1);
-      if (!tc::mbar_wait(mbar, par)) atomicExch(&s.err, 1);
-      tc::fence_after();
-      uint8_t* outt = vt ? gout + tl * (int64_t)kTileBytes : nullptr;
-      uint8_t* buf = s.da2[sl];
-#pragma unroll
-      for (int j = 0; j < NJ; ++j) {
-        const int c = slice * (H / 4) + j * 16;
-        float v[16];
-        tc::tmem_ld16(lane_base + (uint32_t)(sl * 256 + c), v);
-        const uint32_t o0 = tc::swz_offset<128>(row, c, kBwRows), o1 = tc::swz_offset<128>(row, c + 8, kBwRows);
-        const uint4 hb[2] = {*reinterpret_cast<const uint4*>(buf + o0), *reinterpret_cast<const uint4*>(buf + o1)};
-        uint32_t pk[8];
-        tanh_grad16(v, hb, valid, pk);
-        const uint4 lo = make_uint4(pk[0], pk[1], pk[2], pk[3]), hi = make_uint4(pk[4], pk[5], pk[6], pk[7]);
-        if (in_place) {
-          *reinterpret_cast<uint4*>(buf + o0) = lo;
-          *reinterpret_cast<uint4*>(buf + o1) = hi;
-        }
-        if (outt) {
-          *reinterpret_cast<uint4*>(outt + o0) = lo;
-          *reinterpret_cast<uint4*>(outt + o1) = hi;
-        }
-      }
-    };
-    uint4 dzv[2] = {make_uint4(0, 0, 0, 0), make_uint4(0, 0, 0, 0)};
-    auto fetch_dz = [&](int k, uint4& dst) {
-      dst = make_uint4(0, 0, 0, 0);
-      if (tid < kBwRows * 2 && k < my_tiles)
-        dst = __ldg(reinterpret_cast<const uint4*>(g.dz + tile_of(k) * (kBwRows * 32)) + tid);
-    };
-    // The h1/h2 tile images of a pair's two tiles (4 x 64 KB) are asked of L2
-    // one pair ahead, one 128-byte line per thread per image, so that the
-    // loader's bulk copies read L2 instead of waiting for HBM.
-    auto prefetch_pair = [&](int p) {
-#pragma unroll
-      for (int sl = 0; sl < 2; ++sl) {
-        const int k = 2 * p + sl;
-        if (k < my_tiles) {
-          const int64_t off = tile_of(k) * (int64_t)(kBwRows * H * 2) + (int64_t)tid * 128;
-          tc::prefetch_l2(g.h2 + off);
-          tc::prefetch_l2(g.h1 + off);
-        }
-      }
-    };
-    static_assert(kBwRows * H * 2 == 512 * 128, "one line per epilogue thread per tile image");
-    prefetch_pair(0);
-    fetch_dz(0, dzv[0]);
-    fetch_dz(1, dzv[1]);
-    for (int p = 0; p < npairs; ++p) {
-      const uint32_t par = p & 1;
-      prefetch_pair(p + 1);
-      for (int sl = 0; sl < 2; ++sl) {
-        if (tid < kBwRows * 2) reinterpret_cast<uint4*>(s.dz[sl])[tid] = dzv[sl];
-        handover(&s.dzin[sl]);
-      }
-      fetch_dz(2 * p + 2, dzv[0]);
-      fetch_dz(2 * p + 3, dzv[1]);
-      for (int sl = 0; sl < 2; ++sl) {
-        epi(sl, 2 * p + sl, g.da2, true, &s.mma1[sl], par, 0);
-        handover(&s.d2in[sl]);
-      }
-      for (int sl = 0; sl < 2; ++sl) {
-        epi(sl, 2 * p + sl, g.da1, false, &s.mma2[sl], par, 1);
-        handover(&s.bfree[sl]);
-      }
-    }
-  }
-  tc::fence_before();
-  __syncthreads();
-  if (s.err && warp == 16 && lane == 0 && last_issued >= 0)
-    (void)tc::mbar_wait(&s.full[last_issued & 1], (last_issued >> 1) & 1);
-  if (s.err && warp == 18 && lane == 0)
-    for (int sl = 0; sl < 2; ++sl)
-      if (h_issued[sl] > 0) (void)tc::mbar_wait(&s.hin[sl], (h_issued[sl] - 1) & 1);
-  if (tid == 0 && s.err && g.err) atomicExch(g.err, 1);
-  __syncthreads();
-  if (warp == 0) tc::tmem_dealloc(tmem, 512);
 }
 
 // ---------------------------------------------------------------------------
@@ -829,17 +594,7 @@ static pe_status bwd_launch(const float* params, int A, uint8_t* const img[2], c
   if (data_done) {
     // the backward images and the data products came with the fused forward-backward kernel
   } else if constexpr (H == 256) {
-    pe_status s = bwd_images<D, H>(params, A, img, st);
-    if (s != PE_OK) return s;
-    auto kern = bwd_data_pair_kernel<H>;
-    const int bytes = (int)sizeof(BwdPairSmem<H>) + 1024;
-    PE_TRY_CUDA(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes));
-    const int grid = (int)std::min<int64_t>((tiles + 1) / 2, sms);
-    ProfScope ps(PE_PROF_PPO_GRAD, st);
-    for (int ni = 0; ni < 2; ++ni) {
-      BwdArgs a{img[ni], dz[ni], h1[ni], h2[ni], da2[ni], da1[ni], n, err};
-      kern<<<grid, kBwPairThreads, bytes, st>>>(a);
-    }
+    return fail(PE_EINVAL, "the 72B data products run in the fused forward-backward kernel");
   } else {
     pe_status s = bwd_images<D, H>(params, A, img, st);
     if (s != PE_OK) return s;

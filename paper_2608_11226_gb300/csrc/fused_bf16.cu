@@ -4,9 +4,10 @@
 //     -> loss and dz (the head epilogue) -> dh2 = dz W3 -> da2 = bf16(dh2 (1 - h2^2))
 //     -> dh1 = da2 W2 -> da1 = bf16(dh1 (1 - h1^2)),
 // in one kernel, with the arithmetic of mlp_bf16_pair_kernel followed by
-// bwd_data_pair_kernel (the same bits).  h2 and dz never leave the chip
-// between the two halves: da2 overwrites h2 in place in the tile's shared
-// buffer, and dz goes to shared memory beside its tile image.  The tile
+// the backward data products of bwd_bf16.cu (the same bits).  h2 and dz
+// never leave the chip between the two halves: da2 overwrites h2 in place in
+// the tile's shared buffer, and dz goes to shared memory beside its tile
+// image.  The tile
 // images the weight-gradient kernel reads (x, h1, h2, dz, da2, da1) are
 // written as before.
 //
