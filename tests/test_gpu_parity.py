@@ -751,6 +751,23 @@ def test_ppo_bf16_single_step(preset, E, T):
     assert_stats(gs, st, T * E, tol=BF16_TOL)
 
 
+@pytest.mark.parametrize("preset,E,T", [("72b", 320, 128), ("stress", 160, 122)])
+def test_ppo_bf16_several_tiles_per_cta(preset, E, T):
+    """One minibatch large enough that the persistent kernels take more than
+    one tile (pair) per CTA: 72B 40,960 samples = 320 tiles over 152 CTAs
+    (the first 16 run two tile pairs, the second half empty); Stress 19,520
+    samples = 153 tiles (the first CTA runs two).  Adam's first moment after
+    one step is 0.1 x the clipped gradient."""
+    wl = W.make_72b(n_envs=E) if preset == "72b" else W.make_stress(n_envs=E, horizon=T)
+    params, buf, adv, ret = _ppo_inputs(wl, T, seed=4)
+    ppo = W.PPOSpec(epochs=1, minibatch=T * E, ent_coef=0.01)
+    gp, gm, gv, gs = _run_ppo(wl, ppo, params, buf, adv, ret, iteration=1)
+    P, m, v, t, st = _oracle_ppo(wl, ppo, params, buf, adv, ret, iteration=1)
+    assert t == 1 and gs[7] == 1
+    assert bf16_ok(gm, m), (np.abs(gm - m).max() / np.abs(m).max())
+    assert_stats(gs, st, T * E, tol=BF16_TOL)
+
+
 @pytest.mark.parametrize("preset,E,mb,clip", [("72b", 64, 1500, 0.2), ("72b", 64, 1500, 0.01),
                                               ("stress", 32, 900, 0.01)])
 def test_ppo_bf16_ragged_epochs(preset, E, mb, clip):
