@@ -140,6 +140,39 @@ struct Img {
   static_assert(TOTAL + ACT + 3 * 1024 <= 232448, "weights and one activation tile must fit in shared memory");
 };
 
+// the streamed forward image of the Stress network (D = 64, H = 512):
+// 32 KB stages in consumption order -- W1 as 2 N-halves, W2 as 2 N-halves x
+// 8 K-blocks of 64, each 256 rows x 128 bytes (SW128) -- then the head
+constexpr int kStageBytes = 32768;
+constexpr int kStreamStages = 19;  // per tile (H = 512, D = 64)
+
+template <int D, int H>
+struct ImgS {
+  static_assert(D == 64 && H == 512, "streamed layout is laid out for D = 64, H = 512");
+  static constexpr int HEAD_OFF = 18 * kStageBytes;
+  static constexpr int TOTAL = HEAD_OFF + kHeadN * H * 2;  // 592 KB
+  __host__ __device__ static int stage_off(int s) { return s * kStageBytes; }
+  __host__ __device__ static int stage_bytes(int s) { return s < 18 ? kStageBytes : kHeadN * H * 2; }
+};
+
+// byte offset of weight (r, k) of layer mat (1: W1 [H][D], 2: W2 [H][H],
+// 3: the head W3 [16][H]) in a network's forward image (Img for H <= 256,
+// ImgS for the streamed network)
+template <int D, int H>
+__host__ __device__ __forceinline__ uint32_t fwd_img_offset(int mat, int r, int k) {
+  if constexpr (H > 256) {
+    if (mat == 1) return (uint32_t)((r / 256) * kStageBytes) + tc::swz_offset<128>(r % 256, k, 256);
+    if (mat == 2)
+      return (uint32_t)((2 + (r / 256) * (H / 64) + k / 64) * kStageBytes) + tc::swz_offset<128>(r % 256, k % 64, 256);
+    return (uint32_t)ImgS<D, H>::HEAD_OFF + tc::swz_offset<128>(r, k, kHeadN);
+  } else {
+    using I = Img<D, H>;
+    if (mat == 1) return tc::swz_offset<I::RB1>(r, k, H);
+    if (mat == 2) return (uint32_t)I::W1 + tc::swz_offset<128>(r, k, H);
+    return (uint32_t)(I::W1 + I::W2) + tc::swz_offset<128>(r, k, kHeadN);
+  }
+}
+
 constexpr int kBwRows = 128;            // samples per tile (MMA M of the data products)
 constexpr int kBwStage = 32768;         // one streamed W2^T stage: 256 rows x 64 K, SW128
 
@@ -153,6 +186,18 @@ struct BwdImg {
   static constexpr int TOTAL = W3T + STAGES * kBwStage;
   static_assert(W3T % 1024 == 0, "stages start on a swizzle atom");
 };
+
+// byte offset in a network's backward image of W2[o][c] (mat = 2; stored as
+// W2^T[c][o] in the streamed stages) or of W3[a][o] (mat = 3; stored as
+// W3^T[o][a])
+template <int H>
+__host__ __device__ __forceinline__ uint32_t bwd_img_offset(int mat, int row, int col) {
+  using I = BwdImg<H>;
+  if (mat == 3) return tc::swz_offset<32>(col, row, H);
+  const int o = row, c = col;
+  const int stage = (c / 256) * I::KB + o / 64;
+  return (uint32_t)(I::W3T + stage * kBwStage) + tc::swz_offset<128>(c % 256, o % 64, 256);
+}
 
 // d = bf16(g (1 - h^2)) for 16 columns: g from TMEM, h as 16 packed bf16
 __device__ __forceinline__ void tanh_grad16(const float (&g)[16], const uint4 (&h)[2], bool valid,

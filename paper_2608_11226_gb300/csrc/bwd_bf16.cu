@@ -66,12 +66,10 @@ __global__ void bwd_image_kernel(const float* __restrict__ params, int A, uint8_
     if (i < H * 16) {
       const int o = i / 16, a = i % 16;  // W3^T[o][a] = W3[a][o]
       const float v = a < nout ? w3[(int64_t)a * H + o] : 0.0f;
-      *reinterpret_cast<__nv_bfloat16*>(img + tc::swz_offset<32>(o, a, H)) = __float2bfloat16_rn(v);
+      *reinterpret_cast<__nv_bfloat16*>(img + bwd_img_offset<H>(3, a, o)) = __float2bfloat16_rn(v);
     } else {
       const int j = i - H * 16, o = j / H, c = j % H;  // W2[o][c] = W2^T[c][o]
-      const int stage = (c / 256) * I::KB + o / 64;
-      *reinterpret_cast<__nv_bfloat16*>(img + I::W3T + stage * kBwStage + tc::swz_offset<128>(c % 256, o % 64, 256)) =
-          __float2bfloat16_rn(w2[j]);
+      *reinterpret_cast<__nv_bfloat16*>(img + bwd_img_offset<H>(2, o, c)) = __float2bfloat16_rn(w2[j]);
     }
   }
 }
@@ -596,8 +594,6 @@ static pe_status bwd_launch(const float* params, int A, uint8_t* const img[2], c
   } else if constexpr (H == 256) {
     return fail(PE_EINVAL, "the 72B data products run in the fused forward-backward kernel");
   } else {
-    pe_status s = bwd_images<D, H>(params, A, img, st);
-    if (s != PE_OK) return s;
     auto kern = bwd_data_kernel<H>;
     const int bytes = (int)sizeof(BwdSmem<H>) + 1024;
     PE_TRY_CUDA(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes));

@@ -48,18 +48,18 @@ __global__ void weight_image_kernel(const float* __restrict__ params, int A, int
   const int nout = value_net ? 1 : A;
   const int total = H * D + H * H + kHeadN * H;
   for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < total; i += gridDim.x * blockDim.x) {
+    int mat, r, k;
+    float v;
     if (i < H * D) {
-      const int r = i / D, k = i % D;
-      *reinterpret_cast<__nv_bfloat16*>(img + tc::swz_offset<I::RB1>(r, k, H)) = __float2bfloat16_rn(w1[i]);
+      mat = 1, r = i / D, k = i % D, v = w1[i];
     } else if (i < H * D + H * H) {
-      const int j = i - H * D, r = j / H, k = j % H;
-      *reinterpret_cast<__nv_bfloat16*>(img + I::W1 + tc::swz_offset<128>(r, k, H)) = __float2bfloat16_rn(w2[j]);
+      const int j = i - H * D;
+      mat = 2, r = j / H, k = j % H, v = w2[j];
     } else {
-      const int j = i - H * D - H * H, r = j / H, k = j % H;
-      const float v = r < nout ? w3[r * H + k] : 0.0f;
-      *reinterpret_cast<__nv_bfloat16*>(img + I::W1 + I::W2 + tc::swz_offset<128>(r, k, kHeadN)) =
-          __float2bfloat16_rn(v);
+      const int j = i - H * D - H * H;
+      mat = 3, r = j / H, k = j % H, v = r < nout ? w3[r * H + k] : 0.0f;
     }
+    *reinterpret_cast<__nv_bfloat16*>(img + fwd_img_offset<D, H>(mat, r, k)) = __float2bfloat16_rn(v);
   }
 }
 
@@ -77,19 +77,8 @@ __global__ void weight_image_kernel(const float* __restrict__ params, int A, int
 // warps synchronise with a named barrier so that the producer never waits
 // on them.
 // ---------------------------------------------------------------------------
-constexpr int kStageBytes = 32768;
-constexpr int kStreamStages = 19;  // per tile (H = 512, D = 64)
 constexpr int kComputeThreads = 512;
 constexpr int kStreamThreads = kComputeThreads + 32;
-
-template <int D, int H>
-struct ImgS {
-  static_assert(D == 64 && H == 512, "streamed layout is laid out for D = 64, H = 512");
-  static constexpr int HEAD_OFF = 18 * kStageBytes;
-  static constexpr int TOTAL = HEAD_OFF + kHeadN * H * 2;  // 592 KB
-  __host__ __device__ static int stage_off(int s) { return s * kStageBytes; }
-  __host__ __device__ static int stage_bytes(int s) { return s < 18 ? kStageBytes : kHeadN * H * 2; }
-};
 
 template <int D, int H>
 __global__ void weight_image_stream_kernel(const float* __restrict__ params, int A, int value_first,
@@ -104,23 +93,18 @@ __global__ void weight_image_stream_kernel(const float* __restrict__ params, int
   const int nout = value_net ? 1 : A;
   const int total = H * D + H * H + kHeadN * H;
   for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < total; i += gridDim.x * blockDim.x) {
-    uint32_t off;
+    int mat, r, k;
     float v;
     if (i < H * D) {
-      const int r = i / D, k = i % D;
-      off = (r / 256) * kStageBytes + tc::swz_offset<128>(r % 256, k, 256);
-      v = w1[i];
+      mat = 1, r = i / D, k = i % D, v = w1[i];
     } else if (i < H * D + H * H) {
-      const int j = i - H * D, r = j / H, k = j % H;
-      const int stage = 2 + (r / 256) * 8 + k / 64;
-      off = stage * kStageBytes + tc::swz_offset<128>(r % 256, k % 64, 256);
-      v = w2[j];
+      const int j = i - H * D;
+      mat = 2, r = j / H, k = j % H, v = w2[j];
     } else {
-      const int j = i - H * D - H * H, r = j / H, k = j % H;
-      off = I::HEAD_OFF + tc::swz_offset<128>(r, k, kHeadN);
-      v = r < nout ? w3[r * H + k] : 0.0f;
+      const int j = i - H * D - H * H;
+      mat = 3, r = j / H, k = j % H, v = r < nout ? w3[r * H + k] : 0.0f;
     }
-    *reinterpret_cast<__nv_bfloat16*>(img + off) = __float2bfloat16_rn(v);
+    *reinterpret_cast<__nv_bfloat16*>(img + fwd_img_offset<D, H>(mat, r, k)) = __float2bfloat16_rn(v);
   }
 }
 

@@ -19,7 +19,8 @@
 //                products of a network run as one kernel (fused_bf16.cu);
 //   step      -- the gradient's squared norm (summed with the weight
 //                gradients' reduction), clip, Adam on the fp32 master
-//                parameters.
+//                parameters, which also writes the updated weights into the
+//                bf16 weight images (built once per call).
 // Rounding points (which the oracle reproduces): dz, da2 and da1 enter the
 // products as bf16; the layer bias gradients sum the rounded values, the head
 // bias gradient the fp32 dz.
@@ -27,6 +28,7 @@
 
 #include <cmath>
 
+#include "bf16_layout.cuh"
 #include "mlp_f32.cuh"
 
 namespace pe {
@@ -80,8 +82,17 @@ struct AdamBf16Args {
   float beta1, beta2, step_size, inv_sqrt_bc2, eps, max_norm, vf_coef, ent_coef, inv_cnt;
   const double* stat5;
   double* acc;
+  int A;                // policy actions
+  uint8_t* fimg;        // forward weight images of both networks (fstride apart)
+  int64_t fstride;
+  uint8_t* bimg[2];     // backward weight images (policy, value)
 };
 
+// Clip and Adam on the fp32 master parameters, writing every updated weight's
+// bf16 copy straight into the forward and backward weight images (the next
+// minibatch step's operands), so that the images need no rebuild per step;
+// the conversion is the image kernels' own (round to nearest even).
+template <int D, int H>
 __global__ void adam_bf16_kernel(AdamBf16Args a) {
   __shared__ float s_norm;
   if (threadIdx.x < 32) {
@@ -100,7 +111,25 @@ __global__ void adam_bf16_kernel(AdamBf16Args a) {
     const float vp = a.beta2 * a.v[p] + (1.0f - a.beta2) * gp * gp;
     a.m[p] = mp;
     a.v[p] = vp;
-    a.params[p] -= a.step_size * mp / (sqrtf(vp) * a.inv_sqrt_bc2 + a.eps);
+    const float pn = a.params[p] - a.step_size * mp / (sqrtf(vp) * a.inv_sqrt_bc2 + a.eps);
+    a.params[p] = pn;
+    // the weight's place in the images: network, layer, row, column
+    const MlpLayout L = mlp_layout(D, H, a.A);
+    int net = -1, mat = 0;
+    int64_t q = 0;
+    if (p < L.b1) net = 0, mat = 1, q = p - L.w1;
+    else if (p >= L.w2 && p < L.b2) net = 0, mat = 2, q = p - L.w2;
+    else if (p >= L.w3 && p < L.b3) net = 0, mat = 3, q = p - L.w3;
+    else if (p >= L.v1 && p < L.c1) net = 1, mat = 1, q = p - L.v1;
+    else if (p >= L.v2 && p < L.c2) net = 1, mat = 2, q = p - L.v2;
+    else if (p >= L.v3 && p < L.c3) net = 1, mat = 3, q = p - L.v3;
+    if (net >= 0) {
+      const int cols = mat == 1 ? D : H;
+      const int r = (int)(q / cols), k = (int)(q % cols);
+      const __nv_bfloat16 b = __float2bfloat16_rn(pn);
+      *reinterpret_cast<__nv_bfloat16*>(a.fimg + net * a.fstride + fwd_img_offset<D, H>(mat, r, k)) = b;
+      if (mat >= 2) *reinterpret_cast<__nv_bfloat16*>(a.bimg[net] + bwd_img_offset<H>(mat, r, k)) = b;
+    }
   }
   if (blockIdx.x == 0 && threadIdx.x == 0) {
     double v5[5];
@@ -216,6 +245,11 @@ pe_status ppo_update_bf16(const pe_net& net, float* params, float* m, float* v, 
   if (s != PE_OK) return s;
   int64_t t = adam_t;
   const bool fused = bf16_fused_supported(net);
+  // the bf16 weight images of both networks, built once; each Adam step
+  // writes its updated weights into them
+  s = bf16_make_images(net, params, img, st);
+  if (s == PE_OK) s = bf16_bwd_images(net, params, bimg, st);
+  if (s != PE_OK) return s;
   for (int ep = 0; ep < cfg.epochs; ++ep) {
     const Feistel f = make_feistel((uint64_t)N, cfg.seed, ep, cfg.iteration);
     for (int mbi = 0; mbi < pl.nmb; ++mbi) {
@@ -227,8 +261,6 @@ pe_status ppo_update_bf16(const pe_net& net, float* params, float* m, float* v, 
         perm_index_kernel<<<ceil_div(cnt, 256), 256, 0, st>>>(f, start, cnt, idx);
       }
       PE_CHECK_LAUNCH("perm_index_kernel");
-      s = bf16_make_images(net, params, img, st);
-      if (s != PE_OK) return s;
       PpoHead lh;
       lh.act = act;
       lh.logp_old = logp_old;
@@ -243,8 +275,6 @@ pe_status ppo_update_bf16(const pe_net& net, float* params, float* m, float* v, 
       if (fused) {
         // 72B: forward, loss and backward data products of a network in one
         // kernel (its backward images first)
-        s = bf16_bwd_images(net, params, bimg, st);
-        if (s != PE_OK) return s;
         lh.dz = dz[0];
         s = bf16_fused_fwd_bwd(net, img, bimg[0], params, 0, obs, idx, cnt, lh, x, h[0], h[1], da2[0], da1[0], err,
                                st);
@@ -284,9 +314,17 @@ pe_status ppo_update_bf16(const pe_net& net, float* params, float* m, float* v, 
       ad.inv_cnt = 1.0f / (float)cnt;
       ad.stat5 = stat5;
       ad.acc = acc;
+      ad.A = A;
+      ad.fimg = img;
+      ad.fstride = pl.img;
+      ad.bimg[0] = bimg[0];
+      ad.bimg[1] = bimg[1];
       {
         ProfScope ps(PE_PROF_PPO_ADAM, st);
-        adam_bf16_kernel<<<ceil_div(pl.P, 256), 256, 0, st>>>(ad);
+        if (pl.D == 32 && pl.H == 256)
+          adam_bf16_kernel<32, 256><<<ceil_div(pl.P, 256), 256, 0, st>>>(ad);
+        else
+          adam_bf16_kernel<64, 512><<<ceil_div(pl.P, 256), 256, 0, st>>>(ad);
       }
       PE_CHECK_LAUNCH("ppo bf16 step kernels");
     }
