@@ -86,12 +86,18 @@ struct AdamBf16Args {
   uint8_t* fimg;        // forward weight images of both networks (fstride apart)
   int64_t fstride;
   uint8_t* bimg[2];     // backward weight images (policy, value)
+  Feistel nf;           // the next minibatch step's permutation ...
+  int64_t nstart;       // ... and its first position
+  int ncnt;             // its sample count (0: no next step)
+  uint32_t* idx;        // out: its gather indices
 };
 
 // Clip and Adam on the fp32 master parameters, writing every updated weight's
 // bf16 copy straight into the forward and backward weight images (the next
 // minibatch step's operands), so that the images need no rebuild per step;
-// the conversion is the image kernels' own (round to nearest even).
+// the conversion is the image kernels' own (round to nearest even).  The same
+// launch writes the next minibatch step's Feistel gather indices (the current
+// step's kernels, which read them, have finished).
 template <int D, int H>
 __global__ void adam_bf16_kernel(AdamBf16Args a) {
   __shared__ float s_norm;
@@ -131,6 +137,8 @@ __global__ void adam_bf16_kernel(AdamBf16Args a) {
       if (mat >= 2) *reinterpret_cast<__nv_bfloat16*>(a.bimg[net] + bwd_img_offset<H>(mat, r, k)) = b;
     }
   }
+  for (int64_t j = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; j < a.ncnt; j += (int64_t)gridDim.x * blockDim.x)
+    a.idx[j] = feistel_index(a.nf, a.nstart + j);
   if (blockIdx.x == 0 && threadIdx.x == 0) {
     double v5[5];
     for (int k = 0; k < 5; ++k) v5[k] = a.stat5[k];
@@ -250,17 +258,22 @@ pe_status ppo_update_bf16(const pe_net& net, float* params, float* m, float* v, 
   s = bf16_make_images(net, params, img, st);
   if (s == PE_OK) s = bf16_bwd_images(net, params, bimg, st);
   if (s != PE_OK) return s;
+  // the first minibatch step's gather indices; each Adam launch writes the next step's
+  auto mb_count = [&](int mbi) { return (int)std::min<int64_t>(cfg.minibatch, N - (int64_t)mbi * cfg.minibatch); };
+  if (cfg.epochs > 0 && pl.nmb > 0) {
+    ProfScope ps(PE_PROF_PPO_OTHER, st);
+    perm_index_kernel<<<ceil_div(mb_count(0), 256), 256, 0, st>>>(
+        make_feistel((uint64_t)N, cfg.seed, 0, cfg.iteration), 0, mb_count(0), idx);
+  }
+  PE_CHECK_LAUNCH("perm_index_kernel");
   for (int ep = 0; ep < cfg.epochs; ++ep) {
-    const Feistel f = make_feistel((uint64_t)N, cfg.seed, ep, cfg.iteration);
     for (int mbi = 0; mbi < pl.nmb; ++mbi) {
       const int64_t start = (int64_t)mbi * cfg.minibatch;
-      const int cnt = (int)std::min<int64_t>(cfg.minibatch, N - start);
+      const int cnt = mb_count(mbi);
       const int rows = (cnt + kTile - 1) / kTile * kTile;
-      {
-        ProfScope ps(PE_PROF_PPO_OTHER, st);
-        perm_index_kernel<<<ceil_div(cnt, 256), 256, 0, st>>>(f, start, cnt, idx);
-      }
-      PE_CHECK_LAUNCH("perm_index_kernel");
+      // the step after this one (the next minibatch, or the next epoch's first)
+      const bool last_mb = mbi + 1 == pl.nmb;
+      const int nep = last_mb ? ep + 1 : ep, nmbi = last_mb ? 0 : mbi + 1;
       PpoHead lh;
       lh.act = act;
       lh.logp_old = logp_old;
@@ -319,6 +332,10 @@ pe_status ppo_update_bf16(const pe_net& net, float* params, float* m, float* v, 
       ad.fstride = pl.img;
       ad.bimg[0] = bimg[0];
       ad.bimg[1] = bimg[1];
+      ad.idx = idx;
+      ad.ncnt = nep < cfg.epochs ? mb_count(nmbi) : 0;
+      ad.nstart = (int64_t)nmbi * cfg.minibatch;
+      ad.nf = make_feistel((uint64_t)N, cfg.seed, (uint32_t)(nep < cfg.epochs ? nep : 0), cfg.iteration);
       {
         ProfScope ps(PE_PROF_PPO_ADAM, st);
         if (pl.D == 32 && pl.H == 256)
