@@ -7,11 +7,12 @@
 // independent).  Every minibatch step is three phases behind bounded grid
 // barriers:
 //   1. gradient: each CTA takes ceil(cnt / NC) consecutive samples of the
-//      minibatch (Feistel order) in slices of 64, runs forward and backward
-//      with the activations feature-major in shared memory (4x4 register
-//      tiles, packed two-lane FMA), adds the hidden-layer weight gradients of
-//      every slice into shared-memory accumulators, and writes one fp32
-//      partial gradient row; its weights arrive as one bulk copy of a
+//      minibatch (Feistel order) in slices of 128 (one slice for the 7B
+//      minibatch), runs forward and backward with the activations
+//      feature-major in shared memory (4x4 register tiles, packed two-lane
+//      FMA), writes the hidden-layer weight-gradient tiles straight into its
+//      fp32 partial gradient row (later slices add to it) and the rest of the
+//      row after the last slice; its weights arrive as one bulk copy of a
 //      per-role image laid out like shared memory;
 //   2. reduce: a fixed-order fp32 sum of the NC partial rows of each network
 //      and per-CTA sums of squares (deterministic);
@@ -33,7 +34,7 @@
 
 namespace pe {
 
-constexpr int kPpoS = 64;           // samples per slice
+constexpr int kPpoS = 128;          // samples per slice (a 7B CTA's whole share of a minibatch)
 constexpr int kPpoLD = kPpoS + 4;   // row stride of feature-major activations
 constexpr int kPpoNT = 512;         // threads per gradient CTA
 constexpr int kPpoRT = 4;           // sample rows per thread tile in the dense layers
@@ -86,7 +87,7 @@ __global__ void ppo_advstats_kernel(const float* __restrict__ adv, int64_t N, in
   }
 }
 
-// Dense-layer register tiles for the 64-sample slices: a thread owns RT
+// Dense-layer register tiles for the sample slices: a thread owns RT
 // sample rows x 4 neurons; a warp covers 2 row groups x 16 neuron groups (the
 // fastest of the warp shapes measured on the 7B network: 2x16, 4x8, 8x4 and
 // 16x2 lie within 3% of each other).
@@ -150,7 +151,7 @@ template <int TE, int K, int N, int LD, int LDW>
 __device__ __forceinline__ void dense_bwd_wt(const float* __restrict__ inT, const float* __restrict__ WT,
                                              float* hT, int SV) {
   constexpr int RT = 4, EG = TE / RT, NG = N / 4, JOBS = EG * NG;
-  static_assert(K % 4 == 0 && EG == 16, "backward tile layout");
+  static_assert(K % 4 == 0 && EG % 16 == 0, "backward tile layout");
   for (int j = threadIdx.x; j < JOBS; j += blockDim.x) {
     const int eg = j % EG, kg = j / EG;
     if (eg * RT >= SV) continue;  // samples past the slice's valid rows
@@ -248,9 +249,8 @@ struct WGradAcc {
 
 // Shared memory of one gradient CTA: the role's weights (W1 and W2
 // transposed, w2t rows padded to H + 4 floats so that rows 4 apart fall in
-// different banks; the backward pass reads W2 from the same copy), the
-// CTA's accumulated weight gradients of both hidden layers, and one
-// 64-sample slice of feature-major activations.  h2t holds h2, then the
+// different banks; the backward pass reads W2 from the same copy) and one
+// 128-sample slice of feature-major activations.  h2t holds h2, then the
 // layer-2 pre-activation gradient; h1t holds h1, then the layer-1 one.
 template <int H>
 __host__ __device__ constexpr int w2t_ld() { return H + 4; }
@@ -258,7 +258,6 @@ __host__ __device__ constexpr int w2t_ld() { return H + 4; }
 template <int D, int H, int A>
 struct PpoSmem {
   float w1t[D * H], w2t[H * w2t_ld<H>()], w3[A * H], b1[H], b2[H], b3[8];
-  float gw2[H * w2t_ld<H>()], gw1[H * D];  // gw2 rows padded like w2t (conflict-free adds)
   float xt[D * kPpoLD], h1t[H * kPpoLD], h2t[H * kPpoLD];
   float z[kPpoS * A];
   float lpo[kPpoS], advn[kPpoS], ret[kPpoS];
@@ -342,7 +341,7 @@ template <int D, int H, int A, bool POL>
 __device__ __forceinline__ bool ppo_role(PpoSmem<D, H, A>& s, const PpoArgs& g, int c) {
   constexpr int NA = POL ? A : 1;
   constexpr int S = kPpoS, LD = kPpoLD;
-  static_assert(D % 4 == 0 && H % 32 == 0 && S * (D / 4) <= 256 && 256 + S <= kPpoNT && 4 * H <= kPpoNT,
+  static_assert(D % 4 == 0 && H % 32 == 0 && S * (D / 4) <= kPpoNT && S <= kPpoNT && 4 * H <= kPpoNT,
                 "gradient CTA layout");
   const MlpLayout Lp = mlp_layout(D, H, A);
   const int64_t oW1 = POL ? Lp.w1 : Lp.v1, oB1 = POL ? Lp.b1 : Lp.c1;
@@ -351,8 +350,8 @@ __device__ __forceinline__ bool ppo_role(PpoSmem<D, H, A>& s, const PpoArgs& g, 
   const int tid = threadIdx.x;
   const float2 as = *g.advstat;
   // gather one slice (permuted sample order) of nv <= S samples:
-  // observations as float4 rows, per-sample scalars by threads 256..256+S;
-  // rows past nv are zero and marked invalid
+  // observations as float4 rows (one per thread), per-sample scalars by
+  // threads < S; rows past nv are zero and marked invalid
   auto gather = [&](int base, int nv) {
     constexpr int F4 = D / 4;
     if (tid < S * F4) {
@@ -366,8 +365,9 @@ __device__ __forceinline__ bool ppo_role(PpoSmem<D, H, A>& s, const PpoArgs& g, 
       s.xt[(4 * f + 1) * LD + si] = v.y;
       s.xt[(4 * f + 2) * LD + si] = v.z;
       s.xt[(4 * f + 3) * LD + si] = v.w;
-    } else if (tid >= 256 && tid < 256 + S) {
-      const int si = tid - 256;
+    }
+    if (tid < S) {
+      const int si = tid;
       const int ok = si < nv;
       s.valid[si] = ok;
       if (ok) {
@@ -415,8 +415,10 @@ __device__ __forceinline__ bool ppo_role(PpoSmem<D, H, A>& s, const PpoArgs& g, 
     __syncthreads();
     return false;
   }
-  // weight-gradient tiles live in registers only during their phase; each
-  // slice adds them into the CTA's shared-memory accumulators gw2 / gw1
+  // weight-gradient tiles live in registers only during their phase; the
+  // first slice writes them to this CTA's partial gradient row, later slices
+  // (when a CTA's share exceeds S samples) add to it
+  float* row = g.partial + (int64_t)c * g.PS;
   int nsl = 0;
   // head backward: thread (k = tid / 4, quarter q = tid % 4) owns row k of the
   // head weight gradient and of the layer-2 bias gradient over samples 4i + q
@@ -441,11 +443,11 @@ __device__ __forceinline__ bool ppo_role(PpoSmem<D, H, A>& s, const PpoArgs& g, 
     __syncthreads();
     dense_fwd_w<S, H, H, LD, kPpoRT, w2t_ld<H>()>(s.h1t, s.w2t, s.b2, s.h2t, SV);
     __syncthreads();
-    // head: thread (sample si = tid / 8, K-part q = tid % 8) sums k = q, q+8, ...
+    // head: job (sample si = j / 8, K-part q = j % 8) sums k = q, q+8, ...
     // for every action; the 8 parts (adjacent lanes) are shuffle-combined
-    {
-      static_assert(S * 8 == kPpoNT, "one head job per thread");
-      const int q = tid & 7, si = tid >> 3;
+    static_assert((S * 8) % kPpoNT == 0, "whole head jobs per thread");
+    for (int hj = tid; hj < S * 8; hj += kPpoNT) {
+      const int q = hj & 7, si = hj >> 3;
       if (si < SV) {  // warp-uniform: a warp covers 4 samples and SV is a multiple of 8
       float acc[NA];
 #pragma unroll
@@ -544,7 +546,7 @@ __device__ __forceinline__ bool ppo_role(PpoSmem<D, H, A>& s, const PpoArgs& g, 
     // layer-2 weight gradient
     {
       WGradAcc<H, H, kPpoNT> g2;
-      g2.template accumulate<S, LD>(s.h2t, s.h1t, SV, s.gw2, w2t_ld<H>(), nsl == 0);
+      g2.template accumulate<S, LD>(s.h2t, s.h1t, SV, row + oW2, H, nsl == 0);
     }
     __syncthreads();
     // back into layer 1 (in place over h1)
@@ -553,7 +555,7 @@ __device__ __forceinline__ bool ppo_role(PpoSmem<D, H, A>& s, const PpoArgs& g, 
     // layer-1 weight and bias gradients (the bias by the warps the tiles leave idle)
     {
       WGradAcc<H, D, kPpoNT> g1;
-      g1.template accumulate<S, LD>(s.h1t, s.xt, SV, s.gw1, D, nsl == 0);
+      g1.template accumulate<S, LD>(s.h1t, s.xt, SV, row + oW1, D, nsl == 0);
     }
     if (tid >= kPpoNT - H) {
       const int n = tid - (kPpoNT - H), lane = tid & 31;
@@ -566,22 +568,12 @@ __device__ __forceinline__ bool ppo_role(PpoSmem<D, H, A>& s, const PpoArgs& g, 
     }
     ++nsl;
   }
-  // partial gradient row of this CTA (its network's slice of the parameter vector)
-  float* row = g.partial + (int64_t)c * g.PS;
-  // the accumulated hidden-layer weight gradients, coalesced (zero if the
-  // CTA's slices held no sample)
-  __syncthreads();
-  {
-#pragma unroll 8
-    for (int u = 0; u < (H * H + kPpoNT - 1) / kPpoNT; ++u) {
-      const int i = tid + u * kPpoNT;
-      if (i < H * H) {
-        const float v = s.gw2[(i / H) * w2t_ld<H>() + i % H];
-        row[oW2 + i] = nsl ? v : 0.0f;
-      }
-    }
+  // the rest of the partial gradient row (the hidden-layer weight gradients
+  // are zero if the CTA's share held no sample)
+  if (nsl == 0) {
+    for (int i = tid; i < H * H; i += blockDim.x) row[oW2 + i] = 0.0f;
+    for (int i = tid; i < H * D; i += blockDim.x) row[oW1 + i] = 0.0f;
   }
-  for (int i = tid; i < H * D; i += blockDim.x) row[oW1 + i] = nsl ? s.gw1[i] : 0.0f;
 #pragma unroll
   for (int a = 0; a < NA; ++a) {
     g3[a] += __shfl_xor_sync(0xffffffffu, g3[a], 1);
@@ -1090,6 +1082,7 @@ static pe_status ppo_run(const pe_net& net, float* params, float* m, float* v, i
   }
   PE_CHECK_LAUNCH("ppo_image_kernel");
   using Smem = PpoSmem<D, H, A>;
+  static_assert(sizeof(Smem) + 1024 <= 232448, "gradient CTA shared memory");
   auto kern = ppo_grad_kernel<D, H, A>;
   const int bytes = (int)sizeof(Smem);
   PE_TRY_CUDA(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes));
