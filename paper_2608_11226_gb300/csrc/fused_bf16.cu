@@ -302,14 +302,16 @@ __global__ void __launch_bounds__(kFuThreads, 1) ppo_fused_pair_kernel(FusedArgs
         }
       }
     };
-    // head: the PPO loss per row (warps 0-3), dz to its tile image and to
-    // the slot's shared dz tile (zeros for a slot without a tile)
+    // head: the PPO loss per row, dz to its tile image and to the slot's
+    // shared dz tile (zeros for a slot without a tile); slot s by the four
+    // warps of column slice s (one per TMEM lane quadrant), so that the two
+    // slots' losses run side by side
     auto head_epi = [&](int sl, int k) {
-      if (warp >= 4) return;
+      if (slice != sl) return;
       if (k < my_tiles) {
         float v[16];
         tc::tmem_ld16(lane_base + (uint32_t)(sl * 256), v);
-        ppo_head_row(g.save.loss, g.value_net, g.A, s.b3, g.save.gather, tile_of(k), row, g.n, v, warp, s.dz[sl]);
+        ppo_head_row(g.save.loss, g.value_net, g.A, s.b3, g.save.gather, tile_of(k), row, g.n, v, quad, s.dz[sl]);
       } else {
         *reinterpret_cast<uint4*>(s.dz[sl] + row * 32) = make_uint4(0, 0, 0, 0);
         *reinterpret_cast<uint4*>(s.dz[sl] + row * 32 + 16) = make_uint4(0, 0, 0, 0);
