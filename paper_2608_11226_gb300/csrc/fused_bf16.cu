@@ -7,9 +7,8 @@
 // the backward data products of bwd_bf16.cu (the same bits).  h2 and dz
 // never leave the chip between the two halves: da2 overwrites h2 in place in
 // the tile's shared buffer, and dz goes to shared memory beside its tile
-// image.  The tile
-// images the weight-gradient kernel reads (x, h1, h2, dz, da2, da1) are
-// written as before.
+// image.  The tile images the weight-gradient kernel reads (x, h1, h2, dz,
+// da2, da1) are written as before.
 //
 // Two tiles are in flight per CTA (slots 0 and 1), each with its own 64 KB
 // activation buffer (X, then h1, h2, da2), its dz tile and half of TMEM
@@ -21,8 +20,10 @@
 // complete once per tile pair:
 //   epilogue -> issuer (16 arrivals): xin, h1in, h2in, dzin, d2in;
 //   issuer -> epilogue (tcgen05.commit): mma1, mma2, head, mdh2, mdh1.
-// The last epilogue of a tile reads h1 back from the h1 tile image that the
-// same thread wrote in the first one (the same rows and columns), from L2.
+// The loss epilogue of slot s runs on the four warps of column slice s (one
+// per TMEM lane quadrant), so the two slots' losses run side by side.  The
+// last epilogue of a tile reads h1 back from the h1 tile image that the same
+// thread wrote in the first one (the same rows and columns), from L2.
 #include <algorithm>
 
 #include "bf16_layout.cuh"
