@@ -26,6 +26,10 @@
 //   to its tile image.  A loader warp brings the tile's h2 image into the da2
 //   buffer with one bulk copy (da2 then overwrites it in place) and, after
 //   the dh1 MMAs, its h1 image, so the epilogues read h from shared memory.
+//   One launch covers both networks: the policy's tiles, then the value's,
+//   spread over the CTAs as one list (a CTA that crosses from one to the
+//   other reloads W3^T), which balances a tile count that is not a
+//   multiple of the SM count.
 // wgrad_kernel (split over samples): each CTA owns 128 output rows (one
 //   block of layer outputs o) of one network and one 256-column chunk, and
 //   accumulates over its share of the minibatch, 64 samples per stage:
@@ -93,14 +97,16 @@ struct BwdSmem {
 
 __device__ __forceinline__ void bw_compute_sync() { asm volatile("bar.sync 1, 512;" ::: "memory"); }
 
+// per network (policy, value): one launch covers both, their tiles spread
+// over the persistent CTAs together
 struct BwdArgs {
-  const uint8_t* img;   // backward weight image of the network
-  const uint8_t* dz;    // dz tile images (4 KB per tile)
-  const uint8_t* h1;    // h1 tile images
-  const uint8_t* h2;    // h2 tile images
-  uint8_t* da2;         // out: da2 tile images
-  uint8_t* da1;         // out: da1 tile images
-  int64_t n;            // valid samples
+  const uint8_t* img[2];  // backward weight image of each network
+  const uint8_t* dz[2];   // dz tile images (4 KB per tile)
+  const uint8_t* h1[2];   // h1 tile images
+  const uint8_t* h2[2];   // h2 tile images
+  uint8_t* da2[2];        // out: da2 tile images
+  uint8_t* da1[2];        // out: da1 tile images
+  int64_t n;              // valid samples (both networks)
   int32_t* err;
 };
 
@@ -130,19 +136,32 @@ __global__ void __launch_bounds__(kBwThreads, 1) bwd_data_kernel(BwdArgs g) {
   __syncthreads();
   tc::fence_after();
   const uint32_t tmem = s.tmem_base;
-  const int64_t tiles = (g.n + kBwRows - 1) / kBwRows;
-  const int my_tiles = (int)((tiles - blockIdx.x + gridDim.x - 1) / gridDim.x);
+  const int64_t tiles = (g.n + kBwRows - 1) / kBwRows;  // per network
+  const int my_tiles = (int)((2 * tiles - blockIdx.x + gridDim.x - 1) / gridDim.x);
+  // this CTA's k-th tile: its network (ni; the policy's tiles come first, so
+  // a CTA switches network at most once) and its tile index within it
+  auto tile_of = [&](int k, int& ni) -> int64_t {
+    const int64_t q = (int64_t)blockIdx.x + (int64_t)k * gridDim.x;
+    ni = q >= tiles ? 1 : 0;
+    return q - ni * tiles;
+  };
+  int ni0 = 0;
+  if (my_tiles > 0) (void)tile_of(0, ni0);
   if (tid == 0) {
     tc::mbar_expect_tx(&s.bar_w, (uint32_t)I::W3T);
-    tc::bulk_g2s(s.w3t, g.img, (uint32_t)I::W3T, &s.bar_w);
+    tc::bulk_g2s(s.w3t, ni0 ? g.img[1] : g.img[0], (uint32_t)I::W3T, &s.bar_w);
   }
   int last_issued = -1;  // producer: global index of its last issued stage
   int h_issued = 0;      // loader: h copies issued (the hin phases)
+  int cur = ni0;         // MMA issuer: network of the W3^T in shared memory
   if (warp == kBwCompute / 32) {
     // producer: the W2^T stages of every tile, in consumption order
     if (lane == 0) {
       int gs = 0;
       for (int t = 0; t < my_tiles; ++t) {
+        int ni;
+        (void)tile_of(t, ni);
+        const uint8_t* img = ni ? g.img[1] : g.img[0];
         for (int st = 0; st < I::STAGES; ++st, ++gs) {
           const int slot = gs & 1;
           if (gs >= 2 && !tc::mbar_wait(&s.empty[slot], ((gs - 2) >> 1) & 1)) {
@@ -151,7 +170,7 @@ __global__ void __launch_bounds__(kBwThreads, 1) bwd_data_kernel(BwdArgs g) {
             break;
           }
           tc::mbar_expect_tx(&s.full[slot], (uint32_t)kBwStage);
-          tc::bulk_g2s(s.ring[slot], g.img + I::W3T + (int64_t)st * kBwStage, (uint32_t)kBwStage, &s.full[slot]);
+          tc::bulk_g2s(s.ring[slot], img + I::W3T + (int64_t)st * kBwStage, (uint32_t)kBwStage, &s.full[slot]);
           last_issued = gs;
         }
       }
@@ -162,20 +181,23 @@ __global__ void __launch_bounds__(kBwThreads, 1) bwd_data_kernel(BwdArgs g) {
     // the dh1 MMAs have read da2
     if (lane == 0) {
       for (int t = 0; t < my_tiles; ++t) {
-        const int64_t tile = blockIdx.x + (int64_t)t * gridDim.x;
+        int ni;
+        const int64_t tile = tile_of(t, ni);
+        const uint8_t* h2 = ni ? g.h2[1] : g.h2[0];
+        const uint8_t* h1 = ni ? g.h1[1] : g.h1[0];
         if (t > 0 && !tc::mbar_wait(&s.bfree, (t - 1) & 1)) {
           atomicExch(&s.err, 1);
           break;
         }
         tc::mbar_expect_tx(&s.hin, (uint32_t)kTileBytes);
-        tc::bulk_g2s(s.da2, g.h2 + tile * (int64_t)kTileBytes, (uint32_t)kTileBytes, &s.hin);
+        tc::bulk_g2s(s.da2, h2 + tile * (int64_t)kTileBytes, (uint32_t)kTileBytes, &s.hin);
         ++h_issued;
         if (!tc::mbar_wait(&s.dh1, t & 1)) {
           atomicExch(&s.err, 1);
           break;
         }
         tc::mbar_expect_tx(&s.hin, (uint32_t)kTileBytes);
-        tc::bulk_g2s(s.da2, g.h1 + tile * (int64_t)kTileBytes, (uint32_t)kTileBytes, &s.hin);
+        tc::bulk_g2s(s.da2, h1 + tile * (int64_t)kTileBytes, (uint32_t)kTileBytes, &s.hin);
         ++h_issued;
       }
     }
@@ -211,35 +233,45 @@ __global__ void __launch_bounds__(kBwThreads, 1) bwd_data_kernel(BwdArgs g) {
         *reinterpret_cast<uint4*>(outt + o1) = hi;
       }
     };
-    const int tile0 = blockIdx.x;
     uint4 dzv = make_uint4(0, 0, 0, 0);
     if (tid < kBwRows * 2 && my_tiles > 0)
-      dzv = __ldg(reinterpret_cast<const uint4*>(g.dz + (int64_t)tile0 * (kBwRows * 32)) + tid);
+      dzv = __ldg(reinterpret_cast<const uint4*>((ni0 ? g.dz[1] : g.dz[0]) + tile_of(0, ni0) * (kBwRows * 32)) + tid);
     for (int t = 0; t < my_tiles; ++t) {
       // every compute thread takes the same decision (a named barrier with an OR)
       if (tc::bar_any(1, kBwCompute, s.err != 0)) break;
-      const int64_t tile = blockIdx.x + (int64_t)t * gridDim.x;
+      int ni, nn = 0;
+      const int64_t tile = tile_of(t, ni);
+      const int64_t ntile = t + 1 < my_tiles ? tile_of(t + 1, nn) : 0;
       const int nr = (int)(g.n - tile * kBwRows < kBwRows ? g.n - tile * kBwRows : kBwRows);
       const bool valid = row < nr;
       if (t + 1 < my_tiles) {
         // the next tile's h1/h2 images asked of L2 a tile ahead (128-byte lines)
-        const int64_t nxt = (tile + gridDim.x) * (int64_t)kTileBytes;
+        const uint8_t* h2n = (nn ? g.h2[1] : g.h2[0]) + ntile * (int64_t)kTileBytes;
+        const uint8_t* h1n = (nn ? g.h1[1] : g.h1[0]) + ntile * (int64_t)kTileBytes;
         for (int64_t off = (int64_t)tid * 128; off < (int64_t)kTileBytes; off += (int64_t)kBwCompute * 128) {
-          tc::prefetch_l2(g.h2 + nxt + off);
-          tc::prefetch_l2(g.h1 + nxt + off);
+          tc::prefetch_l2(h2n + off);
+          tc::prefetch_l2(h1n + off);
         }
       }
       // dz tile (4 KB, already in the SW32 layout), then the next tile's
       if (tid < kBwRows * 2) {
         reinterpret_cast<uint4*>(s.dz)[tid] = dzv;
         if (t + 1 < my_tiles)
-          dzv = __ldg(reinterpret_cast<const uint4*>(g.dz + (tile + gridDim.x) * (kBwRows * 32)) + tid);
+          dzv = __ldg(reinterpret_cast<const uint4*>((nn ? g.dz[1] : g.dz[0]) + ntile * (kBwRows * 32)) + tid);
       }
       tc::fence_async_smem();
       bw_compute_sync();
       // dh2 (TMEM cols 0..H) = dz W3: one K = 16 MMA per 256 columns
       if (issuer) {
         tc::fence_after();
+        if (ni != cur) {
+          // the value network's W3^T replaces the policy's (every MMA that
+          // read it completed before the previous tile's first epilogue)
+          cur = ni;
+          tc::mbar_expect_tx(&s.bar_w, (uint32_t)I::W3T);
+          tc::bulk_g2s(s.w3t, g.img[1], (uint32_t)I::W3T, &s.bar_w);
+          if (!tc::mbar_wait(&s.bar_w, 1)) atomicExch(&s.err, 1);
+        }
 #pragma unroll
         for (int h = 0; h < I::NH; ++h)
           tc::mma_bf16(tmem + h * 256, tc::desc_strided(dza, 16, 256, tc::kLayoutSW32),
@@ -251,7 +283,7 @@ __global__ void __launch_bounds__(kBwThreads, 1) bwd_data_kernel(BwdArgs g) {
       if (!tc::mbar_wait(&s.hin, 0)) atomicExch(&s.err, 1);  // h2 in the buffer
       tc::fence_after();
       // da2 = bf16(dh2 (1 - h2^2)): in place over h2 (the next A operand) and its tile image
-      epi(valid, g.da2 + tile * (int64_t)kTileBytes, true);
+      epi(valid, (ni ? g.da2[1] : g.da2[0]) + tile * (int64_t)kTileBytes, true);
       tc::fence_before();
       tc::fence_async_smem();
       bw_compute_sync();
@@ -279,7 +311,7 @@ __global__ void __launch_bounds__(kBwThreads, 1) bwd_data_kernel(BwdArgs g) {
       if (!tc::mbar_wait(&s.hin, 1)) atomicExch(&s.err, 1);  // h1 in the buffer
       tc::fence_after();
       // da1 = bf16(dh1 (1 - h1^2)) to its tile image
-      epi(valid, g.da1 + tile * (int64_t)kTileBytes, false);
+      epi(valid, (ni ? g.da1[1] : g.da1[0]) + tile * (int64_t)kTileBytes, false);
       tc::fence_before();
       tc::fence_async_smem();
       __syncwarp();
@@ -294,6 +326,7 @@ __global__ void __launch_bounds__(kBwThreads, 1) bwd_data_kernel(BwdArgs g) {
     (void)tc::mbar_wait(&s.full[last_issued & 1], (last_issued >> 1) & 1);
   if (s.err && warp == kBwCompute / 32 + 1 && lane == 0 && h_issued > 0)
     (void)tc::mbar_wait(&s.hin, (h_issued - 1) & 1);
+  if (s.err && tid == 32 && cur != ni0) (void)tc::mbar_wait(&s.bar_w, 1);
   if (tid == 0 && s.err && g.err) atomicExch(g.err, 1);
   __syncthreads();
   if (warp == 0) tc::tmem_dealloc(tmem, H);
@@ -597,12 +630,20 @@ static pe_status bwd_launch(const float* params, int A, uint8_t* const img[2], c
     auto kern = bwd_data_kernel<H>;
     const int bytes = (int)sizeof(BwdSmem<H>) + 1024;
     PE_TRY_CUDA(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes));
-    const int grid = (int)std::min<int64_t>(tiles, sms);
-    ProfScope ps(PE_PROF_PPO_GRAD, st);
+    const int grid = (int)std::min<int64_t>(2 * tiles, sms);
+    BwdArgs a;
     for (int ni = 0; ni < 2; ++ni) {
-      BwdArgs a{img[ni], dz[ni], h1[ni], h2[ni], da2[ni], da1[ni], n, err};
-      kern<<<grid, kBwThreads, bytes, st>>>(a);
+      a.img[ni] = img[ni];
+      a.dz[ni] = dz[ni];
+      a.h1[ni] = h1[ni];
+      a.h2[ni] = h2[ni];
+      a.da2[ni] = da2[ni];
+      a.da1[ni] = da1[ni];
     }
+    a.n = n;
+    a.err = err;
+    ProfScope ps(PE_PROF_PPO_GRAD, st);
+    kern<<<grid, kBwThreads, bytes, st>>>(a);
   }
   PE_CHECK_LAUNCH("bwd_data_kernel");
   {

@@ -14,7 +14,9 @@
 //     operand into shared memory in the swizzled layout;
 //   - 72B (mlp_bf16_pair_kernel): two tiles in flight per CTA, so that the
 //     epilogue of one overlaps the MMAs of the other; Stress
-//     (mlp_bf16_stream_kernel): one tile, its 592 KB of weights streamed.
+//     (mlp_bf16_stream_kernel): one tile at a time, its 592 KB of weights
+//     streamed, the layer-2 MMAs overlapping the epilogues per 256-column
+//     half.
 // Precision: bf16 observations, weights and hidden activations, fp32
 // accumulation, fp32 bias and tanh -- the quantisation points the oracle
 // emulates.
@@ -70,15 +72,35 @@ __global__ void weight_image_kernel(const float* __restrict__ params, int A, int
 // 32 KB stages, each the B operand of one (N-half, K-block) of a layer:
 //   layer 1: 2 stages (N-halves of W1, K=64), layer 2: 16 stages (2 N-halves x
 //   8 K-blocks of W2), head: 1 stage (W3, 16 rows x 8 K-blocks).
-// A producer warp (warp 16) issues cp.async.bulk for stage s into slot s%2
-// once the MMAs that read the slot's previous stage have completed (signalled
-// by tcgen05.commit on the slot's "empty" barrier); one thread of warp 1
-// waits for the slot's "full" barrier and issues the MMAs.  The 16 compute
-// warps synchronise with a named barrier so that the producer never waits
-// on them.
+// Warp roles: warps 0-15 run the epilogues, warp 16 issues cp.async.bulk for
+// stage s into slot s%2 once the MMAs that read the slot's previous stage
+// have completed (tcgen05.commit on the slot's "empty" barrier), warp 17
+// issues the MMAs.  A layer's 512 accumulator columns fill TMEM, so a tile
+// cannot overlap another tile; instead the epilogues hand over per 256-column
+// half, and the layer-2 MMAs run beside them:
+//   epilogue 1, half A (h1 columns 0-255) -> MMAs of layer-2 N-half 0 over
+//   K-blocks 0-3 run during epilogue 1, half B; once half B is written, the
+//   rest of N-half 0, then N-half 1;
+//   epilogue 2, half A (N-half 0) runs during the N-half 1 MMAs; its first
+//   results wait in registers until the N-half 1 MMAs have read h1's first
+//   four K-blocks, which h2 overwrites in place;
+//   the head accumulates in TMEM columns 256-271, so the next tile's layer-1
+//   N-half 0 can start while warps 0-3 still read the head, and warps 4-15
+//   write the next tile's X during that head epilogue.
+// The accumulation order of every accumulator is that of the serial kernel,
+// so the results are the same bits.  One launch may also cover two networks
+// over the same rows (the policy, then the value network of a PPO forward):
+// the tiles of both form one list spread over the persistent CTAs, which
+// balances a tile count that is not a multiple of the SM count.
 // ---------------------------------------------------------------------------
 constexpr int kComputeThreads = 512;
-constexpr int kStreamThreads = kComputeThreads + 32;
+constexpr int kStreamThreads = kComputeThreads + 64;
+
+// the second network of a two-network stream launch (img == NULL: one network)
+struct MlpSecond {
+  const uint8_t* img;
+  MlpSave save;
+};
 
 template <int D, int H>
 __global__ void weight_image_stream_kernel(const float* __restrict__ params, int A, int value_first,
@@ -110,217 +132,371 @@ __global__ void weight_image_stream_kernel(const float* __restrict__ params, int
 
 template <int D, int H>
 struct MlpStreamSmem {
-  alignas(1024) uint8_t act[kTcRows * H * 2];
+  alignas(1024) uint8_t act[kTcRows * H * 2];  // X (last K-block), then h1, then h2 (in place)
   alignas(1024) uint8_t ring[2][kStageBytes];
-  float b1[H], b2[H], b3[kHeadN];
-  uint64_t full[2], empty[2], bar_mma;
+  float headv[kTcRows][kHeadN];                // the previous tile's head accumulators (warps 0-3)
+  float b1[2][H], b2[2][H], b3[2][kHeadN];     // per network of the launch
+  uint64_t full[2], empty[2], fin;
+  // one completion per tile each: X written (warps 4-15), head read out of
+  // TMEM (warps 0-3), layer-1 N-halves done, h1 halves written, layer-2
+  // N-half 0 done, N-half 1 past K-block 3, N-half 1 done, h2 written, head done
+  uint64_t xin, hd, m1a, m1b, h1a, h1b, m2a, n1lo, m2b, h2in, mh;
   uint32_t tmem_base;
   int32_t err;
 };
-
-__device__ __forceinline__ void compute_sync() { asm volatile("bar.sync 1, 512;" ::: "memory"); }
 
 template <int D, int H>
 __global__ void __launch_bounds__(kStreamThreads, 1)
     mlp_bf16_stream_kernel(const uint8_t* __restrict__ img, const float* __restrict__ params, int A,
                            int value_net, const __nv_bfloat16* __restrict__ obs, int64_t n,
                            float* __restrict__ out, int out_stride, int nout, int32_t* __restrict__ err,
-                           MlpSave save) {
+                           MlpSave save, MlpSecond second) {
   using I = ImgS<D, H>;
+  static_assert(D == 64 && H == 512, "two 256-column halves per layer; X is one 128-byte K-block");
+  constexpr int NJ = H / 2 / 4 / 16;                 // 16-column chunks per warp and half
+  constexpr int KBH = H / 2 / 64;                    // K-blocks of h per half
+  constexpr int kXOff = (H / 64 - 1) * kTcRows * 128;  // X sits in the last K-block of the buffer
+  constexpr int XCPR = D / 8;                        // 16-byte observation chunks per row
+  constexpr int XCH = (kTcRows * XCPR + 383) / 384;  // per X-writing thread (warps 4-15)
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
   MlpStreamSmem<D, H>& s = *reinterpret_cast<MlpStreamSmem<D, H>*>(base);
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const MlpLayout Lp = mlp_layout(D, H, A);
+  const bool two = second.img != nullptr;
+  const int nnet = two ? 2 : 1;
   if (tid == 0) {
     s.err = 0;
     for (int i = 0; i < 2; ++i) {
       tc::mbar_init(&s.full[i], 1);
       tc::mbar_init(&s.empty[i], 1);
     }
-    tc::mbar_init(&s.bar_mma, 1);
+    tc::mbar_init(&s.fin, 1);
+    tc::mbar_init(&s.xin, 12);
+    tc::mbar_init(&s.hd, 4);
+    tc::mbar_init(&s.m1a, 1);
+    tc::mbar_init(&s.m1b, 1);
+    tc::mbar_init(&s.h1a, 16);
+    tc::mbar_init(&s.h1b, 16);
+    tc::mbar_init(&s.m2a, 1);
+    tc::mbar_init(&s.n1lo, 1);
+    tc::mbar_init(&s.m2b, 1);
+    tc::mbar_init(&s.h2in, 16);
+    tc::mbar_init(&s.mh, 1);
     tc::fence_mbar_init();
   }
   if (warp == 0) tc::tmem_alloc(&s.tmem_base, 512);
-  for (int i = tid; i < H; i += blockDim.x) {
-    s.b1[i] = __ldg(params + (value_net ? Lp.c1 : Lp.b1) + i);
-    s.b2[i] = __ldg(params + (value_net ? Lp.c2 : Lp.b2) + i);
+  for (int k = 0; k < nnet; ++k) {
+    const int vn = two ? k : value_net;
+    const int no = two ? (k ? 1 : A) : nout;
+    for (int i = tid; i < H; i += blockDim.x) {
+      s.b1[k][i] = __ldg(params + (vn ? Lp.c1 : Lp.b1) + i);
+      s.b2[k][i] = __ldg(params + (vn ? Lp.c2 : Lp.b2) + i);
+    }
+    if (tid < kHeadN) s.b3[k][tid] = tid < no ? __ldg(params + (vn ? Lp.c3 : Lp.b3) + tid) : 0.0f;
   }
-  if (tid < kHeadN) s.b3[tid] = tid < nout ? __ldg(params + (value_net ? Lp.c3 : Lp.b3) + tid) : 0.0f;
   tc::fence_before();
   __syncthreads();
   tc::fence_after();
   const uint32_t tmem = s.tmem_base;
-  const int64_t tiles = (n + kTcRows - 1) / kTcRows;
-  const int my_tiles = (int)((tiles - blockIdx.x + gridDim.x - 1) / gridDim.x);
-
+  const int64_t tiles = (n + kTcRows - 1) / kTcRows;  // per network
+  const int my_tiles = (int)((tiles * nnet - blockIdx.x + gridDim.x - 1) / gridDim.x);
+  // this CTA's k-th tile: its network (ni) and its tile index within that network
+  auto tile_of = [&](int k, int& ni) -> int64_t {
+    const int64_t g = (int64_t)blockIdx.x + (int64_t)k * gridDim.x;
+    ni = g >= tiles ? 1 : 0;
+    return g - ni * tiles;
+  };
+  // a bounded wait that is skipped once the CTA has an error
+  auto wt = [&](uint64_t* b, uint32_t par) -> bool {
+    if (*reinterpret_cast<volatile int32_t*>(&s.err)) return false;
+    if (tc::mbar_wait(b, par)) return true;
+    atomicExch(&s.err, 1);
+    return false;
+  };
   int last_issued = -1;  // producer: global index of its last issued stage
-  if (warp == kComputeThreads / 32) {
+  if (warp == 16) {
     // producer: every stage of every tile of this CTA, in consumption order
     if (lane == 0) {
       int gs = 0;
-      for (int t = 0; t < my_tiles; ++t) {
-        for (int st = 0; st < kStreamStages; ++st, ++gs) {
+      bool ok = true;
+      for (int t = 0; t < my_tiles && ok; ++t) {
+        int ni;
+        (void)tile_of(t, ni);
+        const uint8_t* timg = ni ? second.img : img;
+        for (int st = 0; st < kStreamStages && ok; ++st) {
           const int slot = gs & 1;
-          if (gs >= 2 && !tc::mbar_wait(&s.empty[slot], ((gs - 2) >> 1) & 1)) {
-            atomicExch(&s.err, 1);
-            t = my_tiles;
+          if (gs >= 2 && !wt(&s.empty[slot], ((gs - 2) >> 1) & 1)) {
+            ok = false;
             break;
           }
           tc::mbar_expect_tx(&s.full[slot], (uint32_t)I::stage_bytes(st));
-          tc::bulk_g2s(s.ring[slot], img + I::stage_off(st), (uint32_t)I::stage_bytes(st), &s.full[slot]);
-          last_issued = gs;
+          tc::bulk_g2s(s.ring[slot], timg + I::stage_off(st), (uint32_t)I::stage_bytes(st), &s.full[slot]);
+          last_issued = gs++;
         }
       }
+    }
+  } else if (warp == 17) {
+    // MMA issuer
+    if (lane == 0) {
+      const uint32_t xa = tc::smem_u32(s.act);
+      constexpr uint32_t kIdN = tc::idesc_bf16(kTcRows, 256);
+      constexpr uint32_t kIdH = tc::idesc_bf16(kTcRows, kHeadN);
+      int gs = 0;
+      auto stage_in = [&]() -> uint32_t {
+        const int slot = gs & 1;
+        (void)wt(&s.full[slot], (gs >> 1) & 1);
+        tc::fence_after();
+        return tc::smem_u32(s.ring[slot]);
+      };
+      auto stage_out = [&]() {
+        tc::mma_commit(&s.empty[gs & 1]);
+        ++gs;
+      };
+      // layer 2: K-blocks [k0, k1) of h1 into N-half h (TMEM columns 256 h ..)
+      auto layer2 = [&](int h, int k0, int k1) {
+#pragma unroll 1
+        for (int kb = k0; kb < k1; ++kb) {
+          const uint32_t ra = stage_in();
+#pragma unroll
+          for (int kk = 0; kk < 4; ++kk)
+            tc::mma_bf16(tmem + h * 256, tc::desc_kmajor(xa + kb * kTcRows * 128 + kk * 32, 1024, tc::kLayoutSW128),
+                         tc::desc_kmajor(ra + kk * 32, 1024, tc::kLayoutSW128), kIdN, (kb | kk) != 0);
+          stage_out();
+        }
+      };
+      for (int t = 0; t < my_tiles; ++t) {
+        const uint32_t par = t & 1;
+        (void)wt(&s.xin, par);
+        tc::fence_after();
+        // layer 1, N-half h; N-half 1 overwrites the columns of the previous tile's head
+#pragma unroll 1
+        for (int h = 0; h < 2; ++h) {
+          if (h == 1 && t > 0) {
+            (void)wt(&s.hd, par ^ 1);
+            tc::fence_after();
+          }
+          const uint32_t ra = stage_in();
+#pragma unroll
+          for (int kk = 0; kk < D / 16; ++kk)
+            tc::mma_bf16(tmem + h * 256, tc::desc_kmajor(xa + kXOff + kk * 32, 1024, tc::kLayoutSW128),
+                         tc::desc_kmajor(ra + kk * 32, 1024, tc::kLayoutSW128), kIdN, kk > 0);
+          stage_out();
+          tc::mma_commit(h ? &s.m1b : &s.m1a);
+        }
+        (void)wt(&s.h1a, par);
+        tc::fence_after();
+        layer2(0, 0, KBH);
+        (void)wt(&s.h1b, par);
+        tc::fence_after();
+        layer2(0, KBH, 2 * KBH);
+        tc::mma_commit(&s.m2a);
+        layer2(1, 0, KBH);
+        tc::mma_commit(&s.n1lo);
+        layer2(1, KBH, 2 * KBH);
+        tc::mma_commit(&s.m2b);
+        // head: TMEM columns 256 .. 271 = H2 W3^T (one 16 KB stage)
+        (void)wt(&s.h2in, par);
+        tc::fence_after();
+        const uint32_t ra = stage_in();
+#pragma unroll 1
+        for (int kb = 0; kb < H / 64; ++kb)
+#pragma unroll
+          for (int kk = 0; kk < 4; ++kk)
+            tc::mma_bf16(tmem + 256, tc::desc_kmajor(xa + kb * kTcRows * 128 + kk * 32, 1024, tc::kLayoutSW128),
+                         tc::desc_kmajor(ra + kb * kHeadN * 128 + kk * 32, 1024, tc::kLayoutSW128), kIdH,
+                         (kb | kk) != 0);
+        stage_out();
+        tc::mma_commit(&s.mh);
+      }
+      // every MMA of this CTA completes before TMEM is released
+      tc::mma_commit(&s.fin);
+      if (!tc::mbar_wait(&s.fin, 0)) atomicExch(&s.err, 1);
     }
   } else {
-    const bool issuer = (tid == 32);
-    const uint32_t xa = tc::smem_u32(s.act);
-    const uint32_t r0a = tc::smem_u32(s.ring[0]), r1a = tc::smem_u32(s.ring[1]);
-    constexpr uint32_t kIdN = tc::idesc_bf16(kTcRows, 256);
-    constexpr uint32_t kIdH = tc::idesc_bf16(kTcRows, kHeadN);
-    uint32_t phase = 0;
-    int gs = 0;  // global stage counter of the issuing thread
+    // epilogue warps: four TMEM lane quadrants x four column slices
     const int quad = warp & 3, slice = warp >> 2, row = quad * 32 + lane;
     const uint32_t lane_addr = tmem + ((uint32_t)(quad * 32) << 16);
+    const int xt = tid - 128;  // X-writing thread index (warps 4-15)
+    uint4 xv[XCH];
+    auto fetch_x = [&](int k) {
+      int ni = 0;
+      const int64_t tl = k < my_tiles ? tile_of(k, ni) : 0;
+      const uint32_t* gather = ni ? second.save.gather : save.gather;
+#pragma unroll
+      for (int q = 0; q < XCH; ++q) {
+        const int i = xt + q * 384, r = i / XCPR, c = i % XCPR;
+        const int64_t rr = tl * kTcRows + r;
+        xv[q] = make_uint4(0, 0, 0, 0);
+        if (k < my_tiles && i < kTcRows * XCPR && rr < n) {
+          const int64_t src = gather ? (int64_t)__ldg(gather + rr) : rr;
+          xv[q] = __ldg(reinterpret_cast<const uint4*>(obs + src * D) + c);
+        }
+      }
+    };
+    auto handover = [&](uint64_t* bar) {
+      tc::fence_async_smem();
+      tc::fence_before();
+      __syncwarp();
+      if (lane == 0) asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(tc::smem_u32(bar)) : "memory");
+    };
+    // columns c .. c + 15 of this thread's row: tanh(acc + bias), packed bf16
+    auto chunk = [&](int c, const float* bias, uint32_t (&pk)[8]) {
+      float v[16];
+      tc::tmem_ld16(lane_addr + (uint32_t)c, v);
+      tc::tanh16_bf16(v, bias + c, pk);
+    };
+    // ... into the activation buffer (the next A operand) and the tile image g
+    auto put = [&](int c, const uint32_t (&pk)[8], uint8_t* g) {
+      const uint32_t o0 = tc::swz_offset<128>(row, c, kTcRows), o1 = tc::swz_offset<128>(row, c + 8, kTcRows);
+      const uint4 lo = make_uint4(pk[0], pk[1], pk[2], pk[3]), hi = make_uint4(pk[4], pk[5], pk[6], pk[7]);
+      *reinterpret_cast<uint4*>(s.act + o0) = lo;
+      *reinterpret_cast<uint4*>(s.act + o1) = hi;
+      if (g) {
+        *reinterpret_cast<uint4*>(g + o0) = lo;
+        *reinterpret_cast<uint4*>(g + o1) = hi;
+      }
+    };
+    // head of this CTA's k-th tile from its 16 accumulators (warps 0-3, one row per thread)
+    auto head_out = [&](int k, const float (&v)[16]) {
+      int ni;
+      const int64_t tl = tile_of(k, ni);
+      if (ni) {
+        ppo_head_row(second.save.loss, 1, A, s.b3[1], second.save.gather, tl, row, n, v, warp);
+      } else if (save.loss.dz) {
+        ppo_head_row(save.loss, value_net, A, s.b3[0], save.gather, tl, row, n, v, warp);
+      } else if (tl * kTcRows + row < n) {
+        float* o = out + (tl * kTcRows + row) * out_stride;
+#pragma unroll
+        for (int j = 0; j < kHeadN; ++j)
+          if (j < nout) o[j] = v[j] + s.b3[0][j];
+      }
+    };
+    if (warp >= 4) fetch_x(0);
     for (int t = 0; t < my_tiles; ++t) {
-      // every compute thread takes the same decision (a named barrier with an OR)
-      if (tc::bar_any(1, kComputeThreads, s.err != 0)) break;
-      const int64_t tile = blockIdx.x + (int64_t)t * gridDim.x;
-      const int64_t rbase = tile * kTcRows;
-      const int nr = (int)(n - rbase < kTcRows ? n - rbase : kTcRows);
-      // observation tile (D = 64 bf16 = one 128-byte K-block per row)
-      for (int i = tid; i < kTcRows * (D / 8); i += kComputeThreads) {
-        const int r = i / (D / 8), c = i % (D / 8);
-        uint4 v = make_uint4(0, 0, 0, 0);
-        if (r < nr) {
-          const int64_t src = save.gather ? (int64_t)__ldg(save.gather + rbase + r) : rbase + r;
-          v = __ldg(reinterpret_cast<const uint4*>(obs + src * D) + c);
-        }
-        const uint32_t off = tc::swz_offset<128>(r, c * 8, kTcRows);
-        *reinterpret_cast<uint4*>(s.act + off) = v;
-        if (save.x)
-          *reinterpret_cast<uint4*>(reinterpret_cast<uint8_t*>(save.x) + tile * (int64_t)(kTcRows * D * 2) + off) = v;
-      }
-      tc::fence_async_smem();
-      compute_sync();
-      // one weight stage: wait for its slot, issue its MMAs, release the slot
-      auto run_stage = [&](int stg, auto&& body) {
-        const int slot = gs & 1;
-        if (!tc::mbar_wait(&s.full[slot], (gs >> 1) & 1)) atomicExch(&s.err, 1);
-        tc::fence_after();
-        body(slot ? r1a : r0a);
-        tc::mma_commit(&s.empty[slot]);
-        ++gs;
-        (void)stg;
-      };
-      // layer 1: D1 (TMEM cols 0..512) = X W1^T, two N-halves
-      if (issuer) {
-        for (int h = 0; h < 2; ++h)
-          run_stage(h, [&](uint32_t ra) {
-#pragma unroll
-            for (int kk = 0; kk < D / 16; ++kk)
-              tc::mma_bf16(tmem + h * 256, tc::desc_kmajor(xa + kk * 32, 1024, tc::kLayoutSW128),
-                           tc::desc_kmajor(ra + kk * 32, 1024, tc::kLayoutSW128), kIdN, kk > 0);
-          });
-        tc::mma_commit(&s.bar_mma);
-      }
-      if (!tc::mbar_wait(&s.bar_mma, phase)) atomicExch(&s.err, 1);
-      phase ^= 1;
-      tc::fence_after();
-      // epilogue 1: 128 columns per warp, chunk by chunk
-#pragma unroll 1
-      for (int j = 0; j < H / 4 / 16; ++j) {
-        const int c = slice * (H / 4) + j * 16;
-        float v[16];
-        tc::tmem_ld16(lane_addr + (uint32_t)c, v);
-        uint32_t p[8];
-        tc::tanh16_bf16(v, s.b1 + c, p);
-        const uint32_t o0 = tc::swz_offset<128>(row, c, kTcRows), o1 = tc::swz_offset<128>(row, c + 8, kTcRows);
-        *reinterpret_cast<uint4*>(s.act + o0) = make_uint4(p[0], p[1], p[2], p[3]);
-        *reinterpret_cast<uint4*>(s.act + o1) = make_uint4(p[4], p[5], p[6], p[7]);
-        if (save.h1) {
-          uint8_t* g = reinterpret_cast<uint8_t*>(save.h1) + tile * (int64_t)(kTcRows * H * 2);
-          *reinterpret_cast<uint4*>(g + o0) = make_uint4(p[0], p[1], p[2], p[3]);
-          *reinterpret_cast<uint4*>(g + o1) = make_uint4(p[4], p[5], p[6], p[7]);
-        }
-      }
-      tc::fence_before();
-      tc::fence_async_smem();
-      compute_sync();
-      // layer 2: D2 (TMEM cols 0..512) = H1 W2^T, 2 N-halves x 8 K-blocks
-      if (issuer) {
-        tc::fence_after();
-        for (int h = 0; h < 2; ++h)
-          for (int kb = 0; kb < H / 64; ++kb)
-            run_stage(2 + h * 8 + kb, [&](uint32_t ra) {
-#pragma unroll
-              for (int kk = 0; kk < 4; ++kk)
-                tc::mma_bf16(tmem + h * 256, tc::desc_kmajor(xa + kb * kTcRows * 128 + kk * 32, 1024, tc::kLayoutSW128),
-                             tc::desc_kmajor(ra + kk * 32, 1024, tc::kLayoutSW128), kIdN, (kb | kk) != 0);
-            });
-        tc::mma_commit(&s.bar_mma);
-      }
-      if (!tc::mbar_wait(&s.bar_mma, phase)) atomicExch(&s.err, 1);
-      phase ^= 1;
-      tc::fence_after();
-#pragma unroll 1
-      for (int j = 0; j < H / 4 / 16; ++j) {
-        const int c = slice * (H / 4) + j * 16;
-        float v[16];
-        tc::tmem_ld16(lane_addr + (uint32_t)c, v);
-        uint32_t p[8];
-        tc::tanh16_bf16(v, s.b2 + c, p);
-        const uint32_t o0 = tc::swz_offset<128>(row, c, kTcRows), o1 = tc::swz_offset<128>(row, c + 8, kTcRows);
-        *reinterpret_cast<uint4*>(s.act + o0) = make_uint4(p[0], p[1], p[2], p[3]);
-        *reinterpret_cast<uint4*>(s.act + o1) = make_uint4(p[4], p[5], p[6], p[7]);
-        if (save.h2) {
-          uint8_t* g = reinterpret_cast<uint8_t*>(save.h2) + tile * (int64_t)(kTcRows * H * 2);
-          *reinterpret_cast<uint4*>(g + o0) = make_uint4(p[0], p[1], p[2], p[3]);
-          *reinterpret_cast<uint4*>(g + o1) = make_uint4(p[4], p[5], p[6], p[7]);
-        }
-      }
-      tc::fence_before();
-      tc::fence_async_smem();
-      compute_sync();
-      // head: D3 (TMEM cols 0..16) = H2 W3^T (one 16 KB stage)
-      if (issuer) {
-        tc::fence_after();
-        run_stage(18, [&](uint32_t ra) {
-#pragma unroll 1
-          for (int kb = 0; kb < H / 64; ++kb)
-#pragma unroll
-            for (int kk = 0; kk < 4; ++kk)
-              tc::mma_bf16(tmem, tc::desc_kmajor(xa + kb * kTcRows * 128 + kk * 32, 1024, tc::kLayoutSW128),
-                           tc::desc_kmajor(ra + kb * kHeadN * 128 + kk * 32, 1024, tc::kLayoutSW128), kIdH,
-                           (kb | kk) != 0);
-        });
-        tc::mma_commit(&s.bar_mma);
-      }
-      if (!tc::mbar_wait(&s.bar_mma, phase)) atomicExch(&s.err, 1);
-      phase ^= 1;
+      const uint32_t par = t & 1;
+      int ni;
+      const int64_t tile = tile_of(t, ni);
+      __nv_bfloat16* const sx = ni ? second.save.x : save.x;
+      __nv_bfloat16* const sh1 = ni ? second.save.h1 : save.h1;
+      __nv_bfloat16* const sh2 = ni ? second.save.h2 : save.h2;
+      uint8_t* const gh1 = sh1 ? reinterpret_cast<uint8_t*>(sh1) + tile * (int64_t)(kTcRows * H * 2) : nullptr;
+      uint8_t* const gh2 = sh2 ? reinterpret_cast<uint8_t*>(sh2) + tile * (int64_t)(kTcRows * H * 2) : nullptr;
+      const float* const b1 = s.b1[ni];
+      const float* const b2 = s.b2[ni];
+      if (t > 0) (void)wt(&s.mh, par ^ 1);  // the previous tile's head is done
       tc::fence_after();
       if (warp < 4) {
-        float v[16];
-        tc::tmem_ld16(lane_addr, v);
-        if (save.loss.dz) {
-          ppo_head_row(save.loss, value_net, A, s.b3, save.gather, tile, row, n, v, warp);
-        } else if (row < nr) {
-          float* o = out + (rbase + row) * out_stride;
+        // its accumulators out of TMEM (the loss comes later, while the
+        // layer-2 MMAs run), so that layer 1 may take the columns
+        if (t > 0) {
+          float v[16];
+          tc::tmem_ld16(lane_addr + 256u, v);
 #pragma unroll
-          for (int j = 0; j < kHeadN; ++j)
-            if (j < nout) o[j] = v[j] + s.b3[j];
+          for (int j = 0; j < kHeadN; j += 4)
+            *reinterpret_cast<float4*>(&s.headv[row][j]) = make_float4(v[j], v[j + 1], v[j + 2], v[j + 3]);
+          tc::fence_before();
+          __syncwarp();
+          if (lane == 0) asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(tc::smem_u32(&s.hd)) : "memory");
+        }
+      } else {
+        // this tile's X (the previous tile's head MMA has read h2)
+#pragma unroll
+        for (int q = 0; q < XCH; ++q) {
+          const int i = xt + q * 384;
+          if (i < kTcRows * XCPR) {
+            const int r = i / XCPR, c = i % XCPR;
+            const uint32_t off = tc::swz_offset<128>(r, c * 8, kTcRows);
+            *reinterpret_cast<uint4*>(s.act + kXOff + off) = xv[q];
+            if (sx)
+              *reinterpret_cast<uint4*>(reinterpret_cast<uint8_t*>(sx) + tile * (int64_t)(kTcRows * D * 2) + off) =
+                  xv[q];
+          }
+        }
+        handover(&s.xin);
+      }
+      // epilogue 1, half A (h1 K-blocks 0-3), then half B (K-blocks 4-7, the
+      // last of which held X: layer-1 N-half 1 is done by then)
+      (void)wt(&s.m1a, par);
+      tc::fence_after();
+#pragma unroll 1
+      for (int j = 0; j < NJ; ++j) {
+        const int c = slice * (H / 8) + j * 16;
+        uint32_t pk[8];
+        chunk(c, b1, pk);
+        put(c, pk, gh1);
+      }
+      handover(&s.h1a);
+      (void)wt(&s.m1b, par);
+      tc::fence_after();
+#pragma unroll 1
+      for (int j = 0; j < NJ; ++j) {
+        const int c = H / 2 + slice * (H / 8) + j * 16;
+        uint32_t pk[8];
+        chunk(c, b1, pk);
+        put(c, pk, gh1);
+      }
+      handover(&s.h1b);
+      // the previous tile's head epilogue, while the rest of layer-2 N-half 0 runs
+      if (warp < 4 && t > 0) {
+        float v[16];
+#pragma unroll
+        for (int j = 0; j < kHeadN; j += 4) {
+          const float4 q = *reinterpret_cast<const float4*>(&s.headv[row][j]);
+          v[j] = q.x, v[j + 1] = q.y, v[j + 2] = q.z, v[j + 3] = q.w;
+        }
+        head_out(t - 1, v);
+      }
+      // epilogue 2, half A: h2 overwrites h1's K-blocks 0-3 only after the
+      // N-half 1 MMAs have read them; the first two chunks wait in registers
+      (void)wt(&s.m2a, par);
+      tc::fence_after();
+      {
+        const int c0 = slice * (H / 8);
+        uint32_t p0[8], p1[8];
+        chunk(c0, b2, p0);
+        chunk(c0 + 16, b2, p1);
+        (void)wt(&s.n1lo, par);
+        tc::fence_after();
+        put(c0, p0, gh2);
+        put(c0 + 16, p1, gh2);
+#pragma unroll 1
+        for (int j = 2; j < NJ; ++j) {
+          const int c = c0 + j * 16;
+          uint32_t pk[8];
+          chunk(c, b2, pk);
+          put(c, pk, gh2);
         }
       }
-      tc::fence_before();
-      compute_sync();
+      (void)wt(&s.m2b, par);
+      tc::fence_after();
+#pragma unroll 1
+      for (int j = 0; j < NJ; ++j) {
+        const int c = H / 2 + slice * (H / 8) + j * 16;
+        uint32_t pk[8];
+        chunk(c, b2, pk);
+        put(c, pk, gh2);
+      }
+      handover(&s.h2in);
+      // the next tile's observation rows, fetched while its X slot waits for this tile's head MMA
+      if (warp >= 4) fetch_x(t + 1);
+    }
+    // the last tile's head
+    if (warp < 4 && my_tiles > 0) {
+      (void)wt(&s.mh, (my_tiles - 1) & 1);
+      tc::fence_after();
+      float v[16];
+      tc::tmem_ld16(lane_addr + 256u, v);
+      head_out(my_tiles - 1, v);
     }
   }
+  tc::fence_before();
   __syncthreads();
-  // on an error, the producer waits (bounded) for its last copy before the
-  // CTA leaves, so that no bulk copy into this CTA's shared memory is in flight
-  if (s.err && warp == kComputeThreads / 32 && lane == 0 && last_issued >= 0)
-    (void)tc::mbar_wait(&s.full[last_issued & 1], (last_issued >> 1) & 1);
+  // on an error, the producer waits (bounded) for the copies it may still
+  // have in flight (at most one per ring slot) before the CTA leaves
+  if (s.err && warp == 16 && lane == 0)
+    for (int q = last_issued - 1; q <= last_issued; ++q)
+      if (q >= 0) (void)tc::mbar_wait(&s.full[q & 1], (q >> 1) & 1);
   if (tid == 0 && s.err) {
     atomicExch(&g_tc_error, 1);
     if (err) atomicExch(err, 1);
@@ -703,21 +879,28 @@ static int64_t bf16_ws_bytes(int64_t E) {
 template <int D, int H>
 static pe_status launch_mlp(const uint8_t* img, const float* params, int A, int value_net,
                             const void* obs, int64_t n, float* out, int out_stride, int nout,
-                            int32_t* err, cudaStream_t st, int prof_kind, MlpSave save = MlpSave{}) {
+                            int32_t* err, cudaStream_t st, int prof_kind, MlpSave save = MlpSave{},
+                            MlpSecond second = MlpSecond{}) {
   if (n <= 0) return PE_OK;
   int dev = 0, sms = 0;
   PE_TRY_CUDA(cudaGetDevice(&dev));
   PE_TRY_CUDA(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
   const int64_t tiles = (n + kTcRows - 1) / kTcRows;
-  const int grid = (int)(tiles < sms ? tiles : sms);
   const __nv_bfloat16* o = reinterpret_cast<const __nv_bfloat16*>(obs);
   if constexpr (NetKind<D, H>::kStream) {
+    // a two-network launch is the PPO forward: policy first, the loss head on both
+    if (second.img && (value_net != 0 || !save.loss.dz || !second.save.loss.dz))
+      return fail(PE_EINVAL, "a two-network forward runs the policy, then the value network, with the loss head");
+    const int64_t all = second.img ? 2 * tiles : tiles;
+    const int grid = (int)(all < sms ? all : sms);
     auto kern = mlp_bf16_stream_kernel<D, H>;
     const int bytes = (int)sizeof(MlpStreamSmem<D, H>) + 1024;
     PE_TRY_CUDA(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes));
     ProfScope ps(prof_kind, st);
-    kern<<<grid, kStreamThreads, bytes, st>>>(img, params, A, value_net, o, n, out, out_stride, nout, err, save);
+    kern<<<grid, kStreamThreads, bytes, st>>>(img, params, A, value_net, o, n, out, out_stride, nout, err, save,
+                                              second);
   } else {
+    if (second.img) return fail(PE_EINVAL, "two-network forward launches are for the streamed network");
     auto kern = mlp_bf16_pair_kernel<D, H>;
     const int bytes = (int)sizeof(MlpPairSmem<D, H>) + 1024;
     PE_TRY_CUDA(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes));
@@ -891,20 +1074,27 @@ pe_status bf16_make_images(const pe_net& net, const float* params, uint8_t* two_
   return fail(PE_EINVAL, "unsupported bf16 network");
 }
 
-pe_status bf16_forward_loss(const pe_net& net, const uint8_t* img, const float* params, int value_net,
-                            const void* obs, const uint32_t* gather, int64_t n, const PpoHead& loss,
-                            __nv_bfloat16* x, __nv_bfloat16* h1, __nv_bfloat16* h2, int32_t* err,
-                            cudaStream_t st) {
-  const MlpSave sv{gather, x, h1, h2, loss};
+// forward of both networks over the same gathered minibatch rows with the PPO
+// loss in the head: the policy (image at img, loss lp, saving x, h[0], h[1])
+// and the value network (image at img + bf16_image_bytes, loss lv, saving
+// h[2], h[3]).  The streamed network runs both in one launch, its tiles
+// spread over the persistent CTAs together.
+pe_status bf16_forward_loss(const pe_net& net, const uint8_t* img, const float* params, const void* obs,
+                            const uint32_t* gather, int64_t n, const PpoHead& lp, const PpoHead& lv,
+                            __nv_bfloat16* x, __nv_bfloat16* const h[4], int32_t* err, cudaStream_t st) {
+  const MlpSave sp{gather, x, h[0], h[1], lp};
+  const MlpSave sv{gather, nullptr, h[2], h[3], lv};
   float* out = nullptr;
-  const int out_stride = 0;
-  const int nout = value_net ? 1 : net.n_actions;
-  if (net.obs_dim == 32 && net.hidden == 256)
-    return launch_mlp<32, 256>(img, params, net.n_actions, value_net, obs, n, out, out_stride, nout, err, st,
-                               PE_PROF_PPO_GRAD, sv);
+  if (net.obs_dim == 32 && net.hidden == 256) {
+    const uint8_t* img_v = img + NetKind<32, 256>::kImgPad;
+    pe_status s = launch_mlp<32, 256>(img, params, net.n_actions, 0, obs, n, out, 0, net.n_actions, err, st,
+                                      PE_PROF_PPO_GRAD, sp);
+    if (s != PE_OK) return s;
+    return launch_mlp<32, 256>(img_v, params, net.n_actions, 1, obs, n, out, 0, 1, err, st, PE_PROF_PPO_GRAD, sv);
+  }
   if (net.obs_dim == 64 && net.hidden == 512)
-    return launch_mlp<64, 512>(img, params, net.n_actions, value_net, obs, n, out, out_stride, nout, err, st,
-                               PE_PROF_PPO_GRAD, sv);
+    return launch_mlp<64, 512>(img, params, net.n_actions, 0, obs, n, out, 0, net.n_actions, err, st,
+                               PE_PROF_PPO_GRAD, sp, MlpSecond{img + NetKind<64, 512>::kImgPad, sv});
   return fail(PE_EINVAL, "unsupported bf16 network");
 }
 

@@ -36,10 +36,9 @@ namespace pe {
 // defined in mlp_bf16.cu / ppo_f32.cu / bwd_bf16.cu
 int64_t bf16_image_bytes(const pe_net& net);
 pe_status bf16_make_images(const pe_net& net, const float* params, uint8_t* two_images, cudaStream_t st);
-pe_status bf16_forward_loss(const pe_net& net, const uint8_t* img, const float* params, int value_net,
-                            const void* obs, const uint32_t* gather, int64_t n, const PpoHead& loss,
-                            __nv_bfloat16* x, __nv_bfloat16* h1, __nv_bfloat16* h2, int32_t* err,
-                            cudaStream_t st);
+pe_status bf16_forward_loss(const pe_net& net, const uint8_t* img, const float* params, const void* obs,
+                            const uint32_t* gather, int64_t n, const PpoHead& lp, const PpoHead& lv,
+                            __nv_bfloat16* x, __nv_bfloat16* const h[4], int32_t* err, cudaStream_t st);
 pe_status launch_advstats(const float* adv, int64_t N, int M, int nmb, int epochs, uint64_t seed,
                           uint32_t iteration, float2* out, cudaStream_t st);
 int64_t bwd_image_bytes(int H);
@@ -296,11 +295,11 @@ pe_status ppo_update_bf16(const pe_net& net, float* params, float* m, float* v, 
         s = bf16_fused_fwd_bwd(net, img + pl.img, bimg[1], params, 1, obs, idx, cnt, lh, nullptr, h[2], h[3], da2[1],
                                da1[1], err, st);
       } else {
+        // Stress: forward and loss of both networks in one launch
+        PpoHead lv = lh;
         lh.dz = dz[0];
-        s = bf16_forward_loss(net, img, params, 0, obs, idx, cnt, lh, x, h[0], h[1], err, st);
-        if (s != PE_OK) return s;
-        lh.dz = dz[1];
-        s = bf16_forward_loss(net, img + pl.img, params, 1, obs, idx, cnt, lh, nullptr, h[2], h[3], err, st);
+        lv.dz = dz[1];
+        s = bf16_forward_loss(net, img, params, obs, idx, cnt, lh, lv, x, h, err, st);
       }
       if (s != PE_OK) return s;
       const int nlb = rows / kTile * 4;

@@ -756,8 +756,10 @@ def test_ppo_bf16_several_tiles_per_cta(preset, E, T):
     """One minibatch large enough that the persistent kernels take more than
     one tile (pair) per CTA: 72B 40,960 samples = 320 tiles over 152 CTAs
     (the first 16 run two tile pairs, the second half empty); Stress 19,520
-    samples = 153 tiles (the first CTA runs two).  Adam's first moment after
-    one step is 0.1 x the clipped gradient."""
+    samples = 153 tiles per network, whose forward and backward-data
+    launches spread the 306 tiles of both networks over the 152 CTAs (two
+    or three each, most CTAs crossing from a policy tile to a value tile).
+    Adam's first moment after one step is 0.1 x the clipped gradient."""
     wl = W.make_72b(n_envs=E) if preset == "72b" else W.make_stress(n_envs=E, horizon=T)
     params, buf, adv, ret = _ppo_inputs(wl, T, seed=4)
     ppo = W.PPOSpec(epochs=1, minibatch=T * E, ent_coef=0.01)
