@@ -23,10 +23,15 @@
 //   da2 = bf16(dh2 (1 - h2^2)) into shared memory (the next A operand) and
 //   its tile image; dh1 = da2 W2 with W2^T streamed through a two-slot ring
 //   of 32 KB stages by a producer warp; epilogue: da1 = bf16(dh1 (1 - h1^2))
-//   to its tile image.  A loader warp brings the tile's h2 image into the da2
-//   buffer with one bulk copy (da2 then overwrites it in place) and, after
-//   the dh1 MMAs, its h1 image, so the epilogues read h from shared memory.
-//   One launch covers both networks: the policy's tiles, then the value's,
+//   to its tile image.  Every step works in 256-column halves so that the
+//   MMAs, the epilogues and the copies overlap: a loader warp brings each
+//   half of the tile's h2 image into the da2 buffer with one bulk copy (da2
+//   then overwrites it in place), the dh1 MMAs over da2's first half start
+//   while the epilogue writes its second half, each half of the h1 image
+//   lands once the dh1 MMAs have read that half of da2, and each half of the
+//   next tile's h2 (and of its dh2 accumulators) follows as soon as the da1
+//   epilogue has read that half of h1 (and of TMEM).  A dedicated warp
+//   issues the MMAs.  One launch covers both networks: the policy's tiles, then the value's,
 //   spread over the CTAs as one list (a CTA that crosses from one to the
 //   other reloads W3^T), which balances a tile count that is not a
 //   multiple of the SM count.
@@ -47,7 +52,7 @@
 namespace pe {
 
 constexpr int kBwCompute = 512;         // 16 compute warps
-constexpr int kBwThreads = kBwCompute + 64;  // + the W2^T producer warp and the h loader warp
+constexpr int kBwThreads = kBwCompute + 96;  // + the W2^T producer, the h loader and the MMA issuer warps
 
 int64_t bwd_image_bytes(int H) {
   if (H == 256) return BwdImg<256>::TOTAL;
@@ -80,22 +85,23 @@ __global__ void bwd_image_kernel(const float* __restrict__ params, int A, uint8_
 
 template <int H>
 struct BwdSmem {
-  // A operand of dh1 = da2 W2 (K-major SW128).  Each tile's h2 image arrives
-  // here first and da2 overwrites it in place (da2 is elementwise in h2);
-  // after the dh1 MMAs the h1 image arrives here for the second epilogue.
+  // A operand of dh1 = da2 W2 (K-major SW128), in 256-column halves (K-blocks
+  // 0-3 and 4-7).  Each half of a tile's h2 image arrives here first and da2
+  // overwrites it in place (da2 is elementwise in h2); once the dh1 MMAs have
+  // read a half of da2, that half of the h1 image arrives for the second
+  // epilogue; once that epilogue has read it, the next tile's h2 half.
   alignas(1024) uint8_t da2[kBwRows * H * 2];
   alignas(1024) uint8_t ring[2][kBwStage];
   alignas(1024) uint8_t w3t[H * 32];           // B operand of dh2 = dz W3 (K-major SW32)
   alignas(1024) uint8_t dz[kBwRows * 32];      // A operand of dh2 (K-major SW32)
-  uint64_t full[2], empty[2], bar_mma, bar_w;
-  uint64_t hin;     // an h image landed in da2 (two completions per tile: h2, then h1)
-  uint64_t dh1;     // the tile's dh1 MMAs are done (da2 may be overwritten by h1)
-  uint64_t bfree;   // the 16 compute warps finished reading h1 (the buffer may take the next h2)
+  uint64_t full[2], empty[2], bar_w, fin;
+  // one completion per tile each: h2 / h1 half landed (bulk copies), dz
+  // written, dh2 N-half done, da2 half written, dh1 N-half 0 done, dh1
+  // N-half 1 past K-block 3, dh1 done, da1 half read out of TMEM and h1
+  uint64_t h2a, h2b, h1a, h1b, dzin, mdh2a, mdh2b, d2a, d2b, m1a, n1lo, m1b, da, db;
   uint32_t tmem_base;
   int32_t err;
 };
-
-__device__ __forceinline__ void bw_compute_sync() { asm volatile("bar.sync 1, 512;" ::: "memory"); }
 
 // per network (policy, value): one launch covers both, their tiles spread
 // over the persistent CTAs together
@@ -113,7 +119,10 @@ struct BwdArgs {
 template <int H>
 __global__ void __launch_bounds__(kBwThreads, 1) bwd_data_kernel(BwdArgs g) {
   using I = BwdImg<H>;
+  static_assert(H == 512, "two 256-column halves per product");
   constexpr int kTileBytes = kBwRows * H * 2;
+  constexpr int kHalfBytes = kTileBytes / 2;  // K-blocks 0-3 or 4-7 of a tile image
+  constexpr int KBH = I::KB / 2;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
   BwdSmem<H>& s = *reinterpret_cast<BwdSmem<H>*>(base);
@@ -124,11 +133,22 @@ __global__ void __launch_bounds__(kBwThreads, 1) bwd_data_kernel(BwdArgs g) {
       tc::mbar_init(&s.full[i], 1);
       tc::mbar_init(&s.empty[i], 1);
     }
-    tc::mbar_init(&s.bar_mma, 1);
     tc::mbar_init(&s.bar_w, 1);
-    tc::mbar_init(&s.hin, 1);
-    tc::mbar_init(&s.dh1, 1);
-    tc::mbar_init(&s.bfree, kBwCompute / 32);
+    tc::mbar_init(&s.fin, 1);
+    tc::mbar_init(&s.h2a, 1);
+    tc::mbar_init(&s.h2b, 1);
+    tc::mbar_init(&s.h1a, 1);
+    tc::mbar_init(&s.h1b, 1);
+    tc::mbar_init(&s.dzin, kBwCompute / 32);
+    tc::mbar_init(&s.mdh2a, 1);
+    tc::mbar_init(&s.mdh2b, 1);
+    tc::mbar_init(&s.d2a, kBwCompute / 32);
+    tc::mbar_init(&s.d2b, kBwCompute / 32);
+    tc::mbar_init(&s.m1a, 1);
+    tc::mbar_init(&s.n1lo, 1);
+    tc::mbar_init(&s.m1b, 1);
+    tc::mbar_init(&s.da, kBwCompute / 32);
+    tc::mbar_init(&s.db, kBwCompute / 32);
     tc::fence_mbar_init();
   }
   if (warp == 0) tc::tmem_alloc(&s.tmem_base, H);
@@ -145,79 +165,153 @@ __global__ void __launch_bounds__(kBwThreads, 1) bwd_data_kernel(BwdArgs g) {
     ni = q >= tiles ? 1 : 0;
     return q - ni * tiles;
   };
+  // a bounded wait that is skipped once the CTA has an error
+  auto wt = [&](uint64_t* b, uint32_t par) -> bool {
+    if (*reinterpret_cast<volatile int32_t*>(&s.err)) return false;
+    if (tc::mbar_wait(b, par)) return true;
+    atomicExch(&s.err, 1);
+    return false;
+  };
   int ni0 = 0;
   if (my_tiles > 0) (void)tile_of(0, ni0);
-  if (tid == 0) {
-    tc::mbar_expect_tx(&s.bar_w, (uint32_t)I::W3T);
-    tc::bulk_g2s(s.w3t, ni0 ? g.img[1] : g.img[0], (uint32_t)I::W3T, &s.bar_w);
-  }
   int last_issued = -1;  // producer: global index of its last issued stage
-  int h_issued = 0;      // loader: h copies issued (the hin phases)
+  int nh[4] = {0, 0, 0, 0};  // loader: copies issued into h2a, h2b, h1a, h1b
   int cur = ni0;         // MMA issuer: network of the W3^T in shared memory
   if (warp == kBwCompute / 32) {
     // producer: the W2^T stages of every tile, in consumption order
     if (lane == 0) {
       int gs = 0;
-      for (int t = 0; t < my_tiles; ++t) {
+      bool ok = true;
+      for (int t = 0; t < my_tiles && ok; ++t) {
         int ni;
         (void)tile_of(t, ni);
         const uint8_t* img = ni ? g.img[1] : g.img[0];
-        for (int st = 0; st < I::STAGES; ++st, ++gs) {
+        for (int st = 0; st < I::STAGES; ++st) {
           const int slot = gs & 1;
-          if (gs >= 2 && !tc::mbar_wait(&s.empty[slot], ((gs - 2) >> 1) & 1)) {
-            atomicExch(&s.err, 1);
-            t = my_tiles;
+          if (gs >= 2 && !wt(&s.empty[slot], ((gs - 2) >> 1) & 1)) {
+            ok = false;
             break;
           }
           tc::mbar_expect_tx(&s.full[slot], (uint32_t)kBwStage);
           tc::bulk_g2s(s.ring[slot], img + I::W3T + (int64_t)st * kBwStage, (uint32_t)kBwStage, &s.full[slot]);
-          last_issued = gs;
+          last_issued = gs++;
         }
       }
     }
   } else if (warp == kBwCompute / 32 + 1) {
-    // loader: per tile, the h2 image into the da2 buffer once the previous
-    // tile's second epilogue has read h1 out of it, then the h1 image once
-    // the dh1 MMAs have read da2
+    // loader: per tile, h1's first half once the dh1 MMAs over da2's first
+    // half are done, its second half once all are; then the next tile's h2
+    // halves as the second epilogue frees the halves of the buffer
     if (lane == 0) {
+      auto copy = [&](int which, uint64_t* bar, const uint8_t* src, int half) {
+        tc::mbar_expect_tx(bar, (uint32_t)kHalfBytes);
+        tc::bulk_g2s(s.da2 + half * kHalfBytes, src + half * kHalfBytes, (uint32_t)kHalfBytes, bar);
+        ++nh[which];
+      };
+      if (my_tiles > 0) {
+        const uint8_t* h2 = (ni0 ? g.h2[1] : g.h2[0]) + tile_of(0, ni0) * (int64_t)kTileBytes;
+        copy(0, &s.h2a, h2, 0);
+        copy(1, &s.h2b, h2, 1);
+      }
       for (int t = 0; t < my_tiles; ++t) {
+        const uint32_t par = t & 1;
         int ni;
-        const int64_t tile = tile_of(t, ni);
-        const uint8_t* h2 = ni ? g.h2[1] : g.h2[0];
-        const uint8_t* h1 = ni ? g.h1[1] : g.h1[0];
-        if (t > 0 && !tc::mbar_wait(&s.bfree, (t - 1) & 1)) {
-          atomicExch(&s.err, 1);
-          break;
+        const int64_t tl = tile_of(t, ni);
+        const uint8_t* h1 = (ni ? g.h1[1] : g.h1[0]) + tl * (int64_t)kTileBytes;
+        if (!wt(&s.n1lo, par)) break;
+        copy(2, &s.h1a, h1, 0);
+        if (!wt(&s.m1b, par)) break;
+        copy(3, &s.h1b, h1, 1);
+        if (t + 1 < my_tiles) {
+          int nn;
+          const int64_t nt = tile_of(t + 1, nn);
+          const uint8_t* h2 = (nn ? g.h2[1] : g.h2[0]) + nt * (int64_t)kTileBytes;
+          if (!wt(&s.da, par)) break;
+          copy(0, &s.h2a, h2, 0);
+          if (!wt(&s.db, par)) break;
+          copy(1, &s.h2b, h2, 1);
         }
-        tc::mbar_expect_tx(&s.hin, (uint32_t)kTileBytes);
-        tc::bulk_g2s(s.da2, h2 + tile * (int64_t)kTileBytes, (uint32_t)kTileBytes, &s.hin);
-        ++h_issued;
-        if (!tc::mbar_wait(&s.dh1, t & 1)) {
-          atomicExch(&s.err, 1);
-          break;
-        }
-        tc::mbar_expect_tx(&s.hin, (uint32_t)kTileBytes);
-        tc::bulk_g2s(s.da2, h1 + tile * (int64_t)kTileBytes, (uint32_t)kTileBytes, &s.hin);
-        ++h_issued;
       }
     }
+  } else if (warp == kBwCompute / 32 + 2) {
+    // MMA issuer
+    if (lane == 0) {
+      tc::mbar_expect_tx(&s.bar_w, (uint32_t)I::W3T);
+      tc::bulk_g2s(s.w3t, ni0 ? g.img[1] : g.img[0], (uint32_t)I::W3T, &s.bar_w);
+      (void)wt(&s.bar_w, 0);
+      const uint32_t da2a = tc::smem_u32(s.da2), dza = tc::smem_u32(s.dz), w3a = tc::smem_u32(s.w3t);
+      constexpr uint32_t kIdN = tc::idesc_bf16(kBwRows, 256);
+      int gs = 0;
+      // dh1 = da2 W2: K-blocks [k0, k1) of da2 into N-half h (TMEM columns 256 h ..)
+      auto dh1 = [&](int h, int k0, int k1) {
+#pragma unroll 1
+        for (int kb = k0; kb < k1; ++kb) {
+          const int slot = gs & 1;
+          (void)wt(&s.full[slot], (gs >> 1) & 1);
+          tc::fence_after();
+          const uint32_t ra = tc::smem_u32(s.ring[slot]);
+#pragma unroll
+          for (int kk = 0; kk < 4; ++kk)
+            tc::mma_bf16(tmem + h * 256, tc::desc_kmajor(da2a + kb * kBwRows * 128 + kk * 32, 1024, tc::kLayoutSW128),
+                         tc::desc_kmajor(ra + kk * 32, 1024, tc::kLayoutSW128), kIdN, (kb | kk) != 0);
+          tc::mma_commit(&s.empty[slot]);
+          ++gs;
+        }
+      };
+      for (int t = 0; t < my_tiles; ++t) {
+        const uint32_t par = t & 1;
+        int ni;
+        (void)tile_of(t, ni);
+        (void)wt(&s.dzin, par);
+        tc::fence_after();
+        if (ni != cur) {
+          // the value network's W3^T replaces the policy's (every MMA that
+          // read it completed before the previous tile's da2 epilogue)
+          cur = ni;
+          tc::mbar_expect_tx(&s.bar_w, (uint32_t)I::W3T);
+          tc::bulk_g2s(s.w3t, g.img[1], (uint32_t)I::W3T, &s.bar_w);
+          (void)wt(&s.bar_w, 1);
+          tc::fence_after();
+        }
+        // dh2 = dz W3, one K = 16 MMA per N-half, each once the previous
+        // tile's da1 epilogue has read that half of TMEM
+#pragma unroll 1
+        for (int h = 0; h < I::NH; ++h) {
+          if (t > 0) {
+            (void)wt(h ? &s.db : &s.da, par ^ 1);
+            tc::fence_after();
+          }
+          tc::mma_bf16(tmem + h * 256, tc::desc_strided(dza, 16, 256, tc::kLayoutSW32),
+                       tc::desc_strided(w3a + h * 256 * 32, 16, 256, tc::kLayoutSW32), kIdN, 0);
+          tc::mma_commit(h ? &s.mdh2b : &s.mdh2a);
+        }
+        (void)wt(&s.d2a, par);
+        tc::fence_after();
+        dh1(0, 0, KBH);
+        (void)wt(&s.d2b, par);
+        tc::fence_after();
+        dh1(0, KBH, 2 * KBH);
+        tc::mma_commit(&s.m1a);
+        dh1(1, 0, KBH);
+        tc::mma_commit(&s.n1lo);
+        dh1(1, KBH, 2 * KBH);
+        tc::mma_commit(&s.m1b);
+      }
+      // every MMA of this CTA completes before TMEM is released
+      tc::mma_commit(&s.fin);
+      if (!tc::mbar_wait(&s.fin, 0)) atomicExch(&s.err, 1);
+    }
   } else {
-    if (!tc::mbar_wait(&s.bar_w, 0)) atomicExch(&s.err, 1);
-    const bool issuer = (tid == 32);
-    const uint32_t da2a = tc::smem_u32(s.da2), dza = tc::smem_u32(s.dz), w3a = tc::smem_u32(s.w3t);
-    const uint32_t r0a = tc::smem_u32(s.ring[0]), r1a = tc::smem_u32(s.ring[1]);
-    constexpr uint32_t kIdN = tc::idesc_bf16(kBwRows, 256);
-    uint32_t phase = 0;
-    int gs = 0;
     const int quad = warp & 3, slice = warp >> 2, row = quad * 32 + lane;
     const uint32_t lane_addr = tmem + ((uint32_t)(quad * 32) << 16);
-    constexpr int NJ = H / 4 / 16;  // 16-column chunks per thread
-    // d = bf16(TMEM (1 - h^2)) for this thread's chunks, h read from the
-    // shared buffer at the offsets d is written to (in place when sbuf)
-    auto epi = [&](bool valid, uint8_t* outt, bool in_place) {
+    constexpr int NJ = H / 2 / 4 / 16;  // 16-column chunks per thread and half
+    // d = bf16(TMEM (1 - h^2)) over this thread's chunks of half hf, h read
+    // from the shared buffer at the offsets d is written to (in place when
+    // in_place), d also to the tile image outt
+    auto epi = [&](int hf, bool valid, uint8_t* outt, bool in_place) {
 #pragma unroll 2
       for (int j = 0; j < NJ; ++j) {
-        const int c = slice * (H / 4) + j * 16;
+        const int c = hf * (H / 2) + slice * (H / 8) + j * 16;
         float v[16];
         tc::tmem_ld16(lane_addr + (uint32_t)c, v);
         const uint32_t o0 = tc::swz_offset<128>(row, c, kBwRows), o1 = tc::swz_offset<128>(row, c + 8, kBwRows);
@@ -233,12 +327,17 @@ __global__ void __launch_bounds__(kBwThreads, 1) bwd_data_kernel(BwdArgs g) {
         *reinterpret_cast<uint4*>(outt + o1) = hi;
       }
     };
+    auto handover = [&](uint64_t* bar) {
+      tc::fence_async_smem();
+      tc::fence_before();
+      __syncwarp();
+      if (lane == 0) asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(tc::smem_u32(bar)) : "memory");
+    };
     uint4 dzv = make_uint4(0, 0, 0, 0);
     if (tid < kBwRows * 2 && my_tiles > 0)
       dzv = __ldg(reinterpret_cast<const uint4*>((ni0 ? g.dz[1] : g.dz[0]) + tile_of(0, ni0) * (kBwRows * 32)) + tid);
     for (int t = 0; t < my_tiles; ++t) {
-      // every compute thread takes the same decision (a named barrier with an OR)
-      if (tc::bar_any(1, kBwCompute, s.err != 0)) break;
+      const uint32_t par = t & 1;
       int ni, nn = 0;
       const int64_t tile = tile_of(t, ni);
       const int64_t ntile = t + 1 < my_tiles ? tile_of(t + 1, nn) : 0;
@@ -253,80 +352,54 @@ __global__ void __launch_bounds__(kBwThreads, 1) bwd_data_kernel(BwdArgs g) {
           tc::prefetch_l2(h1n + off);
         }
       }
-      // dz tile (4 KB, already in the SW32 layout), then the next tile's
+      // dz tile (4 KB, already in the SW32 layout; the previous tile's dh2
+      // MMAs have read the old one), then the next tile's into registers
       if (tid < kBwRows * 2) {
         reinterpret_cast<uint4*>(s.dz)[tid] = dzv;
         if (t + 1 < my_tiles)
           dzv = __ldg(reinterpret_cast<const uint4*>((nn ? g.dz[1] : g.dz[0]) + ntile * (kBwRows * 32)) + tid);
       }
-      tc::fence_async_smem();
-      bw_compute_sync();
-      // dh2 (TMEM cols 0..H) = dz W3: one K = 16 MMA per 256 columns
-      if (issuer) {
-        tc::fence_after();
-        if (ni != cur) {
-          // the value network's W3^T replaces the policy's (every MMA that
-          // read it completed before the previous tile's first epilogue)
-          cur = ni;
-          tc::mbar_expect_tx(&s.bar_w, (uint32_t)I::W3T);
-          tc::bulk_g2s(s.w3t, g.img[1], (uint32_t)I::W3T, &s.bar_w);
-          if (!tc::mbar_wait(&s.bar_w, 1)) atomicExch(&s.err, 1);
-        }
-#pragma unroll
-        for (int h = 0; h < I::NH; ++h)
-          tc::mma_bf16(tmem + h * 256, tc::desc_strided(dza, 16, 256, tc::kLayoutSW32),
-                       tc::desc_strided(w3a + h * 256 * 32, 16, 256, tc::kLayoutSW32), kIdN, 0);
-        tc::mma_commit(&s.bar_mma);
-      }
-      if (!tc::mbar_wait(&s.bar_mma, phase)) atomicExch(&s.err, 1);
-      phase ^= 1;
-      if (!tc::mbar_wait(&s.hin, 0)) atomicExch(&s.err, 1);  // h2 in the buffer
+      handover(&s.dzin);
+      uint8_t* const da2o = (ni ? g.da2[1] : g.da2[0]) + tile * (int64_t)kTileBytes;
+      uint8_t* const da1o = (ni ? g.da1[1] : g.da1[0]) + tile * (int64_t)kTileBytes;
+      // da2 = bf16(dh2 (1 - h2^2)) per half: in place over h2 (the next A
+      // operand) and its tile image
+      (void)wt(&s.mdh2a, par);
+      (void)wt(&s.h2a, par);
       tc::fence_after();
-      // da2 = bf16(dh2 (1 - h2^2)): in place over h2 (the next A operand) and its tile image
-      epi(valid, (ni ? g.da2[1] : g.da2[0]) + tile * (int64_t)kTileBytes, true);
-      tc::fence_before();
-      tc::fence_async_smem();
-      bw_compute_sync();
-      // dh1 (TMEM cols 0..H) = da2 W2, W2^T streamed: stage (h, kb)
-      if (issuer) {
-        tc::fence_after();
-        for (int h = 0; h < I::NH; ++h)
-          for (int kb = 0; kb < I::KB; ++kb) {
-            const int slot = gs & 1;
-            if (!tc::mbar_wait(&s.full[slot], (gs >> 1) & 1)) atomicExch(&s.err, 1);
-            tc::fence_after();
-            const uint32_t ra = slot ? r1a : r0a;
-#pragma unroll
-            for (int kk = 0; kk < 4; ++kk)
-              tc::mma_bf16(tmem + h * 256, tc::desc_kmajor(da2a + kb * kBwRows * 128 + kk * 32, 1024, tc::kLayoutSW128),
-                           tc::desc_kmajor(ra + kk * 32, 1024, tc::kLayoutSW128), kIdN, (kb | kk) != 0);
-            tc::mma_commit(&s.empty[slot]);
-            ++gs;
-          }
-        tc::mma_commit(&s.bar_mma);
-        tc::mma_commit(&s.dh1);  // the loader may now bring h1 over da2
-      }
-      if (!tc::mbar_wait(&s.bar_mma, phase)) atomicExch(&s.err, 1);
-      phase ^= 1;
-      if (!tc::mbar_wait(&s.hin, 1)) atomicExch(&s.err, 1);  // h1 in the buffer
+      epi(0, valid, da2o, true);
+      handover(&s.d2a);
+      (void)wt(&s.mdh2b, par);
+      (void)wt(&s.h2b, par);
       tc::fence_after();
-      // da1 = bf16(dh1 (1 - h1^2)) to its tile image
-      epi(valid, (ni ? g.da1[1] : g.da1[0]) + tile * (int64_t)kTileBytes, false);
-      tc::fence_before();
-      tc::fence_async_smem();
-      __syncwarp();
-      if (lane == 0) asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(tc::smem_u32(&s.bfree)) : "memory");
+      epi(1, valid, da2o, true);
+      handover(&s.d2b);
+      // da1 = bf16(dh1 (1 - h1^2)) per half, to its tile image
+      (void)wt(&s.m1a, par);
+      (void)wt(&s.h1a, par);
+      tc::fence_after();
+      epi(0, valid, da1o, false);
+      handover(&s.da);
+      (void)wt(&s.m1b, par);
+      (void)wt(&s.h1b, par);
+      tc::fence_after();
+      epi(1, valid, da1o, false);
+      handover(&s.db);
     }
   }
+  tc::fence_before();
   __syncthreads();
-  // on an error, the producer and the loader wait (bounded) for their last
-  // copies before the CTA leaves, so that no bulk copy into this CTA's shared
-  // memory is in flight (at most one h copy is outstanding at a time)
-  if (s.err && warp == kBwCompute / 32 && lane == 0 && last_issued >= 0)
-    (void)tc::mbar_wait(&s.full[last_issued & 1], (last_issued >> 1) & 1);
-  if (s.err && warp == kBwCompute / 32 + 1 && lane == 0 && h_issued > 0)
-    (void)tc::mbar_wait(&s.hin, (h_issued - 1) & 1);
-  if (s.err && tid == 32 && cur != ni0) (void)tc::mbar_wait(&s.bar_w, 1);
+  // on an error, the producer, the loader and the issuer wait (bounded) for
+  // the copies they may still have in flight before the CTA leaves
+  if (s.err && warp == kBwCompute / 32 && lane == 0)
+    for (int q = last_issued - 1; q <= last_issued; ++q)
+      if (q >= 0) (void)tc::mbar_wait(&s.full[q & 1], (q >> 1) & 1);
+  if (s.err && warp == kBwCompute / 32 + 1 && lane == 0) {
+    uint64_t* bars[4] = {&s.h2a, &s.h2b, &s.h1a, &s.h1b};
+    for (int k = 0; k < 4; ++k)
+      if (nh[k] > 0) (void)tc::mbar_wait(bars[k], (nh[k] - 1) & 1);
+  }
+  if (s.err && warp == kBwCompute / 32 + 2 && lane == 0) (void)tc::mbar_wait(&s.bar_w, cur != ni0 ? 1 : 0);
   if (tid == 0 && s.err && g.err) atomicExch(g.err, 1);
   __syncthreads();
   if (warp == 0) tc::tmem_dealloc(tmem, H);
