@@ -688,24 +688,27 @@ struct PpoLoop {
 // the k-th barrier's arrivals are numbered k*G .. k*G + G - 1 (no CTA can
 // arrive at barrier k + 1 before all have arrived at k), so each CTA waits
 // for the counter to reach (k + 1) * G; the last arrival releases everyone
-// with its own atomic, and nothing is reset.  The wait is bounded.
+// with its own atomic, and nothing is reset.  The wait is bounded.  Memory
+// order: the block barrier puts the CTA's writes before thread 0's arrival,
+// a release at GPU scope; thread 0's polling loads are acquires at GPU
+// scope, and the second block barrier puts them before the CTA's reads.
 __device__ __forceinline__ bool grid_barrier(unsigned int* bar, int* s_ok, long long limit = 4000000000LL) {
   __syncthreads();
   if (threadIdx.x == 0) {
-    __threadfence();
-    const unsigned int old = atomicAdd(bar, 1u);
+    unsigned int old;
+    asm volatile("atom.release.gpu.global.add.u32 %0, [%1], 1;" : "=r"(old) : "l"(bar) : "memory");
     const unsigned int target = (old / gridDim.x + 1u) * gridDim.x;
-    volatile unsigned int* vb = bar;
     bool ok = true;
     const long long t0 = clock64();
-    while ((int)(*vb - target) < 0) {
+    for (;;) {
+      unsigned int v;
+      asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(bar) : "memory");
+      if ((int)(v - target) >= 0) break;
       if (clock64() - t0 > limit) {  // by default about 2 s at the maximum SM clock
         ok = false;
         break;
       }
-      __nanosleep(32);
     }
-    __threadfence();
     *s_ok = ok;
   }
   __syncthreads();
