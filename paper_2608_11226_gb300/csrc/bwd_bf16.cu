@@ -441,11 +441,34 @@ struct WgArgs {
   const uint8_t* x;   // shared input tile images
   int64_t n;          // valid samples
   int nstages;        // ceil(n / 64)
-  int spc;            // stages per CTA
-  int S;              // sample chunks (CTAs per group)
-  float* part;        // [groups * S][128][kWgMaxCols]
+  int spc[2];         // stages per CTA, per column chunk
+  int S[2];           // sample chunks (CTAs per group), per column chunk
+  float* part;        // one [128][kWgMaxCols] partial block per CTA, in CTA order
   int32_t* err;
 };
+
+// CTA b of the weight-gradient launch: its output group and sample chunk.
+// Groups are ordered (network, row block, column chunk); the CTAs of one
+// (network, row block) are S[0] chunks of column chunk 0, then S[1] of
+// column chunk 1 (with one column chunk, S[0] chunks per group).
+template <int NCH>
+__host__ __device__ __forceinline__ void wg_cta(int b, const int (&S)[2], int& grp, int& chunk) {
+  if (NCH == 2) {
+    const int per = S[0] + S[1], q = b / per, r = b % per;
+    const int nc = r < S[0] ? 0 : 1;
+    grp = 2 * q + nc;
+    chunk = nc ? r - S[0] : r;
+  } else {
+    grp = b / S[0];
+    chunk = b % S[0];
+  }
+}
+
+// first CTA (partial block) of group grp
+template <int NCH>
+__host__ __device__ __forceinline__ int wg_first_cta(int grp, const int (&S)[2]) {
+  return NCH == 2 ? (grp >> 1) * (S[0] + S[1]) + ((grp & 1) ? S[0] : 0) : grp * S[0];
+}
 
 template <int D, int H>
 __global__ void __launch_bounds__(kWgThreads, 1) wgrad_kernel(WgArgs g) {
@@ -456,11 +479,13 @@ __global__ void __launch_bounds__(kWgThreads, 1) wgrad_kernel(WgArgs g) {
   uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
   WgSmem& s = *reinterpret_cast<WgSmem*>(base);
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int grp = blockIdx.x / g.S, chunk = blockIdx.x % g.S;
+  int grp, chunk;
+  wg_cta<NCH>((int)blockIdx.x, g.S, grp, chunk);
   const int ni = grp / (MB * NCH), mb = (grp / NCH) % MB, nc = grp % NCH;
   const bool first = nc == 0;  // column chunk 0 also takes dW1, db1, dW3^T
   const WgNet& nt = g.net[ni];
-  const int k0 = chunk * g.spc, k1 = min(k0 + g.spc, g.nstages);
+  const int spc = nc ? g.spc[1] : g.spc[0];
+  const int k0 = chunk * spc, k1 = min(k0 + spc, g.nstages);
   if (tid == 0) {
     s.err = 0;
     for (int i = 0; i < 2; ++i) {
@@ -596,7 +621,8 @@ constexpr int kWgReduceThreads = 512;  // 27 warps per SM, eight chunk loads in 
 constexpr int kLossPartW = 32;  // loss-kernel partial row: pg, ent, kl, clip, vl, db3[16], dc3
 
 template <int D, int H>
-__global__ void __launch_bounds__(kWgReduceThreads) wgrad_reduce_kernel(const float* __restrict__ part, int S, int A,
+__global__ void __launch_bounds__(kWgReduceThreads) wgrad_reduce_kernel(const float* __restrict__ part, int S0, int S1,
+                                                           int A,
                                                            float* __restrict__ grad, const float* __restrict__ lossp,
                                                            int nlb, double* __restrict__ stat5,
                                                            float* __restrict__ sq) {
@@ -623,10 +649,12 @@ __global__ void __launch_bounds__(kWgReduceThreads) wgrad_reduce_kernel(const fl
       else if (col >= Cn::DW3 && col < Cn::DW3 + nout) dst = (ni ? Lp.v3 : Lp.w3) + (int64_t)(col - Cn::DW3) * H + o;
     }
     if (dst < 0) continue;
-    const float* p = part + ((int64_t)grp * S * 128 + row) * kWgMaxCols + col;
+    const int S[2] = {S0, S1};
+    const int nch = nc ? S1 : S0;
+    const float* p = part + ((int64_t)wg_first_cta<NCH>(grp, S) * 128 + row) * kWgMaxCols + col;
     float acc = 0.0f;
 #pragma unroll 8
-    for (int k = 0; k < S; ++k) acc += p[(int64_t)k * 128 * kWgMaxCols];
+    for (int k = 0; k < nch; ++k) acc += p[(int64_t)k * 128 * kWgMaxCols];
     grad[dst] = acc;
     q = fmaf(acc, acc, q);
   }
@@ -726,18 +754,39 @@ static pe_status bwd_launch(const float* params, int A, uint8_t* const img[2], c
     a.x = x;
     a.n = n;
     a.nstages = (int)((n + kWgSamples - 1) / kWgSamples);
-    const int s_want = std::max(1, std::min(std::min(sms, kWgMaxCtas) / groups, a.nstages));
-    a.spc = (a.nstages + s_want - 1) / s_want;
-    a.S = (a.nstages + a.spc - 1) / a.spc;
+    // CTAs per (network, row block), split between the column chunks in
+    // proportion to the bytes a stage brings in: chunk 0 also loads da1, h2,
+    // x and dz (for the Stress networks 90 KB per stage against 48 KB), so
+    // with equal shares its CTAs would set the launch's length
+    constexpr int NCH = H / 256;
+    const int cap = std::max(NCH, std::min(sms, kWgMaxCtas) / (groups / NCH));
+    int want[2] = {cap, 0};
+    if (NCH == 2) {
+      const double hb = (double)kWgSamples * 128;
+      const double b0 = 10 * hb + kWgSamples * (D * 2 + 32), b1 = 6 * hb;
+      want[0] = std::min(cap - 1, std::max(1, (int)std::lround(cap * b0 / (b0 + b1))));
+      want[1] = cap - want[0];
+    }
+    int ctas = 0;
+    for (int c = 0; c < 2; ++c) {
+      a.spc[c] = a.S[c] = 0;
+      if (c >= NCH) continue;
+      const int s_want = std::max(1, std::min(want[c], a.nstages));
+      a.spc[c] = (a.nstages + s_want - 1) / s_want;
+      a.S[c] = (a.nstages + a.spc[c] - 1) / a.spc[c];
+      ctas += a.S[c];
+    }
+    ctas *= groups / NCH;
     a.part = part;
     a.err = err;
     auto kern = wgrad_kernel<D, H>;
     const int bytes = (int)sizeof(WgSmem) + 1024;
     PE_TRY_CUDA(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes));
     ProfScope ps(PE_PROF_PPO_GRAD, st);
-    kern<<<groups * a.S, kWgThreads, bytes, st>>>(a);
+    kern<<<ctas, kWgThreads, bytes, st>>>(a);
     PE_CHECK_LAUNCH("wgrad_kernel");
-    wgrad_reduce_kernel<D, H><<<kWgReduceBlocks, kWgReduceThreads, 0, st>>>(part, a.S, A, grad, lossp, nlb, stat5, sq);
+    wgrad_reduce_kernel<D, H><<<kWgReduceBlocks, kWgReduceThreads, 0, st>>>(part, a.S[0], a.S[1], A, grad, lossp, nlb,
+                                                                           stat5, sq);
     PE_CHECK_LAUNCH("wgrad_reduce_kernel");
   }
   return PE_OK;
