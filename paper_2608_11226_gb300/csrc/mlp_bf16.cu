@@ -85,8 +85,11 @@ __global__ void weight_image_kernel(const float* __restrict__ params, int A, int
 //   results wait in registers until the N-half 1 MMAs have read h1's first
 //   four K-blocks, which h2 overwrites in place;
 //   the head accumulates in TMEM columns 256-271, so the next tile's layer-1
-//   N-half 0 can start while warps 0-3 still read the head, and warps 4-15
-//   write the next tile's X during that head epilogue.
+//   N-half 0 can start while warps 0-3 copy the head accumulators to shared
+//   memory (they compute the loss later, during the next tile's layer-2
+//   N-half 0 MMAs) and warps 4-15 write the next tile's X (its rows fetched
+//   during the previous epilogue) into the buffer's last K-block, which only
+//   epilogue 1, half B overwrites.
 // The accumulation order of every accumulator is that of the serial kernel,
 // so the results are the same bits.  One launch may also cover two networks
 // over the same rows (the policy, then the value network of a PPO forward):
