@@ -31,16 +31,18 @@
 //   lands once the dh1 MMAs have read that half of da2, and each half of the
 //   next tile's h2 (and of its dh2 accumulators) follows as soon as the da1
 //   epilogue has read that half of h1 (and of TMEM).  A dedicated warp
-//   issues the MMAs.  One launch covers both networks: the policy's tiles, then the value's,
-//   spread over the CTAs as one list (a CTA that crosses from one to the
-//   other reloads W3^T), which balances a tile count that is not a
-//   multiple of the SM count.
+//   issues the MMAs.  One launch covers both networks: the policy's tiles,
+//   then the value's, spread over the CTAs as one list (a CTA that crosses
+//   from one to the other reloads W3^T), which balances a tile count that
+//   is not a multiple of the SM count.
 // wgrad_kernel (split over samples): each CTA owns 128 output rows (one
 //   block of layer outputs o) of one network and one 256-column chunk, and
 //   accumulates over its share of the minibatch, 64 samples per stage:
 //   [dW2 | db2] = da2^T [h1 | 1], and for column chunk 0 also
 //   [dW1 | db1] = da1^T [x | 1] and dW3^T = h2^T dz; it writes its fp32
-//   accumulators as one partial block.  wgrad_reduce_kernel sums the partial
+//   accumulators as one partial block.  Column chunk 0's stages bring more
+//   bytes, so its groups get proportionally more (shorter) sample shares.
+//   wgrad_reduce_kernel sums the partial
 //   blocks of every output in a fixed order (deterministic) into the
 //   canonical gradient vector.
 #include <algorithm>
